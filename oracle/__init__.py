@@ -1,0 +1,37 @@
+"""CPU oracle for the UMIM decode step over a merged context (arXiv 2609.27233).
+
+TEST INFRASTRUCTURE ONLY.  Nothing in the product path imports, links or runs
+this package: only ``tests/``, ``__graft_entry__.smoke()`` and ``bench.py``'s
+CPU-baseline / reference arm use it.  It shares no code with the CUDA library
+(``paper_2609_27233_gb300``) and does not import it.
+
+Every function is a plain, slow, obviously-correct restatement of what the
+paper defines, in float64 for floating point and exact integer / byte logic
+for indices and moved KV bytes:
+
+  merge.merge_spans       App. C.1 (attention-based pooling), Sec. 3.2 Eq. 1
+  rollback.kv_rollback    App. C.6 and App. E ("Decoding-Time Merging and
+                          KV-Cache Update"), Fig. 2 caption
+  attention.decode_attention
+                          the backbone's ordinary attention over the shorter
+                          cache (App. I.1); grouped-query mapping of Llama
+  compaction.build_compressed
+                          App. C.5 and App. E ("Prompt Merging"), App. J.4
+                          ("Compressed-position convention")
+  spans.span_metadata     removed-position count r(t) and compressed index
+                          pi(t) = t - r(t) of App. J.4
+
+bf16 values are represented by their raw bit patterns (numpy uint16) and
+upcast exactly to float64.
+
+Parity status per function (what pins it is in tests/test_oracle_*.py):
+  merge_spans       pinned (library routines, invariants, brute force)
+  kv_rollback       pinned (worked example, length formula, invariants)
+  decode_attention  pinned (library SDPA, closed forms, invariants)
+  build_compressed  pinned (worked example, length formula, library bf16)
+"""
+from . import bf16, spans, merge, rollback, attention, compaction  # noqa: F401
+from .merge import merge_spans, merge_span_reference_steps  # noqa: F401
+from .rollback import kv_rollback  # noqa: F401
+from .attention import decode_attention  # noqa: F401
+from .compaction import build_compressed  # noqa: F401

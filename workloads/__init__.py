@@ -1,0 +1,342 @@
+"""Seeded synthetic inputs for the UMIM decode step over a merged context.
+
+This module only draws random numbers and does the bookkeeping a paged-cache
+allocator would do (which physical page holds which logical page).  It holds
+none of the method's arithmetic: no merge module, no rollback, no attention.
+Both the CUDA path (through its binding) and the CPU oracle consume exactly
+the tensors produced here, so a parity test compares like with like.
+
+Shapes follow the workloads the paper evaluates (Llama-3-8B / 3.1-8B-shaped
+layers, span lengths n in {2,3,4} from the merge rule of Sec. 3.1, 30-40 %
+token coverage matching the reported token reduction, App. I.1 decode
+setting).  The paper's corpora (WikiText-103 and others) are not available, so
+uniform token ids and N(0, sigma^2) embeddings / KV entries stand in for them.
+
+Randomness:
+  * integer structure (token ids, span placement, page permutation, lengths)
+    comes from numpy's PCG64 seeded per workload, so it is identical on any
+    host;
+  * bulk bf16 tensors (embedding tables, KV pools, q) come from a seeded
+    ``torch.Generator`` on the device that will hold them (float32 normal,
+    then rounded to bf16 by torch).
+"""
+from __future__ import annotations
+
+import dataclasses
+import math
+from typing import Optional, Sequence
+
+import numpy as np
+import torch
+
+PAGE_SIZE = 16
+
+# Seeds: one per named workload, 0x5EED000n.
+SEEDS = {
+    "tiny": 0x5EED0001,
+    "llama8b_layer": 0x5EED0002,
+    "prompt_compression": 0x5EED0003,
+    "long_context": 0x5EED0004,
+    "long_context_tr40": 0x5EED0014,
+    "serving": 0x5EED0005,
+}
+
+
+def rng(seed: int) -> np.random.Generator:
+    return np.random.Generator(np.random.PCG64(seed))
+
+
+def torch_gen(seed: int, device) -> torch.Generator:
+    g = torch.Generator(device=device)
+    g.manual_seed(seed)
+    return g
+
+
+# ----------------------------------------------------------------------------
+# span placement
+# ----------------------------------------------------------------------------
+def span_layout(r: np.random.Generator, L: int, *, n_spans: Optional[int] = None,
+                coverage: Optional[float] = None, kmin: int = 2, kmax: int = 4):
+    """Sorted, non-overlapping spans inside [0, L).
+
+    Lengths are drawn uniformly from {kmin..kmax}, either exactly ``n_spans``
+    of them or until they cover ``round(coverage * L)`` positions.  The L - sum(k)
+    free positions are spread over the S+1 gaps by a uniform random
+    composition (stars and bars).  Returns (start[S], length[S]) int32.
+    """
+    lens = []
+    if n_spans is not None:
+        lens = list(r.integers(kmin, kmax + 1, size=n_spans))
+    else:
+        target = int(round(coverage * L))
+        tot = 0
+        while tot < target:
+            k = int(r.integers(kmin, kmax + 1))
+            if tot + k > L:
+                break
+            lens.append(k)
+            tot += k
+    lens = np.asarray(lens, dtype=np.int64)
+    S = len(lens)
+    free = L - int(lens.sum())
+    if free < 0:
+        raise ValueError("spans do not fit")
+    if S == 0:
+        return np.zeros(0, np.int32), np.zeros(0, np.int32)
+    # stars and bars: choose S bar positions among free + S slots
+    bars = np.sort(r.choice(free + S, size=S, replace=False))
+    gaps_before = bars - np.arange(S)          # free positions before span i (cumulative)
+    starts = gaps_before + np.concatenate([[0], np.cumsum(lens)[:-1]])
+    return starts.astype(np.int32), lens.astype(np.int32)
+
+
+def suffix_span(r: np.random.Generator, L: int, kmin: int = 2, kmax: int = 4):
+    k = int(r.integers(kmin, kmax + 1))
+    k = min(k, L)
+    return L - k, k
+
+
+# ----------------------------------------------------------------------------
+# bulk bf16 tensors
+# ----------------------------------------------------------------------------
+def bf16_normal(shape, std: float, seed: int, device="cpu") -> torch.Tensor:
+    g = torch_gen(seed, device)
+    # chunked so that very large tensors never need a full float32 copy
+    out = torch.empty(shape, dtype=torch.bfloat16, device=device)
+    of = out.view(-1)
+    step = 1 << 26
+    for i in range(0, of.numel(), step):
+        j = min(of.numel(), i + step)
+        of[i:j] = torch.randn(j - i, generator=g, device=device, dtype=torch.float32).mul_(std)
+    return out
+
+
+def bf16_uniform(shape, lo: float, hi: float, seed: int, device="cpu") -> torch.Tensor:
+    g = torch_gen(seed, device)
+    x = torch.rand(shape, generator=g, device=device, dtype=torch.float32)
+    return (x * (hi - lo) + lo).to(torch.bfloat16)
+
+
+def bits(t: torch.Tensor) -> np.ndarray:
+    """Raw bf16 bit patterns of a bf16 tensor as a numpy uint16 array."""
+    return t.detach().contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+
+
+# ----------------------------------------------------------------------------
+# merge-module weights (random init; the trained checkpoints are not public)
+# ----------------------------------------------------------------------------
+@dataclasses.dataclass
+class MergeWeights:
+    d_model: int
+    n_heads: int
+    w_kv: torch.Tensor      # [d][d]  W[out][in]
+    b_kv: torch.Tensor      # [d]
+    ln_kv_gamma: torch.Tensor
+    ln_kv_beta: torch.Tensor
+    query: torch.Tensor     # [h][d/h]
+    w_o: torch.Tensor       # [d][d]
+    b_o: torch.Tensor
+    ln_o_gamma: torch.Tensor
+    ln_o_beta: torch.Tensor
+    ln_eps: float = 1e-5
+
+    def tensors(self):
+        return dict(w_kv=self.w_kv, b_kv=self.b_kv, ln_kv_gamma=self.ln_kv_gamma,
+                    ln_kv_beta=self.ln_kv_beta, query=self.query, w_o=self.w_o,
+                    b_o=self.b_o, ln_o_gamma=self.ln_o_gamma, ln_o_beta=self.ln_o_beta)
+
+    def to(self, device):
+        kw = {k: v.to(device) for k, v in self.tensors().items()}
+        return MergeWeights(self.d_model, self.n_heads, ln_eps=self.ln_eps, **kw)
+
+
+def merge_weights(d: int, h: int, seed: int, device="cpu") -> MergeWeights:
+    """Linear weights/biases ~ U(-1/sqrt(d), 1/sqrt(d)) (the usual Linear init),
+    q ~ N(0,1), LayerNorm gamma = 1 + U(-0.1,0.1), beta ~ U(-0.1,0.1); all bf16."""
+    a = 1.0 / math.sqrt(d)
+    s = seed * 16
+    return MergeWeights(
+        d_model=d, n_heads=h,
+        w_kv=bf16_uniform((d, d), -a, a, s + 1, device),
+        b_kv=bf16_uniform((d,), -a, a, s + 2, device),
+        ln_kv_gamma=bf16_uniform((d,), 0.9, 1.1, s + 3, device),
+        ln_kv_beta=bf16_uniform((d,), -0.1, 0.1, s + 4, device),
+        query=bf16_normal((h, d // h), 1.0, s + 5, device),
+        w_o=bf16_uniform((d, d), -a, a, s + 6, device),
+        b_o=bf16_uniform((d,), -a, a, s + 7, device),
+        ln_o_gamma=bf16_uniform((d,), 0.9, 1.1, s + 8, device),
+        ln_o_beta=bf16_uniform((d,), -0.1, 0.1, s + 9, device),
+    )
+
+
+# ----------------------------------------------------------------------------
+# span tokens for the merge module
+# ----------------------------------------------------------------------------
+@dataclasses.dataclass
+class MergeCase:
+    table: torch.Tensor          # [V][d] bf16
+    token_ids: torch.Tensor      # [T] int32, span tokens concatenated
+    span_offsets: torch.Tensor   # [S+1] int32
+    weights: MergeWeights
+
+
+def merge_case(seed: int, *, vocab: int, d: int, h: int = 4, n_spans: int,
+               kmin: int = 2, kmax: int = 4, device="cpu", table=None,
+               weights=None) -> MergeCase:
+    r = rng(seed)
+    lens = r.integers(kmin, kmax + 1, size=n_spans)
+    offs = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    ids = r.integers(0, vocab, size=int(offs[-1])).astype(np.int32)
+    if table is None:
+        table = bf16_normal((vocab, d), 0.02, seed + 101, device)
+    if weights is None:
+        weights = merge_weights(d, h, seed + 202, device)
+    return MergeCase(table=table, token_ids=torch.from_numpy(ids).to(device),
+                     span_offsets=torch.from_numpy(offs).to(device), weights=weights)
+
+
+# ----------------------------------------------------------------------------
+# paged KV cache with spans to roll back
+# ----------------------------------------------------------------------------
+@dataclasses.dataclass
+class DecodeCase:
+    pool: torch.Tensor           # [n_layers][n_pages][2][Hkv][P][D] bf16
+    block_table: torch.Tensor    # [B][max_pages] int32 (-1 = no page)
+    seq_lens: torch.Tensor       # [B] int32
+    span_offsets: torch.Tensor   # [B+1] int32 (CSR over sequences)
+    span_start: torch.Tensor     # [S] int32
+    span_len: torch.Tensor       # [S] int32
+    surrogate_k: torch.Tensor    # [S][n_layers][Hkv][D] bf16
+    surrogate_v: torch.Tensor
+    q: torch.Tensor              # [B][Hq][D] bf16
+    n_q_heads: int
+    page_size: int = PAGE_SIZE
+
+    @property
+    def n_layers(self):
+        return self.pool.shape[0]
+
+    @property
+    def n_pages(self):
+        return self.pool.shape[1]
+
+    @property
+    def n_kv_heads(self):
+        return self.pool.shape[3]
+
+    @property
+    def head_dim(self):
+        return self.pool.shape[5]
+
+    @property
+    def max_pages(self):
+        return self.block_table.shape[1]
+
+
+def decode_case(seed: int, *, lens: Sequence[int], n_q_heads: int, n_kv_heads: int,
+                head_dim: int, n_layers: int = 1, coverage: Optional[float] = None,
+                n_spans: Optional[Sequence[int]] = None, kmin: int = 2, kmax: int = 4,
+                spare_pages: int = 0, extra_max_pages: int = 0, suffix_only: bool = False,
+                device="cpu", pool_device=None, kv_std: float = 1.0) -> DecodeCase:
+    """A paged bf16 KV cache holding ``lens[b]`` entries per sequence, spans to
+    roll back in each sequence, surrogate K/V and one query token per sequence.
+
+    Physical pages are a random permutation of the pool, so logical order and
+    physical order differ.  Every slot of the pool (used or not) holds N(0,1)
+    bf16 values."""
+    r = rng(seed)
+    B = len(lens)
+    P = PAGE_SIZE
+    lens = np.asarray(lens, dtype=np.int64)
+    pages_per = (lens + P - 1) // P
+    max_pages = int(max(1, pages_per.max() if B else 1)) + extra_max_pages
+    n_pages = int(pages_per.sum()) + spare_pages
+    n_pages = max(n_pages, 1)
+    perm = r.permutation(n_pages).astype(np.int32)
+    bt = np.full((B, max_pages), -1, dtype=np.int32)
+    k = 0
+    for b in range(B):
+        for p in range(int(pages_per[b])):
+            bt[b, p] = perm[k]
+            k += 1
+    starts, slens, offs = [], [], [0]
+    for b in range(B):
+        L = int(lens[b])
+        if suffix_only:
+            if L >= 1 and r.random() < (coverage if coverage is not None else 1.0):
+                s, kk = suffix_span(r, L, kmin, kmax)
+                st, ln = np.array([s], np.int32), np.array([kk], np.int32)
+            else:
+                st, ln = np.zeros(0, np.int32), np.zeros(0, np.int32)
+        elif n_spans is not None:
+            st, ln = span_layout(r, L, n_spans=int(n_spans[b]), kmin=kmin, kmax=kmax)
+        else:
+            st, ln = span_layout(r, L, coverage=coverage or 0.0, kmin=kmin, kmax=kmax)
+        starts.append(st)
+        slens.append(ln)
+        offs.append(offs[-1] + len(st))
+    S = offs[-1]
+    span_start = np.concatenate(starts).astype(np.int32) if S else np.zeros(0, np.int32)
+    span_len = np.concatenate(slens).astype(np.int32) if S else np.zeros(0, np.int32)
+    pdev = pool_device or device
+    pool = bf16_normal((n_layers, n_pages, 2, n_kv_heads, P, head_dim), kv_std, seed + 11, pdev)
+    sk = bf16_normal((S, n_layers, n_kv_heads, head_dim), 1.0, seed + 12, device)
+    sv = bf16_normal((S, n_layers, n_kv_heads, head_dim), 1.0, seed + 13, device)
+    q = bf16_normal((B, n_q_heads, head_dim), 1.0, seed + 14, device)
+    t = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(device)
+    return DecodeCase(pool=pool, block_table=t(bt), seq_lens=t(lens.astype(np.int32)),
+                      span_offsets=t(np.asarray(offs, np.int32)), span_start=t(span_start),
+                      span_len=t(span_len), surrogate_k=sk, surrogate_v=sv, q=q,
+                      n_q_heads=n_q_heads)
+
+
+# ----------------------------------------------------------------------------
+# prompts for compaction
+# ----------------------------------------------------------------------------
+@dataclasses.dataclass
+class PromptCase:
+    table: torch.Tensor          # [V][d] bf16
+    token_ids: torch.Tensor      # [B][L] int32
+    span_offsets: torch.Tensor   # [B+1]
+    span_start: torch.Tensor     # [S] position within its prompt
+    span_len: torch.Tensor       # [S]
+    span_token_ids: torch.Tensor  # [T] span tokens concatenated (merge-module input)
+    span_token_offsets: torch.Tensor  # [S+1]
+
+
+def prompt_case(seed: int, *, B: int, L: int, vocab: int, d: int, coverage: float,
+                kmin: int = 2, kmax: int = 4, device="cpu", table=None) -> PromptCase:
+    r = rng(seed)
+    ids = r.integers(0, vocab, size=(B, L)).astype(np.int32)
+    starts, slens, offs = [], [], [0]
+    for b in range(B):
+        st, ln = span_layout(r, L, coverage=coverage, kmin=kmin, kmax=kmax)
+        starts.append(st)
+        slens.append(ln)
+        offs.append(offs[-1] + len(st))
+    span_start = np.concatenate(starts).astype(np.int32)
+    span_len = np.concatenate(slens).astype(np.int32)
+    toks, toffs = [], [0]
+    i = 0
+    for b in range(B):
+        for j in range(offs[b], offs[b + 1]):
+            s, k = int(span_start[j]), int(span_len[j])
+            toks.append(ids[b, s:s + k])
+            toffs.append(toffs[-1] + k)
+    span_tokens = np.concatenate(toks).astype(np.int32) if toks else np.zeros(0, np.int32)
+    if table is None:
+        table = bf16_normal((vocab, d), 0.02, seed + 101, device)
+    t = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(device)
+    return PromptCase(table=table, token_ids=t(ids), span_offsets=t(np.asarray(offs, np.int32)),
+                      span_start=t(span_start), span_len=t(span_len),
+                      span_token_ids=t(span_tokens),
+                      span_token_offsets=t(np.asarray(toffs, np.int32)))
+
+
+# ----------------------------------------------------------------------------
+# serving-loop lengths
+# ----------------------------------------------------------------------------
+def serving_lengths(r: np.random.Generator, B: int, median: int = 1024, sigma: float = 1.0,
+                    lo: int = 256, hi: int = 8192) -> np.ndarray:
+    x = np.exp(np.log(median) + sigma * r.standard_normal(B))
+    return np.clip(np.round(x), lo, hi).astype(np.int32)
