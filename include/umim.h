@@ -1,0 +1,238 @@
+/*
+ * umim.h - C ABI of libumim, a GB300 (sm_103a) implementation of the decode
+ * step over a merged context of UMIM (arXiv 2609.27233, "Distilling
+ * Sequential Computation in Transformer Language Models").
+ *
+ * The step has three parts, each a call below:
+ *   umim_merge_spans       merge module M_phi: span of static token
+ *                          embeddings -> one surrogate embedding
+ *                          (Sec. 3.2 Eq. 1, App. C.1)
+ *   umim_kv_rollback       replace each span's stored KV entries by one
+ *                          surrogate entry and compact the paged cache
+ *                          (App. C.6, App. E "Decoding-Time Merging and
+ *                          KV-Cache Update", Fig. 2)
+ *   umim_decode_attention  grouped-query decode attention over the shorter,
+ *                          compacted paged cache (App. I.1)
+ * and one call for the prompt side:
+ *   umim_build_compressed  packed compressed prompt embeddings with
+ *                          contiguous positions (App. C.5, App. E "Prompt
+ *                          Merging", App. J.4)
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ *  - Pointers named *device* point to GPU memory of the current device; the
+ *    caller allocates and owns every buffer, including the workspace.  The
+ *    library never allocates GPU memory.
+ *  - Every call is asynchronous on `stream`.  The returned umim_status only
+ *    reports what the host can check (null pointers, unsupported shapes, a
+ *    workspace that is too small, a failed launch).  Checks that need device
+ *    data (span lists, token ids, block-table entries) and bounded waits run
+ *    on the GPU and record the first failure in `*dev_status` (a device
+ *    int32 the caller zeroes; NULL means "use a word inside the workspace and
+ *    do not report").  Read it after synchronising the stream.
+ *  - bf16 means IEEE bfloat16 (raw 16-bit patterns); fp32 is IEEE binary32.
+ *  - Paged KV cache: pages of UMIM_PAGE_SIZE (16) entries; one entry holds
+ *    K and V of every KV head of one token position for one layer.
+ *    Layout of the pool, bf16, row-major:
+ *        [n_layers][n_pages][2 (K, V)][n_kv_heads][16][head_dim]
+ *    so one (layer, page, K|V, head) tile of 16 x head_dim values is
+ *    contiguous.  A block table row lists, for logical page p of a sequence,
+ *    the physical page id (or -1 for none).  Entry t of a sequence lives in
+ *    page block_table[t / 16], slot t % 16.
+ *  - Supported: head_dim 64 or 128, page size 16, 1 <= n_q_heads/n_kv_heads
+ *    <= 16, d_model a multiple of 512 (<= 16384), n_heads in {1, 2, 4, 8},
+ *    merge spans of 1..4 tokens.
+ *    Anything else returns UMIM_ERR_UNSUPPORTED.
+ */
+#ifndef UMIM_H_
+#define UMIM_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#include <cuda_runtime_api.h> /* cudaStream_t */
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define UMIM_PAGE_SIZE 16
+#define UMIM_MAX_SPAN_TOKENS 4
+
+typedef enum umim_status {
+  UMIM_OK = 0,
+  UMIM_ERR_INVALID_ARG = 1, /* bad pointer, size, span list, id or page */
+  UMIM_ERR_UNSUPPORTED = 2, /* shape outside the supported set above     */
+  UMIM_ERR_CUDA = 3,        /* a CUDA runtime / driver call failed       */
+  UMIM_ERR_TIMEOUT = 4,     /* a bounded device-side wait gave up        */
+  UMIM_ERR_WORKSPACE = 5    /* workspace pointer or size insufficient    */
+} umim_status;
+
+/* Human-readable name of a status code (static string). */
+const char *umim_status_string(int status);
+
+/* Library version as 10000*major + 100*minor + patch. */
+int umim_version(void);
+
+/* Merge-module parameters phi (App. C.3: |phi| = 2 d^2 + 7 d), all bf16
+ * device arrays, Linear weights stored W[out][in] row-major. */
+typedef struct umim_merge_weights {
+  const void *w_kv;        /* [d][d]   W^{kv}                              */
+  const void *b_kv;        /* [d]      b^{kv}                              */
+  const void *ln_kv_gamma; /* [d]      LN_kv scale                         */
+  const void *ln_kv_beta;  /* [d]      LN_kv shift                         */
+  const void *query;       /* [h][d/h] learnable queries q_i, one per head */
+  const void *w_o;         /* [d][d]   W^{o}                               */
+  const void *b_o;         /* [d]                                          */
+  const void *ln_o_gamma;  /* [d]                                          */
+  const void *ln_o_beta;   /* [d]                                          */
+  int32_t d_model;         /* d                                            */
+  int32_t n_heads;         /* h (the paper uses 4)                         */
+  float ln_eps;            /* LayerNorm epsilon (1e-5 when not trained otherwise) */
+} umim_merge_weights;
+
+/* A paged bf16 KV cache (layout in the header comment). */
+typedef struct umim_paged_kv {
+  void *base;         /* device pool                                   */
+  int32_t n_layers;
+  int32_t n_pages;    /* physical pages per layer                      */
+  int32_t n_kv_heads;
+  int32_t page_size;  /* must be UMIM_PAGE_SIZE                         */
+  int32_t head_dim;   /* 64 or 128                                     */
+} umim_paged_kv;
+
+/* ------------------------------------------------------------------------
+ * Merge module forward (Sec. 3.2 Eq. 1; App. C.1 full form):
+ *   P   = LN_kv(GELU(E_s W_kv^T + b_kv)),  P = [P_1 .. P_h]
+ *   a_i = softmax(P_i q_i / sqrt(d/h)),  o_i = a_i^T P_i
+ *   z_s = LN_o(GELU(W_o [o_1; ..; o_h] + b_o))
+ * GELU is the erf form, LayerNorm uses the biased variance.
+ *
+ * embeddings    device bf16 [vocab][d]  static embedding table e(.)
+ * token_ids     device int32 [n_tokens] the span tokens, concatenated
+ * span_offsets  device int32 [n_spans+1] CSR: span s = token_ids[off[s]..off[s+1])
+ *               (1 <= off[s+1]-off[s] <= 4 is checked on the device)
+ * surrogates    device fp32 [n_spans][d] output z_s
+ * workspace     device, umim_merge_spans_workspace_size() bytes, 256-B aligned
+ * Device-side errors: UMIM_ERR_INVALID_ARG for a token id outside [0, vocab)
+ * (that token reads as zeros) or a malformed span (its z is then computed
+ * from an all-zero pooled vector).
+ * ------------------------------------------------------------------------ */
+size_t umim_merge_spans_workspace_size(int64_t n_tokens, int32_t n_spans, int32_t d_model);
+
+umim_status umim_merge_spans(const void *embeddings, int64_t vocab, const int32_t *token_ids,
+                             int64_t n_tokens, const int32_t *span_offsets, int32_t n_spans,
+                             const umim_merge_weights *weights, float *surrogates, void *workspace,
+                             size_t workspace_bytes, int32_t *dev_status, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Compressed prompt (App. E "Prompt Merging", App. C.5, App. J.4): every
+ * span of prompt b is replaced by bf16(z) (round to nearest even) and every
+ * other token by its embedding row, in order; prompts are packed back to
+ * back; position ids restart at 0 for every prompt (contiguous compressed
+ * positions); cu_seqlens[b] is the first row of prompt b,
+ * cu_seqlens[batch] = total rows = sum_b (L - sum (k - 1)).
+ *
+ * embeddings    device bf16 [vocab][d]
+ * token_ids     device int32 [batch][prompt_len]
+ * span_offsets  device int32 [batch+1] CSR over prompts
+ * span_start    device int32 [n_spans] first position of each span inside its prompt
+ * span_len      device int32 [n_spans] tokens per span (>= 1); spans of a prompt
+ *               sorted, non-overlapping, inside the prompt
+ * surrogates    device fp32 [n_spans][d] (as returned by umim_merge_spans)
+ * out_embeds    device bf16 [out_capacity_rows][d]
+ * position_ids  device int32 [out_capacity_rows]
+ * cu_seqlens    device int32 [batch+1]
+ * workspace     device, umim_build_compressed_workspace_size() bytes, 256-B
+ *               aligned, zero-filled before its first use, then reused
+ * Device-side errors: UMIM_ERR_INVALID_ARG for a bad span list or token id,
+ * or when the compressed rows exceed out_capacity_rows (nothing is written
+ * to out_embeds / position_ids then).
+ * ------------------------------------------------------------------------ */
+size_t umim_build_compressed_workspace_size(int32_t batch, int32_t n_spans);
+
+umim_status umim_build_compressed(const void *embeddings, int64_t vocab, int32_t d_model,
+                                  const int32_t *token_ids, int32_t batch, int32_t prompt_len,
+                                  const int32_t *span_offsets, const int32_t *span_start,
+                                  const int32_t *span_len, int32_t n_spans, const float *surrogates,
+                                  void *out_embeds, int64_t out_capacity_rows, int32_t *position_ids,
+                                  int32_t *cu_seqlens, void *workspace, size_t workspace_bytes,
+                                  int32_t *dev_status, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
+ * KV-cache rollback and compaction (App. E "Decoding-Time Merging and
+ * KV-Cache Update": the cached entries of a merged span are cropped and the
+ * surrogate's single KV state takes their place, L' = L - (n-1) + 1; Fig. 2).
+ * Generalised to any number of sorted, non-overlapping spans per sequence:
+ * each span (s, k) of sequence b replaces its k stored entries, in every
+ * layer, by one entry holding surrogate_k/v[span]; the entries after it
+ * move left.  The result is written IN PLACE into the sequence's own pages
+ * in logical order (new entry j -> page block_table[b][j/16], slot j%16).
+ * Block-table entries p in [ceil(L'/16), ceil(L/16)) are reported in
+ * freed_pages (sequence after sequence, ascending p) and set to -1;
+ * seq_lens[b] becomes L' = L - sum (k - 1).  Slots at or after L' in the
+ * last page keep unspecified contents.  Entries before a sequence's first
+ * span are never read or written.
+ *
+ * kv            host struct describing the device pool (read and written)
+ * block_table   device int32 [batch][max_pages], in/out
+ * seq_lens      device int32 [batch], in/out
+ * span_offsets  device int32 [batch+1] CSR over sequences
+ * span_start    device int32 [n_spans] first replaced entry (logical index)
+ * span_len      device int32 [n_spans] k = stored entries replaced (>= 1);
+ *               the paper's n-1 when the newest token is not cached yet
+ * surrogate_k/v device bf16 [n_spans][n_layers][n_kv_heads][head_dim]
+ * freed_pages   device int32 [batch*max_pages] out, -1 terminated when not
+ *               full; may be NULL
+ * workspace     device, umim_kv_rollback_workspace_size() bytes, 256-B
+ *               aligned, ZERO-FILLED BEFORE ITS FIRST USE and then reused
+ *               unchanged between calls (it carries a call counter)
+ * Preconditions checked on the device before anything is written (a
+ * violation records UMIM_ERR_INVALID_ARG and leaves every buffer
+ * untouched): 0 <= seq_lens[b] <= 16*max_pages; spans sorted,
+ * non-overlapping, k >= 1, s >= 0, s + k <= seq_lens[b]; block-table
+ * entries of used pages in [0, n_pages).  Not checked: that no physical
+ * page is shared by two sequences.  UMIM_ERR_TIMEOUT leaves the cache
+ * contents unspecified.
+ * ------------------------------------------------------------------------ */
+size_t umim_kv_rollback_workspace_size(int32_t batch, int32_t n_spans, int32_t max_pages, int32_t n_layers,
+                                       int32_t n_kv_heads, int32_t head_dim);
+
+umim_status umim_kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t max_pages,
+                             int32_t *seq_lens, int32_t batch, const int32_t *span_offsets,
+                             const int32_t *span_start, const int32_t *span_len, int32_t n_spans,
+                             const void *surrogate_k, const void *surrogate_v, int32_t *freed_pages,
+                             void *workspace, size_t workspace_bytes, int32_t *dev_status,
+                             cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Grouped-query decode attention over the (compacted) paged cache, one
+ * query token per sequence (App. I.1; the backbone's ordinary attention):
+ *   out[b][h] = sum_{j < seq_lens[b]} softmax_j(scale <q[b][h], K[b][g][j]>) V[b][g][j]
+ *   g = h / (n_q_heads / n_kv_heads),  scale = 1/sqrt(head_dim) when 0 is given.
+ * A sequence with seq_lens[b] == 0 gets a zero output.  Reads only: the
+ * cache, block table and lengths are not modified.
+ *
+ * q             device bf16 [batch][n_q_heads][head_dim]
+ * kv, layer     cache and the layer to read
+ * block_table   device int32 [batch][max_pages]
+ * seq_lens      device int32 [batch]
+ * out           device bf16 [batch][n_q_heads][head_dim]
+ * workspace     device, umim_decode_attention_workspace_size() bytes, 256-B aligned
+ * Device-side errors: UMIM_ERR_INVALID_ARG for seq_lens[b] outside
+ * [0, 16*max_pages] or a used block-table entry outside [0, n_pages)
+ * (that page reads as zeros), UMIM_ERR_TIMEOUT for a stalled copy.
+ * ------------------------------------------------------------------------ */
+size_t umim_decode_attention_workspace_size(int32_t batch, int32_t n_q_heads, int32_t n_kv_heads,
+                                            int32_t head_dim);
+
+umim_status umim_decode_attention(const void *q, int32_t n_q_heads, const umim_paged_kv *kv, int32_t layer,
+                                  const int32_t *block_table, int32_t max_pages, const int32_t *seq_lens,
+                                  int32_t batch, float scale, void *out, void *workspace,
+                                  size_t workspace_bytes, int32_t *dev_status, cudaStream_t stream);
+
+#ifdef __cplusplus
+} /* extern "C" */
+#endif
+
+#endif /* UMIM_H_ */

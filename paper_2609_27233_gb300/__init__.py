@@ -1,0 +1,193 @@
+"""Python binding of libumim (GB300 / sm_103a), the decode step over a merged
+context of UMIM (arXiv 2609.27233).
+
+Thin argument marshalling only: every step runs in the library's CUDA
+kernels.  PyTorch provides device memory and the current stream.  The entry
+points keep the C names:
+
+  umim_merge_spans        merge module M_phi (Sec. 3.2 Eq. 1, App. C.1)
+  umim_build_compressed   compressed prompt embeddings + positions (App. E, App. C.5)
+  umim_kv_rollback        KV-cache rollback and in-place compaction (App. E, Fig. 2)
+  umim_decode_attention   GQA decode attention over the compacted paged cache (App. I.1)
+"""
+import ctypes
+
+import torch
+
+from . import _lib
+from ._lib import MergeWeightsC, PagedKVC
+
+UMIM_OK = 0
+STATUS = {0: "UMIM_OK", 1: "UMIM_ERR_INVALID_ARG", 2: "UMIM_ERR_UNSUPPORTED", 3: "UMIM_ERR_CUDA",
+          4: "UMIM_ERR_TIMEOUT", 5: "UMIM_ERR_WORKSPACE"}
+PAGE_SIZE = 16
+
+
+class UmimError(RuntimeError):
+    def __init__(self, code, where=""):
+        self.code = int(code)
+        super().__init__(f"{where}: {STATUS.get(self.code, self.code)}")
+
+
+def lib():
+    return _lib.load()
+
+
+def _p(t):
+    return ctypes.c_void_p(0 if t is None else t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _check(code, where):
+    if code != UMIM_OK:
+        raise UmimError(code, where)
+
+
+def _dev(t):
+    if not t.is_cuda:
+        raise ValueError("expected a CUDA tensor")
+    return t.device
+
+
+def new_status(device):
+    """A zeroed device int32 that receives device-side errors."""
+    return torch.zeros(1, dtype=torch.int32, device=device)
+
+
+def check_status(dev_status, where="device"):
+    v = int(dev_status.item())
+    if v != UMIM_OK:
+        raise UmimError(v, where)
+
+
+def workspace(nbytes, device):
+    """A zero-filled, 256-byte aligned device workspace of at least nbytes."""
+    return torch.zeros(max(int(nbytes), 256), dtype=torch.uint8, device=device)
+
+
+def paged_kv(pool):
+    """umim_paged_kv for a bf16 pool shaped [layers][pages][2][Hkv][16][D]."""
+    if pool.dtype != torch.bfloat16 or pool.dim() != 6 or pool.shape[2] != 2 or not pool.is_contiguous():
+        raise ValueError("pool must be contiguous bf16 [layers][pages][2][Hkv][16][D]")
+    return PagedKVC(pool.data_ptr(), pool.shape[0], pool.shape[1], pool.shape[3], pool.shape[4], pool.shape[5])
+
+
+def merge_weights_c(w):
+    g = (lambda k: getattr(w, k)) if not isinstance(w, dict) else (lambda k: w[k])
+    names = ("w_kv", "b_kv", "ln_kv_gamma", "ln_kv_beta", "query", "w_o", "b_o", "ln_o_gamma", "ln_o_beta")
+    for k in names:
+        t = g(k)
+        if t.dtype != torch.bfloat16 or not t.is_contiguous():
+            raise ValueError(f"merge weight {k} must be contiguous bf16")
+    return MergeWeightsC(*[g(k).data_ptr() for k in names], int(g("d_model")), int(g("n_heads")),
+                         float(g("ln_eps")))
+
+
+# ---------------------------------------------------------------------------
+# workspace sizes
+# ---------------------------------------------------------------------------
+def umim_merge_spans_workspace_size(n_tokens, n_spans, d_model):
+    return int(lib().umim_merge_spans_workspace_size(n_tokens, n_spans, d_model))
+
+
+def umim_build_compressed_workspace_size(batch, n_spans):
+    return int(lib().umim_build_compressed_workspace_size(batch, n_spans))
+
+
+def umim_kv_rollback_workspace_size(batch, n_spans, max_pages, n_layers, n_kv_heads, head_dim):
+    return int(lib().umim_kv_rollback_workspace_size(batch, n_spans, max_pages, n_layers, n_kv_heads, head_dim))
+
+
+def umim_decode_attention_workspace_size(batch, n_q_heads, n_kv_heads, head_dim):
+    return int(lib().umim_decode_attention_workspace_size(batch, n_q_heads, n_kv_heads, head_dim))
+
+
+# ---------------------------------------------------------------------------
+# the four calls
+# ---------------------------------------------------------------------------
+def umim_merge_spans(embeddings, token_ids, span_offsets, weights, surrogates=None, workspace_buf=None,
+                     dev_status=None, stream=None):
+    """Surrogate embeddings z (fp32 [S][d]) of the spans in CSR form."""
+    dev = _dev(embeddings)
+    d = embeddings.shape[1]
+    S = span_offsets.numel() - 1
+    T = token_ids.numel()
+    if surrogates is None:
+        surrogates = torch.empty((S, d), dtype=torch.float32, device=dev)
+    if workspace_buf is None:
+        workspace_buf = workspace(umim_merge_spans_workspace_size(T, S, d), dev)
+    wc = merge_weights_c(weights)
+    code = lib().umim_merge_spans(_p(embeddings), embeddings.shape[0], _p(token_ids), T, _p(span_offsets), S,
+                                  ctypes.byref(wc), _p(surrogates), _p(workspace_buf), workspace_buf.numel(),
+                                  _p(dev_status), _stream(stream))
+    _check(code, "umim_merge_spans")
+    return surrogates
+
+
+def umim_build_compressed(embeddings, token_ids, span_offsets, span_start, span_len, surrogates,
+                          out_embeds=None, position_ids=None, cu_seqlens=None, workspace_buf=None,
+                          dev_status=None, stream=None):
+    """(out_embeds [rows][d] bf16, position_ids [rows], cu_seqlens [B+1]); the
+    first cu_seqlens[-1] rows are the packed compressed prompts."""
+    dev = _dev(embeddings)
+    B, L = token_ids.shape
+    d = embeddings.shape[1]
+    S = span_start.numel()
+    if out_embeds is None:
+        out_embeds = torch.empty((B * L, d), dtype=torch.bfloat16, device=dev)
+    if position_ids is None:
+        position_ids = torch.empty(out_embeds.shape[0], dtype=torch.int32, device=dev)
+    if cu_seqlens is None:
+        cu_seqlens = torch.empty(B + 1, dtype=torch.int32, device=dev)
+    if workspace_buf is None:
+        workspace_buf = workspace(umim_build_compressed_workspace_size(B, S), dev)
+    code = lib().umim_build_compressed(_p(embeddings), embeddings.shape[0], d, _p(token_ids), B, L,
+                                       _p(span_offsets), _p(span_start), _p(span_len), S, _p(surrogates),
+                                       _p(out_embeds), out_embeds.shape[0], _p(position_ids), _p(cu_seqlens),
+                                       _p(workspace_buf), workspace_buf.numel(), _p(dev_status), _stream(stream))
+    _check(code, "umim_build_compressed")
+    return out_embeds, position_ids, cu_seqlens
+
+
+def umim_kv_rollback(pool, block_table, seq_lens, span_offsets, span_start, span_len, surrogate_k, surrogate_v,
+                     freed_pages=None, workspace_buf=None, dev_status=None, stream=None):
+    """In-place rollback of pool / block_table / seq_lens; returns freed_pages
+    (device int32 [B*max_pages], -1 terminated)."""
+    dev = _dev(pool)
+    kv = paged_kv(pool)
+    B, max_pages = block_table.shape
+    S = span_start.numel()
+    if freed_pages is None:
+        freed_pages = torch.empty(max(1, B * max_pages), dtype=torch.int32, device=dev)
+    if workspace_buf is None:
+        workspace_buf = workspace(umim_kv_rollback_workspace_size(B, S, max_pages, kv.n_layers, kv.n_kv_heads,
+                                                                  kv.head_dim), dev)
+    code = lib().umim_kv_rollback(ctypes.byref(kv), _p(block_table), max_pages, _p(seq_lens), B, _p(span_offsets),
+                                  _p(span_start), _p(span_len), S, _p(surrogate_k), _p(surrogate_v),
+                                  _p(freed_pages), _p(workspace_buf), workspace_buf.numel(), _p(dev_status),
+                                  _stream(stream))
+    _check(code, "umim_kv_rollback")
+    return freed_pages
+
+
+def umim_decode_attention(q, pool, layer, block_table, seq_lens, scale=0.0, out=None, workspace_buf=None,
+                          dev_status=None, stream=None):
+    """out [B][Hq][D] bf16 = GQA attention of q over the paged cache."""
+    dev = _dev(q)
+    kv = paged_kv(pool)
+    B, Hq, D = q.shape
+    max_pages = block_table.shape[1]
+    if out is None:
+        out = torch.empty_like(q)
+    if workspace_buf is None:
+        workspace_buf = workspace(umim_decode_attention_workspace_size(B, Hq, kv.n_kv_heads, D), dev)
+    code = lib().umim_decode_attention(_p(q), Hq, ctypes.byref(kv), layer, _p(block_table), max_pages,
+                                       _p(seq_lens), B, float(scale), _p(out), _p(workspace_buf),
+                                       workspace_buf.numel(), _p(dev_status), _stream(stream))
+    _check(code, "umim_decode_attention")
+    return out

@@ -1,0 +1,71 @@
+"""ctypes declarations of libumim's C ABI (include/umim.h).
+
+Loading fails loudly when the shared library has not been built: there is
+no CPU or PyTorch fallback for any call.
+"""
+import ctypes
+import os
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libumim.so")
+
+c_i32 = ctypes.c_int32
+c_i64 = ctypes.c_int64
+c_ptr = ctypes.c_void_p
+c_size = ctypes.c_size_t
+
+
+class MergeWeightsC(ctypes.Structure):
+    _fields_ = [
+        ("w_kv", c_ptr), ("b_kv", c_ptr), ("ln_kv_gamma", c_ptr), ("ln_kv_beta", c_ptr),
+        ("query", c_ptr), ("w_o", c_ptr), ("b_o", c_ptr), ("ln_o_gamma", c_ptr), ("ln_o_beta", c_ptr),
+        ("d_model", c_i32), ("n_heads", c_i32), ("ln_eps", ctypes.c_float),
+    ]
+
+
+class PagedKVC(ctypes.Structure):
+    _fields_ = [
+        ("base", c_ptr), ("n_layers", c_i32), ("n_pages", c_i32), ("n_kv_heads", c_i32),
+        ("page_size", c_i32), ("head_dim", c_i32),
+    ]
+
+
+# name -> (restype, argtypes), exactly as declared in include/umim.h
+SIGNATURES = {
+    "umim_status_string": (ctypes.c_char_p, [ctypes.c_int]),
+    "umim_version": (ctypes.c_int, []),
+    "umim_merge_spans_workspace_size": (c_size, [c_i64, c_i32, c_i32]),
+    "umim_merge_spans": (ctypes.c_int, [c_ptr, c_i64, c_ptr, c_i64, c_ptr, c_i32,
+                                        ctypes.POINTER(MergeWeightsC), c_ptr, c_ptr, c_size, c_ptr, c_ptr]),
+    "umim_build_compressed_workspace_size": (c_size, [c_i32, c_i32]),
+    "umim_build_compressed": (ctypes.c_int, [c_ptr, c_i64, c_i32, c_ptr, c_i32, c_i32, c_ptr, c_ptr, c_ptr,
+                                             c_i32, c_ptr, c_ptr, c_i64, c_ptr, c_ptr, c_ptr, c_size, c_ptr,
+                                             c_ptr]),
+    "umim_kv_rollback_workspace_size": (c_size, [c_i32, c_i32, c_i32, c_i32, c_i32, c_i32]),
+    "umim_kv_rollback": (ctypes.c_int, [ctypes.POINTER(PagedKVC), c_ptr, c_i32, c_ptr, c_i32, c_ptr, c_ptr,
+                                        c_ptr, c_i32, c_ptr, c_ptr, c_ptr, c_ptr, c_size, c_ptr, c_ptr]),
+    "umim_decode_attention_workspace_size": (c_size, [c_i32, c_i32, c_i32, c_i32]),
+    "umim_decode_attention": (ctypes.c_int, [c_ptr, c_i32, ctypes.POINTER(PagedKVC), c_i32, c_ptr, c_i32,
+                                             c_ptr, c_i32, ctypes.c_float, c_ptr, c_ptr, c_size, c_ptr,
+                                             c_ptr]),
+}
+
+_lib = None
+
+
+def load(path: str = LIB_PATH):
+    """Load libumim.so and declare every entry point; raises if it is missing."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise RuntimeError(
+            f"libumim.so not found at {path}: build it first "
+            "(python -c 'import __graft_entry__ as g; g.build()')")
+    lib = ctypes.CDLL(path)
+    for name, (res, args) in SIGNATURES.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    _lib = lib
+    return lib

@@ -1,0 +1,220 @@
+// C ABI of libumim: host-side argument checks, then the kernels of each part.
+#include <algorithm>
+#include <cstring>
+#include <mutex>
+
+#include "common.cuh"
+
+namespace umim {
+
+using EncodeTiledFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                   const cuuint64_t *, const cuuint32_t *, const cuuint32_t *,
+                                   CUtensorMapInterleave, CUtensorMapSwizzle, CUtensorMapL2promotion,
+                                   CUtensorMapFloatOOBfill);
+
+// cuTensorMapEncodeTiled through the runtime's driver entry point (no -lcuda)
+EncodeTiledFn get_encode_tiled() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void *p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  return fn;
+}
+
+// internal entry points (one translation unit per part)
+size_t merge_spans_workspace_bytes(int64_t T, int S, int d);
+umim_status merge_spans(const void *, int64_t, const int32_t *, int64_t, const int32_t *, int,
+                        const umim_merge_weights *, float *, void *, int32_t *, cudaStream_t, int);
+size_t build_compressed_workspace_bytes(int B, int S);
+umim_status build_compressed(const void *, int64_t, int, const int32_t *, int, int, const int32_t *,
+                             const int32_t *, const int32_t *, int, const float *, void *, int64_t, int32_t *,
+                             int32_t *, void *, int32_t *, cudaStream_t, int);
+size_t kv_rollback_workspace_bytes(int B, int S, int max_pages, int n_layers, int n_kv_heads, int head_dim);
+umim_status kv_rollback(const umim_paged_kv *, int32_t *, int32_t, int32_t *, int32_t, const int32_t *,
+                        const int32_t *, const int32_t *, int32_t, const void *, const void *, int32_t *, void *,
+                        size_t, int32_t *, cudaStream_t, int);
+size_t decode_attention_workspace_bytes(int B, int Hq, int Hkv, int D, int num_sms);
+umim_status decode_attention(const void *, int, const umim_paged_kv *, int, const int32_t *, int, const int32_t *,
+                             int, float, void *, void *, int32_t *, cudaStream_t, int);
+
+namespace {
+
+// Make the stream's device current for this runtime instance; return its SM count.
+int prepare_device(cudaStream_t stream) {
+  int dev = 0;
+  if (stream != nullptr && cudaStreamGetDevice(stream, &dev) == cudaSuccess) cudaSetDevice(dev);
+  else cudaGetDevice(&dev);
+  static int cached_dev = -1, cached_sms = 0;
+  if (dev != cached_dev) {
+    int sms = 0;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) sms = 0;
+    cached_sms = sms;
+    cached_dev = dev;
+  }
+  return cached_sms;
+}
+
+int current_sms() {
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+  return sms;
+}
+
+bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+bool kv_ok(const umim_paged_kv *kv) {
+  return kv && kv->base && kv->n_layers > 0 && kv->n_pages > 0 && kv->n_kv_heads > 0 && aligned(kv->base, 16);
+}
+
+bool kv_supported(const umim_paged_kv *kv) {
+  return kv->page_size == UMIM_PAGE_SIZE && (kv->head_dim == 64 || kv->head_dim == 128) && kv->n_kv_heads <= 64;
+}
+
+bool merge_supported(int d, int h) {
+  return d > 0 && d % 512 == 0 && d <= 16384 && (h == 1 || h == 2 || h == 4 || h == 8);
+}
+
+}  // namespace
+}  // namespace umim
+
+using namespace umim;
+
+extern "C" {
+
+const char *umim_status_string(int s) {
+  switch (s) {
+    case UMIM_OK: return "UMIM_OK";
+    case UMIM_ERR_INVALID_ARG: return "UMIM_ERR_INVALID_ARG";
+    case UMIM_ERR_UNSUPPORTED: return "UMIM_ERR_UNSUPPORTED";
+    case UMIM_ERR_CUDA: return "UMIM_ERR_CUDA";
+    case UMIM_ERR_TIMEOUT: return "UMIM_ERR_TIMEOUT";
+    case UMIM_ERR_WORKSPACE: return "UMIM_ERR_WORKSPACE";
+    default: return "UMIM_ERR_UNKNOWN";
+  }
+}
+
+int umim_version(void) { return 100; }
+
+size_t umim_merge_spans_workspace_size(int64_t n_tokens, int32_t n_spans, int32_t d_model) {
+  if (n_tokens < 0 || n_spans < 0 || d_model <= 0) return 0;
+  return merge_spans_workspace_bytes(n_tokens, n_spans, d_model);
+}
+
+umim_status umim_merge_spans(const void *embeddings, int64_t vocab, const int32_t *token_ids, int64_t n_tokens,
+                             const int32_t *span_offsets, int32_t n_spans, const umim_merge_weights *w,
+                             float *surrogates, void *workspace, size_t workspace_bytes, int32_t *dev_status,
+                             cudaStream_t stream) {
+  if (!w || n_spans < 0 || n_tokens < 0 || vocab <= 0) return UMIM_ERR_INVALID_ARG;
+  if (!merge_supported(w->d_model, w->n_heads)) return UMIM_ERR_UNSUPPORTED;
+  if (n_tokens > (int64_t)n_spans * UMIM_MAX_SPAN_TOKENS || n_tokens > INT32_MAX) return UMIM_ERR_INVALID_ARG;
+  if (n_spans == 0) return UMIM_OK;
+  if (!embeddings || !span_offsets || !surrogates || (n_tokens > 0 && !token_ids)) return UMIM_ERR_INVALID_ARG;
+  if (!w->w_kv || !w->b_kv || !w->ln_kv_gamma || !w->ln_kv_beta || !w->query || !w->w_o || !w->b_o ||
+      !w->ln_o_gamma || !w->ln_o_beta)
+    return UMIM_ERR_INVALID_ARG;
+  if (!aligned(embeddings, 16) || !aligned(w->w_kv, 16) || !aligned(w->w_o, 16) || !aligned(surrogates, 16))
+    return UMIM_ERR_INVALID_ARG;
+  if (!workspace || !aligned(workspace, 256) ||
+      workspace_bytes < merge_spans_workspace_bytes(n_tokens, n_spans, w->d_model))
+    return UMIM_ERR_WORKSPACE;
+  const int sms = prepare_device(stream);
+  return merge_spans(embeddings, vocab, token_ids, n_tokens, span_offsets, n_spans, w, surrogates, workspace,
+                     dev_status, stream, sms);
+}
+
+size_t umim_build_compressed_workspace_size(int32_t batch, int32_t n_spans) {
+  if (batch < 0 || n_spans < 0) return 0;
+  return build_compressed_workspace_bytes(batch, n_spans);
+}
+
+umim_status umim_build_compressed(const void *embeddings, int64_t vocab, int32_t d_model, const int32_t *token_ids,
+                                  int32_t batch, int32_t prompt_len, const int32_t *span_offsets,
+                                  const int32_t *span_start, const int32_t *span_len, int32_t n_spans,
+                                  const float *surrogates, void *out_embeds, int64_t out_capacity_rows,
+                                  int32_t *position_ids, int32_t *cu_seqlens, void *workspace,
+                                  size_t workspace_bytes, int32_t *dev_status, cudaStream_t stream) {
+  if (batch < 0 || prompt_len < 0 || n_spans < 0 || vocab <= 0 || out_capacity_rows < 0)
+    return UMIM_ERR_INVALID_ARG;
+  if (d_model <= 0 || d_model % 8 != 0) return UMIM_ERR_UNSUPPORTED;
+  if ((int64_t)batch * prompt_len > INT32_MAX) return UMIM_ERR_UNSUPPORTED;
+  if (batch == 0) return UMIM_OK;
+  if (!embeddings || !token_ids || !span_offsets || !out_embeds || !position_ids || !cu_seqlens)
+    return UMIM_ERR_INVALID_ARG;
+  if (n_spans > 0 && (!span_start || !span_len || !surrogates)) return UMIM_ERR_INVALID_ARG;
+  if (!aligned(embeddings, 16) || !aligned(out_embeds, 16) || (surrogates && !aligned(surrogates, 16)))
+    return UMIM_ERR_INVALID_ARG;
+  if (!workspace || !aligned(workspace, 256) || workspace_bytes < build_compressed_workspace_bytes(batch, n_spans))
+    return UMIM_ERR_WORKSPACE;
+  const int sms = prepare_device(stream);
+  return build_compressed(embeddings, vocab, d_model, token_ids, batch, prompt_len, span_offsets, span_start,
+                          span_len, n_spans, surrogates, out_embeds, out_capacity_rows, position_ids, cu_seqlens,
+                          workspace, dev_status, stream, sms);
+}
+
+size_t umim_kv_rollback_workspace_size(int32_t batch, int32_t n_spans, int32_t max_pages, int32_t n_layers,
+                                       int32_t n_kv_heads, int32_t head_dim) {
+  if (batch < 0 || n_spans < 0 || max_pages < 0 || n_layers <= 0 || n_kv_heads <= 0 ||
+      (head_dim != 64 && head_dim != 128))
+    return 0;
+  return kv_rollback_workspace_bytes(batch, n_spans, max_pages, n_layers, n_kv_heads, head_dim);
+}
+
+umim_status umim_kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t max_pages, int32_t *seq_lens,
+                             int32_t batch, const int32_t *span_offsets, const int32_t *span_start,
+                             const int32_t *span_len, int32_t n_spans, const void *surrogate_k,
+                             const void *surrogate_v, int32_t *freed_pages, void *workspace,
+                             size_t workspace_bytes, int32_t *dev_status, cudaStream_t stream) {
+  if (!kv_ok(kv) || batch < 0 || max_pages < 0 || n_spans < 0) return UMIM_ERR_INVALID_ARG;
+  if (!kv_supported(kv)) return UMIM_ERR_UNSUPPORTED;
+  if ((int64_t)batch * max_pages > INT32_MAX / 16) return UMIM_ERR_UNSUPPORTED;
+  if (batch == 0) return UMIM_OK;
+  if (!block_table || !seq_lens || !span_offsets) return UMIM_ERR_INVALID_ARG;
+  if (n_spans > 0 && (!span_start || !span_len || !surrogate_k || !surrogate_v)) return UMIM_ERR_INVALID_ARG;
+  if (n_spans > 0 && (!aligned(surrogate_k, 16) || !aligned(surrogate_v, 16))) return UMIM_ERR_INVALID_ARG;
+  if (!workspace || !aligned(workspace, 256) ||
+      workspace_bytes < kv_rollback_workspace_bytes(batch, n_spans, max_pages, kv->n_layers, kv->n_kv_heads,
+                                                    kv->head_dim))
+    return UMIM_ERR_WORKSPACE;
+  const int sms = prepare_device(stream);
+  return kv_rollback(kv, block_table, max_pages, seq_lens, batch, span_offsets, span_start, span_len, n_spans,
+                     surrogate_k, surrogate_v, freed_pages, workspace, workspace_bytes, dev_status, stream, sms);
+}
+
+size_t umim_decode_attention_workspace_size(int32_t batch, int32_t n_q_heads, int32_t n_kv_heads,
+                                            int32_t head_dim) {
+  if (batch < 0 || n_q_heads <= 0 || n_kv_heads <= 0 || (head_dim != 64 && head_dim != 128)) return 0;
+  int sms = current_sms();
+  if (sms <= 0) sms = 256;   // no device yet: size for the largest grid this library launches
+  return decode_attention_workspace_bytes(batch, n_q_heads, n_kv_heads, head_dim, sms);
+}
+
+umim_status umim_decode_attention(const void *q, int32_t n_q_heads, const umim_paged_kv *kv, int32_t layer,
+                                  const int32_t *block_table, int32_t max_pages, const int32_t *seq_lens,
+                                  int32_t batch, float scale, void *out, void *workspace, size_t workspace_bytes,
+                                  int32_t *dev_status, cudaStream_t stream) {
+  if (!kv_ok(kv) || batch < 0 || max_pages < 0 || n_q_heads <= 0) return UMIM_ERR_INVALID_ARG;
+  if (!kv_supported(kv)) return UMIM_ERR_UNSUPPORTED;
+  if (n_q_heads % kv->n_kv_heads != 0 || n_q_heads / kv->n_kv_heads > 16) return UMIM_ERR_UNSUPPORTED;
+  if (layer < 0 || layer >= kv->n_layers) return UMIM_ERR_INVALID_ARG;
+  if ((int64_t)batch * kv->n_kv_heads > (int64_t)1 << 24) return UMIM_ERR_UNSUPPORTED;
+  if (batch == 0) return UMIM_OK;
+  if (!q || !block_table || !seq_lens || !out) return UMIM_ERR_INVALID_ARG;
+  if (!aligned(q, 4) || !aligned(out, 2)) return UMIM_ERR_INVALID_ARG;
+  const int sms = prepare_device(stream);
+  if (!workspace || !aligned(workspace, 256) ||
+      workspace_bytes < decode_attention_workspace_bytes(batch, n_q_heads, kv->n_kv_heads, kv->head_dim, sms))
+    return UMIM_ERR_WORKSPACE;
+  if (!(scale > 0.f)) scale = 1.0f / sqrtf((float)kv->head_dim);
+  int32_t *status = dev_status;
+  return decode_attention(q, n_q_heads, kv, layer, block_table, max_pages, seq_lens, batch, scale, out, workspace,
+                          status, stream, sms);
+}
+
+}  // extern "C"

@@ -1,0 +1,335 @@
+// KV-cache rollback and in-place compaction of a paged bf16 cache
+// (App. E "Decoding-Time Merging and KV-Cache Update", Fig. 2): each span's
+// k stored entries become one surrogate entry and later entries move left.
+//
+// Work unit = (sequence b, lane = layer x head group, compacted page p): the
+// 16 compacted entries j in [16p, 16p+16) of one layer and a group of KV
+// heads.  A unit reads its sources (kept entries t = j + r >= j, or the
+// surrogate rows) into registers, publishes "read done", waits until every
+// unit that reads old page p has published, then writes page p.  Because
+// j <= t, the units that read old page p are unit p itself and lower pages
+// of the same (b, lane); tickets are taken in unit order, so a unit only
+// waits for units that already hold a ticket and publish without waiting:
+// no deadlock, no second pass, each moved byte is read once and written
+// once.  Every wait is bounded (UMIM_ERR_TIMEOUT).
+#include <algorithm>
+
+#include "plan.cuh"
+
+namespace umim {
+namespace {
+
+constexpr int kMoveThreads = 256;
+constexpr int kUnitBytes = 32768;                     // data moved per unit
+constexpr int kChunksPerThread = kUnitBytes / 16 / kMoveThreads;   // 8 x 16 B
+
+struct MoveArgs {
+  uint16_t *pool;
+  int32_t n_layers, n_pages, n_kv_heads, head_dim;
+  int32_t heads_per_unit, n_head_groups;
+  int32_t *block_table;
+  int32_t max_pages;
+  int32_t *seq_lens;
+  const int32_t *span_offsets, *span_start, *span_len;
+  const uint16_t *sur_k, *sur_v;
+  int32_t *freed_pages;
+  int32_t freed_capacity;
+  int32_t B;
+  int32_t *status;
+};
+
+// largest i in [lo, hi) with key(i) <= x, or lo - 1
+__device__ __forceinline__ int upper_index(const int32_t *key, int lo, int hi, int x) {
+  int l = lo, h = hi;
+  while (l < h) {
+    const int m = (l + h) >> 1;
+    if (key[m] <= x) l = m + 1;
+    else h = m;
+  }
+  return l - 1;
+}
+
+__device__ __forceinline__ int find_seq(const int32_t *base, int B, int u) {
+  int l = 0, h = B;   // largest b with base[b] <= u
+  while (l < h) {
+    const int m = (l + h) >> 1;
+    if (base[m] <= u) l = m + 1;
+    else h = m;
+  }
+  return l - 1;
+}
+
+__device__ __forceinline__ uint4 ld_v4(const uint16_t *p) {
+  uint4 v;
+  asm volatile("ld.global.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "l"(p));
+  return v;
+}
+
+__device__ __forceinline__ void st_v4(uint16_t *p, uint4 v) {
+  asm volatile("st.global.v4.u32 [%0], {%1, %2, %3, %4};" ::"l"(p), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+               : "memory");
+}
+
+__global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a, PlanArrays arr) {
+  __shared__ int s_unit, s_b, s_lane, s_p, s_last, s_abort;
+  __shared__ int s_src[kPageSize];      // >= 0: kept source position; <= -2: span -(i+2); -1: no write
+  __shared__ int s_dep_lo, s_dep_hi;
+
+  const int tid = threadIdx.x;
+  const PlanHeader *hdr = arr.hdr;
+  const int total = hdr->total_units;
+  const int epoch = hdr->epoch;
+  const int D = a.head_dim;
+  const int cpr = D / 8;                        // 16-byte chunks per (kv, head) row
+  const int64_t row_elems = D;
+  const int64_t slot_stride = row_elems;        // consecutive slots are consecutive rows
+  const int64_t head_stride = (int64_t)kPageSize * D;
+  const int64_t kv_stride = head_stride * a.n_kv_heads;
+  const int64_t page_stride = kv_stride * 2;
+  const int64_t layer_stride = page_stride * a.n_pages;
+
+  while (true) {
+    if (tid == 0) {
+      const int u = atomicAdd(&arr.hdr->ticket, 1);
+      s_unit = u;
+      s_abort = 0;
+      if (u < total) {
+        const int b = find_seq(arr.unit_base, a.B, u);
+        const int rem = u - arr.unit_base[b];
+        const int nd = arr.n_dest[b];
+        s_b = b;
+        s_lane = rem / nd;
+        s_p = arr.first_page[b] + rem % nd;
+      }
+    }
+    __syncthreads();
+    const int u = s_unit;
+    if (u >= total) break;
+    const int b = s_b, lane = s_lane, p = s_p;
+    const int layer = lane / a.n_head_groups;
+    const int hg = lane % a.n_head_groups;
+    const int h0 = hg * a.heads_per_unit;
+    const int nh = min(a.heads_per_unit, a.n_kv_heads - h0);
+    const int lo = a.span_offsets[b], hi = a.span_offsets[b + 1];
+    const int L = arr.seq_L[b], Lp = arr.seq_Lp[b];
+    const int s_first = a.span_start[lo];
+    const int32_t *bt = a.block_table + (int64_t)b * a.max_pages;
+
+    if (tid < kPageSize) {
+      // source of compacted entry j
+      const int j = p * kPageSize + tid;
+      int src = -1;
+      if (j < Lp && j >= s_first) {
+        const int i = upper_index(arr.new_idx, lo, hi, j);
+        if (i >= lo) {
+          if (arr.new_idx[i] == j) src = -(i + 2);
+          else {
+            const int t = j + arr.r_incl[i];
+            src = (t != j) ? t : -1;
+          }
+        }
+      }
+      s_src[tid] = src;
+    } else if (tid >= 32 && tid < 32 + kPageSize) {
+      // which compacted pages read old page p: kept entries t of page p that move
+      const int t = p * kPageSize + (tid - 32);
+      int dpage = -1;
+      if (t < L) {
+        const int i = upper_index(a.span_start, lo, hi, t);
+        if (i >= lo && t >= a.span_start[i] + a.span_len[i]) {
+          const int r = arr.r_incl[i];
+          if (r > 0) dpage = (t - r) / kPageSize;
+        }
+      }
+      int mn = dpage < 0 ? 0x7fffffff : dpage, mx = dpage;
+#pragma unroll
+      for (int o = 8; o >= 1; o >>= 1) {
+        mn = min(mn, __shfl_xor_sync(0xffffu, mn, o, 16));
+        mx = max(mx, __shfl_xor_sync(0xffffu, mx, o, 16));
+      }
+      if (tid == 32) {
+        s_dep_lo = mn;
+        s_dep_hi = mx;
+      }
+    }
+    __syncthreads();
+
+    // ---- read every source chunk of this unit into registers ----
+    uint4 v[kChunksPerThread];
+    const int n_chunks = 2 * nh * kPageSize * cpr;
+    uint32_t fold = 0;
+#pragma unroll
+    for (int it = 0; it < kChunksPerThread; ++it) {
+      const int c = tid + it * kMoveThreads;
+      v[it] = make_uint4(0, 0, 0, 0);
+      if (c < n_chunks) {
+        const int col = c % cpr;
+        const int row = c / cpr;                 // ((kv * nh + h) * 16 + slot)
+        const int slot = row % kPageSize;
+        const int kvh = row / kPageSize;
+        const int h = h0 + kvh % nh;
+        const int kv = kvh / nh;
+        const int src = s_src[slot];
+        if (src >= 0) {
+          const int page = bt[src / kPageSize];
+          const uint16_t *ptr = a.pool + layer * layer_stride + page * page_stride + kv * kv_stride +
+                                h * head_stride + (src % kPageSize) * slot_stride + col * 8;
+          v[it] = ld_v4(ptr);
+        } else if (src <= -2) {
+          const int i = -src - 2;
+          const uint16_t *sur = kv ? a.sur_v : a.sur_k;
+          const uint16_t *ptr = sur + (((int64_t)i * a.n_layers + layer) * a.n_kv_heads + h) * D + col * 8;
+          v[it] = ld_v4(ptr);
+        }
+      }
+      fold ^= v[it].x ^ v[it].y ^ v[it].z ^ v[it].w;
+    }
+    // every loaded value has arrived before this thread reaches the barrier
+    asm volatile("" ::"r"(fold));
+    __syncthreads();
+    if (tid == 0) {
+      __threadfence();
+      st_release(&arr.flags[u], epoch);
+      // wait for the units that read old page p (all have smaller tickets)
+      const int lo_p = s_dep_lo, hi_p = s_dep_hi;
+      for (int q = lo_p; q <= hi_p && q >= 0; ++q) {
+        if (q >= p) break;
+        const int uq = u - (p - q);
+        if (ld_acquire(&arr.flags[uq]) == epoch) continue;
+        const uint64_t t0 = globaltimer();
+        bool ok = false;
+        while (!ok) {
+#pragma unroll 1
+          for (int i = 0; i < 64 && !ok; ++i) ok = (ld_acquire(&arr.flags[uq]) == epoch);
+          if (!ok && globaltimer() - t0 > kWaitLimitNs) break;
+        }
+        if (!ok) {
+          set_error(a.status, UMIM_ERR_TIMEOUT);
+          s_abort = 1;
+          break;
+        }
+      }
+    }
+    __syncthreads();
+    if (!s_abort) {
+#pragma unroll
+      for (int it = 0; it < kChunksPerThread; ++it) {
+        const int c = tid + it * kMoveThreads;
+        if (c < n_chunks) {
+          const int col = c % cpr;
+          const int row = c / cpr;
+          const int slot = row % kPageSize;
+          const int kvh = row / kPageSize;
+          const int h = h0 + kvh % nh;
+          const int kv = kvh / nh;
+          if (s_src[slot] != -1) {
+            const int page = bt[p];
+            uint16_t *ptr = a.pool + layer * layer_stride + page * page_stride + kv * kv_stride +
+                            h * head_stride + slot * slot_stride + col * 8;
+            st_v4(ptr, v[it]);
+          }
+        }
+      }
+    }
+    __syncthreads();
+  }
+
+  // ---- the last CTA to finish truncates block tables and updates lengths ----
+  if (tid == 0) {
+    __threadfence();
+    const int done = atomicAdd(&arr.hdr->done_ctas, 1);
+    s_last = (done == (int)gridDim.x - 1);
+  }
+  __syncthreads();
+  if (!s_last || hdr->skip) return;
+  __threadfence();
+  for (int b = 0; b < a.B; ++b) {
+    if (a.span_offsets[b + 1] == a.span_offsets[b]) continue;
+    const int L = arr.seq_L[b], Lp = arr.seq_Lp[b];
+    const int keep = ceil_div(Lp, kPageSize), had = ceil_div(L, kPageSize);
+    const int fb = arr.freed_base[b];
+    for (int q = keep + tid; q < had; q += kMoveThreads) {
+      int32_t *e = a.block_table + (int64_t)b * a.max_pages + q;
+      const int idx = fb + (q - keep);
+      if (a.freed_pages && idx < a.freed_capacity) a.freed_pages[idx] = *e;
+      *e = -1;
+    }
+    if (tid == 0) a.seq_lens[b] = Lp;
+  }
+  if (tid == 0 && a.freed_pages) {
+    const int n = arr.freed_base[a.B];
+    if (n < a.freed_capacity) a.freed_pages[n] = -1;
+  }
+}
+
+}  // namespace
+
+size_t kv_rollback_workspace_bytes(int B, int S, int max_pages, int n_layers, int n_kv_heads, int head_dim) {
+  const int hpu = std::max(1, kUnitBytes / (2 * kPageSize * head_dim * 2));
+  const int groups = (n_kv_heads + hpu - 1) / hpu;
+  const size_t units = (size_t)B * n_layers * groups * (size_t)max_pages;
+  return plan_bytes(B, S) + align256(sizeof(int32_t) * (units > 0 ? units : 1));
+}
+
+umim_status kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t max_pages, int32_t *seq_lens,
+                        int32_t B, const int32_t *span_offsets, const int32_t *span_start,
+                        const int32_t *span_len, int32_t S, const void *sur_k, const void *sur_v,
+                        int32_t *freed_pages, void *ws, size_t ws_bytes, int32_t *dev_status,
+                        cudaStream_t stream, int num_sms) {
+  const int D = kv->head_dim;
+  const int hpu = std::max(1, kUnitBytes / (2 * kPageSize * D * 2));
+  const int hp = std::min(hpu, (int)kv->n_kv_heads);
+  const int groups = (kv->n_kv_heads + hp - 1) / hp;
+  PlanArrays arr = plan_carve(ws, B, S);
+  int32_t *status = dev_status ? dev_status : &arr.hdr->status;
+
+  PlanArgs pa{};
+  pa.seq_lens = seq_lens;
+  pa.fixed_len = 0;
+  pa.span_offsets = span_offsets;
+  pa.span_start = span_start;
+  pa.span_len = span_len;
+  pa.B = B;
+  pa.S = S;
+  pa.max_span_len = 0;
+  pa.block_table = block_table;
+  pa.max_pages = max_pages;
+  pa.n_pages = kv->n_pages;
+  pa.n_lanes = kv->n_layers * groups;
+  pa.status = status;
+  pa.cu_seqlens_out = nullptr;
+  if (launch_span_plan(pa, arr, stream) != cudaSuccess) return UMIM_ERR_CUDA;
+
+  MoveArgs ma{};
+  ma.pool = static_cast<uint16_t *>(kv->base);
+  ma.n_layers = kv->n_layers;
+  ma.n_pages = kv->n_pages;
+  ma.n_kv_heads = kv->n_kv_heads;
+  ma.head_dim = D;
+  ma.heads_per_unit = hp;
+  ma.n_head_groups = groups;
+  ma.block_table = block_table;
+  ma.max_pages = max_pages;
+  ma.seq_lens = seq_lens;
+  ma.span_offsets = span_offsets;
+  ma.span_start = span_start;
+  ma.span_len = span_len;
+  ma.sur_k = static_cast<const uint16_t *>(sur_k);
+  ma.sur_v = static_cast<const uint16_t *>(sur_v);
+  ma.freed_pages = freed_pages;
+  ma.freed_capacity = (int32_t)std::min<int64_t>((int64_t)B * max_pages, INT32_MAX);
+  ma.B = B;
+  ma.status = status;
+  int per_sm = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, rollback_move_kernel, kMoveThreads, 0) !=
+          cudaSuccess ||
+      per_sm < 1)
+    per_sm = 1;
+  const int grid = std::max(1, num_sms) * per_sm;
+  rollback_move_kernel<<<grid, kMoveThreads, 0, stream>>>(ma, arr);
+  return cudaGetLastError() == cudaSuccess ? UMIM_OK : UMIM_ERR_CUDA;
+}
+
+}  // namespace umim

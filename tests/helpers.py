@@ -1,0 +1,63 @@
+"""Shared helpers of the GPU parity tests: run the CUDA path through the C ABI
+and compare with the CPU oracle on the same seeded inputs."""
+import numpy as np
+import torch
+
+import oracle
+import workloads as W
+
+# tolerances for floating-point outputs (bf16 in, fp32 accumulate)
+MAX_ABS = 1e-2
+REL_L2 = 2e-3
+
+
+def float_close(got, want, what=""):
+    got = np.asarray(got, dtype=np.float64)
+    want = np.asarray(want, dtype=np.float64)
+    assert got.shape == want.shape, (what, got.shape, want.shape)
+    assert np.all(np.isfinite(got)), f"{what}: non-finite output"
+    err = np.abs(got - want)
+    rel = np.linalg.norm(got - want) / max(np.linalg.norm(want), 1e-30)
+    assert err.max() <= MAX_ABS, f"{what}: max abs err {err.max():.3e}"
+    assert rel <= REL_L2, f"{what}: rel L2 err {rel:.3e}"
+    return float(err.max()), float(rel)
+
+
+def umim():
+    import paper_2609_27233_gb300 as m
+    m.lib()
+    return m
+
+
+def dev():
+    return torch.device("cuda:0")
+
+
+def case_to_dev(c, d):
+    return dict(pool=c.pool.to(d), bt=c.block_table.to(d), lens=c.seq_lens.to(d), offs=c.span_offsets.to(d),
+                st=c.span_start.to(d), ln=c.span_len.to(d), sk=c.surrogate_k.to(d), sv=c.surrogate_v.to(d),
+                q=c.q.to(d))
+
+
+def oracle_rollback(c):
+    return oracle.kv_rollback(W.bits(c.pool), c.block_table.cpu().numpy(), c.seq_lens.cpu().numpy(),
+                              c.span_offsets.cpu().numpy(), c.span_start.cpu().numpy(),
+                              c.span_len.cpu().numpy(), W.bits(c.surrogate_k), W.bits(c.surrogate_v))
+
+
+def compare_rollback(g_pool, g_bt, g_lens, g_freed, ref):
+    """Bit-exact: block table, lengths, freed pages, every valid KV byte."""
+    rp, rbt, rl, rfreed = ref
+    bt = g_bt.cpu().numpy()
+    lens = g_lens.cpu().numpy()
+    np.testing.assert_array_equal(bt, rbt)
+    np.testing.assert_array_equal(lens, rl)
+    f = g_freed.cpu().numpy()
+    assert f[:len(rfreed)].tolist() == rfreed
+    if len(rfreed) < len(f):
+        assert f[len(rfreed)] == -1
+    gp = W.bits(g_pool)
+    for b in range(len(rl)):
+        t = np.arange(int(rl[b]))
+        pg, sl = rbt[b, t // 16], t % 16
+        np.testing.assert_array_equal(gp[:, pg, :, :, sl, :], rp[:, pg, :, :, sl, :], err_msg=f"seq {b}")

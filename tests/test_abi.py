@@ -1,0 +1,79 @@
+"""The C ABI library builds, loads and exports every entry point its header
+declares; host-side argument checks work without a GPU (no compute call)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADERS = [os.path.join(ROOT, "include", f) for f in os.listdir(os.path.join(ROOT, "include")) if f.endswith(".h")]
+
+
+def declared_functions():
+    names = set()
+    for h in HEADERS:
+        text = open(h).read()
+        text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+        for m in re.finditer(r"^[A-Za-z_][\w \*]*?\b(umim_\w+)\s*\(", text, flags=re.M):
+            names.add(m.group(1))
+    return names
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2609_27233_gb300 import build, _lib
+    if not os.path.exists(_lib.LIB_PATH):
+        build.build()
+    return _lib.load()
+
+
+def test_header_declares_the_four_calls():
+    names = declared_functions()
+    for n in ("umim_merge_spans", "umim_kv_rollback", "umim_decode_attention", "umim_build_compressed"):
+        assert n in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = declared_functions()
+    assert names
+    for n in names:
+        assert hasattr(lib, n), n
+    from paper_2609_27233_gb300 import _lib
+    assert set(_lib.SIGNATURES) == names
+
+
+def test_status_strings_and_version(lib):
+    assert lib.umim_status_string(0) == b"UMIM_OK"
+    assert lib.umim_status_string(4) == b"UMIM_ERR_TIMEOUT"
+    assert lib.umim_version() >= 100
+
+
+def test_workspace_sizes_are_positive(lib):
+    assert lib.umim_merge_spans_workspace_size(120, 40, 512) > 120 * 512 * 6
+    assert lib.umim_kv_rollback_workspace_size(16, 6560, 256, 1, 8, 128) > 0
+    assert lib.umim_kv_rollback_workspace_size(1, 1, 1, 1, 1, 96) == 0     # head_dim unsupported
+    assert lib.umim_build_compressed_workspace_size(64, 17472) > 0
+    assert lib.umim_decode_attention_workspace_size(16, 32, 8, 128) > 0
+
+
+def test_host_checks_reject_bad_arguments_without_touching_the_gpu(lib):
+    from paper_2609_27233_gb300._lib import PagedKVC, MergeWeightsC
+    null = ctypes.c_void_p(0)
+    kv = PagedKVC(0, 1, 1, 1, 16, 128)                                   # null base
+    assert lib.umim_kv_rollback(ctypes.byref(kv), null, 1, null, 1, null, null, null, 0, null, null, null,
+                                null, 0, null, null) == 1
+    kv = PagedKVC(4096, 1, 1, 1, 8, 128)                                  # page size 8
+    assert lib.umim_decode_attention(null, 1, ctypes.byref(kv), 0, null, 1, null, 1, 0.0, null, null, 0,
+                                     null, null) == 2
+    kv = PagedKVC(4096, 1, 1, 2, 16, 128)                                 # Hq not a multiple of Hkv
+    assert lib.umim_decode_attention(null, 3, ctypes.byref(kv), 0, null, 1, null, 1, 0.0, null, null, 0,
+                                     null, null) == 2
+    w = MergeWeightsC(*([0] * 9), 500, 4, 1e-5)                           # d not a multiple of 512
+    assert lib.umim_merge_spans(null, 10, null, 0, null, 1, ctypes.byref(w), null, null, 0, null, null) == 2
+    w = MergeWeightsC(*([0] * 9), 512, 3, 1e-5)                           # 3 heads
+    assert lib.umim_merge_spans(null, 10, null, 0, null, 1, ctypes.byref(w), null, null, 0, null, null) == 2
+    # empty batches are a no-op that succeeds
+    kv = PagedKVC(4096, 1, 1, 1, 16, 128)
+    assert lib.umim_kv_rollback(ctypes.byref(kv), null, 1, null, 0, null, null, null, 0, null, null, null,
+                                null, 0, null, null) == 0
