@@ -1,0 +1,520 @@
+#!/usr/bin/env python
+"""Benchmark of the UMIM decode step over a merged context on GB300.
+
+One step = the whole hot path on the Llama-3-8B-shaped decode layer
+(16 sequences x 4096 cached tokens, 32 query / 8 KV heads, head_dim 128,
+bf16 paged cache with 16-entry pages, 30 % of positions covered by spans of
+2..4 tokens):
+  1. umim_merge_spans       every span -> surrogate embedding (merge module
+                            at d_model 4096, 4 pooling heads, table 128256 x 4096)
+  2. umim_kv_rollback       every span's entries -> one surrogate entry, in place
+  3. umim_decode_attention  one query token per sequence over the compacted cache
+Metric: merged spans per second through the whole step (value), with the
+decode-attention GB/s and its fraction of the measured HBM bandwidth reported
+beside it.  Every timed step works on its own pristine copy of the cache
+(larger than L2), so no work is skipped and nothing is served from L2.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl umim|reference]
+
+--impl reference times the CPU oracle (the only reference there is: the
+paper publishes no code) on a bounded sample of the same workload.
+"""
+import argparse
+import hashlib
+import json
+import os
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "compacted-KV decode attention GB/s (% of HBM peak); merged spans/sec"
+UNIT = "spans/s"
+WORKLOAD = dict(name="llama8b_layer", B=16, L=4096, Hq=32, Hkv=8, D=128, coverage=0.3, d_model=4096, h=4,
+                vocab=128256)
+
+
+def load_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return dict(hbm=float(p["hbm_gbs"]), bf16=float(p["bf16_tflops"]),
+                    bf16_sus=float(p["bf16_tflops_sustained"]), src="measured")
+    except Exception:
+        return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, src="fallback")
+
+
+# ---------------------------------------------------------------------------
+# workload (host-side structure, identical on every rank apart from the seed)
+# ---------------------------------------------------------------------------
+def make_structure(seed):
+    import workloads as W
+    w = WORKLOAD
+    r = W.rng(seed)
+    token_ids = r.integers(0, w["vocab"], size=(w["B"], w["L"])).astype(np.int32)
+    starts, lens, offs = [], [], [0]
+    for b in range(w["B"]):
+        st, ln = W.span_layout(r, w["L"], coverage=w["coverage"])
+        starts.append(st)
+        lens.append(ln)
+        offs.append(offs[-1] + len(st))
+    span_start = np.concatenate(starts).astype(np.int32)
+    span_len = np.concatenate(lens).astype(np.int32)
+    toks, toffs = [], [0]
+    for b in range(w["B"]):
+        for i in range(offs[b], offs[b + 1]):
+            s, k = int(span_start[i]), int(span_len[i])
+            toks.append(token_ids[b, s:s + k])
+            toffs.append(toffs[-1] + k)
+    return dict(token_ids=token_ids, span_offsets=np.asarray(offs, np.int32), span_start=span_start,
+                span_len=span_len, span_tokens=np.concatenate(toks).astype(np.int32),
+                span_token_offsets=np.asarray(toffs, np.int32))
+
+
+def algorithmic_work(st):
+    """Bytes / FLOPs the method itself must move or compute per step."""
+    w = WORKLOAD
+    B, L, Hkv, D, d = w["B"], w["L"], w["Hkv"], w["D"], w["d_model"]
+    entry = 2 * Hkv * D * 2                    # K and V of every KV head, bf16, one layer
+    S = len(st["span_start"])
+    T = len(st["span_tokens"])
+    moved = 0
+    Lp = []
+    for b in range(B):
+        lo, hi = st["span_offsets"][b], st["span_offsets"][b + 1]
+        ss, ll = st["span_start"][lo:hi], st["span_len"][lo:hi]
+        r = 0
+        prev_end = 0
+        for s, k in zip(ss, ll):
+            if r > 0:
+                moved += int(s - prev_end)     # kept entries between spans that shift left
+            r += int(k) - 1
+            prev_end = int(s + k)
+        if r > 0:
+            moved += L - prev_end
+        Lp.append(L - int((ll - 1).sum()))
+    Lp = np.asarray(Lp)
+    q_bytes = B * w["Hq"] * D * 2
+    return dict(
+        S=S, T=T, Lp=Lp, entry=entry,
+        gemm1_flop=2.0 * T * d * d,
+        gemm2_flop=2.0 * S * d * d,
+        rollback_bytes=float((moved + S) * entry * 2 + 4 * (3 * S + 3 * B)),
+        attention_bytes=float(Lp.sum() * entry + 2 * q_bytes + B * 4 + (Lp + 15).sum() // 16 * 4),
+    )
+
+
+# ---------------------------------------------------------------------------
+# clocks sampled during the timed region
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.lines = []
+        self.proc = None
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(index), "--query-gpu=" + self.FIELDS, "--format=csv,noheader,nounits",
+                 "-lms", "20"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append((time.time(), line.strip()))
+
+    def mark(self):
+        return time.time()
+
+    def stop(self):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self, t0, t1):
+        rows = [l for (t, l) in self.lines if t0 - 0.05 <= t <= t1 + 0.05]
+        if not rows:   # region shorter than one sample: take the nearest
+            rows = [min(self.lines, key=lambda x: abs(x[0] - (t0 + t1) / 2))[1]] if self.lines else []
+        sm, mx, reasons = [], 0.0, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            p = [x.strip() for x in r.split(",")]
+            try:
+                sm.append(float(p[1]))
+                mx = max(mx, float(p[2]))
+            except Exception:
+                continue
+            for n, v in zip(names, p[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": float(np.median(sm)) if sm else None, "sm_max_mhz": mx or None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle on a bounded sample (the cpu_baseline and the reference arm)
+# ---------------------------------------------------------------------------
+class OracleSampler:
+    """Times the oracle on part of one step and scales it to spans/s of a
+    whole step.  The merge-module weights are built once; each sample draws
+    its own spans and sequences."""
+
+    def __init__(self, st, seed):
+        from oracle import merge as M
+        import workloads as W
+        w = WORKLOAD
+        self.st, self.seed = st, seed
+        wt = W.merge_weights(w["d_model"], w["h"], seed + 202)
+        self.wf = M.weights_f64({k: W.bits(v) for k, v in wt.tensors().items()})
+        self.tb = np.zeros((w["vocab"], w["d_model"]), dtype=np.uint16)
+
+    def sample(self, k, n_spans=64, n_seqs=1):
+        import oracle
+        import workloads as W
+        w, st = WORKLOAD, self.st
+        d = w["d_model"]
+        S = len(st["span_start"])
+        r = W.rng(self.seed + 99 + k)
+        which = np.sort(r.choice(S, size=min(n_spans, S), replace=False))
+        toffs, ids = st["span_token_offsets"], st["span_tokens"]
+        used = np.unique(ids[np.concatenate([np.arange(toffs[i], toffs[i + 1]) for i in which])])
+        self.tb[used] = W.bits(W.bf16_normal((len(used), d), 0.02, self.seed + 5 + k))
+        t0 = time.perf_counter()
+        oracle.merge_spans(self.tb, ids, toffs, self.wf, w["h"], which=which)
+        t_merge = (time.perf_counter() - t0) / len(which)
+        t_rb = t_at = 0.0
+        seqs = r.choice(w["B"], size=n_seqs, replace=False)
+        for b in seqs:
+            lo, hi = st["span_offsets"][b], st["span_offsets"][b + 1]
+            n_pages = w["L"] // 16
+            pool = W.bits(W.bf16_normal((1, n_pages, 2, w["Hkv"], 16, w["D"]), 1.0, self.seed + 10 + k))
+            bt = r.permutation(n_pages).astype(np.int32)[None, :]
+            sk = W.bits(W.bf16_normal((hi - lo, 1, w["Hkv"], w["D"]), 1.0, self.seed + 20 + k))
+            sv = W.bits(W.bf16_normal((hi - lo, 1, w["Hkv"], w["D"]), 1.0, self.seed + 30 + k))
+            q = W.bits(W.bf16_normal((1, w["Hq"], w["D"]), 1.0, self.seed + 40 + k))
+            t0 = time.perf_counter()
+            p2, bt2, l2, _ = oracle.kv_rollback(pool, bt, np.array([w["L"]], np.int32), np.array([0, hi - lo]),
+                                                st["span_start"][lo:hi], st["span_len"][lo:hi], sk, sv)
+            t1 = time.perf_counter()
+            oracle.decode_attention(q, p2, 0, bt2, l2)
+            t2 = time.perf_counter()
+            t_rb += t1 - t0
+            t_at += t2 - t1
+        t_rb /= n_seqs
+        t_at /= n_seqs
+        step_s = S * t_merge + w["B"] * (t_rb + t_at)
+        text = (f"oracle on {len(which)} of {S} spans (merge module) and {n_seqs} of {w['B']} sequences "
+                f"(rollback + attention), scaled to one full step")
+        return dict(value=S / step_s, step_s=step_s, sample=text, merge_s_per_span=t_merge,
+                    rollback_s_per_seq=t_rb, attention_s_per_seq=t_at)
+
+
+def cpu_cores():
+    n = os.cpu_count() or 1
+    try:
+        from threadpoolctl import threadpool_info
+        th = [i.get("num_threads", 1) for i in threadpool_info() if i.get("user_api") == "blas"]
+        if th:
+            return int(max(th))
+    except Exception:
+        pass
+    return n
+
+
+# ---------------------------------------------------------------------------
+def traffic_from_profile(label):
+    """DRAM bytes per launch from the committed ncu summary, if the kernel's
+    source is unchanged since the capture."""
+    path = os.path.join(ROOT, "profiles", "ncu_traffic.json")
+    try:
+        with open(path) as f:
+            prof = json.load(f)
+        e = prof[label]
+        src = os.path.join(ROOT, "paper_2609_27233_gb300", "csrc", e["source"])
+        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        if sha != e["source_sha"]:
+            return None
+        return float(e["bytes_per_launch_full"])
+    except Exception:
+        return None
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=100)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="umim", choices=["umim", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    args = ap.parse_args()
+    K, Wm = args.steps, max(3, args.warmup)
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    peaks = load_peaks()
+
+    if args.impl == "reference":
+        if rank != 0:
+            return 0
+        st = make_structure(0x5EED0002)
+        smp = OracleSampler(st, 0x5EED0002)
+        samples = []
+        for k in range(Wm):
+            smp.sample(k, n_spans=8, n_seqs=1)
+        t0 = time.perf_counter()
+        for k in range(K):
+            samples.append(smp.sample(Wm + k, n_spans=32, n_seqs=1))
+        wall = time.perf_counter() - t0
+        v = float(np.mean([s["value"] for s in samples]))
+        line = {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": args.gpus,
+                "steps": K, "warmup": Wm, "ms_per_step": 1000.0 * float(np.mean([s["step_s"] for s in samples])),
+                "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+                "data": "synthetic", "config": config_dict(st),
+                "cpu_baseline": {"value": v, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+                                 "sample": samples[0]["sample"]},
+                "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+                "wall_s": wall}
+        print(json.dumps(line))
+        return 0
+
+    import torch
+    import paper_2609_27233_gb300 as umim
+    import workloads as W
+
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", rank=rank, world_size=world)
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    umim.lib()
+
+    w = WORKLOAD
+    seed = 0x5EED0002 + 1000 * rank
+    st = make_structure(seed)
+    work = algorithmic_work(st)
+    S, T = work["S"], work["T"]
+    B, L, Hq, Hkv, D, d = w["B"], w["L"], w["Hq"], w["Hkv"], w["D"], w["d_model"]
+    n_pages = B * (L // 16)
+    max_pages = L // 16
+    t = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+
+    # model state resident in HBM
+    table = W.bf16_normal((w["vocab"], d), 0.02, seed + 101, dev)
+    weights = W.merge_weights(d, w["h"], seed + 202, dev)
+    span_tokens, span_token_offsets = t(st["span_tokens"]), t(st["span_token_offsets"])
+    span_offsets, span_start, span_len = t(st["span_offsets"]), t(st["span_start"]), t(st["span_len"])
+    sk = W.bf16_normal((S, 1, Hkv, D), 1.0, seed + 12, dev)
+    sv = W.bf16_normal((S, 1, Hkv, D), 1.0, seed + 13, dev)
+    q = W.bf16_normal((B, Hq, D), 1.0, seed + 14, dev)
+    pool0 = W.bf16_normal((1, n_pages, 2, Hkv, 16, D), 1.0, seed + 11, dev)
+    perm = W.rng(seed + 3).permutation(n_pages).astype(np.int32)
+    bt0 = t(perm.reshape(B, max_pages))
+    lens0 = t(np.full(B, L, np.int32))
+
+    # one pristine cache copy per step (each larger than L2)
+    n_copies = Wm + K
+    free = torch.cuda.mem_get_info(dev)[0]
+    copy_bytes = pool0.numel() * 2
+    if n_copies * copy_bytes > 0.6 * free:
+        n_copies = max(Wm + 1, int(0.6 * free // copy_bytes))
+    pools = [torch.empty_like(pool0) for _ in range(n_copies)]
+    bts = [torch.empty_like(bt0) for _ in range(n_copies)]
+    lens = [torch.empty_like(lens0) for _ in range(n_copies)]
+
+    def restore():
+        for i in range(n_copies):
+            pools[i].copy_(pool0)
+            bts[i].copy_(bt0)
+            lens[i].copy_(lens0)
+
+    z = torch.empty((S, d), dtype=torch.float32, device=dev)
+    out = torch.empty_like(q)
+    freed = torch.empty(B * max_pages, dtype=torch.int32, device=dev)
+    status = umim.new_status(dev)
+    ws_m = umim.workspace(umim.umim_merge_spans_workspace_size(T, S, d), dev)
+    ws_r = umim.workspace(umim.umim_kv_rollback_workspace_size(B, S, max_pages, 1, Hkv, D), dev)
+    ws_a = umim.workspace(umim.umim_decode_attention_workspace_size(B, Hq, Hkv, D), dev)
+
+    def step(i, inputs=None):
+        j = i % n_copies
+        if inputs is None:
+            tk, to, so, ss, sl, k_, v_, q_ = (span_tokens, span_token_offsets, span_offsets, span_start, span_len,
+                                             sk, sv, q)
+        else:
+            tk, to, so, ss, sl, k_, v_, q_ = inputs
+        umim.umim_merge_spans(table, tk, to, weights, surrogates=z, workspace_buf=ws_m, dev_status=status)
+        umim.umim_kv_rollback(pools[j], bts[j], lens[j], so, ss, sl, k_, v_, freed_pages=freed,
+                              workspace_buf=ws_r, dev_status=status)
+        umim.umim_decode_attention(q_, pools[j], 0, bts[j], lens[j], out=out, workspace_buf=ws_a,
+                                   dev_status=status)
+
+    def barrier():
+        if world > 1:
+            torch.distributed.barrier()
+
+    def timed(fn, n, offset):
+        barrier()
+        torch.cuda.synchronize()
+        s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s0.record()
+        for i in range(n):
+            if (offset + i) % n_copies == 0 and offset + i > 0:
+                restore()          # only when the steps outnumber the cache copies
+            fn(offset + i)
+        s1.record()
+        torch.cuda.synchronize()
+        barrier()
+        return s0.elapsed_time(s1)
+
+    restore()
+    torch.cuda.synchronize()
+    # warm-up
+    for i in range(Wm):
+        step(i)
+    torch.cuda.synchronize()
+    umim.check_status(status, "warm-up")
+
+    # ---- timed region ----
+    clk = ClockSampler(local)
+    time.sleep(0.3)
+    t_wall0 = time.time()
+    ms = timed(step, K, Wm)
+    t_wall1 = time.time()
+    time.sleep(0.1)
+    clk.stop()
+    umim.check_status(status, "timed steps")
+    clocks = clk.summary(t_wall0, t_wall1)
+    if world > 1:
+        tt = torch.tensor([ms], device=dev)
+        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        ms = float(tt.item())
+    ms_step = ms / K
+    value = world * S * K / (ms / 1000.0)
+
+    # ---- per-kernel times: the same steps again, with kernel tracing on ----
+    restore()
+    torch.cuda.synchronize()
+    umim.trace_start(16 * (K + 2))
+    tms = timed(step, K, Wm)
+    umim.trace_stop()
+    recs = umim.trace_read(16 * (K + 2))
+    kern = {}
+    for lab, v in recs:
+        kern.setdefault(lab, []).append(v)
+    launches_per_step = len(recs) / K
+    avg = {k: float(np.mean(v)) for k, v in kern.items()}
+    work_of = {
+        "merge.gemm1": ("tensor", work["gemm1_flop"] / 1e12, "TFLOP/s", peaks["bf16"]),
+        "merge.gemm2": ("tensor", work["gemm2_flop"] / 1e12, "TFLOP/s", peaks["bf16"]),
+        "rollback.move": ("hbm", work["rollback_bytes"] / 1e9, "GB/s", peaks["hbm"]),
+        "attention.decode": ("hbm", work["attention_bytes"] / 1e9, "GB/s", peaks["hbm"]),
+    }
+    kernels = {}
+    for k, v in sorted(avg.items(), key=lambda x: -x[1]):
+        e = {"ms": round(v, 5), "share": round(v * len(kern[k]) / max(sum(sum(x) for x in kern.values()), 1e-9), 4)}
+        if k in work_of:
+            b, amount, unit, peak = work_of[k]
+            ach = amount / (v / 1000.0)
+            e.update({"bound": b, "achieved": round(ach, 2), "unit": unit, "frac": round(ach / peak, 4)})
+        kernels[k] = e
+    top = max(avg, key=lambda k: avg[k])
+    if top in work_of:
+        b, amount, unit, peak = work_of[top]
+        ach = amount / (avg[top] / 1000.0)
+        tr = traffic_from_profile(top)
+        roof = {"kernel": top, "bound": b, "achieved": round(ach, 2), "peak": peak, "unit": unit,
+                "frac": round(ach / peak, 4), "traffic": tr,
+                "algorithmic_per_launch": amount * (1e12 if unit == "TFLOP/s" else 1e9),
+                "peak_source": peaks["src"] + (" bf16 burst" if b == "tensor" else " HBM copy")}
+    else:
+        roof = {"kernel": top, "bound": "hbm", "achieved": None, "peak": peaks["hbm"], "unit": "GB/s",
+                "frac": None, "traffic": None}
+    att_ms = avg.get("attention.decode", float("nan"))
+    att_gbs = work["attention_bytes"] / 1e9 / (att_ms / 1000.0)
+
+    # ---- end to end through the C ABI with host buffers ----
+    e2e = None
+    if not args.no_e2e:
+        restore()
+        host = [torch.from_numpy(a).pin_memory() for a in (st["span_tokens"], st["span_token_offsets"],
+                                                            st["span_offsets"], st["span_start"], st["span_len"])]
+        host += [x.cpu().pin_memory() for x in (sk, sv, q)]
+        dbuf = [torch.empty_like(h, device=dev) for h in host]
+        h_out = torch.empty(out.shape, dtype=out.dtype).pin_memory()
+        h_lens = torch.empty(B, dtype=torch.int32).pin_memory()
+        h_freed = torch.empty(freed.shape, dtype=torch.int32).pin_memory()
+        h2d = sum(h.numel() * h.element_size() for h in host)
+        d2h = h_out.numel() * 2 + B * 4 + h_freed.numel() * 4
+
+        def e2e_step(i):
+            for dd, hh in zip(dbuf, host):
+                dd.copy_(hh, non_blocking=True)
+            step(i, dbuf)
+            j = i % n_copies
+            h_out.copy_(out, non_blocking=True)
+            h_lens.copy_(lens[j], non_blocking=True)
+            h_freed.copy_(freed, non_blocking=True)
+
+        for i in range(2):
+            e2e_step(i)
+        restore()
+        torch.cuda.synchronize()
+        ems = timed(e2e_step, K, Wm)
+        if world > 1:
+            tt = torch.tensor([ems], device=dev)
+            torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+            ems = float(tt.item())
+        e2e = {"value": world * S * K / (ems / 1000.0), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
+               "d2h_bytes_per_step": int(d2h), "ms_per_step": ems / K}
+        umim.check_status(status, "e2e steps")
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        smp = OracleSampler(st, seed)
+        s = smp.sample(0, n_spans=4096, n_seqs=8)
+        cpu = {"value": s["value"], "unit": UNIT, "cores": cpu_cores(), "kind": "oracle", "sample": s["sample"]}
+
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": Wm,
+                "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+                "dtype": "bf16", "data": "synthetic", "config": config_dict(st),
+                "attention": {"gbs": round(att_gbs, 1), "frac_of_hbm": round(att_gbs / peaks["hbm"], 4),
+                              "frac_of_8tbs_nominal": round(att_gbs / 7900.0, 4)},
+                "roofline": roof, "kernels": kernels, "cpu_baseline": cpu, "e2e": e2e,
+                "gpu_launches": int(round(launches_per_step * K)), "clocks": clocks,
+                "traced_ms_per_step": tms / K}
+        print(json.dumps(line))
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+def config_dict(st):
+    w = WORKLOAD
+    return {"workload": "llama8b_layer decode step over a merged context: 16 seqs x 4096 cached tokens, "
+                        "32/8 heads, head_dim 128, bf16 paged KV (page 16), 30% of positions in spans of 2..4 "
+                        "tokens rolled back, merge module d_model 4096 (4 heads) over a 128256-row table",
+            "batch": w["B"], "context": w["L"], "n_q_heads": w["Hq"], "n_kv_heads": w["Hkv"], "head_dim": w["D"],
+            "spans_per_step": int(len(st["span_start"])), "span_tokens_per_step": int(len(st["span_tokens"])),
+            "d_model": w["d_model"], "l2": "inputs larger than L2: a distinct 268 MB cache copy per step",
+            "parallelism": "replicas (one independent batch per GPU)"}
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -231,6 +231,24 @@ umim_status umim_decode_attention(const void *q, int32_t n_q_heads, const umim_p
                                   int32_t batch, float scale, void *out, void *workspace,
                                   size_t workspace_bytes, int32_t *dev_status, cudaStream_t stream);
 
+/* ------------------------------------------------------------------------
+ * Kernel tracing, for profiling (not part of the method).  Between
+ * umim_trace_start and umim_trace_stop every call above records a CUDA
+ * event on its stream before each kernel it launches and one after its last
+ * kernel, so consecutive events bracket one kernel.  The library creates the
+ * events itself (no device memory).  Process-wide and not thread-safe.
+ *
+ * umim_trace_start  begin recording, at most `capacity` events; returns
+ *                   UMIM_ERR_CUDA if the events cannot be created
+ * umim_trace_stop   stop recording (the recorded events are kept)
+ * umim_trace_read   synchronise on the last event, write up to `cap` kernel
+ *                   durations (ms) and their labels (static strings) in
+ *                   launch order; returns how many were written
+ * ------------------------------------------------------------------------ */
+umim_status umim_trace_start(int32_t capacity);
+void umim_trace_stop(void);
+int32_t umim_trace_read(float *ms, const char **labels, int32_t cap);
+
 #ifdef __cplusplus
 } /* extern "C" */
 #endif

@@ -191,3 +191,22 @@ def umim_decode_attention(q, pool, layer, block_table, seq_lens, scale=0.0, out=
                                        workspace_buf.numel(), _p(dev_status), _stream(stream))
     _check(code, "umim_decode_attention")
     return out
+
+
+# ---------------------------------------------------------------------------
+# kernel tracing (profiling aid)
+# ---------------------------------------------------------------------------
+def trace_start(capacity=4096):
+    _check(lib().umim_trace_start(capacity), "umim_trace_start")
+
+
+def trace_stop():
+    lib().umim_trace_stop()
+
+
+def trace_read(cap=4096):
+    """[(label, milliseconds)] of every kernel launched while tracing."""
+    ms = (ctypes.c_float * cap)()
+    labels = (ctypes.c_char_p * cap)()
+    n = lib().umim_trace_read(ms, labels, cap)
+    return [(labels[i].decode(), float(ms[i])) for i in range(n)]

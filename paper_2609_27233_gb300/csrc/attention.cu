@@ -508,6 +508,7 @@ static umim_status run_attention(const void *q, int Hq, const umim_paged_kv *kv,
   const int total_warps = attn_total_warps(num_sms);
   const int Hkv = kv->n_kv_heads;
   AttnWs ws = attn_carve(workspace, B, Hkv, D, total_warps);
+  trace_mark(stream, "attention.plan");
   attn_plan_kernel<<<1, kPlanThreadsA, 0, stream>>>(seq_lens, B, Hkv, max_pages, total_warps, ws, status);
 
   AttnArgs a{};
@@ -528,11 +529,14 @@ static umim_status run_attention(const void *q, int Hq, const umim_paged_kv *kv,
   auto kern = attn_decode_kernel<D>;
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
     return UMIM_ERR_CUDA;
+  trace_mark(stream, "attention.decode");
   kern<<<total_warps / kAttnWarps, kAttnWarps * 32, smem, stream>>>(map, a, ws);
+  trace_mark(stream, "attention.combine");
   const int threads = 256;
   const int nwarps = B * Hq;
   attn_combine_kernel<D><<<(nwarps * 32 + threads - 1) / threads, threads, 0, stream>>>(
       ws, B, Hq, Hkv, a.G, static_cast<__nv_bfloat16 *>(out));
+  trace_mark(stream, nullptr);
   return cudaGetLastError() == cudaSuccess ? UMIM_OK : UMIM_ERR_CUDA;
 }
 

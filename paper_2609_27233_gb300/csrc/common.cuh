@@ -229,4 +229,8 @@ __device__ __forceinline__ float gelu_erf(float x) {
 
 __host__ __device__ __forceinline__ int ceil_div(int a, int b) { return (a + b - 1) / b; }
 
+// Kernel tracing (trace.cu): records an event labelled with the next kernel,
+// or, with a null label, the end of a call.  No-op unless a trace is active.
+void trace_mark(cudaStream_t stream, const char *label);
+
 }  // namespace umim

@@ -101,6 +101,7 @@ umim_status build_compressed(const void *embeddings, int64_t vocab, int d, const
   pa.n_lanes = 0;
   pa.status = status;
   pa.cu_seqlens_out = cu_seqlens;
+  trace_mark(stream, "compact.plan");
   if (launch_span_plan(pa, arr, stream) != cudaSuccess) return UMIM_ERR_CUDA;
   CompactArgs a;
   a.table = static_cast<const uint4 *>(embeddings);
@@ -117,7 +118,9 @@ umim_status build_compressed(const void *embeddings, int64_t vocab, int d, const
   a.status = status;
   const int64_t rows = (int64_t)B * L;
   const int blocks = (int)std::max<int64_t>(1, std::min<int64_t>((rows + 7) / 8, (int64_t)num_sms * 16));
+  trace_mark(stream, "compact.rows");
   compact_kernel<<<blocks, 256, 0, stream>>>(a, arr);
+  trace_mark(stream, nullptr);
   return cudaGetLastError() == cudaSuccess ? UMIM_OK : UMIM_ERR_CUDA;
 }
 

@@ -25,7 +25,8 @@ constexpr int kStageBytes = (BM + BN) * BK * 2;
 constexpr int kGemmSmem = STAGES * kStageBytes + 1024;
 
 struct GemmArgs {
-  int M, N, K;
+  int M, N, K;                 // A is [M][K]
+  int kb_wrap;                 // B is [N][kb_wrap]; A's column k pairs with B's column k % kb_wrap
   const __nv_bfloat16 *bias;   // [N]
   float *out;                  // [M][N]
   float2 *stats;               // [M][N / BN]
@@ -80,7 +81,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         uint8_t *sb = sa + BM * BK * 2;
         mbar_arrive_expect_tx(&full_bar[s], kStageBytes);
         tma_load_2d(sa, &a_map, &full_bar[s], kb * BK, m0, pol_a);
-        tma_load_2d(sb, &b_map, &full_bar[s], kb * BK, n0, pol_b);
+        tma_load_2d(sb, &b_map, &full_bar[s], (kb * BK) % g.kb_wrap, n0, pol_b);
       }
     }
   } else if (warp == 1) {
@@ -188,7 +189,10 @@ __device__ __forceinline__ float2 row_moments(const float2 *st, int ntiles, int 
 }
 
 // ---------------------------------------------------------------------------
-// LN_kv + attention pooling with the learnable queries, one block per span
+// LN_kv + attention pooling with the learnable queries, one block per span.
+// o is written as two bf16 halves, O[s][0:d] = bf16(o) and
+// O[s][d:2d] = bf16(o - bf16(o)), so that the output projection, run over
+// K = 2d against [W_o | W_o], sees o to about 16 significant bits.
 // ---------------------------------------------------------------------------
 constexpr int kPoolThreads = 256;
 
@@ -274,7 +278,10 @@ __global__ void __launch_bounds__(kPoolThreads)
       o0 += a * ((hr[0] - mom.x) * mom.y * g0 + b0);
       o1 += a * ((hr[1] - mom.x) * mom.y * g1 + b1);
     }
-    *reinterpret_cast<__nv_bfloat162 *>(O + (int64_t)s * d + c) = __floats2bfloat162_rn(o0, o1);
+    const __nv_bfloat162 hi = __floats2bfloat162_rn(o0, o1);
+    const __nv_bfloat162 lo = __floats2bfloat162_rn(o0 - __low2float(hi), o1 - __high2float(hi));
+    *reinterpret_cast<__nv_bfloat162 *>(O + (int64_t)s * 2 * d + c) = hi;
+    *reinterpret_cast<__nv_bfloat162 *>(O + (int64_t)s * 2 * d + d + c) = lo;
   }
 }
 
@@ -309,7 +316,7 @@ size_t merge_spans_workspace_bytes(int64_t T, int S, int d) {
   b += al1k((size_t)std::max<int64_t>(T, 1) * d * 2);          // E (bf16)
   b += al1k((size_t)std::max<int64_t>(T, 1) * d * 4);          // H (fp32)
   b += al1k((size_t)std::max<int64_t>(T, 1) * nt * 8);         // stats of H
-  b += al1k((size_t)std::max(S, 1) * d * 2);                   // o (bf16)
+  b += al1k((size_t)std::max(S, 1) * d * 4);                   // o as bf16 hi | lo
   b += al1k((size_t)std::max(S, 1) * nt * 8);                  // stats of Z
   return b;
 }
@@ -325,14 +332,17 @@ static bool encode_kmajor(EncodeTiledFn enc, CUtensorMap *map, const void *base,
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-static umim_status launch_gemm(EncodeTiledFn enc, const void *A, int64_t M, const void *Bw, int d,
-                               const void *bias, float *out, float2 *stats, int32_t *status, cudaStream_t st) {
+// out[M][d] = GELU(A[M][Ka] B[d][d]^T-with-wrap + bias), Ka = d or 2d
+static umim_status launch_gemm(EncodeTiledFn enc, const void *A, int64_t M, int Ka, const void *Bw, int d,
+                               const void *bias, float *out, float2 *stats, int32_t *status, cudaStream_t st,
+                               const char *label) {
   CUtensorMap am, bm;
-  if (!encode_kmajor(enc, &am, A, M, d, BM) || !encode_kmajor(enc, &bm, Bw, d, d, BN)) return UMIM_ERR_CUDA;
+  if (!encode_kmajor(enc, &am, A, M, Ka, BM) || !encode_kmajor(enc, &bm, Bw, d, d, BN)) return UMIM_ERR_CUDA;
   GemmArgs g;
   g.M = (int)M;
   g.N = d;
-  g.K = d;
+  g.K = Ka;
+  g.kb_wrap = d;
   g.bias = static_cast<const __nv_bfloat16 *>(bias);
   g.out = out;
   g.stats = stats;
@@ -345,6 +355,7 @@ static umim_status launch_gemm(EncodeTiledFn enc, const void *A, int64_t M, cons
     attr_done = true;
   }
   dim3 grid(d / BN, (unsigned)((M + BM - 1) / BM));
+  trace_mark(st, label);
   gemm_bias_gelu_kernel<<<grid, kGemmThreads, kGemmSmem, st>>>(am, bm, g);
   return cudaGetLastError() == cudaSuccess ? UMIM_OK : UMIM_ERR_CUDA;
 }
@@ -363,25 +374,29 @@ umim_status merge_spans(const void *embeddings, int64_t vocab, const int32_t *to
   float2 *st1 = reinterpret_cast<float2 *>(p);
   p += al1k((size_t)std::max<int64_t>(T, 1) * nt * 8);
   __nv_bfloat16 *O = reinterpret_cast<__nv_bfloat16 *>(p);
-  p += al1k((size_t)std::max(S, 1) * d * 2);
+  p += al1k((size_t)std::max(S, 1) * d * 4);
   float2 *st2 = reinterpret_cast<float2 *>(p);
 
   if (S == 0) return UMIM_OK;
   if (T > 0) {
     const int blocks = std::max(1, std::min<int>((int)((T + 7) / 8), num_sms * 8));
+    trace_mark(st, "merge.gather");
     gather_rows_kernel<<<blocks, 256, 0, st>>>(static_cast<const uint4 *>(embeddings), vocab, token_ids, T, d,
                                                reinterpret_cast<uint4 *>(E), status);
-    umim_status r = launch_gemm(enc, E, T, w->w_kv, d, w->b_kv, H, st1, status, st);
+    umim_status r = launch_gemm(enc, E, T, d, w->w_kv, d, w->b_kv, H, st1, status, st, "merge.gemm1");
     if (r != UMIM_OK) return r;
   }
+  trace_mark(st, "merge.pool");
   pool_kernel<<<S, kPoolThreads, 0, st>>>(H, st1, span_offsets, S, T, d, w->n_heads,
                                           static_cast<const __nv_bfloat16 *>(w->ln_kv_gamma),
                                           static_cast<const __nv_bfloat16 *>(w->ln_kv_beta),
                                           static_cast<const __nv_bfloat16 *>(w->query), w->ln_eps, O, status);
-  umim_status r = launch_gemm(enc, O, S, w->w_o, d, w->b_o, surrogates, st2, status, st);
+  umim_status r = launch_gemm(enc, O, S, 2 * d, w->w_o, d, w->b_o, surrogates, st2, status, st, "merge.gemm2");
   if (r != UMIM_OK) return r;
+  trace_mark(st, "merge.ln_o");
   ln_rows_kernel<<<S, 256, 0, st>>>(surrogates, st2, d, static_cast<const __nv_bfloat16 *>(w->ln_o_gamma),
                                     static_cast<const __nv_bfloat16 *>(w->ln_o_beta), w->ln_eps);
+  trace_mark(st, nullptr);
   return cudaGetLastError() == cudaSuccess ? UMIM_OK : UMIM_ERR_CUDA;
 }
 

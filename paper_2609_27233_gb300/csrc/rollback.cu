@@ -300,6 +300,7 @@ umim_status kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t m
   pa.n_lanes = kv->n_layers * groups;
   pa.status = status;
   pa.cu_seqlens_out = nullptr;
+  trace_mark(stream, "rollback.plan");
   if (launch_span_plan(pa, arr, stream) != cudaSuccess) return UMIM_ERR_CUDA;
 
   MoveArgs ma{};
@@ -328,7 +329,9 @@ umim_status kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t m
       per_sm < 1)
     per_sm = 1;
   const int grid = std::max(1, num_sms) * per_sm;
+  trace_mark(stream, "rollback.move");
   rollback_move_kernel<<<grid, kMoveThreads, 0, stream>>>(ma, arr);
+  trace_mark(stream, nullptr);
   return cudaGetLastError() == cudaSuccess ? UMIM_OK : UMIM_ERR_CUDA;
 }
 

@@ -1,5 +1,8 @@
 """Shared helpers of the GPU parity tests: run the CUDA path through the C ABI
 and compare with the CPU oracle on the same seeded inputs."""
+import json
+import os
+
 import numpy as np
 import torch
 
@@ -18,6 +21,11 @@ def float_close(got, want, what=""):
     assert np.all(np.isfinite(got)), f"{what}: non-finite output"
     err = np.abs(got - want)
     rel = np.linalg.norm(got - want) / max(np.linalg.norm(want), 1e-30)
+    log = os.environ.get("UMIM_PARITY_LOG")
+    if log:
+        with open(log, "a") as f:
+            f.write(json.dumps({"test": os.environ.get("PYTEST_CURRENT_TEST", "").split(" ")[0], "what": what,
+                                "max_abs": float(err.max()), "rel_l2": float(rel)}) + "\n")
     assert err.max() <= MAX_ABS, f"{what}: max abs err {err.max():.3e}"
     assert rel <= REL_L2, f"{what}: rel L2 err {rel:.3e}"
     return float(err.max()), float(rel)
