@@ -40,7 +40,7 @@
  *    the physical page id (or -1 for none).  Entry t of a sequence lives in
  *    page block_table[t / 16], slot t % 16.
  *  - Supported: head_dim 64 or 128, page size 16, 1 <= n_q_heads/n_kv_heads
- *    <= 16, d_model a multiple of 512 (<= 16384), n_heads in {1, 2, 4, 8},
+ *    <= 16, d_model a multiple of 512 (<= 8192), n_heads in {1, 2, 4, 8},
  *    merge spans of 1..4 tokens.
  *    Anything else returns UMIM_ERR_UNSUPPORTED.
  */

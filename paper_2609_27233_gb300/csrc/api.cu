@@ -78,7 +78,7 @@ bool kv_supported(const umim_paged_kv *kv) {
 }
 
 bool merge_supported(int d, int h) {
-  return d > 0 && d % 512 == 0 && d <= 16384 && (h == 1 || h == 2 || h == 4 || h == 8);
+  return d > 0 && d % 512 == 0 && d <= 8192 && (h == 1 || h == 2 || h == 4 || h == 8);
 }
 
 }  // namespace
@@ -119,8 +119,10 @@ umim_status umim_merge_spans(const void *embeddings, int64_t vocab, const int32_
   if (!w->w_kv || !w->b_kv || !w->ln_kv_gamma || !w->ln_kv_beta || !w->query || !w->w_o || !w->b_o ||
       !w->ln_o_gamma || !w->ln_o_beta)
     return UMIM_ERR_INVALID_ARG;
-  if (!aligned(embeddings, 16) || !aligned(w->w_kv, 16) || !aligned(w->w_o, 16) || !aligned(surrogates, 16))
-    return UMIM_ERR_INVALID_ARG;
+  if (!aligned(embeddings, 16) || !aligned(surrogates, 16)) return UMIM_ERR_INVALID_ARG;
+  for (const void *p : {w->w_kv, w->b_kv, w->ln_kv_gamma, w->ln_kv_beta, w->query, w->w_o, w->b_o, w->ln_o_gamma,
+                        w->ln_o_beta})
+    if (!aligned(p, 16)) return UMIM_ERR_INVALID_ARG;
   if (!workspace || !aligned(workspace, 256) ||
       workspace_bytes < merge_spans_workspace_bytes(n_tokens, n_spans, w->d_model))
     return UMIM_ERR_WORKSPACE;

@@ -22,8 +22,8 @@
 namespace umim {
 namespace {
 
-constexpr int kAttnWarps = 4;
-constexpr int kAttnStages = 4;
+constexpr int kAttnWarps = 8;
+constexpr int kAttnStages = 3;
 constexpr int kPlanThreadsA = 1024;
 
 struct AttnPlan {
@@ -357,17 +357,28 @@ __global__ void __launch_bounds__(kAttnWarps * 32, 1)
     }
     const uint32_t ks = smem_u32(kt), vs = smem_u32(vt);
 
-    // S = Q K^T   (16 x 16 keys as two n-tiles of 8)
+    // S = Q K^T   (16 x 16 keys as two n-tiles of 8); even and odd k-chunks
+    // accumulate separately to halve the dependent mma chain
     float s[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+    float s2[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
 #pragma unroll
     for (int c = 0; c < KC; ++c) {
       const int key = (lane & 7) + ((lane >> 4) << 3);
       const int c16 = 2 * c + ((lane >> 3) & 1);
       uint32_t b0, b1, b2, b3;
       ldsm_x4(ks + sw_off(key, c16), b0, b1, b2, b3);
-      mma_bf16(s[0], qa[c], b0, b1);
-      mma_bf16(s[1], qa[c], b2, b3);
+      if (c & 1) {
+        mma_bf16(s2[0], qa[c], b0, b1);
+        mma_bf16(s2[1], qa[c], b2, b3);
+      } else {
+        mma_bf16(s[0], qa[c], b0, b1);
+        mma_bf16(s[1], qa[c], b2, b3);
+      }
     }
+#pragma unroll
+    for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) s[nt][e] += s2[nt][e];
     // scale to log2 units and mask keys past the end
 #pragma unroll
     for (int nt = 0; nt < 2; ++nt)

@@ -24,6 +24,16 @@ constexpr int kGemmThreads = 192;   // warp 0: TMA, warp 1: MMA + TMEM owner, wa
 constexpr int kStageBytes = (BM + BN) * BK * 2;
 constexpr int kGemmSmem = STAGES * kStageBytes + 1024;
 
+__device__ __forceinline__ void bf16x8_to_float(uint4 u, float *f) {
+  const __nv_bfloat162 *h = reinterpret_cast<const __nv_bfloat162 *>(&u);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float2 x = __bfloat1622float2(h[i]);
+    f[2 * i] = x.x;
+    f[2 * i + 1] = x.y;
+  }
+}
+
 struct GemmArgs {
   int M, N, K;                 // A is [M][K]
   int kb_wrap;                 // B is [N][kb_wrap]; A's column k pairs with B's column k % kb_wrap
@@ -33,34 +43,40 @@ struct GemmArgs {
   int32_t *status;
 };
 
+// Persistent: each CTA walks tiles blockIdx.x, blockIdx.x + gridDim.x, ...
+// (n fastest, so CTAs running at the same time share the A block in L2).
+// The accumulator is double-buffered in tensor memory (2 x 256 columns):
+// while the epilogue warps drain tile i, the MMA thread accumulates tile i+1.
 __global__ void __launch_bounds__(kGemmThreads, 1)
     gemm_bias_gelu_kernel(const __grid_constant__ CUtensorMap a_map, const __grid_constant__ CUtensorMap b_map,
                           GemmArgs g) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
-  __shared__ uint64_t full_bar[STAGES], empty_bar[STAGES], acc_bar;
+  __shared__ uint64_t full_bar[STAGES], empty_bar[STAGES], acc_full[2], acc_empty[2];
   __shared__ uint32_t tmem_base;
-  __shared__ float s_bias[BN];
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int n0 = blockIdx.x * BN, m0 = blockIdx.y * BM;
   const int num_kb = g.K / BK;
+  const int tiles_n = g.N / BN;
+  const int tiles = tiles_n * ((g.M + BM - 1) / BM);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(&full_bar[s], 1);
       mbar_init(&empty_bar[s], 1);
     }
-    mbar_init(&acc_bar, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&acc_full[i], 1);
+      mbar_init(&acc_empty[i], 4);     // one arrival per epilogue warp
+    }
     fence_mbar_init();
     prefetch_tensormap(&a_map);
     prefetch_tensormap(&b_map);
   }
   if (warp == 1) {
-    tmem_alloc(&tmem_base, BN);
+    tmem_alloc(&tmem_base, 2 * BN);
     tmem_relinquish();
   }
-  for (int i = threadIdx.x; i < BN; i += blockDim.x) s_bias[i] = __bfloat162float(g.bias[n0 + i]);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -70,60 +86,89 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     if (lane == 0) {
       const uint64_t pol_a = policy_evict_first();
       const uint64_t pol_b = policy_evict_last();
-      for (int kb = 0; kb < num_kb; ++kb) {
-        const int s = kb % STAGES;
-        const uint32_t ph = (kb / STAGES) & 1;
-        if (!mbar_wait(&empty_bar[s], ph ^ 1)) {
-          set_error(g.status, UMIM_ERR_TIMEOUT);
-          break;
+      uint32_t it = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x) {
+        const int m0 = (tile / tiles_n) * BM, n0 = (tile % tiles_n) * BN;
+        for (int kb = 0; kb < num_kb; ++kb, ++it) {
+          const int s = it % STAGES;
+          const uint32_t ph = (it / STAGES) & 1;
+          if (!mbar_wait(&empty_bar[s], ph ^ 1)) {
+            set_error(g.status, UMIM_ERR_TIMEOUT);
+            ok = false;
+            break;
+          }
+          uint8_t *sa = smem + s * kStageBytes;
+          uint8_t *sb = sa + BM * BK * 2;
+          mbar_arrive_expect_tx(&full_bar[s], kStageBytes);
+          tma_load_2d(sa, &a_map, &full_bar[s], kb * BK, m0, pol_a);
+          tma_load_2d(sb, &b_map, &full_bar[s], (kb * BK) % g.kb_wrap, n0, pol_b);
         }
-        uint8_t *sa = smem + s * kStageBytes;
-        uint8_t *sb = sa + BM * BK * 2;
-        mbar_arrive_expect_tx(&full_bar[s], kStageBytes);
-        tma_load_2d(sa, &a_map, &full_bar[s], kb * BK, m0, pol_a);
-        tma_load_2d(sb, &b_map, &full_bar[s], (kb * BK) % g.kb_wrap, n0, pol_b);
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_bf16_f32(BM, BN);
-      for (int kb = 0; kb < num_kb; ++kb) {
-        const int s = kb % STAGES;
-        const uint32_t ph = (kb / STAGES) & 1;
-        if (!mbar_wait(&full_bar[s], ph)) {
+      uint32_t it = 0, local = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x, ++local) {
+        const uint32_t buf = local & 1, aph = (local >> 1) & 1;
+        if (!mbar_wait(&acc_empty[buf], aph ^ 1)) {
           set_error(g.status, UMIM_ERR_TIMEOUT);
           break;
         }
         tc_fence_after();
-        const uint32_t a_base = smem_u32(smem + s * kStageBytes);
-        const uint32_t b_base = a_base + BM * BK * 2;
+        const uint32_t d_tmem = tmem + buf * BN;
+        for (int kb = 0; kb < num_kb; ++kb, ++it) {
+          const int s = it % STAGES;
+          const uint32_t ph = (it / STAGES) & 1;
+          if (!mbar_wait(&full_bar[s], ph)) {
+            set_error(g.status, UMIM_ERR_TIMEOUT);
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a_base = smem_u32(smem + s * kStageBytes);
+          const uint32_t b_base = a_base + BM * BK * 2;
 #pragma unroll
-        for (int k = 0; k < BK / 16; ++k) {
-          const uint64_t ad = sw128_kmajor_desc(a_base + k * 32);
-          const uint64_t bd = sw128_kmajor_desc(b_base + k * 32);
-          tc_mma_bf16(tmem, ad, bd, idesc, (kb | k) != 0 ? 1u : 0u);
+          for (int k = 0; k < BK / 16; ++k) {
+            const uint64_t ad = sw128_kmajor_desc(a_base + k * 32);
+            const uint64_t bd = sw128_kmajor_desc(b_base + k * 32);
+            tc_mma_bf16(d_tmem, ad, bd, idesc, (kb | k) != 0 ? 1u : 0u);
+          }
+          tc_commit(&empty_bar[s]);
         }
-        tc_commit(&empty_bar[s]);
+        tc_commit(&acc_full[buf]);
       }
-      tc_commit(&acc_bar);
     }
   } else {
     const int q = warp & 3;   // TMEM lane quadrant this warp may read
-    const int row = m0 + q * 32 + lane;
-    if (!mbar_wait(&acc_bar, 0)) {
-      set_error(g.status, UMIM_ERR_TIMEOUT);
-    } else {
+    uint32_t local = 0;
+    for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x, ++local) {
+      const int m0 = (tile / tiles_n) * BM, n0 = (tile % tiles_n) * BN;
+      const uint32_t buf = local & 1, aph = (local >> 1) & 1;
+      const int row = m0 + q * 32 + lane;
+      if (!mbar_wait(&acc_full[buf], aph)) {
+        set_error(g.status, UMIM_ERR_TIMEOUT);
+        break;
+      }
       tc_fence_after();
       float mean = 0.f, m2 = 0.f, cnt = 0.f;
 #pragma unroll 1
       for (int c = 0; c < BN / 32; ++c) {
         float v[32];
-        tmem_ld_32x32b_x32(tmem + (static_cast<uint32_t>(q * 32) << 16) + c * 32, v);
+        tmem_ld_32x32b_x32(tmem + buf * BN + (static_cast<uint32_t>(q * 32) << 16) + c * 32, v);
+        const uint4 *bp = reinterpret_cast<const uint4 *>(g.bias + n0 + c * 32);
         float sum = 0.f;
 #pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          v[i] = gelu_erf(v[i] + s_bias[c * 32 + i]);
-          sum += v[i];
+        for (int i = 0; i < 4; ++i) {
+          float bb[8];
+          bf16x8_to_float(__ldg(bp + i), bb);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            v[8 * i + e] = gelu_erf(v[8 * i + e] + bb[e]);
+            sum += v[8 * i + e];
+          }
         }
         const float cm = sum * (1.f / 32.f);
         float cm2 = 0.f;
@@ -143,14 +188,18 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           for (int i = 0; i < 8; ++i) dst[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
         }
       }
-      if (row < g.M) g.stats[(int64_t)row * (g.N / BN) + blockIdx.x] = make_float2(mean, m2);
+      if (row < g.M) g.stats[(int64_t)row * tiles_n + n0 / BN] = make_float2(mean, m2);
+      // this warp's quarter of the accumulator has been read
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&acc_empty[buf]);
     }
   }
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, BN);
+    tmem_dealloc(tmem, 2 * BN);
   }
 }
 
@@ -173,44 +222,62 @@ __global__ void gather_rows_kernel(const uint4 *table, int64_t vocab, const int3
   }
 }
 
-// merge the per-tile (mean, M2) of one row into mean and 1/sqrt(var + eps)
-__device__ __forceinline__ float2 row_moments(const float2 *st, int ntiles, int d, float eps) {
-  float mean = 0.f, m2 = 0.f, cnt = 0.f;
-  for (int t = 0; t < ntiles; ++t) {
+// Running (count, mean, M2) of a row; merged pairwise (Chan et al.).
+struct Moments {
+  float n, mean, m2;
+};
+
+__device__ __forceinline__ Moments merge_moments(Moments a, Moments b) {
+  const float n = a.n + b.n;
+  if (b.n == 0.f) return a;
+  if (a.n == 0.f) return b;
+  const float delta = b.mean - a.mean, f = b.n / n;
+  return {n, a.mean + delta * f, a.m2 + b.m2 + delta * delta * a.n * f};
+}
+
+// One warp merges the per-tile (mean, M2) of a row; every lane gets
+// (mean, 1/sqrt(var + eps)).
+__device__ __forceinline__ float2 row_moments_warp(const float2 *st, int ntiles, int d, float eps) {
+  const int lane = threadIdx.x & 31;
+  Moments m{0.f, 0.f, 0.f};
+  for (int t = lane; t < ntiles; t += 32) {
     const float2 v = st[t];
-    const float nt = cnt + (float)BN;
-    const float delta = v.x - mean;
-    mean += delta * ((float)BN / nt);
-    m2 += v.y + delta * delta * (cnt * (float)BN / nt);
-    cnt = nt;
+    m = merge_moments(m, Moments{(float)BN, v.x, v.y});
   }
-  const float var = m2 / (float)d;
-  return make_float2(mean, rsqrtf(var + eps));
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) {
+    Moments x{__shfl_xor_sync(0xffffffffu, m.n, o), __shfl_xor_sync(0xffffffffu, m.mean, o),
+              __shfl_xor_sync(0xffffffffu, m.m2, o)};
+    m = merge_moments(m, x);
+  }
+  return make_float2(m.mean, rsqrtf(m.m2 / (float)d + eps));
 }
 
 // ---------------------------------------------------------------------------
-// LN_kv + attention pooling with the learnable queries, one block per span.
+// LN_kv + attention pooling with the learnable queries, one block per span,
+// d/16 threads with 16 contiguous columns each, H read once.
 // o is written as two bf16 halves, O[s][0:d] = bf16(o) and
 // O[s][d:2d] = bf16(o - bf16(o)), so that the output projection, run over
 // K = 2d against [W_o | W_o], sees o to about 16 significant bits.
 // ---------------------------------------------------------------------------
-constexpr int kPoolThreads = 256;
+constexpr int kColsPerThread = 16;
 
-__global__ void __launch_bounds__(kPoolThreads)
+__global__ void __launch_bounds__(512)
     pool_kernel(const float *H, const float2 *stats, const int32_t *offs, int S, int64_t T, int d, int h,
                 const __nv_bfloat16 *gamma, const __nv_bfloat16 *beta, const __nv_bfloat16 *query, float eps,
                 __nv_bfloat16 *O, int32_t *status) {
   const int s = blockIdx.x;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int ntiles = d / BN;
-  const int cpt = d / kPoolThreads;                // columns per thread, contiguous
-  const int c0 = tid * cpt;
+  const int c0 = tid * kColsPerThread;
   const int dh = d / h;
   const int head = c0 / dh;
-  const int tph = kPoolThreads / h;                // threads per head
+  const int tph = dh / kColsPerThread;             // threads per head
+  const int low_bit = tph & (-tph);
+  const int seg = low_bit < 32 ? low_bit : 32;     // largest power of two dividing tph, at most 32
   __shared__ float2 s_mom[UMIM_MAX_SPAN_TOKENS];
-  __shared__ float s_part[UMIM_MAX_SPAN_TOKENS][kPoolThreads / 32];
-  __shared__ float s_alpha[UMIM_MAX_SPAN_TOKENS][64];
+  __shared__ float s_red[UMIM_MAX_SPAN_TOKENS][512 / 4];
+  __shared__ float s_alpha[UMIM_MAX_SPAN_TOKENS][8];
 
   const int t0 = offs[s], t1 = offs[s + 1];
   int n = t1 - t0;
@@ -218,42 +285,63 @@ __global__ void __launch_bounds__(kPoolThreads)
     if (tid == 0) set_error(status, UMIM_ERR_INVALID_ARG);
     n = 0;
   }
-  if (warp < n) {
-    const float2 m = row_moments(stats + (int64_t)(t0 + warp) * ntiles, ntiles, d, eps);
-    if (lane == 0) s_mom[warp] = m;
+  for (int j = warp; j < n; j += (int)(blockDim.x >> 5)) {
+    const float2 m = row_moments_warp(stats + (int64_t)(t0 + j) * ntiles, ntiles, d, eps);
+    if (lane == 0) s_mom[j] = m;
   }
-  __syncthreads();
-
-  // scores s_j = <P_j[head], q_head> / sqrt(d_h), reduced over the head's threads
-  float part[UMIM_MAX_SPAN_TOKENS] = {0.f, 0.f, 0.f, 0.f};
-  for (int j = 0; j < n; ++j) {
-    const float *hr = H + (int64_t)(t0 + j) * d + c0;
-    const float2 mom = s_mom[j];
-    float acc = 0.f;
-    for (int e = 0; e < cpt; ++e) {
-      const int c = c0 + e;
-      const float p = (hr[e] - mom.x) * mom.y * __bfloat162float(gamma[c]) + __bfloat162float(beta[c]);
-      acc += p * __bfloat162float(query[(int64_t)head * dh + (c - head * dh)]);
-    }
-    part[j] = acc;
+  float g[kColsPerThread], bta[kColsPerThread], q[kColsPerThread];
+  {
+    const uint4 *gp = reinterpret_cast<const uint4 *>(gamma + c0);
+    const uint4 *bp = reinterpret_cast<const uint4 *>(beta + c0);
+    const uint4 *qp = reinterpret_cast<const uint4 *>(query + c0);   // query is [h][dh] = d contiguous values
+    bf16x8_to_float(gp[0], g);
+    bf16x8_to_float(gp[1], g + 8);
+    bf16x8_to_float(bp[0], bta);
+    bf16x8_to_float(bp[1], bta + 8);
+    bf16x8_to_float(qp[0], q);
+    bf16x8_to_float(qp[1], q + 8);
   }
+  float P[UMIM_MAX_SPAN_TOKENS][kColsPerThread];
 #pragma unroll
   for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
-    float v = part[j];
+    if (j < n) {
+      const float4 *hr = reinterpret_cast<const float4 *>(H + (int64_t)(t0 + j) * d + c0);
 #pragma unroll
-    for (int o = 16; o >= 1; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-    if (lane == 0) s_part[j][warp] = v;
+      for (int e = 0; e < 4; ++e) {
+        const float4 x = hr[e];
+        P[j][4 * e] = x.x;
+        P[j][4 * e + 1] = x.y;
+        P[j][4 * e + 2] = x.z;
+        P[j][4 * e + 3] = x.w;
+      }
+    }
   }
   __syncthreads();
-  // softmax over the span for each head (thread `head` of warp 0 handles it)
+  // P = LN_kv(H) and the partial score of this thread's columns
+#pragma unroll
+  for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
+    float part = 0.f;
+    if (j < n) {
+      const float2 mom = s_mom[j];
+#pragma unroll
+      for (int e = 0; e < kColsPerThread; ++e) {
+        P[j][e] = (P[j][e] - mom.x) * mom.y * g[e] + bta[e];
+        part += P[j][e] * q[e];
+      }
+    }
+    for (int o = seg >> 1; o >= 1; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o, seg);
+    if ((tid & (seg - 1)) == 0) s_red[j][tid / seg] = part;
+  }
+  __syncthreads();
+  // softmax over the span for each head
   if (tid < h && n > 0) {
-    const int wph = tph / 32 > 0 ? tph / 32 : 1;    // warps per head
+    const int per = tph / seg;
     float sc[UMIM_MAX_SPAN_TOKENS];
     float mx = -INFINITY;
     const float inv = rsqrtf((float)dh);
     for (int j = 0; j < n; ++j) {
       float v = 0.f;
-      for (int w = 0; w < wph; ++w) v += s_part[j][tid * wph + w];
+      for (int k = 0; k < per; ++k) v += s_red[j][tid * per + k];
       sc[j] = v * inv;
       mx = fmaxf(mx, sc[j]);
     }
@@ -265,39 +353,65 @@ __global__ void __launch_bounds__(kPoolThreads)
     for (int j = 0; j < n; ++j) s_alpha[j][tid] = sc[j] / den;
   }
   __syncthreads();
-  // o = sum_j alpha_j P_j  (bf16, the A operand of the output projection)
-  for (int e = 0; e < cpt; e += 2) {
-    float o0 = 0.f, o1 = 0.f;
-    const int c = c0 + e;
-    const float g0 = __bfloat162float(gamma[c]), g1 = __bfloat162float(gamma[c + 1]);
-    const float b0 = __bfloat162float(beta[c]), b1 = __bfloat162float(beta[c + 1]);
-    for (int j = 0; j < n; ++j) {
-      const float2 mom = s_mom[j];
+  float o[kColsPerThread];
+#pragma unroll
+  for (int e = 0; e < kColsPerThread; ++e) o[e] = 0.f;
+#pragma unroll
+  for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
+    if (j < n) {
       const float a = s_alpha[j][head];
-      const float *hr = H + (int64_t)(t0 + j) * d + c;
-      o0 += a * ((hr[0] - mom.x) * mom.y * g0 + b0);
-      o1 += a * ((hr[1] - mom.x) * mom.y * g1 + b1);
+#pragma unroll
+      for (int e = 0; e < kColsPerThread; ++e) o[e] += a * P[j][e];
     }
-    const __nv_bfloat162 hi = __floats2bfloat162_rn(o0, o1);
-    const __nv_bfloat162 lo = __floats2bfloat162_rn(o0 - __low2float(hi), o1 - __high2float(hi));
-    *reinterpret_cast<__nv_bfloat162 *>(O + (int64_t)s * 2 * d + c) = hi;
-    *reinterpret_cast<__nv_bfloat162 *>(O + (int64_t)s * 2 * d + d + c) = lo;
   }
+  uint4 hi[2], lo[2];
+  __nv_bfloat162 *hh = reinterpret_cast<__nv_bfloat162 *>(hi);
+  __nv_bfloat162 *ll = reinterpret_cast<__nv_bfloat162 *>(lo);
+#pragma unroll
+  for (int e = 0; e < kColsPerThread / 2; ++e) {
+    hh[e] = __floats2bfloat162_rn(o[2 * e], o[2 * e + 1]);
+    ll[e] = __floats2bfloat162_rn(o[2 * e] - __low2float(hh[e]), o[2 * e + 1] - __high2float(hh[e]));
+  }
+  uint4 *dh_ = reinterpret_cast<uint4 *>(O + (int64_t)s * 2 * d + c0);
+  uint4 *dl_ = reinterpret_cast<uint4 *>(O + (int64_t)s * 2 * d + d + c0);
+  dh_[0] = hi[0];
+  dh_[1] = hi[1];
+  dl_[0] = lo[0];
+  dl_[1] = lo[1];
 }
 
 // ---------------------------------------------------------------------------
-// LN_o in place over rows of Z
+// LN_o in place over rows of Z, d/16 threads per row
 // ---------------------------------------------------------------------------
-__global__ void ln_rows_kernel(float *Z, const float2 *stats, int d, const __nv_bfloat16 *gamma,
-                               const __nv_bfloat16 *beta, float eps) {
+__global__ void __launch_bounds__(512)
+    ln_rows_kernel(float *Z, const float2 *stats, int d, const __nv_bfloat16 *gamma, const __nv_bfloat16 *beta,
+                   float eps) {
   const int r = blockIdx.x;
   __shared__ float2 s_m;
-  if (threadIdx.x == 0) s_m = row_moments(stats + (int64_t)r * (d / BN), d / BN, d, eps);
+  if (threadIdx.x < 32) {
+    const float2 m = row_moments_warp(stats + (int64_t)r * (d / BN), d / BN, d, eps);
+    if (threadIdx.x == 0) s_m = m;
+  }
+  const int c0 = threadIdx.x * kColsPerThread;
+  float g[kColsPerThread], b[kColsPerThread];
+  bf16x8_to_float(reinterpret_cast<const uint4 *>(gamma + c0)[0], g);
+  bf16x8_to_float(reinterpret_cast<const uint4 *>(gamma + c0)[1], g + 8);
+  bf16x8_to_float(reinterpret_cast<const uint4 *>(beta + c0)[0], b);
+  bf16x8_to_float(reinterpret_cast<const uint4 *>(beta + c0)[1], b + 8);
+  float4 *row = reinterpret_cast<float4 *>(Z + (int64_t)r * d + c0);
+  float4 x[4];
+#pragma unroll
+  for (int e = 0; e < 4; ++e) x[e] = row[e];
   __syncthreads();
   const float2 m = s_m;
-  float *row = Z + (int64_t)r * d;
-  for (int c = threadIdx.x; c < d; c += blockDim.x)
-    row[c] = (row[c] - m.x) * m.y * __bfloat162float(gamma[c]) + __bfloat162float(beta[c]);
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    x[e].x = (x[e].x - m.x) * m.y * g[4 * e] + b[4 * e];
+    x[e].y = (x[e].y - m.x) * m.y * g[4 * e + 1] + b[4 * e + 1];
+    x[e].z = (x[e].z - m.x) * m.y * g[4 * e + 2] + b[4 * e + 2];
+    x[e].w = (x[e].w - m.x) * m.y * g[4 * e + 3] + b[4 * e + 3];
+    row[e] = x[e];
+  }
 }
 
 inline size_t al1k(size_t x) { return (x + 1023) & ~size_t(1023); }
@@ -335,7 +449,7 @@ static bool encode_kmajor(EncodeTiledFn enc, CUtensorMap *map, const void *base,
 // out[M][d] = GELU(A[M][Ka] B[d][d]^T-with-wrap + bias), Ka = d or 2d
 static umim_status launch_gemm(EncodeTiledFn enc, const void *A, int64_t M, int Ka, const void *Bw, int d,
                                const void *bias, float *out, float2 *stats, int32_t *status, cudaStream_t st,
-                               const char *label) {
+                               const char *label, int num_sms) {
   CUtensorMap am, bm;
   if (!encode_kmajor(enc, &am, A, M, Ka, BM) || !encode_kmajor(enc, &bm, Bw, d, d, BN)) return UMIM_ERR_CUDA;
   GemmArgs g;
@@ -354,7 +468,8 @@ static umim_status launch_gemm(EncodeTiledFn enc, const void *A, int64_t M, int 
       return UMIM_ERR_CUDA;
     attr_done = true;
   }
-  dim3 grid(d / BN, (unsigned)((M + BM - 1) / BM));
+  const int64_t tiles = (int64_t)(d / BN) * ((M + BM - 1) / BM);
+  const int grid = (int)std::min<int64_t>(tiles, std::max(1, num_sms));
   trace_mark(st, label);
   gemm_bias_gelu_kernel<<<grid, kGemmThreads, kGemmSmem, st>>>(am, bm, g);
   return cudaGetLastError() == cudaSuccess ? UMIM_OK : UMIM_ERR_CUDA;
@@ -383,18 +498,18 @@ umim_status merge_spans(const void *embeddings, int64_t vocab, const int32_t *to
     trace_mark(st, "merge.gather");
     gather_rows_kernel<<<blocks, 256, 0, st>>>(static_cast<const uint4 *>(embeddings), vocab, token_ids, T, d,
                                                reinterpret_cast<uint4 *>(E), status);
-    umim_status r = launch_gemm(enc, E, T, d, w->w_kv, d, w->b_kv, H, st1, status, st, "merge.gemm1");
+    umim_status r = launch_gemm(enc, E, T, d, w->w_kv, d, w->b_kv, H, st1, status, st, "merge.gemm1", num_sms);
     if (r != UMIM_OK) return r;
   }
   trace_mark(st, "merge.pool");
-  pool_kernel<<<S, kPoolThreads, 0, st>>>(H, st1, span_offsets, S, T, d, w->n_heads,
+  pool_kernel<<<S, d / kColsPerThread, 0, st>>>(H, st1, span_offsets, S, T, d, w->n_heads,
                                           static_cast<const __nv_bfloat16 *>(w->ln_kv_gamma),
                                           static_cast<const __nv_bfloat16 *>(w->ln_kv_beta),
                                           static_cast<const __nv_bfloat16 *>(w->query), w->ln_eps, O, status);
-  umim_status r = launch_gemm(enc, O, S, 2 * d, w->w_o, d, w->b_o, surrogates, st2, status, st, "merge.gemm2");
+  umim_status r = launch_gemm(enc, O, S, 2 * d, w->w_o, d, w->b_o, surrogates, st2, status, st, "merge.gemm2", num_sms);
   if (r != UMIM_OK) return r;
   trace_mark(st, "merge.ln_o");
-  ln_rows_kernel<<<S, 256, 0, st>>>(surrogates, st2, d, static_cast<const __nv_bfloat16 *>(w->ln_o_gamma),
+  ln_rows_kernel<<<S, d / kColsPerThread, 0, st>>>(surrogates, st2, d, static_cast<const __nv_bfloat16 *>(w->ln_o_gamma),
                                     static_cast<const __nv_bfloat16 *>(w->ln_o_beta), w->ln_eps);
   trace_mark(st, nullptr);
   return cudaGetLastError() == cudaSuccess ? UMIM_OK : UMIM_ERR_CUDA;

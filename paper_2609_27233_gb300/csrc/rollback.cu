@@ -72,29 +72,45 @@ __device__ __forceinline__ void st_v4(uint16_t *p, uint4 v) {
                : "memory");
 }
 
+template <int D>
 __global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a, PlanArrays arr) {
+  constexpr int CPR = D / 8;                                   // 16-byte chunks per (kv, head) row
+  constexpr int NH = kUnitBytes / (2 * kPageSize * D * 2);     // KV heads per unit
+  constexpr int CHUNKS = 2 * NH * kPageSize * CPR;
+  static_assert(CHUNKS == kChunksPerThread * kMoveThreads, "unit size");
+  constexpr int64_t kNoWrite = INT64_MIN;
+
   __shared__ int s_unit, s_b, s_lane, s_p, s_last, s_abort;
-  __shared__ int s_src[kPageSize];      // >= 0: kept source position; <= -2: span -(i+2); -1: no write
+  // per compacted slot: element offset of its source row (kv 0, first head of
+  // the unit), or -(i + 1) for the surrogate of span i, or kNoWrite
+  __shared__ int64_t s_src[kPageSize];
   __shared__ int s_dep_lo, s_dep_hi;
 
   const int tid = threadIdx.x;
   const PlanHeader *hdr = arr.hdr;
   const int total = hdr->total_units;
   const int epoch = hdr->epoch;
-  const int D = a.head_dim;
-  const int cpr = D / 8;                        // 16-byte chunks per (kv, head) row
-  const int64_t row_elems = D;
-  const int64_t slot_stride = row_elems;        // consecutive slots are consecutive rows
+  const int Hkv = a.n_kv_heads;
   const int64_t head_stride = (int64_t)kPageSize * D;
-  const int64_t kv_stride = head_stride * a.n_kv_heads;
+  const int64_t kv_stride = head_stride * Hkv;
   const int64_t page_stride = kv_stride * 2;
   const int64_t layer_stride = page_stride * a.n_pages;
 
+  // Chunk c = tid + it * 256 of a unit is 16-byte column c % CPR of row
+  // c / CPR = ((kv * NH + h) * 16 + slot).  256 is a multiple of 16 * CPR, so
+  // a thread's column and slot are the same for every it; only (kv, h) vary.
+  const int my_col = tid % CPR;
+  const int my_slot = (tid / CPR) % kPageSize;
+  const int my_kvh0 = tid / (CPR * kPageSize);
+  constexpr int KVH_STEP = kMoveThreads / (CPR * kPageSize);
+
+  // set once on a timed-out wait, never cleared: the call has failed and the
+  // remaining units skip their writes
+  if (tid == 0) s_abort = 0;
   while (true) {
     if (tid == 0) {
       const int u = atomicAdd(&arr.hdr->ticket, 1);
       s_unit = u;
-      s_abort = 0;
       if (u < total) {
         const int b = find_seq(arr.unit_base, a.B, u);
         const int rem = u - arr.unit_base[b];
@@ -109,31 +125,31 @@ __global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a,
     if (u >= total) break;
     const int b = s_b, lane = s_lane, p = s_p;
     const int layer = lane / a.n_head_groups;
-    const int hg = lane % a.n_head_groups;
-    const int h0 = hg * a.heads_per_unit;
-    const int nh = min(a.heads_per_unit, a.n_kv_heads - h0);
+    const int h0 = (lane % a.n_head_groups) * NH;
+    const int nh = min(NH, Hkv - h0);
     const int lo = a.span_offsets[b], hi = a.span_offsets[b + 1];
-    const int L = arr.seq_L[b], Lp = arr.seq_Lp[b];
-    const int s_first = a.span_start[lo];
     const int32_t *bt = a.block_table + (int64_t)b * a.max_pages;
+    const int64_t layer_base = layer * layer_stride + h0 * head_stride;
 
     if (tid < kPageSize) {
-      // source of compacted entry j
+      const int L = arr.seq_Lp[b];
       const int j = p * kPageSize + tid;
-      int src = -1;
-      if (j < Lp && j >= s_first) {
+      int64_t src = kNoWrite;
+      if (j < L && j >= a.span_start[lo]) {
         const int i = upper_index(arr.new_idx, lo, hi, j);
         if (i >= lo) {
-          if (arr.new_idx[i] == j) src = -(i + 2);
-          else {
+          if (arr.new_idx[i] == j) {
+            src = -(int64_t)i - 1;
+          } else {
             const int t = j + arr.r_incl[i];
-            src = (t != j) ? t : -1;
+            if (t != j) src = layer_base + (int64_t)bt[t / kPageSize] * page_stride + (t % kPageSize) * D;
           }
         }
       }
       s_src[tid] = src;
     } else if (tid >= 32 && tid < 32 + kPageSize) {
       // which compacted pages read old page p: kept entries t of page p that move
+      const int L = arr.seq_L[b];
       const int t = p * kPageSize + (tid - 32);
       int dpage = -1;
       if (t < L) {
@@ -158,30 +174,20 @@ __global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a,
 
     // ---- read every source chunk of this unit into registers ----
     uint4 v[kChunksPerThread];
-    const int n_chunks = 2 * nh * kPageSize * cpr;
+    const int64_t src = s_src[my_slot];
     uint32_t fold = 0;
 #pragma unroll
     for (int it = 0; it < kChunksPerThread; ++it) {
-      const int c = tid + it * kMoveThreads;
+      const int kvh = my_kvh0 + it * KVH_STEP;
+      const int h = kvh % NH, kv = kvh / NH;
       v[it] = make_uint4(0, 0, 0, 0);
-      if (c < n_chunks) {
-        const int col = c % cpr;
-        const int row = c / cpr;                 // ((kv * nh + h) * 16 + slot)
-        const int slot = row % kPageSize;
-        const int kvh = row / kPageSize;
-        const int h = h0 + kvh % nh;
-        const int kv = kvh / nh;
-        const int src = s_src[slot];
+      if (h < nh) {
         if (src >= 0) {
-          const int page = bt[src / kPageSize];
-          const uint16_t *ptr = a.pool + layer * layer_stride + page * page_stride + kv * kv_stride +
-                                h * head_stride + (src % kPageSize) * slot_stride + col * 8;
-          v[it] = ld_v4(ptr);
-        } else if (src <= -2) {
-          const int i = -src - 2;
+          v[it] = ld_v4(a.pool + src + kv * kv_stride + h * head_stride + my_col * 8);
+        } else if (src != kNoWrite) {
+          const int64_t i = -src - 1;
           const uint16_t *sur = kv ? a.sur_v : a.sur_k;
-          const uint16_t *ptr = sur + (((int64_t)i * a.n_layers + layer) * a.n_kv_heads + h) * D + col * 8;
-          v[it] = ld_v4(ptr);
+          v[it] = ld_v4(sur + ((i * a.n_layers + layer) * Hkv + h0 + h) * D + my_col * 8);
         }
       }
       fold ^= v[it].x ^ v[it].y ^ v[it].z ^ v[it].w;
@@ -190,12 +196,11 @@ __global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a,
     asm volatile("" ::"r"(fold));
     __syncthreads();
     if (tid == 0) {
-      __threadfence();
+      // release: every load of this CTA (ordered before by the barrier) is done
       st_release(&arr.flags[u], epoch);
-      // wait for the units that read old page p (all have smaller tickets)
+      // wait for the units that read old page p (all hold smaller tickets)
       const int lo_p = s_dep_lo, hi_p = s_dep_hi;
-      for (int q = lo_p; q <= hi_p && q >= 0; ++q) {
-        if (q >= p) break;
+      for (int q = lo_p; q <= hi_p && q >= 0 && q < p; ++q) {
         const int uq = u - (p - q);
         if (ld_acquire(&arr.flags[uq]) == epoch) continue;
         const uint64_t t0 = globaltimer();
@@ -213,27 +218,17 @@ __global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a,
       }
     }
     __syncthreads();
-    if (!s_abort) {
+    if (!s_abort && src != kNoWrite) {
+      const int64_t dst = layer_base + (int64_t)bt[p] * page_stride + my_slot * D + my_col * 8;
 #pragma unroll
       for (int it = 0; it < kChunksPerThread; ++it) {
-        const int c = tid + it * kMoveThreads;
-        if (c < n_chunks) {
-          const int col = c % cpr;
-          const int row = c / cpr;
-          const int slot = row % kPageSize;
-          const int kvh = row / kPageSize;
-          const int h = h0 + kvh % nh;
-          const int kv = kvh / nh;
-          if (s_src[slot] != -1) {
-            const int page = bt[p];
-            uint16_t *ptr = a.pool + layer * layer_stride + page * page_stride + kv * kv_stride +
-                            h * head_stride + slot * slot_stride + col * 8;
-            st_v4(ptr, v[it]);
-          }
-        }
+        const int kvh = my_kvh0 + it * KVH_STEP;
+        const int h = kvh % NH, kv = kvh / NH;
+        if (h < nh) st_v4(a.pool + dst + kv * kv_stride + h * head_stride, v[it]);
       }
     }
-    __syncthreads();
+    // s_src / s_abort are rewritten only after the next ticket barrier,
+    // which every thread reaches after its stores
   }
 
   // ---- the last CTA to finish truncates block tables and updates lengths ----
@@ -279,8 +274,7 @@ umim_status kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t m
                         int32_t *freed_pages, void *ws, size_t ws_bytes, int32_t *dev_status,
                         cudaStream_t stream, int num_sms) {
   const int D = kv->head_dim;
-  const int hpu = std::max(1, kUnitBytes / (2 * kPageSize * D * 2));
-  const int hp = std::min(hpu, (int)kv->n_kv_heads);
+  const int hp = kUnitBytes / (2 * kPageSize * D * 2);     // heads per unit (the kernel's NH)
   const int groups = (kv->n_kv_heads + hp - 1) / hp;
   PlanArrays arr = plan_carve(ws, B, S);
   int32_t *status = dev_status ? dev_status : &arr.hdr->status;
@@ -323,14 +317,13 @@ umim_status kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t m
   ma.freed_capacity = (int32_t)std::min<int64_t>((int64_t)B * max_pages, INT32_MAX);
   ma.B = B;
   ma.status = status;
+  auto kern = (D == 128) ? rollback_move_kernel<128> : rollback_move_kernel<64>;
   int per_sm = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, rollback_move_kernel, kMoveThreads, 0) !=
-          cudaSuccess ||
-      per_sm < 1)
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kMoveThreads, 0) != cudaSuccess || per_sm < 1)
     per_sm = 1;
   const int grid = std::max(1, num_sms) * per_sm;
   trace_mark(stream, "rollback.move");
-  rollback_move_kernel<<<grid, kMoveThreads, 0, stream>>>(ma, arr);
+  kern<<<grid, kMoveThreads, 0, stream>>>(ma, arr);
   trace_mark(stream, nullptr);
   return cudaGetLastError() == cudaSuccess ? UMIM_OK : UMIM_ERR_CUDA;
 }
