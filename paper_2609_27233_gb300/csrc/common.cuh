@@ -211,13 +211,14 @@ __device__ __forceinline__ uint64_t sw128_kmajor_desc(uint32_t smem_addr) {
   return d;
 }
 
-// Instruction descriptor: bf16 x bf16 -> fp32, both operands K-major, M x N tile.
-__host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
-  return (1u << 4)                                   // D format: fp32
-         | (1u << 7)                                 // A format: bf16
-         | (1u << 10)                                // B format: bf16
-         | (static_cast<uint32_t>(N >> 3) << 17)     // N / 8
-         | (static_cast<uint32_t>(M >> 4) << 24);    // M / 16
+// Instruction descriptor of kind::f16: both operands bf16 (or both fp16),
+// fp32 accumulate, both K-major, M x N tile.
+__host__ __device__ constexpr uint32_t idesc_f32acc(int M, int N, bool fp16_operands) {
+  return (1u << 4)                                             // D format: fp32
+         | (fp16_operands ? 0u : 1u) << 7                      // A format: fp16 = 0, bf16 = 1
+         | (fp16_operands ? 0u : 1u) << 10                     // B format (same type as A)
+         | (static_cast<uint32_t>(N >> 3) << 17)               // N / 8
+         | (static_cast<uint32_t>(M >> 4) << 24);              // M / 16
 }
 
 // ---------------------------------------------------------------------------

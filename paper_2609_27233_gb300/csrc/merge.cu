@@ -2,7 +2,7 @@
 //   gather     E   = rows of the embedding table for every span token
 //   GEMM1      H   = GELU(E W_kv^T + b_kv)        tcgen05, fp32 out + row stats
 //   pool       P   = LN_kv(H);  a_i = softmax(P_i q_i / sqrt(d_h));  o_i = a_i^T P_i
-//   GEMM2      Z   = GELU(o W_o^T + b_o)          tcgen05, fp32 out + row stats
+//   GEMM2      Z   = GELU(o W_o^T + b_o)          tcgen05 on fp16 operands, fp32 out + row stats
 //   LN_o       z   = LN_o(Z)                      in place in the output
 //
 // The two d x d projections are the only dense contractions of the module
@@ -13,6 +13,8 @@
 // spans d/256 output tiles, so each tile's epilogue writes the (mean, M2) of
 // its 256 columns per row and the next kernel merges them (Chan et al.).
 #include <algorithm>
+
+#include <cuda_fp16.h>
 
 #include "common.cuh"
 
@@ -35,8 +37,8 @@ __device__ __forceinline__ void bf16x8_to_float(uint4 u, float *f) {
 }
 
 struct GemmArgs {
-  int M, N, K;                 // A is [M][K]
-  int kb_wrap;                 // B is [N][kb_wrap]; A's column k pairs with B's column k % kb_wrap
+  int M, N, K;                 // A is [M][K], B is [N][K]
+  uint32_t idesc;              // tcgen05 instruction descriptor (operand types)
   const __nv_bfloat16 *bias;   // [N]
   float *out;                  // [M][N]
   float2 *stats;               // [M][N / BN]
@@ -102,13 +104,13 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           uint8_t *sb = sa + BM * BK * 2;
           mbar_arrive_expect_tx(&full_bar[s], kStageBytes);
           tma_load_2d(sa, &a_map, &full_bar[s], kb * BK, m0, pol_a);
-          tma_load_2d(sb, &b_map, &full_bar[s], (kb * BK) % g.kb_wrap, n0, pol_b);
+          tma_load_2d(sb, &b_map, &full_bar[s], kb * BK, n0, pol_b);
         }
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {
-      constexpr uint32_t idesc = idesc_bf16_f32(BM, BN);
+      const uint32_t idesc = g.idesc;
       uint32_t it = 0, local = 0;
       bool ok = true;
       for (int tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x, ++local) {
@@ -255,17 +257,15 @@ __device__ __forceinline__ float2 row_moments_warp(const float2 *st, int ntiles,
 
 // ---------------------------------------------------------------------------
 // LN_kv + attention pooling with the learnable queries, one block per span,
-// d/16 threads with 16 contiguous columns each, H read once.
-// o is written as two bf16 halves, O[s][0:d] = bf16(o) and
-// O[s][d:2d] = bf16(o - bf16(o)), so that the output projection, run over
-// K = 2d against [W_o | W_o], sees o to about 16 significant bits.
+// d/16 threads with 16 contiguous columns each, H read once.  o is written
+// in fp16 (11 significant bits) as the A operand of the output projection.
 // ---------------------------------------------------------------------------
 constexpr int kColsPerThread = 16;
 
 __global__ void __launch_bounds__(512)
     pool_kernel(const float *H, const float2 *stats, const int32_t *offs, int S, int64_t T, int d, int h,
                 const __nv_bfloat16 *gamma, const __nv_bfloat16 *beta, const __nv_bfloat16 *query, float eps,
-                __nv_bfloat16 *O, int32_t *status) {
+                __half *O, int32_t *status) {
   const int s = blockIdx.x;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int ntiles = d / BN;
@@ -364,20 +364,27 @@ __global__ void __launch_bounds__(512)
       for (int e = 0; e < kColsPerThread; ++e) o[e] += a * P[j][e];
     }
   }
-  uint4 hi[2], lo[2];
-  __nv_bfloat162 *hh = reinterpret_cast<__nv_bfloat162 *>(hi);
-  __nv_bfloat162 *ll = reinterpret_cast<__nv_bfloat162 *>(lo);
+  uint4 packed[2];
+  __half2 *hp = reinterpret_cast<__half2 *>(packed);
 #pragma unroll
-  for (int e = 0; e < kColsPerThread / 2; ++e) {
-    hh[e] = __floats2bfloat162_rn(o[2 * e], o[2 * e + 1]);
-    ll[e] = __floats2bfloat162_rn(o[2 * e] - __low2float(hh[e]), o[2 * e + 1] - __high2float(hh[e]));
+  for (int e = 0; e < kColsPerThread / 2; ++e) hp[e] = __floats2half2_rn(o[2 * e], o[2 * e + 1]);
+  uint4 *dst = reinterpret_cast<uint4 *>(O + (int64_t)s * d + c0);
+  dst[0] = packed[0];
+  dst[1] = packed[1];
+}
+
+// W_o from bf16 to fp16 (exact for values in fp16's normal range)
+__global__ void bf16_to_f16_kernel(const uint4 *in, uint4 *out, int64_t n_vec) {
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n_vec; i += (int64_t)gridDim.x * blockDim.x) {
+    const uint4 u = in[i];
+    float f[8];
+    bf16x8_to_float(u, f);
+    uint4 o;
+    __half2 *h = reinterpret_cast<__half2 *>(&o);
+#pragma unroll
+    for (int e = 0; e < 4; ++e) h[e] = __floats2half2_rn(f[2 * e], f[2 * e + 1]);
+    out[i] = o;
   }
-  uint4 *dh_ = reinterpret_cast<uint4 *>(O + (int64_t)s * 2 * d + c0);
-  uint4 *dl_ = reinterpret_cast<uint4 *>(O + (int64_t)s * 2 * d + d + c0);
-  dh_[0] = hi[0];
-  dh_[1] = hi[1];
-  dl_[0] = lo[0];
-  dl_[1] = lo[1];
 }
 
 // ---------------------------------------------------------------------------
@@ -430,33 +437,36 @@ size_t merge_spans_workspace_bytes(int64_t T, int S, int d) {
   b += al1k((size_t)std::max<int64_t>(T, 1) * d * 2);          // E (bf16)
   b += al1k((size_t)std::max<int64_t>(T, 1) * d * 4);          // H (fp32)
   b += al1k((size_t)std::max<int64_t>(T, 1) * nt * 8);         // stats of H
-  b += al1k((size_t)std::max(S, 1) * d * 4);                   // o as bf16 hi | lo
+  b += al1k((size_t)std::max(S, 1) * d * 2);                   // o (fp16)
+  b += al1k((size_t)d * d * 2);                                 // W_o (fp16)
   b += al1k((size_t)std::max(S, 1) * nt * 8);                  // stats of Z
   return b;
 }
 
 static bool encode_kmajor(EncodeTiledFn enc, CUtensorMap *map, const void *base, int64_t rows, int K,
-                          int box_rows) {
+                          int box_rows, bool fp16) {
   const cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)rows};
   const cuuint64_t strides[1] = {(cuuint64_t)K * 2};
   const cuuint32_t box[2] = {(cuuint32_t)BK, (cuuint32_t)box_rows};
   const cuuint32_t es[2] = {1, 1};
-  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, es,
+  return enc(map, fp16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+             const_cast<void *>(base), dims, strides, box, es,
              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// out[M][d] = GELU(A[M][Ka] B[d][d]^T-with-wrap + bias), Ka = d or 2d
-static umim_status launch_gemm(EncodeTiledFn enc, const void *A, int64_t M, int Ka, const void *Bw, int d,
+// out[M][d] = GELU(A[M][d] B[d][d]^T + bias); A and B both bf16 or both fp16
+static umim_status launch_gemm(EncodeTiledFn enc, const void *A, int64_t M, const void *Bw, int d, bool fp16,
                                const void *bias, float *out, float2 *stats, int32_t *status, cudaStream_t st,
                                const char *label, int num_sms) {
   CUtensorMap am, bm;
-  if (!encode_kmajor(enc, &am, A, M, Ka, BM) || !encode_kmajor(enc, &bm, Bw, d, d, BN)) return UMIM_ERR_CUDA;
+  if (!encode_kmajor(enc, &am, A, M, d, BM, fp16) || !encode_kmajor(enc, &bm, Bw, d, d, BN, fp16))
+    return UMIM_ERR_CUDA;
   GemmArgs g;
   g.M = (int)M;
   g.N = d;
-  g.K = Ka;
-  g.kb_wrap = d;
+  g.K = d;
+  g.idesc = idesc_f32acc(BM, BN, fp16);
   g.bias = static_cast<const __nv_bfloat16 *>(bias);
   g.out = out;
   g.stats = stats;
@@ -488,8 +498,10 @@ umim_status merge_spans(const void *embeddings, int64_t vocab, const int32_t *to
   p += al1k((size_t)std::max<int64_t>(T, 1) * d * 4);
   float2 *st1 = reinterpret_cast<float2 *>(p);
   p += al1k((size_t)std::max<int64_t>(T, 1) * nt * 8);
-  __nv_bfloat16 *O = reinterpret_cast<__nv_bfloat16 *>(p);
-  p += al1k((size_t)std::max(S, 1) * d * 4);
+  __half *O = reinterpret_cast<__half *>(p);
+  p += al1k((size_t)std::max(S, 1) * d * 2);
+  __half *Wo16 = reinterpret_cast<__half *>(p);
+  p += al1k((size_t)d * d * 2);
   float2 *st2 = reinterpret_cast<float2 *>(p);
 
   if (S == 0) return UMIM_OK;
@@ -498,7 +510,7 @@ umim_status merge_spans(const void *embeddings, int64_t vocab, const int32_t *to
     trace_mark(st, "merge.gather");
     gather_rows_kernel<<<blocks, 256, 0, st>>>(static_cast<const uint4 *>(embeddings), vocab, token_ids, T, d,
                                                reinterpret_cast<uint4 *>(E), status);
-    umim_status r = launch_gemm(enc, E, T, d, w->w_kv, d, w->b_kv, H, st1, status, st, "merge.gemm1", num_sms);
+    umim_status r = launch_gemm(enc, E, T, w->w_kv, d, false, w->b_kv, H, st1, status, st, "merge.gemm1", num_sms);
     if (r != UMIM_OK) return r;
   }
   trace_mark(st, "merge.pool");
@@ -506,7 +518,10 @@ umim_status merge_spans(const void *embeddings, int64_t vocab, const int32_t *to
                                           static_cast<const __nv_bfloat16 *>(w->ln_kv_gamma),
                                           static_cast<const __nv_bfloat16 *>(w->ln_kv_beta),
                                           static_cast<const __nv_bfloat16 *>(w->query), w->ln_eps, O, status);
-  umim_status r = launch_gemm(enc, O, S, 2 * d, w->w_o, d, w->b_o, surrogates, st2, status, st, "merge.gemm2", num_sms);
+  trace_mark(st, "merge.wo_f16");
+  bf16_to_f16_kernel<<<std::max(1, num_sms) * 4, 256, 0, st>>>(static_cast<const uint4 *>(w->w_o), reinterpret_cast<uint4 *>(Wo16),
+                                                  (int64_t)d * d / 8);
+  umim_status r = launch_gemm(enc, O, S, Wo16, d, true, w->b_o, surrogates, st2, status, st, "merge.gemm2", num_sms);
   if (r != UMIM_OK) return r;
   trace_mark(st, "merge.ln_o");
   ln_rows_kernel<<<S, d / kColsPerThread, 0, st>>>(surrogates, st2, d, static_cast<const __nv_bfloat16 *>(w->ln_o_gamma),

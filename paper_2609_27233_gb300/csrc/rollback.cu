@@ -22,6 +22,7 @@ namespace {
 constexpr int kMoveThreads = 256;
 constexpr int kUnitBytes = 32768;                     // data moved per unit
 constexpr int kChunksPerThread = kUnitBytes / 16 / kMoveThreads;   // 8 x 16 B
+constexpr int64_t kNoWrite = INT64_MIN;
 
 struct MoveArgs {
   uint16_t *pool;
@@ -72,21 +73,41 @@ __device__ __forceinline__ void st_v4(uint16_t *p, uint4 v) {
                : "memory");
 }
 
+__device__ __forceinline__ void cp_async_16(void *smem, const void *gmem) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(smem)), "l"(gmem) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+constexpr int kRing = 3;   // units in flight per CTA
+
+struct UnitMeta {
+  int unit, b, lane, p, nh, h0, dep_lo, dep_hi;
+  int64_t src[kPageSize];   // source row offset (kv 0, head h0), -(i+1) for surrogate i, or kNoWrite
+};
+
 template <int D>
 __global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a, PlanArrays arr) {
   constexpr int CPR = D / 8;                                   // 16-byte chunks per (kv, head) row
   constexpr int NH = kUnitBytes / (2 * kPageSize * D * 2);     // KV heads per unit
   constexpr int CHUNKS = 2 * NH * kPageSize * CPR;
   static_assert(CHUNKS == kChunksPerThread * kMoveThreads, "unit size");
-  constexpr int64_t kNoWrite = INT64_MIN;
+  // Chunk c = tid + it * 256 of a unit is 16-byte column c % CPR of row
+  // c / CPR = ((kv * NH + h) * 16 + slot).  256 is a multiple of 16 * CPR, so
+  // a thread's column and slot are the same for every it; only (kv, h) vary.
+  const int tid = threadIdx.x, lane_id = tid & 31;
+  const int my_col = tid % CPR;
+  const int my_slot = (tid / CPR) % kPageSize;
+  const int my_kvh0 = tid / (CPR * kPageSize);
+  constexpr int KVH_STEP = kMoveThreads / (CPR * kPageSize);
 
-  __shared__ int s_unit, s_b, s_lane, s_p, s_last, s_abort;
-  // per compacted slot: element offset of its source row (kv 0, first head of
-  // the unit), or -(i + 1) for the surrogate of span i, or kNoWrite
-  __shared__ int64_t s_src[kPageSize];
-  __shared__ int s_dep_lo, s_dep_hi;
+  extern __shared__ __align__(16) uint8_t ring[];              // kRing x 32 KB of unit data
+  __shared__ UnitMeta meta[kRing + 1];
+  __shared__ int s_last, s_abort;
 
-  const int tid = threadIdx.x;
   const PlanHeader *hdr = arr.hdr;
   const int total = hdr->total_units;
   const int epoch = hdr->epoch;
@@ -96,44 +117,36 @@ __global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a,
   const int64_t page_stride = kv_stride * 2;
   const int64_t layer_stride = page_stride * a.n_pages;
 
-  // Chunk c = tid + it * 256 of a unit is 16-byte column c % CPR of row
-  // c / CPR = ((kv * NH + h) * 16 + slot).  256 is a multiple of 16 * CPR, so
-  // a thread's column and slot are the same for every it; only (kv, h) vary.
-  const int my_col = tid % CPR;
-  const int my_slot = (tid / CPR) % kPageSize;
-  const int my_kvh0 = tid / (CPR * kPageSize);
-  constexpr int KVH_STEP = kMoveThreads / (CPR * kPageSize);
-
-  // set once on a timed-out wait, never cleared: the call has failed and the
-  // remaining units skip their writes
-  if (tid == 0) s_abort = 0;
-  while (true) {
-    if (tid == 0) {
-      const int u = atomicAdd(&arr.hdr->ticket, 1);
-      s_unit = u;
+  // warp 0: take the next ticket and describe the unit in meta[m]
+  auto describe = [&](int m) {
+    int u = 0, b = 0, ln = 0, p = 0;
+    if (lane_id == 0) {
+      u = atomicAdd(&arr.hdr->ticket, 1);
       if (u < total) {
-        const int b = find_seq(arr.unit_base, a.B, u);
+        b = find_seq(arr.unit_base, a.B, u);
         const int rem = u - arr.unit_base[b];
         const int nd = arr.n_dest[b];
-        s_b = b;
-        s_lane = rem / nd;
-        s_p = arr.first_page[b] + rem % nd;
+        ln = rem / nd;
+        p = arr.first_page[b] + rem % nd;
       }
     }
-    __syncthreads();
-    const int u = s_unit;
-    if (u >= total) break;
-    const int b = s_b, lane = s_lane, p = s_p;
-    const int layer = lane / a.n_head_groups;
-    const int h0 = (lane % a.n_head_groups) * NH;
-    const int nh = min(NH, Hkv - h0);
+    u = __shfl_sync(0xffffffffu, u, 0);
+    UnitMeta &M = meta[m];
+    if (u >= total) {
+      if (lane_id == 0) M.unit = u;
+      return;
+    }
+    b = __shfl_sync(0xffffffffu, b, 0);
+    ln = __shfl_sync(0xffffffffu, ln, 0);
+    p = __shfl_sync(0xffffffffu, p, 0);
+    const int layer = ln / a.n_head_groups;
+    const int h0 = (ln % a.n_head_groups) * NH;
     const int lo = a.span_offsets[b], hi = a.span_offsets[b + 1];
     const int32_t *bt = a.block_table + (int64_t)b * a.max_pages;
-    const int64_t layer_base = layer * layer_stride + h0 * head_stride;
-
-    if (tid < kPageSize) {
+    if (lane_id < kPageSize) {
+      // source of compacted entry j
       const int L = arr.seq_Lp[b];
-      const int j = p * kPageSize + tid;
+      const int j = p * kPageSize + lane_id;
       int64_t src = kNoWrite;
       if (j < L && j >= a.span_start[lo]) {
         const int i = upper_index(arr.new_idx, lo, hi, j);
@@ -142,16 +155,19 @@ __global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a,
             src = -(int64_t)i - 1;
           } else {
             const int t = j + arr.r_incl[i];
-            if (t != j) src = layer_base + (int64_t)bt[t / kPageSize] * page_stride + (t % kPageSize) * D;
+            if (t != j)
+              src = layer * layer_stride + h0 * head_stride + (int64_t)bt[t / kPageSize] * page_stride +
+                    (t % kPageSize) * D;
           }
         }
       }
-      s_src[tid] = src;
-    } else if (tid >= 32 && tid < 32 + kPageSize) {
-      // which compacted pages read old page p: kept entries t of page p that move
+      M.src[lane_id] = src;
+    }
+    // which compacted pages read old page p: kept entries t of page p that move
+    int dpage = -1;
+    if (lane_id >= 16) {
       const int L = arr.seq_L[b];
-      const int t = p * kPageSize + (tid - 32);
-      int dpage = -1;
+      const int t = p * kPageSize + (lane_id - 16);
       if (t < L) {
         const int i = upper_index(a.span_start, lo, hi, t);
         if (i >= lo && t >= a.span_start[i] + a.span_len[i]) {
@@ -159,48 +175,78 @@ __global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a,
           if (r > 0) dpage = (t - r) / kPageSize;
         }
       }
-      int mn = dpage < 0 ? 0x7fffffff : dpage, mx = dpage;
-#pragma unroll
-      for (int o = 8; o >= 1; o >>= 1) {
-        mn = min(mn, __shfl_xor_sync(0xffffu, mn, o, 16));
-        mx = max(mx, __shfl_xor_sync(0xffffu, mx, o, 16));
-      }
-      if (tid == 32) {
-        s_dep_lo = mn;
-        s_dep_hi = mx;
-      }
     }
-    __syncthreads();
-
-    // ---- read every source chunk of this unit into registers ----
-    uint4 v[kChunksPerThread];
-    const int64_t src = s_src[my_slot];
-    uint32_t fold = 0;
+    int mn = dpage < 0 ? 0x7fffffff : dpage, mx = dpage;
 #pragma unroll
-    for (int it = 0; it < kChunksPerThread; ++it) {
-      const int kvh = my_kvh0 + it * KVH_STEP;
-      const int h = kvh % NH, kv = kvh / NH;
-      v[it] = make_uint4(0, 0, 0, 0);
-      if (h < nh) {
-        if (src >= 0) {
-          v[it] = ld_v4(a.pool + src + kv * kv_stride + h * head_stride + my_col * 8);
-        } else if (src != kNoWrite) {
-          const int64_t i = -src - 1;
-          const uint16_t *sur = kv ? a.sur_v : a.sur_k;
-          v[it] = ld_v4(sur + ((i * a.n_layers + layer) * Hkv + h0 + h) * D + my_col * 8);
+    for (int o = 8; o >= 1; o >>= 1) {
+      mn = min(mn, __shfl_xor_sync(0xffffffffu, mn, o));
+      mx = max(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    }
+    mn = __shfl_sync(0xffffffffu, mn, 16);
+    mx = __shfl_sync(0xffffffffu, mx, 16);
+    if (lane_id == 0) {
+      M.unit = u;
+      M.b = b;
+      M.lane = layer;
+      M.p = p;
+      M.h0 = h0;
+      M.nh = min(NH, Hkv - h0);
+      M.dep_lo = mn;
+      M.dep_hi = mx;
+    }
+  };
+
+  // every thread: start the copies of the unit in meta[m] into ring stage st
+  auto issue = [&](int m, int st) {
+    const UnitMeta &M = meta[m];
+    if (M.unit < total) {
+      const int64_t src = M.src[my_slot];
+      uint8_t *dst = ring + st * kUnitBytes;
+#pragma unroll
+      for (int it = 0; it < kChunksPerThread; ++it) {
+        const int kvh = my_kvh0 + it * KVH_STEP;
+        const int h = kvh % NH, kv = kvh / NH;
+        if (h < M.nh && src != kNoWrite) {
+          const uint16_t *g;
+          if (src >= 0) {
+            g = a.pool + src + kv * kv_stride + h * head_stride + my_col * 8;
+          } else {
+            const int64_t i = -src - 1;
+            g = (kv ? a.sur_v : a.sur_k) + ((i * a.n_layers + M.lane) * Hkv + M.h0 + h) * D + my_col * 8;
+          }
+          cp_async_16(dst + (tid + it * kMoveThreads) * 16, g);
         }
       }
-      fold ^= v[it].x ^ v[it].y ^ v[it].z ^ v[it].w;
     }
-    // every loaded value has arrived before this thread reaches the barrier
-    asm volatile("" ::"r"(fold));
+    cp_async_commit();   // one group per ring slot, empty or not
+  };
+
+  if (tid == 0) s_abort = 0;
+  // prologue: kRing - 1 units in flight
+  int head = 0;   // units described so far by this CTA
+  for (int k = 0; k < kRing - 1; ++k) {
+    if (tid < 32) describe(head % (kRing + 1));
     __syncthreads();
+    issue(head % (kRing + 1), head % kRing);
+    ++head;
+  }
+  for (int cur = 0;; ++cur) {
+    // describe and start one more unit, then wait for the oldest one's copies
+    if (tid < 32) describe(head % (kRing + 1));
+    __syncthreads();
+    issue(head % (kRing + 1), head % kRing);
+    ++head;
+    cp_async_wait<kRing - 1>();
+    __syncthreads();
+    const UnitMeta &M = meta[cur % (kRing + 1)];
+    const int u = M.unit;
+    if (u >= total) break;     // tickets are taken in order: nothing younger exists either
+    const int p = M.p;
     if (tid == 0) {
-      // release: every load of this CTA (ordered before by the barrier) is done
+      // release: every copy of this unit has landed (wait_group + barrier)
       st_release(&arr.flags[u], epoch);
       // wait for the units that read old page p (all hold smaller tickets)
-      const int lo_p = s_dep_lo, hi_p = s_dep_hi;
-      for (int q = lo_p; q <= hi_p && q >= 0 && q < p; ++q) {
+      for (int q = M.dep_lo; q <= M.dep_hi && q >= 0 && q < p; ++q) {
         const int uq = u - (p - q);
         if (ld_acquire(&arr.flags[uq]) == epoch) continue;
         const uint64_t t0 = globaltimer();
@@ -218,18 +264,24 @@ __global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a,
       }
     }
     __syncthreads();
+    const int64_t src = M.src[my_slot];
     if (!s_abort && src != kNoWrite) {
-      const int64_t dst = layer_base + (int64_t)bt[p] * page_stride + my_slot * D + my_col * 8;
+      const int32_t *bt = a.block_table + (int64_t)M.b * a.max_pages;
+      const int64_t dst = M.lane * layer_stride + M.h0 * head_stride + (int64_t)bt[p] * page_stride +
+                          my_slot * D + my_col * 8;
+      const uint8_t *stage = ring + (cur % kRing) * kUnitBytes;
 #pragma unroll
       for (int it = 0; it < kChunksPerThread; ++it) {
         const int kvh = my_kvh0 + it * KVH_STEP;
         const int h = kvh % NH, kv = kvh / NH;
-        if (h < nh) st_v4(a.pool + dst + kv * kv_stride + h * head_stride, v[it]);
+        if (h < M.nh) {
+          const uint4 v = *reinterpret_cast<const uint4 *>(stage + (tid + it * kMoveThreads) * 16);
+          st_v4(a.pool + dst + kv * kv_stride + h * head_stride, v);
+        }
       }
     }
-    // s_src / s_abort are rewritten only after the next ticket barrier,
-    // which every thread reaches after its stores
   }
+  cp_async_wait<0>();
 
   // ---- the last CTA to finish truncates block tables and updates lengths ----
   if (tid == 0) {
@@ -318,12 +370,15 @@ umim_status kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t m
   ma.B = B;
   ma.status = status;
   auto kern = (D == 128) ? rollback_move_kernel<128> : rollback_move_kernel<64>;
+  const int smem = kRing * kUnitBytes;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
+    return UMIM_ERR_CUDA;
   int per_sm = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kMoveThreads, 0) != cudaSuccess || per_sm < 1)
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kMoveThreads, smem) != cudaSuccess || per_sm < 1)
     per_sm = 1;
   const int grid = std::max(1, num_sms) * per_sm;
   trace_mark(stream, "rollback.move");
-  kern<<<grid, kMoveThreads, 0, stream>>>(ma, arr);
+  kern<<<grid, kMoveThreads, smem, stream>>>(ma, arr);
   trace_mark(stream, nullptr);
   return cudaGetLastError() == cudaSuccess ? UMIM_OK : UMIM_ERR_CUDA;
 }
