@@ -175,7 +175,7 @@ umim_status umim_kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int3
                              size_t workspace_bytes, int32_t *dev_status, cudaStream_t stream) {
   if (!kv_ok(kv) || batch < 0 || max_pages < 0 || n_spans < 0) return UMIM_ERR_INVALID_ARG;
   if (!kv_supported(kv)) return UMIM_ERR_UNSUPPORTED;
-  if ((int64_t)batch * max_pages > INT32_MAX / 16) return UMIM_ERR_UNSUPPORTED;
+  if ((int64_t)batch * max_pages > INT32_MAX / 16 || batch > 65535) return UMIM_ERR_UNSUPPORTED;
   if (batch == 0) return UMIM_OK;
   if (!block_table || !seq_lens || !span_offsets) return UMIM_ERR_INVALID_ARG;
   if (n_spans > 0 && (!span_start || !span_len || !surrogate_k || !surrogate_v)) return UMIM_ERR_INVALID_ARG;

@@ -1,6 +1,6 @@
 // Merge module M_phi forward (App. C.1; Sec. 3.2 Eq. 1) for a batch of spans:
 //   gather     E   = rows of the embedding table for every span token
-//   GEMM1      H   = GELU(E W_kv^T + b_kv)        tcgen05, fp32 out + row stats
+//   GEMM1      H   = GELU(E W_kv^T + b_kv)        tcgen05, fp16 out + row stats of the fp32 values
 //   pool       P   = LN_kv(H);  a_i = softmax(P_i q_i / sqrt(d_h));  o_i = a_i^T P_i
 //   GEMM2      Z   = GELU(o W_o^T + b_o)          tcgen05 on fp16 operands, fp32 out + row stats
 //   LN_o       z   = LN_o(Z)                      in place in the output
@@ -36,11 +36,12 @@ __device__ __forceinline__ void bf16x8_to_float(uint4 u, float *f) {
   }
 }
 
+template <typename OutT>
 struct GemmArgs {
   int M, N, K;                 // A is [M][K], B is [N][K]
   uint32_t idesc;              // tcgen05 instruction descriptor (operand types)
   const __nv_bfloat16 *bias;   // [N]
-  float *out;                  // [M][N]
+  OutT *out;                   // [M][N]
   float2 *stats;               // [M][N / BN]
   int32_t *status;
 };
@@ -49,9 +50,28 @@ struct GemmArgs {
 // (n fastest, so CTAs running at the same time share the A block in L2).
 // The accumulator is double-buffered in tensor memory (2 x 256 columns):
 // while the epilogue warps drain tile i, the MMA thread accumulates tile i+1.
+__device__ __forceinline__ void store32(float *dst, const float (&v)[32]) {
+  float4 *d4 = reinterpret_cast<float4 *>(dst);
+#pragma unroll
+  for (int i = 0; i < 8; ++i) d4[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+}
+
+__device__ __forceinline__ void store32(__half *dst, const float (&v)[32]) {
+  uint4 *d4 = reinterpret_cast<uint4 *>(dst);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    uint4 u;
+    __half2 *h = reinterpret_cast<__half2 *>(&u);
+#pragma unroll
+    for (int e = 0; e < 4; ++e) h[e] = __floats2half2_rn(v[8 * i + 2 * e], v[8 * i + 2 * e + 1]);
+    d4[i] = u;
+  }
+}
+
+template <typename OutT>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     gemm_bias_gelu_kernel(const __grid_constant__ CUtensorMap a_map, const __grid_constant__ CUtensorMap b_map,
-                          GemmArgs g) {
+                          GemmArgs<OutT> g) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   __shared__ uint64_t full_bar[STAGES], empty_bar[STAGES], acc_full[2], acc_empty[2];
   __shared__ uint32_t tmem_base;
@@ -184,11 +204,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         mean += delta * (32.f / nt);
         m2 += cm2 + delta * delta * (cnt * 32.f / nt);
         cnt = nt;
-        if (row < g.M) {
-          float4 *dst = reinterpret_cast<float4 *>(g.out + (int64_t)row * g.N + n0 + c * 32);
-#pragma unroll
-          for (int i = 0; i < 8; ++i) dst[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
-        }
+        if (row < g.M) store32(g.out + (int64_t)row * g.N + n0 + c * 32, v);
       }
       if (row < g.M) g.stats[(int64_t)row * tiles_n + n0 / BN] = make_float2(mean, m2);
       // this warp's quarter of the accumulator has been read
@@ -263,7 +279,7 @@ __device__ __forceinline__ float2 row_moments_warp(const float2 *st, int ntiles,
 constexpr int kColsPerThread = 16;
 
 __global__ void __launch_bounds__(512)
-    pool_kernel(const float *H, const float2 *stats, const int32_t *offs, int S, int64_t T, int d, int h,
+    pool_kernel(const __half *H, const float2 *stats, const int32_t *offs, int S, int64_t T, int d, int h,
                 const __nv_bfloat16 *gamma, const __nv_bfloat16 *beta, const __nv_bfloat16 *query, float eps,
                 __half *O, int32_t *status) {
   const int s = blockIdx.x;
@@ -305,14 +321,17 @@ __global__ void __launch_bounds__(512)
 #pragma unroll
   for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
     if (j < n) {
-      const float4 *hr = reinterpret_cast<const float4 *>(H + (int64_t)(t0 + j) * d + c0);
+      const uint4 *hr = reinterpret_cast<const uint4 *>(H + (int64_t)(t0 + j) * d + c0);
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const float4 x = hr[e];
-        P[j][4 * e] = x.x;
-        P[j][4 * e + 1] = x.y;
-        P[j][4 * e + 2] = x.z;
-        P[j][4 * e + 3] = x.w;
+      for (int e = 0; e < 2; ++e) {
+        const uint4 x = hr[e];
+        const __half2 *h2 = reinterpret_cast<const __half2 *>(&x);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const float2 f = __half22float2(h2[k]);
+          P[j][8 * e + 2 * k] = f.x;
+          P[j][8 * e + 2 * k + 1] = f.y;
+        }
       }
     }
   }
@@ -435,7 +454,7 @@ size_t merge_spans_workspace_bytes(int64_t T, int S, int d) {
   const int nt = d / BN;
   size_t b = 0;
   b += al1k((size_t)std::max<int64_t>(T, 1) * d * 2);          // E (bf16)
-  b += al1k((size_t)std::max<int64_t>(T, 1) * d * 4);          // H (fp32)
+  b += al1k((size_t)std::max<int64_t>(T, 1) * d * 2);          // H (fp16)
   b += al1k((size_t)std::max<int64_t>(T, 1) * nt * 8);         // stats of H
   b += al1k((size_t)std::max(S, 1) * d * 2);                   // o (fp16)
   b += al1k((size_t)d * d * 2);                                 // W_o (fp16)
@@ -456,13 +475,14 @@ static bool encode_kmajor(EncodeTiledFn enc, CUtensorMap *map, const void *base,
 }
 
 // out[M][d] = GELU(A[M][d] B[d][d]^T + bias); A and B both bf16 or both fp16
+template <typename OutT>
 static umim_status launch_gemm(EncodeTiledFn enc, const void *A, int64_t M, const void *Bw, int d, bool fp16,
-                               const void *bias, float *out, float2 *stats, int32_t *status, cudaStream_t st,
+                               const void *bias, OutT *out, float2 *stats, int32_t *status, cudaStream_t st,
                                const char *label, int num_sms) {
   CUtensorMap am, bm;
   if (!encode_kmajor(enc, &am, A, M, d, BM, fp16) || !encode_kmajor(enc, &bm, Bw, d, d, BN, fp16))
     return UMIM_ERR_CUDA;
-  GemmArgs g;
+  GemmArgs<OutT> g;
   g.M = (int)M;
   g.N = d;
   g.K = d;
@@ -473,15 +493,15 @@ static umim_status launch_gemm(EncodeTiledFn enc, const void *A, int64_t M, cons
   g.status = status;
   static bool attr_done = false;
   if (!attr_done) {
-    if (cudaFuncSetAttribute(gemm_bias_gelu_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kGemmSmem) !=
-        cudaSuccess)
+    if (cudaFuncSetAttribute(gemm_bias_gelu_kernel<OutT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             kGemmSmem) != cudaSuccess)
       return UMIM_ERR_CUDA;
     attr_done = true;
   }
   const int64_t tiles = (int64_t)(d / BN) * ((M + BM - 1) / BM);
   const int grid = (int)std::min<int64_t>(tiles, std::max(1, num_sms));
   trace_mark(st, label);
-  gemm_bias_gelu_kernel<<<grid, kGemmThreads, kGemmSmem, st>>>(am, bm, g);
+  gemm_bias_gelu_kernel<OutT><<<grid, kGemmThreads, kGemmSmem, st>>>(am, bm, g);
   return cudaGetLastError() == cudaSuccess ? UMIM_OK : UMIM_ERR_CUDA;
 }
 
@@ -494,8 +514,8 @@ umim_status merge_spans(const void *embeddings, int64_t vocab, const int32_t *to
   char *p = static_cast<char *>(workspace);
   __nv_bfloat16 *E = reinterpret_cast<__nv_bfloat16 *>(p);
   p += al1k((size_t)std::max<int64_t>(T, 1) * d * 2);
-  float *H = reinterpret_cast<float *>(p);
-  p += al1k((size_t)std::max<int64_t>(T, 1) * d * 4);
+  __half *H = reinterpret_cast<__half *>(p);
+  p += al1k((size_t)std::max<int64_t>(T, 1) * d * 2);
   float2 *st1 = reinterpret_cast<float2 *>(p);
   p += al1k((size_t)std::max<int64_t>(T, 1) * nt * 8);
   __half *O = reinterpret_cast<__half *>(p);

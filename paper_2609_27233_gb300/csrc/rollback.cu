@@ -26,6 +26,7 @@ constexpr int64_t kNoWrite = INT64_MIN;
 
 struct MoveArgs {
   uint16_t *pool;
+  int32_t n_lanes;
   int32_t n_layers, n_pages, n_kv_heads, head_dim;
   int32_t heads_per_unit, n_head_groups;
   int32_t *block_table;
@@ -83,14 +84,71 @@ __device__ __forceinline__ void cp_async_wait() {
 }
 
 constexpr int kRing = 3;   // units in flight per CTA
+constexpr int kMeta = kRing + 2;
+
+struct PageDesc {
+  int64_t *src;    // [pages][16] source row offset within a layer (no head offset), -(i+1) for span i, kNoWrite
+  int2 *dep;       // [pages] range of compacted pages that read this old page
+};
+
+// One warp per (sequence, compacted page): where each of its 16 entries comes
+// from, and which compacted pages read the same page of the old layout.
+__global__ void __launch_bounds__(256) rollback_map_kernel(MoveArgs a, PlanArrays arr, PageDesc pd, int D) {
+  if (arr.hdr->skip) return;
+  const int b = blockIdx.y;
+  const int k = blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  const int nd = arr.n_dest[b];
+  if (k >= nd) return;
+  const int p = arr.first_page[b] + k;
+  const int idx = arr.unit_base[b] / a.n_lanes + k;
+  const int lo = a.span_offsets[b], hi = a.span_offsets[b + 1];
+  const int32_t *bt = a.block_table + (int64_t)b * a.max_pages;
+  const int64_t page_stride = (int64_t)kPageSize * D * a.n_kv_heads * 2;
+  int dpage = -1;
+  if (lane < kPageSize) {
+    const int L = arr.seq_Lp[b];
+    const int j = p * kPageSize + lane;
+    int64_t src = kNoWrite;
+    if (j < L && j >= a.span_start[lo]) {
+      const int i = upper_index(arr.new_idx, lo, hi, j);
+      if (i >= lo) {
+        if (arr.new_idx[i] == j) {
+          src = -(int64_t)i - 1;
+        } else {
+          const int t = j + arr.r_incl[i];
+          if (t != j) src = (int64_t)bt[t / kPageSize] * page_stride + (t % kPageSize) * D;
+        }
+      }
+    }
+    pd.src[(int64_t)idx * kPageSize + lane] = src;
+  } else {
+    const int L = arr.seq_L[b];
+    const int t = p * kPageSize + (lane - kPageSize);
+    if (t < L) {
+      const int i = upper_index(a.span_start, lo, hi, t);
+      if (i >= lo && t >= a.span_start[i] + a.span_len[i]) {
+        const int r = arr.r_incl[i];
+        if (r > 0) dpage = (t - r) / kPageSize;
+      }
+    }
+  }
+  int mn = dpage < 0 ? 0x7fffffff : dpage, mx = dpage;
+#pragma unroll
+  for (int o = 8; o >= 1; o >>= 1) {
+    mn = min(mn, __shfl_xor_sync(0xffffffffu, mn, o));
+    mx = max(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+  }
+  if (lane == kPageSize) pd.dep[idx] = make_int2(mn, mx);
+}
 
 struct UnitMeta {
-  int unit, b, lane, p, nh, h0, dep_lo, dep_hi;
-  int64_t src[kPageSize];   // source row offset (kv 0, head h0), -(i+1) for surrogate i, or kNoWrite
+  int unit, b, layer, p, nh, h0, dep_lo, dep_hi;
+  int64_t src[kPageSize];
 };
 
 template <int D>
-__global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a, PlanArrays arr) {
+__global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a, PlanArrays arr, PageDesc pd) {
   constexpr int CPR = D / 8;                                   // 16-byte chunks per (kv, head) row
   constexpr int NH = kUnitBytes / (2 * kPageSize * D * 2);     // KV heads per unit
   constexpr int CHUNKS = 2 * NH * kPageSize * CPR;
@@ -98,15 +156,15 @@ __global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a,
   // Chunk c = tid + it * 256 of a unit is 16-byte column c % CPR of row
   // c / CPR = ((kv * NH + h) * 16 + slot).  256 is a multiple of 16 * CPR, so
   // a thread's column and slot are the same for every it; only (kv, h) vary.
-  const int tid = threadIdx.x, lane_id = tid & 31;
+  const int tid = threadIdx.x, lane_id = tid & 31, warp = tid >> 5;
   const int my_col = tid % CPR;
   const int my_slot = (tid / CPR) % kPageSize;
   const int my_kvh0 = tid / (CPR * kPageSize);
   constexpr int KVH_STEP = kMoveThreads / (CPR * kPageSize);
 
   extern __shared__ __align__(16) uint8_t ring[];              // kRing x 32 KB of unit data
-  __shared__ UnitMeta meta[kRing + 1];
-  __shared__ int s_last, s_abort;
+  __shared__ UnitMeta meta[kMeta];
+  __shared__ int s_last, s_abort, s_done;
 
   const PlanHeader *hdr = arr.hdr;
   const int total = hdr->total_units;
@@ -114,12 +172,11 @@ __global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a,
   const int Hkv = a.n_kv_heads;
   const int64_t head_stride = (int64_t)kPageSize * D;
   const int64_t kv_stride = head_stride * Hkv;
-  const int64_t page_stride = kv_stride * 2;
-  const int64_t layer_stride = page_stride * a.n_pages;
+  const int64_t layer_stride = kv_stride * 2 * a.n_pages;
 
-  // warp 0: take the next ticket and describe the unit in meta[m]
+  // warp 1: take the next ticket and copy that unit's precomputed description
   auto describe = [&](int m) {
-    int u = 0, b = 0, ln = 0, p = 0;
+    int u = 0, b = 0, ln = 0, k = 0;
     if (lane_id == 0) {
       u = atomicAdd(&arr.hdr->ticket, 1);
       if (u < total) {
@@ -127,7 +184,7 @@ __global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a,
         const int rem = u - arr.unit_base[b];
         const int nd = arr.n_dest[b];
         ln = rem / nd;
-        p = arr.first_page[b] + rem % nd;
+        k = rem % nd;
       }
     }
     u = __shfl_sync(0xffffffffu, u, 0);
@@ -138,61 +195,20 @@ __global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a,
     }
     b = __shfl_sync(0xffffffffu, b, 0);
     ln = __shfl_sync(0xffffffffu, ln, 0);
-    p = __shfl_sync(0xffffffffu, p, 0);
-    const int layer = ln / a.n_head_groups;
-    const int h0 = (ln % a.n_head_groups) * NH;
-    const int lo = a.span_offsets[b], hi = a.span_offsets[b + 1];
-    const int32_t *bt = a.block_table + (int64_t)b * a.max_pages;
-    if (lane_id < kPageSize) {
-      // source of compacted entry j
-      const int L = arr.seq_Lp[b];
-      const int j = p * kPageSize + lane_id;
-      int64_t src = kNoWrite;
-      if (j < L && j >= a.span_start[lo]) {
-        const int i = upper_index(arr.new_idx, lo, hi, j);
-        if (i >= lo) {
-          if (arr.new_idx[i] == j) {
-            src = -(int64_t)i - 1;
-          } else {
-            const int t = j + arr.r_incl[i];
-            if (t != j)
-              src = layer * layer_stride + h0 * head_stride + (int64_t)bt[t / kPageSize] * page_stride +
-                    (t % kPageSize) * D;
-          }
-        }
-      }
-      M.src[lane_id] = src;
-    }
-    // which compacted pages read old page p: kept entries t of page p that move
-    int dpage = -1;
-    if (lane_id >= 16) {
-      const int L = arr.seq_L[b];
-      const int t = p * kPageSize + (lane_id - 16);
-      if (t < L) {
-        const int i = upper_index(a.span_start, lo, hi, t);
-        if (i >= lo && t >= a.span_start[i] + a.span_len[i]) {
-          const int r = arr.r_incl[i];
-          if (r > 0) dpage = (t - r) / kPageSize;
-        }
-      }
-    }
-    int mn = dpage < 0 ? 0x7fffffff : dpage, mx = dpage;
-#pragma unroll
-    for (int o = 8; o >= 1; o >>= 1) {
-      mn = min(mn, __shfl_xor_sync(0xffffffffu, mn, o));
-      mx = max(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-    }
-    mn = __shfl_sync(0xffffffffu, mn, 16);
-    mx = __shfl_sync(0xffffffffu, mx, 16);
+    k = __shfl_sync(0xffffffffu, k, 0);
+    const int idx = arr.unit_base[b] / a.n_lanes + k;
+    if (lane_id < kPageSize) M.src[lane_id] = pd.src[(int64_t)idx * kPageSize + lane_id];
     if (lane_id == 0) {
+      const int2 dep = pd.dep[idx];
+      const int h0 = (ln % a.n_head_groups) * NH;
       M.unit = u;
       M.b = b;
-      M.lane = layer;
-      M.p = p;
+      M.layer = ln / a.n_head_groups;
+      M.p = arr.first_page[b] + k;
       M.h0 = h0;
       M.nh = min(NH, Hkv - h0);
-      M.dep_lo = mn;
-      M.dep_hi = mx;
+      M.dep_lo = dep.x;
+      M.dep_hi = dep.y;
     }
   };
 
@@ -202,6 +218,7 @@ __global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a,
     if (M.unit < total) {
       const int64_t src = M.src[my_slot];
       uint8_t *dst = ring + st * kUnitBytes;
+      const int64_t base = M.layer * layer_stride + M.h0 * head_stride + my_col * 8;
 #pragma unroll
       for (int it = 0; it < kChunksPerThread; ++it) {
         const int kvh = my_kvh0 + it * KVH_STEP;
@@ -209,10 +226,10 @@ __global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a,
         if (h < M.nh && src != kNoWrite) {
           const uint16_t *g;
           if (src >= 0) {
-            g = a.pool + src + kv * kv_stride + h * head_stride + my_col * 8;
+            g = a.pool + base + src + kv * kv_stride + h * head_stride;
           } else {
             const int64_t i = -src - 1;
-            g = (kv ? a.sur_v : a.sur_k) + ((i * a.n_layers + M.lane) * Hkv + M.h0 + h) * D + my_col * 8;
+            g = (kv ? a.sur_v : a.sur_k) + ((i * a.n_layers + M.layer) * Hkv + M.h0 + h) * D + my_col * 8;
           }
           cp_async_16(dst + (tid + it * kMoveThreads) * 16, g);
         }
@@ -222,53 +239,54 @@ __global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a,
   };
 
   if (tid == 0) s_abort = 0;
-  // prologue: kRing - 1 units in flight
-  int head = 0;   // units described so far by this CTA
+  // prologue: units 0 .. kRing-2 in flight, unit kRing-1 described
+  if (warp == 1) describe(0);
+  __syncthreads();
   for (int k = 0; k < kRing - 1; ++k) {
-    if (tid < 32) describe(head % (kRing + 1));
+    issue(k % kMeta, k % kRing);
+    if (warp == 1) describe((k + 1) % kMeta);
     __syncthreads();
-    issue(head % (kRing + 1), head % kRing);
-    ++head;
   }
   for (int cur = 0;; ++cur) {
-    // describe and start one more unit, then wait for the oldest one's copies
-    if (tid < 32) describe(head % (kRing + 1));
+    const int head = cur + kRing - 1;
+    issue(head % kMeta, head % kRing);
+    cp_async_wait<kRing - 1>();          // this thread's copies of unit `cur` have landed
     __syncthreads();
-    issue(head % (kRing + 1), head % kRing);
-    ++head;
-    cp_async_wait<kRing - 1>();
-    __syncthreads();
-    const UnitMeta &M = meta[cur % (kRing + 1)];
-    const int u = M.unit;
-    if (u >= total) break;     // tickets are taken in order: nothing younger exists either
-    const int p = M.p;
+    const UnitMeta &M = meta[cur % kMeta];
     if (tid == 0) {
-      // release: every copy of this unit has landed (wait_group + barrier)
-      st_release(&arr.flags[u], epoch);
-      // wait for the units that read old page p (all hold smaller tickets)
-      for (int q = M.dep_lo; q <= M.dep_hi && q >= 0 && q < p; ++q) {
-        const int uq = u - (p - q);
-        if (ld_acquire(&arr.flags[uq]) == epoch) continue;
-        const uint64_t t0 = globaltimer();
-        bool ok = false;
-        while (!ok) {
+      const int u = M.unit;
+      s_done = u >= total;    // tickets are taken in order: nothing younger is valid either
+      if (u < total) {
+        const int p = M.p;
+        // release: every copy of this unit has landed (wait_group + barrier)
+        st_release(&arr.flags[u], epoch);
+        // wait for the units that read old page p (all hold smaller tickets)
+        for (int q = M.dep_lo; q <= M.dep_hi && q >= 0 && q < p; ++q) {
+          const int uq = u - (p - q);
+          if (ld_acquire(&arr.flags[uq]) == epoch) continue;
+          const uint64_t t0 = globaltimer();
+          bool ok = false;
+          while (!ok) {
 #pragma unroll 1
-          for (int i = 0; i < 64 && !ok; ++i) ok = (ld_acquire(&arr.flags[uq]) == epoch);
-          if (!ok && globaltimer() - t0 > kWaitLimitNs) break;
-        }
-        if (!ok) {
-          set_error(a.status, UMIM_ERR_TIMEOUT);
-          s_abort = 1;
-          break;
+            for (int i = 0; i < 64 && !ok; ++i) ok = (ld_acquire(&arr.flags[uq]) == epoch);
+            if (!ok && globaltimer() - t0 > kWaitLimitNs) break;
+          }
+          if (!ok) {
+            set_error(a.status, UMIM_ERR_TIMEOUT);
+            s_abort = 1;
+            break;
+          }
         }
       }
     }
+    if (warp == 1) describe((head + 1) % kMeta);
     __syncthreads();
+    if (s_done) break;
     const int64_t src = M.src[my_slot];
     if (!s_abort && src != kNoWrite) {
       const int32_t *bt = a.block_table + (int64_t)M.b * a.max_pages;
-      const int64_t dst = M.lane * layer_stride + M.h0 * head_stride + (int64_t)bt[p] * page_stride +
-                          my_slot * D + my_col * 8;
+      const int64_t dst = M.layer * layer_stride + M.h0 * head_stride +
+                          (int64_t)bt[M.p] * (kv_stride * 2) + my_slot * D + my_col * 8;
       const uint8_t *stage = ring + (cur % kRing) * kUnitBytes;
 #pragma unroll
       for (int it = 0; it < kChunksPerThread; ++it) {
@@ -280,6 +298,7 @@ __global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a,
         }
       }
     }
+    __syncthreads();   // stage cur % kRing is refilled by the next issue
   }
   cp_async_wait<0>();
 
@@ -317,7 +336,9 @@ size_t kv_rollback_workspace_bytes(int B, int S, int max_pages, int n_layers, in
   const int hpu = std::max(1, kUnitBytes / (2 * kPageSize * head_dim * 2));
   const int groups = (n_kv_heads + hpu - 1) / hpu;
   const size_t units = (size_t)B * n_layers * groups * (size_t)max_pages;
-  return plan_bytes(B, S) + align256(sizeof(int32_t) * (units > 0 ? units : 1));
+  const size_t pages = (size_t)B * max_pages;
+  return plan_bytes(B, S) + align256(sizeof(int32_t) * (units > 0 ? units : 1)) +
+         align256(sizeof(int64_t) * kPageSize * (pages > 0 ? pages : 1)) + align256(sizeof(int2) * (pages > 0 ? pages : 1));
 }
 
 umim_status kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t max_pages, int32_t *seq_lens,
@@ -330,6 +351,13 @@ umim_status kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t m
   const int groups = (kv->n_kv_heads + hp - 1) / hp;
   PlanArrays arr = plan_carve(ws, B, S);
   int32_t *status = dev_status ? dev_status : &arr.hdr->status;
+  const size_t units = (size_t)B * kv->n_layers * groups * (size_t)max_pages;
+  const size_t pages = (size_t)B * max_pages;
+  PageDesc pd;
+  pd.src = reinterpret_cast<int64_t *>(reinterpret_cast<char *>(arr.flags) +
+                                       align256(sizeof(int32_t) * (units > 0 ? units : 1)));
+  pd.dep = reinterpret_cast<int2 *>(reinterpret_cast<char *>(pd.src) +
+                                    align256(sizeof(int64_t) * kPageSize * (pages > 0 ? pages : 1)));
 
   PlanArgs pa{};
   pa.seq_lens = seq_lens;
@@ -351,6 +379,7 @@ umim_status kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t m
 
   MoveArgs ma{};
   ma.pool = static_cast<uint16_t *>(kv->base);
+  ma.n_lanes = kv->n_layers * groups;
   ma.n_layers = kv->n_layers;
   ma.n_pages = kv->n_pages;
   ma.n_kv_heads = kv->n_kv_heads;
@@ -377,8 +406,11 @@ umim_status kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t m
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kMoveThreads, smem) != cudaSuccess || per_sm < 1)
     per_sm = 1;
   const int grid = std::max(1, num_sms) * per_sm;
+  trace_mark(stream, "rollback.map");
+  rollback_map_kernel<<<dim3((unsigned)std::max(1, ceil_div(max_pages, 8)), (unsigned)B), 256, 0, stream>>>(ma, arr,
+                                                                                                         pd, D);
   trace_mark(stream, "rollback.move");
-  kern<<<grid, kMoveThreads, smem, stream>>>(ma, arr);
+  kern<<<grid, kMoveThreads, smem, stream>>>(ma, arr, pd);
   trace_mark(stream, nullptr);
   return cudaGetLastError() == cudaSuccess ? UMIM_OK : UMIM_ERR_CUDA;
 }
