@@ -272,124 +272,150 @@ __device__ __forceinline__ float2 row_moments_warp(const float2 *st, int ntiles,
 }
 
 // ---------------------------------------------------------------------------
-// LN_kv + attention pooling with the learnable queries, one block per span,
-// d/16 threads with 16 contiguous columns each, H read once.  o is written
-// in fp16 (11 significant bits) as the A operand of the output projection.
+// LN_kv + attention pooling with the learnable queries, one warp per span.
+// Lane l owns columns [256 k + 8 l, 256 k + 8 l + 8) of column chunk k.
+// Pass 1 accumulates the scores <P_j[head], q_head>; pass 2 re-reads the
+// span's H rows (now in L2) and forms o = sum_j alpha_j P_j, written in fp16
+// (11 significant bits) as the A operand of the output projection.
 // ---------------------------------------------------------------------------
-constexpr int kColsPerThread = 16;
+constexpr int kPoolWarps = 8;
 
-__global__ void __launch_bounds__(512)
+__global__ void __launch_bounds__(kPoolWarps * 32)
     pool_kernel(const __half *H, const float2 *stats, const int32_t *offs, int S, int64_t T, int d, int h,
                 const __nv_bfloat16 *gamma, const __nv_bfloat16 *beta, const __nv_bfloat16 *query, float eps,
                 __half *O, int32_t *status) {
-  const int s = blockIdx.x;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int ntiles = d / BN;
-  const int c0 = tid * kColsPerThread;
-  const int dh = d / h;
-  const int head = c0 / dh;
-  const int tph = dh / kColsPerThread;             // threads per head
-  const int low_bit = tph & (-tph);
-  const int seg = low_bit < 32 ? low_bit : 32;     // largest power of two dividing tph, at most 32
-  __shared__ float2 s_mom[UMIM_MAX_SPAN_TOKENS];
-  __shared__ float s_red[UMIM_MAX_SPAN_TOKENS][512 / 4];
-  __shared__ float s_alpha[UMIM_MAX_SPAN_TOKENS][8];
-
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int s = blockIdx.x * kPoolWarps + warp;
+  __shared__ float s_sc[kPoolWarps][UMIM_MAX_SPAN_TOKENS][8];
+  __shared__ float s_al[kPoolWarps][UMIM_MAX_SPAN_TOKENS][8];
+  if (s >= S) return;
   const int t0 = offs[s], t1 = offs[s + 1];
   int n = t1 - t0;
   if (t0 < 0 || n < 1 || n > UMIM_MAX_SPAN_TOKENS || t1 > T) {
-    if (tid == 0) set_error(status, UMIM_ERR_INVALID_ARG);
+    if (lane == 0) set_error(status, UMIM_ERR_INVALID_ARG);
     n = 0;
   }
-  for (int j = warp; j < n; j += (int)(blockDim.x >> 5)) {
-    const float2 m = row_moments_warp(stats + (int64_t)(t0 + j) * ntiles, ntiles, d, eps);
-    if (lane == 0) s_mom[j] = m;
-  }
-  float g[kColsPerThread], bta[kColsPerThread], q[kColsPerThread];
-  {
-    const uint4 *gp = reinterpret_cast<const uint4 *>(gamma + c0);
-    const uint4 *bp = reinterpret_cast<const uint4 *>(beta + c0);
-    const uint4 *qp = reinterpret_cast<const uint4 *>(query + c0);   // query is [h][dh] = d contiguous values
-    bf16x8_to_float(gp[0], g);
-    bf16x8_to_float(gp[1], g + 8);
-    bf16x8_to_float(bp[0], bta);
-    bf16x8_to_float(bp[1], bta + 8);
-    bf16x8_to_float(qp[0], q);
-    bf16x8_to_float(qp[1], q + 8);
-  }
-  float P[UMIM_MAX_SPAN_TOKENS][kColsPerThread];
+  const int ntiles = d / BN;
+  const int dh = d / h;
+  // lanes per segment: a power of two dividing dh / 8, so no segment straddles a head
+  const int q8 = dh / 8;
+  const int seg = min(32, q8 & (-q8));
+  float mu[UMIM_MAX_SPAN_TOKENS], rs[UMIM_MAX_SPAN_TOKENS];
 #pragma unroll
   for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
+    mu[j] = 0.f;
+    rs[j] = 0.f;
     if (j < n) {
-      const uint4 *hr = reinterpret_cast<const uint4 *>(H + (int64_t)(t0 + j) * d + c0);
+      const float2 m = row_moments_warp(stats + (int64_t)(t0 + j) * ntiles, ntiles, d, eps);
+      mu[j] = m.x;
+      rs[j] = m.y;
+    }
+  }
+  for (int i = lane; i < UMIM_MAX_SPAN_TOKENS * 8; i += 32) s_sc[warp][i / 8][i % 8] = 0.f;
+  __syncwarp();
+  const __half *Hs = H + (int64_t)t0 * d;
+  // pass 1: scores
+#pragma unroll 2
+  for (int c = lane * 8; c < d; c += 256) {
+    const int head = c / dh;
+    float g[8], b[8], q[8];
+    bf16x8_to_float(*reinterpret_cast<const uint4 *>(gamma + c), g);
+    bf16x8_to_float(*reinterpret_cast<const uint4 *>(beta + c), b);
+    bf16x8_to_float(*reinterpret_cast<const uint4 *>(query + c), q);   // query [h][dh] is d contiguous values
 #pragma unroll
-      for (int e = 0; e < 2; ++e) {
-        const uint4 x = hr[e];
+    for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
+      if (j < n) {
+        const uint4 x = *reinterpret_cast<const uint4 *>(Hs + (int64_t)j * d + c);
         const __half2 *h2 = reinterpret_cast<const __half2 *>(&x);
+        float part = 0.f;
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          const float2 f = __half22float2(h2[k]);
-          P[j][8 * e + 2 * k] = f.x;
-          P[j][8 * e + 2 * k + 1] = f.y;
+        for (int e = 0; e < 4; ++e) {
+          const float2 f = __half22float2(h2[e]);
+          part += ((f.x - mu[j]) * rs[j] * g[2 * e] + b[2 * e]) * q[2 * e];
+          part += ((f.y - mu[j]) * rs[j] * g[2 * e + 1] + b[2 * e + 1]) * q[2 * e + 1];
         }
+        for (int o = seg >> 1; o >= 1; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o, seg);
+        if ((lane & (seg - 1)) == 0) atomicAdd(&s_sc[warp][j][head], part);
       }
     }
   }
-  __syncthreads();
-  // P = LN_kv(H) and the partial score of this thread's columns
-#pragma unroll
-  for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
-    float part = 0.f;
-    if (j < n) {
-      const float2 mom = s_mom[j];
-#pragma unroll
-      for (int e = 0; e < kColsPerThread; ++e) {
-        P[j][e] = (P[j][e] - mom.x) * mom.y * g[e] + bta[e];
-        part += P[j][e] * q[e];
-      }
-    }
-    for (int o = seg >> 1; o >= 1; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o, seg);
-    if ((tid & (seg - 1)) == 0) s_red[j][tid / seg] = part;
-  }
-  __syncthreads();
-  // softmax over the span for each head
-  if (tid < h && n > 0) {
-    const int per = tph / seg;
+  __syncwarp();
+  // softmax over the span, one lane per head
+  if (lane < h && n > 0) {
+    const float inv = rsqrtf((float)dh);
     float sc[UMIM_MAX_SPAN_TOKENS];
     float mx = -INFINITY;
-    const float inv = rsqrtf((float)dh);
-    for (int j = 0; j < n; ++j) {
-      float v = 0.f;
-      for (int k = 0; k < per; ++k) v += s_red[j][tid * per + k];
-      sc[j] = v * inv;
+#pragma unroll
+    for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
+      sc[j] = j < n ? s_sc[warp][j][lane] * inv : -INFINITY;
       mx = fmaxf(mx, sc[j]);
     }
     float den = 0.f;
-    for (int j = 0; j < n; ++j) {
-      sc[j] = expf(sc[j] - mx);
+#pragma unroll
+    for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
+      sc[j] = j < n ? expf(sc[j] - mx) : 0.f;
       den += sc[j];
     }
-    for (int j = 0; j < n; ++j) s_alpha[j][tid] = sc[j] / den;
+#pragma unroll
+    for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) s_al[warp][j][lane] = sc[j] / den;
   }
-  __syncthreads();
-  float o[kColsPerThread];
+  __syncwarp();
+  // pass 2: o = sum_j alpha_j P_j
+  __half *Os = O + (int64_t)s * d;
+#pragma unroll 2
+  for (int c = lane * 8; c < d; c += 256) {
+    const int head = c / dh;
+    float g[8], b[8], o[8];
+    bf16x8_to_float(*reinterpret_cast<const uint4 *>(gamma + c), g);
+    bf16x8_to_float(*reinterpret_cast<const uint4 *>(beta + c), b);
 #pragma unroll
-  for (int e = 0; e < kColsPerThread; ++e) o[e] = 0.f;
+    for (int e = 0; e < 8; ++e) o[e] = 0.f;
 #pragma unroll
-  for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
-    if (j < n) {
-      const float a = s_alpha[j][head];
+    for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
+      if (j < n) {
+        const float al = s_al[warp][j][head];
+        const uint4 x = *reinterpret_cast<const uint4 *>(Hs + (int64_t)j * d + c);
+        const __half2 *h2 = reinterpret_cast<const __half2 *>(&x);
 #pragma unroll
-      for (int e = 0; e < kColsPerThread; ++e) o[e] += a * P[j][e];
+        for (int e = 0; e < 4; ++e) {
+          const float2 f = __half22float2(h2[e]);
+          o[2 * e] += al * ((f.x - mu[j]) * rs[j] * g[2 * e] + b[2 * e]);
+          o[2 * e + 1] += al * ((f.y - mu[j]) * rs[j] * g[2 * e + 1] + b[2 * e + 1]);
+        }
+      }
     }
-  }
-  uint4 packed[2];
-  __half2 *hp = reinterpret_cast<__half2 *>(packed);
+    uint4 packed;
+    __half2 *hp = reinterpret_cast<__half2 *>(&packed);
 #pragma unroll
-  for (int e = 0; e < kColsPerThread / 2; ++e) hp[e] = __floats2half2_rn(o[2 * e], o[2 * e + 1]);
-  uint4 *dst = reinterpret_cast<uint4 *>(O + (int64_t)s * d + c0);
-  dst[0] = packed[0];
-  dst[1] = packed[1];
+    for (int e = 0; e < 4; ++e) hp[e] = __floats2half2_rn(o[2 * e], o[2 * e + 1]);
+    *reinterpret_cast<uint4 *>(Os + c) = packed;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// LN_o in place over rows of Z, one warp per row
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256)
+    ln_rows_kernel(float *Z, const float2 *stats, int S, int d, const __nv_bfloat16 *gamma,
+                   const __nv_bfloat16 *beta, float eps) {
+  const int r = blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (r >= S) return;
+  const float2 m = row_moments_warp(stats + (int64_t)r * (d / BN), d / BN, d, eps);
+  float *row = Z + (int64_t)r * d;
+#pragma unroll 4
+  for (int c = lane * 4; c < d; c += 128) {
+    float4 x = *reinterpret_cast<float4 *>(row + c);
+    const __nv_bfloat162 *g2 = reinterpret_cast<const __nv_bfloat162 *>(gamma + c);
+    const __nv_bfloat162 *b2 = reinterpret_cast<const __nv_bfloat162 *>(beta + c);
+    const float2 g0 = __bfloat1622float2(g2[0]), g1 = __bfloat1622float2(g2[1]);
+    const float2 b0 = __bfloat1622float2(b2[0]), b1 = __bfloat1622float2(b2[1]);
+    x.x = (x.x - m.x) * m.y * g0.x + b0.x;
+    x.y = (x.y - m.x) * m.y * g0.y + b0.y;
+    x.z = (x.z - m.x) * m.y * g1.x + b1.x;
+    x.w = (x.w - m.x) * m.y * g1.y + b1.y;
+    *reinterpret_cast<float4 *>(row + c) = x;
+  }
 }
 
 // W_o from bf16 to fp16 (exact for values in fp16's normal range)
@@ -403,40 +429,6 @@ __global__ void bf16_to_f16_kernel(const uint4 *in, uint4 *out, int64_t n_vec) {
 #pragma unroll
     for (int e = 0; e < 4; ++e) h[e] = __floats2half2_rn(f[2 * e], f[2 * e + 1]);
     out[i] = o;
-  }
-}
-
-// ---------------------------------------------------------------------------
-// LN_o in place over rows of Z, d/16 threads per row
-// ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(512)
-    ln_rows_kernel(float *Z, const float2 *stats, int d, const __nv_bfloat16 *gamma, const __nv_bfloat16 *beta,
-                   float eps) {
-  const int r = blockIdx.x;
-  __shared__ float2 s_m;
-  if (threadIdx.x < 32) {
-    const float2 m = row_moments_warp(stats + (int64_t)r * (d / BN), d / BN, d, eps);
-    if (threadIdx.x == 0) s_m = m;
-  }
-  const int c0 = threadIdx.x * kColsPerThread;
-  float g[kColsPerThread], b[kColsPerThread];
-  bf16x8_to_float(reinterpret_cast<const uint4 *>(gamma + c0)[0], g);
-  bf16x8_to_float(reinterpret_cast<const uint4 *>(gamma + c0)[1], g + 8);
-  bf16x8_to_float(reinterpret_cast<const uint4 *>(beta + c0)[0], b);
-  bf16x8_to_float(reinterpret_cast<const uint4 *>(beta + c0)[1], b + 8);
-  float4 *row = reinterpret_cast<float4 *>(Z + (int64_t)r * d + c0);
-  float4 x[4];
-#pragma unroll
-  for (int e = 0; e < 4; ++e) x[e] = row[e];
-  __syncthreads();
-  const float2 m = s_m;
-#pragma unroll
-  for (int e = 0; e < 4; ++e) {
-    x[e].x = (x[e].x - m.x) * m.y * g[4 * e] + b[4 * e];
-    x[e].y = (x[e].y - m.x) * m.y * g[4 * e + 1] + b[4 * e + 1];
-    x[e].z = (x[e].z - m.x) * m.y * g[4 * e + 2] + b[4 * e + 2];
-    x[e].w = (x[e].w - m.x) * m.y * g[4 * e + 3] + b[4 * e + 3];
-    row[e] = x[e];
   }
 }
 
@@ -534,7 +526,7 @@ umim_status merge_spans(const void *embeddings, int64_t vocab, const int32_t *to
     if (r != UMIM_OK) return r;
   }
   trace_mark(st, "merge.pool");
-  pool_kernel<<<S, d / kColsPerThread, 0, st>>>(H, st1, span_offsets, S, T, d, w->n_heads,
+  pool_kernel<<<(S + kPoolWarps - 1) / kPoolWarps, kPoolWarps * 32, 0, st>>>(H, st1, span_offsets, S, T, d, w->n_heads,
                                           static_cast<const __nv_bfloat16 *>(w->ln_kv_gamma),
                                           static_cast<const __nv_bfloat16 *>(w->ln_kv_beta),
                                           static_cast<const __nv_bfloat16 *>(w->query), w->ln_eps, O, status);
@@ -544,7 +536,7 @@ umim_status merge_spans(const void *embeddings, int64_t vocab, const int32_t *to
   umim_status r = launch_gemm(enc, O, S, Wo16, d, true, w->b_o, surrogates, st2, status, st, "merge.gemm2", num_sms);
   if (r != UMIM_OK) return r;
   trace_mark(st, "merge.ln_o");
-  ln_rows_kernel<<<S, d / kColsPerThread, 0, st>>>(surrogates, st2, d, static_cast<const __nv_bfloat16 *>(w->ln_o_gamma),
+  ln_rows_kernel<<<(S + 7) / 8, 256, 0, st>>>(surrogates, st2, S, d, static_cast<const __nv_bfloat16 *>(w->ln_o_gamma),
                                     static_cast<const __nv_bfloat16 *>(w->ln_o_beta), w->ln_eps);
   trace_mark(st, nullptr);
   return cudaGetLastError() == cudaSuccess ? UMIM_OK : UMIM_ERR_CUDA;

@@ -4,14 +4,16 @@
 //
 // Work unit = (sequence b, lane = layer x head group, compacted page p): the
 // 16 compacted entries j in [16p, 16p+16) of one layer and a group of KV
-// heads.  A unit reads its sources (kept entries t = j + r >= j, or the
-// surrogate rows) into registers, publishes "read done", waits until every
-// unit that reads old page p has published, then writes page p.  Because
-// j <= t, the units that read old page p are unit p itself and lower pages
-// of the same (b, lane); tickets are taken in unit order, so a unit only
-// waits for units that already hold a ticket and publish without waiting:
-// no deadlock, no second pass, each moved byte is read once and written
-// once.  Every wait is bounded (UMIM_ERR_TIMEOUT).
+// heads.  A unit copies its sources (kept entries t = j + r >= j, or the
+// surrogate rows) into shared memory, publishes "read done", waits until
+// every unit that reads old page p has published, then writes page p.
+// Because j <= t, the units that read old page p are unit p itself and lower
+// pages of the same (b, lane), i.e. smaller unit indices.  The launch is
+// cooperative (every CTA resident) and CTA c handles units c, c + grid,
+// c + 2 grid, ... in increasing order, publishing each as soon as its copies
+// land, so the smallest unpublished unit always makes progress: no deadlock,
+// no second pass, each moved byte read once and written once.  Every wait is
+// bounded (UMIM_ERR_TIMEOUT).
 #include <algorithm>
 
 #include "plan.cuh"
@@ -174,11 +176,13 @@ __global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a,
   const int64_t kv_stride = head_stride * Hkv;
   const int64_t layer_stride = kv_stride * 2 * a.n_pages;
 
-  // warp 1: take the next ticket and copy that unit's precomputed description
+  // warp 1: describe this CTA's next unit (units blockIdx.x, blockIdx.x +
+  // gridDim.x, ... in increasing order) from its precomputed description
+  int next_unit = blockIdx.x;
   auto describe = [&](int m) {
     int u = 0, b = 0, ln = 0, k = 0;
     if (lane_id == 0) {
-      u = atomicAdd(&arr.hdr->ticket, 1);
+      u = next_unit;
       if (u < total) {
         b = find_seq(arr.unit_base, a.B, u);
         const int rem = u - arr.unit_base[b];
@@ -187,6 +191,7 @@ __global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a,
         k = rem % nd;
       }
     }
+    next_unit += gridDim.x;
     u = __shfl_sync(0xffffffffu, u, 0);
     UnitMeta &M = meta[m];
     if (u >= total) {
@@ -255,12 +260,12 @@ __global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a,
     const UnitMeta &M = meta[cur % kMeta];
     if (tid == 0) {
       const int u = M.unit;
-      s_done = u >= total;    // tickets are taken in order: nothing younger is valid either
+      s_done = u >= total;    // this CTA's units increase: nothing younger is valid either
       if (u < total) {
         const int p = M.p;
         // release: every copy of this unit has landed (wait_group + barrier)
         st_release(&arr.flags[u], epoch);
-        // wait for the units that read old page p (all hold smaller tickets)
+        // wait for the units that read old page p (all have smaller indices)
         for (int q = M.dep_lo; q <= M.dep_hi && q >= 0 && q < p; ++q) {
           const int uq = u - (p - q);
           if (ld_acquire(&arr.flags[uq]) == epoch) continue;
@@ -405,12 +410,15 @@ umim_status kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t m
   int per_sm = 0;
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kMoveThreads, smem) != cudaSuccess || per_sm < 1)
     per_sm = 1;
-  const int grid = std::max(1, num_sms) * per_sm;
+  const int grid = std::max(1, num_sms) * per_sm;   // every CTA resident (cooperative launch)
   trace_mark(stream, "rollback.map");
   rollback_map_kernel<<<dim3((unsigned)std::max(1, ceil_div(max_pages, 8)), (unsigned)B), 256, 0, stream>>>(ma, arr,
                                                                                                          pd, D);
   trace_mark(stream, "rollback.move");
-  kern<<<grid, kMoveThreads, smem, stream>>>(ma, arr, pd);
+  void *args[] = {&ma, &arr, &pd};
+  if (cudaLaunchCooperativeKernel(reinterpret_cast<const void *>(kern), dim3(grid), dim3(kMoveThreads), args,
+                                  (size_t)smem, stream) != cudaSuccess)
+    return UMIM_ERR_CUDA;
   trace_mark(stream, nullptr);
   return cudaGetLastError() == cudaSuccess ? UMIM_OK : UMIM_ERR_CUDA;
 }
