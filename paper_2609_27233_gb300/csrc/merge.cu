@@ -272,123 +272,206 @@ __device__ __forceinline__ float2 row_moments_warp(const float2 *st, int ntiles,
 }
 
 // ---------------------------------------------------------------------------
-// LN_kv + attention pooling with the learnable queries, one warp per span.
-// Lane l owns columns [256 k + 8 l, 256 k + 8 l + 8) of column chunk k.
-// Pass 1 accumulates the scores <P_j[head], q_head>; pass 2 re-reads the
-// span's H rows (now in L2) and forms o = sum_j alpha_j P_j, written in fp16
+// LN_kv + attention pooling with the learnable queries.
+// Persistent CTAs; span s goes to CTA s mod grid.  A producer warp copies each
+// span's H rows (fp16) and row statistics into a 3-stage shared-memory ring
+// with bulk asynchronous copies completing an mbarrier; 8 consumer warps
+// compute from shared memory: P = LN_kv(H), the scores <P_j[head], q_head>,
+// the softmax over the span and o = sum_j alpha_j P_j, written in fp16
 // (11 significant bits) as the A operand of the output projection.
+// 16-byte column chunk cc (columns 8 cc .. 8 cc + 7) belongs to consumer
+// thread cc mod 256.
 // ---------------------------------------------------------------------------
-constexpr int kPoolWarps = 8;
+constexpr int kPoolRing = 3;
+constexpr int kPoolConsumers = 256;
 
-__global__ void __launch_bounds__(kPoolWarps * 32)
+__device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                   smem_u32(dst)),
+               "l"(src), "r"(bytes), "r"(smem_u32(bar))
+               : "memory");
+}
+
+__device__ __forceinline__ void consumer_sync() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
+
+__host__ __device__ inline int pool_stage_bytes(int d) { return (UMIM_MAX_SPAN_TOKENS * (d * 2 + (d / BN) * 8) + 127) & ~127; }
+
+__global__ void __launch_bounds__(kPoolConsumers + 32, 1)
     pool_kernel(const __half *H, const float2 *stats, const int32_t *offs, int S, int64_t T, int d, int h,
                 const __nv_bfloat16 *gamma, const __nv_bfloat16 *beta, const __nv_bfloat16 *query, float eps,
                 __half *O, int32_t *status) {
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int s = blockIdx.x * kPoolWarps + warp;
-  __shared__ float s_sc[kPoolWarps][UMIM_MAX_SPAN_TOKENS][8];
-  __shared__ float s_al[kPoolWarps][UMIM_MAX_SPAN_TOKENS][8];
-  if (s >= S) return;
-  const int t0 = offs[s], t1 = offs[s + 1];
-  int n = t1 - t0;
-  if (t0 < 0 || n < 1 || n > UMIM_MAX_SPAN_TOKENS || t1 > T) {
-    if (lane == 0) set_error(status, UMIM_ERR_INVALID_ARG);
-    n = 0;
-  }
+  extern __shared__ __align__(128) uint8_t pool_smem[];
+  __shared__ uint64_t full[kPoolRing], empty[kPoolRing];
+  __shared__ int s_n[kPoolRing];
+  __shared__ float2 s_mom[UMIM_MAX_SPAN_TOKENS];
+  __shared__ float s_red[UMIM_MAX_SPAN_TOKENS][128];
+  __shared__ float s_al[UMIM_MAX_SPAN_TOKENS][8];
+  __shared__ int s_abort;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int ntiles = d / BN;
+  const int sbytes = pool_stage_bytes(d);
   const int dh = d / h;
-  // lanes per segment: a power of two dividing dh / 8, so no segment straddles a head
   const int q8 = dh / 8;
-  const int seg = min(32, q8 & (-q8));
-  float mu[UMIM_MAX_SPAN_TOKENS], rs[UMIM_MAX_SPAN_TOKENS];
+  const int seg = min(32, q8 & (-q8));   // lanes per segment: never straddles a head
+  const int seg_per_head = q8 / seg;
+
+  if (tid == 0) {
+    for (int i = 0; i < kPoolRing; ++i) {
+      mbar_init(&full[i], 1);
+      mbar_init(&empty[i], kPoolConsumers / 32);
+    }
+    s_abort = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+
+  if (warp == kPoolConsumers / 32) {
+    // ---- producer ----
+    if (lane == 0) {
+      int k = 0;
+      for (int s = blockIdx.x; s < S; s += gridDim.x, ++k) {
+        const int st = k % kPoolRing;
+        if (!mbar_wait(&empty[st], ((k / kPoolRing) & 1) ^ 1)) {
+          set_error(status, UMIM_ERR_TIMEOUT);
+          break;
+        }
+        const int t0 = offs[s], t1 = offs[s + 1];
+        int n = t1 - t0;
+        if (t0 < 0 || n < 1 || n > UMIM_MAX_SPAN_TOKENS || t1 > T) {
+          set_error(status, UMIM_ERR_INVALID_ARG);
+          n = 0;
+        }
+        s_n[st] = n;
+        uint8_t *sh = pool_smem + st * sbytes;
+        uint8_t *ss = sh + UMIM_MAX_SPAN_TOKENS * d * 2;
+        if (n > 0) {
+          mbar_arrive_expect_tx(&full[st], n * (d * 2 + ntiles * 8));
+          for (int j = 0; j < n; ++j) {
+            bulk_g2s(sh + j * d * 2, H + (int64_t)(t0 + j) * d, d * 2, &full[st]);
+            bulk_g2s(ss + j * ntiles * 8, stats + (int64_t)(t0 + j) * ntiles, ntiles * 8, &full[st]);
+          }
+        } else {
+          mbar_arrive(&full[st]);
+        }
+      }
+    }
+    return;
+  }
+
+  // ---- consumers ----
+  int k = 0;
+  for (int s = blockIdx.x; s < S; s += gridDim.x, ++k) {
+    const int st = k % kPoolRing;
+    if (!mbar_wait(&full[st], (k / kPoolRing) & 1)) {
+      set_error(status, UMIM_ERR_TIMEOUT);
+      s_abort = 1;
+    }
+    consumer_sync();
+    if (s_abort) break;
+    const int n = s_n[st];
+    const __half *sh = reinterpret_cast<const __half *>(pool_smem + st * sbytes);
+    const float2 *ss = reinterpret_cast<const float2 *>(pool_smem + st * sbytes + UMIM_MAX_SPAN_TOKENS * d * 2);
+    if (warp < n) {
+      // merge the per-tile (mean, M2) of row `warp`
+      Moments m{0.f, 0.f, 0.f};
+      for (int t = lane; t < ntiles; t += 32) m = merge_moments(m, Moments{(float)BN, ss[warp * ntiles + t].x,
+                                                                           ss[warp * ntiles + t].y});
 #pragma unroll
-  for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
-    mu[j] = 0.f;
-    rs[j] = 0.f;
-    if (j < n) {
-      const float2 m = row_moments_warp(stats + (int64_t)(t0 + j) * ntiles, ntiles, d, eps);
+      for (int o = 16; o >= 1; o >>= 1) {
+        Moments x{__shfl_xor_sync(0xffffffffu, m.n, o), __shfl_xor_sync(0xffffffffu, m.mean, o),
+                  __shfl_xor_sync(0xffffffffu, m.m2, o)};
+        m = merge_moments(m, x);
+      }
+      if (lane == 0) s_mom[warp] = make_float2(m.mean, rsqrtf(m.m2 / (float)d + eps));
+    }
+    consumer_sync();
+    float mu[UMIM_MAX_SPAN_TOKENS], rs[UMIM_MAX_SPAN_TOKENS];
+#pragma unroll
+    for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
+      const float2 m = j < n ? s_mom[j] : make_float2(0.f, 0.f);
       mu[j] = m.x;
       rs[j] = m.y;
     }
-  }
-  for (int i = lane; i < UMIM_MAX_SPAN_TOKENS * 8; i += 32) s_sc[warp][i / 8][i % 8] = 0.f;
-  __syncwarp();
-  const __half *Hs = H + (int64_t)t0 * d;
-  // pass 1: scores
-#pragma unroll 2
-  for (int c = lane * 8; c < d; c += 256) {
-    const int head = c / dh;
-    float g[8], b[8], q[8];
-    bf16x8_to_float(*reinterpret_cast<const uint4 *>(gamma + c), g);
-    bf16x8_to_float(*reinterpret_cast<const uint4 *>(beta + c), b);
-    bf16x8_to_float(*reinterpret_cast<const uint4 *>(query + c), q);   // query [h][dh] is d contiguous values
+    // scores
+    for (int cc = tid; cc < d / 8; cc += kPoolConsumers) {
+      const int c = cc * 8;
+      float g[8], b[8], q[8];
+      bf16x8_to_float(*reinterpret_cast<const uint4 *>(gamma + c), g);
+      bf16x8_to_float(*reinterpret_cast<const uint4 *>(beta + c), b);
+      bf16x8_to_float(*reinterpret_cast<const uint4 *>(query + c), q);   // query [h][dh]: d contiguous values
 #pragma unroll
-    for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
-      if (j < n) {
-        const uint4 x = *reinterpret_cast<const uint4 *>(Hs + (int64_t)j * d + c);
-        const __half2 *h2 = reinterpret_cast<const __half2 *>(&x);
-        float part = 0.f;
+      for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
+        if (j < n) {
+          const uint4 x = *reinterpret_cast<const uint4 *>(sh + j * d + c);
+          const __half2 *h2 = reinterpret_cast<const __half2 *>(&x);
+          float part = 0.f;
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float2 f = __half22float2(h2[e]);
-          part += ((f.x - mu[j]) * rs[j] * g[2 * e] + b[2 * e]) * q[2 * e];
-          part += ((f.y - mu[j]) * rs[j] * g[2 * e + 1] + b[2 * e + 1]) * q[2 * e + 1];
-        }
-        for (int o = seg >> 1; o >= 1; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o, seg);
-        if ((lane & (seg - 1)) == 0) atomicAdd(&s_sc[warp][j][head], part);
-      }
-    }
-  }
-  __syncwarp();
-  // softmax over the span, one lane per head
-  if (lane < h && n > 0) {
-    const float inv = rsqrtf((float)dh);
-    float sc[UMIM_MAX_SPAN_TOKENS];
-    float mx = -INFINITY;
-#pragma unroll
-    for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
-      sc[j] = j < n ? s_sc[warp][j][lane] * inv : -INFINITY;
-      mx = fmaxf(mx, sc[j]);
-    }
-    float den = 0.f;
-#pragma unroll
-    for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
-      sc[j] = j < n ? expf(sc[j] - mx) : 0.f;
-      den += sc[j];
-    }
-#pragma unroll
-    for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) s_al[warp][j][lane] = sc[j] / den;
-  }
-  __syncwarp();
-  // pass 2: o = sum_j alpha_j P_j
-  __half *Os = O + (int64_t)s * d;
-#pragma unroll 2
-  for (int c = lane * 8; c < d; c += 256) {
-    const int head = c / dh;
-    float g[8], b[8], o[8];
-    bf16x8_to_float(*reinterpret_cast<const uint4 *>(gamma + c), g);
-    bf16x8_to_float(*reinterpret_cast<const uint4 *>(beta + c), b);
-#pragma unroll
-    for (int e = 0; e < 8; ++e) o[e] = 0.f;
-#pragma unroll
-    for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
-      if (j < n) {
-        const float al = s_al[warp][j][head];
-        const uint4 x = *reinterpret_cast<const uint4 *>(Hs + (int64_t)j * d + c);
-        const __half2 *h2 = reinterpret_cast<const __half2 *>(&x);
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float2 f = __half22float2(h2[e]);
-          o[2 * e] += al * ((f.x - mu[j]) * rs[j] * g[2 * e] + b[2 * e]);
-          o[2 * e + 1] += al * ((f.y - mu[j]) * rs[j] * g[2 * e + 1] + b[2 * e + 1]);
+          for (int e = 0; e < 4; ++e) {
+            const float2 f = __half22float2(h2[e]);
+            part += ((f.x - mu[j]) * rs[j] * g[2 * e] + b[2 * e]) * q[2 * e];
+            part += ((f.y - mu[j]) * rs[j] * g[2 * e + 1] + b[2 * e + 1]) * q[2 * e + 1];
+          }
+          for (int o = seg >> 1; o >= 1; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o, seg);
+          if ((lane & (seg - 1)) == 0) s_red[j][cc / seg] = part;
         }
       }
     }
-    uint4 packed;
-    __half2 *hp = reinterpret_cast<__half2 *>(&packed);
+    consumer_sync();
+    if (tid < h && n > 0) {
+      const float inv = rsqrtf((float)dh);
+      float sc[UMIM_MAX_SPAN_TOKENS];
+      float mx = -INFINITY;
 #pragma unroll
-    for (int e = 0; e < 4; ++e) hp[e] = __floats2half2_rn(o[2 * e], o[2 * e + 1]);
-    *reinterpret_cast<uint4 *>(Os + c) = packed;
+      for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
+        float v = 0.f;
+        if (j < n)
+          for (int i = 0; i < seg_per_head; ++i) v += s_red[j][tid * seg_per_head + i];
+        sc[j] = j < n ? v * inv : -INFINITY;
+        mx = fmaxf(mx, sc[j]);
+      }
+      float den = 0.f;
+#pragma unroll
+      for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
+        sc[j] = j < n ? expf(sc[j] - mx) : 0.f;
+        den += sc[j];
+      }
+#pragma unroll
+      for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) s_al[j][tid] = sc[j] / den;
+    }
+    consumer_sync();
+    // o = sum_j alpha_j P_j
+    for (int cc = tid; cc < d / 8; cc += kPoolConsumers) {
+      const int c = cc * 8;
+      const int head = c / dh;
+      float g[8], b[8], o[8];
+      bf16x8_to_float(*reinterpret_cast<const uint4 *>(gamma + c), g);
+      bf16x8_to_float(*reinterpret_cast<const uint4 *>(beta + c), b);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) o[e] = 0.f;
+#pragma unroll
+      for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
+        if (j < n) {
+          const float al = s_al[j][head];
+          const uint4 x = *reinterpret_cast<const uint4 *>(sh + j * d + c);
+          const __half2 *h2 = reinterpret_cast<const __half2 *>(&x);
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const float2 f = __half22float2(h2[e]);
+            o[2 * e] += al * ((f.x - mu[j]) * rs[j] * g[2 * e] + b[2 * e]);
+            o[2 * e + 1] += al * ((f.y - mu[j]) * rs[j] * g[2 * e + 1] + b[2 * e + 1]);
+          }
+        }
+      }
+      uint4 packed;
+      __half2 *hp = reinterpret_cast<__half2 *>(&packed);
+#pragma unroll
+      for (int e = 0; e < 4; ++e) hp[e] = __floats2half2_rn(o[2 * e], o[2 * e + 1]);
+      *reinterpret_cast<uint4 *>(O + (int64_t)s * d + c) = packed;
+    }
+    // this warp no longer reads the stage
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&empty[st]);
+    consumer_sync();   // s_mom / s_red / s_al are rewritten for the next span
   }
 }
 
@@ -526,7 +609,16 @@ umim_status merge_spans(const void *embeddings, int64_t vocab, const int32_t *to
     if (r != UMIM_OK) return r;
   }
   trace_mark(st, "merge.pool");
-  pool_kernel<<<(S + kPoolWarps - 1) / kPoolWarps, kPoolWarps * 32, 0, st>>>(H, st1, span_offsets, S, T, d, w->n_heads,
+  const int psmem = kPoolRing * pool_stage_bytes(d);
+  if (cudaFuncSetAttribute(pool_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, psmem) != cudaSuccess)
+    return UMIM_ERR_CUDA;
+  int pool_per_sm = 1;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&pool_per_sm, pool_kernel, kPoolConsumers + 32, psmem) !=
+          cudaSuccess ||
+      pool_per_sm < 1)
+    pool_per_sm = 1;
+  const int pool_grid = std::max(1, std::min(S, std::max(1, num_sms) * pool_per_sm));
+  pool_kernel<<<pool_grid, kPoolConsumers + 32, psmem, st>>>(H, st1, span_offsets, S, T, d, w->n_heads,
                                           static_cast<const __nv_bfloat16 *>(w->ln_kv_gamma),
                                           static_cast<const __nv_bfloat16 *>(w->ln_kv_beta),
                                           static_cast<const __nv_bfloat16 *>(w->query), w->ln_eps, O, status);

@@ -22,15 +22,12 @@ namespace umim {
 namespace {
 
 constexpr int kMoveThreads = 256;
-constexpr int kUnitBytes = 32768;                     // data moved per unit
-constexpr int kChunksPerThread = kUnitBytes / 16 / kMoveThreads;   // 8 x 16 B
 constexpr int64_t kNoWrite = INT64_MIN;
 
 struct MoveArgs {
   uint16_t *pool;
   int32_t n_lanes;
   int32_t n_layers, n_pages, n_kv_heads, head_dim;
-  int32_t heads_per_unit, n_head_groups;
   int32_t *block_table;
   int32_t max_pages;
   int32_t *seq_lens;
@@ -75,18 +72,6 @@ __device__ __forceinline__ void st_v4(uint16_t *p, uint4 v) {
   asm volatile("st.global.v4.u32 [%0], {%1, %2, %3, %4};" ::"l"(p), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
                : "memory");
 }
-
-__device__ __forceinline__ void cp_async_16(void *smem, const void *gmem) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(smem)), "l"(gmem) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
-}
-
-constexpr int kRing = 3;   // units in flight per CTA
-constexpr int kMeta = kRing + 2;
 
 struct PageDesc {
   int64_t *src;    // [pages][16] source row offset within a layer (no head offset), -(i+1) for span i, kNoWrite
@@ -144,29 +129,20 @@ __global__ void __launch_bounds__(256) rollback_map_kernel(MoveArgs a, PlanArray
   if (lane == kPageSize) pd.dep[idx] = make_int2(mn, mx);
 }
 
-struct UnitMeta {
-  int unit, b, layer, p, nh, h0, dep_lo, dep_hi;
-  int64_t src[kPageSize];
-};
-
+// One warp per unit = one (layer, K|V, head) 16 x D tile of a compacted
+// page.  Lane l moves 16-byte chunks c = l + 32 it of the tile: row c / CPR
+// (the slot), column c % CPR.
 template <int D>
-__global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a, PlanArrays arr, PageDesc pd) {
-  constexpr int CPR = D / 8;                                   // 16-byte chunks per (kv, head) row
-  constexpr int NH = kUnitBytes / (2 * kPageSize * D * 2);     // KV heads per unit
-  constexpr int CHUNKS = 2 * NH * kPageSize * CPR;
-  static_assert(CHUNKS == kChunksPerThread * kMoveThreads, "unit size");
-  // Chunk c = tid + it * 256 of a unit is 16-byte column c % CPR of row
-  // c / CPR = ((kv * NH + h) * 16 + slot).  256 is a multiple of 16 * CPR, so
-  // a thread's column and slot are the same for every it; only (kv, h) vary.
-  const int tid = threadIdx.x, lane_id = tid & 31, warp = tid >> 5;
-  const int my_col = tid % CPR;
-  const int my_slot = (tid / CPR) % kPageSize;
-  const int my_kvh0 = tid / (CPR * kPageSize);
-  constexpr int KVH_STEP = kMoveThreads / (CPR * kPageSize);
-
-  extern __shared__ __align__(16) uint8_t ring[];              // kRing x 32 KB of unit data
-  __shared__ UnitMeta meta[kMeta];
-  __shared__ int s_last, s_abort, s_done;
+__global__ void __launch_bounds__(kMoveThreads, 4) rollback_move_kernel(MoveArgs a, PlanArrays arr, PageDesc pd) {
+  constexpr int CPR = D / 8;                       // 16-byte chunks per row
+  constexpr int PER_LANE = kPageSize * CPR / 32;   // 8 (D=128) or 4 (D=64)
+  constexpr int SLOT_STEP = 32 / CPR;              // slots advanced per it
+  const int lane = threadIdx.x & 31;
+  const int gw = blockIdx.x * (kMoveThreads / 32) + (threadIdx.x >> 5);
+  const int nw = gridDim.x * (kMoveThreads / 32);
+  const int my_col = lane % CPR;
+  const int my_slot0 = lane / CPR;
+  __shared__ int s_last;
 
   const PlanHeader *hdr = arr.hdr;
   const int total = hdr->total_units;
@@ -174,140 +150,84 @@ __global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a,
   const int Hkv = a.n_kv_heads;
   const int64_t head_stride = (int64_t)kPageSize * D;
   const int64_t kv_stride = head_stride * Hkv;
-  const int64_t layer_stride = kv_stride * 2 * a.n_pages;
+  const int64_t page_stride = kv_stride * 2;
+  const int64_t layer_stride = page_stride * a.n_pages;
+  bool abort = false;
 
-  // warp 1: describe this CTA's next unit (units blockIdx.x, blockIdx.x +
-  // gridDim.x, ... in increasing order) from its precomputed description
-  int next_unit = blockIdx.x;
-  auto describe = [&](int m) {
-    int u = 0, b = 0, ln = 0, k = 0;
-    if (lane_id == 0) {
-      u = next_unit;
-      if (u < total) {
-        b = find_seq(arr.unit_base, a.B, u);
-        const int rem = u - arr.unit_base[b];
-        const int nd = arr.n_dest[b];
-        ln = rem / nd;
-        k = rem % nd;
-      }
-    }
-    next_unit += gridDim.x;
-    u = __shfl_sync(0xffffffffu, u, 0);
-    UnitMeta &M = meta[m];
-    if (u >= total) {
-      if (lane_id == 0) M.unit = u;
-      return;
-    }
-    b = __shfl_sync(0xffffffffu, b, 0);
-    ln = __shfl_sync(0xffffffffu, ln, 0);
-    k = __shfl_sync(0xffffffffu, k, 0);
+  for (int u = gw; u < total && !abort; u += nw) {
+    // unit -> (sequence, tile lane, compacted page)
+    const int b = find_seq(arr.unit_base, a.B, u);
+    const int rem = u - arr.unit_base[b];
+    const int nd = arr.n_dest[b];
+    const int tl = rem / nd, k = rem % nd;
+    const int layer = tl / (2 * Hkv);
+    const int kv = (tl / Hkv) & 1;
+    const int h = tl % Hkv;
     const int idx = arr.unit_base[b] / a.n_lanes + k;
-    if (lane_id < kPageSize) M.src[lane_id] = pd.src[(int64_t)idx * kPageSize + lane_id];
-    if (lane_id == 0) {
-      const int2 dep = pd.dep[idx];
-      const int h0 = (ln % a.n_head_groups) * NH;
-      M.unit = u;
-      M.b = b;
-      M.layer = ln / a.n_head_groups;
-      M.p = arr.first_page[b] + k;
-      M.h0 = h0;
-      M.nh = min(NH, Hkv - h0);
-      M.dep_lo = dep.x;
-      M.dep_hi = dep.y;
-    }
-  };
+    const int p = arr.first_page[b] + k;
+    const int64_t my_src = lane < kPageSize ? pd.src[(int64_t)idx * kPageSize + lane] : kNoWrite;
+    const int2 dep = pd.dep[idx];
+    const int64_t tile = layer * layer_stride + kv * kv_stride + h * head_stride + my_col * 8;
+    const uint16_t *sur = kv ? a.sur_v : a.sur_k;
 
-  // every thread: start the copies of the unit in meta[m] into ring stage st
-  auto issue = [&](int m, int st) {
-    const UnitMeta &M = meta[m];
-    if (M.unit < total) {
-      const int64_t src = M.src[my_slot];
-      uint8_t *dst = ring + st * kUnitBytes;
-      const int64_t base = M.layer * layer_stride + M.h0 * head_stride + my_col * 8;
+    uint4 v[PER_LANE];
+    uint32_t write_mask = 0;
+    uint32_t fold = 0;
 #pragma unroll
-      for (int it = 0; it < kChunksPerThread; ++it) {
-        const int kvh = my_kvh0 + it * KVH_STEP;
-        const int h = kvh % NH, kv = kvh / NH;
-        if (h < M.nh && src != kNoWrite) {
-          const uint16_t *g;
-          if (src >= 0) {
-            g = a.pool + base + src + kv * kv_stride + h * head_stride;
-          } else {
-            const int64_t i = -src - 1;
-            g = (kv ? a.sur_v : a.sur_k) + ((i * a.n_layers + M.layer) * Hkv + M.h0 + h) * D + my_col * 8;
-          }
-          cp_async_16(dst + (tid + it * kMoveThreads) * 16, g);
-        }
+    for (int it = 0; it < PER_LANE; ++it) {
+      const int slot = my_slot0 + it * SLOT_STEP;
+      const int64_t src = __shfl_sync(0xffffffffu, my_src, slot);
+      if (src != kNoWrite) write_mask |= 1u << it;
+      v[it] = make_uint4(0, 0, 0, 0);
+      if (src >= 0) {
+        v[it] = ld_v4(a.pool + tile + src);
+      } else if (src != kNoWrite) {
+        const int64_t i = -src - 1;
+        v[it] = ld_v4(sur + ((i * a.n_layers + layer) * Hkv + h) * D + my_col * 8);
       }
+      fold ^= v[it].x ^ v[it].y ^ v[it].z ^ v[it].w;
     }
-    cp_async_commit();   // one group per ring slot, empty or not
-  };
-
-  if (tid == 0) s_abort = 0;
-  // prologue: units 0 .. kRing-2 in flight, unit kRing-1 described
-  if (warp == 1) describe(0);
-  __syncthreads();
-  for (int k = 0; k < kRing - 1; ++k) {
-    issue(k % kMeta, k % kRing);
-    if (warp == 1) describe((k + 1) % kMeta);
-    __syncthreads();
-  }
-  for (int cur = 0;; ++cur) {
-    const int head = cur + kRing - 1;
-    issue(head % kMeta, head % kRing);
-    cp_async_wait<kRing - 1>();          // this thread's copies of unit `cur` have landed
-    __syncthreads();
-    const UnitMeta &M = meta[cur % kMeta];
-    if (tid == 0) {
-      const int u = M.unit;
-      s_done = u >= total;    // this CTA's units increase: nothing younger is valid either
-      if (u < total) {
-        const int p = M.p;
-        // release: every copy of this unit has landed (wait_group + barrier)
-        st_release(&arr.flags[u], epoch);
-        // wait for the units that read old page p (all have smaller indices)
-        for (int q = M.dep_lo; q <= M.dep_hi && q >= 0 && q < p; ++q) {
-          const int uq = u - (p - q);
-          if (ld_acquire(&arr.flags[uq]) == epoch) continue;
-          const uint64_t t0 = globaltimer();
-          bool ok = false;
-          while (!ok) {
+    // every loaded value of this lane has arrived before the warp barrier
+    asm volatile("" ::"r"(fold));
+    __syncwarp();
+    int ok = 1;
+    if (lane == 0) {
+      // release: the warp's loads are ordered before it by the warp barrier
+      st_release(&arr.flags[u], epoch);
+      // wait for the units that read this tile of old page p (smaller indices)
+      for (int q = dep.x; q <= dep.y && q >= 0 && q < p; ++q) {
+        const int uq = u - (p - q);
+        if (ld_acquire(&arr.flags[uq]) == epoch) continue;
+        const uint64_t t0 = globaltimer();
+        bool got = false;
+        while (!got) {
 #pragma unroll 1
-            for (int i = 0; i < 64 && !ok; ++i) ok = (ld_acquire(&arr.flags[uq]) == epoch);
-            if (!ok && globaltimer() - t0 > kWaitLimitNs) break;
-          }
-          if (!ok) {
-            set_error(a.status, UMIM_ERR_TIMEOUT);
-            s_abort = 1;
-            break;
-          }
+          for (int i = 0; i < 64 && !got; ++i) got = (ld_acquire(&arr.flags[uq]) == epoch);
+          if (!got && globaltimer() - t0 > kWaitLimitNs) break;
+        }
+        if (!got) {
+          set_error(a.status, UMIM_ERR_TIMEOUT);
+          ok = 0;
+          break;
         }
       }
     }
-    if (warp == 1) describe((head + 1) % kMeta);
-    __syncthreads();
-    if (s_done) break;
-    const int64_t src = M.src[my_slot];
-    if (!s_abort && src != kNoWrite) {
-      const int32_t *bt = a.block_table + (int64_t)M.b * a.max_pages;
-      const int64_t dst = M.layer * layer_stride + M.h0 * head_stride +
-                          (int64_t)bt[M.p] * (kv_stride * 2) + my_slot * D + my_col * 8;
-      const uint8_t *stage = ring + (cur % kRing) * kUnitBytes;
+    ok = __shfl_sync(0xffffffffu, ok, 0);
+    if (!ok) {
+      abort = true;
+      break;
+    }
+    const int64_t dst = tile + (int64_t)a.block_table[(int64_t)b * a.max_pages + p] * page_stride;
 #pragma unroll
-      for (int it = 0; it < kChunksPerThread; ++it) {
-        const int kvh = my_kvh0 + it * KVH_STEP;
-        const int h = kvh % NH, kv = kvh / NH;
-        if (h < M.nh) {
-          const uint4 v = *reinterpret_cast<const uint4 *>(stage + (tid + it * kMoveThreads) * 16);
-          st_v4(a.pool + dst + kv * kv_stride + h * head_stride, v);
-        }
-      }
+    for (int it = 0; it < PER_LANE; ++it) {
+      const int slot = my_slot0 + it * SLOT_STEP;
+      if (write_mask & (1u << it)) st_v4(a.pool + dst + slot * D, v[it]);
     }
-    __syncthreads();   // stage cur % kRing is refilled by the next issue
   }
-  cp_async_wait<0>();
 
   // ---- the last CTA to finish truncates block tables and updates lengths ----
+  const int tid = threadIdx.x;
+  __syncthreads();
   if (tid == 0) {
     __threadfence();
     const int done = atomicAdd(&arr.hdr->done_ctas, 1);
@@ -338,9 +258,8 @@ __global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a,
 }  // namespace
 
 size_t kv_rollback_workspace_bytes(int B, int S, int max_pages, int n_layers, int n_kv_heads, int head_dim) {
-  const int hpu = std::max(1, kUnitBytes / (2 * kPageSize * head_dim * 2));
-  const int groups = (n_kv_heads + hpu - 1) / hpu;
-  const size_t units = (size_t)B * n_layers * groups * (size_t)max_pages;
+  (void)head_dim;
+  const size_t units = (size_t)B * n_layers * 2 * n_kv_heads * (size_t)max_pages;
   const size_t pages = (size_t)B * max_pages;
   return plan_bytes(B, S) + align256(sizeof(int32_t) * (units > 0 ? units : 1)) +
          align256(sizeof(int64_t) * kPageSize * (pages > 0 ? pages : 1)) + align256(sizeof(int2) * (pages > 0 ? pages : 1));
@@ -352,11 +271,10 @@ umim_status kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t m
                         int32_t *freed_pages, void *ws, size_t ws_bytes, int32_t *dev_status,
                         cudaStream_t stream, int num_sms) {
   const int D = kv->head_dim;
-  const int hp = kUnitBytes / (2 * kPageSize * D * 2);     // heads per unit (the kernel's NH)
-  const int groups = (kv->n_kv_heads + hp - 1) / hp;
+  const int lanes = kv->n_layers * 2 * kv->n_kv_heads;   // one unit per (layer, K|V, head) tile
   PlanArrays arr = plan_carve(ws, B, S);
   int32_t *status = dev_status ? dev_status : &arr.hdr->status;
-  const size_t units = (size_t)B * kv->n_layers * groups * (size_t)max_pages;
+  const size_t units = (size_t)B * lanes * (size_t)max_pages;
   const size_t pages = (size_t)B * max_pages;
   PageDesc pd;
   pd.src = reinterpret_cast<int64_t *>(reinterpret_cast<char *>(arr.flags) +
@@ -376,7 +294,7 @@ umim_status kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t m
   pa.block_table = block_table;
   pa.max_pages = max_pages;
   pa.n_pages = kv->n_pages;
-  pa.n_lanes = kv->n_layers * groups;
+  pa.n_lanes = lanes;
   pa.status = status;
   pa.cu_seqlens_out = nullptr;
   trace_mark(stream, "rollback.plan");
@@ -384,13 +302,11 @@ umim_status kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t m
 
   MoveArgs ma{};
   ma.pool = static_cast<uint16_t *>(kv->base);
-  ma.n_lanes = kv->n_layers * groups;
+  ma.n_lanes = lanes;
   ma.n_layers = kv->n_layers;
   ma.n_pages = kv->n_pages;
   ma.n_kv_heads = kv->n_kv_heads;
   ma.head_dim = D;
-  ma.heads_per_unit = hp;
-  ma.n_head_groups = groups;
   ma.block_table = block_table;
   ma.max_pages = max_pages;
   ma.seq_lens = seq_lens;
@@ -404,9 +320,7 @@ umim_status kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t m
   ma.B = B;
   ma.status = status;
   auto kern = (D == 128) ? rollback_move_kernel<128> : rollback_move_kernel<64>;
-  const int smem = kRing * kUnitBytes;
-  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
-    return UMIM_ERR_CUDA;
+  const int smem = 0;
   int per_sm = 0;
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kMoveThreads, smem) != cudaSuccess || per_sm < 1)
     per_sm = 1;
