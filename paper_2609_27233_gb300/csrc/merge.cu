@@ -276,11 +276,16 @@ __device__ __forceinline__ float2 row_moments_warp(const float2 *st, int ntiles,
 // Persistent CTAs; span s goes to CTA s mod grid.  A producer warp copies each
 // span's H rows (fp16) and row statistics into a 3-stage shared-memory ring
 // with bulk asynchronous copies completing an mbarrier; 8 consumer warps
-// compute from shared memory: P = LN_kv(H), the scores <P_j[head], q_head>,
-// the softmax over the span and o = sum_j alpha_j P_j, written in fp16
-// (11 significant bits) as the A operand of the output projection.
-// 16-byte column chunk cc (columns 8 cc .. 8 cc + 7) belongs to consumer
-// thread cc mod 256.
+// compute from shared memory.  With P_jc = (H_jc - mu_j) r_j gamma_c + beta_c,
+//   <P_j[head], q_head> = r_j (sum_c H_jc gamma_c q_c - mu_j A_head) + B_head,
+//   A_head = sum_c gamma_c q_c,  B_head = sum_c beta_c q_c   (c in head),
+// and, because the softmax weights alpha_j sum to one,
+//   o_c = sum_j alpha_j P_jc = gamma_c (sum_j w_j H_jc - C_head) + beta_c,
+//   w_j = alpha_j r_j,  C_head = sum_j w_j mu_j,
+// so each element costs one multiply-add per span row in each pass.  o is
+// written in fp16 (11 significant bits) as the A operand of the output
+// projection.  16-byte column chunk cc (columns 8 cc .. 8 cc + 7) belongs to
+// consumer thread cc mod 256; CH chunks per thread.
 // ---------------------------------------------------------------------------
 constexpr int kPoolRing = 3;
 constexpr int kPoolConsumers = 256;
@@ -294,9 +299,12 @@ __device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t by
 
 __device__ __forceinline__ void consumer_sync() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
 
-__host__ __device__ inline int pool_stage_bytes(int d) { return (UMIM_MAX_SPAN_TOKENS * (d * 2 + (d / BN) * 8) + 127) & ~127; }
+__host__ __device__ inline int pool_stage_bytes(int d) {
+  return (UMIM_MAX_SPAN_TOKENS * (d * 2 + (d / BN) * 8) + 127) & ~127;
+}
 
-__global__ void __launch_bounds__(kPoolConsumers + 32, 1)
+template <int CH>
+__global__ void __launch_bounds__(kPoolConsumers + 32, CH <= 2 ? 2 : 1)
     pool_kernel(const __half *H, const float2 *stats, const int32_t *offs, int S, int64_t T, int d, int h,
                 const __nv_bfloat16 *gamma, const __nv_bfloat16 *beta, const __nv_bfloat16 *query, float eps,
                 __half *O, int32_t *status) {
@@ -305,7 +313,8 @@ __global__ void __launch_bounds__(kPoolConsumers + 32, 1)
   __shared__ int s_n[kPoolRing];
   __shared__ float2 s_mom[UMIM_MAX_SPAN_TOKENS];
   __shared__ float s_red[UMIM_MAX_SPAN_TOKENS][128];
-  __shared__ float s_al[UMIM_MAX_SPAN_TOKENS][8];
+  __shared__ float s_w[UMIM_MAX_SPAN_TOKENS][8];
+  __shared__ float s_A[8], s_B[8], s_C[8];
   __shared__ int s_abort;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int ntiles = d / BN;
@@ -322,6 +331,10 @@ __global__ void __launch_bounds__(kPoolConsumers + 32, 1)
     }
     s_abort = 0;
     fence_mbar_init();
+  }
+  if (tid < 8) {
+    s_A[tid] = 0.f;
+    s_B[tid] = 0.f;
   }
   __syncthreads();
 
@@ -358,7 +371,36 @@ __global__ void __launch_bounds__(kPoolConsumers + 32, 1)
     return;
   }
 
-  // ---- consumers ----
+  // ---- consumers: per-column constants, kept for every span of this CTA ----
+  float g[CH][8], b[CH][8], gq[CH][8];
+#pragma unroll
+  for (int i = 0; i < CH; ++i) {
+    const int cc = tid + i * kPoolConsumers;
+    if (cc < d / 8) {
+      const int c = cc * 8;
+      float q[8];
+      bf16x8_to_float(*reinterpret_cast<const uint4 *>(gamma + c), g[i]);
+      bf16x8_to_float(*reinterpret_cast<const uint4 *>(beta + c), b[i]);
+      bf16x8_to_float(*reinterpret_cast<const uint4 *>(query + c), q);   // query [h][dh]: d contiguous values
+      float a = 0.f, bb = 0.f;
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        gq[i][e] = g[i][e] * q[e];
+        a += gq[i][e];
+        bb += b[i][e] * q[e];
+      }
+      for (int o = seg >> 1; o >= 1; o >>= 1) {
+        a += __shfl_xor_sync(0xffffffffu, a, o, seg);
+        bb += __shfl_xor_sync(0xffffffffu, bb, o, seg);
+      }
+      if ((lane & (seg - 1)) == 0) {
+        atomicAdd(&s_A[c / dh], a);
+        atomicAdd(&s_B[c / dh], bb);
+      }
+    }
+  }
+  consumer_sync();
+
   int k = 0;
   for (int s = blockIdx.x; s < S; s += gridDim.x, ++k) {
     const int st = k % kPoolRing;
@@ -384,39 +426,31 @@ __global__ void __launch_bounds__(kPoolConsumers + 32, 1)
       }
       if (lane == 0) s_mom[warp] = make_float2(m.mean, rsqrtf(m.m2 / (float)d + eps));
     }
-    consumer_sync();
-    float mu[UMIM_MAX_SPAN_TOKENS], rs[UMIM_MAX_SPAN_TOKENS];
+    // pass 1: sum_c H_jc gamma_c q_c per (row, segment)
 #pragma unroll
-    for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
-      const float2 m = j < n ? s_mom[j] : make_float2(0.f, 0.f);
-      mu[j] = m.x;
-      rs[j] = m.y;
-    }
-    // scores
-    for (int cc = tid; cc < d / 8; cc += kPoolConsumers) {
-      const int c = cc * 8;
-      float g[8], b[8], q[8];
-      bf16x8_to_float(*reinterpret_cast<const uint4 *>(gamma + c), g);
-      bf16x8_to_float(*reinterpret_cast<const uint4 *>(beta + c), b);
-      bf16x8_to_float(*reinterpret_cast<const uint4 *>(query + c), q);   // query [h][dh]: d contiguous values
+    for (int i = 0; i < CH; ++i) {
+      const int cc = tid + i * kPoolConsumers;
+      if (cc < d / 8) {
 #pragma unroll
-      for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
-        if (j < n) {
-          const uint4 x = *reinterpret_cast<const uint4 *>(sh + j * d + c);
-          const __half2 *h2 = reinterpret_cast<const __half2 *>(&x);
-          float part = 0.f;
+        for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
+          if (j < n) {
+            const uint4 x = *reinterpret_cast<const uint4 *>(sh + j * d + cc * 8);
+            const __half2 *h2 = reinterpret_cast<const __half2 *>(&x);
+            float part = 0.f;
 #pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const float2 f = __half22float2(h2[e]);
-            part += ((f.x - mu[j]) * rs[j] * g[2 * e] + b[2 * e]) * q[2 * e];
-            part += ((f.y - mu[j]) * rs[j] * g[2 * e + 1] + b[2 * e + 1]) * q[2 * e + 1];
+            for (int e = 0; e < 4; ++e) {
+              const float2 f = __half22float2(h2[e]);
+              part = fmaf(f.x, gq[i][2 * e], part);
+              part = fmaf(f.y, gq[i][2 * e + 1], part);
+            }
+            for (int o = seg >> 1; o >= 1; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o, seg);
+            if ((lane & (seg - 1)) == 0) s_red[j][cc / seg] = part;
           }
-          for (int o = seg >> 1; o >= 1; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o, seg);
-          if ((lane & (seg - 1)) == 0) s_red[j][cc / seg] = part;
         }
       }
     }
     consumer_sync();
+    // softmax over the span for each head, then w_j = alpha_j r_j and C_head
     if (tid < h && n > 0) {
       const float inv = rsqrtf((float)dh);
       float sc[UMIM_MAX_SPAN_TOKENS];
@@ -424,9 +458,13 @@ __global__ void __launch_bounds__(kPoolConsumers + 32, 1)
 #pragma unroll
       for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
         float v = 0.f;
-        if (j < n)
+        if (j < n) {
           for (int i = 0; i < seg_per_head; ++i) v += s_red[j][tid * seg_per_head + i];
-        sc[j] = j < n ? v * inv : -INFINITY;
+          const float2 m = s_mom[j];
+          sc[j] = (m.y * (v - m.x * s_A[tid]) + s_B[tid]) * inv;
+        } else {
+          sc[j] = -INFINITY;
+        }
         mx = fmaxf(mx, sc[j]);
       }
       float den = 0.f;
@@ -435,43 +473,56 @@ __global__ void __launch_bounds__(kPoolConsumers + 32, 1)
         sc[j] = j < n ? expf(sc[j] - mx) : 0.f;
         den += sc[j];
       }
-#pragma unroll
-      for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) s_al[j][tid] = sc[j] / den;
-    }
-    consumer_sync();
-    // o = sum_j alpha_j P_j
-    for (int cc = tid; cc < d / 8; cc += kPoolConsumers) {
-      const int c = cc * 8;
-      const int head = c / dh;
-      float g[8], b[8], o[8];
-      bf16x8_to_float(*reinterpret_cast<const uint4 *>(gamma + c), g);
-      bf16x8_to_float(*reinterpret_cast<const uint4 *>(beta + c), b);
-#pragma unroll
-      for (int e = 0; e < 8; ++e) o[e] = 0.f;
+      float C = 0.f;
 #pragma unroll
       for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
-        if (j < n) {
-          const float al = s_al[j][head];
-          const uint4 x = *reinterpret_cast<const uint4 *>(sh + j * d + c);
-          const __half2 *h2 = reinterpret_cast<const __half2 *>(&x);
+        const float2 m = j < n ? s_mom[j] : make_float2(0.f, 0.f);
+        const float wj = sc[j] / den * m.y;
+        s_w[j][tid] = wj;
+        C += wj * m.x;
+      }
+      s_C[tid] = C;
+    }
+    consumer_sync();
+    // pass 2: o_c = gamma_c (sum_j w_j H_jc - C_head) + beta_c
 #pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const float2 f = __half22float2(h2[e]);
-            o[2 * e] += al * ((f.x - mu[j]) * rs[j] * g[2 * e] + b[2 * e]);
-            o[2 * e + 1] += al * ((f.y - mu[j]) * rs[j] * g[2 * e + 1] + b[2 * e + 1]);
+    for (int i = 0; i < CH; ++i) {
+      const int cc = tid + i * kPoolConsumers;
+      if (cc < d / 8) {
+        const int head = cc * 8 / dh;
+        float x[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) x[e] = 0.f;
+#pragma unroll
+        for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
+          if (j < n) {
+            const float wj = s_w[j][head];
+            const uint4 hv = *reinterpret_cast<const uint4 *>(sh + j * d + cc * 8);
+            const __half2 *h2 = reinterpret_cast<const __half2 *>(&hv);
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const float2 f = __half22float2(h2[e]);
+              x[2 * e] = fmaf(wj, f.x, x[2 * e]);
+              x[2 * e + 1] = fmaf(wj, f.y, x[2 * e + 1]);
+            }
           }
         }
-      }
-      uint4 packed;
-      __half2 *hp = reinterpret_cast<__half2 *>(&packed);
+        const float C = n > 0 ? s_C[head] : 0.f;
+        uint4 packed;
+        __half2 *hp = reinterpret_cast<__half2 *>(&packed);
 #pragma unroll
-      for (int e = 0; e < 4; ++e) hp[e] = __floats2half2_rn(o[2 * e], o[2 * e + 1]);
-      *reinterpret_cast<uint4 *>(O + (int64_t)s * d + c) = packed;
+        for (int e = 0; e < 4; ++e) {
+          const float o0 = n > 0 ? fmaf(g[i][2 * e], x[2 * e] - C, b[i][2 * e]) : 0.f;
+          const float o1 = n > 0 ? fmaf(g[i][2 * e + 1], x[2 * e + 1] - C, b[i][2 * e + 1]) : 0.f;
+          hp[e] = __floats2half2_rn(o0, o1);
+        }
+        *reinterpret_cast<uint4 *>(O + (int64_t)s * d + cc * 8) = packed;
+      }
     }
     // this warp no longer reads the stage
     __syncwarp();
     if (lane == 0) mbar_arrive(&empty[st]);
-    consumer_sync();   // s_mom / s_red / s_al are rewritten for the next span
+    consumer_sync();   // s_mom / s_red / s_w / s_C are rewritten for the next span
   }
 }
 
@@ -610,15 +661,16 @@ umim_status merge_spans(const void *embeddings, int64_t vocab, const int32_t *to
   }
   trace_mark(st, "merge.pool");
   const int psmem = kPoolRing * pool_stage_bytes(d);
-  if (cudaFuncSetAttribute(pool_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, psmem) != cudaSuccess)
+  const int chunks = d / 8 / kPoolConsumers;   // 16-byte column chunks per consumer thread (d <= 8192)
+  auto pk = chunks <= 1 ? pool_kernel<1> : (chunks == 2 ? pool_kernel<2> : pool_kernel<4>);
+  if (cudaFuncSetAttribute(pk, cudaFuncAttributeMaxDynamicSharedMemorySize, psmem) != cudaSuccess)
     return UMIM_ERR_CUDA;
   int pool_per_sm = 1;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&pool_per_sm, pool_kernel, kPoolConsumers + 32, psmem) !=
-          cudaSuccess ||
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&pool_per_sm, pk, kPoolConsumers + 32, psmem) != cudaSuccess ||
       pool_per_sm < 1)
     pool_per_sm = 1;
   const int pool_grid = std::max(1, std::min(S, std::max(1, num_sms) * pool_per_sm));
-  pool_kernel<<<pool_grid, kPoolConsumers + 32, psmem, st>>>(H, st1, span_offsets, S, T, d, w->n_heads,
+  pk<<<pool_grid, kPoolConsumers + 32, psmem, st>>>(H, st1, span_offsets, S, T, d, w->n_heads,
                                           static_cast<const __nv_bfloat16 *>(w->ln_kv_gamma),
                                           static_cast<const __nv_bfloat16 *>(w->ln_kv_beta),
                                           static_cast<const __nv_bfloat16 *>(w->query), w->ln_eps, O, status);
