@@ -187,17 +187,13 @@ __global__ void __launch_bounds__(kMoveThreads, 4) rollback_move_kernel(MoveArgs
       }
       fold ^= v[it].x ^ v[it].y ^ v[it].z ^ v[it].w;
     }
-    // The flag value is made to depend on every loaded word, so no lane passes
-    // the warp barrier, and lane 0 cannot even issue the flag store, before
-    // all of this unit's loads have returned their data: once the flag is
-    // visible the source slots may be overwritten.  No release fence is
-    // needed (and none waits for the previous unit's stores to drain).
-    int flag_val = epoch;
-    asm volatile("" : "+r"(flag_val) : "r"(fold) : "memory");
+    // every loaded value of this lane has arrived before the warp barrier
+    asm volatile("" ::"r"(fold) : "memory");
     __syncwarp();
     int ok = 1;
     if (lane == 0) {
-      st_relaxed(&arr.flags[u], flag_val);
+      // release: the warp's loads are ordered before it by the warp barrier
+      st_release(&arr.flags[u], epoch);
       // wait for the units that read this tile of old page p (smaller indices)
       for (int q = dep.x; q <= dep.y && q >= 0 && q < p; ++q) {
         const int uq = u - (p - q);
