@@ -232,6 +232,36 @@ umim_status umim_decode_attention(const void *q, int32_t n_q_heads, const umim_p
                                   size_t workspace_bytes, int32_t *dev_status, cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
+ * Decode attention for callers that cannot allocate GPU memory.
+ * The paper has no counterpart to this call; it is a convenience of this
+ * library.  A serving engine that gives all device memory to its own block
+ * allocator up front, or a plug-in running inside another framework that
+ * forbids allocations outside its arena, may be unable to provide the
+ * workspace that umim_decode_attention needs.  This variant computes exactly
+ * the same result but takes its scratch (split-K plan and fp32 partials)
+ * from an array of UMIM_STATIC_SCRATCH_BYTES compiled into the library; every
+ * GPU that loads the library holds that array until the process exits.
+ *  - Arguments and results are those of umim_decode_attention, without the
+ *    workspace.  It allocates nothing and calls no allocating routine.
+ *  - A batch whose scratch would exceed the array (about
+ *    (batch * n_kv_heads + 8 * SMs) * 16 * (head_dim + 2) * 4 bytes) is
+ *    rejected with UMIM_ERR_WORKSPACE before anything is launched.
+ *  - The first call on a device looks up the array's device address
+ *    (cudaGetSymbolAddress) and the SM count; make that first call before
+ *    any stream capture begins.
+ *  - All calls share the one array.  Nothing in it has to start at zero
+ *    (each call rewrites every field it reads), but calls whose kernels
+ *    overlap on the GPU (different streams, no ordering between them) race
+ *    on it and give wrong results: order such calls on one stream.
+ * ------------------------------------------------------------------------ */
+#define UMIM_STATIC_SCRATCH_BYTES (32u << 20)
+
+umim_status umim_decode_attention_static(const void *q, int32_t n_q_heads, const umim_paged_kv *kv,
+                                         int32_t layer, const int32_t *block_table, int32_t max_pages,
+                                         const int32_t *seq_lens, int32_t batch, float scale, void *out,
+                                         int32_t *dev_status, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
  * Kernel tracing, for profiling (not part of the method).  Between
  * umim_trace_start and umim_trace_stop every call above records a CUDA
  * event on its stream before each kernel it launches and one after its last

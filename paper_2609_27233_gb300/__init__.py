@@ -193,6 +193,23 @@ def umim_decode_attention(q, pool, layer, block_table, seq_lens, scale=0.0, out=
     return out
 
 
+def umim_decode_attention_static(q, pool, layer, block_table, seq_lens, scale=0.0, out=None, dev_status=None,
+                                 stream=None):
+    """Decode attention without a workspace argument, for callers that cannot
+    allocate GPU memory at call time: the library's fixed scratch array is
+    used instead (see include/umim.h for the size limit and the rule that
+    overlapping calls must not run concurrently)."""
+    kv = paged_kv(pool)
+    B, Hq, D = q.shape
+    if out is None:
+        out = torch.empty_like(q)
+    code = lib().umim_decode_attention_static(_p(q), Hq, ctypes.byref(kv), layer, _p(block_table),
+                                              block_table.shape[1], _p(seq_lens), B, float(scale), _p(out),
+                                              _p(dev_status), _stream(stream))
+    _check(code, "umim_decode_attention_static")
+    return out
+
+
 # ---------------------------------------------------------------------------
 # kernel tracing (profiling aid)
 # ---------------------------------------------------------------------------

@@ -48,6 +48,8 @@ SIGNATURES = {
     "umim_decode_attention": (ctypes.c_int, [c_ptr, c_i32, ctypes.POINTER(PagedKVC), c_i32, c_ptr, c_i32,
                                              c_ptr, c_i32, ctypes.c_float, c_ptr, c_ptr, c_size, c_ptr,
                                              c_ptr]),
+    "umim_decode_attention_static": (ctypes.c_int, [c_ptr, c_i32, ctypes.POINTER(PagedKVC), c_i32, c_ptr, c_i32,
+                                                    c_ptr, c_i32, ctypes.c_float, c_ptr, c_ptr, c_ptr]),
     "umim_trace_start": (ctypes.c_int, [c_i32]),
     "umim_trace_stop": (None, []),
     "umim_trace_read": (c_i32, [ctypes.POINTER(ctypes.c_float), ctypes.POINTER(ctypes.c_char_p), c_i32]),
