@@ -107,6 +107,7 @@ __device__ int scan1024(int v, int &total) {
 __global__ void __launch_bounds__(kPlanThreadsA)
     attn_plan_kernel(const int32_t *seq_lens, int B, int Hkv, int max_pages, int total_warps, AttnWs ws,
                      int32_t *status) {
+  griddep_wait();
   const int nseg = B * Hkv;
   // pass 1: segment offsets (segment (b, g) has n_b pages)
   int carry = 0;
@@ -223,6 +224,7 @@ __global__ void __launch_bounds__(kAttnWarps * 32, 1)
     if (warp == 0) prefetch_tensormap(&kv_map);
   }
   __syncwarp();
+  griddep_wait();
 
   const int W = ws.plan->W, total = ws.plan->total, nseg = ws.plan->n_seg;
   const int start = gw * W;
@@ -452,6 +454,7 @@ __global__ void __launch_bounds__(kAttnWarps * 32, 1)
 // ---------------------------------------------------------------------------
 template <int D>
 __global__ void attn_combine_kernel(AttnWs ws, int B, int Hq, int Hkv, int G, __nv_bfloat16 *out) {
+  griddep_wait();
   const int warp_global = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (warp_global >= B * Hq) return;
@@ -520,7 +523,9 @@ static umim_status run_attention(const void *q, int Hq, const umim_paged_kv *kv,
   const int Hkv = kv->n_kv_heads;
   AttnWs ws = attn_carve(workspace, B, Hkv, D, total_warps);
   trace_mark(stream, "attention.plan");
-  attn_plan_kernel<<<1, kPlanThreadsA, 0, stream>>>(seq_lens, B, Hkv, max_pages, total_warps, ws, status);
+  if (launch_pdl(attn_plan_kernel, dim3(1), dim3(kPlanThreadsA), 0, stream, seq_lens, B, Hkv, max_pages,
+                 total_warps, ws, status) != cudaSuccess)
+    return UMIM_ERR_CUDA;
 
   AttnArgs a{};
   a.q = static_cast<const __nv_bfloat16 *>(q);
@@ -541,12 +546,15 @@ static umim_status run_attention(const void *q, int Hq, const umim_paged_kv *kv,
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
     return UMIM_ERR_CUDA;
   trace_mark(stream, "attention.decode");
-  kern<<<total_warps / kAttnWarps, kAttnWarps * 32, smem, stream>>>(map, a, ws);
+  if (launch_pdl(kern, dim3(total_warps / kAttnWarps), dim3(kAttnWarps * 32), smem, stream, map, a, ws) !=
+      cudaSuccess)
+    return UMIM_ERR_CUDA;
   trace_mark(stream, "attention.combine");
   const int threads = 256;
   const int nwarps = B * Hq;
-  attn_combine_kernel<D><<<(nwarps * 32 + threads - 1) / threads, threads, 0, stream>>>(
-      ws, B, Hq, Hkv, a.G, static_cast<__nv_bfloat16 *>(out));
+  if (launch_pdl(attn_combine_kernel<D>, dim3((nwarps * 32 + threads - 1) / threads), dim3(threads), 0, stream, ws,
+                 B, Hq, Hkv, a.G, static_cast<__nv_bfloat16 *>(out)) != cudaSuccess)
+    return UMIM_ERR_CUDA;
   trace_mark(stream, nullptr);
   return cudaGetLastError() == cudaSuccess ? UMIM_OK : UMIM_ERR_CUDA;
 }

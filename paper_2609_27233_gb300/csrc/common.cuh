@@ -230,6 +230,29 @@ __device__ __forceinline__ float gelu_erf(float x) {
 
 __host__ __device__ __forceinline__ int ceil_div(int a, int b) { return (a + b - 1) / b; }
 
+// Programmatic dependent launch: a kernel launched with launch_pdl may start
+// while the previous kernel of the stream is finishing; griddep_wait() blocks
+// until that kernel has completed and its writes are visible.  Every kernel
+// calls it before its first access to memory another kernel may have written
+// (it is a no-op for a kernel launched the ordinary way).
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
+                              Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+}
+
 // Kernel tracing (trace.cu): records an event labelled with the next kernel,
 // or, with a null label, the end of a call.  No-op unless a trace is active.
 void trace_mark(cudaStream_t stream, const char *label);

@@ -36,6 +36,7 @@ __device__ __forceinline__ int last_le(const int32_t *key, int lo, int hi, int x
 }
 
 __global__ void __launch_bounds__(256) compact_kernel(CompactArgs a, PlanArrays arr) {
+  griddep_wait();
   const PlanHeader *hdr = arr.hdr;
   if (hdr->skip) return;
   const int total = hdr->total_rows;
@@ -119,9 +120,9 @@ umim_status build_compressed(const void *embeddings, int64_t vocab, int d, const
   const int64_t rows = (int64_t)B * L;
   const int blocks = (int)std::max<int64_t>(1, std::min<int64_t>((rows + 7) / 8, (int64_t)num_sms * 16));
   trace_mark(stream, "compact.rows");
-  compact_kernel<<<blocks, 256, 0, stream>>>(a, arr);
+  if (launch_pdl(compact_kernel, dim3(blocks), dim3(256), 0, stream, a, arr) != cudaSuccess) return UMIM_ERR_CUDA;
   trace_mark(stream, nullptr);
-  return cudaGetLastError() == cudaSuccess ? UMIM_OK : UMIM_ERR_CUDA;
+  return UMIM_OK;
 }
 
 }  // namespace umim

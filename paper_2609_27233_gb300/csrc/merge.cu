@@ -103,6 +103,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = tmem_base;
+  griddep_wait();
 
   if (warp == 0) {
     if (lane == 0) {
@@ -226,6 +227,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 // ---------------------------------------------------------------------------
 __global__ void gather_rows_kernel(const uint4 *table, int64_t vocab, const int32_t *ids, int64_t T, int d,
                                    uint4 *out, int32_t *status) {
+  griddep_wait();
   const int vec = d / 8;   // 16-byte vectors per row
   const int64_t warp = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const int64_t nwarps = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
@@ -337,6 +339,7 @@ __global__ void __launch_bounds__(kPoolConsumers + 32, CH <= 2 ? 2 : 1)
     s_B[tid] = 0.f;
   }
   __syncthreads();
+  griddep_wait();
 
   if (warp == kPoolConsumers / 32) {
     // ---- producer ----
@@ -554,6 +557,7 @@ __global__ void __launch_bounds__(256)
 
 // W_o from bf16 to fp16 (exact for values in fp16's normal range)
 __global__ void bf16_to_f16_kernel(const uint4 *in, uint4 *out, int64_t n_vec) {
+  griddep_wait();
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n_vec; i += (int64_t)gridDim.x * blockDim.x) {
     const uint4 u = in[i];
     float f[8];
@@ -627,8 +631,10 @@ static umim_status launch_gemm(EncodeTiledFn enc, const void *A, int64_t M, cons
   const int64_t tiles = (int64_t)(d / BN) * ((M + BM - 1) / BM);
   const int grid = (int)std::min<int64_t>(tiles, std::max(1, num_sms));
   trace_mark(st, label);
-  gemm_bias_gelu_kernel<OutT><<<grid, kGemmThreads, kGemmSmem, st>>>(am, bm, g);
-  return cudaGetLastError() == cudaSuccess ? UMIM_OK : UMIM_ERR_CUDA;
+  return launch_pdl(gemm_bias_gelu_kernel<OutT>, dim3(grid), dim3(kGemmThreads), kGemmSmem, st, am, bm, g) ==
+                 cudaSuccess
+             ? UMIM_OK
+             : UMIM_ERR_CUDA;
 }
 
 umim_status merge_spans(const void *embeddings, int64_t vocab, const int32_t *token_ids, int64_t T,
@@ -654,8 +660,9 @@ umim_status merge_spans(const void *embeddings, int64_t vocab, const int32_t *to
   if (T > 0) {
     const int blocks = std::max(1, std::min<int>((int)((T + 7) / 8), num_sms * 8));
     trace_mark(st, "merge.gather");
-    gather_rows_kernel<<<blocks, 256, 0, st>>>(static_cast<const uint4 *>(embeddings), vocab, token_ids, T, d,
-                                               reinterpret_cast<uint4 *>(E), status);
+    if (launch_pdl(gather_rows_kernel, dim3(blocks), dim3(256), 0, st, static_cast<const uint4 *>(embeddings), vocab,
+                   token_ids, T, d, reinterpret_cast<uint4 *>(E), status) != cudaSuccess)
+      return UMIM_ERR_CUDA;
     umim_status r = launch_gemm(enc, E, T, w->w_kv, d, false, w->b_kv, H, st1, status, st, "merge.gemm1", num_sms);
     if (r != UMIM_OK) return r;
   }
@@ -670,20 +677,25 @@ umim_status merge_spans(const void *embeddings, int64_t vocab, const int32_t *to
       pool_per_sm < 1)
     pool_per_sm = 1;
   const int pool_grid = std::max(1, std::min(S, std::max(1, num_sms) * pool_per_sm));
-  pk<<<pool_grid, kPoolConsumers + 32, psmem, st>>>(H, st1, span_offsets, S, T, d, w->n_heads,
-                                          static_cast<const __nv_bfloat16 *>(w->ln_kv_gamma),
-                                          static_cast<const __nv_bfloat16 *>(w->ln_kv_beta),
-                                          static_cast<const __nv_bfloat16 *>(w->query), w->ln_eps, O, status);
+  if (launch_pdl(pk, dim3(pool_grid), dim3(kPoolConsumers + 32), psmem, st, (const __half *)H, (const float2 *)st1,
+                 span_offsets, S, T, d, (int)w->n_heads, static_cast<const __nv_bfloat16 *>(w->ln_kv_gamma),
+                 static_cast<const __nv_bfloat16 *>(w->ln_kv_beta), static_cast<const __nv_bfloat16 *>(w->query),
+                 w->ln_eps, O, status) != cudaSuccess)
+    return UMIM_ERR_CUDA;
   trace_mark(st, "merge.wo_f16");
-  bf16_to_f16_kernel<<<std::max(1, num_sms) * 4, 256, 0, st>>>(static_cast<const uint4 *>(w->w_o), reinterpret_cast<uint4 *>(Wo16),
-                                                  (int64_t)d * d / 8);
+  if (launch_pdl(bf16_to_f16_kernel, dim3(std::max(1, num_sms) * 4), dim3(256), 0, st,
+                 static_cast<const uint4 *>(w->w_o), reinterpret_cast<uint4 *>(Wo16), (int64_t)d * d / 8) !=
+      cudaSuccess)
+    return UMIM_ERR_CUDA;
   umim_status r = launch_gemm(enc, O, S, Wo16, d, true, w->b_o, surrogates, st2, status, st, "merge.gemm2", num_sms);
   if (r != UMIM_OK) return r;
   trace_mark(st, "merge.ln_o");
-  ln_rows_kernel<<<(S + 7) / 8, 256, 0, st>>>(surrogates, st2, S, d, static_cast<const __nv_bfloat16 *>(w->ln_o_gamma),
-                                    static_cast<const __nv_bfloat16 *>(w->ln_o_beta), w->ln_eps);
+  if (launch_pdl(ln_rows_kernel, dim3((S + 7) / 8), dim3(256), 0, st, surrogates, (const float2 *)st2, S, d,
+                 static_cast<const __nv_bfloat16 *>(w->ln_o_gamma), static_cast<const __nv_bfloat16 *>(w->ln_o_beta),
+                 w->ln_eps) != cudaSuccess)
+    return UMIM_ERR_CUDA;
   trace_mark(st, nullptr);
-  return cudaGetLastError() == cudaSuccess ? UMIM_OK : UMIM_ERR_CUDA;
+  return UMIM_OK;
 }
 
 }  // namespace umim

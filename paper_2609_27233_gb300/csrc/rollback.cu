@@ -78,70 +78,35 @@ struct PageDesc {
   int2 *dep;       // [pages] range of compacted pages that read this old page
 };
 
-// One warp per (sequence, compacted page): where each of its 16 entries comes
-// from, and which compacted pages read the same page of the old layout.
-__global__ void __launch_bounds__(256) rollback_map_kernel(MoveArgs a, PlanArrays arr, PageDesc pd, int D) {
-  if (arr.hdr->skip) return;
-  const int b = blockIdx.y;
-  const int k = blockIdx.x * 8 + (threadIdx.x >> 5);
-  const int lane = threadIdx.x & 31;
-  const int nd = arr.n_dest[b];
-  if (k >= nd) return;
-  const int p = arr.first_page[b] + k;
-  const int idx = arr.unit_base[b] / a.n_lanes + k;
-  const int lo = a.span_offsets[b], hi = a.span_offsets[b + 1];
-  const int32_t *bt = a.block_table + (int64_t)b * a.max_pages;
-  const int64_t page_stride = (int64_t)kPageSize * D * a.n_kv_heads * 2;
-  int dpage = -1;
-  if (lane < kPageSize) {
-    const int L = arr.seq_Lp[b];
-    const int j = p * kPageSize + lane;
-    int64_t src = kNoWrite;
-    if (j < L && j >= a.span_start[lo]) {
-      const int i = upper_index(arr.new_idx, lo, hi, j);
-      if (i >= lo) {
-        if (arr.new_idx[i] == j) {
-          src = -(int64_t)i - 1;
-        } else {
-          const int t = j + arr.r_incl[i];
-          if (t != j) src = (int64_t)bt[t / kPageSize] * page_stride + (t % kPageSize) * D;
-        }
-      }
-    }
-    pd.src[(int64_t)idx * kPageSize + lane] = src;
-  } else {
-    const int L = arr.seq_L[b];
-    const int t = p * kPageSize + (lane - kPageSize);
-    if (t < L) {
-      const int i = upper_index(a.span_start, lo, hi, t);
-      if (i >= lo && t >= a.span_start[i] + a.span_len[i]) {
-        const int r = arr.r_incl[i];
-        if (r > 0) dpage = (t - r) / kPageSize;
-      }
-    }
-  }
-  int mn = dpage < 0 ? 0x7fffffff : dpage, mx = dpage;
-#pragma unroll
-  for (int o = 8; o >= 1; o >>= 1) {
-    mn = min(mn, __shfl_xor_sync(0xffffffffu, mn, o));
-    mx = max(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-  }
-  if (lane == kPageSize) pd.dep[idx] = make_int2(mn, mx);
+__device__ __forceinline__ void cp_async_16(uint32_t smem, const void *gmem) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem), "l"(gmem) : "memory");
 }
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_1() { asm volatile("cp.async.wait_group 1;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_0() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
 
-// One warp per unit = one (layer, K|V, head) 16 x D tile of a compacted
-// page.  Lane l moves 16-byte chunks c = l + 32 it of the tile: row c / CPR
-// (the slot), column c % CPR.
+constexpr int kMoveWarps = kMoveThreads / 32;
+
+// One warp per unit = one (layer, K|V, head) 16 x D tile of a compacted page.
+// Lane l moves 16-byte chunks c = l + 32 it of the tile: row c / CPR (the
+// slot), column c % CPR.  Each warp runs a two-deep pipeline over its units
+// (gw, gw + warps, ...): the copies of unit i+1 into one half of the warp's
+// shared buffer are in flight while unit i is published, its dependencies
+// are checked and it is written out from the other half.  The release that
+// publishes unit i therefore only orders stores issued one iteration ago.
 template <int D>
-__global__ void __launch_bounds__(kMoveThreads, 4) rollback_move_kernel(MoveArgs a, PlanArrays arr, PageDesc pd) {
+__global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a, PlanArrays arr, PageDesc pd) {
   constexpr int CPR = D / 8;                       // 16-byte chunks per row
   constexpr int PER_LANE = kPageSize * CPR / 32;   // 8 (D=128) or 4 (D=64)
   constexpr int SLOT_STEP = 32 / CPR;              // slots advanced per it
-  const int lane = threadIdx.x & 31;
-  const int gw = blockIdx.x * (kMoveThreads / 32) + (threadIdx.x >> 5);
-  const int nw = gridDim.x * (kMoveThreads / 32);
+  constexpr int TILE_BYTES = kPageSize * D * 2;
+  extern __shared__ __align__(16) uint8_t move_smem[];
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  const int gw = blockIdx.x * kMoveWarps + wid;
+  const int nw = gridDim.x * kMoveWarps;
   const int my_col = lane % CPR;
   const int my_slot0 = lane / CPR;
+  const uint32_t wbuf = smem_u32(move_smem + wid * 2 * TILE_BYTES);
   __shared__ int s_last;
 
   const PlanHeader *hdr = arr.hdr;
@@ -152,10 +117,22 @@ __global__ void __launch_bounds__(kMoveThreads, 4) rollback_move_kernel(MoveArgs
   const int64_t kv_stride = head_stride * Hkv;
   const int64_t page_stride = kv_stride * 2;
   const int64_t layer_stride = page_stride * a.n_pages;
-  bool abort = false;
 
-  for (int u = gw; u < total && !abort; u += nw) {
-    // unit -> (sequence, tile lane, compacted page)
+  struct Unit {
+    int u, b, p;
+    int2 dep;
+    int64_t tile;       // element offset of the tile (layer, kv, head) within a page, plus this lane's column
+    uint32_t mask;      // which of this lane's chunks are written
+  };
+  // describe unit u and start its copies into buffer half `half`
+  auto start = [&](int u, int half) {
+    Unit U;
+    U.u = u;
+    U.mask = 0;
+    if (u >= total) {
+      cp_async_commit();
+      return U;
+    }
     const int b = find_seq(arr.unit_base, a.B, u);
     const int rem = u - arr.unit_base[b];
     const int nd = arr.n_dest[b];
@@ -163,40 +140,47 @@ __global__ void __launch_bounds__(kMoveThreads, 4) rollback_move_kernel(MoveArgs
     const int layer = tl / (2 * Hkv);
     const int kv = (tl / Hkv) & 1;
     const int h = tl % Hkv;
-    const int idx = arr.unit_base[b] / a.n_lanes + k;
-    const int p = arr.first_page[b] + k;
-    const int64_t my_src = lane < kPageSize ? pd.src[(int64_t)idx * kPageSize + lane] : kNoWrite;
-    const int2 dep = pd.dep[idx];
-    const int64_t tile = layer * layer_stride + kv * kv_stride + h * head_stride + my_col * 8;
+    const int64_t idx = (int64_t)b * a.max_pages + k;
+    U.b = b;
+    U.p = arr.first_page[b] + k;
+    U.dep = pd.dep[idx];
+    U.tile = layer * layer_stride + kv * kv_stride + h * head_stride + my_col * 8;
+    const int64_t my_src = lane < kPageSize ? pd.src[idx * kPageSize + lane] : kNoWrite;
     const uint16_t *sur = kv ? a.sur_v : a.sur_k;
-
-    uint4 v[PER_LANE];
-    uint32_t write_mask = 0;
-    uint32_t fold = 0;
+    const uint32_t dst = wbuf + half * TILE_BYTES;
 #pragma unroll
     for (int it = 0; it < PER_LANE; ++it) {
       const int slot = my_slot0 + it * SLOT_STEP;
       const int64_t src = __shfl_sync(0xffffffffu, my_src, slot);
-      if (src != kNoWrite) write_mask |= 1u << it;
-      v[it] = make_uint4(0, 0, 0, 0);
+      if (src == kNoWrite) continue;
+      U.mask |= 1u << it;
+      const uint16_t *g;
       if (src >= 0) {
-        v[it] = ld_v4(a.pool + tile + src);
-      } else if (src != kNoWrite) {
+        g = a.pool + U.tile + src;
+      } else {
         const int64_t i = -src - 1;
-        v[it] = ld_v4(sur + ((i * a.n_layers + layer) * Hkv + h) * D + my_col * 8);
+        g = sur + ((i * a.n_layers + layer) * Hkv + h) * D + my_col * 8;
       }
-      fold ^= v[it].x ^ v[it].y ^ v[it].z ^ v[it].w;
+      cp_async_16(dst + (lane + it * 32) * 16, g);
     }
-    // every loaded value of this lane has arrived before the warp barrier
-    asm volatile("" ::"r"(fold) : "memory");
-    __syncwarp();
+    cp_async_commit();
+    return U;
+  };
+
+  bool abort = false;
+  int half = 0;
+  Unit cur = start(gw, 0);
+  while (cur.u < total) {
+    const Unit nxt = start(cur.u + nw, half ^ 1);
+    cp_async_wait_1();     // this lane's copies of `cur` have landed
+    __syncwarp();          // ... and every other lane's
     int ok = 1;
     if (lane == 0) {
-      // release: the warp's loads are ordered before it by the warp barrier
-      st_release(&arr.flags[u], epoch);
+      // release: the copies of this unit are complete and ordered before it
+      st_release(&arr.flags[cur.u], epoch);
       // wait for the units that read this tile of old page p (smaller indices)
-      for (int q = dep.x; q <= dep.y && q >= 0 && q < p; ++q) {
-        const int uq = u - (p - q);
+      for (int q = cur.dep.x; q <= cur.dep.y && q >= 0 && q < cur.p; ++q) {
+        const int uq = cur.u - (cur.p - q);
         if (ld_acquire(&arr.flags[uq]) == epoch) continue;
         const uint64_t t0 = globaltimer();
         bool got = false;
@@ -217,13 +201,24 @@ __global__ void __launch_bounds__(kMoveThreads, 4) rollback_move_kernel(MoveArgs
       abort = true;
       break;
     }
-    const int64_t dst = tile + (int64_t)a.block_table[(int64_t)b * a.max_pages + p] * page_stride;
+    const int64_t dst = cur.tile + (int64_t)a.block_table[(int64_t)cur.b * a.max_pages + cur.p] * page_stride;
+    const uint32_t src_s = wbuf + half * TILE_BYTES;
 #pragma unroll
     for (int it = 0; it < PER_LANE; ++it) {
-      const int slot = my_slot0 + it * SLOT_STEP;
-      if (write_mask & (1u << it)) st_v4(a.pool + dst + slot * D, v[it]);
+      if (cur.mask & (1u << it)) {
+        uint4 v;
+        asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+                     : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                     : "r"(src_s + (lane + it * 32) * 16));
+        st_v4(a.pool + dst + (my_slot0 + it * SLOT_STEP) * D, v);
+      }
     }
+    __syncwarp();          // the buffer half is refilled two units later
+    cur = nxt;
+    half ^= 1;
   }
+  (void)abort;
+  cp_async_wait_0();
 
   // ---- the last CTA to finish truncates block tables and updates lengths ----
   const int tid = threadIdx.x;
@@ -297,6 +292,10 @@ umim_status kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t m
   pa.n_lanes = lanes;
   pa.status = status;
   pa.cu_seqlens_out = nullptr;
+  pa.page_src = pd.src;
+  pa.page_dep = pd.dep;
+  pa.page_stride = (int64_t)kPageSize * D * kv->n_kv_heads * 2;
+  pa.head_dim = D;
   trace_mark(stream, "rollback.plan");
   if (launch_span_plan(pa, arr, stream) != cudaSuccess) return UMIM_ERR_CUDA;
 
@@ -320,14 +319,13 @@ umim_status kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t m
   ma.B = B;
   ma.status = status;
   auto kern = (D == 128) ? rollback_move_kernel<128> : rollback_move_kernel<64>;
-  const int smem = 0;
+  const int smem = kMoveWarps * 2 * kPageSize * D * 2;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
+    return UMIM_ERR_CUDA;
   int per_sm = 0;
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kMoveThreads, smem) != cudaSuccess || per_sm < 1)
     per_sm = 1;
   const int grid = std::max(1, num_sms) * per_sm;   // every CTA resident (cooperative launch)
-  trace_mark(stream, "rollback.map");
-  rollback_map_kernel<<<dim3((unsigned)std::max(1, ceil_div(max_pages, 8)), (unsigned)B), 256, 0, stream>>>(ma, arr,
-                                                                                                         pd, D);
   trace_mark(stream, "rollback.move");
   void *args[] = {&ma, &arr, &pd};
   if (cudaLaunchCooperativeKernel(reinterpret_cast<const void *>(kern), dim3(grid), dim3(kMoveThreads), args,
