@@ -87,64 +87,6 @@ __global__ void __launch_bounds__(kPlanThreads) span_plan_kernel(PlanArgs a, Pla
     }
   }
   __syncthreads();
-  // rollback: describe every compacted page of this sequence (two 16-lane
-  // halves of a warp per page: sources of its entries, readers of the old page)
-  if (a.block_table && !s_err && hi > lo) {
-    const int Lp = L - s_carry;
-    const int fp = a.span_start[lo] / kPageSize;
-    const int nd = ceil_div(Lp, kPageSize) - fp;
-    const int32_t *bt = a.block_table + (int64_t)b * a.max_pages;
-    const int lane = threadIdx.x & 31;
-    for (int k = threadIdx.x >> 5; k < nd; k += kPlanThreads / 32) {
-      const int p = fp + k;
-      const int64_t idx = (int64_t)b * a.max_pages + k;
-      int dpage = -1;
-      if (lane < kPageSize) {
-        const int j = p * kPageSize + lane;
-        int64_t src = INT64_MIN;
-        if (j < Lp && j >= a.span_start[lo]) {
-          int l2 = lo, h2 = hi;   // last span whose compressed index <= j
-          while (l2 < h2) {
-            const int m = (l2 + h2) >> 1;
-            if (arr.new_idx[m] <= j) l2 = m + 1;
-            else h2 = m;
-          }
-          const int i = l2 - 1;
-          if (i >= lo) {
-            if (arr.new_idx[i] == j) {
-              src = -(int64_t)i - 1;
-            } else {
-              const int t = j + arr.r_incl[i];
-              if (t != j) src = (int64_t)bt[t / kPageSize] * a.page_stride + (t % kPageSize) * a.head_dim;
-            }
-          }
-        }
-        a.page_src[idx * kPageSize + lane] = src;
-      } else {
-        const int t = p * kPageSize + (lane - kPageSize);
-        if (t < L) {
-          int l2 = lo, h2 = hi;   // last span starting at or before t
-          while (l2 < h2) {
-            const int m = (l2 + h2) >> 1;
-            if (a.span_start[m] <= t) l2 = m + 1;
-            else h2 = m;
-          }
-          const int i = l2 - 1;
-          if (i >= lo && t >= a.span_start[i] + a.span_len[i]) {
-            const int r = arr.r_incl[i];
-            if (r > 0) dpage = (t - r) / kPageSize;
-          }
-        }
-      }
-      int mn = dpage < 0 ? 0x7fffffff : dpage, mx = dpage;
-#pragma unroll
-      for (int o = 8; o >= 1; o >>= 1) {
-        mn = min(mn, __shfl_xor_sync(0xffffffffu, mn, o));
-        mx = max(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-      }
-      if (lane == kPageSize) a.page_dep[idx] = make_int2(mn, mx);
-    }
-  }
   if (threadIdx.x == 0) {
     const int err = s_err;
     const int Lp = err ? L : L - s_carry;

@@ -93,14 +93,6 @@ struct PlanArgs {
   int32_t n_lanes;           // units per compacted page (layers x head groups)
   int32_t *status;           // resolved status word
   int32_t *cu_seqlens_out;   // compaction: [B+1] or nullptr
-  // rollback only: per (sequence, compacted page k), at index b * max_pages + k,
-  // the source of each of its 16 entries (row offset within a layer, no head
-  // offset; -(i+1) for the surrogate of span i; INT64_MIN for no write) and
-  // the range of compacted pages that read the same page of the old layout
-  int64_t *page_src;         // [B * max_pages][16]
-  int2 *page_dep;            // [B * max_pages]
-  int64_t page_stride;       // elements per page within a layer
-  int32_t head_dim;
 };
 
 // Launches the plan kernel (B blocks; the last block to finish does the

@@ -78,36 +78,95 @@ struct PageDesc {
   int2 *dep;       // [pages] range of compacted pages that read this old page
 };
 
-__device__ __forceinline__ void cp_async_16(uint32_t smem, const void *gmem) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem), "l"(gmem) : "memory");
+// One warp per (sequence, compacted page): where each of its 16 entries comes
+// from, and which compacted pages read the same page of the old layout.
+__global__ void __launch_bounds__(256) rollback_map_kernel(MoveArgs a, PlanArrays arr, PageDesc pd, int D) {
+  griddep_wait();
+  if (arr.hdr->skip) return;
+  const int b = blockIdx.y;
+  const int k = blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  const int nd = arr.n_dest[b];
+  if (k >= nd) return;
+  const int p = arr.first_page[b] + k;
+  const int idx = arr.unit_base[b] / a.n_lanes + k;
+  const int lo = a.span_offsets[b], hi = a.span_offsets[b + 1];
+  const int32_t *bt = a.block_table + (int64_t)b * a.max_pages;
+  const int64_t page_stride = (int64_t)kPageSize * D * a.n_kv_heads * 2;
+  int dpage = -1;
+  if (lane < kPageSize) {
+    const int L = arr.seq_Lp[b];
+    const int j = p * kPageSize + lane;
+    int64_t src = kNoWrite;
+    if (j < L && j >= a.span_start[lo]) {
+      const int i = upper_index(arr.new_idx, lo, hi, j);
+      if (i >= lo) {
+        if (arr.new_idx[i] == j) {
+          src = -(int64_t)i - 1;
+        } else {
+          const int t = j + arr.r_incl[i];
+          if (t != j) src = (int64_t)bt[t / kPageSize] * page_stride + (t % kPageSize) * D;
+        }
+      }
+    }
+    pd.src[(int64_t)idx * kPageSize + lane] = src;
+  } else {
+    const int L = arr.seq_L[b];
+    const int t = p * kPageSize + (lane - kPageSize);
+    if (t < L) {
+      const int i = upper_index(a.span_start, lo, hi, t);
+      if (i >= lo && t >= a.span_start[i] + a.span_len[i]) {
+        const int r = arr.r_incl[i];
+        if (r > 0) dpage = (t - r) / kPageSize;
+      }
+    }
+  }
+  int mn = dpage < 0 ? 0x7fffffff : dpage, mx = dpage;
+#pragma unroll
+  for (int o = 8; o >= 1; o >>= 1) {
+    mn = min(mn, __shfl_xor_sync(0xffffffffu, mn, o));
+    mx = max(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+  }
+  if (lane == kPageSize) pd.dep[idx] = make_int2(mn, mx);
 }
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-__device__ __forceinline__ void cp_async_wait_1() { asm volatile("cp.async.wait_group 1;" ::: "memory"); }
-__device__ __forceinline__ void cp_async_wait_0() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
 
-constexpr int kMoveWarps = kMoveThreads / 32;
+constexpr int kMovers = kMoveThreads / 32 - 1;   // mover warps per CTA; the last warp publishes
 
-// One warp per unit = one (layer, K|V, head) 16 x D tile of a compacted page.
-// Lane l moves 16-byte chunks c = l + 32 it of the tile: row c / CPR (the
-// slot), column c % CPR.  Each warp runs a two-deep pipeline over its units
-// (gw, gw + warps, ...): the copies of unit i+1 into one half of the warp's
-// shared buffer are in flight while unit i is published, its dependencies
-// are checked and it is written out from the other half.  The release that
-// publishes unit i therefore only orders stores issued one iteration ago.
+__device__ __forceinline__ void st_release_cta_shared(int *p, int v) {
+  asm volatile("st.release.cta.shared.b32 [%0], %1;" ::"r"(smem_u32(p)), "r"(v) : "memory");
+}
+__device__ __forceinline__ int ld_acquire_cta_shared(const int *p) {
+  int v;
+  asm volatile("ld.acquire.cta.shared.b32 %0, [%1];" : "=r"(v) : "r"(smem_u32(p)) : "memory");
+  return v;
+}
+__device__ __forceinline__ void fence_acq_rel_gpu() { asm volatile("fence.acq_rel.gpu;" ::: "memory"); }
+__device__ __forceinline__ void st_relaxed_gpu(int32_t *p, int32_t v) {
+  asm volatile("st.relaxed.gpu.global.b32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+// One mover warp per unit = one (layer, K|V, head) 16 x D tile of a compacted
+// page.  Lane l moves 16-byte chunks c = l + 32 it of the tile: row c / CPR
+// (the slot), column c % CPR.  Mover m of the grid handles units m, m + M,
+// m + 2M, ... (M movers).  When a unit's loads have returned, the mover
+// reports it in its shared-memory mailbox (CTA-scope release) and goes on to
+// wait for the units that read its destination page and to write it.  The
+// CTA's publisher warp collects reported units, issues one GPU-scope fence
+// for the whole batch and then marks their read-done flags: the fence orders
+// every reported load before every flag store that follows it, and movers
+// never pay for a GPU-scope fence themselves.
 template <int D>
-__global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a, PlanArrays arr, PageDesc pd) {
+__global__ void __launch_bounds__(kMoveThreads, 4) rollback_move_kernel(MoveArgs a, PlanArrays arr, PageDesc pd) {
   constexpr int CPR = D / 8;                       // 16-byte chunks per row
   constexpr int PER_LANE = kPageSize * CPR / 32;   // 8 (D=128) or 4 (D=64)
   constexpr int SLOT_STEP = 32 / CPR;              // slots advanced per it
-  constexpr int TILE_BYTES = kPageSize * D * 2;
-  extern __shared__ __align__(16) uint8_t move_smem[];
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-  const int gw = blockIdx.x * kMoveWarps + wid;
-  const int nw = gridDim.x * kMoveWarps;
+  const int nm = gridDim.x * kMovers;
   const int my_col = lane % CPR;
   const int my_slot0 = lane / CPR;
-  const uint32_t wbuf = smem_u32(move_smem + wid * 2 * TILE_BYTES);
   __shared__ int s_last;
+  __shared__ int s_mail[kMovers];   // units reported loaded by each mover (a count)
+  __shared__ int s_finished;        // movers that left their loop
 
   const PlanHeader *hdr = arr.hdr;
   const int total = hdr->total_units;
@@ -118,107 +177,121 @@ __global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a,
   const int64_t page_stride = kv_stride * 2;
   const int64_t layer_stride = page_stride * a.n_pages;
 
-  struct Unit {
-    int u, b, p;
-    int2 dep;
-    int64_t tile;       // element offset of the tile (layer, kv, head) within a page, plus this lane's column
-    uint32_t mask;      // which of this lane's chunks are written
-  };
-  // describe unit u and start its copies into buffer half `half`
-  auto start = [&](int u, int half) {
-    Unit U;
-    U.u = u;
-    U.mask = 0;
-    if (u >= total) {
-      cp_async_commit();
-      return U;
-    }
-    const int b = find_seq(arr.unit_base, a.B, u);
-    const int rem = u - arr.unit_base[b];
-    const int nd = arr.n_dest[b];
-    const int tl = rem / nd, k = rem % nd;
-    const int layer = tl / (2 * Hkv);
-    const int kv = (tl / Hkv) & 1;
-    const int h = tl % Hkv;
-    const int64_t idx = (int64_t)b * a.max_pages + k;
-    U.b = b;
-    U.p = arr.first_page[b] + k;
-    U.dep = pd.dep[idx];
-    U.tile = layer * layer_stride + kv * kv_stride + h * head_stride + my_col * 8;
-    const int64_t my_src = lane < kPageSize ? pd.src[idx * kPageSize + lane] : kNoWrite;
-    const uint16_t *sur = kv ? a.sur_v : a.sur_k;
-    const uint32_t dst = wbuf + half * TILE_BYTES;
-#pragma unroll
-    for (int it = 0; it < PER_LANE; ++it) {
-      const int slot = my_slot0 + it * SLOT_STEP;
-      const int64_t src = __shfl_sync(0xffffffffu, my_src, slot);
-      if (src == kNoWrite) continue;
-      U.mask |= 1u << it;
-      const uint16_t *g;
-      if (src >= 0) {
-        g = a.pool + U.tile + src;
-      } else {
-        const int64_t i = -src - 1;
-        g = sur + ((i * a.n_layers + layer) * Hkv + h) * D + my_col * 8;
-      }
-      cp_async_16(dst + (lane + it * 32) * 16, g);
-    }
-    cp_async_commit();
-    return U;
-  };
+  if (threadIdx.x < kMovers) s_mail[threadIdx.x] = 0;
+  if (threadIdx.x == 0) s_finished = 0;
+  __syncthreads();
 
-  bool abort = false;
-  int half = 0;
-  Unit cur = start(gw, 0);
-  while (cur.u < total) {
-    const Unit nxt = start(cur.u + nw, half ^ 1);
-    cp_async_wait_1();     // this lane's copies of `cur` have landed
-    __syncwarp();          // ... and every other lane's
-    int ok = 1;
-    if (lane == 0) {
-      // release: the copies of this unit are complete and ordered before it
-      st_release(&arr.flags[cur.u], epoch);
-      // wait for the units that read this tile of old page p (smaller indices)
-      for (int q = cur.dep.x; q <= cur.dep.y && q >= 0 && q < cur.p; ++q) {
-        const int uq = cur.u - (cur.p - q);
-        if (ld_acquire(&arr.flags[uq]) == epoch) continue;
-        const uint64_t t0 = globaltimer();
-        bool got = false;
-        while (!got) {
-#pragma unroll 1
-          for (int i = 0; i < 64 && !got; ++i) got = (ld_acquire(&arr.flags[uq]) == epoch);
-          if (!got && globaltimer() - t0 > kWaitLimitNs) break;
-        }
-        if (!got) {
-          set_error(a.status, UMIM_ERR_TIMEOUT);
-          ok = 0;
-          break;
-        }
-      }
-    }
-    ok = __shfl_sync(0xffffffffu, ok, 0);
-    if (!ok) {
-      abort = true;
-      break;
-    }
-    const int64_t dst = cur.tile + (int64_t)a.block_table[(int64_t)cur.b * a.max_pages + cur.p] * page_stride;
-    const uint32_t src_s = wbuf + half * TILE_BYTES;
+  if (wid == kMovers) {
+    // ---- publisher ----
+    int published[kMovers];
 #pragma unroll
-    for (int it = 0; it < PER_LANE; ++it) {
-      if (cur.mask & (1u << it)) {
-        uint4 v;
-        asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
-                     : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-                     : "r"(src_s + (lane + it * 32) * 16));
-        st_v4(a.pool + dst + (my_slot0 + it * SLOT_STEP) * D, v);
+    for (int m = 0; m < kMovers; ++m) published[m] = 0;
+    uint64_t t_idle = globaltimer();
+    while (true) {
+      int mail[kMovers];
+      bool any = false;
+      // finished before the mailboxes: a mover's last report precedes its exit
+      const int fin = ld_acquire_cta_shared(&s_finished);
+#pragma unroll
+      for (int m = 0; m < kMovers; ++m) {
+        mail[m] = ld_acquire_cta_shared(&s_mail[m]);
+        any |= mail[m] > published[m];
+      }
+      if (any) {
+        fence_acq_rel_gpu();   // every reported load happens before the flags below
+#pragma unroll
+        for (int m = 0; m < kMovers; ++m) {
+          const int mover = blockIdx.x * kMovers + m;
+          for (int k = published[m] + lane; k < mail[m]; k += 32) st_relaxed_gpu(&arr.flags[mover + k * nm], epoch);
+          published[m] = mail[m];
+        }
+        t_idle = globaltimer();
+      } else if (fin == kMovers) {
+        break;
+      } else if (globaltimer() - t_idle > kWaitLimitNs) {
+        set_error(a.status, UMIM_ERR_TIMEOUT);
+        break;
+      } else {
+        __nanosleep(32);
       }
     }
-    __syncwarp();          // the buffer half is refilled two units later
-    cur = nxt;
-    half ^= 1;
+  } else {
+    // ---- mover ----
+    const int mover = blockIdx.x * kMovers + wid;
+    int k = 0;
+    for (int u = mover; u < total; u += nm, ++k) {
+      // unit -> (sequence, tile lane, compacted page)
+      const int b = find_seq(arr.unit_base, a.B, u);
+      const int rem = u - arr.unit_base[b];
+      const int nd = arr.n_dest[b];
+      const int tl = rem / nd, kk = rem % nd;
+      const int layer = tl / (2 * Hkv);
+      const int kv = (tl / Hkv) & 1;
+      const int h = tl % Hkv;
+      const int idx = arr.unit_base[b] / a.n_lanes + kk;
+      const int p = arr.first_page[b] + kk;
+      const int64_t my_src = lane < kPageSize ? pd.src[(int64_t)idx * kPageSize + lane] : kNoWrite;
+      const int2 dep = pd.dep[idx];
+      const int64_t tile = layer * layer_stride + kv * kv_stride + h * head_stride + my_col * 8;
+      const uint16_t *sur = kv ? a.sur_v : a.sur_k;
+
+      uint4 v[PER_LANE];
+      uint32_t write_mask = 0;
+      uint32_t fold = 0;
+#pragma unroll
+      for (int it = 0; it < PER_LANE; ++it) {
+        const int slot = my_slot0 + it * SLOT_STEP;
+        const int64_t src = __shfl_sync(0xffffffffu, my_src, slot);
+        if (src != kNoWrite) write_mask |= 1u << it;
+        v[it] = make_uint4(0, 0, 0, 0);
+        if (src >= 0) {
+          v[it] = ld_v4(a.pool + tile + src);
+        } else if (src != kNoWrite) {
+          const int64_t i = -src - 1;
+          v[it] = ld_v4(sur + ((i * a.n_layers + layer) * Hkv + h) * D + my_col * 8);
+        }
+        fold ^= v[it].x ^ v[it].y ^ v[it].z ^ v[it].w;
+      }
+      // every loaded value of this lane has arrived before the warp barrier
+      asm volatile("" ::"r"(fold) : "memory");
+      __syncwarp();
+      int ok = 1;
+      if (lane == 0) {
+        // report: units 0 .. k of this mover have been read
+        st_release_cta_shared(&s_mail[wid], k + 1);
+        // wait for the units that read this tile of old page p (smaller indices)
+        for (int q = dep.x; q <= dep.y && q >= 0 && q < p; ++q) {
+          const int uq = u - (p - q);
+          if (ld_acquire(&arr.flags[uq]) == epoch) continue;
+          const uint64_t t0 = globaltimer();
+          bool got = false;
+          while (!got) {
+#pragma unroll 1
+            for (int i = 0; i < 64 && !got; ++i) got = (ld_acquire(&arr.flags[uq]) == epoch);
+            if (!got && globaltimer() - t0 > kWaitLimitNs) break;
+          }
+          if (!got) {
+            set_error(a.status, UMIM_ERR_TIMEOUT);
+            ok = 0;
+            break;
+          }
+        }
+      }
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) break;
+      const int64_t dst = tile + (int64_t)a.block_table[(int64_t)b * a.max_pages + p] * page_stride;
+#pragma unroll
+      for (int it = 0; it < PER_LANE; ++it) {
+        const int slot = my_slot0 + it * SLOT_STEP;
+        if (write_mask & (1u << it)) st_v4(a.pool + dst + slot * D, v[it]);
+      }
+    }
+    __syncwarp();
+    if (lane == 0) {
+      __threadfence_block();   // the last report is visible before the exit count
+      atomicAdd(&s_finished, 1);
+    }
   }
-  (void)abort;
-  cp_async_wait_0();
 
   // ---- the last CTA to finish truncates block tables and updates lengths ----
   const int tid = threadIdx.x;
@@ -292,10 +365,6 @@ umim_status kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t m
   pa.n_lanes = lanes;
   pa.status = status;
   pa.cu_seqlens_out = nullptr;
-  pa.page_src = pd.src;
-  pa.page_dep = pd.dep;
-  pa.page_stride = (int64_t)kPageSize * D * kv->n_kv_heads * 2;
-  pa.head_dim = D;
   trace_mark(stream, "rollback.plan");
   if (launch_span_plan(pa, arr, stream) != cudaSuccess) return UMIM_ERR_CUDA;
 
@@ -319,13 +388,15 @@ umim_status kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t m
   ma.B = B;
   ma.status = status;
   auto kern = (D == 128) ? rollback_move_kernel<128> : rollback_move_kernel<64>;
-  const int smem = kMoveWarps * 2 * kPageSize * D * 2;
-  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
-    return UMIM_ERR_CUDA;
+  const int smem = 0;
   int per_sm = 0;
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kMoveThreads, smem) != cudaSuccess || per_sm < 1)
     per_sm = 1;
   const int grid = std::max(1, num_sms) * per_sm;   // every CTA resident (cooperative launch)
+  trace_mark(stream, "rollback.map");
+  if (launch_pdl(rollback_map_kernel, dim3((unsigned)std::max(1, ceil_div(max_pages, 8)), (unsigned)B), dim3(256), 0,
+                 stream, ma, arr, pd, (int)D) != cudaSuccess)
+    return UMIM_ERR_CUDA;
   trace_mark(stream, "rollback.move");
   void *args[] = {&ma, &arr, &pd};
   if (cudaLaunchCooperativeKernel(reinterpret_cast<const void *>(kern), dim3(grid), dim3(kMoveThreads), args,
