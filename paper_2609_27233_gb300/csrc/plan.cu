@@ -111,6 +111,10 @@ __global__ void __launch_bounds__(kPlanThreads) span_plan_kernel(PlanArgs a, Pla
   __threadfence();
   const int err = atomicOr(&arr.hdr->error, 0);
   int cu_units = 0, cu_rows = 0, cu_freed = 0;
+  __shared__ int s_max_dest;
+  if (threadIdx.x == 0) s_max_dest = 0;
+  __syncthreads();
+  for (int j = threadIdx.x; j < a.B; j += kPlanThreads) atomicMax(&s_max_dest, arr.n_dest[j]);
   for (int base = 0; base < a.B; base += kPlanThreads) {
     const int j = base + threadIdx.x;
     int u = 0, r = 0, f = 0;
@@ -142,6 +146,7 @@ __global__ void __launch_bounds__(kPlanThreads) span_plan_kernel(PlanArgs a, Pla
     PlanHeader *h = arr.hdr;
     h->total_units = err ? 0 : cu_units;
     h->total_rows = cu_rows;
+    h->max_dest = err ? 0 : s_max_dest;
     h->skip = err ? 1 : 0;
     h->epoch = h->epoch + 1;
     h->ticket = 0;

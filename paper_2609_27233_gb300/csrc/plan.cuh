@@ -25,7 +25,8 @@ struct PlanHeader {
   int32_t error;        // OR of plan errors this call
   int32_t skip;         // 1: the call found invalid input, write nothing
   int32_t total_rows;   // sum of compressed lengths
-  int32_t pad[55];      // header is 256 bytes
+  int32_t max_dest;     // largest number of compacted pages of one sequence
+  int32_t pad[54];      // header is 256 bytes
 };
 static_assert(sizeof(PlanHeader) == 256, "header size");
 

@@ -147,8 +147,12 @@ __device__ __forceinline__ void st_relaxed_gpu(int32_t *p, int32_t v) {
 
 // One mover warp per unit = one (layer, K|V, head) 16 x D tile of a compacted
 // page.  Lane l moves 16-byte chunks c = l + 32 it of the tile: row c / CPR
-// (the slot), column c % CPR.  Mover m of the grid handles units m, m + M,
-// m + 2M, ... (M movers).  When a unit's loads have returned, the mover
+// (the slot), column c % CPR.  Units are visited page-row by page-row:
+// processing slot i covers compacted page k = i / (B * tiles) of sequence b
+// and tile t, (b, t) = divmod(i mod (B * tiles), tiles); slots with k beyond
+// the sequence's pages do nothing.  A unit waits only for units of earlier
+// rows, which were picked up at least a whole row of slots before it.  Mover m
+// of the grid handles slots m, m + M, m + 2M, ... (M movers).  When a unit's loads have returned, the mover
 // reports it in its shared-memory mailbox (CTA-scope release) and goes on to
 // wait for the units that read its destination page and to write it.  The
 // CTA's publisher warp collects reported units, issues one GPU-scope fence
@@ -176,6 +180,8 @@ __global__ void __launch_bounds__(kMoveThreads, 4) rollback_move_kernel(MoveArgs
   const int64_t kv_stride = head_stride * Hkv;
   const int64_t page_stride = kv_stride * 2;
   const int64_t layer_stride = page_stride * a.n_pages;
+  const int row_size = a.B * a.n_lanes;
+  const int64_t n_slots = total > 0 ? (int64_t)hdr->max_dest * row_size : 0;
 
   if (threadIdx.x < kMovers) s_mail[threadIdx.x] = 0;
   if (threadIdx.x == 0) s_finished = 0;
@@ -202,7 +208,14 @@ __global__ void __launch_bounds__(kMoveThreads, 4) rollback_move_kernel(MoveArgs
 #pragma unroll
         for (int m = 0; m < kMovers; ++m) {
           const int mover = blockIdx.x * kMovers + m;
-          for (int k = published[m] + lane; k < mail[m]; k += 32) st_relaxed_gpu(&arr.flags[mover + k * nm], epoch);
+          for (int k = published[m] + lane; k < mail[m]; k += 32) {
+            const int64_t i = mover + (int64_t)k * nm;
+            const int kk = (int)(i / row_size);
+            const int pos = (int)(i - (int64_t)kk * row_size);
+            const int b = pos / a.n_lanes, tl = pos % a.n_lanes;
+            const int nd = arr.n_dest[b];
+            if (kk < nd) st_relaxed_gpu(&arr.flags[arr.unit_base[b] + tl * nd + kk], epoch);
+          }
           published[m] = mail[m];
         }
         t_idle = globaltimer();
@@ -219,12 +232,17 @@ __global__ void __launch_bounds__(kMoveThreads, 4) rollback_move_kernel(MoveArgs
     // ---- mover ----
     const int mover = blockIdx.x * kMovers + wid;
     int k = 0;
-    for (int u = mover; u < total; u += nm, ++k) {
-      // unit -> (sequence, tile lane, compacted page)
-      const int b = find_seq(arr.unit_base, a.B, u);
-      const int rem = u - arr.unit_base[b];
+    for (int64_t i = mover; i < n_slots; i += nm, ++k) {
+      // slot -> (compacted page row kk, sequence, tile lane)
+      const int kk = (int)(i / row_size);
+      const int pos = (int)(i - (int64_t)kk * row_size);
+      const int b = pos / a.n_lanes, tl = pos % a.n_lanes;
       const int nd = arr.n_dest[b];
-      const int tl = rem / nd, kk = rem % nd;
+      if (kk >= nd) {
+        if (lane == 0) st_release_cta_shared(&s_mail[wid], k + 1);
+        continue;
+      }
+      const int u = arr.unit_base[b] + tl * nd + kk;
       const int layer = tl / (2 * Hkv);
       const int kv = (tl / Hkv) & 1;
       const int h = tl % Hkv;
