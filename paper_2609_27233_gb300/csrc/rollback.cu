@@ -132,6 +132,13 @@ __global__ void __launch_bounds__(256) rollback_map_kernel(MoveArgs a, PlanArray
 
 constexpr int kMovers = kMoveThreads / 32 - 1;   // mover warps per CTA; the last warp publishes
 
+__device__ __forceinline__ void cp_async_16(uint32_t smem, const void *gmem) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem), "l"(gmem) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_1() { asm volatile("cp.async.wait_group 1;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_0() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
+
 __device__ __forceinline__ void st_release_cta_shared(int *p, int v) {
   asm volatile("st.release.cta.shared.b32 [%0], %1;" ::"r"(smem_u32(p)), "r"(v) : "memory");
 }
@@ -160,10 +167,11 @@ __device__ __forceinline__ void st_relaxed_gpu(int32_t *p, int32_t v) {
 // every reported load before every flag store that follows it, and movers
 // never pay for a GPU-scope fence themselves.
 template <int D>
-__global__ void __launch_bounds__(kMoveThreads, 4) rollback_move_kernel(MoveArgs a, PlanArrays arr, PageDesc pd) {
+__global__ void __launch_bounds__(kMoveThreads, 3) rollback_move_kernel(MoveArgs a, PlanArrays arr, PageDesc pd) {
   constexpr int CPR = D / 8;                       // 16-byte chunks per row
   constexpr int PER_LANE = kPageSize * CPR / 32;   // 8 (D=128) or 4 (D=64)
   constexpr int SLOT_STEP = 32 / CPR;              // slots advanced per it
+  extern __shared__ __align__(16) uint8_t move_smem[];
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
   const int nm = gridDim.x * kMovers;
   const int my_col = lane % CPR;
@@ -230,80 +238,114 @@ __global__ void __launch_bounds__(kMoveThreads, 4) rollback_move_kernel(MoveArgs
     }
   } else {
     // ---- mover ----
-    const int mover = blockIdx.x * kMovers + wid;
-    int k = 0;
-    for (int64_t i = mover; i < n_slots; i += nm, ++k) {
-      // slot -> (compacted page row kk, sequence, tile lane)
-      const int kk = (int)(i / row_size);
-      const int pos = (int)(i - (int64_t)kk * row_size);
-      const int b = pos / a.n_lanes, tl = pos % a.n_lanes;
-      const int nd = arr.n_dest[b];
-      if (kk >= nd) {
-        if (lane == 0) st_release_cta_shared(&s_mail[wid], k + 1);
-        continue;
-      }
-      const int u = arr.unit_base[b] + tl * nd + kk;
-      const int layer = tl / (2 * Hkv);
-      const int kv = (tl / Hkv) & 1;
-      const int h = tl % Hkv;
-      const int idx = arr.unit_base[b] / a.n_lanes + kk;
-      const int p = arr.first_page[b] + kk;
-      const int64_t my_src = lane < kPageSize ? pd.src[(int64_t)idx * kPageSize + lane] : kNoWrite;
-      const int2 dep = pd.dep[idx];
-      const int64_t tile = layer * layer_stride + kv * kv_stride + h * head_stride + my_col * 8;
-      const uint16_t *sur = kv ? a.sur_v : a.sur_k;
-
-      uint4 v[PER_LANE];
-      uint32_t write_mask = 0;
-      uint32_t fold = 0;
+    // Two halves of a per-mover shared buffer: the copies of the next slot
+    // land in one half while the current slot is reported, waited for and
+    // written out from the other.
+    constexpr int TILE_BYTES = kPageSize * D * 2;
+    const uint32_t mbuf = smem_u32(move_smem + wid * 2 * TILE_BYTES);
+    struct Slot {
+      int u, layer, kv, h, p, dst_page;
+      int2 dep;
+      uint32_t mask;   // this lane's chunks that are written
+      bool work;
+    };
+    auto start = [&](int64_t i, int half) {
+      Slot d;
+      d.work = false;
+      d.mask = 0;
+      if (i < n_slots) {
+        const int kk = (int)(i / row_size);
+        const int pos = (int)(i - (int64_t)kk * row_size);
+        const int b = pos / a.n_lanes, tl = pos % a.n_lanes;
+        const int nd = arr.n_dest[b];
+        if (kk < nd) {
+          const int ub = arr.unit_base[b];
+          d.work = true;
+          d.u = ub + tl * nd + kk;
+          d.layer = tl / (2 * Hkv);
+          d.kv = (tl / Hkv) & 1;
+          d.h = tl % Hkv;
+          d.p = arr.first_page[b] + kk;
+          const int64_t idx = ub / a.n_lanes + kk;
+          const int64_t my_src = lane < kPageSize ? pd.src[idx * kPageSize + lane] : kNoWrite;
+          d.dep = pd.dep[idx];
+          d.dst_page = a.block_table[(int64_t)b * a.max_pages + d.p];
+          const int64_t tile = d.layer * layer_stride + d.kv * kv_stride + d.h * head_stride + my_col * 8;
+          const uint16_t *sur = d.kv ? a.sur_v : a.sur_k;
+          const uint32_t dst = mbuf + half * TILE_BYTES;
 #pragma unroll
-      for (int it = 0; it < PER_LANE; ++it) {
-        const int slot = my_slot0 + it * SLOT_STEP;
-        const int64_t src = __shfl_sync(0xffffffffu, my_src, slot);
-        if (src != kNoWrite) write_mask |= 1u << it;
-        v[it] = make_uint4(0, 0, 0, 0);
-        if (src >= 0) {
-          v[it] = ld_v4(a.pool + tile + src);
-        } else if (src != kNoWrite) {
-          const int64_t i = -src - 1;
-          v[it] = ld_v4(sur + ((i * a.n_layers + layer) * Hkv + h) * D + my_col * 8);
+          for (int it = 0; it < PER_LANE; ++it) {
+            const int slot = my_slot0 + it * SLOT_STEP;
+            const int64_t src = __shfl_sync(0xffffffffu, my_src, slot);
+            if (src == kNoWrite) continue;
+            d.mask |= 1u << it;
+            const uint16_t *g;
+            if (src >= 0) {
+              g = a.pool + tile + src;
+            } else {
+              const int64_t si = -src - 1;
+              g = sur + ((si * a.n_layers + d.layer) * Hkv + d.h) * D + my_col * 8;
+            }
+            cp_async_16(dst + (lane + it * 32) * 16, g);
+          }
         }
-        fold ^= v[it].x ^ v[it].y ^ v[it].z ^ v[it].w;
       }
-      // every loaded value of this lane has arrived before the warp barrier
-      asm volatile("" ::"r"(fold) : "memory");
-      __syncwarp();
+      cp_async_commit();   // one group per slot, empty or not
+      return d;
+    };
+    const int mover = blockIdx.x * kMovers + wid;
+    int k = 0, half = 0;
+    Slot cur = start(mover, 0);
+    for (int64_t i = mover; i < n_slots; i += nm, ++k) {
+      const Slot nxt = start(i + nm, half ^ 1);
+      cp_async_wait_1();      // this lane's copies of the current slot have landed
+      __syncwarp();           // ... and every other lane's
       int ok = 1;
       if (lane == 0) {
-        // report: units 0 .. k of this mover have been read
+        // report: slots 0 .. k of this mover have been read
         st_release_cta_shared(&s_mail[wid], k + 1);
-        // wait for the units that read this tile of old page p (smaller indices)
-        for (int q = dep.x; q <= dep.y && q >= 0 && q < p; ++q) {
-          const int uq = u - (p - q);
-          if (ld_acquire(&arr.flags[uq]) == epoch) continue;
-          const uint64_t t0 = globaltimer();
-          bool got = false;
-          while (!got) {
+        // wait for the units that read this tile of old page p (earlier rows)
+        if (cur.work) {
+          for (int q = cur.dep.x; q <= cur.dep.y && q >= 0 && q < cur.p; ++q) {
+            const int uq = cur.u - (cur.p - q);
+            if (ld_acquire(&arr.flags[uq]) == epoch) continue;
+            const uint64_t t0 = globaltimer();
+            bool got = false;
+            while (!got) {
 #pragma unroll 1
-            for (int i = 0; i < 64 && !got; ++i) got = (ld_acquire(&arr.flags[uq]) == epoch);
-            if (!got && globaltimer() - t0 > kWaitLimitNs) break;
-          }
-          if (!got) {
-            set_error(a.status, UMIM_ERR_TIMEOUT);
-            ok = 0;
-            break;
+              for (int w = 0; w < 64 && !got; ++w) got = (ld_acquire(&arr.flags[uq]) == epoch);
+              if (!got && globaltimer() - t0 > kWaitLimitNs) break;
+            }
+            if (!got) {
+              set_error(a.status, UMIM_ERR_TIMEOUT);
+              ok = 0;
+              break;
+            }
           }
         }
       }
       ok = __shfl_sync(0xffffffffu, ok, 0);
       if (!ok) break;
-      const int64_t dst = tile + (int64_t)a.block_table[(int64_t)b * a.max_pages + p] * page_stride;
+      if (cur.work) {
+        const int64_t dst = cur.layer * layer_stride + cur.kv * kv_stride + cur.h * head_stride + my_col * 8 +
+                            (int64_t)cur.dst_page * page_stride;
+        const uint32_t src_s = mbuf + half * TILE_BYTES;
 #pragma unroll
-      for (int it = 0; it < PER_LANE; ++it) {
-        const int slot = my_slot0 + it * SLOT_STEP;
-        if (write_mask & (1u << it)) st_v4(a.pool + dst + slot * D, v[it]);
+        for (int it = 0; it < PER_LANE; ++it) {
+          if (cur.mask & (1u << it)) {
+            uint4 v;
+            asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+                         : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                         : "r"(src_s + (lane + it * 32) * 16));
+            st_v4(a.pool + dst + (my_slot0 + it * SLOT_STEP) * D, v);
+          }
+        }
       }
+      __syncwarp();           // this half is refilled two slots later
+      cur = nxt;
+      half ^= 1;
     }
+    cp_async_wait_0();
     __syncwarp();
     if (lane == 0) {
       __threadfence_block();   // the last report is visible before the exit count
@@ -406,7 +448,9 @@ umim_status kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t m
   ma.B = B;
   ma.status = status;
   auto kern = (D == 128) ? rollback_move_kernel<128> : rollback_move_kernel<64>;
-  const int smem = 0;
+  const int smem = kMovers * 2 * kPageSize * D * 2;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
+    return UMIM_ERR_CUDA;
   int per_sm = 0;
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kMoveThreads, smem) != cudaSuccess || per_sm < 1)
     per_sm = 1;
