@@ -21,7 +21,7 @@
 namespace umim {
 namespace {
 
-constexpr int kMoveThreads = 224;   // 6 mover warps + 1 publisher warp
+constexpr int kMoveThreads = 256;
 constexpr int64_t kNoWrite = INT64_MIN;
 
 struct MoveArgs {
@@ -104,11 +104,8 @@ __global__ void __launch_bounds__(256) rollback_map_kernel(MoveArgs a, PlanArray
         if (arr.new_idx[i] == j) {
           src = -(int64_t)i - 1;
         } else {
-          // t == j (an entry that does not move, before the first span that
-          // removes anything) is read and written back unchanged, so that the
-          // written slots of a page form one contiguous range
           const int t = j + arr.r_incl[i];
-          src = (int64_t)bt[t / kPageSize] * page_stride + (t % kPageSize) * D;
+          if (t != j) src = (int64_t)bt[t / kPageSize] * page_stride + (t % kPageSize) * D;
         }
       }
     }
@@ -134,8 +131,6 @@ __global__ void __launch_bounds__(256) rollback_map_kernel(MoveArgs a, PlanArray
 }
 
 constexpr int kMovers = kMoveThreads / 32 - 1;   // mover warps per CTA; the last warp publishes
-
-
 
 __device__ __forceinline__ void st_release_cta_shared(int *p, int v) {
   asm volatile("st.release.cta.shared.b32 [%0], %1;" ::"r"(smem_u32(p)), "r"(v) : "memory");
@@ -164,47 +159,18 @@ __device__ __forceinline__ void st_relaxed_gpu(int32_t *p, int32_t v) {
 // for the whole batch and then marks their read-done flags: the fence orders
 // every reported load before every flag store that follows it, and movers
 // never pay for a GPU-scope fence themselves.
-__device__ __forceinline__ void bulk_load(uint32_t smem_dst, const void *gsrc, uint32_t bytes, uint32_t mbar) {
-  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-                   smem_dst),
-               "l"(gsrc), "r"(bytes), "r"(mbar)
-               : "memory");
-}
-__device__ __forceinline__ void bulk_store(void *gdst, uint32_t smem_src, uint32_t bytes) {
-  asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(gdst), "r"(smem_src), "r"(bytes)
-               : "memory");
-}
-__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
-__device__ __forceinline__ void bulk_wait_read_1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }
-__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
-__device__ __forceinline__ void fence_proxy_async_all() { asm volatile("fence.proxy.async;" ::: "memory"); }
-
-constexpr int kRing = 4;   // tiles per mover: one being written out, two in flight, one being refilled
-
-struct TileMeta {
-  int u, p, dep_lo, dep_hi, j_lo, j_hi, work;
-  int64_t dst;             // element offset of the destination tile in the pool
-};
-
-// Mover warps move tiles with the tensor-memory-access engine: the source
-// rows of a tile (runs of consecutive rows of one old page, or a surrogate
-// row) are bulk-copied into a slot of the mover's shared-memory ring,
-// completing the slot's mbarrier; once the tile is read, the mover reports it
-// to the CTA's publisher, waits for the units that read its destination page
-// and writes the tile back with one bulk copy.  Slots are visited page-row by
-// page-row (see the publisher comment above).
 template <int D>
-__global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a, PlanArrays arr, PageDesc pd) {
-  constexpr int ROW = D * 2;                        // bytes of one (kv, head) row
-  constexpr int TILE_BYTES = kPageSize * ROW;
-  extern __shared__ __align__(128) uint8_t move_smem[];
+__global__ void __launch_bounds__(kMoveThreads, 4) rollback_move_kernel(MoveArgs a, PlanArrays arr, PageDesc pd) {
+  constexpr int CPR = D / 8;                       // 16-byte chunks per row
+  constexpr int PER_LANE = kPageSize * CPR / 32;   // 8 (D=128) or 4 (D=64)
+  constexpr int SLOT_STEP = 32 / CPR;              // slots advanced per it
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
   const int nm = gridDim.x * kMovers;
+  const int my_col = lane % CPR;
+  const int my_slot0 = lane / CPR;
   __shared__ int s_last;
-  __shared__ int s_mail[kMovers];   // slots reported read by each mover (a count)
+  __shared__ int s_mail[kMovers];   // units reported loaded by each mover (a count)
   __shared__ int s_finished;        // movers that left their loop
-  __shared__ uint64_t s_full[kMovers][kRing];
-  __shared__ TileMeta s_meta[kMovers][kRing];
 
   const PlanHeader *hdr = arr.hdr;
   const int total = hdr->total_units;
@@ -218,12 +184,7 @@ __global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a,
   const int64_t n_slots = total > 0 ? (int64_t)hdr->max_dest * row_size : 0;
 
   if (threadIdx.x < kMovers) s_mail[threadIdx.x] = 0;
-  if (threadIdx.x == 0) {
-    s_finished = 0;
-    for (int m = 0; m < kMovers; ++m)
-      for (int r = 0; r < kRing; ++r) mbar_init(&s_full[m][r], 1);
-    fence_mbar_init();
-  }
+  if (threadIdx.x == 0) s_finished = 0;
   __syncthreads();
 
   if (wid == kMovers) {
@@ -243,7 +204,7 @@ __global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a,
         any |= mail[m] > published[m];
       }
       if (any) {
-        fence_acq_rel_gpu();   // every reported read happens before the flags below
+        fence_acq_rel_gpu();   // every reported load happens before the flags below
 #pragma unroll
         for (int m = 0; m < kMovers; ++m) {
           const int mover = blockIdx.x * kMovers + m;
@@ -270,126 +231,79 @@ __global__ void __launch_bounds__(kMoveThreads) rollback_move_kernel(MoveArgs a,
   } else {
     // ---- mover ----
     const int mover = blockIdx.x * kMovers + wid;
-    const uint32_t ring = smem_u32(move_smem + wid * kRing * TILE_BYTES);
-    // describe the k-th slot of this mover and start its copies into ring slot r
-    auto issue = [&](int k, int r) {
-      const int64_t i = mover + (int64_t)k * nm;
-      uint64_t *bar = &s_full[wid][r];
-      TileMeta &M = s_meta[wid][r];
-      int work = 0;
-      int kk = 0, b = 0, tl = 0, nd = 0;
-      if (i < n_slots) {
-        kk = (int)(i / row_size);
-        const int pos = (int)(i - (int64_t)kk * row_size);
-        b = pos / a.n_lanes;
-        tl = pos % a.n_lanes;
-        nd = arr.n_dest[b];
-        work = kk < nd;
+    int k = 0;
+    for (int64_t i = mover; i < n_slots; i += nm, ++k) {
+      // slot -> (compacted page row kk, sequence, tile lane)
+      const int kk = (int)(i / row_size);
+      const int pos = (int)(i - (int64_t)kk * row_size);
+      const int b = pos / a.n_lanes, tl = pos % a.n_lanes;
+      const int nd = arr.n_dest[b];
+      if (kk >= nd) {
+        if (lane == 0) st_release_cta_shared(&s_mail[wid], k + 1);
+        continue;
       }
-      if (!work) {
-        if (lane == 0) {
-          M.work = 0;
-          mbar_arrive(bar);
-        }
-        return;
-      }
-      const int ub = arr.unit_base[b];
+      const int u = arr.unit_base[b] + tl * nd + kk;
       const int layer = tl / (2 * Hkv);
       const int kv = (tl / Hkv) & 1;
       const int h = tl % Hkv;
+      const int idx = arr.unit_base[b] / a.n_lanes + kk;
       const int p = arr.first_page[b] + kk;
-      const int64_t idx = ub / a.n_lanes + kk;
-      const int64_t src = lane < kPageSize ? pd.src[idx * kPageSize + lane] : kNoWrite;
-      const int64_t tile = layer * layer_stride + kv * kv_stride + h * head_stride;
-      // written range [j_lo, j_hi) and runs of rows that are consecutive in memory
-      const unsigned wr = __ballot_sync(0xffffffffu, lane < kPageSize && src != kNoWrite);
-      const int j_lo = wr ? __ffs(wr) - 1 : 0;
-      const int j_hi = wr ? 32 - __clz(wr) : 0;
-      const int64_t prev = __shfl_up_sync(0xffffffffu, src, 1);
-      const bool in = lane >= j_lo && lane < j_hi;
-      const bool start = in && (lane == j_lo || src < 0 || prev < 0 || src != prev + D);
-      const unsigned starts = __ballot_sync(0xffffffffu, start);
-      if (lane == 0) {
-        M.work = 1;
-        M.u = ub + tl * nd + kk;
-        M.p = p;
-        const int2 dep = pd.dep[idx];
-        M.dep_lo = dep.x;
-        M.dep_hi = dep.y;
-        M.j_lo = j_lo;
-        M.j_hi = j_hi;
-        M.dst = tile + (int64_t)a.block_table[(int64_t)b * a.max_pages + p] * page_stride;
-        mbar_arrive_expect_tx(bar, (uint32_t)(j_hi - j_lo) * ROW);
-      }
-      __syncwarp();
-      if (start) {
-        const unsigned later = starts & ~((2u << lane) - 1u);   // run starts after this lane
-        const int end = later ? __ffs(later) - 1 : j_hi;
-        const uint32_t dst = ring + r * TILE_BYTES + lane * ROW;
-        if (src >= 0) {
-          bulk_load(dst, a.pool + tile + src, (uint32_t)(end - lane) * ROW, smem_u32(bar));
-        } else {
-          const int64_t si = -src - 1;
-          const uint16_t *sur = (kv ? a.sur_v : a.sur_k) + ((si * a.n_layers + layer) * Hkv + h) * D;
-          bulk_load(dst, sur, ROW, smem_u32(bar));
-        }
-      }
-    };
+      const int64_t my_src = lane < kPageSize ? pd.src[(int64_t)idx * kPageSize + lane] : kNoWrite;
+      const int2 dep = pd.dep[idx];
+      const int64_t tile = layer * layer_stride + kv * kv_stride + h * head_stride + my_col * 8;
+      const uint16_t *sur = kv ? a.sur_v : a.sur_k;
 
-    bool ok = true;
-    int k = 0;
-    for (int q = 0; q < kRing - 2; ++q) issue(q, q);
-    for (int64_t i = mover; i < n_slots; i += nm, ++k) {
-      // refill the slot of k-2 (its write-out has been read from shared memory)
-      if (lane == 0) bulk_wait_read_1();
-      __syncwarp();
-      issue(k + kRing - 2, (k + kRing - 2) % kRing);
-      const int r = k % kRing;
-      if (!mbar_wait(&s_full[wid][r], (k / kRing) & 1)) {
-        if (lane == 0) set_error(a.status, UMIM_ERR_TIMEOUT);
-        ok = false;
+      uint4 v[PER_LANE];
+      uint32_t write_mask = 0;
+      uint32_t fold = 0;
+#pragma unroll
+      for (int it = 0; it < PER_LANE; ++it) {
+        const int slot = my_slot0 + it * SLOT_STEP;
+        const int64_t src = __shfl_sync(0xffffffffu, my_src, slot);
+        if (src != kNoWrite) write_mask |= 1u << it;
+        v[it] = make_uint4(0, 0, 0, 0);
+        if (src >= 0) {
+          v[it] = ld_v4(a.pool + tile + src);
+        } else if (src != kNoWrite) {
+          const int64_t i = -src - 1;
+          v[it] = ld_v4(sur + ((i * a.n_layers + layer) * Hkv + h) * D + my_col * 8);
+        }
+        fold ^= v[it].x ^ v[it].y ^ v[it].z ^ v[it].w;
       }
-      if (lane == 0 && ok) {
-        // report: slots 0 .. k of this mover have been read
+      // every loaded value of this lane has arrived before the warp barrier
+      asm volatile("" ::"r"(fold) : "memory");
+      __syncwarp();
+      int ok = 1;
+      if (lane == 0) {
+        // report: units 0 .. k of this mover have been read
         st_release_cta_shared(&s_mail[wid], k + 1);
-        const TileMeta &M = s_meta[wid][r];
-        if (M.work) {
-          // wait for the units that read this tile of old page p (earlier rows)
-          for (int q = M.dep_lo; q <= M.dep_hi && q >= 0 && q < M.p && ok; ++q) {
-            const int uq = M.u - (M.p - q);
-            if (ld_acquire(&arr.flags[uq]) == epoch) continue;
-            const uint64_t t0 = globaltimer();
-            bool got = false;
-            while (!got) {
+        // wait for the units that read this tile of old page p (smaller indices)
+        for (int q = dep.x; q <= dep.y && q >= 0 && q < p; ++q) {
+          const int uq = u - (p - q);
+          if (ld_acquire(&arr.flags[uq]) == epoch) continue;
+          const uint64_t t0 = globaltimer();
+          bool got = false;
+          while (!got) {
 #pragma unroll 1
-              for (int w = 0; w < 64 && !got; ++w) got = (ld_acquire(&arr.flags[uq]) == epoch);
-              if (!got && globaltimer() - t0 > kWaitLimitNs) break;
-            }
-            if (!got) {
-              set_error(a.status, UMIM_ERR_TIMEOUT);
-              ok = false;
-            }
+            for (int i = 0; i < 64 && !got; ++i) got = (ld_acquire(&arr.flags[uq]) == epoch);
+            if (!got && globaltimer() - t0 > kWaitLimitNs) break;
           }
-          if (ok) {
-            // order the acquires above before the asynchronous write-out
-            fence_proxy_async_all();
-            bulk_store(a.pool + M.dst + (int64_t)M.j_lo * D, ring + r * TILE_BYTES + M.j_lo * ROW,
-                       (uint32_t)(M.j_hi - M.j_lo) * ROW);
+          if (!got) {
+            set_error(a.status, UMIM_ERR_TIMEOUT);
+            ok = 0;
+            break;
           }
         }
-        bulk_commit();
       }
-      ok = __shfl_sync(0xffffffffu, (int)ok, 0) != 0;
+      ok = __shfl_sync(0xffffffffu, ok, 0);
       if (!ok) break;
-    }
-    // after an early exit, let the copies still in flight land (each wait bounded)
-    if (!ok) {
-      for (int q = 1; q <= kRing - 2; ++q) {
-        const int kq = k + q;
-        if (mover + (int64_t)kq * nm < n_slots) mbar_wait(&s_full[wid][kq % kRing], (kq / kRing) & 1);
+      const int64_t dst = tile + (int64_t)a.block_table[(int64_t)b * a.max_pages + p] * page_stride;
+#pragma unroll
+      for (int it = 0; it < PER_LANE; ++it) {
+        const int slot = my_slot0 + it * SLOT_STEP;
+        if (write_mask & (1u << it)) st_v4(a.pool + dst + slot * D, v[it]);
       }
     }
-    if (lane == 0) bulk_wait_all();
     __syncwarp();
     if (lane == 0) {
       __threadfence_block();   // the last report is visible before the exit count
@@ -492,9 +406,7 @@ umim_status kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t m
   ma.B = B;
   ma.status = status;
   auto kern = (D == 128) ? rollback_move_kernel<128> : rollback_move_kernel<64>;
-  const int smem = kMovers * kRing * kPageSize * D * 2;
-  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
-    return UMIM_ERR_CUDA;
+  const int smem = 0;
   int per_sm = 0;
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kMoveThreads, smem) != cudaSuccess || per_sm < 1)
     per_sm = 1;
