@@ -12,6 +12,8 @@ for indices and moved KV bytes:
   merge.merge_spans       App. C.1 (attention-based pooling), Sec. 3.2 Eq. 1
   rollback.kv_rollback    App. C.6 and App. E ("Decoding-Time Merging and
                           KV-Cache Update"), Fig. 2 caption
+  append.kv_append        App. E and Fig. 2 step (2): one KV entry appended
+                          per layer when no rule matches
   attention.decode_attention
                           the backbone's ordinary attention over the shorter
                           cache (App. I.1); grouped-query mapping of Llama
@@ -27,11 +29,13 @@ upcast exactly to float64.
 Parity status per function (what pins it is in tests/test_oracle_*.py):
   merge_spans       pinned (library routines, invariants, brute force)
   kv_rollback       pinned (worked example, length formula, invariants)
+  kv_append         pinned (logical-list model, rollback identities)
   decode_attention  pinned (library SDPA, closed forms, invariants)
   build_compressed  pinned (worked example, length formula, library bf16)
 """
-from . import bf16, spans, merge, rollback, attention, compaction  # noqa: F401
+from . import bf16, spans, merge, rollback, append, attention, compaction  # noqa: F401
 from .merge import merge_spans, merge_span_reference_steps  # noqa: F401
 from .rollback import kv_rollback  # noqa: F401
+from .append import kv_append  # noqa: F401
 from .attention import decode_attention  # noqa: F401
 from .compaction import build_compressed  # noqa: F401

@@ -69,17 +69,17 @@ def kv_rollback(pool, block_table, seq_lens, span_offsets, span_start, span_len,
         # step 1: logical entries
         t_all = np.arange(L)
         entries = view[bt[b, t_all // P], t_all % P]           # [L][layers][2][Hkv][D]
-        # step 2: the new list, walking positions left to right
+        # step 2: the new list, left to right: the kept entries before each
+        # span, then the span's surrogate entry, then the entries after the
+        # last span
         new = []
-        t, i = 0, lo
-        while t < L:
-            if i < hi and t == int(span_start[i]):
-                new.append(np.stack([surrogate_k[i], surrogate_v[i]], axis=1))  # [layers][2][Hkv][D]
-                t += int(span_len[i])
-                i += 1
-            else:
-                new.append(entries[t])
-                t += 1
+        t = 0
+        for i in range(lo, hi):
+            s, k = int(span_start[i]), int(span_len[i])
+            new.extend(entries[t:s])
+            new.append(np.stack([surrogate_k[i], surrogate_v[i]], axis=1))  # [layers][2][Hkv][D]
+            t = s + k
+        new.extend(entries[t:L])
         new = np.stack(new)
         Lp = len(new)
         assert Lp == compressed_length(L, span_len[lo:hi])
