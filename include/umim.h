@@ -206,6 +206,36 @@ umim_status umim_kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int3
                              cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
+ * Decode-step KV append (App. E "Decoding-Time Merging and KV-Cache Update"
+ * and Fig. 2 step (2): a generated token that completes no merge is
+ * forwarded normally and one KV entry is appended).  For each sequence b
+ * with L = seq_lens[b], in every layer, the K and V rows of entry L are
+ * written to page block_table[b][L/16], slot L%16, from new_k/new_v[b];
+ * when L % 16 == 0 that page is new_pages[b] (the caller's allocator picks
+ * it) and is recorded in block_table[b][L/16]; seq_lens[b] becomes L + 1.
+ * With merging, the decode loop appends first and then, when the suffix
+ * matches a rule, rolls the last k stored entries back to one surrogate
+ * entry with umim_kv_rollback (k counts the appended entry).
+ *
+ * kv            host struct describing the device pool (written)
+ * block_table   device int32 [batch][max_pages], in/out
+ * seq_lens      device int32 [batch], in/out
+ * new_k/new_v   device bf16 [batch][n_layers][n_kv_heads][head_dim], 16-B aligned
+ * new_pages     device int32 [batch] or NULL: read only for sequences whose
+ *               length is a multiple of 16
+ * dev_status    device int32 or NULL (device-side errors are then not
+ *               reported)
+ * No workspace.  Device-side errors: UMIM_ERR_INVALID_ARG, and that
+ * sequence is left unchanged (the others are appended), when seq_lens[b] is
+ * outside [0, 16*max_pages), or the destination page (new_pages[b] at a page
+ * boundary, else block_table[b][L/16]) is outside [0, n_pages).  Not
+ * checked: that the new page is free.
+ * ------------------------------------------------------------------------ */
+umim_status umim_kv_append(const umim_paged_kv *kv, int32_t *block_table, int32_t max_pages, int32_t *seq_lens,
+                           int32_t batch, const void *new_k, const void *new_v, const int32_t *new_pages,
+                           int32_t *dev_status, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
  * Grouped-query decode attention over the (compacted) paged cache, one
  * query token per sequence (App. I.1; the backbone's ordinary attention):
  *   out[b][h] = sum_{j < seq_lens[b]} softmax_j(scale <q[b][h], K[b][g][j]>) V[b][g][j]

@@ -8,6 +8,7 @@ points keep the C names:
   umim_merge_spans        merge module M_phi (Sec. 3.2 Eq. 1, App. C.1)
   umim_build_compressed   compressed prompt embeddings + positions (App. E, App. C.5)
   umim_kv_rollback        KV-cache rollback and in-place compaction (App. E, Fig. 2)
+  umim_kv_append          decode-step append of one KV entry per layer (App. E, Fig. 2)
   umim_decode_attention   GQA decode attention over the compacted paged cache (App. I.1)
 """
 import ctypes
@@ -108,7 +109,7 @@ def umim_decode_attention_workspace_size(batch, n_q_heads, n_kv_heads, head_dim)
 
 
 # ---------------------------------------------------------------------------
-# the four calls
+# the calls
 # ---------------------------------------------------------------------------
 def umim_merge_spans(embeddings, token_ids, span_offsets, weights, surrogates=None, workspace_buf=None,
                      dev_status=None, stream=None):
@@ -173,6 +174,16 @@ def umim_kv_rollback(pool, block_table, seq_lens, span_offsets, span_start, span
                                   _stream(stream))
     _check(code, "umim_kv_rollback")
     return freed_pages
+
+
+def umim_kv_append(pool, block_table, seq_lens, new_k, new_v, new_pages=None, dev_status=None, stream=None):
+    """In-place append of one entry per layer to every sequence (new_k/new_v
+    [B][n_layers][Hkv][D] bf16; new_pages [B] int32, read at page boundaries)."""
+    kv = paged_kv(pool)
+    B, max_pages = block_table.shape
+    code = lib().umim_kv_append(ctypes.byref(kv), _p(block_table), max_pages, _p(seq_lens), B, _p(new_k),
+                                _p(new_v), _p(new_pages), _p(dev_status), _stream(stream))
+    _check(code, "umim_kv_append")
 
 
 def umim_decode_attention(q, pool, layer, block_table, seq_lens, scale=0.0, out=None, workspace_buf=None,

@@ -340,3 +340,117 @@ def serving_lengths(r: np.random.Generator, B: int, median: int = 1024, sigma: f
                     lo: int = 256, hi: int = 8192) -> np.ndarray:
     x = np.exp(np.log(median) + sigma * r.standard_normal(B))
     return np.clip(np.round(x), lo, hi).astype(np.int32)
+
+
+# ----------------------------------------------------------------------------
+# the decode loop of a serving engine (append, sometimes merge, attend)
+# ----------------------------------------------------------------------------
+class PageAllocator:
+    """First-in first-out free-page list of a paged cache: the bookkeeping a
+    serving engine's block allocator does (which physical page a sequence
+    gets when its length reaches a page boundary)."""
+
+    def __init__(self, free_pages):
+        import collections
+        self.free = collections.deque(int(p) for p in free_pages)
+
+    def take(self, lens) -> np.ndarray:
+        """new_pages[b]: a page for every sequence whose length is a multiple
+        of the page size (it opens a page with its next entry), else -1."""
+        new_pages = np.full(len(lens), -1, np.int32)
+        for b, L in enumerate(lens):
+            if int(L) % PAGE_SIZE == 0:
+                new_pages[b] = self.free.popleft()
+        return new_pages
+
+    def give_back(self, pages):
+        self.free.extend(int(p) for p in pages)
+
+
+@dataclasses.dataclass
+class ServingLoop:
+    """A decode loop over a paged cache: every step appends one entry per
+    sequence and layer, then each sequence with probability p merges its last
+    k ~ U{kmin..kmax} stored entries (the new one included) into one
+    surrogate entry, then attention runs per layer.  Initial KV entries,
+    appended entries, surrogates and queries are N(0,1) bf16 drawn from seeds
+    derived from (seed, step, layer), so any of them can be drawn again
+    without replaying the loop."""
+    seed: int
+    n_layers: int
+    n_q_heads: int
+    n_kv_heads: int
+    head_dim: int
+    steps: int
+    p: float
+    kmin: int
+    kmax: int
+    lens: np.ndarray          # [B] initial lengths
+    block_table: np.ndarray   # [B][max_pages] initial layout (-1 = no page)
+    n_pages: int
+    free_pages: list          # pages not in the initial layout, allocator order
+
+    @property
+    def B(self):
+        return len(self.lens)
+
+    def _seed(self, kind, step=0, layer=0):
+        return self.seed + 7919 * kind + 104729 * step + layer
+
+    def init_layer(self, layer, device):
+        """Initial contents of one layer of the pool, [n_pages][2][Hkv][P][D]."""
+        return bf16_normal((self.n_pages, 2, self.n_kv_heads, PAGE_SIZE, self.head_dim), 1.0,
+                           self._seed(1, 0, layer), device)
+
+    def init_pool(self, device):
+        pool = torch.empty((self.n_layers, self.n_pages, 2, self.n_kv_heads, PAGE_SIZE, self.head_dim),
+                           dtype=torch.bfloat16, device=device)
+        for layer in range(self.n_layers):
+            pool[layer] = self.init_layer(layer, device)
+        return pool
+
+    def new_entries(self, step, device):
+        shape = (self.B, self.n_layers, self.n_kv_heads, self.head_dim)
+        return (bf16_normal(shape, 1.0, self._seed(2, step, 0), device),
+                bf16_normal(shape, 1.0, self._seed(2, step, 1), device))
+
+    def rollbacks(self, step):
+        """[(b, k)]: the sequences that merge their last k stored entries after
+        this step's append, in increasing b."""
+        r = rng(self._seed(3, step))
+        hit = r.random(self.B) < self.p
+        ks = r.integers(self.kmin, self.kmax + 1, size=self.B)
+        return [(b, int(ks[b])) for b in range(self.B) if hit[b]]
+
+    def surrogates(self, step, n, device):
+        shape = (n, self.n_layers, self.n_kv_heads, self.head_dim)
+        return (bf16_normal(shape, 1.0, self._seed(4, step, 0), device),
+                bf16_normal(shape, 1.0, self._seed(4, step, 1), device))
+
+    def q(self, step, layer, device):
+        return bf16_normal((self.B, self.n_q_heads, self.head_dim), 1.0, self._seed(5, step, layer), device)
+
+
+def serving_loop(seed: int, *, B: int, n_layers: int, n_q_heads: int, n_kv_heads: int, head_dim: int,
+                 steps: int, p: float = 0.1, kmin: int = 2, kmax: int = 4, lens=None, median: int = 1024,
+                 sigma: float = 1.0, lo: int = 256, hi: int = 8192) -> ServingLoop:
+    """Lengths lognormal(ln median, sigma) clipped to [lo, hi] unless given;
+    every sequence has room for `steps` appends; physical pages are a random
+    permutation, the pages not in the initial layout form the free list."""
+    r = rng(seed)
+    lens = serving_lengths(r, B, median, sigma, lo, hi) if lens is None else np.asarray(lens, np.int32)
+    P = PAGE_SIZE
+    pages_now = (lens.astype(np.int64) + P - 1) // P
+    pages_max = (lens.astype(np.int64) + steps + P - 1) // P
+    max_pages = int(max(1, pages_max.max()))
+    n_pages = int(pages_max.sum()) + B
+    perm = r.permutation(n_pages).astype(np.int32)
+    bt = np.full((B, max_pages), -1, np.int32)
+    k = 0
+    for b in range(B):
+        for pg in range(int(pages_now[b])):
+            bt[b, pg] = perm[k]
+            k += 1
+    return ServingLoop(seed=seed, n_layers=n_layers, n_q_heads=n_q_heads, n_kv_heads=n_kv_heads,
+                       head_dim=head_dim, steps=steps, p=p, kmin=kmin, kmax=kmax, lens=lens.astype(np.int32),
+                       block_table=bt, n_pages=n_pages, free_pages=[int(x) for x in perm[k:]])
