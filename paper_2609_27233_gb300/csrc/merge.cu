@@ -535,6 +535,7 @@ __global__ void __launch_bounds__(kPoolConsumers + 32, CH <= 2 ? 2 : 1)
 __global__ void __launch_bounds__(256)
     ln_rows_kernel(float *Z, const float2 *stats, int S, int d, const __nv_bfloat16 *gamma,
                    const __nv_bfloat16 *beta, float eps) {
+  griddep_wait();
   const int r = blockIdx.x * 8 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (r >= S) return;

@@ -34,6 +34,7 @@ def _run(case):
     (23, 3000, 4096, 4, 97, 2, 4),                       # Llama-3-8B width, several M / all N tiles
     (24, 700, 2048, 8, 60, 1, 4),                        # 8 pooling heads
     (25, 700, 1536, 2, 33, 4, 4),                        # 2 heads, only 4-token spans
+    (27, 700, 1536, 8, 21, 1, 4),                        # head width 192: 24 chunks, 3 column groups per head
 ])
 def test_merge_matches_oracle(seed, vocab, d, h, S, kmin, kmax):
     case = W.merge_case(seed, vocab=vocab, d=d, h=h, n_spans=S, kmin=kmin, kmax=kmax)
