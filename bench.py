@@ -17,6 +17,11 @@ beside it.  Every timed step works on its own pristine copy of the cache
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl umim|reference]
   python bench.py --workload serving
 
+--workload prompt_compression times the prompt-side path (64 prompts of 2048
+tokens, merge module at d_model 4096 over all 17k spans, then the packed
+compressed prompts); --workload long_context times rollback + decode
+attention on 4 sequences of 32768 tokens (28/4 heads, 40 % coverage; add
+--coverage 0.6 for the 40 % token-reduction reading).
 --workload serving times the serving decode loop instead (128 sequences of
 lognormal length, 32 layers of 32/8 heads, 256 steps; every step appends one
 entry per sequence and layer, merges the last 2..4 stored entries of each
@@ -229,6 +234,21 @@ class OracleSampler:
                     rollback_s_per_seq=t_rb, attention_s_per_seq=t_at)
 
 
+def reduce_over_ranks(ms, units, device):
+    """(max of ms over ranks, sum of units over ranks): the whole job's
+    elapsed time is the slowest rank's, and every rank processed its own
+    batch.  One process (or no process group) returns the inputs."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return float(ms), float(units)
+    t = torch.tensor([float(ms)], dtype=torch.float64, device=device)
+    u = torch.tensor([float(units)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dist.all_reduce(u, op=dist.ReduceOp.SUM)
+    return float(t.item()), float(u.item())
+
+
 def cpu_cores():
     n = os.cpu_count() or 1
     try:
@@ -267,10 +287,14 @@ def main():
     ap.add_argument("--impl", default="umim", choices=["umim", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--workload", default="llama8b_layer", choices=["llama8b_layer", "serving"])
+    ap.add_argument("--workload", default="llama8b_layer",
+                    choices=["llama8b_layer", "serving", "prompt_compression", "long_context"])
+    ap.add_argument("--coverage", type=float, default=0.4, help="long_context span coverage")
     args = ap.parse_args()
     if args.workload == "serving" and args.impl == "umim":
         return serving_bench(args)
+    if args.workload in ("prompt_compression", "long_context") and args.impl == "umim":
+        return side_bench(args)
     K, Wm = args.steps, max(3, args.warmup)
 
     rank = int(os.environ.get("RANK", "0"))
@@ -409,12 +433,9 @@ def main():
     clk.stop()
     umim.check_status(status, "timed steps")
     clocks = clk.summary(t_wall0, t_wall1)
-    if world > 1:
-        tt = torch.tensor([ms], device=dev)
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        ms = float(tt.item())
+    ms, units = reduce_over_ranks(ms, S * K, dev)
     ms_step = ms / K
-    value = world * S * K / (ms / 1000.0)
+    value = units / (ms / 1000.0)
 
     # ---- per-kernel times: the same steps again, with kernel tracing on ----
     restore()
@@ -485,11 +506,8 @@ def main():
         restore()
         torch.cuda.synchronize()
         ems = timed(e2e_step, K, Wm)
-        if world > 1:
-            tt = torch.tensor([ems], device=dev)
-            torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-            ems = float(tt.item())
-        e2e = {"value": world * S * K / (ems / 1000.0), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
+        ems, eunits = reduce_over_ranks(ems, S * K, dev)
+        e2e = {"value": eunits / (ems / 1000.0), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
                "d2h_bytes_per_step": int(d2h), "ms_per_step": ems / K}
         umim.check_status(status, "e2e steps")
 
@@ -656,6 +674,176 @@ def serving_bench(args):
                             "us_mean": round(1000 * float(np.mean(v)), 2)} for k, v in
                         sorted(kern.items(), key=lambda x: -np.sum(x[1]))},
             "gpu_launches": len(recs), "clocks": clocks, "traced_ms_per_step": tms / sl.steps}
+    print(json.dumps(line))
+    return 0
+
+
+def kernel_table(recs, K, work_of):
+    kern = {}
+    for lab, v in recs:
+        kern.setdefault(lab, []).append(v)
+    total = max(sum(sum(x) for x in kern.values()), 1e-9)
+    out = {}
+    for k, v in sorted(kern.items(), key=lambda x: -np.mean(x[1])):
+        mean = float(np.mean(v))
+        e = {"ms": round(mean, 5), "launches_per_step": round(len(v) / K, 2), "share": round(sum(v) / total, 4)}
+        if k in work_of:
+            b, amount, unit, peak = work_of[k]
+            ach = amount / (mean / 1000.0)
+            e.update({"bound": b, "achieved": round(ach, 2), "unit": unit, "frac": round(ach / peak, 4)})
+        out[k] = e
+    return out
+
+
+def side_bench(args):
+    """Prompt compression (merge + packed compressed prompts) or long-context
+    rollback + attention, timed like the default step (CUDA events around K
+    steps after W warm-up steps, then a traced run for per-kernel times)."""
+    import torch
+    import paper_2609_27233_gb300 as umim
+    import workloads as W
+
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    umim.lib()
+    peaks = load_peaks()
+    K, Wm = args.steps, max(3, args.warmup)
+    status = umim.new_status(dev)
+
+    if args.workload == "prompt_compression":
+        seed = W.SEEDS["prompt_compression"]
+        B, L, V, d = 64, 2048, 128256, 4096
+        table = W.bf16_normal((V, d), 0.02, seed + 101, dev)
+        pc = W.prompt_case(seed, B=B, L=L, vocab=V, d=d, coverage=0.4, device=dev, table=table)
+        weights = W.merge_weights(d, 4, seed + 202, dev)
+        S, T = pc.span_start.numel(), pc.span_token_ids.numel()
+        z = torch.empty((S, d), dtype=torch.float32, device=dev)
+        ws_m = umim.workspace(umim.umim_merge_spans_workspace_size(T, S, d), dev)
+        ws_c = umim.workspace(umim.umim_build_compressed_workspace_size(B, S), dev)
+        rows = B * L - int((pc.span_len.cpu().numpy() - 1).sum())
+        out = torch.empty((rows, d), dtype=torch.bfloat16, device=dev)
+        pos = torch.empty(rows, dtype=torch.int32, device=dev)
+        cu = torch.empty(B + 1, dtype=torch.int32, device=dev)
+
+        def step(i):
+            umim.umim_merge_spans(table, pc.span_token_ids, pc.span_token_offsets, weights, surrogates=z,
+                                  workspace_buf=ws_m, dev_status=status)
+            umim.umim_build_compressed(table, pc.token_ids, pc.span_offsets, pc.span_start, pc.span_len, z,
+                                       out_embeds=out, position_ids=pos, cu_seqlens=cu, workspace_buf=ws_c,
+                                       dev_status=status)
+
+        restore = None
+        kept = rows - S
+        comp_bytes = rows * d * 2 + kept * d * 2 + S * d * 4 + B * L * 4 + rows * 4
+        work_of = {
+            "merge.gemm1": ("tensor", 2.0 * T * d * d / 1e12, "TFLOP/s", peaks["bf16"]),
+            "merge.gemm2": ("tensor", 2.0 * S * d * d / 1e12, "TFLOP/s", peaks["bf16"]),
+            "compact.rows": ("hbm", comp_bytes / 1e9, "GB/s", peaks["hbm"]),
+        }
+        units, unit, metric = S, "spans/s", "prompt compression: merged spans/s (merge module + packed prompts)"
+        cfg = {"workload": "prompt compression: 64 prompts x 2048 uniform token ids over a 128256 x 4096 bf16 "
+                           "table, 40% of tokens in spans of 2..4, merge module d_model 4096 (4 heads), packed "
+                           "compressed prompts with position ids",
+               "spans": S, "span_tokens": T, "compressed_rows": rows,
+               "l2": "inputs larger than L2: the 1.05 GB table and 787 MB of packed output per step"}
+    else:
+        name = "long_context" if abs(args.coverage - 0.4) < 1e-9 else "long_context_tr40"
+        seed = W.SEEDS[name]
+        c = W.decode_case(seed, lens=[32768] * 4, n_q_heads=28, n_kv_heads=4, head_dim=128,
+                          coverage=args.coverage, device=dev)
+        B, Hq, Hkv, D = 4, 28, 4, 128
+        max_pages = c.max_pages
+        n_copies = min(Wm + K, max(Wm + 1, int(0.5 * torch.cuda.mem_get_info(dev)[0] // (c.pool.numel() * 2))))
+        pools = [torch.empty_like(c.pool) for _ in range(n_copies)]
+        bts = [torch.empty_like(c.block_table) for _ in range(n_copies)]
+        lens = [torch.empty_like(c.seq_lens) for _ in range(n_copies)]
+
+        def restore():
+            for i in range(n_copies):
+                pools[i].copy_(c.pool)
+                bts[i].copy_(c.block_table)
+                lens[i].copy_(c.seq_lens)
+
+        S = c.span_start.numel()
+        freed = torch.empty(B * max_pages, dtype=torch.int32, device=dev)
+        out = torch.empty_like(c.q)
+        ws_r = umim.workspace(umim.umim_kv_rollback_workspace_size(B, S, max_pages, 1, Hkv, D), dev)
+        ws_a = umim.workspace(umim.umim_decode_attention_workspace_size(B, Hq, Hkv, D), dev)
+
+        def step(i):
+            j = i % n_copies
+            umim.umim_kv_rollback(pools[j], bts[j], lens[j], c.span_offsets, c.span_start, c.span_len,
+                                  c.surrogate_k, c.surrogate_v, freed_pages=freed, workspace_buf=ws_r,
+                                  dev_status=status)
+            umim.umim_decode_attention(c.q, pools[j], 0, bts[j], lens[j], out=out, workspace_buf=ws_a,
+                                       dev_status=status)
+
+        entry = 2 * Hkv * D * 2
+        offs, st_, ln_ = (c.span_offsets.cpu().numpy(), c.span_start.cpu().numpy(), c.span_len.cpu().numpy())
+        moved, Lp = 0, []
+        for b in range(B):
+            lo, hi = offs[b], offs[b + 1]
+            r, prev = 0, 0
+            for s_, k_ in zip(st_[lo:hi], ln_[lo:hi]):
+                if r > 0:
+                    moved += int(s_) - prev
+                r += int(k_) - 1
+                prev = int(s_ + k_)
+            if r > 0:
+                moved += 32768 - prev
+            Lp.append(32768 - int((ln_[lo:hi] - 1).sum()))
+        rb_bytes = (moved + S) * entry * 2
+        at_bytes = sum(Lp) * entry + 2 * B * Hq * D * 2
+        work_of = {"rollback.move": ("hbm", rb_bytes / 1e9, "GB/s", peaks["hbm"]),
+                   "attention.decode": ("hbm", at_bytes / 1e9, "GB/s", peaks["hbm"])}
+        units, unit, metric = S, "spans/s", "long-context decode: merged spans/s (rollback + attention)"
+        cfg = {"workload": f"long-context decode: 4 seqs x 32768 tokens, 28/4 heads, head_dim 128, bf16 paged KV "
+                           f"(page 16), {int(round(100 * args.coverage))}% of positions in spans of 2..4 rolled "
+                           f"back, then decode attention",
+               "spans": S, "compacted_lengths": Lp,
+               "l2": "inputs larger than L2: a distinct 268 MB cache copy per step"}
+
+    def timed(n, offset):
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for i in range(n):
+            if restore is not None and (offset + i) % n_copies == 0 and offset + i > 0:
+                restore()
+            step(offset + i)
+        e1.record()
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1)
+
+    if restore is not None:
+        restore()
+    for i in range(Wm):
+        step(i)
+    torch.cuda.synchronize()
+    umim.check_status(status, "warm-up")
+    if restore is not None:
+        restore()
+    clk = ClockSampler(0)
+    time.sleep(0.3)
+    w0 = time.time()
+    ms = timed(K, Wm)
+    w1 = time.time()
+    time.sleep(0.1)
+    clk.stop()
+    umim.check_status(status, "timed steps")
+    if restore is not None:
+        restore()
+    torch.cuda.synchronize()
+    umim.trace_start(64 * (K + 2))
+    tms = timed(K, Wm)
+    umim.trace_stop()
+    recs = umim.trace_read(64 * (K + 2))
+    kernels = kernel_table(recs, K, work_of)
+    line = {"metric": metric, "value": units * K / (ms / 1000.0), "unit": unit, "n_gpus": 1, "steps": K,
+            "warmup": Wm, "ms_per_step": ms / K, "higher_is_better": True, "dtype": "bf16", "data": "synthetic",
+            "config": cfg, "kernels": kernels, "gpu_launches": len(recs), "clocks": clk.summary(w0, w1),
+            "traced_ms_per_step": tms / K, "peaks": {"hbm_gbs": peaks["hbm"], "bf16_tflops": peaks["bf16"],
+                                                     "source": peaks["src"]}}
     print(json.dumps(line))
     return 0
 

@@ -450,36 +450,69 @@ __global__ void __launch_bounds__(kAttnWarps * 32, 1)
 }
 
 // ---------------------------------------------------------------------------
-// combine: one warp per (b, query head)
+// combine: one CTA per (b, query head); its warps split the pieces of the
+// segment, each merges its share in one pass with a running maximum, and the
+// warps' (m, l, acc) are merged through shared memory.
 // ---------------------------------------------------------------------------
+constexpr int kCombineWarps = 8;
+
 template <int D>
-__global__ void attn_combine_kernel(AttnWs ws, int B, int Hq, int Hkv, int G, __nv_bfloat16 *out) {
+__global__ void __launch_bounds__(kCombineWarps * 32)
+    attn_combine_kernel(AttnWs ws, int B, int Hq, int Hkv, int G, __nv_bfloat16 *out) {
+  constexpr int E = D / 32;
+  __shared__ float s_m[kCombineWarps], s_l[kCombineWarps];
+  __shared__ float s_acc[kCombineWarps][D];
   griddep_wait();
-  const int warp_global = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const int lane = threadIdx.x & 31;
-  if (warp_global >= B * Hq) return;
-  const int b = warp_global / Hq, h = warp_global % Hq;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int b = blockIdx.x / Hq, h = blockIdx.x % Hq;
   const int seg = b * Hkv + h / G, row = h % G;
   const int p0 = ws.piece_base[seg], p1 = ws.piece_base[seg + 1];
-  constexpr int E = D / 32;
-  float o[E];
+  float M = -INFINITY, l = 0.f, o[E];
 #pragma unroll
   for (int e = 0; e < E; ++e) o[e] = 0.f;
-  float M = -INFINITY;
-  for (int pc = p0; pc < p1; ++pc) M = fmaxf(M, ws.part_ml[(int64_t)pc * 16 + row].x);
-  float den = 0.f;
-  for (int pc = p0; pc < p1; ++pc) {
+  for (int pc = p0 + warp; pc < p1; pc += kCombineWarps) {
     const float2 ml = ws.part_ml[(int64_t)pc * 16 + row];
-    const float w = exp2f(ml.x - M);
-    den += w * ml.y;
-    const float *acc = ws.part_acc + ((int64_t)pc * 16 + row) * D;
+    const float *acc = ws.part_acc + ((int64_t)pc * 16 + row) * D + lane * E;
+    float a[E];
 #pragma unroll
-    for (int e = 0; e < E; ++e) o[e] += w * acc[lane * E + e];
+    for (int e = 0; e < E; ++e) a[e] = acc[e];
+    const float nm = fmaxf(M, ml.x);
+    if (nm == -INFINITY) continue;   // nothing but empty pieces so far
+    const float c_old = exp2f(M - nm), c_new = exp2f(ml.x - nm);
+    l = l * c_old + ml.y * c_new;
+#pragma unroll
+    for (int e = 0; e < E; ++e) o[e] = o[e] * c_old + a[e] * c_new;
+    M = nm;
   }
-  const float inv = den > 0.f ? 1.f / den : 0.f;
-  __nv_bfloat16 *dst = out + ((int64_t)b * Hq + h) * D + lane * E;
+  if (lane == 0) {
+    s_m[warp] = M;
+    s_l[warp] = l;
+  }
 #pragma unroll
-  for (int e = 0; e < E; ++e) dst[e] = __float2bfloat16_rn(o[e] * inv);
+  for (int e = 0; e < E; ++e) s_acc[warp][lane * E + e] = o[e];
+  __syncthreads();
+  if (warp == 0) {
+    float Mx = -INFINITY;
+#pragma unroll
+    for (int w = 0; w < kCombineWarps; ++w) Mx = fmaxf(Mx, s_m[w]);
+    float den = 0.f, r[E];
+#pragma unroll
+    for (int e = 0; e < E; ++e) r[e] = 0.f;
+    if (Mx != -INFINITY) {
+#pragma unroll
+      for (int w = 0; w < kCombineWarps; ++w) {
+        if (s_m[w] == -INFINITY) continue;
+        const float c = exp2f(s_m[w] - Mx);
+        den += c * s_l[w];
+#pragma unroll
+        for (int e = 0; e < E; ++e) r[e] += c * s_acc[w][lane * E + e];
+      }
+    }
+    const float inv = den > 0.f ? 1.f / den : 0.f;
+    __nv_bfloat16 *dst = out + ((int64_t)b * Hq + h) * D + lane * E;
+#pragma unroll
+    for (int e = 0; e < E; ++e) dst[e] = __float2bfloat16_rn(r[e] * inv);
+  }
 }
 
 }  // namespace
@@ -550,10 +583,8 @@ static umim_status run_attention(const void *q, int Hq, const umim_paged_kv *kv,
       cudaSuccess)
     return UMIM_ERR_CUDA;
   trace_mark(stream, "attention.combine");
-  const int threads = 256;
-  const int nwarps = B * Hq;
-  if (launch_pdl(attn_combine_kernel<D>, dim3((nwarps * 32 + threads - 1) / threads), dim3(threads), 0, stream, ws,
-                 B, Hq, Hkv, a.G, static_cast<__nv_bfloat16 *>(out)) != cudaSuccess)
+  if (launch_pdl(attn_combine_kernel<D>, dim3((unsigned)(B * Hq)), dim3(kCombineWarps * 32), 0, stream, ws, B, Hq,
+                 Hkv, a.G, static_cast<__nv_bfloat16 *>(out)) != cudaSuccess)
     return UMIM_ERR_CUDA;
   trace_mark(stream, nullptr);
   return cudaGetLastError() == cudaSuccess ? UMIM_OK : UMIM_ERR_CUDA;

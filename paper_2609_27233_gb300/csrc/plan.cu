@@ -5,7 +5,7 @@
 namespace umim {
 namespace {
 
-constexpr int kPlanThreads = 256;
+constexpr int kPlanThreads = 1024;
 
 // Inclusive block-wide scan; every thread gets the block total.
 __device__ int block_scan_incl(int v, int &total) {
