@@ -178,6 +178,8 @@ umim_status umim_kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int3
   if (!kv_ok(kv) || batch < 0 || max_pages < 0 || n_spans < 0) return UMIM_ERR_INVALID_ARG;
   if (!kv_supported(kv)) return UMIM_ERR_UNSUPPORTED;
   if ((int64_t)batch * max_pages > INT32_MAX / 16 || batch > 65535) return UMIM_ERR_UNSUPPORTED;
+  // work units (sequence x page x layer x K|V x head) are indexed in 32 bits
+  if ((int64_t)batch * max_pages * kv->n_layers * 2 * kv->n_kv_heads >= INT32_MAX / 2) return UMIM_ERR_UNSUPPORTED;
   if (batch == 0) return UMIM_OK;
   if (!block_table || !seq_lens || !span_offsets) return UMIM_ERR_INVALID_ARG;
   if (n_spans > 0 && (!span_start || !span_len || !surrogate_k || !surrogate_v)) return UMIM_ERR_INVALID_ARG;

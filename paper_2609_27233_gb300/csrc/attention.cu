@@ -450,69 +450,76 @@ __global__ void __launch_bounds__(kAttnWarps * 32, 1)
 }
 
 // ---------------------------------------------------------------------------
-// combine: one CTA per (b, query head); its warps split the pieces of the
-// segment, each merges its share in one pass with a running maximum, and the
-// warps' (m, l, acc) are merged through shared memory.
+// combine: WPR warps per (b, query head) row, 256 threads per CTA.  The warps
+// of a row split its segment's pieces, each merges its share in one pass with
+// a running maximum, and (WPR > 1) the warps' (m, l, acc) are merged through
+// shared memory.  WPR grows with the pieces per segment (few, long sequences
+// split into many pieces).
 // ---------------------------------------------------------------------------
-constexpr int kCombineWarps = 8;
+constexpr int kCombineThreads = 256;
 
-template <int D>
-__global__ void __launch_bounds__(kCombineWarps * 32)
+template <int D, int WPR>
+__global__ void __launch_bounds__(kCombineThreads)
     attn_combine_kernel(AttnWs ws, int B, int Hq, int Hkv, int G, __nv_bfloat16 *out) {
   constexpr int E = D / 32;
-  __shared__ float s_m[kCombineWarps], s_l[kCombineWarps];
-  __shared__ float s_acc[kCombineWarps][D];
+  constexpr int RPB = kCombineThreads / 32 / WPR;   // rows per CTA
+  __shared__ float s_m[kCombineThreads / 32], s_l[kCombineThreads / 32];
+  __shared__ float s_acc[WPR > 1 ? kCombineThreads / 32 : 1][D];
   griddep_wait();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int b = blockIdx.x / Hq, h = blockIdx.x % Hq;
+  const int row_g = blockIdx.x * RPB + warp / WPR, sub = warp % WPR;
+  const bool live = row_g < B * Hq;
+  const int b = live ? row_g / Hq : 0, h = live ? row_g % Hq : 0;
   const int seg = b * Hkv + h / G, row = h % G;
-  const int p0 = ws.piece_base[seg], p1 = ws.piece_base[seg + 1];
+  const int p0 = live ? ws.piece_base[seg] : 0, p1 = live ? ws.piece_base[seg + 1] : 0;
   float M = -INFINITY, l = 0.f, o[E];
 #pragma unroll
   for (int e = 0; e < E; ++e) o[e] = 0.f;
-  for (int pc = p0 + warp; pc < p1; pc += kCombineWarps) {
+  for (int pc = p0 + sub; pc < p1; pc += WPR) {
     const float2 ml = ws.part_ml[(int64_t)pc * 16 + row];
     const float *acc = ws.part_acc + ((int64_t)pc * 16 + row) * D + lane * E;
-    float a[E];
+    float av[E];
 #pragma unroll
-    for (int e = 0; e < E; ++e) a[e] = acc[e];
+    for (int e = 0; e < E; ++e) av[e] = acc[e];
     const float nm = fmaxf(M, ml.x);
     if (nm == -INFINITY) continue;   // nothing but empty pieces so far
     const float c_old = exp2f(M - nm), c_new = exp2f(ml.x - nm);
     l = l * c_old + ml.y * c_new;
 #pragma unroll
-    for (int e = 0; e < E; ++e) o[e] = o[e] * c_old + a[e] * c_new;
+    for (int e = 0; e < E; ++e) o[e] = o[e] * c_old + av[e] * c_new;
     M = nm;
   }
-  if (lane == 0) {
-    s_m[warp] = M;
-    s_l[warp] = l;
-  }
+  if constexpr (WPR > 1) {
+    if (lane == 0) {
+      s_m[warp] = M;
+      s_l[warp] = l;
+    }
 #pragma unroll
-  for (int e = 0; e < E; ++e) s_acc[warp][lane * E + e] = o[e];
-  __syncthreads();
-  if (warp == 0) {
+    for (int e = 0; e < E; ++e) s_acc[warp][lane * E + e] = o[e];
+    __syncthreads();
+    if (sub != 0) return;
     float Mx = -INFINITY;
 #pragma unroll
-    for (int w = 0; w < kCombineWarps; ++w) Mx = fmaxf(Mx, s_m[w]);
-    float den = 0.f, r[E];
+    for (int w = 0; w < WPR; ++w) Mx = fmaxf(Mx, s_m[warp + w]);
+    l = 0.f;
 #pragma unroll
-    for (int e = 0; e < E; ++e) r[e] = 0.f;
+    for (int e = 0; e < E; ++e) o[e] = 0.f;
     if (Mx != -INFINITY) {
 #pragma unroll
-      for (int w = 0; w < kCombineWarps; ++w) {
-        if (s_m[w] == -INFINITY) continue;
-        const float c = exp2f(s_m[w] - Mx);
-        den += c * s_l[w];
+      for (int w = 0; w < WPR; ++w) {
+        if (s_m[warp + w] == -INFINITY) continue;
+        const float c = exp2f(s_m[warp + w] - Mx);
+        l += c * s_l[warp + w];
 #pragma unroll
-        for (int e = 0; e < E; ++e) r[e] += c * s_acc[w][lane * E + e];
+        for (int e = 0; e < E; ++e) o[e] += c * s_acc[warp + w][lane * E + e];
       }
     }
-    const float inv = den > 0.f ? 1.f / den : 0.f;
-    __nv_bfloat16 *dst = out + ((int64_t)b * Hq + h) * D + lane * E;
-#pragma unroll
-    for (int e = 0; e < E; ++e) dst[e] = __float2bfloat16_rn(r[e] * inv);
   }
+  if (!live) return;
+  const float inv = l > 0.f ? 1.f / l : 0.f;
+  __nv_bfloat16 *dst = out + ((int64_t)b * Hq + h) * D + lane * E;
+#pragma unroll
+  for (int e = 0; e < E; ++e) dst[e] = __float2bfloat16_rn(o[e] * inv);
 }
 
 }  // namespace
@@ -583,8 +590,15 @@ static umim_status run_attention(const void *q, int Hq, const umim_paged_kv *kv,
       cudaSuccess)
     return UMIM_ERR_CUDA;
   trace_mark(stream, "attention.combine");
-  if (launch_pdl(attn_combine_kernel<D>, dim3((unsigned)(B * Hq)), dim3(kCombineWarps * 32), 0, stream, ws, B, Hq,
-                 Hkv, a.G, static_cast<__nv_bfloat16 *>(out)) != cudaSuccess)
+  // warps per row: about half the pieces a segment has (1 + warps / segments)
+  const int per_seg = 1 + total_warps / std::max(1, B * Hkv);
+  const int wpr = per_seg >= 16 ? 8 : per_seg >= 8 ? 4 : per_seg >= 4 ? 2 : 1;
+  const int rows_per_cta = kCombineThreads / 32 / wpr;
+  auto comb = wpr == 8 ? attn_combine_kernel<D, 8>
+              : wpr == 4 ? attn_combine_kernel<D, 4>
+              : wpr == 2 ? attn_combine_kernel<D, 2> : attn_combine_kernel<D, 1>;
+  if (launch_pdl(comb, dim3((unsigned)((B * Hq + rows_per_cta - 1) / rows_per_cta)), dim3(kCombineThreads), 0, stream,
+                 ws, B, Hq, Hkv, a.G, static_cast<__nv_bfloat16 *>(out)) != cudaSuccess)
     return UMIM_ERR_CUDA;
   trace_mark(stream, nullptr);
   return cudaGetLastError() == cudaSuccess ? UMIM_OK : UMIM_ERR_CUDA;

@@ -110,7 +110,7 @@ __global__ void __launch_bounds__(kPlanThreads) span_plan_kernel(PlanArgs a, Pla
   // ---- last block: prefix sums over sequences, per-call header reset ----
   __threadfence();
   const int err = atomicOr(&arr.hdr->error, 0);
-  int cu_units = 0, cu_rows = 0, cu_freed = 0;
+  int cu_units = 0, cu_rows = 0, cu_freed = 0, cu_active = 0;
   __shared__ int s_max_dest;
   if (threadIdx.x == 0) s_max_dest = 0;
   __syncthreads();
@@ -124,19 +124,23 @@ __global__ void __launch_bounds__(kPlanThreads) span_plan_kernel(PlanArgs a, Pla
       r = Lp;
       f = ceil_div(L, kPageSize) - ceil_div(Lp, kPageSize);
     }
-    int tu, tr, tf;
+    const int act = (j < a.B && arr.n_dest[j] > 0) ? 1 : 0;
+    int tu, tr, tf, ta;
     const int iu = block_scan_incl(u, tu);
     const int ir = block_scan_incl(r, tr);
     const int iff = block_scan_incl(f, tf);
+    const int ia = block_scan_incl(act, ta);
     if (j < a.B) {
       arr.unit_base[j] = cu_units + iu - u;
       arr.row_base[j] = cu_rows + ir - r;
       arr.freed_base[j] = cu_freed + iff - f;
+      if (act) arr.active[cu_active + ia - 1] = j;
       if (a.cu_seqlens_out && !err) a.cu_seqlens_out[j] = cu_rows + ir - r;
     }
     cu_units += tu;
     cu_rows += tr;
     cu_freed += tf;
+    cu_active += ta;
   }
   if (threadIdx.x == 0) {
     arr.unit_base[a.B] = cu_units;
@@ -147,6 +151,7 @@ __global__ void __launch_bounds__(kPlanThreads) span_plan_kernel(PlanArgs a, Pla
     h->total_units = err ? 0 : cu_units;
     h->total_rows = cu_rows;
     h->max_dest = err ? 0 : s_max_dest;
+    h->n_active = err ? 0 : cu_active;
     h->skip = err ? 1 : 0;
     h->epoch = h->epoch + 1;
     h->ticket = 0;

@@ -17,8 +17,8 @@ namespace umim {
 
 struct PlanHeader {
   int32_t status;       // status word used when the caller passes no dev_status
-  int32_t epoch;        // call counter (rollback read-done flags)
-  int32_t ticket;       // next rollback unit
+  int32_t epoch;        // call counter
+  int32_t ticket;       // rollback grid-barrier arrivals
   int32_t done_ctas;    // rollback CTAs that finished
   int32_t total_units;  // rollback units this call (0 when skipped)
   int32_t blocks_done;  // plan blocks that finished
@@ -26,7 +26,8 @@ struct PlanHeader {
   int32_t skip;         // 1: the call found invalid input, write nothing
   int32_t total_rows;   // sum of compressed lengths
   int32_t max_dest;     // largest number of compacted pages of one sequence
-  int32_t pad[54];      // header is 256 bytes
+  int32_t n_active;     // sequences with compacted pages to write (rollback)
+  int32_t pad[53];      // header is 256 bytes
 };
 static_assert(sizeof(PlanHeader) == 256, "header size");
 
@@ -38,10 +39,11 @@ struct PlanArrays {
   int32_t *seq_Lp;      // [B]
   int32_t *first_page;  // [B]   first compacted page (rollback)
   int32_t *n_dest;      // [B]   compacted pages written per lane (rollback)
+  int32_t *active;      // [B]   the sequences with n_dest > 0, in order (rollback)
   int32_t *unit_base;   // [B+1] rollback units, prefix
   int32_t *row_base;    // [B+1] compressed rows, prefix (cu_seqlens)
   int32_t *freed_base;  // [B+1] released pages, prefix
-  int32_t *flags;       // [max units] rollback read-done flags
+  int32_t *flags;       // end of the plan: the caller's own data follows
 };
 
 // Bytes of the plan part of a workspace, 256-B aligned pieces.
@@ -50,7 +52,7 @@ inline size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 inline size_t plan_bytes(int B, int S) {
   size_t b = align256(sizeof(PlanHeader));
   b += 2 * align256(sizeof(int32_t) * (size_t)(S > 0 ? S : 1));
-  b += 4 * align256(sizeof(int32_t) * (size_t)(B > 0 ? B : 1));
+  b += 5 * align256(sizeof(int32_t) * (size_t)(B > 0 ? B : 1));
   b += 3 * align256(sizeof(int32_t) * (size_t)(B + 1));
   return b;
 }
@@ -73,6 +75,7 @@ inline PlanArrays plan_carve(void *ws, int B, int S) {
   a.seq_Lp = reinterpret_cast<int32_t *>(take(b4));
   a.first_page = reinterpret_cast<int32_t *>(take(b4));
   a.n_dest = reinterpret_cast<int32_t *>(take(b4));
+  a.active = reinterpret_cast<int32_t *>(take(b4));
   a.unit_base = reinterpret_cast<int32_t *>(take(b14));
   a.row_base = reinterpret_cast<int32_t *>(take(b14));
   a.freed_base = reinterpret_cast<int32_t *>(take(b14));

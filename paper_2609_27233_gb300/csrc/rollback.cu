@@ -2,18 +2,19 @@
 // (App. E "Decoding-Time Merging and KV-Cache Update", Fig. 2): each span's
 // k stored entries become one surrogate entry and later entries move left.
 //
-// Work unit = (sequence b, lane = layer x head group, compacted page p): the
-// 16 compacted entries j in [16p, 16p+16) of one layer and a group of KV
-// heads.  A unit copies its sources (kept entries t = j + r >= j, or the
-// surrogate rows) into shared memory, publishes "read done", waits until
-// every unit that reads old page p has published, then writes page p.
-// Because j <= t, the units that read old page p are unit p itself and lower
-// pages of the same (b, lane), i.e. smaller unit indices.  The launch is
-// cooperative (every CTA resident) and CTA c handles units c, c + grid,
-// c + 2 grid, ... in increasing order, publishing each as soon as its copies
-// land, so the smallest unpublished unit always makes progress: no deadlock,
-// no second pass, each moved byte read once and written once.  Every wait is
-// bounded (UMIM_ERR_TIMEOUT).
+// Work unit = one (layer, K|V, kv-head) 16 x D tile of one compacted page of
+// one sequence: its 16 entries j come from kept entries t = j + r >= j or
+// from surrogate rows, and it is written to the same physical page that held
+// old page j / 16.  Units are visited row by row (row = compacted page index,
+// over the sequences that have pages to write) in rounds: round r gives every
+// mover warp of the cooperative grid one unit, its loads land, a grid-wide
+// barrier follows, then its stores.  Because j <= t, the units that read a
+// unit's destination tile sit in the same column at the same or a lower row,
+// i.e. in the same or an earlier round, so every read of a location precedes
+// its write; and a round's loads read only tiles at or beyond their own rows,
+// which no earlier round writes, so round r + 1's loads are in flight while
+// round r waits at the barrier and stores.  One pass: each moved byte is read
+// once and written once.  The barrier wait is bounded (UMIM_ERR_TIMEOUT).
 #include <algorithm>
 
 #include "plan.cuh"
@@ -21,7 +22,7 @@
 namespace umim {
 namespace {
 
-constexpr int kMoveThreads = 256;
+constexpr int kMoveThreads = 256;   // 7 mover warps + 1 warp that runs the grid barrier
 constexpr int64_t kNoWrite = INT64_MIN;
 
 struct MoveArgs {
@@ -50,16 +51,6 @@ __device__ __forceinline__ int upper_index(const int32_t *key, int lo, int hi, i
   return l - 1;
 }
 
-__device__ __forceinline__ int find_seq(const int32_t *base, int B, int u) {
-  int l = 0, h = B;   // largest b with base[b] <= u
-  while (l < h) {
-    const int m = (l + h) >> 1;
-    if (base[m] <= u) l = m + 1;
-    else h = m;
-  }
-  return l - 1;
-}
-
 __device__ __forceinline__ uint4 ld_v4(const uint16_t *p) {
   uint4 v;
   asm volatile("ld.global.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
@@ -75,17 +66,16 @@ __device__ __forceinline__ void st_v4(uint16_t *p, uint4 v) {
 
 struct PageDesc {
   int64_t *src;    // [pages][16] source row offset within a layer (no head offset), -(i+1) for span i, kNoWrite
-  int2 *dep;       // [pages] range of compacted pages that read this old page
 };
 
-// One warp per (sequence, compacted page): where each of its 16 entries comes
-// from, and which compacted pages read the same page of the old layout.
+// Sixteen threads per (sequence, compacted page): where each of its 16
+// entries comes from (kNoWrite: the entry does not move).
 __global__ void __launch_bounds__(256) rollback_map_kernel(MoveArgs a, PlanArrays arr, PageDesc pd, int D) {
   griddep_wait();
   if (arr.hdr->skip) return;
   const int b = blockIdx.y;
-  const int k = blockIdx.x * 8 + (threadIdx.x >> 5);
-  const int lane = threadIdx.x & 31;
+  const int k = blockIdx.x * 16 + (threadIdx.x >> 4);
+  const int slot = threadIdx.x & 15;
   const int nd = arr.n_dest[b];
   if (k >= nd) return;
   const int p = arr.first_page[b] + k;
@@ -93,221 +83,210 @@ __global__ void __launch_bounds__(256) rollback_map_kernel(MoveArgs a, PlanArray
   const int lo = a.span_offsets[b], hi = a.span_offsets[b + 1];
   const int32_t *bt = a.block_table + (int64_t)b * a.max_pages;
   const int64_t page_stride = (int64_t)kPageSize * D * a.n_kv_heads * 2;
-  int dpage = -1;
-  if (lane < kPageSize) {
-    const int L = arr.seq_Lp[b];
-    const int j = p * kPageSize + lane;
-    int64_t src = kNoWrite;
-    if (j < L && j >= a.span_start[lo]) {
-      const int i = upper_index(arr.new_idx, lo, hi, j);
-      if (i >= lo) {
-        if (arr.new_idx[i] == j) {
-          src = -(int64_t)i - 1;
-        } else {
-          const int t = j + arr.r_incl[i];
-          if (t != j) src = (int64_t)bt[t / kPageSize] * page_stride + (t % kPageSize) * D;
-        }
-      }
-    }
-    pd.src[(int64_t)idx * kPageSize + lane] = src;
-  } else {
-    const int L = arr.seq_L[b];
-    const int t = p * kPageSize + (lane - kPageSize);
-    if (t < L) {
-      const int i = upper_index(a.span_start, lo, hi, t);
-      if (i >= lo && t >= a.span_start[i] + a.span_len[i]) {
-        const int r = arr.r_incl[i];
-        if (r > 0) dpage = (t - r) / kPageSize;
+  const int L = arr.seq_Lp[b];
+  const int j = p * kPageSize + slot;
+  int64_t src = kNoWrite;
+  if (j < L && j >= a.span_start[lo]) {
+    const int i = upper_index(arr.new_idx, lo, hi, j);
+    if (i >= lo) {
+      if (arr.new_idx[i] == j) {
+        src = -(int64_t)i - 1;
+      } else {
+        const int t = j + arr.r_incl[i];
+        if (t != j) src = (int64_t)bt[t / kPageSize] * page_stride + (t % kPageSize) * D;
       }
     }
   }
-  int mn = dpage < 0 ? 0x7fffffff : dpage, mx = dpage;
-#pragma unroll
-  for (int o = 8; o >= 1; o >>= 1) {
-    mn = min(mn, __shfl_xor_sync(0xffffffffu, mn, o));
-    mx = max(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+  pd.src[(int64_t)idx * kPageSize + slot] = src;
+}
+
+constexpr int kMovers = kMoveThreads / 32 - 1;
+constexpr int kSmemSeqs = 1024;   // active sequences whose plan values a CTA keeps in shared memory
+
+// Grid barrier in two halves, run by lane 0 of the CTA's barrier warp (which
+// has no loads of its own in flight, so its fence does not wait for them).
+// arrive: after a __syncthreads that follows every load of the round, count
+// this CTA in; wait: until every CTA has counted itself in for the round.
+__device__ __forceinline__ void grid_arrive(int32_t *count) {
+  __threadfence();   // the CTA's completed loads before the arrival
+  atomicAdd(count, 1);
+}
+__device__ __forceinline__ bool grid_wait(const int32_t *count, int target) {
+  if (ld_acquire(count) >= target) return true;
+  const uint64_t t0 = globaltimer();
+  while (true) {
+#pragma unroll 1
+    for (int i = 0; i < 64; ++i)
+      if (ld_acquire(count) >= target) return true;
+    if (globaltimer() - t0 > kWaitLimitNs) return false;
   }
-  if (lane == kPageSize) pd.dep[idx] = make_int2(mn, mx);
 }
 
-constexpr int kMovers = kMoveThreads / 32 - 1;   // mover warps per CTA; the last warp publishes
-
-__device__ __forceinline__ void st_release_cta_shared(int *p, int v) {
-  asm volatile("st.release.cta.shared.b32 [%0], %1;" ::"r"(smem_u32(p)), "r"(v) : "memory");
-}
-__device__ __forceinline__ int ld_acquire_cta_shared(const int *p) {
-  int v;
-  asm volatile("ld.acquire.cta.shared.b32 %0, [%1];" : "=r"(v) : "r"(smem_u32(p)) : "memory");
-  return v;
-}
-__device__ __forceinline__ void fence_acq_rel_gpu() { asm volatile("fence.acq_rel.gpu;" ::: "memory"); }
-__device__ __forceinline__ void st_relaxed_gpu(int32_t *p, int32_t v) {
-  asm volatile("st.relaxed.gpu.global.b32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
-}
-
-// One mover warp per unit = one (layer, K|V, head) 16 x D tile of a compacted
-// page.  Lane l moves 16-byte chunks c = l + 32 it of the tile: row c / CPR
-// (the slot), column c % CPR.  Units are visited page-row by page-row:
-// processing slot i covers compacted page k = i / (B * tiles) of sequence b
-// and tile t, (b, t) = divmod(i mod (B * tiles), tiles); slots with k beyond
-// the sequence's pages do nothing.  A unit waits only for units of earlier
-// rows, which were picked up at least a whole row of slots before it.  Mover m
-// of the grid handles slots m, m + M, m + 2M, ... (M movers).  When a unit's loads have returned, the mover
-// reports it in its shared-memory mailbox (CTA-scope release) and goes on to
-// wait for the units that read its destination page and to write it.  The
-// CTA's publisher warp collects reported units, issues one GPU-scope fence
-// for the whole batch and then marks their read-done flags: the fence orders
-// every reported load before every flag store that follows it, and movers
-// never pay for a GPU-scope fence themselves.
+// Mover warps: lane l moves 16-byte chunks c = l + 32 it of a tile, row
+// (slot) c / CPR, column c % CPR.  Step r: round r + 1's loads land and the
+// CTA arrives at barrier r + 1; then, while that barrier fills up, round r's
+// tile (barrier r has passed) is stored and round r + 2's loads are issued
+// into the registers it held; then barrier r + 1 is waited for.  A CTA
+// arrives at barrier r + 1 only after passing barrier r, so one counter of
+// arrivals serves every round: barrier r has passed once it reaches
+// (r + 1) x grid.
 template <int D>
-__global__ void __launch_bounds__(kMoveThreads, 4) rollback_move_kernel(MoveArgs a, PlanArrays arr, PageDesc pd) {
+__global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs a, PlanArrays arr, PageDesc pd) {
   constexpr int CPR = D / 8;                       // 16-byte chunks per row
   constexpr int PER_LANE = kPageSize * CPR / 32;   // 8 (D=128) or 4 (D=64)
-  constexpr int SLOT_STEP = 32 / CPR;              // slots advanced per it
+  constexpr int SLOT_STEP = 32 / CPR;              // rows advanced per it
+  constexpr int kHead = kPageSize * D;             // elements of one (K|V, head) tile
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
   const int nm = gridDim.x * kMovers;
   const int my_col = lane % CPR;
   const int my_slot0 = lane / CPR;
-  __shared__ int s_last;
-  __shared__ int s_mail[kMovers];   // units reported loaded by each mover (a count)
-  __shared__ int s_finished;        // movers that left their loop
+  __shared__ int s_last, s_abort;
+  __shared__ int s_sq[kSmemSeqs], s_nd[kSmemSeqs], s_ub[kSmemSeqs], s_fp[kSmemSeqs];
 
   const PlanHeader *hdr = arr.hdr;
   const int total = hdr->total_units;
-  const int epoch = hdr->epoch;
   const int Hkv = a.n_kv_heads;
-  const int64_t head_stride = (int64_t)kPageSize * D;
-  const int64_t kv_stride = head_stride * Hkv;
-  const int64_t page_stride = kv_stride * 2;
-  const int64_t layer_stride = page_stride * a.n_pages;
-  const int row_size = a.B * a.n_lanes;
-  const int64_t n_slots = total > 0 ? (int64_t)hdr->max_dest * row_size : 0;
+  const int64_t layer_stride = (int64_t)2 * kHead * Hkv * a.n_pages;
+  const int kv_stride32 = kHead * Hkv, page_stride32 = 2 * kHead * Hkv;
+  // a row holds the tiles of the sequences that have pages to write
+  const int n_active = total > 0 ? hdr->n_active : 0;
+  const int row_size = max(1, n_active * a.n_lanes);
+  // slot indices fit in 32 bits: batch x max_pages x tile lanes < 2^30 is checked on the host
+  const int max_dest = total > 0 ? hdr->max_dest : 0;
+  const int n_slots = max_dest * row_size;
+  const int rounds = (n_slots + nm - 1) / nm;
 
-  if (threadIdx.x < kMovers) s_mail[threadIdx.x] = 0;
-  if (threadIdx.x == 0) s_finished = 0;
+  if (threadIdx.x == 0) s_abort = 0;
+  // plan values of the active sequences (row position order), from shared
+  // memory when there are few enough of them
+  const bool seq_in_smem = n_active <= kSmemSeqs;
+  if (seq_in_smem) {
+    for (int j = threadIdx.x; j < n_active; j += blockDim.x) {
+      const int b = arr.active[j];
+      s_sq[j] = b;
+      s_nd[j] = arr.n_dest[b];
+      s_ub[j] = arr.unit_base[b];
+      s_fp[j] = arr.first_page[b];
+    }
+  }
   __syncthreads();
+  auto seq_of = [&](int j) { return seq_in_smem ? s_sq[j] : arr.active[j]; };
+  auto nd_of = [&](int j) { return seq_in_smem ? s_nd[j] : arr.n_dest[arr.active[j]]; };
+  auto ub_of = [&](int j) { return seq_in_smem ? s_ub[j] : arr.unit_base[arr.active[j]]; };
+  auto fp_of = [&](int j) { return seq_in_smem ? s_fp[j] : arr.first_page[arr.active[j]]; };
 
-  if (wid == kMovers) {
-    // ---- publisher ----
-    int published[kMovers];
+  // slot i = kk * row_size + pos, kk the compacted page row
+  struct Desc {
+    int valid, tl;
+    int64_t src;    // this lane's row source (lanes < 16)
+    int32_t page;   // destination physical page
+  };
+  auto describe = [&](int kk, int pos) {
+    Desc x{0, 0, kNoWrite, 0};
+    if (kk >= max_dest) return x;
+    const int j = pos / a.n_lanes, tl = pos - j * a.n_lanes;
+    if (kk >= nd_of(j)) return x;
+    const int b = seq_of(j);
+    const int idx = ub_of(j) / a.n_lanes + kk;
+    x.valid = 1;
+    x.tl = tl;
+    x.src = lane < kPageSize ? pd.src[(int64_t)idx * kPageSize + lane] : kNoWrite;
+    x.page = a.block_table[(int64_t)b * a.max_pages + fp_of(j) + kk];
+    return x;
+  };
+  const int step_kk = nm / row_size, step_pos = nm - step_kk * row_size;
+  auto advance = [&](int &kk, int &pos) {
+    kk += step_kk;
+    pos += step_pos;
+    if (pos >= row_size) {
+      pos -= row_size;
+      ++kk;
+    }
+  };
+  // a tile in registers, with where it goes
+  struct Tile {
+    uint4 v[PER_LANE];
+    uint32_t mask;
+    int64_t dst;
+  };
+  auto load = [&](const Desc &x, Tile &t) {
+    t.mask = 0;
+    t.dst = 0;
 #pragma unroll
-    for (int m = 0; m < kMovers; ++m) published[m] = 0;
-    uint64_t t_idle = globaltimer();
-    while (true) {
-      int mail[kMovers];
-      bool any = false;
-      // finished before the mailboxes: a mover's last report precedes its exit
-      const int fin = ld_acquire_cta_shared(&s_finished);
+    for (int it = 0; it < PER_LANE; ++it) t.v[it] = make_uint4(0, 0, 0, 0);
+    if (!x.valid) return;
+    const int layer = x.tl / (2 * Hkv), kv = (x.tl / Hkv) & 1, h = x.tl % Hkv;
+    const int64_t tile = layer * layer_stride + (int)(kv * kv_stride32 + h * kHead + my_col * 8);
+    const uint16_t *sur = kv ? a.sur_v : a.sur_k;
+    t.dst = tile + (int64_t)x.page * page_stride32;
 #pragma unroll
-      for (int m = 0; m < kMovers; ++m) {
-        mail[m] = ld_acquire_cta_shared(&s_mail[m]);
-        any |= mail[m] > published[m];
-      }
-      if (any) {
-        fence_acq_rel_gpu();   // every reported load happens before the flags below
-#pragma unroll
-        for (int m = 0; m < kMovers; ++m) {
-          const int mover = blockIdx.x * kMovers + m;
-          for (int k = published[m] + lane; k < mail[m]; k += 32) {
-            const int64_t i = mover + (int64_t)k * nm;
-            const int kk = (int)(i / row_size);
-            const int pos = (int)(i - (int64_t)kk * row_size);
-            const int b = pos / a.n_lanes, tl = pos % a.n_lanes;
-            const int nd = arr.n_dest[b];
-            if (kk < nd) st_relaxed_gpu(&arr.flags[arr.unit_base[b] + tl * nd + kk], epoch);
-          }
-          published[m] = mail[m];
-        }
-        t_idle = globaltimer();
-      } else if (fin == kMovers) {
-        break;
-      } else if (globaltimer() - t_idle > kWaitLimitNs) {
-        set_error(a.status, UMIM_ERR_TIMEOUT);
-        break;
-      } else {
-        __nanosleep(32);
+    for (int it = 0; it < PER_LANE; ++it) {
+      const int slot = my_slot0 + it * SLOT_STEP;
+      const int64_t src = __shfl_sync(0xffffffffu, x.src, slot);
+      if (src != kNoWrite) t.mask |= 1u << it;
+      if (src >= 0) {
+        t.v[it] = ld_v4(a.pool + tile + src);
+      } else if (src != kNoWrite) {
+        const int64_t si = -src - 1;
+        t.v[it] = ld_v4(sur + ((si * a.n_layers + layer) * Hkv + h) * D + my_col * 8);
       }
     }
-  } else {
-    // ---- mover ----
-    const int mover = blockIdx.x * kMovers + wid;
-    int k = 0;
-    for (int64_t i = mover; i < n_slots; i += nm, ++k) {
-      // slot -> (compacted page row kk, sequence, tile lane)
-      const int kk = (int)(i / row_size);
-      const int pos = (int)(i - (int64_t)kk * row_size);
-      const int b = pos / a.n_lanes, tl = pos % a.n_lanes;
-      const int nd = arr.n_dest[b];
-      if (kk >= nd) {
-        if (lane == 0) st_release_cta_shared(&s_mail[wid], k + 1);
-        continue;
-      }
-      const int u = arr.unit_base[b] + tl * nd + kk;
-      const int layer = tl / (2 * Hkv);
-      const int kv = (tl / Hkv) & 1;
-      const int h = tl % Hkv;
-      const int idx = arr.unit_base[b] / a.n_lanes + kk;
-      const int p = arr.first_page[b] + kk;
-      const int64_t my_src = lane < kPageSize ? pd.src[(int64_t)idx * kPageSize + lane] : kNoWrite;
-      const int2 dep = pd.dep[idx];
-      const int64_t tile = layer * layer_stride + kv * kv_stride + h * head_stride + my_col * 8;
-      const uint16_t *sur = kv ? a.sur_v : a.sur_k;
-
-      uint4 v[PER_LANE];
-      uint32_t write_mask = 0;
-      uint32_t fold = 0;
+  };
+  auto store = [&](const Tile &t) {
 #pragma unroll
-      for (int it = 0; it < PER_LANE; ++it) {
-        const int slot = my_slot0 + it * SLOT_STEP;
-        const int64_t src = __shfl_sync(0xffffffffu, my_src, slot);
-        if (src != kNoWrite) write_mask |= 1u << it;
-        v[it] = make_uint4(0, 0, 0, 0);
-        if (src >= 0) {
-          v[it] = ld_v4(a.pool + tile + src);
-        } else if (src != kNoWrite) {
-          const int64_t i = -src - 1;
-          v[it] = ld_v4(sur + ((i * a.n_layers + layer) * Hkv + h) * D + my_col * 8);
-        }
-        fold ^= v[it].x ^ v[it].y ^ v[it].z ^ v[it].w;
-      }
-      // every loaded value of this lane has arrived before the warp barrier
-      asm volatile("" ::"r"(fold) : "memory");
-      __syncwarp();
-      int ok = 1;
-      if (lane == 0) {
-        // report: units 0 .. k of this mover have been read
-        st_release_cta_shared(&s_mail[wid], k + 1);
-        // wait for the units that read this tile of old page p (smaller indices)
-        for (int q = dep.x; q <= dep.y && q >= 0 && q < p; ++q) {
-          const int uq = u - (p - q);
-          if (ld_acquire(&arr.flags[uq]) == epoch) continue;
-          const uint64_t t0 = globaltimer();
-          bool got = false;
-          while (!got) {
-#pragma unroll 1
-            for (int i = 0; i < 64 && !got; ++i) got = (ld_acquire(&arr.flags[uq]) == epoch);
-            if (!got && globaltimer() - t0 > kWaitLimitNs) break;
-          }
-          if (!got) {
-            set_error(a.status, UMIM_ERR_TIMEOUT);
-            ok = 0;
-            break;
-          }
-        }
-      }
-      ok = __shfl_sync(0xffffffffu, ok, 0);
-      if (!ok) break;
-      const int64_t dst = tile + (int64_t)a.block_table[(int64_t)b * a.max_pages + p] * page_stride;
-#pragma unroll
-      for (int it = 0; it < PER_LANE; ++it) {
-        const int slot = my_slot0 + it * SLOT_STEP;
-        if (write_mask & (1u << it)) st_v4(a.pool + dst + slot * D, v[it]);
-      }
+    for (int it = 0; it < PER_LANE; ++it) {
+      const int slot = my_slot0 + it * SLOT_STEP;
+      if (t.mask & (1u << it)) st_v4(a.pool + t.dst + slot * D, t.v[it]);
     }
-    __syncwarp();
-    if (lane == 0) {
-      __threadfence_block();   // the last report is visible before the exit count
-      atomicAdd(&s_finished, 1);
+  };
+  auto landed = [&](const Tile &t) {
+    uint32_t fold = 0;
+#pragma unroll
+    for (int it = 0; it < PER_LANE; ++it) fold ^= t.v[it].x ^ t.v[it].y ^ t.v[it].z ^ t.v[it].w;
+    asm volatile("" ::"r"(fold) : "memory");   // every loaded value of the tile has arrived
+  };
+  // barrier halves, CTA-wide: arrive after this CTA's loads of the round landed
+  auto arrive = [&]() {
+    __syncthreads();
+    if (wid == kMovers && lane == 0) grid_arrive(&arr.hdr->ticket);
+  };
+  auto wait = [&](int r) -> bool {
+    if (wid == kMovers && lane == 0 && !grid_wait(&arr.hdr->ticket, (r + 1) * (int)gridDim.x)) {
+      set_error(a.status, UMIM_ERR_TIMEOUT);
+      s_abort = 1;
+    }
+    __syncthreads();
+    return !s_abort;
+  };
+  // step r (tile r in `cur`, round r + 1's loads in flight in `next`, barrier r passed)
+  auto step = [&](int r, Tile &cur, Tile &next, Desc &d_next2, int &kk2, int &pos2) -> bool {
+    landed(next);                 // round r + 1's loads
+    arrive();                     // barrier r + 1
+    store(cur);                   // round r
+    load(d_next2, cur);           // round r + 2 into the registers just stored
+    d_next2 = describe(kk2, pos2);
+    advance(kk2, pos2);
+    return wait(r + 1);
+  };
+
+  // the barrier warp takes a slot past the end: it describes, loads and stores nothing
+  const int mover = wid < kMovers ? blockIdx.x * kMovers + wid : n_slots + nm;
+  int kk = mover / row_size, pos = mover - kk * row_size;   // round 0
+  Tile A, B;
+  load(describe(kk, pos), A);                                // round 0
+  advance(kk, pos);
+  load(describe(kk, pos), B);                                // round 1
+  advance(kk, pos);
+  Desc d_next2 = describe(kk, pos);                          // round 2
+  advance(kk, pos);
+  if (rounds > 0) {
+    landed(A);
+    arrive();
+    if (wait(0)) {
+      for (int r = 0; r < rounds; r += 2) {
+        if (!step(r, A, B, d_next2, kk, pos)) break;
+        if (r + 1 < rounds && !step(r + 1, B, A, d_next2, kk, pos)) break;
+      }
     }
   }
 
@@ -345,10 +324,10 @@ __global__ void __launch_bounds__(kMoveThreads, 4) rollback_move_kernel(MoveArgs
 
 size_t kv_rollback_workspace_bytes(int B, int S, int max_pages, int n_layers, int n_kv_heads, int head_dim) {
   (void)head_dim;
-  const size_t units = (size_t)B * n_layers * 2 * n_kv_heads * (size_t)max_pages;
+  (void)n_layers;
+  (void)n_kv_heads;
   const size_t pages = (size_t)B * max_pages;
-  return plan_bytes(B, S) + align256(sizeof(int32_t) * (units > 0 ? units : 1)) +
-         align256(sizeof(int64_t) * kPageSize * (pages > 0 ? pages : 1)) + align256(sizeof(int2) * (pages > 0 ? pages : 1));
+  return plan_bytes(B, S) + align256(sizeof(int64_t) * kPageSize * (pages > 0 ? pages : 1));
 }
 
 umim_status kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t max_pages, int32_t *seq_lens,
@@ -360,13 +339,8 @@ umim_status kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t m
   const int lanes = kv->n_layers * 2 * kv->n_kv_heads;   // one unit per (layer, K|V, head) tile
   PlanArrays arr = plan_carve(ws, B, S);
   int32_t *status = dev_status ? dev_status : &arr.hdr->status;
-  const size_t units = (size_t)B * lanes * (size_t)max_pages;
-  const size_t pages = (size_t)B * max_pages;
   PageDesc pd;
-  pd.src = reinterpret_cast<int64_t *>(reinterpret_cast<char *>(arr.flags) +
-                                       align256(sizeof(int32_t) * (units > 0 ? units : 1)));
-  pd.dep = reinterpret_cast<int2 *>(reinterpret_cast<char *>(pd.src) +
-                                    align256(sizeof(int64_t) * kPageSize * (pages > 0 ? pages : 1)));
+  pd.src = reinterpret_cast<int64_t *>(arr.flags);   // the page descriptions follow the plan
 
   PlanArgs pa{};
   pa.seq_lens = seq_lens;
@@ -412,7 +386,7 @@ umim_status kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t m
     per_sm = 1;
   const int grid = std::max(1, num_sms) * per_sm;   // every CTA resident (cooperative launch)
   trace_mark(stream, "rollback.map");
-  if (launch_pdl(rollback_map_kernel, dim3((unsigned)std::max(1, ceil_div(max_pages, 8)), (unsigned)B), dim3(256), 0,
+  if (launch_pdl(rollback_map_kernel, dim3((unsigned)std::max(1, ceil_div(max_pages, 16)), (unsigned)B), dim3(256), 0,
                  stream, ma, arr, pd, (int)D) != cudaSuccess)
     return UMIM_ERR_CUDA;
   trace_mark(stream, "rollback.move");
