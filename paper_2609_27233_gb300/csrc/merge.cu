@@ -2,8 +2,9 @@
 //   gather     E   = rows of the embedding table for every span token
 //   GEMM1      H   = GELU(E W_kv^T + b_kv)        tcgen05, fp16 out + row stats of the fp32 values
 //   pool       P   = LN_kv(H);  a_i = softmax(P_i q_i / sqrt(d_h));  o_i = a_i^T P_i
-//   GEMM2      Z   = GELU(o W_o^T + b_o)          tcgen05 on fp16 operands, fp32 out + row stats
-//   LN_o       z   = LN_o(Z)                      in place in the output
+//   GEMM2      Z   = GELU(o W_o^T + b_o)          tcgen05 on fp16 operands, fp16 out + row stats
+//                                                 of the fp32 values
+//   LN_o       z   = LN_o(Z)                      fp32 into the output
 //
 // The two d x d projections are the only dense contractions of the module
 // and run on the 5th-generation tensor cores: operands staged by TMA in
@@ -22,7 +23,7 @@ namespace umim {
 namespace {
 
 constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4;
-constexpr int kGemmThreads = 192;   // warp 0: TMA, warp 1: MMA + TMEM owner, warps 2-5: epilogue
+constexpr int kGemmThreads = 224;   // warp 0: TMA, warp 1: MMA + TMEM owner, warps 2-5: epilogue, warp 6: side job
 constexpr int kStageBytes = (BM + BN) * BK * 2;
 constexpr int kGemmSmem = STAGES * kStageBytes + 1024;
 
@@ -43,6 +44,10 @@ struct GemmArgs {
   const __nv_bfloat16 *bias;   // [N]
   OutT *out;                   // [M][N]
   float2 *stats;               // [M][N / BN]
+  // side job of warp 6: bf16 -> fp16 of cvt_n 16-byte vectors (0: none)
+  const uint4 *cvt_in;
+  uint4 *cvt_out;
+  int64_t cvt_n;
   int32_t *status;
 };
 
@@ -50,12 +55,6 @@ struct GemmArgs {
 // (n fastest, so CTAs running at the same time share the A block in L2).
 // The accumulator is double-buffered in tensor memory (2 x 256 columns):
 // while the epilogue warps drain tile i, the MMA thread accumulates tile i+1.
-__device__ __forceinline__ void store32(float *dst, const float (&v)[32]) {
-  float4 *d4 = reinterpret_cast<float4 *>(dst);
-#pragma unroll
-  for (int i = 0; i < 8; ++i) d4[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
-}
-
 __device__ __forceinline__ void store32(__half *dst, const float (&v)[32]) {
   uint4 *d4 = reinterpret_cast<uint4 *>(dst);
 #pragma unroll
@@ -162,6 +161,31 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           tc_commit(&empty_bar[s]);
         }
         tc_commit(&acc_full[buf]);
+      }
+    }
+  } else if (warp == 6) {
+    // side job, converted while the tensor cores work (the memory traffic is
+    // small next to the tile loads), 8 loads in flight per lane
+    const int64_t step = (int64_t)gridDim.x * 32;
+    for (int64_t i0 = (int64_t)blockIdx.x * 32 + lane; i0 < g.cvt_n; i0 += 8 * step) {
+      uint4 u[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        const int64_t i = i0 + k * step;
+        if (i < g.cvt_n) u[k] = __ldg(g.cvt_in + i);
+      }
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        const int64_t i = i0 + k * step;
+        if (i < g.cvt_n) {
+          float f[8];
+          bf16x8_to_float(u[k], f);
+          uint4 o;
+          __half2 *hh = reinterpret_cast<__half2 *>(&o);
+#pragma unroll
+          for (int e = 0; e < 4; ++e) hh[e] = __floats2half2_rn(f[2 * e], f[2 * e + 1]);
+          g.cvt_out[i] = o;
+        }
       }
     }
   } else {
@@ -530,29 +554,35 @@ __global__ void __launch_bounds__(kPoolConsumers + 32, CH <= 2 ? 2 : 1)
 }
 
 // ---------------------------------------------------------------------------
-// LN_o in place over rows of Z, one warp per row
+// LN_o over rows of Z (fp16, the GELU output of the projection; its row
+// statistics were taken from the fp32 values), one warp per row, z in fp32
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(256)
-    ln_rows_kernel(float *Z, const float2 *stats, int S, int d, const __nv_bfloat16 *gamma,
+    ln_rows_kernel(const __half *Z, float *out, const float2 *stats, int S, int d, const __nv_bfloat16 *gamma,
                    const __nv_bfloat16 *beta, float eps) {
   griddep_wait();
   const int r = blockIdx.x * 8 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (r >= S) return;
   const float2 m = row_moments_warp(stats + (int64_t)r * (d / BN), d / BN, d, eps);
-  float *row = Z + (int64_t)r * d;
-#pragma unroll 4
-  for (int c = lane * 4; c < d; c += 128) {
-    float4 x = *reinterpret_cast<float4 *>(row + c);
-    const __nv_bfloat162 *g2 = reinterpret_cast<const __nv_bfloat162 *>(gamma + c);
-    const __nv_bfloat162 *b2 = reinterpret_cast<const __nv_bfloat162 *>(beta + c);
-    const float2 g0 = __bfloat1622float2(g2[0]), g1 = __bfloat1622float2(g2[1]);
-    const float2 b0 = __bfloat1622float2(b2[0]), b1 = __bfloat1622float2(b2[1]);
-    x.x = (x.x - m.x) * m.y * g0.x + b0.x;
-    x.y = (x.y - m.x) * m.y * g0.y + b0.y;
-    x.z = (x.z - m.x) * m.y * g1.x + b1.x;
-    x.w = (x.w - m.x) * m.y * g1.y + b1.y;
-    *reinterpret_cast<float4 *>(row + c) = x;
+  const __half *row = Z + (int64_t)r * d;
+  float *dst = out + (int64_t)r * d;
+#pragma unroll 2
+  for (int c = lane * 8; c < d; c += 256) {
+    const uint4 u = *reinterpret_cast<const uint4 *>(row + c);
+    const __half2 *h2 = reinterpret_cast<const __half2 *>(&u);
+    float g[8], b[8];
+    bf16x8_to_float(*reinterpret_cast<const uint4 *>(gamma + c), g);
+    bf16x8_to_float(*reinterpret_cast<const uint4 *>(beta + c), b);
+    float y[8];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const float2 x = __half22float2(h2[e]);
+      y[2 * e] = (x.x - m.x) * m.y * g[2 * e] + b[2 * e];
+      y[2 * e + 1] = (x.y - m.x) * m.y * g[2 * e + 1] + b[2 * e + 1];
+    }
+    *reinterpret_cast<float4 *>(dst + c) = make_float4(y[0], y[1], y[2], y[3]);
+    *reinterpret_cast<float4 *>(dst + c + 4) = make_float4(y[4], y[5], y[6], y[7]);
   }
 }
 
@@ -584,7 +614,7 @@ EncodeTiledFn get_encode_tiled();
 size_t merge_spans_workspace_bytes(int64_t T, int S, int d) {
   const int nt = d / BN;
   size_t b = 0;
-  b += al1k((size_t)std::max<int64_t>(T, 1) * d * 2);          // E (bf16)
+  b += al1k((size_t)std::max<int64_t>(std::max<int64_t>(T, S), 1) * d * 2);   // E (bf16), later Z (fp16)
   b += al1k((size_t)std::max<int64_t>(T, 1) * d * 2);          // H (fp16)
   b += al1k((size_t)std::max<int64_t>(T, 1) * nt * 8);         // stats of H
   b += al1k((size_t)std::max(S, 1) * d * 2);                   // o (fp16)
@@ -609,7 +639,8 @@ static bool encode_kmajor(EncodeTiledFn enc, CUtensorMap *map, const void *base,
 template <typename OutT>
 static umim_status launch_gemm(EncodeTiledFn enc, const void *A, int64_t M, const void *Bw, int d, bool fp16,
                                const void *bias, OutT *out, float2 *stats, int32_t *status, cudaStream_t st,
-                               const char *label, int num_sms) {
+                               const char *label, int num_sms, const void *cvt_in = nullptr, void *cvt_out = nullptr,
+                               int64_t cvt_n = 0) {
   CUtensorMap am, bm;
   if (!encode_kmajor(enc, &am, A, M, d, BM, fp16) || !encode_kmajor(enc, &bm, Bw, d, d, BN, fp16))
     return UMIM_ERR_CUDA;
@@ -621,6 +652,9 @@ static umim_status launch_gemm(EncodeTiledFn enc, const void *A, int64_t M, cons
   g.bias = static_cast<const __nv_bfloat16 *>(bias);
   g.out = out;
   g.stats = stats;
+  g.cvt_in = static_cast<const uint4 *>(cvt_in);
+  g.cvt_out = static_cast<uint4 *>(cvt_out);
+  g.cvt_n = cvt_n;
   g.status = status;
   static bool attr_done = false;
   if (!attr_done) {
@@ -646,7 +680,8 @@ umim_status merge_spans(const void *embeddings, int64_t vocab, const int32_t *to
   const int d = w->d_model, nt = d / BN;
   char *p = static_cast<char *>(workspace);
   __nv_bfloat16 *E = reinterpret_cast<__nv_bfloat16 *>(p);
-  p += al1k((size_t)std::max<int64_t>(T, 1) * d * 2);
+  __half *Z16 = reinterpret_cast<__half *>(p);   // E is dead once GEMM1 has run
+  p += al1k((size_t)std::max<int64_t>(std::max<int64_t>(T, S), 1) * d * 2);
   __half *H = reinterpret_cast<__half *>(p);
   p += al1k((size_t)std::max<int64_t>(T, 1) * d * 2);
   float2 *st1 = reinterpret_cast<float2 *>(p);
@@ -658,13 +693,22 @@ umim_status merge_spans(const void *embeddings, int64_t vocab, const int32_t *to
   float2 *st2 = reinterpret_cast<float2 *>(p);
 
   if (S == 0) return UMIM_OK;
+  bool wo_in_gemm1 = false;
   if (T > 0) {
     const int blocks = std::max(1, std::min<int>((int)((T + 7) / 8), num_sms * 8));
     trace_mark(st, "merge.gather");
     if (launch_pdl(gather_rows_kernel, dim3(blocks), dim3(256), 0, st, static_cast<const uint4 *>(embeddings), vocab,
                    token_ids, T, d, reinterpret_cast<uint4 *>(E), status) != cudaSuccess)
       return UMIM_ERR_CUDA;
-    umim_status r = launch_gemm(enc, E, T, w->w_kv, d, false, w->b_kv, H, st1, status, st, "merge.gemm1", num_sms);
+    // W_o -> fp16 rides along in a side warp of GEMM1 when its share is small
+    // next to the tiles its CTA computes; else a kernel of its own
+    const int64_t tiles1 = (int64_t)(d / BN) * ((T + BM - 1) / BM);
+    const int64_t grid1 = std::min<int64_t>(tiles1, std::max(1, num_sms));
+    const int64_t n_vec = (int64_t)d * d / 8;
+    wo_in_gemm1 = n_vec <= 128 * 32 * grid1 * (tiles1 / grid1);
+    umim_status r = launch_gemm(enc, E, T, w->w_kv, d, false, w->b_kv, H, st1, status, st, "merge.gemm1", num_sms,
+                                wo_in_gemm1 ? w->w_o : nullptr, wo_in_gemm1 ? Wo16 : nullptr,
+                                wo_in_gemm1 ? n_vec : 0);
     if (r != UMIM_OK) return r;
   }
   trace_mark(st, "merge.pool");
@@ -683,15 +727,18 @@ umim_status merge_spans(const void *embeddings, int64_t vocab, const int32_t *to
                  static_cast<const __nv_bfloat16 *>(w->ln_kv_beta), static_cast<const __nv_bfloat16 *>(w->query),
                  w->ln_eps, O, status) != cudaSuccess)
     return UMIM_ERR_CUDA;
-  trace_mark(st, "merge.wo_f16");
-  if (launch_pdl(bf16_to_f16_kernel, dim3(std::max(1, num_sms) * 4), dim3(256), 0, st,
-                 static_cast<const uint4 *>(w->w_o), reinterpret_cast<uint4 *>(Wo16), (int64_t)d * d / 8) !=
-      cudaSuccess)
-    return UMIM_ERR_CUDA;
-  umim_status r = launch_gemm(enc, O, S, Wo16, d, true, w->b_o, surrogates, st2, status, st, "merge.gemm2", num_sms);
+  if (!wo_in_gemm1) {
+    trace_mark(st, "merge.wo_f16");
+    if (launch_pdl(bf16_to_f16_kernel, dim3(std::max(1, num_sms) * 4), dim3(256), 0, st,
+                   static_cast<const uint4 *>(w->w_o), reinterpret_cast<uint4 *>(Wo16), (int64_t)d * d / 8) !=
+        cudaSuccess)
+      return UMIM_ERR_CUDA;
+  }
+  umim_status r = launch_gemm(enc, O, S, Wo16, d, true, w->b_o, Z16, st2, status, st, "merge.gemm2", num_sms);
   if (r != UMIM_OK) return r;
   trace_mark(st, "merge.ln_o");
-  if (launch_pdl(ln_rows_kernel, dim3((S + 7) / 8), dim3(256), 0, st, surrogates, (const float2 *)st2, S, d,
+  if (launch_pdl(ln_rows_kernel, dim3((S + 7) / 8), dim3(256), 0, st, (const __half *)Z16, surrogates,
+                 (const float2 *)st2, S, d,
                  static_cast<const __nv_bfloat16 *>(w->ln_o_gamma), static_cast<const __nv_bfloat16 *>(w->ln_o_beta),
                  w->ln_eps) != cudaSuccess)
     return UMIM_ERR_CUDA;
