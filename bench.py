@@ -633,6 +633,13 @@ def serving_bench(args):
     surs = [sl.surrogates(s, len(plan[s]["st"]), dev) for s in range(sl.steps)]
     qs = [sl.q(0, layer, dev) for layer in range(NL)]
     d_plan = [dict(new_pages=t(x["new_pages"]), offs=t(x["offs"]), st=t(x["st"]), ln=t(x["ln"])) for x in plan]
+    for x, dp in zip(plan, d_plan):
+        # the same merges as per-sequence (k, surrogate row) for the fused call
+        mk, mr = np.zeros(B, np.int32), np.full(B, -1, np.int32)
+        for b in range(B):
+            if x["offs"][b + 1] > x["offs"][b]:
+                mk[b], mr[b] = x["ln"][x["offs"][b]], x["offs"][b]
+        dp["merge_k"], dp["merge_row"] = t(mk), t(mr)
     status = umim.new_status(dev)
     max_pages = sl.block_table.shape[1]
     ws_r = umim.workspace(umim.umim_kv_rollback_workspace_size(B, B, max_pages, NL, sl.n_kv_heads, sl.head_dim),
@@ -640,15 +647,21 @@ def serving_bench(args):
     ws_a = umim.workspace(umim.umim_decode_attention_workspace_size(B, sl.n_q_heads, sl.n_kv_heads,
                                                                     sl.head_dim), dev)
     freed = torch.empty(B * max_pages, dtype=torch.int32, device=dev)
+    released = torch.empty(B, dtype=torch.int32, device=dev)
     outs = [torch.empty_like(qs[0]) for _ in range(NL)]
+    fused = [False]
 
     def step(s):
         nk, nv = entries[s]
         dp = d_plan[s]
-        umim.umim_kv_append(pool, bt, lens, nk, nv, dp["new_pages"], dev_status=status)
         sk, sv = surs[s]
-        umim.umim_kv_rollback(pool, bt, lens, dp["offs"], dp["st"], dp["ln"], sk, sv, freed_pages=freed,
-                              workspace_buf=ws_r, dev_status=status)
+        if fused[0]:
+            umim.umim_decode_append_merge(pool, bt, lens, nk, nv, dp["new_pages"], dp["merge_k"], dp["merge_row"],
+                                          sk, sv, released=released, dev_status=status)
+        else:
+            umim.umim_kv_append(pool, bt, lens, nk, nv, dp["new_pages"], dev_status=status)
+            umim.umim_kv_rollback(pool, bt, lens, dp["offs"], dp["st"], dp["ln"], sk, sv, freed_pages=freed,
+                                  workspace_buf=ws_r, dev_status=status)
         for layer in range(NL):
             umim.umim_decode_attention(qs[layer], pool, layer, bt, lens, out=outs[layer], workspace_buf=ws_a,
                                        dev_status=status)
@@ -694,6 +707,20 @@ def serving_bench(args):
     kern = {}
     for lab, v in recs:
         kern.setdefault(lab, []).append(v)
+    # the same loop with the append and the merge in one call per step
+    fused[0] = True
+    reset()
+    f_ms = run()
+    umim.check_status(status, "fused loop")
+    assert np.array_equal(lens.cpu().numpy(), plan[-1]["lens_after"]), "fused loop: lengths differ"
+    reset()
+    umim.trace_start(200 * sl.steps)
+    run()
+    umim.trace_stop()
+    f_kern = {}
+    for lab, v in umim.trace_read(200 * sl.steps):
+        f_kern.setdefault(lab, []).append(v)
+    fused[0] = False
     entry = 2 * sl.n_kv_heads * sl.head_dim * 2
     att_bytes = sum(float(x["lens_after"].sum()) * entry + 2 * B * sl.n_q_heads * sl.head_dim * 2
                     for x in plan) * NL
@@ -715,7 +742,12 @@ def serving_bench(args):
             "kernels": {k: {"launches": len(v), "ms_total": round(float(np.sum(v)), 3),
                             "us_mean": round(1000 * float(np.mean(v)), 2)} for k, v in
                         sorted(kern.items(), key=lambda x: -np.sum(x[1]))},
-            "gpu_launches": len(recs), "clocks": clocks, "traced_ms_per_step": tms / sl.steps}
+            "gpu_launches": len(recs), "clocks": clocks, "traced_ms_per_step": tms / sl.steps,
+            "fused_append_merge": {
+                "value": B * sl.steps / (f_ms / 1000.0), "unit": "tokens/s", "ms_per_step": f_ms / sl.steps,
+                "kernels": {k: {"launches": len(v), "ms_total": round(float(np.sum(v)), 3),
+                                "us_mean": round(1000 * float(np.mean(v)), 2)} for k, v in
+                            sorted(f_kern.items(), key=lambda x: -np.sum(x[1]))}}}
     print(json.dumps(line))
     return 0
 

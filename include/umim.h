@@ -236,6 +236,44 @@ umim_status umim_kv_append(const umim_paged_kv *kv, int32_t *block_table, int32_
                            int32_t *dev_status, cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
+ * Decode step with decoding-time merging (App. E "Decoding-Time Merging and
+ * KV-Cache Update"; Fig. 2 steps (2) and (3)): after each generated token
+ * the recent suffix is checked against the merge rules; without a match the
+ * token's KV entry is appended, with a match the n-gram's cached entries are
+ * cropped and the surrogate's single KV entry takes their place.  One call
+ * does both for a batch, in place, per sequence b with L = seq_lens[b]:
+ *   merge_k[b] == 0 (or merge_k NULL): new_k/new_v[b] are appended at slot L
+ *     exactly as umim_kv_append does (new_pages[b] opens the page when
+ *     L % 16 == 0);
+ *   merge_k[b] = k in [1, 16]: the new token and the k - 1 stored entries
+ *     before it form the merged span, so surrogate row merge_row[b] is
+ *     written at slot s = L + 1 - k in every layer, seq_lens[b] becomes
+ *     s + 1, and the one page that no longer holds an entry, if any (the
+ *     page the append would have opened included), is set to -1 in the block
+ *     table and reported in released_pages[b] (-1 otherwise).
+ * The result is identical to umim_kv_append followed by umim_kv_rollback of
+ * the suffix spans (s, k); no entry moves, since a suffix has nothing after
+ * it.  k counts stored entries after the append, i.e. the paper's n.
+ *
+ * new_k/new_v       device bf16 [batch][n_layers][n_kv_heads][head_dim]
+ * new_pages         device int32 [batch] or NULL (read at page boundaries)
+ * merge_k           device int32 [batch] or NULL (no merges)
+ * merge_row         device int32 [batch]: row of the surrogate arrays for a
+ *                   merging sequence
+ * surrogate_k/v     device bf16 [n_merge_rows][n_layers][n_kv_heads][head_dim]
+ * released_pages    device int32 [batch] out, or NULL
+ * No workspace.  Device-side errors: UMIM_ERR_INVALID_ARG, and that sequence
+ * is left unchanged, when seq_lens[b] is outside [0, 16*max_pages), k is
+ * outside [0, min(16, L + 1)], merge_row[b] is outside [0, n_merge_rows), or
+ * a page to write is outside [0, n_pages).
+ * ------------------------------------------------------------------------ */
+umim_status umim_decode_append_merge(const umim_paged_kv *kv, int32_t *block_table, int32_t max_pages,
+                                     int32_t *seq_lens, int32_t batch, const void *new_k, const void *new_v,
+                                     const int32_t *new_pages, const int32_t *merge_k, const int32_t *merge_row,
+                                     int32_t n_merge_rows, const void *surrogate_k, const void *surrogate_v,
+                                     int32_t *released_pages, int32_t *dev_status, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
  * Grouped-query decode attention over the (compacted) paged cache, one
  * query token per sequence (App. I.1; the backbone's ordinary attention):
  *   out[b][h] = sum_{j < seq_lens[b]} softmax_j(scale <q[b][h], K[b][g][j]>) V[b][g][j]

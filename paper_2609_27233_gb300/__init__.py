@@ -9,6 +9,7 @@ points keep the C names:
   umim_build_compressed   compressed prompt embeddings + positions (App. E, App. C.5)
   umim_kv_rollback        KV-cache rollback and in-place compaction (App. E, Fig. 2)
   umim_kv_append          decode-step append of one KV entry per layer (App. E, Fig. 2)
+  umim_decode_append_merge  append or suffix merge per sequence in one call (App. E decoding loop)
   umim_decode_attention   GQA decode attention over the compacted paged cache (App. I.1)
 """
 import ctypes
@@ -184,6 +185,26 @@ def umim_kv_append(pool, block_table, seq_lens, new_k, new_v, new_pages=None, de
     code = lib().umim_kv_append(ctypes.byref(kv), _p(block_table), max_pages, _p(seq_lens), B, _p(new_k),
                                 _p(new_v), _p(new_pages), _p(dev_status), _stream(stream))
     _check(code, "umim_kv_append")
+
+
+def umim_decode_append_merge(pool, block_table, seq_lens, new_k, new_v, new_pages=None, merge_k=None,
+                             merge_row=None, surrogate_k=None, surrogate_v=None, released=None, dev_status=None,
+                             stream=None):
+    """In place: append new_k/new_v [B][n_layers][Hkv][D] to every sequence,
+    or, where merge_k[b] = k > 0, write surrogate row merge_row[b] in place of
+    the last k entries (the new one included).  Returns released [B] int32
+    (the page a merge freed, or -1)."""
+    kv = paged_kv(pool)
+    B, max_pages = block_table.shape
+    if released is None:
+        released = torch.empty(B, dtype=torch.int32, device=pool.device)
+    n_rows = 0 if surrogate_k is None else surrogate_k.shape[0]
+    code = lib().umim_decode_append_merge(ctypes.byref(kv), _p(block_table), max_pages, _p(seq_lens), B, _p(new_k),
+                                          _p(new_v), _p(new_pages), _p(merge_k), _p(merge_row), n_rows,
+                                          _p(surrogate_k), _p(surrogate_v), _p(released), _p(dev_status),
+                                          _stream(stream))
+    _check(code, "umim_decode_append_merge")
+    return released
 
 
 def umim_decode_attention(q, pool, layer, block_table, seq_lens, scale=0.0, out=None, workspace_buf=None,

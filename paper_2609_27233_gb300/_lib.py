@@ -46,6 +46,8 @@ SIGNATURES = {
                                         c_ptr, c_i32, c_ptr, c_ptr, c_ptr, c_ptr, c_size, c_ptr, c_ptr]),
     "umim_kv_append": (ctypes.c_int, [ctypes.POINTER(PagedKVC), c_ptr, c_i32, c_ptr, c_i32, c_ptr, c_ptr, c_ptr,
                                       c_ptr, c_ptr]),
+    "umim_decode_append_merge": (ctypes.c_int, [ctypes.POINTER(PagedKVC), c_ptr, c_i32, c_ptr, c_i32, c_ptr, c_ptr,
+                                                c_ptr, c_ptr, c_ptr, c_i32, c_ptr, c_ptr, c_ptr, c_ptr, c_ptr]),
     "umim_decode_attention_workspace_size": (c_size, [c_i32, c_i32, c_i32, c_i32]),
     "umim_decode_attention": (ctypes.c_int, [c_ptr, c_i32, ctypes.POINTER(PagedKVC), c_i32, c_ptr, c_i32,
                                              c_ptr, c_i32, ctypes.c_float, c_ptr, c_ptr, c_size, c_ptr,

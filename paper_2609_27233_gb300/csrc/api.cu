@@ -41,6 +41,9 @@ umim_status kv_rollback(const umim_paged_kv *, int32_t *, int32_t, int32_t *, in
                         size_t, int32_t *, cudaStream_t, int);
 umim_status kv_append(const umim_paged_kv *, int32_t *, int32_t, int32_t *, int32_t, const void *, const void *,
                       const int32_t *, int32_t *, cudaStream_t);
+umim_status decode_append_merge(const umim_paged_kv *, int32_t *, int32_t, int32_t *, int32_t, const void *,
+                                const void *, const int32_t *, const int32_t *, const int32_t *, int32_t, const void *,
+                                const void *, int32_t *, int32_t *, cudaStream_t);
 size_t decode_attention_workspace_bytes(int B, int Hq, int Hkv, int D, int num_sms);
 umim_status decode_attention(const void *, int, const umim_paged_kv *, int, const int32_t *, int, const int32_t *,
                              int, float, void *, void *, int32_t *, cudaStream_t, int);
@@ -204,6 +207,24 @@ umim_status umim_kv_append(const umim_paged_kv *kv, int32_t *block_table, int32_
   if (!aligned(new_k, 16) || !aligned(new_v, 16)) return UMIM_ERR_INVALID_ARG;
   prepare_device(stream);
   return kv_append(kv, block_table, max_pages, seq_lens, batch, new_k, new_v, new_pages, dev_status, stream);
+}
+
+umim_status umim_decode_append_merge(const umim_paged_kv *kv, int32_t *block_table, int32_t max_pages,
+                                     int32_t *seq_lens, int32_t batch, const void *new_k, const void *new_v,
+                                     const int32_t *new_pages, const int32_t *merge_k, const int32_t *merge_row,
+                                     int32_t n_merge_rows, const void *surrogate_k, const void *surrogate_v,
+                                     int32_t *released_pages, int32_t *dev_status, cudaStream_t stream) {
+  if (!kv_ok(kv) || batch < 0 || max_pages < 0 || n_merge_rows < 0) return UMIM_ERR_INVALID_ARG;
+  if (!kv_supported(kv)) return UMIM_ERR_UNSUPPORTED;
+  if ((int64_t)batch * max_pages > INT32_MAX / 16) return UMIM_ERR_UNSUPPORTED;
+  if (batch == 0) return UMIM_OK;
+  if (!block_table || !seq_lens || !new_k || !new_v) return UMIM_ERR_INVALID_ARG;
+  if (!aligned(new_k, 16) || !aligned(new_v, 16)) return UMIM_ERR_INVALID_ARG;
+  if (merge_k && n_merge_rows > 0 && (!merge_row || !surrogate_k || !surrogate_v)) return UMIM_ERR_INVALID_ARG;
+  if (n_merge_rows > 0 && (!aligned(surrogate_k, 16) || !aligned(surrogate_v, 16))) return UMIM_ERR_INVALID_ARG;
+  prepare_device(stream);
+  return decode_append_merge(kv, block_table, max_pages, seq_lens, batch, new_k, new_v, new_pages, merge_k,
+                             merge_row, n_merge_rows, surrogate_k, surrogate_v, released_pages, dev_status, stream);
 }
 
 size_t umim_decode_attention_workspace_size(int32_t batch, int32_t n_q_heads, int32_t n_kv_heads,

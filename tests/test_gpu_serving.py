@@ -4,7 +4,8 @@ Every step appends one KV entry per sequence and layer (umim_kv_append),
 then each sequence with probability p merges its last k stored entries, the
 new one included, into one surrogate entry (umim_kv_rollback of a suffix
 span, App. E), then decode attention runs for every layer
-(umim_decode_attention).
+(umim_decode_attention).  Each loop also runs with the append and the merge
+fused into one umim_decode_append_merge call.
 
 * Small loops: the oracle replays the same steps on a host copy of the cache
   and everything is compared after every step: block tables, lengths, freed
@@ -47,11 +48,13 @@ def _spans(rolls, lens, B):
 
 
 class GpuLoop:
-    """The CUDA path: the library's three calls on device buffers."""
+    """The CUDA path: the library's three calls on device buffers, or with
+    fused=True the append and the suffix merge in one umim_decode_append_merge
+    call (the released pages then come back one per sequence)."""
 
-    def __init__(self, sl, dv):
+    def __init__(self, sl, dv, fused=False):
         self.m = umim()
-        self.sl, self.dv = sl, dv
+        self.sl, self.dv, self.fused = sl, dv, fused
         self.pool = sl.init_pool(dv)
         self.bt = torch.from_numpy(sl.block_table.copy()).to(dv)
         self.lens = torch.from_numpy(sl.lens.copy()).to(dv)
@@ -63,16 +66,33 @@ class GpuLoop:
         self.at_ws = self.m.workspace(self.m.umim_decode_attention_workspace_size(
             B, sl.n_q_heads, sl.n_kv_heads, sl.head_dim), dv)
         self.freed = torch.empty(B * max_pages, dtype=torch.int32, device=dv)
+        self.released = torch.empty(B, dtype=torch.int32, device=dv)
 
     def step(self, step, new_pages, offs, st, ln):
         m, sl, dv = self.m, self.sl, self.dv
         nk, nv = sl.new_entries(step, dv)
+        if self.fused:
+            B = len(offs) - 1
+            merge_k = np.zeros(B, np.int32)
+            merge_row = np.full(B, -1, np.int32)
+            for b in range(B):
+                if offs[b + 1] > offs[b]:
+                    merge_k[b], merge_row[b] = ln[offs[b]], offs[b]
+            sk, sv = sl.surrogates(step, len(st), dv)
+            t = lambda x: torch.from_numpy(x).to(dv)
+            m.umim_decode_append_merge(self.pool, self.bt, self.lens, nk, nv, t(new_pages), t(merge_k), t(merge_row),
+                                       sk, sv, released=self.released, dev_status=self.status)
+            return self._attend(step)
         m.umim_kv_append(self.pool, self.bt, self.lens, nk, nv, torch.from_numpy(new_pages).to(dv),
                          dev_status=self.status)
         sk, sv = sl.surrogates(step, len(st), dv)
         m.umim_kv_rollback(self.pool, self.bt, self.lens, torch.from_numpy(offs).to(dv),
                            torch.from_numpy(st).to(dv), torch.from_numpy(ln).to(dv), sk, sv,
                            freed_pages=self.freed, workspace_buf=self.rb_ws, dev_status=self.status)
+        return self._attend(step)
+
+    def _attend(self, step):
+        m, sl, dv = self.m, self.sl, self.dv
         outs = []
         for layer in range(sl.n_layers):
             outs.append(m.umim_decode_attention(sl.q(step, layer, dv), self.pool, layer, self.bt, self.lens,
@@ -85,23 +105,28 @@ def _check_indices(g, o_bt, o_lens, o_freed, step):
     assert int(g.status.item()) == 0, f"step {step}: device status {int(g.status.item())}"
     np.testing.assert_array_equal(g.bt.cpu().numpy(), o_bt, err_msg=f"step {step}")
     np.testing.assert_array_equal(g.lens.cpu().numpy(), o_lens, err_msg=f"step {step}")
+    if g.fused:
+        r = g.released.cpu().numpy()
+        assert r[r >= 0].tolist() == list(o_freed), f"step {step}"
+        return
     f = g.freed.cpu().numpy()
     assert f[:len(o_freed)].tolist() == list(o_freed), f"step {step}"
     if len(o_freed) < len(f):
         assert f[len(o_freed)] == -1
 
 
+@pytest.mark.parametrize("fused", [False, True], ids=["three_calls", "fused"])
 @pytest.mark.parametrize("seed,B,layers,hq,hkv,d,steps,p", [
     (31, 6, 3, 16, 4, 128, 40, 0.3),
     (32, 5, 2, 8, 2, 64, 36, 0.5),
 ])
-def test_small_serving_loop_matches_oracle_every_step(seed, B, layers, hq, hkv, d, steps, p):
+def test_small_serving_loop_matches_oracle_every_step(seed, B, layers, hq, hkv, d, steps, p, fused):
     lens = W.rng(seed).integers(1, 200, size=B).astype(np.int32)
     lens[0] = 16
     sl = W.serving_loop(seed, B=B, n_layers=layers, n_q_heads=hq, n_kv_heads=hkv, head_dim=d, steps=steps, p=p,
                         lens=lens)
     dv = dev()
-    g = GpuLoop(sl, dv)
+    g = GpuLoop(sl, dv, fused)
     # every tensor is drawn on the GPU's generator and copied to the host for the oracle
     o_pool = W.bits(sl.init_pool(dv))
     o_bt, o_lens = sl.block_table.copy(), sl.lens.copy()
@@ -179,11 +204,12 @@ def _materialise(ids, layer, dv, init_layer, draw):
     return out
 
 
-def test_full_serving_workload_matches_oracle():
+@pytest.mark.parametrize("fused", [False, True], ids=["three_calls", "fused"])
+def test_full_serving_workload_matches_oracle(fused):
     sl = W.serving_loop(W.SEEDS["serving"], B=128, n_layers=32, n_q_heads=32, n_kv_heads=8, head_dim=128,
                         steps=256, p=0.1)
     dv = dev()
-    g = GpuLoop(sl, dv)
+    g = GpuLoop(sl, dv, fused)
     B = sl.B
     o_pool = _id_pool(sl)
     o_bt, o_lens = sl.block_table.copy(), sl.lens.copy()
