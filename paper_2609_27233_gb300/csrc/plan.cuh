@@ -18,7 +18,7 @@ namespace umim {
 struct PlanHeader {
   int32_t status;       // status word used when the caller passes no dev_status
   int32_t epoch;        // call counter
-  int32_t ticket;       // rollback grid-barrier arrivals
+  int32_t ticket;       // rollback: set when a mover gave up waiting
   int32_t done_ctas;    // rollback CTAs that finished
   int32_t total_units;  // rollback units this call (0 when skipped)
   int32_t blocks_done;  // plan blocks that finished

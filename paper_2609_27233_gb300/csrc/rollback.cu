@@ -5,16 +5,21 @@
 // Work unit = one (layer, K|V, kv-head) 16 x D tile of one compacted page of
 // one sequence: its 16 entries j come from kept entries t = j + r >= j or
 // from surrogate rows, and it is written to the same physical page that held
-// old page j / 16.  Units are visited row by row (row = compacted page index,
-// over the sequences that have pages to write) in rounds: round r gives every
-// mover warp of the cooperative grid one unit, its loads land, a grid-wide
-// barrier follows, then its stores.  Because j <= t, the units that read a
-// unit's destination tile sit in the same column at the same or a lower row,
-// i.e. in the same or an earlier round, so every read of a location precedes
-// its write; and a round's loads read only tiles at or beyond their own rows,
-// which no earlier round writes, so round r + 1's loads are in flight while
-// round r waits at the barrier and stores.  One pass: each moved byte is read
-// once and written once.  The barrier wait is bounded (UMIM_ERR_TIMEOUT).
+// old page j / 16.  Units are numbered row by row (row = compacted page
+// index, over the sequences that have pages to write) and dealt round-robin
+// to the mover warps of a cooperative grid; each warp loads two units ahead
+// of its stores.  A unit may overwrite its page once every unit that reads
+// that old page has its loads landed.  Because j <= t, the readers of old
+// page p are the units of the same sequence at compacted rows whose entries
+// come from p: at most two rows, both at or before p's own row (a unit reads
+// and writes only its own (layer, K|V, head) column, so within p's row the
+// reader is the unit itself).  So every unit counts itself into its row's
+// "landed" counter when its loads have arrived (release), and waits (acquire,
+// bounded) for the counters of its page's reader rows before it stores.
+// Every wait is for units numbered before the waiting one, each warp takes
+// its units in increasing order and all warps are resident, so the earliest
+// unstored unit can always proceed: no deadlock, and no grid-wide barrier.
+// One pass: each moved byte is read once and written once.
 #include <algorithm>
 
 #include "plan.cuh"
@@ -22,7 +27,8 @@
 namespace umim {
 namespace {
 
-constexpr int kMoveThreads = 256;   // 7 mover warps + 1 warp that runs the grid barrier
+constexpr int kMoveThreads = 256;   // 8 mover warps
+constexpr int kMovers = kMoveThreads / 32;
 constexpr int64_t kNoWrite = INT64_MIN;
 
 struct MoveArgs {
@@ -64,12 +70,25 @@ __device__ __forceinline__ void st_v4(uint16_t *p, uint4 v) {
                : "memory");
 }
 
+__device__ __forceinline__ void red_release_add(int32_t *p, int32_t v) {
+  asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+// Per compacted row (global row index over the active sequences).
+struct RowDep {
+  int32_t lo, hi;   // reader rows of this row's old page that precede it (lo > hi: none)
+  int32_t landed;   // units of this row whose loads have arrived (n_lanes: all)
+  int32_t pad;
+};
+
 struct PageDesc {
-  int64_t *src;    // [pages][16] source row offset within a layer (no head offset), -(i+1) for span i, kNoWrite
+  int64_t *src;    // [rows][16] source row offset within a layer (no head offset), -(i+1) for span i, kNoWrite
+  RowDep *dep;     // [rows]
 };
 
 // Sixteen threads per (sequence, compacted page): where each of its 16
-// entries comes from (kNoWrite: the entry does not move).
+// entries comes from (kNoWrite: the entry does not move), and which
+// compacted rows read the old entries of the page.
 __global__ void __launch_bounds__(256) rollback_map_kernel(MoveArgs a, PlanArrays arr, PageDesc pd, int D) {
   griddep_wait();
   if (arr.hdr->skip) return;
@@ -77,59 +96,73 @@ __global__ void __launch_bounds__(256) rollback_map_kernel(MoveArgs a, PlanArray
   const int k = blockIdx.x * 16 + (threadIdx.x >> 4);
   const int slot = threadIdx.x & 15;
   const int nd = arr.n_dest[b];
-  if (k >= nd) return;
-  const int p = arr.first_page[b] + k;
-  const int idx = arr.unit_base[b] / a.n_lanes + k;
-  const int lo = a.span_offsets[b], hi = a.span_offsets[b + 1];
-  const int32_t *bt = a.block_table + (int64_t)b * a.max_pages;
-  const int64_t page_stride = (int64_t)kPageSize * D * a.n_kv_heads * 2;
-  const int L = arr.seq_Lp[b];
-  const int j = p * kPageSize + slot;
+  const bool row_ok = k < nd;
   int64_t src = kNoWrite;
-  if (j < L && j >= a.span_start[lo]) {
-    const int i = upper_index(arr.new_idx, lo, hi, j);
-    if (i >= lo) {
-      if (arr.new_idx[i] == j) {
-        src = -(int64_t)i - 1;
-      } else {
-        const int t = j + arr.r_incl[i];
-        if (t != j) src = (int64_t)bt[t / kPageSize] * page_stride + (t % kPageSize) * D;
+  int rd_lo = INT32_MAX, rd_hi = -1;
+  int idx = 0;
+  if (row_ok) {
+    const int fp = arr.first_page[b];
+    const int p = fp + k;
+    idx = arr.unit_base[b] / a.n_lanes + k;
+    const int lo = a.span_offsets[b], hi = a.span_offsets[b + 1];
+    const int32_t *bt = a.block_table + (int64_t)b * a.max_pages;
+    const int64_t page_stride = (int64_t)kPageSize * D * a.n_kv_heads * 2;
+    const int j = p * kPageSize + slot;
+    if (j < arr.seq_Lp[b] && j >= a.span_start[lo]) {
+      const int i = upper_index(arr.new_idx, lo, hi, j);
+      if (i >= lo) {
+        if (arr.new_idx[i] == j) {
+          src = -(int64_t)i - 1;
+        } else {
+          const int t = j + arr.r_incl[i];
+          if (t != j) src = (int64_t)bt[t / kPageSize] * page_stride + (t % kPageSize) * D;
+        }
+      }
+    }
+    // the old entry t in this slot of page p: the compacted row that reads it
+    const int t = j;
+    if (t < arr.seq_L[b]) {
+      const int i = upper_index(a.span_start, lo, hi, t);
+      if (i >= lo && t >= a.span_start[i] + a.span_len[i] && arr.r_incl[i] > 0) {
+        rd_lo = rd_hi = (t - arr.r_incl[i]) / kPageSize - fp;
       }
     }
   }
+  for (int o = 8; o > 0; o >>= 1) {   // over the row's 16 slots
+    rd_lo = min(rd_lo, __shfl_xor_sync(0xffffffffu, rd_lo, o, 16));
+    rd_hi = max(rd_hi, __shfl_xor_sync(0xffffffffu, rd_hi, o, 16));
+  }
+  if (!row_ok) return;
   pd.src[(int64_t)idx * kPageSize + slot] = src;
-}
-
-constexpr int kMovers = kMoveThreads / 32 - 1;
-constexpr int kSmemSeqs = 1024;   // active sequences whose plan values a CTA keeps in shared memory
-
-// Grid barrier in two halves, run by lane 0 of the CTA's barrier warp (which
-// has no loads of its own in flight, so its fence does not wait for them).
-// arrive: after a __syncthreads that follows every load of the round, count
-// this CTA in; wait: until every CTA has counted itself in for the round.
-__device__ __forceinline__ void grid_arrive(int32_t *count) {
-  __threadfence();   // the CTA's completed loads before the arrival
-  atomicAdd(count, 1);
-}
-__device__ __forceinline__ bool grid_wait(const int32_t *count, int target) {
-  if (ld_acquire(count) >= target) return true;
-  const uint64_t t0 = globaltimer();
-  while (true) {
-#pragma unroll 1
-    for (int i = 0; i < 64; ++i)
-      if (ld_acquire(count) >= target) return true;
-    if (globaltimer() - t0 > kWaitLimitNs) return false;
+  if (slot == 0) {
+    rd_hi = min(rd_hi, k - 1);   // the row itself reads only its own units' columns
+    RowDep d;
+    d.lo = rd_lo <= rd_hi ? idx - k + rd_lo : 1;
+    d.hi = rd_lo <= rd_hi ? idx - k + rd_hi : 0;
+    d.landed = 0;
+    d.pad = 0;
+    pd.dep[idx] = d;
   }
 }
 
-// Mover warps: lane l moves 16-byte chunks c = l + 32 it of a tile, row
-// (slot) c / CPR, column c % CPR.  Step r: round r + 1's loads land and the
-// CTA arrives at barrier r + 1; then, while that barrier fills up, round r's
-// tile (barrier r has passed) is stored and round r + 2's loads are issued
-// into the registers it held; then barrier r + 1 is waited for.  A CTA
-// arrives at barrier r + 1 only after passing barrier r, so one counter of
-// arrivals serves every round: barrier r has passed once it reaches
-// (r + 1) x grid.
+constexpr int kSmemSeqs = 1024;   // active sequences whose plan values a CTA keeps in shared memory
+
+// Waits until *cnt >= target; false when it gave up (time limit, or another
+// warp gave up: *abort != 0).
+__device__ __forceinline__ bool wait_landed(const int32_t *cnt, int target, const int32_t *abort) {
+  const uint64_t t0 = globaltimer();
+  while (true) {
+#pragma unroll 1
+    for (int i = 0; i < 32; ++i)
+      if (ld_acquire(cnt) >= target) return true;
+    if (ld_acquire(abort) != 0 || globaltimer() - t0 > kWaitLimitNs) return false;
+  }
+}
+
+// Mover warps: lane l moves 16-byte chunks c = l + 32 it of a unit, row
+// (slot) c / CPR, column c % CPR.  Step: the next unit's loads land and it is
+// counted in; this unit waits for its page's readers and is stored; the unit
+// after next is loaded into its registers.
 template <int D>
 __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs a, PlanArrays arr, PageDesc pd) {
   constexpr int CPR = D / 8;                       // 16-byte chunks per row
@@ -140,23 +173,22 @@ __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs
   const int nm = gridDim.x * kMovers;
   const int my_col = lane % CPR;
   const int my_slot0 = lane / CPR;
-  __shared__ int s_last, s_abort;
+  __shared__ int s_last;
   __shared__ int s_sq[kSmemSeqs], s_nd[kSmemSeqs], s_ub[kSmemSeqs], s_fp[kSmemSeqs];
 
   const PlanHeader *hdr = arr.hdr;
+  int32_t *abort_flag = &arr.hdr->ticket;
   const int total = hdr->total_units;
   const int Hkv = a.n_kv_heads;
   const int64_t layer_stride = (int64_t)2 * kHead * Hkv * a.n_pages;
   const int kv_stride32 = kHead * Hkv, page_stride32 = 2 * kHead * Hkv;
-  // a row holds the tiles of the sequences that have pages to write
+  // a row holds the units of the sequences that have pages to write
   const int n_active = total > 0 ? hdr->n_active : 0;
   const int row_size = max(1, n_active * a.n_lanes);
-  // slot indices fit in 32 bits: batch x max_pages x tile lanes < 2^30 is checked on the host
+  // unit indices fit in 32 bits: batch x max_pages x tile lanes < 2^30 is checked on the host
   const int max_dest = total > 0 ? hdr->max_dest : 0;
   const int n_slots = max_dest * row_size;
-  const int rounds = (n_slots + nm - 1) / nm;
 
-  if (threadIdx.x == 0) s_abort = 0;
   // plan values of the active sequences (row position order), from shared
   // memory when there are few enough of them
   const bool seq_in_smem = n_active <= kSmemSeqs;
@@ -175,54 +207,41 @@ __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs
   auto ub_of = [&](int j) { return seq_in_smem ? s_ub[j] : arr.unit_base[arr.active[j]]; };
   auto fp_of = [&](int j) { return seq_in_smem ? s_fp[j] : arr.first_page[arr.active[j]]; };
 
-  // slot i = kk * row_size + pos, kk the compacted page row
-  struct Desc {
-    int valid, tl;
-    int64_t src;    // this lane's row source (lanes < 16)
-    int32_t page;   // destination physical page
-  };
-  auto describe = [&](int kk, int pos) {
-    Desc x{0, 0, kNoWrite, 0};
-    if (kk >= max_dest) return x;
-    const int j = pos / a.n_lanes, tl = pos - j * a.n_lanes;
-    if (kk >= nd_of(j)) return x;
-    const int b = seq_of(j);
-    const int idx = ub_of(j) / a.n_lanes + kk;
-    x.valid = 1;
-    x.tl = tl;
-    x.src = lane < kPageSize ? pd.src[(int64_t)idx * kPageSize + lane] : kNoWrite;
-    x.page = a.block_table[(int64_t)b * a.max_pages + fp_of(j) + kk];
-    return x;
-  };
-  const int step_kk = nm / row_size, step_pos = nm - step_kk * row_size;
-  auto advance = [&](int &kk, int &pos) {
-    kk += step_kk;
-    pos += step_pos;
-    if (pos >= row_size) {
-      pos -= row_size;
-      ++kk;
-    }
-  };
-  // a tile in registers, with where it goes
+  // a unit in registers, with where it goes and what it waits for
   struct Tile {
     uint4 v[PER_LANE];
     uint32_t mask;
+    int valid;
     int64_t dst;
+    int32_t row, dlo, dhi;
   };
-  auto load = [&](const Desc &x, Tile &t) {
+  // slot i = kk * row_size + pos, kk the compacted page row
+  auto load = [&](int kk, int pos, Tile &t) {
     t.mask = 0;
+    t.valid = 0;
     t.dst = 0;
+    t.row = 0;
+    t.dlo = 1;
+    t.dhi = 0;
 #pragma unroll
     for (int it = 0; it < PER_LANE; ++it) t.v[it] = make_uint4(0, 0, 0, 0);
-    if (!x.valid) return;
-    const int layer = x.tl / (2 * Hkv), kv = (x.tl / Hkv) & 1, h = x.tl % Hkv;
+    if (kk >= max_dest) return;
+    const int j = pos / a.n_lanes, tl = pos - j * a.n_lanes;
+    if (kk >= nd_of(j)) return;
+    const int b = seq_of(j);
+    const int idx = ub_of(j) / a.n_lanes + kk;
+    const int64_t my_src = lane < kPageSize ? pd.src[(int64_t)idx * kPageSize + lane] : kNoWrite;
+    const int page = a.block_table[(int64_t)b * a.max_pages + fp_of(j) + kk];
+    const int layer = tl / (2 * Hkv), kv = (tl / Hkv) & 1, h = tl % Hkv;
     const int64_t tile = layer * layer_stride + (int)(kv * kv_stride32 + h * kHead + my_col * 8);
     const uint16_t *sur = kv ? a.sur_v : a.sur_k;
-    t.dst = tile + (int64_t)x.page * page_stride32;
+    t.valid = 1;
+    t.row = idx;
+    t.dst = tile + (int64_t)page * page_stride32;
 #pragma unroll
     for (int it = 0; it < PER_LANE; ++it) {
       const int slot = my_slot0 + it * SLOT_STEP;
-      const int64_t src = __shfl_sync(0xffffffffu, x.src, slot);
+      const int64_t src = __shfl_sync(0xffffffffu, my_src, slot);
       if (src != kNoWrite) t.mask |= 1u << it;
       if (src >= 0) {
         t.v[it] = ld_v4(a.pool + tile + src);
@@ -231,6 +250,8 @@ __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs
         t.v[it] = ld_v4(sur + ((si * a.n_layers + layer) * Hkv + h) * D + my_col * 8);
       }
     }
+    t.dlo = pd.dep[idx].lo;
+    t.dhi = pd.dep[idx].hi;
   };
   auto store = [&](const Tile &t) {
 #pragma unroll
@@ -239,58 +260,64 @@ __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs
       if (t.mask & (1u << it)) st_v4(a.pool + t.dst + slot * D, t.v[it]);
     }
   };
-  auto landed = [&](const Tile &t) {
+  // the unit's loads have arrived; count it into its row
+  auto land_and_count = [&](const Tile &t) {
     uint32_t fold = 0;
 #pragma unroll
     for (int it = 0; it < PER_LANE; ++it) fold ^= t.v[it].x ^ t.v[it].y ^ t.v[it].z ^ t.v[it].w;
-    asm volatile("" ::"r"(fold) : "memory");   // every loaded value of the tile has arrived
+    asm volatile("" ::"r"(fold) : "memory");
+    __syncwarp();
+    if (t.valid && lane == 0) red_release_add(&pd.dep[t.row].landed, 1);
   };
-  // barrier halves, CTA-wide: arrive after this CTA's loads of the round landed
-  auto arrive = [&]() {
-    __syncthreads();
-    if (wid == kMovers && lane == 0) grid_arrive(&arr.hdr->ticket);
-  };
-  auto wait = [&](int r) -> bool {
-    if (wid == kMovers && lane == 0 && !grid_wait(&arr.hdr->ticket, (r + 1) * (int)gridDim.x)) {
-      set_error(a.status, UMIM_ERR_TIMEOUT);
-      s_abort = 1;
-    }
-    __syncthreads();
-    return !s_abort;
-  };
-  // step r (tile r in `cur`, round r + 1's loads in flight in `next`, barrier r passed)
-  auto step = [&](int r, Tile &cur, Tile &next, Desc &d_next2, int &kk2, int &pos2) -> bool {
-    landed(next);                 // round r + 1's loads
-    arrive();                     // barrier r + 1
-    store(cur);                   // round r
-    load(d_next2, cur);           // round r + 2 into the registers just stored
-    d_next2 = describe(kk2, pos2);
-    advance(kk2, pos2);
-    return wait(r + 1);
+  // every reader of the unit's old page has its loads landed
+  auto readers_done = [&](const Tile &t) -> bool {
+    for (int rw = t.dlo; rw <= t.dhi; ++rw)
+      if (!wait_landed(&pd.dep[rw].landed, a.n_lanes, abort_flag)) return false;
+    return true;
   };
 
-  // the barrier warp takes a slot past the end: it describes, loads and stores nothing
-  const int mover = wid < kMovers ? blockIdx.x * kMovers + wid : n_slots + nm;
-  int kk = mover / row_size, pos = mover - kk * row_size;   // round 0
+  const int mover = blockIdx.x * kMovers + wid;
+  const int my_units = mover < n_slots ? (n_slots - 1 - mover) / nm + 1 : 0;
+  const int step_kk = nm / row_size, step_pos = nm - step_kk * row_size;
+  int kk = mover / row_size, pos = mover - kk * row_size;
+  auto advance = [&]() {
+    kk += step_kk;
+    pos += step_pos;
+    if (pos >= row_size) {
+      pos -= row_size;
+      ++kk;
+    }
+  };
   Tile A, B;
-  load(describe(kk, pos), A);                                // round 0
-  advance(kk, pos);
-  load(describe(kk, pos), B);                                // round 1
-  advance(kk, pos);
-  Desc d_next2 = describe(kk, pos);                          // round 2
-  advance(kk, pos);
-  if (rounds > 0) {
-    landed(A);
-    arrive();
-    if (wait(0)) {
-      for (int r = 0; r < rounds; r += 2) {
-        if (!step(r, A, B, d_next2, kk, pos)) break;
-        if (r + 1 < rounds && !step(r + 1, B, A, d_next2, kk, pos)) break;
+  if (my_units > 0) {
+    load(kk, pos, A);
+    advance();
+    load(kk, pos, B);
+    advance();
+    land_and_count(A);
+    // unit u in `cur` (landed, counted), unit u + 1 in flight in `next`
+    auto step = [&](Tile &cur, Tile &next) -> bool {
+      land_and_count(next);
+      if (!readers_done(cur)) return false;
+      store(cur);
+      load(kk, pos, cur);   // unit u + 2
+      advance();
+      return true;
+    };
+    for (int u = 0; u < my_units; u += 2) {
+      bool ok = step(A, B);
+      if (ok && u + 1 < my_units) ok = step(B, A);
+      if (!ok) {
+        if (lane == 0) {
+          set_error(a.status, UMIM_ERR_TIMEOUT);
+          atomicExch(abort_flag, 1);
+        }
+        break;
       }
     }
   }
 
-  // ---- the last CTA to finish truncates block tables and updates lengths ----
+// ---- the last CTA to finish truncates block tables and updates lengths ----
   const int tid = threadIdx.x;
   __syncthreads();
   if (tid == 0) {
@@ -326,8 +353,8 @@ size_t kv_rollback_workspace_bytes(int B, int S, int max_pages, int n_layers, in
   (void)head_dim;
   (void)n_layers;
   (void)n_kv_heads;
-  const size_t pages = (size_t)B * max_pages;
-  return plan_bytes(B, S) + align256(sizeof(int64_t) * kPageSize * (pages > 0 ? pages : 1));
+  const size_t pages = (size_t)B * max_pages > 0 ? (size_t)B * max_pages : 1;
+  return plan_bytes(B, S) + align256(sizeof(int64_t) * kPageSize * pages) + align256(sizeof(RowDep) * pages);
 }
 
 umim_status kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t max_pages, int32_t *seq_lens,
@@ -341,6 +368,8 @@ umim_status kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t m
   int32_t *status = dev_status ? dev_status : &arr.hdr->status;
   PageDesc pd;
   pd.src = reinterpret_cast<int64_t *>(arr.flags);   // the page descriptions follow the plan
+  const size_t pages = (size_t)B * max_pages > 0 ? (size_t)B * max_pages : 1;
+  pd.dep = reinterpret_cast<RowDep *>(reinterpret_cast<char *>(pd.src) + align256(sizeof(int64_t) * kPageSize * pages));
 
   PlanArgs pa{};
   pa.seq_lens = seq_lens;
