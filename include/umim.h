@@ -312,7 +312,7 @@ umim_status umim_decode_attention(const void *q, int32_t n_q_heads, const umim_p
  *  - Arguments and results are those of umim_decode_attention, without the
  *    workspace.  It allocates nothing and calls no allocating routine.
  *  - A batch whose scratch would exceed the array (about
- *    (batch * n_kv_heads + 8 * SMs) * 16 * (head_dim + 2) * 4 bytes) is
+ *    (batch * n_kv_heads + 12 * SMs) * 16 * (head_dim + 2) * 4 bytes) is
  *    rejected with UMIM_ERR_WORKSPACE before anything is launched.
  *  - The first call on a device looks up the array's device address
  *    (cudaGetSymbolAddress) and the SM count; make that first call before

@@ -176,6 +176,7 @@ __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs
   __shared__ int s_last;
   __shared__ int s_sq[kSmemSeqs], s_nd[kSmemSeqs], s_ub[kSmemSeqs], s_fp[kSmemSeqs];
 
+  griddep_wait();
   const PlanHeader *hdr = arr.hdr;
   int32_t *abort_flag = &arr.hdr->ticket;
   const int total = hdr->total_units;
@@ -419,10 +420,21 @@ umim_status kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t m
                  stream, ma, arr, pd, (int)D) != cudaSuccess)
     return UMIM_ERR_CUDA;
   trace_mark(stream, "rollback.move");
-  void *args[] = {&ma, &arr, &pd};
-  if (cudaLaunchCooperativeKernel(reinterpret_cast<const void *>(kern), dim3(grid), dim3(kMoveThreads), args,
-                                  (size_t)smem, stream) != cudaSuccess)
-    return UMIM_ERR_CUDA;
+  // cooperative (every CTA resident), and allowed to launch while the map
+  // kernel finishes (the kernel waits for it before reading the plan)
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(kMoveThreads);
+  cfg.dynamicSmemBytes = (size_t)smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  if (cudaLaunchKernelEx(&cfg, kern, ma, arr, pd) != cudaSuccess) return UMIM_ERR_CUDA;
   trace_mark(stream, nullptr);
   return cudaGetLastError() == cudaSuccess ? UMIM_OK : UMIM_ERR_CUDA;
 }
