@@ -22,6 +22,14 @@ for indices and moved KV bytes:
                           ("Compressed-position convention")
   spans.span_metadata     removed-position count r(t) and compressed index
                           pi(t) = t - r(t) of App. J.4
+  rules.match_prompt / match_prompts
+                          App. E ("Rule Matching", "Prompt Merging"):
+                          left-to-right, longest-first n-gram matching
+  rules.SuffixState / match_suffixes
+                          App. E ("Decoding-Time Merging"): longest-first
+                          test of the raw generated suffix after every token
+  rules.lookup            App. E (potential engineering optimizations):
+                          surrogates precomputed per rule, fetched by id
 
 bf16 values are represented by their raw bit patterns (numpy uint16) and
 upcast exactly to float64.
@@ -32,8 +40,13 @@ Parity status per function (what pins it is in tests/test_oracle_*.py):
   kv_append         pinned (logical-list model, rollback identities)
   decode_attention  pinned (library SDPA, closed forms, invariants)
   build_compressed  pinned (worked example, length formula, library bf16)
+  match_prompt(s)   pinned (worked example, independent greedy-condition
+                    checker, closed forms)
+  SuffixState       pinned (worked example, list model with markers,
+                    equality with prompt matching for 2-gram rules)
+  lookup            pinned (equals merging the matched spans)
 """
-from . import bf16, spans, merge, rollback, append, attention, compaction  # noqa: F401
+from . import bf16, spans, merge, rollback, append, attention, compaction, rules  # noqa: F401
 from .merge import merge_spans, merge_span_reference_steps  # noqa: F401
 from .rollback import kv_rollback  # noqa: F401
 from .append import kv_append  # noqa: F401
