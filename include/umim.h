@@ -300,6 +300,117 @@ umim_status umim_decode_attention(const void *q, int32_t n_q_heads, const umim_p
                                   size_t workspace_bytes, int32_t *dev_status, cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
+ * Merge rules (App. E "Rule Matching").  A rule is a token n-gram, n in
+ * {2, 3, 4}; its rule id is its row in the list given to umim_rules_build.
+ * The table is open addressing over 16-byte slots (the n-gram packed as four
+ * 24-bit token ids, and the rule id) in a caller-owned device buffer.
+ *
+ * umim_rule_table_bytes: buffer size for n_rules rules (a power of two times
+ * 16 bytes, at least 24 * n_rules: load factor <= 2/3; 64 MB for the 2.2
+ * million rules of a Llama-3 rule set, which then stays in L2).
+ *
+ * umim_rules_build: fills the table.
+ * table         device, table_bytes (16 times a power of two, >= 24 *
+ *               n_rules and >= 256), 16-B aligned; overwritten
+ * rule_tokens   device int32 [n_rules][4], 16-B aligned: the n token ids of
+ *               a rule (each in [0, 0xFFFFFF)) followed by 4 - n entries -1
+ * Device-side errors: UMIM_ERR_INVALID_ARG when a rule row is malformed or
+ * an n-gram occurs twice (the table is then not usable).  Token ids are
+ * limited to 24 bits (every published vocabulary fits).
+ * ------------------------------------------------------------------------ */
+size_t umim_rule_table_bytes(int64_t n_rules);
+
+umim_status umim_rules_build(void *table, size_t table_bytes, const int32_t *rule_tokens, int64_t n_rules,
+                             int32_t *dev_status, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Prompt merging's span selection (App. E "Rule Matching", "Prompt
+ * Merging"): each prompt is scanned from left to right; at a position the
+ * 4-, 3- and then 2-gram starting there is tested and the first that is a
+ * rule becomes a span, the scan continuing after it; otherwise the scan moves
+ * on by one token.  Output: the spans as the CSR that umim_build_compressed
+ * takes, each span's rule id (the row of a surrogate lookup table), and
+ * optionally the span tokens as the CSR that umim_merge_spans takes.
+ *
+ * token_ids       device int32 [batch][max_len]; tokens past a prompt's
+ *                 length are not read
+ * prompt_lens     device int32 [batch], each in [0, max_len], or NULL (all
+ *                 max_len)
+ * span_offsets    device int32 [batch + 1] out: spans of prompt b are
+ *                 span_offsets[b] .. span_offsets[b+1]-1
+ * span_start      device int32 [batch * (max_len/2)] out: start, relative to
+ *                 the prompt (capacity: a prompt of length L has at most L/2)
+ * span_len        device int32, same capacity: n
+ * span_rule       device int32, same capacity: rule id
+ * merge_token_ids device int32 [batch * max_len] out, or NULL: the tokens of
+ *                 every span, span after span
+ * merge_offsets   device int32 [batch * (max_len/2) + 1] out (with
+ *                 merge_token_ids): CSR offsets of the spans' tokens
+ * workspace       device, umim_match_prompts_workspace_size() bytes, 256-B
+ *                 aligned
+ * Host-side errors: batch * max_len >= 2^31.  Device-side errors:
+ * UMIM_ERR_INVALID_ARG for a prompt length outside [0, max_len] (clamped) or
+ * a token id outside [0, 0xFFFFFF) (no n-gram containing it matches).
+ * ------------------------------------------------------------------------ */
+size_t umim_match_prompts_workspace_size(int32_t batch, int32_t max_len);
+
+umim_status umim_match_prompts(const void *table, size_t table_bytes, const int32_t *token_ids, int32_t batch,
+                               int32_t max_len, const int32_t *prompt_lens, int32_t *span_offsets,
+                               int32_t *span_start, int32_t *span_len, int32_t *span_rule,
+                               int32_t *merge_token_ids, int32_t *merge_offsets, void *workspace,
+                               size_t workspace_bytes, int32_t *dev_status, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Decoding-time span selection (App. E "Rule Matching", "Decoding-Time
+ * Merging"): after each generated token, the raw-token suffix ending at it is
+ * tested longest first (4, 3, 2 tokens).  A merged span counts as one marker
+ * that no later suffix includes, and generation starts with an empty suffix
+ * (the prompt is not part of it).  Per sequence the state is the last up to
+ * three raw generated tokens:
+ *   typedef: int32 raw[3] (right-aligned: the last n_raw entries are the
+ *   suffix, oldest first), int32 n_raw in [0, 3].  A zeroed state is the
+ *   start of generation.
+ * Per sequence b, for new_tokens[b]:
+ *   merge_k[b]    n of the merge it completes (the k of
+ *                 umim_decode_append_merge), or 0
+ *   merge_rule[b] its rule id, or -1
+ *   merge_row[b]  its rank among this step's merging sequences (in sequence
+ *                 order), or -1: the row of the surrogate arrays that
+ *                 umim_decode_append_merge reads
+ *   rows_rule     device int32 [batch] out, or NULL: rule id of each row
+ *   n_merges      device int32 [1] out, or NULL: number of merging sequences
+ * state is updated in place.  Device-side errors: UMIM_ERR_INVALID_ARG for
+ * n_raw outside [0, 3] (read as 0) or a token outside [0, 0xFFFFFF) (no
+ * merge; the suffix restarts after it).
+ * ------------------------------------------------------------------------ */
+typedef struct {
+  int32_t raw[3];
+  int32_t n_raw;
+} umim_suffix_state;
+
+umim_status umim_match_suffix(const void *table, size_t table_bytes, umim_suffix_state *state,
+                              const int32_t *new_tokens, int32_t batch, int32_t *merge_k, int32_t *merge_rule,
+                              int32_t *merge_row, int32_t *rows_rule, int32_t *n_merges, int32_t *dev_status,
+                              cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Surrogate lookup (App. E, potential engineering optimizations): a
+ * surrogate depends only on its span's tokens, so one per rule can be
+ * computed ahead of time (umim_merge_spans over the rules' n-grams) and
+ * fetched by rule id instead of running the merge module.
+ * lut        device fp32 [n_rules][d], 16-B aligned (d a multiple of 4)
+ * rule_ids   device int32 [n_max]
+ * n_dev      device int32 [1] or NULL: rows to fetch, min(*n_dev, n_max)
+ *            (e.g. span_offsets[batch] of umim_match_prompts); NULL: n_max
+ * out        device fp32 [n_max][d], 16-B aligned
+ * Device-side errors: UMIM_ERR_INVALID_ARG for a rule id outside
+ * [0, n_rules) (that row is written as zeros).
+ * ------------------------------------------------------------------------ */
+umim_status umim_lookup_surrogates(const float *lut, int64_t n_rules, int32_t d, const int32_t *rule_ids,
+                                   int32_t n_max, const int32_t *n_dev, float *out, int32_t *dev_status,
+                                   cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
  * Decode attention for callers that cannot allocate GPU memory.
  * The paper has no counterpart to this call; it is a convenience of this
  * library.  A serving engine that gives all device memory to its own block

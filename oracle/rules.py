@@ -35,7 +35,7 @@ def rule_dict(rules):
     Returns {tuple: rule id}."""
     d = {}
     for r, g in enumerate(rules):
-        g = tuple(int(x) for x in g)
+        g = g if type(g) is tuple else tuple(int(x) for x in g)
         if not 2 <= len(g) <= 4:
             raise ValueError(f"rule {r} has length {len(g)}")
         if g in d:

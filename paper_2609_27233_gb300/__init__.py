@@ -11,6 +11,9 @@ points keep the C names:
   umim_kv_append          decode-step append of one KV entry per layer (App. E, Fig. 2)
   umim_decode_append_merge  append or suffix merge per sequence in one call (App. E decoding loop)
   umim_decode_attention   GQA decode attention over the compacted paged cache (App. I.1)
+  umim_rules_build, umim_match_prompts, umim_match_suffix, umim_lookup_surrogates
+                          merge-rule table, longest-first span selection for prompts
+                          and for decoding, and precomputed surrogates by rule id (App. E)
 """
 import ctypes
 
@@ -245,6 +248,87 @@ def umim_decode_attention_static(q, pool, layer, block_table, seq_lens, scale=0.
 # ---------------------------------------------------------------------------
 # kernel tracing (profiling aid)
 # ---------------------------------------------------------------------------
+def umim_rule_table_bytes(n_rules):
+    return int(lib().umim_rule_table_bytes(n_rules))
+
+
+def umim_rules_build(rule_tokens, table=None, dev_status=None, stream=None):
+    """Rule table for rule_tokens [R][4] int32 (n token ids, then -1s).
+    Returns the table (a uint8 device buffer)."""
+    R = rule_tokens.shape[0]
+    nbytes = umim_rule_table_bytes(R)
+    if table is None:
+        table = torch.empty(nbytes, dtype=torch.uint8, device=rule_tokens.device)
+    code = lib().umim_rules_build(_p(table), table.numel(), _p(rule_tokens), R, _p(dev_status), _stream(stream))
+    _check(code, "umim_rules_build")
+    return table
+
+
+def umim_match_prompts_workspace_size(batch, max_len):
+    return int(lib().umim_match_prompts_workspace_size(batch, max_len))
+
+
+def umim_match_prompts(table, token_ids, prompt_lens=None, merge_inputs=False, workspace_buf=None, dev_status=None,
+                       stream=None):
+    """Longest-first span selection for a batch of prompts token_ids [B][L].
+    Returns a dict of device int32 tensors: span_offsets [B+1], span_start,
+    span_len, span_rule (capacity B*(L//2)), and with merge_inputs the span
+    tokens and their CSR offsets (merge_token_ids, merge_offsets)."""
+    dev = _dev(token_ids)
+    B, L = token_ids.shape
+    cap = max(1, B * (L // 2))
+    i32 = lambda n: torch.empty(n, dtype=torch.int32, device=dev)
+    out = dict(span_offsets=i32(B + 1), span_start=i32(cap), span_len=i32(cap), span_rule=i32(cap),
+               merge_token_ids=i32(max(1, B * L)) if merge_inputs else None,
+               merge_offsets=i32(cap + 1) if merge_inputs else None)
+    if workspace_buf is None:
+        workspace_buf = workspace(umim_match_prompts_workspace_size(B, L), dev)
+    code = lib().umim_match_prompts(_p(table), table.numel(), _p(token_ids), B, L, _p(prompt_lens),
+                                    _p(out["span_offsets"]), _p(out["span_start"]), _p(out["span_len"]),
+                                    _p(out["span_rule"]), _p(out["merge_token_ids"]), _p(out["merge_offsets"]),
+                                    _p(workspace_buf), workspace_buf.numel(), _p(dev_status), _stream(stream))
+    _check(code, "umim_match_prompts")
+    return out
+
+
+def new_suffix_state(batch, device):
+    """Decoding state of umim_match_suffix at the start of generation: [B][4] int32 zeros."""
+    return torch.zeros((batch, 4), dtype=torch.int32, device=device)
+
+
+def umim_match_suffix(table, state, new_tokens, merge_k=None, merge_rule=None, merge_row=None, rows_rule=None,
+                      n_merges=None, dev_status=None, stream=None):
+    """One decoding step of span selection; state [B][4] is updated in place.
+    Returns (merge_k, merge_rule, merge_row, rows_rule, n_merges)."""
+    dev = _dev(new_tokens)
+    B = new_tokens.shape[0]
+    i32 = lambda n: torch.empty(n, dtype=torch.int32, device=dev)
+    merge_k = i32(B) if merge_k is None else merge_k
+    merge_rule = i32(B) if merge_rule is None else merge_rule
+    merge_row = i32(B) if merge_row is None else merge_row
+    if rows_rule is None:   # entries past n_merges are not written
+        rows_rule = torch.full((max(1, B),), -1, dtype=torch.int32, device=dev)
+    n_merges = i32(1) if n_merges is None else n_merges
+    code = lib().umim_match_suffix(_p(table), table.numel(), _p(state), _p(new_tokens), B, _p(merge_k),
+                                   _p(merge_rule), _p(merge_row), _p(rows_rule), _p(n_merges), _p(dev_status),
+                                   _stream(stream))
+    _check(code, "umim_match_suffix")
+    return merge_k, merge_rule, merge_row, rows_rule, n_merges
+
+
+def umim_lookup_surrogates(lut, rule_ids, n_dev=None, out=None, dev_status=None, stream=None):
+    """out [n][d] fp32 = lut[rule_ids[:n]] with n = min(*n_dev, len(rule_ids))
+    (rows past n are left as they were)."""
+    R, d = lut.shape
+    n_max = rule_ids.shape[0]
+    if out is None:
+        out = torch.zeros((max(1, n_max), d), dtype=torch.float32, device=lut.device)
+    code = lib().umim_lookup_surrogates(_p(lut), R, d, _p(rule_ids), n_max, _p(n_dev), _p(out), _p(dev_status),
+                                        _stream(stream))
+    _check(code, "umim_lookup_surrogates")
+    return out
+
+
 def trace_start(capacity=4096):
     _check(lib().umim_trace_start(capacity), "umim_trace_start")
 

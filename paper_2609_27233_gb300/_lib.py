@@ -48,6 +48,14 @@ SIGNATURES = {
                                       c_ptr, c_ptr]),
     "umim_decode_append_merge": (ctypes.c_int, [ctypes.POINTER(PagedKVC), c_ptr, c_i32, c_ptr, c_i32, c_ptr, c_ptr,
                                                 c_ptr, c_ptr, c_ptr, c_i32, c_ptr, c_ptr, c_ptr, c_ptr, c_ptr]),
+    "umim_rule_table_bytes": (c_size, [c_i64]),
+    "umim_rules_build": (ctypes.c_int, [c_ptr, c_size, c_ptr, c_i64, c_ptr, c_ptr]),
+    "umim_match_prompts_workspace_size": (c_size, [c_i32, c_i32]),
+    "umim_match_prompts": (ctypes.c_int, [c_ptr, c_size, c_ptr, c_i32, c_i32, c_ptr, c_ptr, c_ptr, c_ptr, c_ptr,
+                                          c_ptr, c_ptr, c_ptr, c_size, c_ptr, c_ptr]),
+    "umim_match_suffix": (ctypes.c_int, [c_ptr, c_size, c_ptr, c_ptr, c_i32, c_ptr, c_ptr, c_ptr, c_ptr, c_ptr,
+                                         c_ptr, c_ptr]),
+    "umim_lookup_surrogates": (ctypes.c_int, [c_ptr, c_i64, c_i32, c_ptr, c_i32, c_ptr, c_ptr, c_ptr, c_ptr]),
     "umim_decode_attention_workspace_size": (c_size, [c_i32, c_i32, c_i32, c_i32]),
     "umim_decode_attention": (ctypes.c_int, [c_ptr, c_i32, ctypes.POINTER(PagedKVC), c_i32, c_ptr, c_i32,
                                              c_ptr, c_i32, ctypes.c_float, c_ptr, c_ptr, c_size, c_ptr,

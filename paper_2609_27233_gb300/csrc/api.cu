@@ -44,6 +44,15 @@ umim_status kv_append(const umim_paged_kv *, int32_t *, int32_t, int32_t *, int3
 umim_status decode_append_merge(const umim_paged_kv *, int32_t *, int32_t, int32_t *, int32_t, const void *,
                                 const void *, const int32_t *, const int32_t *, const int32_t *, int32_t, const void *,
                                 const void *, int32_t *, int32_t *, cudaStream_t);
+size_t rule_table_bytes(int64_t n_rules);
+umim_status rules_build(void *, size_t, const int32_t *, int64_t, int32_t *, cudaStream_t, int);
+size_t match_prompts_workspace_bytes(int B, int L);
+umim_status match_prompts(const void *, size_t, const int32_t *, int, int, const int32_t *, int32_t *, int32_t *,
+                          int32_t *, int32_t *, int32_t *, int32_t *, void *, int32_t *, cudaStream_t, int);
+umim_status match_suffix(const void *, size_t, void *, const int32_t *, int, int32_t *, int32_t *, int32_t *,
+                         int32_t *, int32_t *, int32_t *, cudaStream_t);
+umim_status lookup_surrogates(const float *, int64_t, int, const int32_t *, int, const int32_t *, float *, int32_t *,
+                              cudaStream_t, int);
 size_t decode_attention_workspace_bytes(int B, int Hq, int Hkv, int D, int num_sms);
 umim_status decode_attention(const void *, int, const umim_paged_kv *, int, const int32_t *, int, const int32_t *,
                              int, float, void *, void *, int32_t *, cudaStream_t, int);
@@ -73,6 +82,15 @@ int current_sms() {
 }
 
 bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+constexpr int64_t kMaxRules = int64_t(1) << 29;
+
+// a rule table buffer: 16-B aligned, a power of two of 16-byte slots, at least 16 of them
+bool table_ok(const void *t, size_t bytes) {
+  const uint64_t slots = bytes / 16;
+  return t && aligned(t, 16) && bytes % 16 == 0 && slots >= 16 && (slots & (slots - 1)) == 0 &&
+         slots <= (uint64_t(1) << 31);
+}
 
 bool kv_ok(const umim_paged_kv *kv) {
   return kv && kv->base && kv->n_layers > 0 && kv->n_pages > 0 && kv->n_kv_heads > 0 && aligned(kv->base, 16);
@@ -225,6 +243,74 @@ umim_status umim_decode_append_merge(const umim_paged_kv *kv, int32_t *block_tab
   prepare_device(stream);
   return decode_append_merge(kv, block_table, max_pages, seq_lens, batch, new_k, new_v, new_pages, merge_k,
                              merge_row, n_merge_rows, surrogate_k, surrogate_v, released_pages, dev_status, stream);
+}
+
+size_t umim_rule_table_bytes(int64_t n_rules) {
+  if (n_rules < 0 || n_rules > kMaxRules) return 0;
+  return rule_table_bytes(n_rules);
+}
+
+umim_status umim_rules_build(void *table, size_t table_bytes, const int32_t *rule_tokens, int64_t n_rules,
+                             int32_t *dev_status, cudaStream_t stream) {
+  if (n_rules < 0 || n_rules > kMaxRules || !table_ok(table, table_bytes)) return UMIM_ERR_INVALID_ARG;
+  if ((uint64_t)table_bytes < 24ull * (uint64_t)n_rules) return UMIM_ERR_WORKSPACE;
+  if (n_rules > 0 && (!rule_tokens || !aligned(rule_tokens, 16))) return UMIM_ERR_INVALID_ARG;
+  const int sms = prepare_device(stream);
+  return rules_build(table, table_bytes, rule_tokens, n_rules, dev_status, stream, sms);
+}
+
+size_t umim_match_prompts_workspace_size(int32_t batch, int32_t max_len) {
+  if (batch < 0 || max_len < 0) return 0;
+  return match_prompts_workspace_bytes(batch, max_len);
+}
+
+umim_status umim_match_prompts(const void *table, size_t table_bytes, const int32_t *token_ids, int32_t batch,
+                               int32_t max_len, const int32_t *prompt_lens, int32_t *span_offsets,
+                               int32_t *span_start, int32_t *span_len, int32_t *span_rule,
+                               int32_t *merge_token_ids, int32_t *merge_offsets, void *workspace,
+                               size_t workspace_bytes, int32_t *dev_status, cudaStream_t stream) {
+  if (!table_ok(table, table_bytes) || batch < 0 || max_len < 0 || !span_offsets) return UMIM_ERR_INVALID_ARG;
+  if ((int64_t)batch * max_len >= INT32_MAX) return UMIM_ERR_UNSUPPORTED;
+  if ((merge_token_ids == nullptr) != (merge_offsets == nullptr)) return UMIM_ERR_INVALID_ARG;
+  const int sms = prepare_device(stream);
+  if (batch == 0) {
+    if (cudaMemsetAsync(span_offsets, 0, sizeof(int32_t), stream) != cudaSuccess) return UMIM_ERR_CUDA;
+    if (merge_offsets && cudaMemsetAsync(merge_offsets, 0, sizeof(int32_t), stream) != cudaSuccess)
+      return UMIM_ERR_CUDA;
+    return UMIM_OK;
+  }
+  if (!token_ids || !span_start || !span_len || !span_rule) return UMIM_ERR_INVALID_ARG;
+  if (!workspace || !aligned(workspace, 256) || workspace_bytes < match_prompts_workspace_bytes(batch, max_len))
+    return UMIM_ERR_WORKSPACE;
+  return match_prompts(table, table_bytes, token_ids, batch, max_len, prompt_lens, span_offsets, span_start,
+                       span_len, span_rule, merge_token_ids, merge_offsets, workspace, dev_status, stream, sms);
+}
+
+umim_status umim_match_suffix(const void *table, size_t table_bytes, umim_suffix_state *state,
+                              const int32_t *new_tokens, int32_t batch, int32_t *merge_k, int32_t *merge_rule,
+                              int32_t *merge_row, int32_t *rows_rule, int32_t *n_merges, int32_t *dev_status,
+                              cudaStream_t stream) {
+  static_assert(sizeof(umim_suffix_state) == 16, "suffix state is one 16-byte vector");
+  if (!table_ok(table, table_bytes) || batch < 0) return UMIM_ERR_INVALID_ARG;
+  prepare_device(stream);
+  if (batch == 0) {
+    if (n_merges && cudaMemsetAsync(n_merges, 0, sizeof(int32_t), stream) != cudaSuccess) return UMIM_ERR_CUDA;
+    return UMIM_OK;
+  }
+  if (!state || !aligned(state, 16) || !new_tokens || !merge_k || !merge_rule || !merge_row)
+    return UMIM_ERR_INVALID_ARG;
+  return match_suffix(table, table_bytes, state, new_tokens, batch, merge_k, merge_rule, merge_row, rows_rule,
+                      n_merges, dev_status, stream);
+}
+
+umim_status umim_lookup_surrogates(const float *lut, int64_t n_rules, int32_t d, const int32_t *rule_ids,
+                                   int32_t n_max, const int32_t *n_dev, float *out, int32_t *dev_status,
+                                   cudaStream_t stream) {
+  if (n_rules < 0 || d <= 0 || d % 4 != 0 || n_max < 0) return UMIM_ERR_INVALID_ARG;
+  if (n_max == 0) return UMIM_OK;
+  if (!lut || !aligned(lut, 16) || !rule_ids || !out || !aligned(out, 16)) return UMIM_ERR_INVALID_ARG;
+  const int sms = prepare_device(stream);
+  return lookup_surrogates(lut, n_rules, d, rule_ids, n_max, n_dev, out, dev_status, stream, sms);
 }
 
 size_t umim_decode_attention_workspace_size(int32_t batch, int32_t n_q_heads, int32_t n_kv_heads,

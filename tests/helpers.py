@@ -69,3 +69,29 @@ def compare_rollback(g_pool, g_bt, g_lens, g_freed, ref):
         t = np.arange(int(rl[b]))
         pg, sl = rbt[b, t // 16], t % 16
         np.testing.assert_array_equal(gp[:, pg, :, :, sl, :], rp[:, pg, :, :, sl, :], err_msg=f"seq {b}")
+
+
+def oracle_append_merge(pool, bt, lens, nk, nv, new_pages, merge_k, sk, sv):
+    """kv_append, then kv_rollback of the suffix span (L + 1 - k, k) of every
+    merging sequence (surrogate rows in sequence order); released pages per
+    sequence from the rollback's freed list."""
+    L0 = lens.copy()
+    pool, bt, lens, rej = oracle.kv_append(pool, bt, lens, nk, nv, new_pages)
+    assert rej == []
+    B = len(L0)
+    offs = np.zeros(B + 1, np.int32)
+    st, ln = [], []
+    for b in range(B):
+        offs[b + 1] = offs[b]
+        if merge_k[b] > 0:
+            st.append(int(L0[b]) + 1 - int(merge_k[b]))
+            ln.append(int(merge_k[b]))
+            offs[b + 1] += 1
+    pool, bt2, lens2, freed = oracle.kv_rollback(pool, bt, lens, offs, np.array(st, np.int32),
+                                                 np.array(ln, np.int32), sk, sv)
+    released = np.full(B, -1, np.int32)
+    fi = iter(freed)
+    for b in range(B):
+        if (int(lens[b]) + 15) // 16 > (int(lens2[b]) + 15) // 16:
+            released[b] = next(fi)
+    return pool, bt2, lens2, released

@@ -7,7 +7,7 @@ import torch
 
 import oracle
 import workloads as W
-from helpers import dev, umim
+from helpers import dev, oracle_append_merge, umim
 
 pytestmark = pytest.mark.gpu
 
@@ -104,32 +104,6 @@ def test_no_page_list_needed_inside_pages():
 # ---------------------------------------------------------------------------
 # append or suffix merge in one call (the decode loop's cache update)
 # ---------------------------------------------------------------------------
-def _oracle_append_merge(pool, bt, lens, nk, nv, new_pages, merge_k, sk, sv):
-    """kv_append, then kv_rollback of the suffix span (L + 1 - k, k) of every
-    merging sequence (surrogate rows in sequence order); released pages per
-    sequence from the rollback's freed list."""
-    L0 = lens.copy()
-    pool, bt, lens, rej = oracle.kv_append(pool, bt, lens, nk, nv, new_pages)
-    assert rej == []
-    B = len(L0)
-    offs = np.zeros(B + 1, np.int32)
-    st, ln = [], []
-    for b in range(B):
-        offs[b + 1] = offs[b]
-        if merge_k[b] > 0:
-            st.append(int(L0[b]) + 1 - int(merge_k[b]))
-            ln.append(int(merge_k[b]))
-            offs[b + 1] += 1
-    pool, bt2, lens2, freed = oracle.kv_rollback(pool, bt, lens, offs, np.array(st, np.int32),
-                                                 np.array(ln, np.int32), sk, sv)
-    released = np.full(B, -1, np.int32)
-    fi = iter(freed)
-    for b in range(B):
-        if (int(lens[b]) + 15) // 16 > (int(lens2[b]) + 15) // 16:
-            released[b] = next(fi)
-    return pool, bt2, lens2, released
-
-
 @pytest.mark.parametrize("seed,lens,hkv,d,layers,steps", [
     (41, [0, 1, 15, 16, 17, 31, 32, 100, 255, 256], 8, 128, 3, 30),
     (42, [3, 16, 47, 64, 2047], 2, 64, 2, 24),
@@ -164,7 +138,7 @@ def test_append_merge_matches_append_then_suffix_rollback(seed, lens, hkv, d, la
         t = lambda x: torch.from_numpy(x).to(dv)
         rel = m.umim_decode_append_merge(pool, bt, sl, nk, nv, t(new_pages), t(merge_k), t(merge_row), sk, sv,
                                          dev_status=status)
-        o_pool, o_bt, o_lens, o_rel = _oracle_append_merge(o_pool, o_bt, o_lens, W.bits(nk), W.bits(nv), new_pages,
+        o_pool, o_bt, o_lens, o_rel = oracle_append_merge(o_pool, o_bt, o_lens, W.bits(nk), W.bits(nv), new_pages,
                                                            merge_k, W.bits(sk)[:S], W.bits(sv)[:S])
         alloc.give_back([p for p in o_rel if p >= 0])
         n_merged += S

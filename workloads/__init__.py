@@ -39,7 +39,13 @@ SEEDS = {
     "long_context": 0x5EED0004,
     "long_context_tr40": 0x5EED0014,
     "serving": 0x5EED0005,
+    "rule_matching": 0x5EED0006,
 }
+
+# Retained merge rules per n-gram length for the Llama-3 tokenizer (the paper's
+# table of rule counts, frequency threshold 5): 2-, 3- and 4-grams.
+LLAMA3_RULE_COUNTS = (216_700, 684_793, 1_266_080)
+LLAMA3_VOCAB = 128_256
 
 
 def rng(seed: int) -> np.random.Generator:
@@ -331,6 +337,86 @@ def prompt_case(seed: int, *, B: int, L: int, vocab: int, d: int, coverage: floa
                       span_start=t(span_start), span_len=t(span_len),
                       span_token_ids=t(span_tokens),
                       span_token_offsets=t(np.asarray(toffs, np.int32)))
+
+
+# ----------------------------------------------------------------------------
+# merge rules and prompts that use them
+# ----------------------------------------------------------------------------
+def _distinct_rows(a: np.ndarray) -> np.ndarray:
+    """Rows of a with repeats removed (first occurrence kept), order kept."""
+    if len(a) == 0:
+        return a
+    order = np.lexsort(a.T[::-1])
+    srt = a[order]
+    first = np.ones(len(a), bool)
+    first[1:] = np.any(srt[1:] != srt[:-1], axis=1)
+    keep = np.zeros(len(a), bool)
+    keep[order[first]] = True
+    return a[keep]
+
+
+def random_rules(seed: int, counts, vocab: int) -> np.ndarray:
+    """Distinct n-grams: counts[0] 2-grams, counts[1] 3-grams, counts[2]
+    4-grams with uniform token ids in [0, vocab), in that order, each as a
+    row [4] int32 padded with -1 (the rule id is the row), rows shuffled."""
+    r = rng(seed)
+    out = []
+    for n, c in zip((2, 3, 4), counts):
+        got = np.zeros((0, n), np.int32)
+        while len(got) < c:
+            more = r.integers(0, vocab, size=(c - len(got) + 16, n)).astype(np.int32)
+            got = _distinct_rows(np.concatenate([got, more]))
+        rows = np.full((c, 4), -1, np.int32)
+        rows[:, :n] = got[:c]
+        out.append(rows)
+    rules = np.concatenate(out) if out else np.zeros((0, 4), np.int32)
+    return rules[r.permutation(len(rules))]
+
+
+def rule_prompts(seed: int, rules: np.ndarray, *, B: int, L: int, vocab: int, coverage: float,
+                 lens=None) -> np.ndarray:
+    """Prompts [B][L] int32 of uniform random tokens in which occurrences of
+    rules are planted at non-overlapping places until they cover about
+    ``coverage`` of each prompt: a length n uniform in {2, 3, 4} (among the
+    lengths the rule set has), then a rule of that length uniformly, placed by
+    stars and bars as in span_layout.  lens[b] < L leaves the tail of row b as
+    padding (-1)."""
+    r = rng(seed)
+    ids = r.integers(0, vocab, size=(B, L)).astype(np.int32)
+    n_of = (rules >= 0).sum(axis=1) if len(rules) else np.zeros(0, np.int64)
+    by_n = [np.nonzero(n_of == n)[0] for n in (2, 3, 4)]
+    by_n = [g for g in by_n if len(g)]
+    for b in range(B):
+        Lb = L if lens is None else int(lens[b])
+        chosen, tot = [], 0
+        target = int(round(coverage * Lb))
+        while by_n and tot < target:
+            g = by_n[int(r.integers(0, len(by_n)))]
+            j = int(g[int(r.integers(0, len(g)))])
+            if tot + n_of[j] > Lb:
+                break
+            chosen.append(j)
+            tot += int(n_of[j])
+        S = len(chosen)
+        if S:
+            ks = n_of[chosen]
+            bars = np.sort(r.choice(Lb - tot + S, size=S, replace=False))
+            starts = bars - np.arange(S) + np.concatenate([[0], np.cumsum(ks)[:-1]])
+            for j, s0 in zip(chosen, starts):
+                ids[b, s0:s0 + n_of[j]] = rules[j, :n_of[j]]
+        ids[b, Lb:] = -1
+    return ids
+
+
+def rule_tuples(rules: np.ndarray):
+    """Rule rows [R][4] (-1 padded) as a list of token tuples, rule id order."""
+    n_of = (rules >= 0).sum(axis=1)
+    out = [None] * len(rules)
+    for n in (2, 3, 4):
+        idx = np.nonzero(n_of == n)[0]
+        for i, g in zip(idx.tolist(), rules[idx, :n].tolist()):
+            out[i] = tuple(g)
+    return out
 
 
 # ----------------------------------------------------------------------------
