@@ -268,19 +268,21 @@ def umim_match_prompts_workspace_size(batch, max_len):
     return int(lib().umim_match_prompts_workspace_size(batch, max_len))
 
 
-def umim_match_prompts(table, token_ids, prompt_lens=None, merge_inputs=False, workspace_buf=None, dev_status=None,
-                       stream=None):
+def umim_match_prompts(table, token_ids, prompt_lens=None, merge_inputs=False, out=None, workspace_buf=None,
+                       dev_status=None, stream=None):
     """Longest-first span selection for a batch of prompts token_ids [B][L].
-    Returns a dict of device int32 tensors: span_offsets [B+1], span_start,
-    span_len, span_rule (capacity B*(L//2)), and with merge_inputs the span
-    tokens and their CSR offsets (merge_token_ids, merge_offsets)."""
+    Returns (or fills, when out is given) a dict of device int32 tensors:
+    span_offsets [B+1], span_start, span_len, span_rule (capacity B*(L//2)),
+    and with merge_inputs the span tokens and their CSR offsets
+    (merge_token_ids, merge_offsets)."""
     dev = _dev(token_ids)
     B, L = token_ids.shape
     cap = max(1, B * (L // 2))
     i32 = lambda n: torch.empty(n, dtype=torch.int32, device=dev)
-    out = dict(span_offsets=i32(B + 1), span_start=i32(cap), span_len=i32(cap), span_rule=i32(cap),
-               merge_token_ids=i32(max(1, B * L)) if merge_inputs else None,
-               merge_offsets=i32(cap + 1) if merge_inputs else None)
+    if out is None:
+        out = dict(span_offsets=i32(B + 1), span_start=i32(cap), span_len=i32(cap), span_rule=i32(cap),
+                   merge_token_ids=i32(max(1, B * L)) if merge_inputs else None,
+                   merge_offsets=i32(cap + 1) if merge_inputs else None)
     if workspace_buf is None:
         workspace_buf = workspace(umim_match_prompts_workspace_size(B, L), dev)
     code = lib().umim_match_prompts(_p(table), table.numel(), _p(token_ids), B, L, _p(prompt_lens),

@@ -542,26 +542,38 @@ __global__ void __launch_bounds__(kSuffixThreads)
 // ---------------------------------------------------------------------------
 // surrogate lookup
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(256) lut_gather_kernel(const float4 *lut, int64_t n_rules, int d4,
-                                                         const int32_t *ids, int n_max, const int32_t *n_dev,
-                                                         float4 *out, int32_t *status) {
+// one CTA per row (grid-stride): 16-byte chunks, four loads in flight per thread
+constexpr int kGatherThreads = 256, kGatherUnroll = 4;
+
+__global__ void __launch_bounds__(kGatherThreads) lut_gather_kernel(const float4 *lut, int64_t n_rules, int d4,
+                                                                    const int32_t *ids, int n_max,
+                                                                    const int32_t *n_dev, float4 *out,
+                                                                    int32_t *status) {
   griddep_wait();
   const int n = n_dev ? min(max(*n_dev, 0), n_max) : n_max;
-  const int64_t total = (int64_t)n * d4;
-  for (int64_t g = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; g < total; g += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t i = g / d4;
-    const int c = (int)(g - i * d4);
-    const int32_t id = ids[i];
-    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (id < 0 || id >= n_rules) {
-      if (c == 0) set_error(status, UMIM_ERR_INVALID_ARG);
-    } else {
-      const float4 *src = lut + (int64_t)id * d4 + c;
-      asm volatile("ld.global.nc.L1::no_allocate.v4.f32 {%0, %1, %2, %3}, [%4];"
-                   : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
-                   : "l"(src));
+  for (int row = blockIdx.x; row < n; row += gridDim.x) {
+    const int32_t id = ids[row];
+    const bool ok = id >= 0 && id < n_rules;
+    if (!ok && threadIdx.x == 0) set_error(status, UMIM_ERR_INVALID_ARG);
+    const float4 *src = lut + (int64_t)(ok ? id : 0) * d4;
+    float4 *dst = out + (int64_t)row * d4;
+    for (int c0 = threadIdx.x; c0 < d4; c0 += kGatherThreads * kGatherUnroll) {
+      float4 v[kGatherUnroll];
+#pragma unroll
+      for (int u = 0; u < kGatherUnroll; ++u) {
+        const int c = c0 + u * kGatherThreads;
+        v[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (ok && c < d4)
+          asm volatile("ld.global.nc.L1::no_allocate.v4.f32 {%0, %1, %2, %3}, [%4];"
+                       : "=f"(v[u].x), "=f"(v[u].y), "=f"(v[u].z), "=f"(v[u].w)
+                       : "l"(src + c));
+      }
+#pragma unroll
+      for (int u = 0; u < kGatherUnroll; ++u) {
+        const int c = c0 + u * kGatherThreads;
+        if (c < d4) dst[c] = v[u];
+      }
     }
-    out[g] = v;
   }
 }
 
@@ -644,10 +656,9 @@ umim_status match_suffix(const void *table, size_t table_bytes, void *state, con
 umim_status lookup_surrogates(const float *lut, int64_t n_rules, int d, const int32_t *ids, int n_max,
                               const int32_t *n_dev, float *out, int32_t *status, cudaStream_t stream, int num_sms) {
   const int d4 = d / 4;
-  const int64_t total = (int64_t)n_max * d4;
-  const int grid = (int)std::max<int64_t>(1, std::min<int64_t>((total + 255) / 256, (int64_t)num_sms * 8));
+  const int grid = std::max(1, std::min(n_max, std::max(1, num_sms) * 8));
   trace_mark(stream, "lut.gather");
-  if (launch_pdl(lut_gather_kernel, dim3(grid), dim3(256), 0, stream, reinterpret_cast<const float4 *>(lut), n_rules,
+  if (launch_pdl(lut_gather_kernel, dim3(grid), dim3(kGatherThreads), 0, stream, reinterpret_cast<const float4 *>(lut), n_rules,
                  d4, ids, n_max, n_dev, reinterpret_cast<float4 *>(out), status) != cudaSuccess)
     return UMIM_ERR_CUDA;
   trace_mark(stream, nullptr);
