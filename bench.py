@@ -295,6 +295,9 @@ def main():
     ap.add_argument("--workload", default="llama8b_layer",
                     choices=["llama8b_layer", "serving", "prompt_compression", "long_context", "rule_matching"])
     ap.add_argument("--coverage", type=float, default=0.4, help="long_context span coverage")
+    ap.add_argument("--lut-rows", type=int, default=0,
+                    help="rule_matching: keep only this many lookup-table rows (rule id mod rows), to bound "
+                         "device memory under a profiler; 0 = one row per rule")
     args = ap.parse_args()
     if args.workload == "serving" and args.impl == "umim":
         return serving_bench(args)
@@ -836,10 +839,11 @@ def side_bench(args):
         table = umim.umim_rules_build(torch.from_numpy(rules_np).to(dev), dev_status=status)
         emb = W.bf16_normal((V, d), 0.02, seed + 101, dev)
         # one precomputed surrogate per rule (fp32); any values do for timing the copies
-        lut = torch.empty((R, d), dtype=torch.float32, device=dev)
+        lut_rows = args.lut_rows if 0 < args.lut_rows < R else R
+        lut = torch.empty((lut_rows, d), dtype=torch.float32, device=dev)
         g = torch.Generator(device=dev)
         g.manual_seed(seed + 303)
-        for r0 in range(0, R, 1 << 16):
+        for r0 in range(0, lut_rows, 1 << 16):
             lut[r0:r0 + (1 << 16)].normal_(0.0, 1.0, generator=g)
         cap = B * (L // 2)
         i32 = lambda n: torch.empty(n, dtype=torch.int32, device=dev)
@@ -853,10 +857,14 @@ def side_bench(args):
         ws_c = umim.workspace(umim.umim_build_compressed_workspace_size(B, cap), dev)
         n_dev = mo["span_offsets"][B:]
 
+        rule_ids = mo["span_rule"] if lut_rows == R else torch.empty_like(mo["span_rule"])
+
         def step(i):
             t = toks[i % n_sets]
             umim.umim_match_prompts(table, t, out=mo, workspace_buf=ws_m, dev_status=status)
-            umim.umim_lookup_surrogates(lut, mo["span_rule"], n_dev=n_dev, out=sur, dev_status=status)
+            if lut_rows < R:
+                torch.remainder(mo["span_rule"], lut_rows, out=rule_ids)
+            umim.umim_lookup_surrogates(lut, rule_ids, n_dev=n_dev, out=sur, dev_status=status)
             umim.umim_build_compressed(emb, t, mo["span_offsets"], mo["span_start"], mo["span_len"], sur,
                                        out_embeds=out, position_ids=pos, cu_seqlens=cu, workspace_buf=ws_c,
                                        dev_status=status)
@@ -902,6 +910,7 @@ def side_bench(args):
                            "3-grams, 1,266,080 4-grams); longest-first matching, surrogates fetched from a "
                            "2.17M x 4096 fp32 lookup table, packed bf16 compressed prompts with position ids",
                "rules": R, "rule_table_mb": round(table.numel() / 2 ** 20, 1), "lut_gb": round(lut.numel() * 4 / 1e9, 1),
+               "lut_rows": lut_rows,
                "spans_per_step": S, "compressed_rows": rows, "prompt_tokens_per_step": B * L,
                "decode_suffix_match_us_per_call": round(suffix_us, 2),
                "decode_suffix_match_kernel_us": round(suffix_kernel_us, 2), "decode_suffix_batch": Bs,
