@@ -36,7 +36,10 @@ upcast exactly to float64.
 
 Parity status per function (what pins it is in tests/test_oracle_*.py):
   merge_spans       pinned (library routines, invariants, brute force)
-  kv_rollback       pinned (worked example, length formula, invariants)
+  kv_rollback       pinned (worked example, length formula, invariants); its
+                    key re-rotation to compressed positions pinned by the
+                    complex-exponential RoPE identity, the rotation bound and
+                    inner-product invariance (tests/test_oracle_rope.py)
   kv_append         pinned (logical-list model, rollback identities)
   decode_attention  pinned (library SDPA, closed forms, invariants)
   build_compressed  pinned (worked example, length formula, library bf16)

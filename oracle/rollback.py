@@ -25,19 +25,47 @@ Here k counts STORED entries replaced (the paper's n - 1 when the newest token
 is not yet cached; n when it is).  Slots of the last page at or beyond L' are
 left as they are and are not part of the result.  KV bytes are handled as raw
 bf16 bit patterns, so the result is exact.
+
+Position-aware variant (App. J.4, compressed positions pi(t) = t - r(t), and
+its RoPE discussion): the cache stores keys already rotated for their
+position, so a kept entry that moves from t to pi(t) carries a key rotated
+for t.  With rope_inv_freq (the angular frequencies w_m, m < rotary_dim / 2)
+every moved kept entry's K rows (all layers and KV heads) are rotated by
+-r(t) w_m on the pairs (m, m + rotary_dim / 2) (the half-split pairing of
+Llama-style RoPE), which gives the key the rotation of its compressed
+position: R(pi(t)) k = R(-r(t)) R(t) k.  Computed in float64 and rounded to
+bf16 (ties to even); V rows, columns at or beyond rotary_dim, surrogate
+entries and entries that do not move are unchanged.
 """
 import numpy as np
 
+from . import bf16
 from .spans import check_spans, compressed_length
 
 
+def rerotate_keys(k_bits, shift, inv_freq, rotary_dim):
+    """K rows [..][D] (bf16 bits) rotated by -shift * w_m on the pairs
+    (m, m + rotary_dim/2): x' = x cos + y sin, y' = y cos - x sin."""
+    k = bf16.to_f64(k_bits)
+    half = rotary_dim // 2
+    ang = float(shift) * np.asarray(inv_freq, dtype=np.float64)[:half]
+    c, s = np.cos(ang), np.sin(ang)
+    x, y = k[..., :half], k[..., half:rotary_dim]
+    out = np.array(k_bits, copy=True)
+    out[..., :half] = bf16.from_f64(x * c + y * s)
+    out[..., half:rotary_dim] = bf16.from_f64(y * c - x * s)
+    return out
+
+
 def kv_rollback(pool, block_table, seq_lens, span_offsets, span_start, span_len,
-                surrogate_k, surrogate_v, page_size=16):
+                surrogate_k, surrogate_v, page_size=16, rope_inv_freq=None, rotary_dim=None):
     """pool         [n_layers][n_pages][2][Hkv][P][D] uint16 (bf16 bits)
     block_table  [B][max_pages] int32
     seq_lens     [B] int32
     span_offsets [B+1], span_start [S], span_len [S] int32
     surrogate_k/v [S][n_layers][Hkv][D] uint16
+    rope_inv_freq [rotary_dim/2] (float32 values) or None: re-rotate moved keys
+    rotary_dim   even, <= D (default D)
     Returns (pool', block_table', seq_lens', freed_pages list)."""
     P = page_size
     pool = np.array(pool, copy=True)
@@ -58,6 +86,20 @@ def kv_rollback(pool, block_table, seq_lens, span_offsets, span_start, span_len,
         used = bt[b, :(L + P - 1) // P]
         if np.any(used < 0) or np.any(used >= n_pages):
             raise ValueError("block table entry out of range")
+    D = pool.shape[5]
+    if rope_inv_freq is not None:
+        rotary_dim = D if rotary_dim is None else int(rotary_dim)
+        if rotary_dim % 2 or not 0 < rotary_dim <= D or len(rope_inv_freq) < rotary_dim // 2:
+            raise ValueError("rotary_dim")
+
+    def kept(run, shift):
+        """entries of a kept run [n][layers][2][Hkv][D]; moved runs re-rotated."""
+        if rope_inv_freq is None or shift == 0 or len(run) == 0:
+            return list(run)
+        run = np.array(run, copy=True)
+        run[:, :, 0] = rerotate_keys(run[:, :, 0], shift, rope_inv_freq, rotary_dim)
+        return list(run)
+
     # [page][slot][layer][K|V][Hkv][D] view of the pool (writes go through it)
     view = pool.transpose(1, 4, 0, 2, 3, 5)
     freed = []
@@ -74,12 +116,14 @@ def kv_rollback(pool, block_table, seq_lens, span_offsets, span_start, span_len,
         # last span
         new = []
         t = 0
+        r = 0   # positions removed before the current run
         for i in range(lo, hi):
             s, k = int(span_start[i]), int(span_len[i])
-            new.extend(entries[t:s])
+            new.extend(kept(entries[t:s], r))
             new.append(np.stack([surrogate_k[i], surrogate_v[i]], axis=1))  # [layers][2][Hkv][D]
             t = s + k
-        new.extend(entries[t:L])
+            r += k - 1
+        new.extend(kept(entries[t:L], r))
         new = np.stack(new)
         Lp = len(new)
         assert Lp == compressed_length(L, span_len[lo:hi])
