@@ -295,6 +295,9 @@ def main():
     ap.add_argument("--workload", default="llama8b_layer",
                     choices=["llama8b_layer", "serving", "prompt_compression", "long_context", "rule_matching"])
     ap.add_argument("--coverage", type=float, default=0.4, help="long_context span coverage")
+    ap.add_argument("--rope", action="store_true",
+                    help="llama8b_layer / long_context: re-rotate moved keys to their compressed positions "
+                         "(umim_kv_rollback_rope, Llama-3 RoPE frequencies) instead of moving them verbatim")
     ap.add_argument("--lut-rows", type=int, default=0,
                     help="rule_matching: keep only this many lookup-table rows (rule id mod rows), to bound "
                          "device memory under a profiler; 0 = one row per rule")
@@ -391,6 +394,7 @@ def main():
     ws_m = umim.workspace(umim.umim_merge_spans_workspace_size(T, S, d), dev)
     ws_r = umim.workspace(umim.umim_kv_rollback_workspace_size(B, S, max_pages, 1, Hkv, D), dev)
     ws_a = umim.workspace(umim.umim_decode_attention_workspace_size(B, Hq, Hkv, D), dev)
+    rope = llama3_inv_freq(D, dev) if args.rope else None
 
     def step(i, inputs=None, outs=None):
         j = i % n_copies
@@ -402,7 +406,7 @@ def main():
         o_, f_ = (out, freed) if outs is None else outs
         umim.umim_merge_spans(table, tk, to, weights, surrogates=z, workspace_buf=ws_m, dev_status=status)
         umim.umim_kv_rollback(pools[j], bts[j], lens[j], so, ss, sl, k_, v_, freed_pages=f_,
-                              workspace_buf=ws_r, dev_status=status)
+                              workspace_buf=ws_r, dev_status=status, rope_inv_freq=rope)
         umim.umim_decode_attention(q_, pools[j], 0, bts[j], lens[j], out=o_, workspace_buf=ws_a,
                                    dev_status=status)
 
@@ -576,6 +580,8 @@ def main():
                 "roofline": roof, "kernels": kernels, "cpu_baseline": cpu, "e2e": e2e,
                 "gpu_launches": int(round(launches_per_step * K)), "clocks": clocks,
                 "traced_ms_per_step": tms / K}
+        if args.rope:
+            line["config"]["rope"] = "moved keys re-rotated to their compressed positions (umim_kv_rollback_rope)"
         print(json.dumps(line))
     if world > 1:
         torch.distributed.destroy_process_group()
@@ -939,12 +945,13 @@ def side_bench(args):
         out = torch.empty_like(c.q)
         ws_r = umim.workspace(umim.umim_kv_rollback_workspace_size(B, S, max_pages, 1, Hkv, D), dev)
         ws_a = umim.workspace(umim.umim_decode_attention_workspace_size(B, Hq, Hkv, D), dev)
+        rope = llama3_inv_freq(D, dev) if args.rope else None
 
         def step(i):
             j = i % n_copies
             umim.umim_kv_rollback(pools[j], bts[j], lens[j], c.span_offsets, c.span_start, c.span_len,
                                   c.surrogate_k, c.surrogate_v, freed_pages=freed, workspace_buf=ws_r,
-                                  dev_status=status)
+                                  dev_status=status, rope_inv_freq=rope)
             umim.umim_decode_attention(c.q, pools[j], 0, bts[j], lens[j], out=out, workspace_buf=ws_a,
                                        dev_status=status)
 
@@ -970,7 +977,7 @@ def side_bench(args):
         cfg = {"workload": f"long-context decode: 4 seqs x 32768 tokens, 28/4 heads, head_dim 128, bf16 paged KV "
                            f"(page 16), {int(round(100 * args.coverage))}% of positions in spans of 2..4 rolled "
                            f"back, then decode attention",
-               "spans": S, "compacted_lengths": Lp,
+               "spans": S, "compacted_lengths": Lp, "rope": bool(args.rope),
                "l2": "inputs larger than L2: a distinct 268 MB cache copy per step"}
 
     def timed(n, offset):
@@ -1016,6 +1023,12 @@ def side_bench(args):
                                                      "source": peaks["src"]}}
     print(json.dumps(line))
     return 0
+
+
+def llama3_inv_freq(D, dev):
+    """RoPE angular frequencies w_m = 500000^(-2m/D) (Llama-3's base), fp32 on the device."""
+    import torch
+    return torch.from_numpy((500000.0 ** (-np.arange(0, D, 2, dtype=np.float64) / D)).astype(np.float32)).to(dev)
 
 
 def config_dict(st):

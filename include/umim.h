@@ -206,6 +206,33 @@ umim_status umim_kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int3
                              cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
+ * Position-aware rollback (App. J.4: a kept token at original position t
+ * takes the compressed position pi(t) = t - r(t), r(t) the positions removed
+ * before it; and its discussion of RoPE).  The cache holds keys already
+ * rotated for their positions, so this variant of umim_kv_rollback also
+ * rotates every moved kept entry's K rows (all layers and KV heads) by
+ * -r(t) * rope_inv_freq[m] on the pairs (m, m + rotary_dim/2),
+ * m < rotary_dim/2 (the half-split pairing of Llama-style RoPE):
+ *   x' = x cos(r w_m) + y sin(r w_m),  y' = y cos(r w_m) - x sin(r w_m),
+ * computed in fp32 and rounded to bf16 (nearest even), which gives each
+ * moved key the rotation of its compressed position.  V rows, columns at or
+ * beyond rotary_dim, surrogate entries (computed by the caller at their
+ * compressed positions) and entries that do not move are unchanged; block
+ * tables, lengths and freed pages are those of umim_kv_rollback.
+ * rope_inv_freq  device fp32 [rotary_dim / 2]: the angular frequencies (any
+ *                RoPE variant: base, scaling and all are folded into them)
+ * rotary_dim     a multiple of 16, <= head_dim
+ * Other arguments, workspace and errors: as umim_kv_rollback; a bad
+ * rotary_dim or a NULL rope_inv_freq is UMIM_ERR_INVALID_ARG.
+ * ------------------------------------------------------------------------ */
+umim_status umim_kv_rollback_rope(const umim_paged_kv *kv, int32_t *block_table, int32_t max_pages,
+                                  int32_t *seq_lens, int32_t batch, const int32_t *span_offsets,
+                                  const int32_t *span_start, const int32_t *span_len, int32_t n_spans,
+                                  const void *surrogate_k, const void *surrogate_v, const float *rope_inv_freq,
+                                  int32_t rotary_dim, int32_t *freed_pages, void *workspace, size_t workspace_bytes,
+                                  int32_t *dev_status, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
  * Decode-step KV append (App. E "Decoding-Time Merging and KV-Cache Update"
  * and Fig. 2 step (2): a generated token that completes no merge is
  * forwarded normally and one KV entry is appended).  For each sequence b

@@ -160,9 +160,12 @@ def umim_build_compressed(embeddings, token_ids, span_offsets, span_start, span_
 
 
 def umim_kv_rollback(pool, block_table, seq_lens, span_offsets, span_start, span_len, surrogate_k, surrogate_v,
-                     freed_pages=None, workspace_buf=None, dev_status=None, stream=None):
+                     freed_pages=None, workspace_buf=None, dev_status=None, stream=None, rope_inv_freq=None,
+                     rotary_dim=None):
     """In-place rollback of pool / block_table / seq_lens; returns freed_pages
-    (device int32 [B*max_pages], -1 terminated)."""
+    (device int32 [B*max_pages], -1 terminated).  With rope_inv_freq (device
+    fp32 [rotary_dim/2]) moved keys are re-rotated to their compressed
+    positions (umim_kv_rollback_rope)."""
     dev = _dev(pool)
     kv = paged_kv(pool)
     B, max_pages = block_table.shape
@@ -172,11 +175,19 @@ def umim_kv_rollback(pool, block_table, seq_lens, span_offsets, span_start, span
     if workspace_buf is None:
         workspace_buf = workspace(umim_kv_rollback_workspace_size(B, S, max_pages, kv.n_layers, kv.n_kv_heads,
                                                                   kv.head_dim), dev)
-    code = lib().umim_kv_rollback(ctypes.byref(kv), _p(block_table), max_pages, _p(seq_lens), B, _p(span_offsets),
-                                  _p(span_start), _p(span_len), S, _p(surrogate_k), _p(surrogate_v),
-                                  _p(freed_pages), _p(workspace_buf), workspace_buf.numel(), _p(dev_status),
-                                  _stream(stream))
-    _check(code, "umim_kv_rollback")
+    if rope_inv_freq is None:
+        code = lib().umim_kv_rollback(ctypes.byref(kv), _p(block_table), max_pages, _p(seq_lens), B,
+                                      _p(span_offsets), _p(span_start), _p(span_len), S, _p(surrogate_k),
+                                      _p(surrogate_v), _p(freed_pages), _p(workspace_buf), workspace_buf.numel(),
+                                      _p(dev_status), _stream(stream))
+        _check(code, "umim_kv_rollback")
+    else:
+        rd = kv.head_dim if rotary_dim is None else int(rotary_dim)
+        code = lib().umim_kv_rollback_rope(ctypes.byref(kv), _p(block_table), max_pages, _p(seq_lens), B,
+                                           _p(span_offsets), _p(span_start), _p(span_len), S, _p(surrogate_k),
+                                           _p(surrogate_v), _p(rope_inv_freq), rd, _p(freed_pages),
+                                           _p(workspace_buf), workspace_buf.numel(), _p(dev_status), _stream(stream))
+        _check(code, "umim_kv_rollback_rope")
     return freed_pages
 
 

@@ -44,6 +44,9 @@ SIGNATURES = {
     "umim_kv_rollback_workspace_size": (c_size, [c_i32, c_i32, c_i32, c_i32, c_i32, c_i32]),
     "umim_kv_rollback": (ctypes.c_int, [ctypes.POINTER(PagedKVC), c_ptr, c_i32, c_ptr, c_i32, c_ptr, c_ptr,
                                         c_ptr, c_i32, c_ptr, c_ptr, c_ptr, c_ptr, c_size, c_ptr, c_ptr]),
+    "umim_kv_rollback_rope": (ctypes.c_int, [ctypes.POINTER(PagedKVC), c_ptr, c_i32, c_ptr, c_i32, c_ptr, c_ptr,
+                                             c_ptr, c_i32, c_ptr, c_ptr, c_ptr, c_i32, c_ptr, c_ptr, c_size, c_ptr,
+                                             c_ptr]),
     "umim_kv_append": (ctypes.c_int, [ctypes.POINTER(PagedKVC), c_ptr, c_i32, c_ptr, c_i32, c_ptr, c_ptr, c_ptr,
                                       c_ptr, c_ptr]),
     "umim_decode_append_merge": (ctypes.c_int, [ctypes.POINTER(PagedKVC), c_ptr, c_i32, c_ptr, c_i32, c_ptr, c_ptr,

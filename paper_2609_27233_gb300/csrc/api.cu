@@ -38,7 +38,7 @@ umim_status build_compressed(const void *, int64_t, int, const int32_t *, int, i
 size_t kv_rollback_workspace_bytes(int B, int S, int max_pages, int n_layers, int n_kv_heads, int head_dim);
 umim_status kv_rollback(const umim_paged_kv *, int32_t *, int32_t, int32_t *, int32_t, const int32_t *,
                         const int32_t *, const int32_t *, int32_t, const void *, const void *, int32_t *, void *,
-                        size_t, int32_t *, cudaStream_t, int);
+                        size_t, int32_t *, cudaStream_t, int, const float *, int);
 umim_status kv_append(const umim_paged_kv *, int32_t *, int32_t, int32_t *, int32_t, const void *, const void *,
                       const int32_t *, int32_t *, cudaStream_t);
 umim_status decode_append_merge(const umim_paged_kv *, int32_t *, int32_t, int32_t *, int32_t, const void *,
@@ -191,13 +191,17 @@ size_t umim_kv_rollback_workspace_size(int32_t batch, int32_t n_spans, int32_t m
   return kv_rollback_workspace_bytes(batch, n_spans, max_pages, n_layers, n_kv_heads, head_dim);
 }
 
-umim_status umim_kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t max_pages, int32_t *seq_lens,
+namespace {
+umim_status rollback_checked(const umim_paged_kv *kv, int32_t *block_table, int32_t max_pages, int32_t *seq_lens,
                              int32_t batch, const int32_t *span_offsets, const int32_t *span_start,
                              const int32_t *span_len, int32_t n_spans, const void *surrogate_k,
                              const void *surrogate_v, int32_t *freed_pages, void *workspace,
-                             size_t workspace_bytes, int32_t *dev_status, cudaStream_t stream) {
+                             size_t workspace_bytes, int32_t *dev_status, cudaStream_t stream,
+                             const float *rope_inv_freq, int32_t rotary_dim) {
   if (!kv_ok(kv) || batch < 0 || max_pages < 0 || n_spans < 0) return UMIM_ERR_INVALID_ARG;
   if (!kv_supported(kv)) return UMIM_ERR_UNSUPPORTED;
+  if (rope_inv_freq && (rotary_dim <= 0 || rotary_dim % 16 != 0 || rotary_dim > kv->head_dim))
+    return UMIM_ERR_INVALID_ARG;
   if ((int64_t)batch * max_pages > INT32_MAX / 16 || batch > 65535) return UMIM_ERR_UNSUPPORTED;
   // work units (sequence x page x layer x K|V x head) are indexed in 32 bits
   if ((int64_t)batch * max_pages * kv->n_layers * 2 * kv->n_kv_heads >= INT32_MAX / 2) return UMIM_ERR_UNSUPPORTED;
@@ -211,7 +215,31 @@ umim_status umim_kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int3
     return UMIM_ERR_WORKSPACE;
   const int sms = prepare_device(stream);
   return kv_rollback(kv, block_table, max_pages, seq_lens, batch, span_offsets, span_start, span_len, n_spans,
-                     surrogate_k, surrogate_v, freed_pages, workspace, workspace_bytes, dev_status, stream, sms);
+                     surrogate_k, surrogate_v, freed_pages, workspace, workspace_bytes, dev_status, stream, sms,
+                     rope_inv_freq, rotary_dim);
+}
+}  // namespace
+
+umim_status umim_kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t max_pages, int32_t *seq_lens,
+                             int32_t batch, const int32_t *span_offsets, const int32_t *span_start,
+                             const int32_t *span_len, int32_t n_spans, const void *surrogate_k,
+                             const void *surrogate_v, int32_t *freed_pages, void *workspace,
+                             size_t workspace_bytes, int32_t *dev_status, cudaStream_t stream) {
+  return rollback_checked(kv, block_table, max_pages, seq_lens, batch, span_offsets, span_start, span_len, n_spans,
+                          surrogate_k, surrogate_v, freed_pages, workspace, workspace_bytes, dev_status, stream,
+                          nullptr, 0);
+}
+
+umim_status umim_kv_rollback_rope(const umim_paged_kv *kv, int32_t *block_table, int32_t max_pages,
+                                  int32_t *seq_lens, int32_t batch, const int32_t *span_offsets,
+                                  const int32_t *span_start, const int32_t *span_len, int32_t n_spans,
+                                  const void *surrogate_k, const void *surrogate_v, const float *rope_inv_freq,
+                                  int32_t rotary_dim, int32_t *freed_pages, void *workspace, size_t workspace_bytes,
+                                  int32_t *dev_status, cudaStream_t stream) {
+  if (!rope_inv_freq) return UMIM_ERR_INVALID_ARG;
+  return rollback_checked(kv, block_table, max_pages, seq_lens, batch, span_offsets, span_start, span_len, n_spans,
+                          surrogate_k, surrogate_v, freed_pages, workspace, workspace_bytes, dev_status, stream,
+                          rope_inv_freq, rotary_dim);
 }
 
 umim_status umim_kv_append(const umim_paged_kv *kv, int32_t *block_table, int32_t max_pages, int32_t *seq_lens,

@@ -44,6 +44,8 @@ struct MoveArgs {
   int32_t freed_capacity;
   int32_t B;
   int32_t *status;
+  const float *rope_inv_freq;   // [rotary_dim / 2] or nullptr: keys move verbatim
+  int32_t rotary_dim;
 };
 
 // largest i in [lo, hi) with key(i) <= x, or lo - 1
@@ -84,6 +86,7 @@ struct RowDep {
 struct PageDesc {
   int64_t *src;    // [rows][16] source row offset within a layer (no head offset), -(i+1) for span i, kNoWrite
   RowDep *dep;     // [rows]
+  int32_t *shift;  // [rows][16] r of a moved kept entry (positions removed before it), else 0
 };
 
 // Sixteen threads per (sequence, compacted page): where each of its 16
@@ -98,6 +101,7 @@ __global__ void __launch_bounds__(256) rollback_map_kernel(MoveArgs a, PlanArray
   const int nd = arr.n_dest[b];
   const bool row_ok = k < nd;
   int64_t src = kNoWrite;
+  int32_t shift = 0;
   int rd_lo = INT32_MAX, rd_hi = -1;
   int idx = 0;
   if (row_ok) {
@@ -115,7 +119,10 @@ __global__ void __launch_bounds__(256) rollback_map_kernel(MoveArgs a, PlanArray
           src = -(int64_t)i - 1;
         } else {
           const int t = j + arr.r_incl[i];
-          if (t != j) src = (int64_t)bt[t / kPageSize] * page_stride + (t % kPageSize) * D;
+          if (t != j) {
+            src = (int64_t)bt[t / kPageSize] * page_stride + (t % kPageSize) * D;
+            shift = t - j;
+          }
         }
       }
     }
@@ -134,6 +141,7 @@ __global__ void __launch_bounds__(256) rollback_map_kernel(MoveArgs a, PlanArray
   }
   if (!row_ok) return;
   pd.src[(int64_t)idx * kPageSize + slot] = src;
+  pd.shift[(int64_t)idx * kPageSize + slot] = shift;
   if (slot == 0) {
     rd_hi = min(rd_hi, k - 1);   // the row itself reads only its own units' columns
     RowDep d;
@@ -163,7 +171,7 @@ __device__ __forceinline__ bool wait_landed(const int32_t *cnt, int target, cons
 // (slot) c / CPR, column c % CPR.  Step: the next unit's loads land and it is
 // counted in; this unit waits for its page's readers and is stored; the unit
 // after next is loaded into its registers.
-template <int D>
+template <int D, bool ROPE>
 __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs a, PlanArrays arr, PageDesc pd) {
   constexpr int CPR = D / 8;                       // 16-byte chunks per row
   constexpr int PER_LANE = kPageSize * CPR / 32;   // 8 (D=128) or 4 (D=64)
@@ -175,7 +183,10 @@ __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs
   const int my_slot0 = lane / CPR;
   __shared__ int s_last;
   __shared__ int s_sq[kSmemSeqs], s_nd[kSmemSeqs], s_ub[kSmemSeqs], s_fp[kSmemSeqs];
+  __shared__ float s_w[ROPE ? D / 2 : 1];   // RoPE angular frequencies
 
+  if (ROPE)
+    for (int i = threadIdx.x; i < a.rotary_dim / 2; i += blockDim.x) s_w[i] = a.rope_inv_freq[i];
   griddep_wait();
   const PlanHeader *hdr = arr.hdr;
   int32_t *abort_flag = &arr.hdr->ticket;
@@ -212,14 +223,17 @@ __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs
   struct Tile {
     uint4 v[PER_LANE];
     uint32_t mask;
-    int valid;
+    int valid, rot;     // rot: a K tile whose moved entries get re-rotated
     int64_t dst;
     int32_t row, dlo, dhi;
+    int32_t shift;      // lanes < 16: the shift of slot `lane`
   };
   // slot i = kk * row_size + pos, kk the compacted page row
   auto load = [&](int kk, int pos, Tile &t) {
     t.mask = 0;
     t.valid = 0;
+    t.rot = 0;
+    t.shift = 0;
     t.dst = 0;
     t.row = 0;
     t.dlo = 1;
@@ -239,6 +253,10 @@ __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs
     t.valid = 1;
     t.row = idx;
     t.dst = tile + (int64_t)page * page_stride32;
+    if (ROPE) {
+      t.rot = kv == 0;
+      t.shift = lane < kPageSize ? pd.shift[(int64_t)idx * kPageSize + lane] : 0;
+    }
 #pragma unroll
     for (int it = 0; it < PER_LANE; ++it) {
       const int slot = my_slot0 + it * SLOT_STEP;
@@ -270,6 +288,66 @@ __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs
     __syncwarp();
     if (t.valid && lane == 0) red_release_add(&pd.dep[t.row].landed, 1);
   };
+  // RoPE: a moved key (shift r) is rotated by -r w_m on the pairs (m, m + rotary_dim/2):
+  // x' = x cos + y sin, y' = y cos - x sin.  The lane holding chunk c of a slot's
+  // row takes its partner chunk from the lane holding c +- rotary_dim/16.  The
+  // angle is r w rounded plus its exact rounding error (an fma), the error
+  // folded into the sine and cosine to first order; the rounded angle is
+  // reduced to [-pi, pi] (Cody and Waite's three-part reduction) for the
+  // hardware sine and cosine, whose error there (about 2^-21) is far below
+  // the bf16 result's resolution.
+  auto rotate = [&](Tile &t) {
+    if (!ROPE || !t.rot) return;
+    const int hc = a.rotary_dim / 16;   // 16-byte chunks in each half of the rotated columns
+    const bool in_x = my_col < hc, in_y = my_col >= hc && my_col < 2 * hc;
+    const int partner = lane - my_col + (in_x ? my_col + hc : (in_y ? my_col - hc : my_col));
+    const int m0 = (in_x || in_y) ? 8 * (in_x ? my_col : my_col - hc) : 0;   // lanes past rotary_dim: unused
+    const int mine = in_y ? 1 : 0;   // of each element pair (2q, 2q+1) this lane evaluates element 2q + mine
+#pragma unroll
+    for (int it = 0; it < PER_LANE; ++it) {
+      const int slot = my_slot0 + it * SLOT_STEP;
+      const float rf = (float)__shfl_sync(0xffffffffu, t.shift, slot);   // 0: the identity (same bytes)
+      uint4 pv;
+      pv.x = __shfl_sync(0xffffffffu, t.v[it].x, partner);
+      pv.y = __shfl_sync(0xffffffffu, t.v[it].y, partner);
+      pv.z = __shfl_sync(0xffffffffu, t.v[it].z, partner);
+      pv.w = __shfl_sync(0xffffffffu, t.v[it].w, partner);
+      // the x and y lanes of a pair need the same angles: each evaluates half and they swap
+      float sn_m[4], cs_m[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const float w = s_w[m0 + 2 * q + mine];
+        const float ang = rf * w;
+        const float err = fmaf(rf, w, -ang);
+        const float kq = rintf(ang * 0.15915493667125702f);
+        float red = fmaf(-kq, 6.28125f, ang);
+        red = fmaf(-kq, 0.0019354820251464844f, red);
+        red = fmaf(-kq, -1.7484555314695172e-07f, red);
+        const float sn = __sinf(red), cs = __cosf(red);
+        sn_m[q] = fmaf(err, cs, sn);
+        cs_m[q] = fmaf(-err, sn, cs);
+      }
+      const uint32_t own[4] = {t.v[it].x, t.v[it].y, t.v[it].z, t.v[it].w};
+      const uint32_t oth[4] = {pv.x, pv.y, pv.z, pv.w};
+      uint32_t out[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const float sn_o = __shfl_sync(0xffffffffu, sn_m[q], partner);
+        const float cs_o = __shfl_sync(0xffffffffu, cs_m[q], partner);
+        float res[2];
+#pragma unroll
+        for (int hlf = 0; hlf < 2; ++hlf) {
+          const float sn = hlf == mine ? sn_m[q] : sn_o, cs = hlf == mine ? cs_m[q] : cs_o;
+          const float x = __uint_as_float(hlf ? (own[q] & 0xFFFF0000u) : (own[q] << 16));
+          const float y = __uint_as_float(hlf ? (oth[q] & 0xFFFF0000u) : (oth[q] << 16));
+          res[hlf] = in_x ? fmaf(x, cs, y * sn) : fmaf(x, cs, -(y * sn));
+        }
+        const __nv_bfloat162 b2 = __floats2bfloat162_rn(res[0], res[1]);
+        out[q] = *reinterpret_cast<const uint32_t *>(&b2);
+      }
+      if (in_x || in_y) t.v[it] = make_uint4(out[0], out[1], out[2], out[3]);
+    }
+  };
   // every reader of the unit's old page has its loads landed
   auto readers_done = [&](const Tile &t) -> bool {
     for (int rw = t.dlo; rw <= t.dhi; ++rw)
@@ -296,13 +374,16 @@ __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs
     load(kk, pos, B);
     advance();
     land_and_count(A);
-    // unit u in `cur` (landed, counted), unit u + 1 in flight in `next`
+    rotate(A);
+    // unit u in `cur` (landed, counted, rotated), unit u + 1 in flight in `next`;
+    // the next unit is rotated while unit u + 2's loads are in flight
     auto step = [&](Tile &cur, Tile &next) -> bool {
       land_and_count(next);
       if (!readers_done(cur)) return false;
       store(cur);
       load(kk, pos, cur);   // unit u + 2
       advance();
+      rotate(next);
       return true;
     };
     for (int u = 0; u < my_units; u += 2) {
@@ -355,14 +436,15 @@ size_t kv_rollback_workspace_bytes(int B, int S, int max_pages, int n_layers, in
   (void)n_layers;
   (void)n_kv_heads;
   const size_t pages = (size_t)B * max_pages > 0 ? (size_t)B * max_pages : 1;
-  return plan_bytes(B, S) + align256(sizeof(int64_t) * kPageSize * pages) + align256(sizeof(RowDep) * pages);
+  return plan_bytes(B, S) + align256(sizeof(int64_t) * kPageSize * pages) + align256(sizeof(RowDep) * pages) +
+         align256(sizeof(int32_t) * kPageSize * pages);
 }
 
 umim_status kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t max_pages, int32_t *seq_lens,
                         int32_t B, const int32_t *span_offsets, const int32_t *span_start,
                         const int32_t *span_len, int32_t S, const void *sur_k, const void *sur_v,
                         int32_t *freed_pages, void *ws, size_t ws_bytes, int32_t *dev_status,
-                        cudaStream_t stream, int num_sms) {
+                        cudaStream_t stream, int num_sms, const float *rope_inv_freq, int rotary_dim) {
   const int D = kv->head_dim;
   const int lanes = kv->n_layers * 2 * kv->n_kv_heads;   // one unit per (layer, K|V, head) tile
   PlanArrays arr = plan_carve(ws, B, S);
@@ -371,6 +453,7 @@ umim_status kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t m
   pd.src = reinterpret_cast<int64_t *>(arr.flags);   // the page descriptions follow the plan
   const size_t pages = (size_t)B * max_pages > 0 ? (size_t)B * max_pages : 1;
   pd.dep = reinterpret_cast<RowDep *>(reinterpret_cast<char *>(pd.src) + align256(sizeof(int64_t) * kPageSize * pages));
+  pd.shift = reinterpret_cast<int32_t *>(reinterpret_cast<char *>(pd.dep) + align256(sizeof(RowDep) * pages));
 
   PlanArgs pa{};
   pa.seq_lens = seq_lens;
@@ -409,7 +492,11 @@ umim_status kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t m
   ma.freed_capacity = (int32_t)std::min<int64_t>((int64_t)B * max_pages, INT32_MAX);
   ma.B = B;
   ma.status = status;
-  auto kern = (D == 128) ? rollback_move_kernel<128> : rollback_move_kernel<64>;
+  ma.rope_inv_freq = rope_inv_freq;
+  ma.rotary_dim = rope_inv_freq ? rotary_dim : 0;
+  const bool rope = rope_inv_freq != nullptr;
+  auto kern = D == 128 ? (rope ? rollback_move_kernel<128, true> : rollback_move_kernel<128, false>)
+                       : (rope ? rollback_move_kernel<64, true> : rollback_move_kernel<64, false>);
   const int smem = 0;
   int per_sm = 0;
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kMoveThreads, smem) != cudaSuccess || per_sm < 1)
