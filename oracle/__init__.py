@@ -30,6 +30,10 @@ for indices and moved KV bytes:
                           test of the raw generated suffix after every token
   rules.lookup            App. E (potential engineering optimizations):
                           surrogates precomputed per rule, fetched by id
+  prefill.prefill_attention
+                          App. E ("Prompt Merging"), App. C.5: the backbone's
+                          causal grouped-query attention over the packed
+                          compressed prompts
 
 bf16 values are represented by their raw bit patterns (numpy uint16) and
 upcast exactly to float64.
@@ -48,8 +52,10 @@ Parity status per function (what pins it is in tests/test_oracle_*.py):
   SuffixState       pinned (worked example, list model with markers,
                     equality with prompt matching for 2-gram rules)
   lookup            pinned (equals merging the matched spans)
+  prefill_attention pinned (library causal SDPA, closed forms, packing,
+                    last row = decode attention)
 """
-from . import bf16, spans, merge, rollback, append, attention, compaction, rules  # noqa: F401
+from . import bf16, spans, merge, rollback, append, attention, compaction, rules, prefill  # noqa: F401
 from .merge import merge_spans, merge_span_reference_steps  # noqa: F401
 from .rollback import kv_rollback  # noqa: F401
 from .append import kv_append  # noqa: F401
