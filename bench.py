@@ -27,6 +27,9 @@ to speed it up: longest-first rule matching against a table of the Llama-3
 rule counts (2.17 million 2- to 4-grams), surrogates fetched from a per-rule
 lookup table instead of the merge module, then the packed prompts; it also
 reports the per-call time of decoding-time suffix matching for 128 sequences.
+--workload prefill times causal prefill attention (one Llama-3-8B layer) over
+the compressed prompts of the prompt-compression workload and, beside it,
+over the same prompts uncompressed.
 --workload serving times the serving decode loop instead (128 sequences of
 lognormal length, 32 layers of 32/8 heads, 256 steps; every step appends one
 entry per sequence and layer, merges the last 2..4 stored entries of each
@@ -293,7 +296,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--workload", default="llama8b_layer",
-                    choices=["llama8b_layer", "serving", "prompt_compression", "long_context", "rule_matching"])
+                    choices=["llama8b_layer", "serving", "prompt_compression", "long_context", "rule_matching",
+                             "prefill"])
     ap.add_argument("--coverage", type=float, default=0.4, help="long_context span coverage")
     ap.add_argument("--rope", action="store_true",
                     help="llama8b_layer / long_context: re-rotate moved keys to their compressed positions "
@@ -304,7 +308,7 @@ def main():
     args = ap.parse_args()
     if args.workload == "serving" and args.impl == "umim":
         return serving_bench(args)
-    if args.workload in ("prompt_compression", "long_context", "rule_matching") and args.impl == "umim":
+    if args.workload in ("prompt_compression", "long_context", "rule_matching", "prefill") and args.impl == "umim":
         return side_bench(args)
     K, Wm = args.steps, max(3, args.warmup)
 
@@ -922,6 +926,56 @@ def side_bench(args):
                "decode_suffix_match_kernel_us": round(suffix_kernel_us, 2), "decode_suffix_batch": Bs,
                "l2": "the 64 MB rule table stays in L2 between steps (it is persistent); the looked-up rows, "
                      "the 1.05 GB embedding table and the packed output are larger than L2"}
+    elif args.workload == "prefill":
+        seed = W.SEEDS["prompt_compression"]
+        B, L, Hq, Hkv, D = 64, 2048, 32, 8, 128
+        pc = W.prompt_case(seed, B=B, L=L, vocab=128256, d=8, coverage=0.4)
+        offs_np, ln_np = pc.span_offsets.numpy(), pc.span_len.numpy()
+        lens_c = [L - int((ln_np[offs_np[b]:offs_np[b + 1]] - 1).sum()) for b in range(B)]
+        Tc, Tu = sum(lens_c), B * L
+        cu_c = torch.tensor(np.concatenate([[0], np.cumsum(lens_c)]), dtype=torch.int32, device=dev)
+        cu_u = torch.arange(0, Tu + 1, L, dtype=torch.int32, device=dev)
+        qkv_u = [W.bf16_normal((Tu, h, D), 1.0, seed + 401 + i, dev) for i, h in enumerate((Hq, Hkv, Hkv))]
+        qkv_c = [x[:Tc] for x in qkv_u]   # the compressed rows (values do not matter for timing)
+        out = torch.empty_like(qkv_u[0])
+        ws_p = umim.workspace(umim.umim_prefill_attention_workspace_size(B), dev)
+        phase = ["compressed"]
+
+        def step(i):
+            if phase[0] == "compressed":
+                umim.umim_prefill_attention(*qkv_c, cu_c, out=out, workspace_buf=ws_p, dev_status=status)
+            else:
+                umim.umim_prefill_attention(*qkv_u, cu_u, out=out, workspace_buf=ws_p, dev_status=status)
+
+        def causal_flops(lens):
+            return float(sum(2.0 * D * Hq * Lb * (Lb + 1) for Lb in lens))
+
+        restore = None
+        fl_c = causal_flops(lens_c)
+        work_of = {"prefill.attention": ("tensor", fl_c / 1e12, "TFLOP/s", peaks["bf16"])}
+        units, unit = Tc, "compressed rows/s"
+        metric = "prefill attention over compressed prompts: compressed prompt rows/s (one Llama-3-8B layer)"
+        # the uncompressed prompts, for the ratio the paper's prefill speedup rests on
+        phase[0] = "uncompressed"
+        for i in range(max(3, args.warmup)):
+            step(i)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for i in range(args.steps):
+            step(i)
+        e1.record()
+        torch.cuda.synchronize()
+        unc_ms = e0.elapsed_time(e1) / args.steps
+        phase[0] = "compressed"
+        cfg = {"workload": "prefill attention of one Llama-3-8B layer (32/8 heads, head_dim 128, causal, bf16) "
+                           "over 64 prompts of 2048 tokens compressed at 40% span coverage (the prompt-compression "
+                           "workload's packed output shape), against the same prompts uncompressed",
+               "compressed_rows": Tc, "uncompressed_rows": Tu, "mean_compressed_length": round(Tc / B, 1),
+               "uncompressed_ms": round(unc_ms, 4),
+               "uncompressed_tflops": round(causal_flops([L] * B) / unc_ms / 1e9, 1),
+               "kernel": "mma.sync m16n8k16 (P split into bf16 high + remainder), cp.async double buffering",
+               "l2": "q/k/v of one layer are 0.96 GB (compressed) / 1.34 GB (uncompressed): larger than L2"}
     else:
         name = "long_context" if abs(args.coverage - 0.4) < 1e-9 else "long_context_tr40"
         seed = W.SEEDS[name]
@@ -1016,6 +1070,8 @@ def side_bench(args):
     umim.trace_stop()
     recs = umim.trace_read(64 * (K + 2))
     kernels = kernel_table(recs, K, work_of)
+    if args.workload == "prefill":
+        cfg["speedup_from_compression"] = round(cfg["uncompressed_ms"] / (ms / K), 3)
     line = {"metric": metric, "value": units * K / (ms / 1000.0), "unit": unit, "n_gpus": 1, "steps": K,
             "warmup": Wm, "ms_per_step": ms / K, "higher_is_better": True, "dtype": "bf16", "data": "synthetic",
             "config": cfg, "kernels": kernels, "gpu_launches": len(recs), "clocks": clk.summary(w0, w1),

@@ -327,6 +327,35 @@ umim_status umim_decode_attention(const void *q, int32_t n_q_heads, const umim_p
                                   size_t workspace_bytes, int32_t *dev_status, cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
+ * Prefill attention over packed compressed prompts (App. E "Prompt
+ * Merging", App. C.5: the compressed embeddings, with contiguous positions,
+ * go through the frozen backbone's prefill, whose causal self-attention then
+ * runs over the shorter sequences).  Sequence b owns rows cu_seqlens[b] ..
+ * cu_seqlens[b+1]-1 (the cu_seqlens umim_build_compressed writes); per
+ * sequence, with rows i, j counted inside it:
+ *   out[i, h] = sum_{j <= i} softmax_j(scale <q[i, h], k[j, g]>) v[j, g],
+ *   g = h / (n_q_heads / n_kv_heads),  scale = 1/sqrt(head_dim) if scale <= 0.
+ * Rotary embeddings are already applied to q and k by the caller.
+ * q            device bf16 [n_rows][n_q_heads][head_dim], 16-B aligned
+ * k, v         device bf16 [n_rows][n_kv_heads][head_dim], 16-B aligned
+ * cu_seqlens   device int32 [batch + 1], cu_seqlens[0] = 0, nondecreasing,
+ *              cu_seqlens[batch] <= n_rows
+ * out          device bf16 [n_rows][n_q_heads][head_dim] (rows outside every
+ *              sequence are not written)
+ * workspace    device, umim_prefill_attention_workspace_size() bytes, 256-B
+ *              aligned
+ * head_dim 64 or 128; n_q_heads a multiple of n_kv_heads (else
+ * UMIM_ERR_UNSUPPORTED).  Device-side errors: UMIM_ERR_INVALID_ARG for
+ * offsets that break the rules above (nothing is written).
+ * ------------------------------------------------------------------------ */
+size_t umim_prefill_attention_workspace_size(int32_t batch);
+
+umim_status umim_prefill_attention(const void *q, const void *k, const void *v, int32_t n_rows, int32_t n_q_heads,
+                                   int32_t n_kv_heads, int32_t head_dim, const int32_t *cu_seqlens, int32_t batch,
+                                   float scale, void *out, void *workspace, size_t workspace_bytes,
+                                   int32_t *dev_status, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
  * Merge rules (App. E "Rule Matching").  A rule is a token n-gram, n in
  * {2, 3, 4}; its rule id is its row in the list given to umim_rules_build.
  * The table is open addressing over 16-byte slots (the n-gram packed as four

@@ -61,3 +61,4 @@ from .rollback import kv_rollback  # noqa: F401
 from .append import kv_append  # noqa: F401
 from .attention import decode_attention  # noqa: F401
 from .compaction import build_compressed  # noqa: F401
+from .prefill import prefill_attention  # noqa: F401

@@ -11,6 +11,7 @@ points keep the C names:
   umim_kv_append          decode-step append of one KV entry per layer (App. E, Fig. 2)
   umim_decode_append_merge  append or suffix merge per sequence in one call (App. E decoding loop)
   umim_decode_attention   GQA decode attention over the compacted paged cache (App. I.1)
+  umim_prefill_attention  causal GQA attention over the packed compressed prompts (App. E, App. C.5)
   umim_rules_build, umim_match_prompts, umim_match_suffix, umim_lookup_surrogates
                           merge-rule table, longest-first span selection for prompts
                           and for decoding, and precomputed surrogates by rule id (App. E)
@@ -106,6 +107,10 @@ def umim_build_compressed_workspace_size(batch, n_spans):
 
 def umim_kv_rollback_workspace_size(batch, n_spans, max_pages, n_layers, n_kv_heads, head_dim):
     return int(lib().umim_kv_rollback_workspace_size(batch, n_spans, max_pages, n_layers, n_kv_heads, head_dim))
+
+
+def umim_prefill_attention_workspace_size(batch):
+    return int(lib().umim_prefill_attention_workspace_size(batch))
 
 
 def umim_decode_attention_workspace_size(batch, n_q_heads, n_kv_heads, head_dim):
@@ -259,6 +264,24 @@ def umim_decode_attention_static(q, pool, layer, block_table, seq_lens, scale=0.
 # ---------------------------------------------------------------------------
 # kernel tracing (profiling aid)
 # ---------------------------------------------------------------------------
+def umim_prefill_attention(q, k, v, cu_seqlens, scale=0.0, out=None, workspace_buf=None, dev_status=None,
+                           stream=None):
+    """out [T][Hq][D] bf16: causal grouped-query attention within each packed
+    sequence of q [T][Hq][D], k / v [T][Hkv][D] (cu_seqlens [B+1] on the device)."""
+    dev = _dev(q)
+    T, Hq, D = q.shape
+    Hkv = k.shape[1]
+    B = cu_seqlens.numel() - 1
+    if out is None:
+        out = torch.empty_like(q)
+    if workspace_buf is None:
+        workspace_buf = workspace(umim_prefill_attention_workspace_size(B), dev)
+    code = lib().umim_prefill_attention(_p(q), _p(k), _p(v), T, Hq, Hkv, D, _p(cu_seqlens), B, float(scale), _p(out),
+                                        _p(workspace_buf), workspace_buf.numel(), _p(dev_status), _stream(stream))
+    _check(code, "umim_prefill_attention")
+    return out
+
+
 def umim_rule_table_bytes(n_rules):
     return int(lib().umim_rule_table_bytes(n_rules))
 

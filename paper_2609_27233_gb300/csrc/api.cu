@@ -53,6 +53,9 @@ umim_status match_suffix(const void *, size_t, void *, const int32_t *, int, int
                          int32_t *, int32_t *, int32_t *, cudaStream_t);
 umim_status lookup_surrogates(const float *, int64_t, int, const int32_t *, int, const int32_t *, float *, int32_t *,
                               cudaStream_t, int);
+size_t prefill_attention_workspace_bytes(int B);
+umim_status prefill_attention(const void *, const void *, const void *, int, int, int, int, const int32_t *, int,
+                              float, void *, void *, int32_t *, cudaStream_t);
 size_t decode_attention_workspace_bytes(int B, int Hq, int Hkv, int D, int num_sms);
 umim_status decode_attention(const void *, int, const umim_paged_kv *, int, const int32_t *, int, const int32_t *,
                              int, float, void *, void *, int32_t *, cudaStream_t, int);
@@ -339,6 +342,28 @@ umim_status umim_lookup_surrogates(const float *lut, int64_t n_rules, int32_t d,
   if (!lut || !aligned(lut, 16) || !rule_ids || !out || !aligned(out, 16)) return UMIM_ERR_INVALID_ARG;
   const int sms = prepare_device(stream);
   return lookup_surrogates(lut, n_rules, d, rule_ids, n_max, n_dev, out, dev_status, stream, sms);
+}
+
+size_t umim_prefill_attention_workspace_size(int32_t batch) {
+  if (batch < 0) return 0;
+  return prefill_attention_workspace_bytes(batch);
+}
+
+umim_status umim_prefill_attention(const void *q, const void *k, const void *v, int32_t n_rows, int32_t n_q_heads,
+                                   int32_t n_kv_heads, int32_t head_dim, const int32_t *cu_seqlens, int32_t batch,
+                                   float scale, void *out, void *workspace, size_t workspace_bytes,
+                                   int32_t *dev_status, cudaStream_t stream) {
+  if (n_rows < 0 || batch < 0 || n_q_heads <= 0 || n_kv_heads <= 0) return UMIM_ERR_INVALID_ARG;
+  if ((head_dim != 64 && head_dim != 128) || n_q_heads % n_kv_heads != 0 || n_q_heads > 65535)
+    return UMIM_ERR_UNSUPPORTED;
+  if (batch == 0 || n_rows == 0) return UMIM_OK;
+  if (!q || !k || !v || !out || !cu_seqlens) return UMIM_ERR_INVALID_ARG;
+  if (!aligned(q, 16) || !aligned(k, 16) || !aligned(v, 16) || !aligned(out, 16)) return UMIM_ERR_INVALID_ARG;
+  if (!workspace || !aligned(workspace, 256) || workspace_bytes < prefill_attention_workspace_bytes(batch))
+    return UMIM_ERR_WORKSPACE;
+  prepare_device(stream);
+  return prefill_attention(q, k, v, n_rows, n_q_heads, n_kv_heads, head_dim, cu_seqlens, batch, scale, out,
+                           workspace, dev_status, stream);
 }
 
 size_t umim_decode_attention_workspace_size(int32_t batch, int32_t n_q_heads, int32_t n_kv_heads,
