@@ -497,6 +497,23 @@ umim_status umim_decode_attention_static(const void *q, int32_t n_q_heads, const
                                          int32_t *dev_status, cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
+ * Self-test of the bounded waits (not part of the method).  Every wait of
+ * the library on another agent (an mbarrier completed by TMA or the tensor
+ * cores, a counter raised by another CTA) gives up after a time limit (1 s
+ * inside the calls above), records UMIM_ERR_TIMEOUT in the status word and
+ * returns, so the context stays usable.  This call waits, with limit_us
+ * (1 .. 1e6) microseconds, on something that never happens:
+ *   which 0: an mbarrier that nobody arrives on;
+ *   which 1: flags[0] >= 1 with flags[1] as the abort word (the rollback
+ *            movers' wait); the caller keeps both at 0.
+ * flags       device int32 [2] (which 1) or NULL
+ * elapsed_ns  device uint64 [1] out, or NULL: how long the wait lasted
+ * The expected outcome is UMIM_ERR_TIMEOUT in dev_status.
+ * ------------------------------------------------------------------------ */
+umim_status umim_selftest_bounded_wait(int32_t which, uint32_t limit_us, const int32_t *flags,
+                                       uint64_t *elapsed_ns, int32_t *dev_status, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
  * Kernel tracing, for profiling (not part of the method).  Between
  * umim_trace_start and umim_trace_stop every call above records a CUDA
  * event on its stream before each kernel it launches and one after its last

@@ -282,6 +282,18 @@ def umim_prefill_attention(q, k, v, cu_seqlens, scale=0.0, out=None, workspace_b
     return out
 
 
+def umim_selftest_bounded_wait(which, limit_us, device, dev_status=None, stream=None):
+    """Run one of the library's bounded waits on something that never happens
+    (0: an mbarrier, 1: a counter); returns (status, elapsed_ns)."""
+    flags = torch.zeros(2, dtype=torch.int32, device=device)
+    elapsed = torch.zeros(1, dtype=torch.int64, device=device)
+    status = new_status(device) if dev_status is None else dev_status
+    code = lib().umim_selftest_bounded_wait(int(which), int(limit_us), _p(flags), _p(elapsed), _p(status),
+                                            _stream(stream))
+    _check(code, "umim_selftest_bounded_wait")
+    return status, elapsed
+
+
 def umim_rule_table_bytes(n_rules):
     return int(lib().umim_rule_table_bytes(n_rules))
 

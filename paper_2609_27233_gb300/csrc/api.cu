@@ -53,6 +53,7 @@ umim_status match_suffix(const void *, size_t, void *, const int32_t *, int, int
                          int32_t *, int32_t *, int32_t *, cudaStream_t);
 umim_status lookup_surrogates(const float *, int64_t, int, const int32_t *, int, const int32_t *, float *, int32_t *,
                               cudaStream_t, int);
+umim_status selftest_bounded_wait(int, uint32_t, const int32_t *, uint64_t *, int32_t *, cudaStream_t);
 size_t prefill_attention_workspace_bytes(int B);
 umim_status prefill_attention(const void *, const void *, const void *, int, int, int, int, const int32_t *, int,
                               float, void *, void *, int32_t *, cudaStream_t);
@@ -342,6 +343,14 @@ umim_status umim_lookup_surrogates(const float *lut, int64_t n_rules, int32_t d,
   if (!lut || !aligned(lut, 16) || !rule_ids || !out || !aligned(out, 16)) return UMIM_ERR_INVALID_ARG;
   const int sms = prepare_device(stream);
   return lookup_surrogates(lut, n_rules, d, rule_ids, n_max, n_dev, out, dev_status, stream, sms);
+}
+
+umim_status umim_selftest_bounded_wait(int32_t which, uint32_t limit_us, const int32_t *flags,
+                                       uint64_t *elapsed_ns, int32_t *dev_status, cudaStream_t stream) {
+  if ((which != 0 && which != 1) || limit_us == 0 || limit_us > 1000000u) return UMIM_ERR_INVALID_ARG;
+  if (which == 1 && !flags) return UMIM_ERR_INVALID_ARG;
+  prepare_device(stream);
+  return selftest_bounded_wait(which, limit_us, flags, elapsed_ns, dev_status, stream);
 }
 
 size_t umim_prefill_attention_workspace_size(int32_t batch) {

@@ -158,13 +158,7 @@ constexpr int kSmemSeqs = 1024;   // active sequences whose plan values a CTA ke
 // Waits until *cnt >= target; false when it gave up (time limit, or another
 // warp gave up: *abort != 0).
 __device__ __forceinline__ bool wait_landed(const int32_t *cnt, int target, const int32_t *abort) {
-  const uint64_t t0 = globaltimer();
-  while (true) {
-#pragma unroll 1
-    for (int i = 0; i < 32; ++i)
-      if (ld_acquire(cnt) >= target) return true;
-    if (ld_acquire(abort) != 0 || globaltimer() - t0 > kWaitLimitNs) return false;
-  }
+  return wait_count_for(cnt, target, abort, kWaitLimitNs);
 }
 
 // Mover warps: lane l moves 16-byte chunks c = l + 32 it of a unit, row
