@@ -64,10 +64,16 @@ umim_status decode_attention(const void *, int, const umim_paged_kv *, int, cons
 namespace {
 
 // Make the stream's device current for this runtime instance; return its SM count.
+// A stream being captured into a CUDA graph refuses cudaStreamGetDevice (and the
+// refusal invalidates the capture), so there the current device is taken.
 int prepare_device(cudaStream_t stream) {
   int dev = 0;
-  if (stream != nullptr && cudaStreamGetDevice(stream, &dev) == cudaSuccess) cudaSetDevice(dev);
-  else cudaGetDevice(&dev);
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  if (stream != nullptr && cudaStreamIsCapturing(stream, &cs) == cudaSuccess && cs == cudaStreamCaptureStatusNone &&
+      cudaStreamGetDevice(stream, &dev) == cudaSuccess)
+    cudaSetDevice(dev);
+  else
+    cudaGetDevice(&dev);
   static int cached_dev = -1, cached_sms = 0;
   if (dev != cached_dev) {
     int sms = 0;

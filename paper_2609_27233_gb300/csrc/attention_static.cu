@@ -70,8 +70,12 @@ umim_status umim_decode_attention_static(const void *q, int32_t n_q_heads, const
   if (!q || !block_table || !seq_lens || !out) return UMIM_ERR_INVALID_ARG;
   if ((reinterpret_cast<uintptr_t>(q) % 4) != 0 || (reinterpret_cast<uintptr_t>(out) % 2) != 0)
     return UMIM_ERR_INVALID_ARG;
+  // a stream being captured into a CUDA graph refuses cudaStreamGetDevice (the refusal would
+  // invalidate the capture): there the current device is the stream's
   int dev = 0;
-  if (stream != nullptr && cudaStreamGetDevice(stream, &dev) == cudaSuccess) {
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  if (stream != nullptr && cudaStreamIsCapturing(stream, &cs) == cudaSuccess && cs == cudaStreamCaptureStatusNone &&
+      cudaStreamGetDevice(stream, &dev) == cudaSuccess) {
     if (cudaSetDevice(dev) != cudaSuccess) return UMIM_ERR_CUDA;
   }
   void *scratch = nullptr;

@@ -266,3 +266,95 @@ def test_full_serving_workload_matches_oracle(fused):
                 float_close(got_out[b:b + 1], want, f"step {step} layer {layer} seq {b}")
             del init_layer
     assert n_rolled > 0
+
+
+def test_captured_step_replays_the_eager_fused_loop_bit_for_bit():
+    """The fused serving step (update + attention for every layer) captured
+    once as a CUDA graph and replayed with each step's inputs copied into its
+    static buffers gives, bit for bit, what the eager calls give."""
+    B, layers, hq, hkv, d, steps = 6, 3, 16, 4, 128, 30
+    lens = W.rng(35).integers(1, 200, size=B).astype(np.int32)
+    sl = W.serving_loop(35, B=B, n_layers=layers, n_q_heads=hq, n_kv_heads=hkv, head_dim=d, steps=steps, p=0.5,
+                        lens=lens)
+    dv = dev()
+    m = umim()
+    # host bookkeeping of the loop: pages handed out, merges per step
+    alloc = W.PageAllocator(sl.free_pages)
+    o_lens, o_bt = sl.lens.copy(), sl.block_table.copy()
+    o_pool = np.zeros((1, sl.n_pages, 2, 1, 16, 1), np.uint16)   # indices only: values are irrelevant here
+    sched = []
+    for step in range(steps):
+        new_pages = alloc.take(o_lens)
+        zeros = np.zeros((B, 1, 1, 1), np.uint16)
+        o_pool, o_bt, o_lens, _ = oracle.kv_append(o_pool, o_bt, o_lens, zeros, zeros, new_pages)
+        offs, st, ln = _spans(sl.rollbacks(step), o_lens, B)
+        S = len(st)
+        o_pool, o_bt, o_lens, freed = oracle.kv_rollback(o_pool, o_bt, o_lens, offs, st, ln,
+                                                        np.zeros((S, 1, 1, 1), np.uint16),
+                                                        np.zeros((S, 1, 1, 1), np.uint16))
+        alloc.give_back(freed)
+        mk, mr = np.zeros(B, np.int32), np.full(B, -1, np.int32)
+        for b in range(B):
+            if offs[b + 1] > offs[b]:
+                mk[b], mr[b] = ln[offs[b]], offs[b]
+        sched.append((new_pages, mk, mr, S))
+    t = lambda a: torch.from_numpy(a).to(dv)
+    entries = [sl.new_entries(s, dv) for s in range(steps)]
+    surs = [sl.surrogates(s, sched[s][3], dv) for s in range(steps)]
+    qs = [sl.q(0, layer, dv) for layer in range(layers)]
+    ws_a = m.workspace(m.umim_decode_attention_workspace_size(B, hq, hkv, d), dv)
+
+    def fresh():
+        return sl.init_pool(dv), t(sl.block_table.copy()), t(sl.lens.copy())
+
+    # eager
+    pool, bt, ln_ = fresh()
+    status = m.new_status(dv)
+    rel = torch.empty(B, dtype=torch.int32, device=dv)
+    eager = []
+    for s in range(steps):
+        np_, mk, mr, S = sched[s]
+        m.umim_decode_append_merge(pool, bt, ln_, entries[s][0], entries[s][1], t(np_), t(mk), t(mr), surs[s][0],
+                                   surs[s][1], released=rel, dev_status=status)
+        outs = [m.umim_decode_attention(qs[l], pool, l, bt, ln_, workspace_buf=ws_a, dev_status=status)
+                for l in range(layers)]
+        eager.append(([o.clone() for o in outs], rel.clone()))
+    e_pool, e_bt, e_len = pool.clone(), bt.clone(), ln_.clone()
+    # captured once, replayed every step
+    pool, bt, ln_ = fresh()
+    n_max = max(1, max(x[3] for x in sched))
+    st_nk, st_nv = torch.empty_like(entries[0][0]), torch.empty_like(entries[0][1])
+    st_np, st_mk, st_mr = (torch.empty(B, dtype=torch.int32, device=dv) for _ in range(3))
+    st_sk = torch.zeros((n_max, layers, hkv, d), dtype=torch.bfloat16, device=dv)
+    st_sv = torch.zeros_like(st_sk)
+    g_outs = [torch.empty_like(qs[0]) for _ in range(layers)]
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        m.umim_decode_append_merge(pool, bt, ln_, st_nk, st_nv, st_np, st_mk, st_mr, st_sk, st_sv, released=rel,
+                                   dev_status=status)
+        for l in range(layers):
+            m.umim_decode_attention(qs[l], pool, l, bt, ln_, out=g_outs[l], workspace_buf=ws_a, dev_status=status)
+    for s in range(steps):
+        np_, mk, mr, S = sched[s]
+        st_nk.copy_(entries[s][0])
+        st_nv.copy_(entries[s][1])
+        st_np.copy_(t(np_))
+        st_mk.copy_(t(mk))
+        st_mr.copy_(t(mr))
+        if S:
+            st_sk[:S].copy_(surs[s][0])
+            st_sv[:S].copy_(surs[s][1])
+        graph.replay()
+        for l in range(layers):
+            assert torch.equal(g_outs[l], eager[s][0][l]), (s, l)
+        assert torch.equal(rel, eager[s][1]), s
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    assert torch.equal(bt, e_bt) and torch.equal(ln_, e_len)
+    tl = e_len.cpu().numpy()
+    btn = e_bt.cpu().numpy()
+    gp, ep = W.bits(pool), W.bits(e_pool)
+    for b in range(B):
+        tt = np.arange(int(tl[b]))
+        pg, slot = btn[b, tt // 16], tt % 16
+        np.testing.assert_array_equal(gp[:, pg, :, :, slot, :], ep[:, pg, :, :, slot, :])
