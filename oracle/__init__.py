@@ -34,6 +34,11 @@ for indices and moved KV bytes:
                           App. E ("Prompt Merging"), App. C.5: the backbone's
                           causal grouped-query attention over the packed
                           compressed prompts
+  distill.align / soft_ce
+                          App. F (Algorithm 1, the masked distillation
+                          loss): teacher / student alignment masks packed
+                          into pairs, the soft cross-entropy and its
+                          gradient with respect to the student logits
 
 bf16 values are represented by their raw bit patterns (numpy uint16) and
 upcast exactly to float64.
@@ -54,8 +59,11 @@ Parity status per function (what pins it is in tests/test_oracle_*.py):
   lookup            pinned (equals merging the matched spans)
   prefill_attention pinned (library causal SDPA, closed forms, packing,
                     last row = decode attention)
+  align / soft_ce   pinned (the paper's alignment example, the compressed-
+                    position map, library soft cross-entropy and KL,
+                    autograd)
 """
-from . import bf16, spans, merge, rollback, append, attention, compaction, rules, prefill  # noqa: F401
+from . import bf16, spans, merge, rollback, append, attention, compaction, rules, prefill, distill  # noqa: F401
 from .merge import merge_spans, merge_span_reference_steps  # noqa: F401
 from .rollback import kv_rollback  # noqa: F401
 from .append import kv_append  # noqa: F401
