@@ -30,6 +30,9 @@ reports the per-call time of decoding-time suffix matching for 128 sequences.
 --workload prefill times causal prefill attention (one Llama-3-8B layer) over
 the compressed prompts of the prompt-compression workload and, beside it,
 over the same prompts uncompressed.
+--workload distill times the training-side step (App. F, Algorithm 1): the
+alignment of teacher and student rows, then the full-vocabulary soft-target
+cross-entropy and its gradient over 8 x 512 tokens of Llama-3 logits.
 --workload serving times the serving decode loop instead (128 sequences of
 lognormal length, 32 layers of 32/8 heads, 256 steps; every step appends one
 entry per sequence and layer, merges the last 2..4 stored entries of each
@@ -297,7 +300,7 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--workload", default="llama8b_layer",
                     choices=["llama8b_layer", "serving", "prompt_compression", "long_context", "rule_matching",
-                             "prefill"])
+                             "prefill", "distill"])
     ap.add_argument("--coverage", type=float, default=0.4, help="long_context span coverage")
     ap.add_argument("--rope", action="store_true",
                     help="llama8b_layer / long_context: re-rotate moved keys to their compressed positions "
@@ -308,7 +311,8 @@ def main():
     args = ap.parse_args()
     if args.workload == "serving" and args.impl == "umim":
         return serving_bench(args)
-    if args.workload in ("prompt_compression", "long_context", "rule_matching", "prefill") and args.impl == "umim":
+    if args.workload in ("prompt_compression", "long_context", "rule_matching", "prefill", "distill") and \
+            args.impl == "umim":
         return side_bench(args)
     K, Wm = args.steps, max(3, args.warmup)
 
@@ -1023,6 +1027,46 @@ def side_bench(args):
                "uncompressed_tflops": round(causal_flops([L] * B) / unc_ms / 1e9, 1),
                "kernel": "mma.sync m16n8k16 (P split into bf16 high + remainder), cp.async double buffering",
                "l2": "q/k/v of one layer are 0.96 GB (compressed) / 1.34 GB (uncompressed): larger than L2"}
+    elif args.workload == "distill":
+        seed = W.SEEDS["distillation"]
+        B, L, V = 8, 512, W.LLAMA3_VOCAB
+        c = W.distill_case(seed, lens=[L] * B, vocab=V, coverage=0.4, device=dev)
+        T_rows = B * L
+        i32 = lambda n: torch.empty(n, dtype=torch.int32, device=dev)
+        al = dict(pair_offsets=i32(B + 1), teacher_rows=i32(T_rows), student_rows=i32(T_rows), student_cu=i32(B + 1))
+        ws_al = umim.workspace(umim.umim_distill_align_workspace_size(B, c.span_start.numel()), dev)
+        umim.umim_distill_align(c.seq_lens, c.span_offsets, c.span_start, c.span_len, T_rows, out=al,
+                                workspace_buf=ws_al, dev_status=status)
+        R_S = int(al["student_cu"][B].item())
+        N = int(al["pair_offsets"][B].item())
+        stu = W.distill_logits(seed + 7, R_S, c.teacher_logits.shape[1], 2.0, dev)
+        loss = torch.empty(1, dtype=torch.float32, device=dev)
+        pl = torch.empty(T_rows, dtype=torch.float32, device=dev)
+        grad = torch.empty_like(stu)
+        ws_ce = umim.workspace(umim.umim_distill_soft_ce_workspace_size(R_S, T_rows), dev)
+        n_dev = al["pair_offsets"][B:]
+
+        def step(i):
+            umim.umim_distill_align(c.seq_lens, c.span_offsets, c.span_start, c.span_len, T_rows, out=al,
+                                    workspace_buf=ws_al, dev_status=status)
+            umim.umim_distill_soft_ce(c.teacher_logits, stu, al["teacher_rows"], al["student_rows"], n_pairs=n_dev,
+                                      vocab=V, loss=loss, pair_loss=pl, grad=grad, workspace_buf=ws_ce,
+                                      dev_status=status)
+
+        restore = None
+        ce_bytes = 2.0 * N * V * 2 + R_S * V * 2 + N * 16 + R_S * 4
+        work_of = {"distill.soft_ce": ("hbm", ce_bytes / 1e9, "GB/s", peaks["hbm"])}
+        units, unit = N, "aligned pairs/s"
+        metric = "aligned predictive distillation: aligned pairs/s (alignment + full-vocabulary soft-target " \
+                 "cross-entropy and its gradient)"
+        cfg = {"workload": "aligned predictive distillation of a Llama-3.1-8B-vocabulary batch: 8 sequences x 512 "
+                           "tokens (the paper's training length), 40% of tokens in spans of 2..4, bf16 teacher "
+                           "logits [4096][128256] and student logits over the compressed rows, N(0, 2^2); "
+                           "loss and bf16 gradient over the full vocabulary",
+               "pairs": N, "teacher_rows": T_rows, "student_rows": R_S, "vocab": V,
+               "algorithmic_gb_soft_ce": round(ce_bytes / 1e9, 4),
+               "l2": "inputs larger than L2: 1.05 GB of teacher logits and 0.77 GB of student logits read, "
+                     "0.77 GB of gradient written per step"}
     else:
         name = "long_context" if abs(args.coverage - 0.4) < 1e-9 else "long_context_tr40"
         seed = W.SEEDS[name]

@@ -467,6 +467,81 @@ umim_status umim_lookup_surrogates(const float *lut, int64_t n_rules, int32_t d,
                                    cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
+ * Aligned predictive distillation, the training objective of the merge
+ * module (App. F "Predictive Distillation Loss and Alignment Metrics",
+ * Algorithm 1 and the masked distillation loss).  The frozen backbone runs on
+ * the original sequences (teacher) and on the compressed ones (student); the
+ * two calls below pair their rows and compute the loss and its gradient with
+ * respect to the student logits.
+ *
+ * umim_distill_align: the masks and Pack of Algorithm 1 as row indices.  For
+ * sample b with original length L_b and sorted, non-overlapping spans
+ * (s_i, n_i), the keep mask marks every retained token and, for each span,
+ * only its last position s_i + n_i - 1; the teacher mask is the keep mask
+ * from the first span's start s_b on (N_b = its number of ones); the student
+ * mask marks the last N_b positions of the compressed sequence (length
+ * L~_b = L_b - sum (n_i - 1)); Pack pairs them in order.  A sample without
+ * spans has no pairs.  Rows are numbered over the packed batches: teacher
+ * row of (b, t) = sum_{b'<b} L_b' + t; student row of (b, j) =
+ * sum_{b'<b} L~_b' + j, the row order of umim_build_compressed's output.
+ * seq_lens      device int32 [batch] L_b
+ * span_offsets  device int32 [batch + 1] CSR over the spans; span_start /
+ *               span_len device int32 [n_spans], start relative to the sample
+ * pair_offsets  device int32 [batch + 1] out: pairs of sample b are
+ *               pair_offsets[b] .. pair_offsets[b+1]-1, in Pack order
+ * teacher_rows, student_rows  device int32 [capacity] out
+ * student_cu    device int32 [batch + 1] out, or NULL: prefix sums of L~_b
+ * workspace     device, umim_distill_align_workspace_size() bytes, 256-B
+ *               aligned, zero-filled before its first use
+ * Device-side errors: UMIM_ERR_INVALID_ARG (nothing written) for spans that
+ * are unsorted, overlap, are empty or pass L_b, a negative length, bad
+ * offsets, more pairs than capacity or more than 2^31 - 1 teacher rows.
+ *
+ * umim_distill_soft_ce: over the N aligned pairs (teacher row t_k, student
+ * row s_k), with P = softmax over the whole vocabulary of a logits row,
+ *   loss = -(1/N) sum_k sum_v P^T_k(v) log(P^S_k(v) + eps)
+ * and the gradient with respect to the student logits of row s_k
+ *   -(1/N) (a_v - P^S_k(v) sum_u a_u),  a_u = P^T_k(u) P^S_k(u) / (P^S_k(u) + eps);
+ * student rows in no pair have a zero gradient.  Computed in fp32 from bf16
+ * logits; each logit is read once.
+ * teacher_logits  device bf16 [n_teacher_rows][ld], 16-B aligned
+ * student_logits  device bf16 [n_student_rows][ld], 16-B aligned
+ * vocab, ld       vocabulary size (1 .. 163840) and row stride in elements
+ *                 (a multiple of 8, >= vocab rounded up to a multiple of 8;
+ *                 the elements from vocab up to that are read, never used)
+ * teacher_rows, student_rows  device int32 [max_pairs] (e.g. from
+ *                 umim_distill_align); each student row at most once
+ * n_pairs         device int32 [1] or NULL: N (NULL: N = max_pairs), e.g.
+ *                 pair_offsets + batch of umim_distill_align
+ * eps             the loss's stability constant (>= 0, finite)
+ * loss            device fp32 [1] out
+ * pair_loss       device fp32 [max_pairs] out, or NULL: each pair's
+ *                 -sum_v P^T log(P^S + eps)
+ * grad            device bf16 [n_student_rows][ld] out, or NULL (loss only);
+ *                 elements [0, vocab) of every row written
+ * workspace       device, umim_distill_soft_ce_workspace_size() bytes, 256-B
+ *                 aligned (no initial contents required)
+ * Host-side errors: UMIM_ERR_UNSUPPORTED for a vocabulary above 163840.
+ * Device-side errors: UMIM_ERR_INVALID_ARG (nothing written) for N outside
+ * [0, max_pairs], a row outside its logits or a student row in two pairs.
+ * ------------------------------------------------------------------------ */
+size_t umim_distill_align_workspace_size(int32_t batch, int32_t n_spans);
+
+umim_status umim_distill_align(const int32_t *seq_lens, int32_t batch, const int32_t *span_offsets,
+                               const int32_t *span_start, const int32_t *span_len, int32_t n_spans,
+                               int32_t *pair_offsets, int32_t *teacher_rows, int32_t *student_rows,
+                               int32_t capacity, int32_t *student_cu, void *workspace, size_t workspace_bytes,
+                               int32_t *dev_status, cudaStream_t stream);
+
+size_t umim_distill_soft_ce_workspace_size(int32_t n_student_rows, int32_t max_pairs);
+
+umim_status umim_distill_soft_ce(const void *teacher_logits, int32_t n_teacher_rows, const void *student_logits,
+                                 int32_t n_student_rows, int32_t vocab, int64_t ld, const int32_t *teacher_rows,
+                                 const int32_t *student_rows, int32_t max_pairs, const int32_t *n_pairs, float eps,
+                                 float *loss, float *pair_loss, void *grad, void *workspace,
+                                 size_t workspace_bytes, int32_t *dev_status, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
  * Decode attention for callers that cannot allocate GPU memory.
  * The paper has no counterpart to this call; it is a convenience of this
  * library.  A serving engine that gives all device memory to its own block

@@ -15,6 +15,10 @@ points keep the C names:
   umim_rules_build, umim_match_prompts, umim_match_suffix, umim_lookup_surrogates
                           merge-rule table, longest-first span selection for prompts
                           and for decoding, and precomputed surrogates by rule id (App. E)
+  umim_distill_align, umim_distill_soft_ce
+                          aligned predictive distillation: teacher/student row pairing
+                          and the full-vocabulary soft-target cross-entropy with its
+                          gradient (App. F, Algorithm 1)
 """
 import ctypes
 
@@ -375,6 +379,68 @@ def umim_lookup_surrogates(lut, rule_ids, n_dev=None, out=None, dev_status=None,
                                         _stream(stream))
     _check(code, "umim_lookup_surrogates")
     return out
+
+
+def umim_distill_align_workspace_size(batch, n_spans):
+    return int(lib().umim_distill_align_workspace_size(batch, n_spans))
+
+
+def umim_distill_align(seq_lens, span_offsets, span_start, span_len, capacity, out=None, workspace_buf=None,
+                       dev_status=None, stream=None):
+    """Teacher/student row pairs of Algorithm 1 (App. F).  Returns (or fills,
+    when out is given) a dict of device int32 tensors: pair_offsets [B+1],
+    teacher_rows and student_rows [capacity], student_cu [B+1]."""
+    dev = _dev(seq_lens)
+    B = seq_lens.numel()
+    S = span_start.numel()
+    i32 = lambda n: torch.empty(n, dtype=torch.int32, device=dev)
+    if out is None:
+        out = dict(pair_offsets=i32(B + 1), teacher_rows=i32(max(1, capacity)),
+                   student_rows=i32(max(1, capacity)), student_cu=i32(B + 1))
+    if workspace_buf is None:
+        workspace_buf = workspace(umim_distill_align_workspace_size(B, S), dev)
+    code = lib().umim_distill_align(_p(seq_lens), B, _p(span_offsets), _p(span_start), _p(span_len), S,
+                                    _p(out["pair_offsets"]), _p(out["teacher_rows"]), _p(out["student_rows"]),
+                                    int(capacity), _p(out.get("student_cu")), _p(workspace_buf),
+                                    workspace_buf.numel(), _p(dev_status), _stream(stream))
+    _check(code, "umim_distill_align")
+    return out
+
+
+def umim_distill_soft_ce_workspace_size(n_student_rows, max_pairs):
+    return int(lib().umim_distill_soft_ce_workspace_size(n_student_rows, max_pairs))
+
+
+def umim_distill_soft_ce(teacher_logits, student_logits, teacher_rows, student_rows, n_pairs=None, vocab=None,
+                         eps=1e-8, with_grad=True, loss=None, pair_loss=None, grad=None, workspace_buf=None,
+                         dev_status=None, stream=None):
+    """Soft-target cross-entropy over the aligned pairs and its gradient with
+    respect to the student logits (bf16 [R][ld] rows; vocab defaults to ld).
+    n_pairs: device int32 [1] (pairs used: its value) or None (all of
+    teacher_rows).  Returns (loss [1] fp32, pair_loss [max_pairs] fp32,
+    grad bf16 like student_logits or None)."""
+    dev = _dev(student_logits)
+    R_T, ld = teacher_logits.shape
+    R_S = student_logits.shape[0]
+    if student_logits.shape[1] != ld or teacher_logits.dtype != torch.bfloat16 or \
+            student_logits.dtype != torch.bfloat16:
+        raise ValueError("logits must be bf16 [rows][ld] with the same ld")
+    V = ld if vocab is None else int(vocab)
+    P = teacher_rows.numel()
+    if loss is None:
+        loss = torch.empty(1, dtype=torch.float32, device=dev)
+    if pair_loss is None:
+        pair_loss = torch.empty(max(1, P), dtype=torch.float32, device=dev)
+    if with_grad and grad is None:
+        grad = torch.empty_like(student_logits)
+    if workspace_buf is None:
+        workspace_buf = workspace(umim_distill_soft_ce_workspace_size(R_S, P), dev)
+    code = lib().umim_distill_soft_ce(_p(teacher_logits), R_T, _p(student_logits), R_S, V, ld, _p(teacher_rows),
+                                      _p(student_rows), P, _p(n_pairs), float(eps), _p(loss), _p(pair_loss),
+                                      _p(grad if with_grad else None), _p(workspace_buf), workspace_buf.numel(),
+                                      _p(dev_status), _stream(stream))
+    _check(code, "umim_distill_soft_ce")
+    return loss, pair_loss, (grad if with_grad else None)
 
 
 def trace_start(capacity=4096):

@@ -63,6 +63,12 @@ SIGNATURES = {
     "umim_match_suffix": (ctypes.c_int, [c_ptr, c_size, c_ptr, c_ptr, c_i32, c_ptr, c_ptr, c_ptr, c_ptr, c_ptr,
                                          c_ptr, c_ptr]),
     "umim_lookup_surrogates": (ctypes.c_int, [c_ptr, c_i64, c_i32, c_ptr, c_i32, c_ptr, c_ptr, c_ptr, c_ptr]),
+    "umim_distill_align_workspace_size": (c_size, [c_i32, c_i32]),
+    "umim_distill_align": (ctypes.c_int, [c_ptr, c_i32, c_ptr, c_ptr, c_ptr, c_i32, c_ptr, c_ptr, c_ptr, c_i32,
+                                          c_ptr, c_ptr, c_size, c_ptr, c_ptr]),
+    "umim_distill_soft_ce_workspace_size": (c_size, [c_i32, c_i32]),
+    "umim_distill_soft_ce": (ctypes.c_int, [c_ptr, c_i32, c_ptr, c_i32, c_i32, c_i64, c_ptr, c_ptr, c_i32, c_ptr,
+                                            ctypes.c_float, c_ptr, c_ptr, c_ptr, c_ptr, c_size, c_ptr, c_ptr]),
     "umim_decode_attention_workspace_size": (c_size, [c_i32, c_i32, c_i32, c_i32]),
     "umim_decode_attention": (ctypes.c_int, [c_ptr, c_i32, ctypes.POINTER(PagedKVC), c_i32, c_ptr, c_i32,
                                              c_ptr, c_i32, ctypes.c_float, c_ptr, c_ptr, c_size, c_ptr,

@@ -1,5 +1,6 @@
 // C ABI of libumim: host-side argument checks, then the kernels of each part.
 #include <algorithm>
+#include <cmath>
 #include <cstring>
 #include <mutex>
 
@@ -57,6 +58,14 @@ umim_status selftest_bounded_wait(int, uint32_t, const int32_t *, uint64_t *, in
 size_t prefill_attention_workspace_bytes(int B);
 umim_status prefill_attention(const void *, const void *, const void *, int, int, int, int, const int32_t *, int,
                               float, void *, void *, int32_t *, cudaStream_t);
+size_t distill_align_workspace_bytes(int B, int S);
+umim_status distill_align(const int32_t *, int32_t, const int32_t *, const int32_t *, const int32_t *, int32_t,
+                          int32_t *, int32_t *, int32_t *, int32_t, int32_t *, void *, int32_t *, cudaStream_t);
+size_t distill_soft_ce_workspace_bytes(int R_S, int max_pairs);
+int distill_soft_ce_vecs(int64_t V);
+umim_status distill_soft_ce(const void *, int32_t, const void *, int32_t, int32_t, int64_t, const int32_t *,
+                            const int32_t *, int32_t, const int32_t *, float, float *, float *, void *, void *,
+                            int32_t *, cudaStream_t, int);
 size_t decode_attention_workspace_bytes(int B, int Hq, int Hkv, int D, int num_sms);
 umim_status decode_attention(const void *, int, const umim_paged_kv *, int, const int32_t *, int, const int32_t *,
                              int, float, void *, void *, int32_t *, cudaStream_t, int);
@@ -379,6 +388,58 @@ umim_status umim_prefill_attention(const void *q, const void *k, const void *v, 
   prepare_device(stream);
   return prefill_attention(q, k, v, n_rows, n_q_heads, n_kv_heads, head_dim, cu_seqlens, batch, scale, out,
                            workspace, dev_status, stream);
+}
+
+size_t umim_distill_align_workspace_size(int32_t batch, int32_t n_spans) {
+  if (batch < 0 || n_spans < 0) return 0;
+  return distill_align_workspace_bytes(batch, n_spans);
+}
+
+umim_status umim_distill_align(const int32_t *seq_lens, int32_t batch, const int32_t *span_offsets,
+                               const int32_t *span_start, const int32_t *span_len, int32_t n_spans,
+                               int32_t *pair_offsets, int32_t *teacher_rows, int32_t *student_rows,
+                               int32_t capacity, int32_t *student_cu, void *workspace, size_t workspace_bytes,
+                               int32_t *dev_status, cudaStream_t stream) {
+  if (batch < 0 || n_spans < 0 || capacity < 0 || !pair_offsets) return UMIM_ERR_INVALID_ARG;
+  prepare_device(stream);
+  if (batch == 0) {
+    if (cudaMemsetAsync(pair_offsets, 0, sizeof(int32_t), stream) != cudaSuccess) return UMIM_ERR_CUDA;
+    if (student_cu && cudaMemsetAsync(student_cu, 0, sizeof(int32_t), stream) != cudaSuccess) return UMIM_ERR_CUDA;
+    return UMIM_OK;
+  }
+  if (!seq_lens || !span_offsets || (n_spans > 0 && (!span_start || !span_len))) return UMIM_ERR_INVALID_ARG;
+  if (capacity > 0 && (!teacher_rows || !student_rows)) return UMIM_ERR_INVALID_ARG;
+  if (!workspace || !aligned(workspace, 256) || workspace_bytes < distill_align_workspace_bytes(batch, n_spans))
+    return UMIM_ERR_WORKSPACE;
+  return distill_align(seq_lens, batch, span_offsets, span_start, span_len, n_spans, pair_offsets, teacher_rows,
+                       student_rows, capacity, student_cu, workspace, dev_status, stream);
+}
+
+size_t umim_distill_soft_ce_workspace_size(int32_t n_student_rows, int32_t max_pairs) {
+  if (n_student_rows < 0 || max_pairs < 0) return 0;
+  return distill_soft_ce_workspace_bytes(n_student_rows, max_pairs);
+}
+
+umim_status umim_distill_soft_ce(const void *teacher_logits, int32_t n_teacher_rows, const void *student_logits,
+                                 int32_t n_student_rows, int32_t vocab, int64_t ld, const int32_t *teacher_rows,
+                                 const int32_t *student_rows, int32_t max_pairs, const int32_t *n_pairs, float eps,
+                                 float *loss, float *pair_loss, void *grad, void *workspace,
+                                 size_t workspace_bytes, int32_t *dev_status, cudaStream_t stream) {
+  if (n_teacher_rows < 0 || n_student_rows < 0 || max_pairs < 0 || vocab < 1 || !loss) return UMIM_ERR_INVALID_ARG;
+  if (!(eps >= 0.f) || !std::isfinite(eps)) return UMIM_ERR_INVALID_ARG;
+  if (ld % 8 != 0 || ld < ((int64_t)vocab + 7) / 8 * 8) return UMIM_ERR_INVALID_ARG;
+  if (distill_soft_ce_vecs(vocab) == 0) return UMIM_ERR_UNSUPPORTED;
+  if (n_teacher_rows > 0 && (!teacher_logits || !aligned(teacher_logits, 16))) return UMIM_ERR_INVALID_ARG;
+  if (n_student_rows > 0 && (!student_logits || !aligned(student_logits, 16))) return UMIM_ERR_INVALID_ARG;
+  if (grad && !aligned(grad, 16)) return UMIM_ERR_INVALID_ARG;
+  if (max_pairs > 0 && (!teacher_rows || !student_rows)) return UMIM_ERR_INVALID_ARG;
+  if (!workspace || !aligned(workspace, 256) ||
+      workspace_bytes < distill_soft_ce_workspace_bytes(n_student_rows, max_pairs))
+    return UMIM_ERR_WORKSPACE;
+  const int sms = prepare_device(stream);
+  return distill_soft_ce(teacher_logits, n_teacher_rows, student_logits, n_student_rows, vocab, ld, teacher_rows,
+                         student_rows, max_pairs, n_pairs, eps, loss, pair_loss, grad, workspace, dev_status,
+                         stream, sms);
 }
 
 size_t umim_decode_attention_workspace_size(int32_t batch, int32_t n_q_heads, int32_t n_kv_heads,

@@ -77,3 +77,28 @@ def test_host_checks_reject_bad_arguments_without_touching_the_gpu(lib):
     kv = PagedKVC(4096, 1, 1, 1, 16, 128)
     assert lib.umim_kv_rollback(ctypes.byref(kv), null, 1, null, 0, null, null, null, 0, null, null, null,
                                 null, 0, null, null) == 0
+
+
+def test_distillation_host_checks(lib):
+    null = ctypes.c_void_p(0)
+    fake = ctypes.c_void_p(1 << 20)      # never dereferenced: every call below fails its host checks
+    loss = ctypes.c_void_p(1 << 21)
+    assert lib.umim_distill_soft_ce_workspace_size(3000, 3000) > 3000 * 8
+    assert lib.umim_distill_align_workspace_size(8, 1000) > 0
+    ce = lambda V, ld, eps=1e-8, ws=null, grad=null, lo=loss: lib.umim_distill_soft_ce(
+        fake, 4, fake, 4, V, ld, fake, fake, 4, null, eps, lo, null, grad, ws, 1 << 20, null, null)
+    assert ce(163841, 163848) == 2               # vocabulary above the supported maximum
+    assert ce(1000, 1001) == 1                   # row stride not a multiple of 8
+    assert ce(1001, 1000) == 1                   # stride shorter than the vocabulary
+    assert ce(1000, 1000, eps=-1.0) == 1         # negative eps
+    assert ce(1000, 1000, eps=float("inf")) == 1
+    assert ce(1000, 1000, lo=null) == 1          # no loss output
+    assert ce(1000, 1000, grad=ctypes.c_void_p((1 << 20) + 2)) == 1   # misaligned gradient
+    assert ce(1000, 1000) == 5                   # no workspace
+    assert ce(1000, 1000, ws=ctypes.c_void_p((1 << 20) + 16)) == 5    # misaligned workspace
+    assert lib.umim_distill_align(null, -1, null, null, null, 0, fake, null, null, 0, null, null, 0, null,
+                                  null) == 1
+    assert lib.umim_distill_align(fake, 2, fake, null, null, 3, fake, fake, fake, 10, null, fake, 1 << 20, null,
+                                  null) == 1     # spans but no span arrays
+    assert lib.umim_distill_align(fake, 2, fake, fake, fake, 3, fake, fake, fake, 10, null, null, 0, null,
+                                  null) == 5     # no workspace

@@ -40,6 +40,7 @@ SEEDS = {
     "long_context_tr40": 0x5EED0014,
     "serving": 0x5EED0005,
     "rule_matching": 0x5EED0006,
+    "distillation": 0x5EED0007,
 }
 
 # Retained merge rules per n-gram length for the Llama-3 tokenizer (the paper's
@@ -540,3 +541,42 @@ def serving_loop(seed: int, *, B: int, n_layers: int, n_q_heads: int, n_kv_heads
     return ServingLoop(seed=seed, n_layers=n_layers, n_q_heads=n_q_heads, n_kv_heads=n_kv_heads,
                        head_dim=head_dim, steps=steps, p=p, kmin=kmin, kmax=kmax, lens=lens.astype(np.int32),
                        block_table=bt, n_pages=n_pages, free_pages=[int(x) for x in perm[k:]])
+
+
+# ----------------------------------------------------------------------------
+# aligned predictive distillation (training side)
+# ----------------------------------------------------------------------------
+@dataclasses.dataclass
+class DistillCase:
+    seq_lens: torch.Tensor        # [B] int32 original lengths
+    span_offsets: torch.Tensor    # [B+1]
+    span_start: torch.Tensor      # [S] position within its sample
+    span_len: torch.Tensor        # [S]
+    teacher_logits: torch.Tensor  # [sum L][ld] bf16: the backbone's logits on the original sequences
+
+
+def distill_case(seed: int, *, lens: Sequence[int], vocab: int, coverage: float = 0.4, kmin: int = 2,
+                 kmax: int = 4, ld: Optional[int] = None, std: float = 2.0, device="cpu") -> DistillCase:
+    """Samples of the given lengths with seeded spans (as span_layout) and
+    N(0, std^2) teacher logits over the vocabulary, rows of stride ld
+    (default: vocab rounded up to a multiple of 8).  The student logits are a
+    separate draw (distill_logits) once the caller knows how many compressed
+    rows there are."""
+    r = rng(seed)
+    starts, slens, offs = [], [], [0]
+    for L in lens:
+        st, ln = span_layout(r, int(L), coverage=coverage, kmin=kmin, kmax=kmax)
+        starts.append(st)
+        slens.append(ln)
+        offs.append(offs[-1] + len(st))
+    ld = ((vocab + 7) // 8) * 8 if ld is None else ld
+    t = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(device)
+    cat = lambda xs: np.concatenate(xs).astype(np.int32) if xs else np.zeros(0, np.int32)
+    return DistillCase(seq_lens=t(np.asarray(lens, np.int32)), span_offsets=t(np.asarray(offs, np.int32)),
+                       span_start=t(cat(starts)), span_len=t(cat(slens)),
+                       teacher_logits=distill_logits(seed + 1, int(sum(lens)), ld, std, device))
+
+
+def distill_logits(seed: int, rows: int, ld: int, std: float = 2.0, device="cpu") -> torch.Tensor:
+    """[rows][ld] bf16 logits, N(0, std^2)."""
+    return bf16_normal((rows, ld), std, seed, device)
