@@ -26,6 +26,8 @@
 //    in pair order, by the last CTA to finish.
 #include <algorithm>
 #include <cmath>
+#include <cstdio>
+#include <cstdlib>
 #include <mutex>
 
 #include "common.cuh"
@@ -258,12 +260,10 @@ __global__ void __launch_bounds__(256) align_rows_kernel(AlignArgs a, AlignArray
 // ===========================================================================
 // soft-target cross-entropy
 // ===========================================================================
-constexpr int kCeCluster = 8;     // CTAs per student row (portable cluster size)
-constexpr int kCeThreads = 512;
-constexpr int kCeWarps = kCeThreads / 32;
-constexpr int kCeMaxVecs = 5;     // 16-byte vectors per thread per row
+constexpr int kCeMaxCluster = 16;  // CTAs per student row, at most (16 is a non-portable cluster size)
+constexpr int kCeMaxVecs = 5;      // 16-byte vectors per thread per row
 constexpr int kCeMaxStages = 3;
-constexpr size_t kCeSmemLimit = 227 * 1024 - 2048;   // dynamic shared memory: room left for the static part
+constexpr size_t kCeSmemLimit = 200 * 1024;   // dynamic shared memory per SM: room left for the static part
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 
@@ -339,18 +339,6 @@ __device__ __forceinline__ uint32_t cluster_count() {
 __device__ __forceinline__ void cluster_sync_all() {
   asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
-// float4 at the same shared-memory offset in CTA `rank` of this cluster
-__device__ __forceinline__ float4 ld_peer_f4(const float4 *local, uint32_t rank) {
-  uint32_t ra;
-  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(ra) : "r"(smem_u32(local)), "r"(rank));
-  float4 v;
-  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
-               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
-               : "r"(ra)
-               : "memory");
-  return v;
-}
-
 __device__ __forceinline__ void bulk_load(void *dst, const void *src, uint32_t bytes, uint64_t *bar,
                                           uint64_t policy) {
   asm volatile(
@@ -360,20 +348,58 @@ __device__ __forceinline__ void bulk_load(void *dst, const void *src, uint32_t b
       : "memory");
 }
 
-// (max, sum of exp2(x - max)) of two sets merged; an empty set is (-inf, 0)
-__device__ __forceinline__ void lse_merge(float &m, float &z, float m2, float z2) {
-  const float M = fmaxf(m, m2);
-  if (M == -INFINITY) return;
-  z = z * exp2f(m - M) + z2 * exp2f(m2 - M);
+__device__ __forceinline__ uint32_t cluster_size() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(r));
+  return r;
+}
+
+// The hardware's approximate base-2 exponential, logarithm and reciprocal
+// (PTX ex2/lg2/rcp.approx.ftz: relative errors of about 2^-22; subnormal
+// results flush to zero).
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+__device__ __forceinline__ float lg2_approx(float x) {
+  float y;
+  asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+__device__ __forceinline__ float rcp_approx(float x) {
+  float y;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// Softmax statistics over a warp: from each lane's (m, z) with
+// z = sum exp(x - m) over its values (m = -inf: no values), every lane gets
+// the warp's max and its sum exp(x - max).  The max first, then one rescale
+// per lane, then a plain sum: xor butterflies give every lane the same bits.
+__device__ __forceinline__ void warp_lse(float &m, float &z) {
+  float M = m;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+  float w = (m == -INFINITY) ? 0.f : z * ex2_approx((m - M) * kLog2e);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) w += __shfl_xor_sync(0xffffffffu, w, o);
   m = M;
+  z = w;
+}
+
+__device__ __forceinline__ float warp_sum(float x) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+  return x;
 }
 
 __device__ __forceinline__ void unpack8(const uint4 u, float *f) {
   const uint32_t w[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
   for (int j = 0; j < 4; ++j) {
-    f[2 * j] = __uint_as_float(w[j] << 16) * kLog2e;
-    f[2 * j + 1] = __uint_as_float(w[j] & 0xffff0000u) * kLog2e;
+    f[2 * j] = __uint_as_float(w[j] << 16);
+    f[2 * j + 1] = __uint_as_float(w[j] & 0xffff0000u);
   }
 }
 
@@ -399,17 +425,39 @@ __device__ __forceinline__ void store8(uint16_t *row, int64_t e, int V, const fl
   }
 }
 
-template <int KV>
-__global__ void __launch_bounds__(kCeThreads, 1) ce_kernel(CeArgs a) {
+// The exchange between the CTAs of a row's cluster: every warp pushes its
+// partial (a float4) into slot [rank][warp] of buffer (kind, b) in every CTA
+// of the cluster with st.async, which counts its bytes on that CTA's mbarrier
+// (kind, b); a CTA's warps wait on their own mbarrier and then read all C x NW
+// partials locally.  No fence and no CTA- or cluster-wide barrier is needed
+// per row.  Buffers alternate with the row's parity; each mbarrier phase is
+// armed (arrive + expected bytes) by thread 0 one row ahead, right after the
+// previous phase of that buffer completed, so its byte count never runs
+// negative.
+__device__ __forceinline__ uint32_t peer_addr(const void *local, uint32_t rank) {
+  uint32_t ra;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(ra) : "r"(smem_u32(local)), "r"(rank));
+  return ra;
+}
+__device__ __forceinline__ void st_async_f4(uint32_t raddr, float4 v, uint32_t rbar) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.f32 [%0], {%1, %2, %3, %4}, [%5];" ::"r"(
+                   raddr),
+               "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w), "r"(rbar)
+               : "memory");
+}
+
+template <int KV, int T>
+__global__ void __launch_bounds__(T, 512 / T) ce_kernel(CeArgs a) {
+  constexpr int NW = T / 32;
+  constexpr int NX = kCeMaxCluster * NW;   // partial slots per buffer
   extern __shared__ __align__(128) uint8_t ce_smem[];
   __shared__ __align__(8) uint64_t full_bar[kCeMaxStages];
-  __shared__ float4 slot_stats;          // this CTA's (m_T, z_T, m_S, z_S), read by the cluster
-  __shared__ float4 slot_sums;           // this CTA's (sum P^T log2 q, sum a, -, -)
-  __shared__ float4 warp_part[kCeWarps];
-  __shared__ float4 bcast;
+  __shared__ __align__(8) uint64_t xbar[2][2];        // [stats | sums][row parity]
+  __shared__ __align__(16) float4 xbuf[2][2][NX];     // [stats | sums][row parity][rank * NW + warp]
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const uint32_t rank = cluster_ctarank();
+  const int C = (int)cluster_size();
   const int cid = (int)cluster_idx(), ncl = (int)cluster_count();
   const int nvec = (a.V + 7) >> 3;
   const int vbeg = (int)rank * a.chunk_vecs;
@@ -417,15 +465,21 @@ __global__ void __launch_bounds__(kCeThreads, 1) ce_kernel(CeArgs a) {
   const int S = a.stages;
   uint4 *stage_base = reinterpret_cast<uint4 *>(ce_smem);   // [S][2][chunk_vecs]
   const uint32_t tx_bytes = 2u * (uint32_t)vcnt * 16u;
+  const uint32_t x_bytes = (uint32_t)(C * NW * 16);
 
+  if (a.hdr->error) return;   // the prep kernel rejected the pairs: write nothing (every CTA alike)
   if (tid == 0) {
     for (int s = 0; s < S; ++s) mbar_init(&full_bar[s], 1);
+    for (int k = 0; k < 2; ++k)
+      for (int b = 0; b < 2; ++b) mbar_init(&xbar[k][b], 1);
     fence_mbar_init();
+    for (int k = 0; k < 2; ++k)
+      for (int b = 0; b < 2; ++b) mbar_arrive_expect_tx(&xbar[k][b], x_bytes);   // rows 0 and 1
   }
-  __syncthreads();
-  if (a.hdr->error) return;   // the prep kernel rejected the pairs: write nothing
+  cluster_sync_all();   // every CTA's mbarriers exist before anyone pushes to them
   const int N = a.hdr->n_pairs;
   const float invN = N > 0 ? 1.0f / (float)N : 0.f;
+  const float eps = a.eps;
 
   // producer state (thread 0): next item to consider, copies issued
   int issue_w = cid, issued = 0;
@@ -456,33 +510,41 @@ __global__ void __launch_bounds__(kCeThreads, 1) ce_kernel(CeArgs a) {
   if (tid == 0)
     for (int s = 0; s < S; ++s) issue_next();
 
+  // wait for phase `parity` of mbarrier m; a wait that gives up marks the CTA failed
+  auto xwait = [&](uint64_t *m, uint32_t parity) {
+    if (!failed && !mbar_wait(m, parity)) {
+      failed = true;
+      set_error(a.status, UMIM_ERR_TIMEOUT);
+    }
+  };
+
   int consumed = 0;
+  int p_next = cid < a.R_S ? a.row_pair[cid] : -1;
   for (int w = cid; w < a.R_S; w += ncl) {
-    const int p = a.row_pair[w];
+    const int p = p_next;
+    if (w + ncl < a.R_S) p_next = a.row_pair[w + ncl];
     uint16_t *grow = a.grad ? a.grad + (int64_t)w * a.ld : nullptr;
     if (p < 0) {   // a student row in no pair: zero gradient
       if (grow) {
         float z[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-        for (int vi = tid; vi < vcnt; vi += kCeThreads) store8(grow, (int64_t)(vbeg + vi) * 8, a.V, z);
+        for (int vi = tid; vi < vcnt; vi += T) store8(grow, (int64_t)(vbeg + vi) * 8, a.V, z);
       }
       continue;
     }
-    const int s = consumed % S;
-    const uint32_t parity = (uint32_t)(consumed / S) & 1u;
-    ++consumed;
-    if (!failed && !mbar_wait(&full_bar[s], parity)) {
-      failed = true;
-      set_error(a.status, UMIM_ERR_TIMEOUT);
-    }
+    const int c = consumed++;
+    const int s = c % S;
+    const int xb = c & 1;
+    const uint32_t xpar = (uint32_t)(c >> 1) & 1u;
+    xwait(&full_bar[s], (uint32_t)(c / S) & 1u);
     if (tid == 0 && !failed) pending &= ~(1u << s);
     const uint4 *st = stage_base + (size_t)s * 2 * a.chunk_vecs;
 
-    // ---- pass 1: logits (scaled by log2 e) into registers, local max and sum ----
+    // ---- pass 1: logits into registers, this thread's max, then exp(x - max) and its sum ----
     float xt[KV * 8], xs[KV * 8];
     float mt = -INFINITY, ms = -INFINITY;
 #pragma unroll
     for (int k = 0; k < KV; ++k) {
-      const int vi = tid + k * kCeThreads;
+      const int vi = tid + k * T;
       if (vi < vcnt) {
         unpack8(st[vi], xt + 8 * k);
         unpack8(st[a.chunk_vecs + vi], xs + 8 * k);
@@ -508,127 +570,97 @@ __global__ void __launch_bounds__(kCeThreads, 1) ce_kernel(CeArgs a) {
         ms = fmaxf(ms, xs[8 * k + j]);
       }
     }
-    __syncthreads();   // stage s is in registers: it may be refilled
-    if (tid == 0 && !failed) issue_next();
+    const float bt = (mt == -INFINITY) ? 0.f : -mt * kLog2e;
+    const float bs = (ms == -INFINITY) ? 0.f : -ms * kLog2e;
     float zt = 0.f, zs = 0.f;
 #pragma unroll
     for (int i = 0; i < KV * 8; ++i) {
-      xt[i] = (mt == -INFINITY) ? 0.f : exp2f(xt[i] - mt);
-      xs[i] = (ms == -INFINITY) ? 0.f : exp2f(xs[i] - ms);
+      xt[i] = ex2_approx(fmaf(xt[i], kLog2e, bt));   // -inf -> 0
+      xs[i] = ex2_approx(fmaf(xs[i], kLog2e, bs));
       zt += xt[i];
       zs += xs[i];
     }
-    // ---- softmax statistics over the cluster ----
+    // ---- softmax statistics of the whole row ----
     {
       float m1 = mt, z1 = zt, m2 = ms, z2 = zs;
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        lse_merge(m1, z1, __shfl_xor_sync(0xffffffffu, m1, o), __shfl_xor_sync(0xffffffffu, z1, o));
-        lse_merge(m2, z2, __shfl_xor_sync(0xffffffffu, m2, o), __shfl_xor_sync(0xffffffffu, z2, o));
-      }
-      if (lane == 0) warp_part[warp] = make_float4(m1, z1, m2, z2);
-      __syncthreads();
-      if (warp == 0) {
-        float4 v = lane < kCeWarps ? warp_part[lane] : make_float4(-INFINITY, 0.f, -INFINITY, 0.f);
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-          lse_merge(v.x, v.y, __shfl_xor_sync(0xffffffffu, v.x, o), __shfl_xor_sync(0xffffffffu, v.y, o));
-          lse_merge(v.z, v.w, __shfl_xor_sync(0xffffffffu, v.z, o), __shfl_xor_sync(0xffffffffu, v.w, o));
-        }
-        if (lane == 0) slot_stats = v;
-      }
-      cluster_sync_all();
-      if (tid == 0) {
-        float4 r[kCeCluster];
-#pragma unroll
-        for (int c = 0; c < kCeCluster; ++c) r[c] = ld_peer_f4(&slot_stats, (uint32_t)c);
-        float4 g = r[0];
-#pragma unroll
-        for (int c = 1; c < kCeCluster; ++c) {
-          lse_merge(g.x, g.y, r[c].x, r[c].y);
-          lse_merge(g.z, g.w, r[c].z, r[c].w);
-        }
-        bcast = g;
-      }
-      __syncthreads();
+      warp_lse(m1, z1);
+      warp_lse(m2, z2);
+      if (lane < C)
+        st_async_f4(peer_addr(&xbuf[0][xb][rank * NW + warp], (uint32_t)lane), make_float4(m1, z1, m2, z2),
+                    peer_addr(&xbar[0][xb], (uint32_t)lane));
     }
-    const float4 gs = bcast;
-    // P(v) = exp2(x - m_local) * exp2(m_local - M) / Z
-    const float ct = (mt == -INFINITY) ? 0.f : exp2f(mt - gs.x) / gs.y;
-    const float cs = (ms == -INFINITY) ? 0.f : exp2f(ms - gs.z) / gs.w;
+    xwait(&xbar[0][xb], xpar);
+    if (tid == 0) {
+      if (!failed) mbar_arrive_expect_tx(&xbar[0][xb], x_bytes);   // row c + 2
+      if (!failed) issue_next();                                     // every warp is past stage s
+    }
+    float4 g = make_float4(-INFINITY, 0.f, -INFINITY, 0.f);
+    for (int j = lane; j < C * NW; j += 32) {
+      const float4 v = xbuf[0][xb][j];
+      const float Mt = fmaxf(g.x, v.x), Ms = fmaxf(g.z, v.z);
+      g.y = (Mt == -INFINITY) ? 0.f : g.y * ex2_approx((g.x - Mt) * kLog2e) + v.y * ex2_approx((v.x - Mt) * kLog2e);
+      g.w = (Ms == -INFINITY) ? 0.f : g.w * ex2_approx((g.z - Ms) * kLog2e) + v.w * ex2_approx((v.z - Ms) * kLog2e);
+      g.x = Mt;
+      g.z = Ms;
+    }
+    warp_lse(g.x, g.y);
+    warp_lse(g.z, g.w);
+    // P(v) = exp(x - m_thread) * exp(m_thread - M) / Z
+    const float ct = (mt == -INFINITY) ? 0.f : ex2_approx((mt - g.x) * kLog2e) / g.y;
+    const float cs = (ms == -INFINITY) ? 0.f : ex2_approx((ms - g.z) * kLog2e) / g.w;
 
     // ---- pass 2: P^T, P^S, the loss terms and a ----
     float lsum = 0.f, asum = 0.f;
 #pragma unroll
     for (int i = 0; i < KV * 8; ++i) {
       const float pt = xt[i] * ct, ps = xs[i] * cs;
-      const float q = ps + a.eps;
-      const float r = q > 0.f ? __fdividef(ps, q) : 0.f;
-      lsum += pt > 0.f ? pt * __log2f(q) : 0.f;
-      const float av = pt * r;
+      const float q = fmaxf(ps + eps, 1.17549435e-38f);   // log2 stays finite when eps = 0
+      lsum = fmaf(pt, lg2_approx(q), lsum);
+      const float av = pt * (ps * rcp_approx(q));
       asum += av;
       xt[i] = av;
       xs[i] = ps;
     }
-    {
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        lsum += __shfl_xor_sync(0xffffffffu, lsum, o);
-        asum += __shfl_xor_sync(0xffffffffu, asum, o);
-      }
-      if (lane == 0) warp_part[warp] = make_float4(lsum, asum, 0.f, 0.f);
-      __syncthreads();
-      if (warp == 0) {
-        float4 v = lane < kCeWarps ? warp_part[lane] : make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-          v.x += __shfl_xor_sync(0xffffffffu, v.x, o);
-          v.y += __shfl_xor_sync(0xffffffffu, v.y, o);
-        }
-        if (lane == 0) slot_sums = v;
-      }
-      cluster_sync_all();
-      if (tid == 0) {
-        float4 r[kCeCluster];
-#pragma unroll
-        for (int c = 0; c < kCeCluster; ++c) r[c] = ld_peer_f4(&slot_sums, (uint32_t)c);
-        float l = 0.f, A = 0.f;
-#pragma unroll
-        for (int c = 0; c < kCeCluster; ++c) {
-          l += r[c].x;
-          A += r[c].y;
-        }
-        bcast = make_float4(l, A, 0.f, 0.f);
-        if (rank == 0) a.pair_loss[p] = -l * kLn2;
-      }
-      __syncthreads();
+    lsum = warp_sum(lsum);
+    asum = warp_sum(asum);
+    if (lane < C)
+      st_async_f4(peer_addr(&xbuf[1][xb][rank * NW + warp], (uint32_t)lane), make_float4(lsum, asum, 0.f, 0.f),
+                  peer_addr(&xbar[1][xb], (uint32_t)lane));
+    xwait(&xbar[1][xb], xpar);
+    if (tid == 0 && !failed) mbar_arrive_expect_tx(&xbar[1][xb], x_bytes);   // row c + 2
+    float Lp = 0.f, A = 0.f;
+    for (int j = lane; j < C * NW; j += 32) {
+      const float4 v = xbuf[1][xb][j];
+      Lp += v.x;
+      A += v.y;
     }
-    const float A = bcast.y;
+    Lp = warp_sum(Lp);
+    A = warp_sum(A);
+    if (rank == 0 && tid == 0) a.pair_loss[p] = -Lp * kLn2;
 
     // ---- pass 3: gradient -(1/N) (a_v - P^S(v) A) ----
     if (grow) {
 #pragma unroll
       for (int k = 0; k < KV; ++k) {
-        const int vi = tid + k * kCeThreads;
+        const int vi = tid + k * T;
         if (vi < vcnt) {
-          float g[8];
+          float gr[8];
 #pragma unroll
-          for (int j = 0; j < 8; ++j) g[j] = (xs[8 * k + j] * A - xt[8 * k + j]) * invN;
-          store8(grow, (int64_t)(vbeg + vi) * 8, a.V, g);
+          for (int j = 0; j < 8; ++j) gr[j] = (xs[8 * k + j] * A - xt[8 * k + j]) * invN;
+          store8(grow, (int64_t)(vbeg + vi) * 8, a.V, gr);
         }
       }
     }
   }
 
-  // no CTA leaves while a peer may still read its shared memory
+  // no CTA leaves while a peer may still push to or read its shared memory
   cluster_sync_all();
 
   // a copy whose wait gave up may still be in flight: wait for it, bounded
   if (tid == 0 && failed) {
     for (int s = 0; s < S; ++s)
       if (pending & (1u << s)) {
-        // the outstanding phase of stage s is the last one issued there
-        const int last = ((issued - 1 - s) / S) * S + s;
+        const int last = ((issued - 1 - s) / S) * S + s;   // the last copy issued to stage s
         if (last >= 0) mbar_wait_for(&full_bar[s], (uint32_t)(last / S) & 1u, kWaitLimitNs);
       }
   }
@@ -643,8 +675,8 @@ __global__ void __launch_bounds__(kCeThreads, 1) ce_kernel(CeArgs a) {
   __syncthreads();
   if (!s_last) return;
   __threadfence();
-  __shared__ double dpart[kCeWarps];
-  const int per = (N + kCeThreads - 1) / kCeThreads;
+  __shared__ double dpart[NW];
+  const int per = (N + T - 1) / T;
   double acc = 0.0;
   for (int i = 0; i < per; ++i) {
     const int q = tid * per + i;
@@ -656,63 +688,118 @@ __global__ void __launch_bounds__(kCeThreads, 1) ce_kernel(CeArgs a) {
   __syncthreads();
   if (tid == 0) {
     double t = 0.0;
-    for (int w2 = 0; w2 < kCeWarps; ++w2) t += dpart[w2];
+    for (int w2 = 0; w2 < NW; ++w2) t += dpart[w2];
     a.loss[0] = N > 0 ? (float)(t / (double)N) : 0.f;
   }
 }
 
-template <int KV>
-struct CeLaunch {
-  static void *fn() { return reinterpret_cast<void *>(ce_kernel<KV>); }
-};
+using CeKernel = void (*)(CeArgs);
 
-void *ce_kernel_ptr(int kv) {
-  switch (kv) {
-    case 1: return CeLaunch<1>::fn();
-    case 2: return CeLaunch<2>::fn();
-    case 3: return CeLaunch<3>::fn();
-    case 4: return CeLaunch<4>::fn();
-    default: return CeLaunch<5>::fn();
-  }
+CeKernel ce_kernel_for(int kv, int T) {
+  static const CeKernel k256[kCeMaxVecs] = {ce_kernel<1, 256>, ce_kernel<2, 256>, ce_kernel<3, 256>,
+                                            ce_kernel<4, 256>, ce_kernel<5, 256>};
+  static const CeKernel k512[kCeMaxVecs] = {ce_kernel<1, 512>, ce_kernel<2, 512>, ce_kernel<3, 512>,
+                                            ce_kernel<4, 512>, ce_kernel<5, 512>};
+  return (T == 256 ? k256 : k512)[kv - 1];
 }
 
-// Clusters of the main kernel that can be resident at once (cached per
-// device, vectors per thread and shared-memory size).
-int ce_max_clusters(int kv, size_t smem, int num_sms) {
+// 16-byte vectors per thread per row with T threads per CTA and C CTAs per row
+int ce_vecs(int64_t V, int T, int C) {
+  const int64_t nvec = (V + 7) / 8;
+  const int64_t chunk = (nvec + C - 1) / C;
+  return (int)std::max<int64_t>(1, (chunk + T - 1) / T);
+}
+
+// How a call runs: T threads per CTA, C CTAs (one cluster) per student row.
+struct CeLayout {
+  int T, C, kv, chunk_vecs, stages;
+  size_t smem;
+  int resident;   // clusters that can be resident at once
+};
+
+// Clusters of a layout that can be resident at once (0: it cannot launch);
+// cached per device and layout.
+int ce_resident_clusters(int kv, int T, int C, size_t smem, int num_sms) {
   struct Entry {
-    int dev, kv;
+    int dev, kv, T, C;
     size_t smem;
     int n;
   };
-  static Entry cache[16];
+  static Entry cache[32];
   static int n_cache = 0;
   static std::mutex mu;
   int dev = 0;
   cudaGetDevice(&dev);
   std::lock_guard<std::mutex> lock(mu);
-  for (int i = 0; i < n_cache; ++i)
-    if (cache[i].dev == dev && cache[i].kv == kv && cache[i].smem == smem) return cache[i].n;
-  void *fn = ce_kernel_ptr(kv);
+  for (int i = 0; i < n_cache; ++i) {
+    const Entry &e = cache[i];
+    if (e.dev == dev && e.kv == kv && e.T == T && e.C == C && e.smem == smem) return e.n;
+  }
+  const CeKernel fn = ce_kernel_for(kv, T);
   // the largest size any call may request, so that no later call finds a smaller limit
   cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kCeSmemLimit);
+  if (C > 8) cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(kCeCluster * std::max(1, num_sms / kCeCluster));
-  cfg.blockDim = dim3(kCeThreads);
+  cfg.gridDim = dim3((unsigned)(C * std::max(1, 2 * num_sms / C)));
+  cfg.blockDim = dim3((unsigned)T);
   cfg.dynamicSmemBytes = smem;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = kCeCluster;
+  attr[0].val.clusterDim.x = (unsigned)C;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   int n = 0;
-  if (cudaOccupancyMaxActiveClusters(&n, fn, &cfg) != cudaSuccess || n <= 0) {
+  if (cudaOccupancyMaxActiveClusters(&n, fn, &cfg) != cudaSuccess) {
     cudaGetLastError();
-    n = std::max(1, num_sms / kCeCluster);
+    n = 0;
   }
-  if (n_cache < 16) cache[n_cache++] = Entry{dev, kv, smem, n};
+  if (n_cache < 32) cache[n_cache++] = Entry{dev, kv, T, C, smem, n};
   return n;
+}
+
+bool ce_try_layout(int64_t V, int T, int C, int num_sms, CeLayout &L) {
+  const int kv = ce_vecs(V, T, C);
+  if (kv > kCeMaxVecs) return false;
+  const int nvec = (int)((V + 7) / 8);
+  L.T = T;
+  L.C = C;
+  L.kv = kv;
+  L.chunk_vecs = (nvec + C - 1) / C;
+  const size_t stage_bytes = (size_t)2 * L.chunk_vecs * 16;
+  // 256-thread CTAs run two to an SM: each keeps to half of the shared memory
+  const size_t limit = T == 256 ? kCeSmemLimit / 2 : kCeSmemLimit;
+  L.stages = (int)std::min<size_t>(kCeMaxStages, limit / stage_bytes);
+  if (L.stages < 2) return false;
+  L.smem = stage_bytes * L.stages;
+  L.resident = ce_resident_clusters(kv, T, C, L.smem, num_sms);
+  return L.resident > 0;
+}
+
+// 256-thread CTAs (two per SM, so one computes while the other waits at a
+// cluster barrier), with the fewest CTAs per row that keep each thread at
+// <= 4 vectors per row (5 at 16 CTAs); 512-thread CTAs in clusters of 8 when
+// that cannot be resident.  UMIM_SOFT_CE_LAYOUT="T,C" picks a layout (for
+// measurements).
+bool ce_layout(int64_t V, int num_sms, CeLayout &L) {
+  static int env_T = -1, env_C = -1;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    const char *e = getenv("UMIM_SOFT_CE_LAYOUT");
+    int t = 0, c = 0;
+    if (e && sscanf(e, "%d,%d", &t, &c) == 2 && (t == 256 || t == 512) && c >= 1 && c <= kCeMaxCluster &&
+        (c & (c - 1)) == 0) {
+      env_T = t;
+      env_C = c;
+    }
+  });
+  if (env_T > 0 && ce_try_layout(V, env_T, env_C, num_sms, L)) return true;
+  for (int C = 1; C <= kCeMaxCluster; C *= 2)
+    if ((ce_vecs(V, 256, C) <= 4 || C == kCeMaxCluster) && ce_try_layout(V, 256, C, num_sms, L)) return true;
+  for (int C = 1; C <= 8; C *= 2)
+    if ((ce_vecs(V, 512, C) <= 4 || C == 8) && ce_try_layout(V, 512, C, num_sms, L)) return true;
+  return false;
 }
 
 }  // namespace
@@ -752,19 +839,16 @@ umim_status distill_align(const int32_t *seq_lens, int32_t B, const int32_t *spa
 size_t distill_soft_ce_workspace_bytes(int R_S, int max_pairs) { return ce_ws_bytes(R_S, max_pairs); }
 
 // vectors per thread per row for a vocabulary (0: unsupported)
-int distill_soft_ce_vecs(int64_t V) {
-  const int64_t nvec = (V + 7) / 8;
-  const int64_t chunk = (nvec + kCeCluster - 1) / kCeCluster;
-  const int64_t kv = (chunk + kCeThreads - 1) / kCeThreads;
-  return (V >= 1 && kv <= kCeMaxVecs) ? (int)std::max<int64_t>(kv, 1) : 0;
-}
+// nonzero when the vocabulary is supported (at most 16 CTAs x 256 threads x 5 vectors x 8 values)
+int distill_soft_ce_vecs(int64_t V) { return (V >= 1 && ce_vecs(V, 256, kCeMaxCluster) <= kCeMaxVecs) ? 1 : 0; }
 
 umim_status distill_soft_ce(const void *teacher, int32_t R_T, const void *student, int32_t R_S, int32_t V, int64_t ld,
                             const int32_t *teacher_rows, const int32_t *student_rows, int32_t max_pairs,
                             const int32_t *n_dev, float eps, float *loss, float *pair_loss, void *grad, void *ws,
                             int32_t *dev_status, cudaStream_t stream, int num_sms) {
-  const int kv = distill_soft_ce_vecs(V);
-  if (kv == 0) return UMIM_ERR_UNSUPPORTED;
+  if (!distill_soft_ce_vecs(V)) return UMIM_ERR_UNSUPPORTED;
+  CeLayout lay;
+  if (!ce_layout(V, num_sms, lay)) return UMIM_ERR_UNSUPPORTED;
   char *p = static_cast<char *>(ws);
   CeHeader *hdr = reinterpret_cast<CeHeader *>(p);
   p += a256(sizeof(CeHeader));
@@ -790,12 +874,8 @@ umim_status distill_soft_ce(const void *teacher, int32_t R_T, const void *studen
   a.row_pair = row_pair;
   a.hdr = hdr;
   a.status = dev_status ? dev_status : &hdr->status;
-  const int nvec = (V + 7) / 8;
-  a.chunk_vecs = (nvec + kCeCluster - 1) / kCeCluster;
-  const size_t stage_bytes = (size_t)2 * a.chunk_vecs * 16;
-  a.stages = (int)std::min<size_t>(kCeMaxStages, kCeSmemLimit / stage_bytes);
-  if (a.stages < 2) return UMIM_ERR_UNSUPPORTED;
-  const size_t smem = stage_bytes * a.stages;
+  a.chunk_vecs = lay.chunk_vecs;
+  a.stages = lay.stages;
 
   if (cudaMemsetAsync(hdr, 0, sizeof(CeHeader), stream) != cudaSuccess) return UMIM_ERR_CUDA;
   if (R_S > 0 && cudaMemsetAsync(row_pair, 0xFF, sizeof(int32_t) * (size_t)R_S, stream) != cudaSuccess)
@@ -805,29 +885,21 @@ umim_status distill_soft_ce(const void *teacher, int32_t R_T, const void *studen
   ce_prep_kernel<<<prep_blocks, 256, 0, stream>>>(a);
   if (cudaGetLastError() != cudaSuccess) return UMIM_ERR_CUDA;
 
-  const int max_cl = ce_max_clusters(kv, smem, num_sms);
-  const int n_cl = std::max(1, std::min(R_S, max_cl));
+  const int n_cl = std::max(1, std::min(R_S, lay.resident));
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((unsigned)(n_cl * kCeCluster));
-  cfg.blockDim = dim3(kCeThreads);
-  cfg.dynamicSmemBytes = smem;
+  cfg.gridDim = dim3((unsigned)(n_cl * lay.C));
+  cfg.blockDim = dim3((unsigned)lay.T);
+  cfg.dynamicSmemBytes = lay.smem;
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = kCeCluster;
+  attr[0].val.clusterDim.x = (unsigned)lay.C;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   trace_mark(stream, "distill.soft_ce");
-  cudaError_t e;
-  switch (kv) {
-    case 1: e = cudaLaunchKernelEx(&cfg, ce_kernel<1>, a); break;
-    case 2: e = cudaLaunchKernelEx(&cfg, ce_kernel<2>, a); break;
-    case 3: e = cudaLaunchKernelEx(&cfg, ce_kernel<3>, a); break;
-    case 4: e = cudaLaunchKernelEx(&cfg, ce_kernel<4>, a); break;
-    default: e = cudaLaunchKernelEx(&cfg, ce_kernel<5>, a); break;
-  }
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, ce_kernel_for(lay.kv, lay.T), a);
   trace_mark(stream, nullptr);
   return e == cudaSuccess ? UMIM_OK : UMIM_ERR_CUDA;
 }
