@@ -1163,9 +1163,20 @@ def side_bench(args):
     kernels = kernel_table(recs, K, work_of)
     if args.workload == "prefill":
         cfg["speedup_from_compression"] = round(cfg["uncompressed_ms"] / (ms / K), 3)
+    # the dominant kernel against its bound
+    roof = None
+    measured = [k for k in kernels if k in work_of]
+    if measured:
+        top = max(measured, key=lambda k: kernels[k]["share"])
+        b, amount, unit_r, peak = work_of[top]
+        roof = {"kernel": top, "bound": b, "achieved": kernels[top]["achieved"], "peak": peak, "unit": unit_r,
+                "frac": kernels[top]["frac"], "traffic": traffic_from_profile(top),
+                "algorithmic_per_launch": amount * (1e12 if unit_r == "TFLOP/s" else 1e9),
+                "peak_source": peaks["src"] + (" bf16 burst" if b == "tensor" else " HBM copy")}
     line = {"metric": metric, "value": units * K / (ms / 1000.0), "unit": unit, "n_gpus": 1, "steps": K,
             "warmup": Wm, "ms_per_step": ms / K, "higher_is_better": True, "dtype": "bf16", "data": "synthetic",
-            "config": cfg, "kernels": kernels, "gpu_launches": len(recs), "clocks": clk.summary(w0, w1),
+            "config": cfg, "roofline": roof, "kernels": kernels, "gpu_launches": len(recs),
+            "clocks": clk.summary(w0, w1),
             "traced_ms_per_step": tms / K, "peaks": {"hbm_gbs": peaks["hbm"], "bf16_tflops": peaks["bf16"],
                                                      "source": peaks["src"]}}
     print(json.dumps(line))
