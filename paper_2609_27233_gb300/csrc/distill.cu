@@ -594,20 +594,30 @@ __global__ void __launch_bounds__(T, 512 / T) ce_kernel(CeArgs a) {
       if (!failed) mbar_arrive_expect_tx(&xbar[0][xb], x_bytes);   // row c + 2
       if (!failed) issue_next();                                     // every warp is past stage s
     }
-    float4 g = make_float4(-INFINITY, 0.f, -INFINITY, 0.f);
+    // the row's max over the C x NW partials, then one rescale per partial
+    float Mt = -INFINITY, Ms = -INFINITY;
     for (int j = lane; j < C * NW; j += 32) {
       const float4 v = xbuf[0][xb][j];
-      const float Mt = fmaxf(g.x, v.x), Ms = fmaxf(g.z, v.z);
-      g.y = (Mt == -INFINITY) ? 0.f : g.y * ex2_approx((g.x - Mt) * kLog2e) + v.y * ex2_approx((v.x - Mt) * kLog2e);
-      g.w = (Ms == -INFINITY) ? 0.f : g.w * ex2_approx((g.z - Ms) * kLog2e) + v.w * ex2_approx((v.z - Ms) * kLog2e);
-      g.x = Mt;
-      g.z = Ms;
+      Mt = fmaxf(Mt, v.x);
+      Ms = fmaxf(Ms, v.z);
     }
-    warp_lse(g.x, g.y);
-    warp_lse(g.z, g.w);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      Mt = fmaxf(Mt, __shfl_xor_sync(0xffffffffu, Mt, o));
+      Ms = fmaxf(Ms, __shfl_xor_sync(0xffffffffu, Ms, o));
+    }
+    const float nMt = (Mt == -INFINITY) ? 0.f : -Mt * kLog2e, nMs = (Ms == -INFINITY) ? 0.f : -Ms * kLog2e;
+    float Zt = 0.f, Zs = 0.f;
+    for (int j = lane; j < C * NW; j += 32) {
+      const float4 v = xbuf[0][xb][j];
+      Zt = fmaf(v.y, ex2_approx(fmaf(v.x, kLog2e, nMt)), Zt);   // empty partials: z = 0
+      Zs = fmaf(v.w, ex2_approx(fmaf(v.z, kLog2e, nMs)), Zs);
+    }
+    Zt = warp_sum(Zt);
+    Zs = warp_sum(Zs);
     // P(v) = exp(x - m_thread) * exp(m_thread - M) / Z
-    const float ct = (mt == -INFINITY) ? 0.f : ex2_approx((mt - g.x) * kLog2e) / g.y;
-    const float cs = (ms == -INFINITY) ? 0.f : ex2_approx((ms - g.z) * kLog2e) / g.w;
+    const float ct = (mt == -INFINITY) ? 0.f : ex2_approx(fmaf(mt, kLog2e, nMt)) * rcp_approx(Zt);
+    const float cs = (ms == -INFINITY) ? 0.f : ex2_approx(fmaf(ms, kLog2e, nMs)) * rcp_approx(Zs);
 
     // ---- pass 2: P^T, P^S, the loss terms and a ----
     float lsum = 0.f, asum = 0.f;
@@ -777,11 +787,13 @@ bool ce_try_layout(int64_t V, int T, int C, int num_sms, CeLayout &L) {
   return L.resident > 0;
 }
 
-// 256-thread CTAs (two per SM, so one computes while the other waits at a
-// cluster barrier), with the fewest CTAs per row that keep each thread at
-// <= 4 vectors per row (5 at 16 CTAs); 512-thread CTAs in clusters of 8 when
-// that cannot be resident.  UMIM_SOFT_CE_LAYOUT="T,C" picks a layout (for
-// measurements).
+// Two candidates: 256-thread CTAs (two per SM, one computing while the other
+// waits for its exchange) and 512-thread CTAs, each with the fewest CTAs per
+// row that keep a thread at <= 4 vectors per row (5 at the largest cluster);
+// the one with more threads resident wins -- cluster placement within a GPC
+// can leave SMs idle (on a GB300 at the Llama-3 vocabulary: 14 clusters of
+// 16 x 256 threads on 112 SMs, 15 clusters of 8 x 512 on 120).
+// UMIM_SOFT_CE_LAYOUT="T,C" picks a layout (for measurements).
 bool ce_layout(int64_t V, int num_sms, CeLayout &L) {
   static int env_T = -1, env_C = -1;
   static std::once_flag once;
@@ -795,11 +807,24 @@ bool ce_layout(int64_t V, int num_sms, CeLayout &L) {
     }
   });
   if (env_T > 0 && ce_try_layout(V, env_T, env_C, num_sms, L)) return true;
-  for (int C = 1; C <= kCeMaxCluster; C *= 2)
-    if ((ce_vecs(V, 256, C) <= 4 || C == kCeMaxCluster) && ce_try_layout(V, 256, C, num_sms, L)) return true;
-  for (int C = 1; C <= 8; C *= 2)
-    if ((ce_vecs(V, 512, C) <= 4 || C == 8) && ce_try_layout(V, 512, C, num_sms, L)) return true;
-  return false;
+  // per thread count, the fewest CTAs per row with <= 4 vectors per thread (5 at the largest cluster)
+  CeLayout best{};
+  bool found = false;
+  for (const int T : {256, 512}) {
+    const int Cmax = T == 256 ? kCeMaxCluster : 8;
+    for (int C = 1; C <= Cmax; C *= 2) {
+      if (ce_vecs(V, T, C) > 4 && C < Cmax) continue;
+      CeLayout cand;
+      if (ce_try_layout(V, T, C, num_sms, cand)) {
+        // more resident threads wins (a cluster size that leaves SMs of a GPC idle loses)
+        if (!found || (int64_t)cand.resident * cand.C * cand.T > (int64_t)best.resident * best.C * best.T) best = cand;
+        found = true;
+      }
+      break;
+    }
+  }
+  if (found) L = best;
+  return found;
 }
 
 }  // namespace
