@@ -989,7 +989,7 @@ def side_bench(args):
         qkv_u = [W.bf16_normal((Tu, h, D), 1.0, seed + 401 + i, dev) for i, h in enumerate((Hq, Hkv, Hkv))]
         qkv_c = [x[:Tc] for x in qkv_u]   # the compressed rows (values do not matter for timing)
         out = torch.empty_like(qkv_u[0])
-        ws_p = umim.workspace(umim.umim_prefill_attention_workspace_size(B), dev)
+        ws_p = umim.workspace(umim.umim_prefill_attention_workspace_size(B, Tu, Hkv, D), dev)
         phase = ["compressed"]
 
         def step(i):
@@ -1025,7 +1025,8 @@ def side_bench(args):
                "compressed_rows": Tc, "uncompressed_rows": Tu, "mean_compressed_length": round(Tc / B, 1),
                "uncompressed_ms": round(unc_ms, 4),
                "uncompressed_tflops": round(causal_flops([L] * B) / unc_ms / 1e9, 1),
-               "kernel": "mma.sync m16n8k16 (P split into bf16 high + remainder), cp.async double buffering",
+               "kernel": "tcgen05.mma (S and O in tensor memory; P from shared memory as bf16 high + remainder), "
+                         "TMA-fed K / V^T ring, V transposed per call",
                "l2": "q/k/v of one layer are 0.96 GB (compressed) / 1.34 GB (uncompressed): larger than L2"}
     elif args.workload == "distill":
         seed = W.SEEDS["distillation"]

@@ -343,12 +343,14 @@ umim_status umim_decode_attention(const void *q, int32_t n_q_heads, const umim_p
  * out          device bf16 [n_rows][n_q_heads][head_dim] (rows outside every
  *              sequence are not written)
  * workspace    device, umim_prefill_attention_workspace_size() bytes, 256-B
- *              aligned
+ *              aligned (it holds the tile plan and a transposed copy of v,
+ *              each sequence padded to 64 keys: about
+ *              n_kv_heads * head_dim * (n_rows + 64 * batch) * 2 bytes)
  * head_dim 64 or 128; n_q_heads a multiple of n_kv_heads (else
  * UMIM_ERR_UNSUPPORTED).  Device-side errors: UMIM_ERR_INVALID_ARG for
  * offsets that break the rules above (nothing is written).
  * ------------------------------------------------------------------------ */
-size_t umim_prefill_attention_workspace_size(int32_t batch);
+size_t umim_prefill_attention_workspace_size(int32_t batch, int32_t n_rows, int32_t n_kv_heads, int32_t head_dim);
 
 umim_status umim_prefill_attention(const void *q, const void *k, const void *v, int32_t n_rows, int32_t n_q_heads,
                                    int32_t n_kv_heads, int32_t head_dim, const int32_t *cu_seqlens, int32_t batch,

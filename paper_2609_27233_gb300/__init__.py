@@ -113,8 +113,8 @@ def umim_kv_rollback_workspace_size(batch, n_spans, max_pages, n_layers, n_kv_he
     return int(lib().umim_kv_rollback_workspace_size(batch, n_spans, max_pages, n_layers, n_kv_heads, head_dim))
 
 
-def umim_prefill_attention_workspace_size(batch):
-    return int(lib().umim_prefill_attention_workspace_size(batch))
+def umim_prefill_attention_workspace_size(batch, n_rows, n_kv_heads, head_dim):
+    return int(lib().umim_prefill_attention_workspace_size(batch, n_rows, n_kv_heads, head_dim))
 
 
 def umim_decode_attention_workspace_size(batch, n_q_heads, n_kv_heads, head_dim):
@@ -279,7 +279,7 @@ def umim_prefill_attention(q, k, v, cu_seqlens, scale=0.0, out=None, workspace_b
     if out is None:
         out = torch.empty_like(q)
     if workspace_buf is None:
-        workspace_buf = workspace(umim_prefill_attention_workspace_size(B), dev)
+        workspace_buf = workspace(umim_prefill_attention_workspace_size(B, T, Hkv, D), dev)
     code = lib().umim_prefill_attention(_p(q), _p(k), _p(v), T, Hq, Hkv, D, _p(cu_seqlens), B, float(scale), _p(out),
                                         _p(workspace_buf), workspace_buf.numel(), _p(dev_status), _stream(stream))
     _check(code, "umim_prefill_attention")

@@ -55,9 +55,9 @@ umim_status match_suffix(const void *, size_t, void *, const int32_t *, int, int
 umim_status lookup_surrogates(const float *, int64_t, int, const int32_t *, int, const int32_t *, float *, int32_t *,
                               cudaStream_t, int);
 umim_status selftest_bounded_wait(int, uint32_t, const int32_t *, uint64_t *, int32_t *, cudaStream_t);
-size_t prefill_attention_workspace_bytes(int B);
+size_t prefill_attention_workspace_bytes(int B, int T, int Hkv, int D);
 umim_status prefill_attention(const void *, const void *, const void *, int, int, int, int, const int32_t *, int,
-                              float, void *, void *, int32_t *, cudaStream_t);
+                              float, void *, void *, int32_t *, cudaStream_t, int);
 size_t distill_align_workspace_bytes(int B, int S);
 umim_status distill_align(const int32_t *, int32_t, const int32_t *, const int32_t *, const int32_t *, int32_t,
                           int32_t *, int32_t *, int32_t *, int32_t, int32_t *, void *, int32_t *, cudaStream_t);
@@ -368,9 +368,9 @@ umim_status umim_selftest_bounded_wait(int32_t which, uint32_t limit_us, const i
   return selftest_bounded_wait(which, limit_us, flags, elapsed_ns, dev_status, stream);
 }
 
-size_t umim_prefill_attention_workspace_size(int32_t batch) {
-  if (batch < 0) return 0;
-  return prefill_attention_workspace_bytes(batch);
+size_t umim_prefill_attention_workspace_size(int32_t batch, int32_t n_rows, int32_t n_kv_heads, int32_t head_dim) {
+  if (batch < 0 || n_rows < 0 || n_kv_heads <= 0 || (head_dim != 64 && head_dim != 128)) return 0;
+  return prefill_attention_workspace_bytes(batch, n_rows, n_kv_heads, head_dim);
 }
 
 umim_status umim_prefill_attention(const void *q, const void *k, const void *v, int32_t n_rows, int32_t n_q_heads,
@@ -383,11 +383,12 @@ umim_status umim_prefill_attention(const void *q, const void *k, const void *v, 
   if (batch == 0 || n_rows == 0) return UMIM_OK;
   if (!q || !k || !v || !out || !cu_seqlens) return UMIM_ERR_INVALID_ARG;
   if (!aligned(q, 16) || !aligned(k, 16) || !aligned(v, 16) || !aligned(out, 16)) return UMIM_ERR_INVALID_ARG;
-  if (!workspace || !aligned(workspace, 256) || workspace_bytes < prefill_attention_workspace_bytes(batch))
+  if (!workspace || !aligned(workspace, 256) ||
+      workspace_bytes < prefill_attention_workspace_bytes(batch, n_rows, n_kv_heads, head_dim))
     return UMIM_ERR_WORKSPACE;
-  prepare_device(stream);
+  const int sms = prepare_device(stream);
   return prefill_attention(q, k, v, n_rows, n_q_heads, n_kv_heads, head_dim, cu_seqlens, batch, scale, out,
-                           workspace, dev_status, stream);
+                           workspace, dev_status, stream, sms);
 }
 
 size_t umim_distill_align_workspace_size(int32_t batch, int32_t n_spans) {

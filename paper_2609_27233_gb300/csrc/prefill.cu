@@ -4,280 +4,496 @@
 // then runs over the shorter sequences).  Sequence b owns rows
 // cu_seqlens[b] .. cu_seqlens[b+1]-1 of q [T][Hq][D], k, v [T][Hkv][D].
 //
-// Work unit: 64 query rows of one sequence and one query head, one CTA of 4
-// warps (16 rows each).  K and V tiles of 64 keys are staged in shared memory
-// by cp.async (double-buffered; rows past the sequence are zero-filled) in
-// the 128-byte-swizzled layout the decode kernel uses; S = Q K^T and O += P V
-// run as mma.sync m16n8k16 (P split into a bf16 high part and a bf16
-// remainder, as in decode); the softmax is online in fp32 with the causal
-// mask applied on the diagonal tile.  A plan kernel turns cu_seqlens into
-// per-sequence query-tile offsets (and validates them); tiles run heaviest
+// On the 5th-generation tensor cores: one CTA takes 128 query rows of one
+// sequence and one query head.  Warp 0 loads tiles with TMA (Q once; K and
+// V^T tiles of 64 keys into a 3-stage ring), warp 1 issues tcgen05.mma
+// (S = Q K^T into one of two tensor-memory buffers, then O += P V into a
+// tensor-memory accumulator), warps 2-5 run the online softmax, one thread
+// per query row: S from tensor memory (tcgen05.ld), causal mask, running max,
+// P = exp2(S - max) written to shared memory as a bf16 high part and a bf16
+// remainder (two MMAs per P V product keep P's rounding out of the error
+// budget), row sums.  The running max is only moved when it grows by more
+// than 2^8, so the accumulator in tensor memory is rescaled rarely (the
+// result is the same: P and the row sum use the same stale max).  The S MMA
+// of the next tile runs while the softmax works on the current one.
+//
+// V is transposed first (per sequence, padded to a multiple of 64 keys) so
+// that both products read K-major operands and every TMA copy starts on a
+// 16-byte boundary.  A plan kernel turns cu_seqlens into per-sequence tile
+// offsets and padded key offsets (and validates them); tiles run heaviest
 // (last in their sequence) first.
 #include "common.cuh"
-#include "mma.cuh"
 
 namespace umim {
+
+using EncodeTiledFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                   const cuuint64_t *, const cuuint32_t *, const cuuint32_t *,
+                                   CUtensorMapInterleave, CUtensorMapSwizzle, CUtensorMapL2promotion,
+                                   CUtensorMapFloatOOBfill);
+EncodeTiledFn get_encode_tiled();
+
 namespace {
 
-constexpr int kPfWarps = 4;
-constexpr int kPfRows = 16 * kPfWarps;   // query rows per CTA
-constexpr int kPfKeys = 64;              // keys per K / V tile
+constexpr int kPfRows = 128;             // query rows per CTA (the MMA's M)
+constexpr int kPfKeys = 64;              // keys per K / V tile (the S MMA's N)
+constexpr int kPfStages = 3;             // K / V^T ring
+constexpr int kPfThreads = 192;          // warp 0 TMA, warp 1 MMA + tensor memory, warps 2-5 softmax
 constexpr int kPfPlanThreads = 1024;
+constexpr uint32_t kPfTmemCols = 256;    // S buffers at columns 0 and 64, O at 128
 
 struct PfArgs {
-  const __nv_bfloat16 *q, *k, *v;   // [T][H][D]
   __nv_bfloat16 *out;               // [T][Hq][D]
   const int32_t *cu;                // [B + 1]
   int32_t *cu_tiles;                // [B + 1] workspace: query-tile offsets
+  int32_t *pcu;                     // [B + 1] workspace: key offsets padded to 64 in V^T
+  const __nv_bfloat16 *v;           // [T][Hkv][D]
+  __nv_bfloat16 *vt;                // [Hkv][D][Tp] workspace
+  int64_t Tp;                       // row length of V^T (a multiple of 64)
   int32_t B, T, Hq, Hkv, G;
   float scale_log2;
   int32_t *status;
 };
 
+// One block: validates cu_seqlens, writes the prefix sums of query tiles and
+// of sequence lengths rounded up to 64 keys.
 __global__ void __launch_bounds__(kPfPlanThreads) prefill_plan_kernel(PfArgs a) {
   griddep_wait();
-  __shared__ int s_wsum[kPfPlanThreads / 32];
+  __shared__ int s_wsum[2][kPfPlanThreads / 32];
   __shared__ int s_err;
   const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
   if (tid == 0) s_err = (a.cu[0] != 0 || a.cu[a.B] > a.T) ? 1 : 0;
   __syncthreads();
-  int carry = 0;
+  int carry_t = 0, carry_p = 0;
   for (int base = 0; base < a.B; base += kPfPlanThreads) {
     const int b = base + tid;
-    int n = 0;
+    int n = 0, pk = 0;
     if (b < a.B) {
       const int len = a.cu[b + 1] - a.cu[b];
       if (len < 0) s_err = 1;
       n = len > 0 ? (len + kPfRows - 1) / kPfRows : 0;
+      pk = len > 0 ? (len + kPfKeys - 1) / kPfKeys * kPfKeys : 0;
     }
-    int incl = n;
+    int it = n, ip = pk;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
-      const int y = __shfl_up_sync(0xffffffffu, incl, o);
-      if (lane >= o) incl += y;
+      const int y = __shfl_up_sync(0xffffffffu, it, o), z = __shfl_up_sync(0xffffffffu, ip, o);
+      if (lane >= o) {
+        it += y;
+        ip += z;
+      }
     }
-    if (lane == 31) s_wsum[wid] = incl;
+    if (lane == 31) {
+      s_wsum[0][wid] = it;
+      s_wsum[1][wid] = ip;
+    }
     __syncthreads();
-    int before = 0, total = 0;
+    int bt = 0, tt = 0, bp = 0, tp = 0;
     for (int w = 0; w < kPfPlanThreads / 32; ++w) {
-      if (w < wid) before += s_wsum[w];
-      total += s_wsum[w];
+      if (w < wid) {
+        bt += s_wsum[0][w];
+        bp += s_wsum[1][w];
+      }
+      tt += s_wsum[0][w];
+      tp += s_wsum[1][w];
     }
-    if (b < a.B) a.cu_tiles[b] = carry + before + incl - n;
-    carry += total;
+    if (b < a.B) {
+      a.cu_tiles[b] = carry_t + bt + it - n;
+      a.pcu[b] = carry_p + bp + ip - pk;
+    }
+    carry_t += tt;
+    carry_p += tp;
     __syncthreads();
   }
   if (tid == 0) {
     if (s_err) set_error(a.status, UMIM_ERR_INVALID_ARG);
-    a.cu_tiles[a.B] = s_err ? 0 : carry;   // invalid offsets: no work at all
+    a.cu_tiles[a.B] = s_err ? 0 : carry_t;   // invalid offsets: no work at all
+    a.pcu[a.B] = s_err ? 0 : carry_p;
   }
 }
 
-// byte offset of 16-byte chunk c16 of key row r in a [64 rows][D] tile stored
-// as D / 64 boxes of [64 rows][128 B], 128-byte swizzled
-__device__ __forceinline__ uint32_t pf_sw(int r, int c16) {
-  return (c16 >> 3) * (kPfKeys * 128) + r * 128 + ((((c16 & 7) ^ (r & 7))) << 4);
-}
-
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src, bool fill) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(fill ? 16 : 0)
-               : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
-}
-
-template <int D>
-__global__ void __launch_bounds__(kPfWarps * 32) prefill_attn_kernel(PfArgs a) {
-  constexpr int KC = D / 16;              // k-chunks of Q K^T
-  constexpr int NT = D / 8;               // n-tiles of the output
-  constexpr int CPR = D / 8;              // 16-byte chunks per row
-  constexpr int kTile = kPfKeys * D * 2;  // bytes of one K (or V) tile
-  extern __shared__ __align__(1024) uint8_t pf_smem[];
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(pf_smem) + 1023) & ~uintptr_t(1023));
-
-  griddep_wait();
-  const int total = a.cu_tiles[a.B];
-  if ((int)blockIdx.x >= total) return;
-  const int t = total - 1 - (int)blockIdx.x;   // a sequence's last (heaviest) tiles first
-  int lo = 0, hi = a.B;                        // sequence: last b with cu_tiles[b] <= t
+// last index b in [0, B) with key[b] <= x
+__device__ __forceinline__ int pf_find(const int32_t *key, int B, int x) {
+  int lo = 0, hi = B;
   while (hi - lo > 1) {
     const int mid = (lo + hi) >> 1;
-    if (a.cu_tiles[mid] <= t) lo = mid;
+    if (key[mid] <= x) lo = mid;
     else hi = mid;
   }
-  const int b = lo;
-  const int qt = t - a.cu_tiles[b];
-  const int s0 = a.cu[b], len = a.cu[b + 1] - s0;
-  const int q0 = qt * kPfRows;
-  const int h = blockIdx.y, g = h / a.G;
-  const int n_kv = qt + 1;   // causal: keys up to the tile's last query row
+  return lo;
+}
 
-  auto load_kv = [&](int kt, int buf) {
-    uint8_t *kd = base + buf * 2 * kTile;
-    uint8_t *vd = kd + kTile;
-    for (int c = threadIdx.x; c < kPfKeys * CPR; c += kPfWarps * 32) {
-      const int r = c / CPR, c16 = c % CPR;
-      const int key = kt * kPfKeys + r;
-      const bool ok = key < len;
-      const int64_t row = (int64_t)s0 + (ok ? key : 0);
-      const int64_t off = (row * a.Hkv + g) * D + c16 * 8;
-      cp_async16(smem_u32(kd + pf_sw(r, c16)), a.k + off, ok);
-      cp_async16(smem_u32(vd + pf_sw(r, c16)), a.v + off, ok);
-    }
-    cp_async_commit();
-  };
-  load_kv(0, 0);
-
-  // Q fragments of this warp's 16 rows
-  const int qr = lane >> 2, qc = lane & 3;
-  const int r0 = q0 + warp * 16 + qr, r1 = r0 + 8;   // rows within the sequence
-  uint32_t qa[KC][4];
-  {
-    const __nv_bfloat16 *q0p = a.q + (((int64_t)s0 + r0) * a.Hq + h) * D;
-    const __nv_bfloat16 *q1p = a.q + (((int64_t)s0 + r1) * a.Hq + h) * D;
-#pragma unroll
-    for (int c = 0; c < KC; ++c) {
-      const int k0 = c * 16 + 2 * qc;
-      qa[c][0] = r0 < len ? *reinterpret_cast<const uint32_t *>(q0p + k0) : 0u;
-      qa[c][1] = r1 < len ? *reinterpret_cast<const uint32_t *>(q1p + k0) : 0u;
-      qa[c][2] = r0 < len ? *reinterpret_cast<const uint32_t *>(q0p + k0 + 8) : 0u;
-      qa[c][3] = r1 < len ? *reinterpret_cast<const uint32_t *>(q1p + k0 + 8) : 0u;
-    }
+// V^T: vt[g][d][pcu[b] + t] = v[cu[b] + t][g][d] for t < len_b, 0 up to the
+// next multiple of 64.  One CTA per 64 padded keys and KV head, through a
+// shared-memory tile.
+template <int D>
+__global__ void __launch_bounds__(256) vt_kernel(PfArgs a) {
+  griddep_wait();
+  __shared__ uint32_t tile[kPfKeys][D / 2 + 1];   // bf16 pairs, padded against bank conflicts
+  const int k0 = blockIdx.x * kPfKeys, g = blockIdx.y;
+  if (k0 >= a.pcu[a.B]) return;
+  const int b = pf_find(a.pcu, a.B, k0);
+  const int len = a.cu[b + 1] - a.cu[b];
+  const int t0 = k0 - a.pcu[b];
+  constexpr int CPR = D / 8;   // 16-byte chunks per key row
+  for (int i = threadIdx.x; i < kPfKeys * CPR; i += blockDim.x) {
+    const int r = i / CPR, c = i % CPR;
+    uint4 u = make_uint4(0, 0, 0, 0);
+    if (t0 + r < len)
+      u = __ldg(reinterpret_cast<const uint4 *>(a.v + ((int64_t)(a.cu[b] + t0 + r) * a.Hkv + g) * D) + c);
+    tile[r][4 * c] = u.x;
+    tile[r][4 * c + 1] = u.y;
+    tile[r][4 * c + 2] = u.z;
+    tile[r][4 * c + 3] = u.w;
   }
-  float acc[NT][4];
+  __syncthreads();
+  // each thread writes 8 keys of one d row (16 bytes)
+  for (int i = threadIdx.x; i < D * (kPfKeys / 8); i += blockDim.x) {
+    const int d = i / (kPfKeys / 8), c = i % (kPfKeys / 8);
+    uint32_t w[4];
 #pragma unroll
-  for (int j = 0; j < NT; ++j) acc[j][0] = acc[j][1] = acc[j][2] = acc[j][3] = 0.f;
-  float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
-
-  for (int kt = 0; kt < n_kv; ++kt) {
-    if (kt + 1 < n_kv) {
-      load_kv(kt + 1, (kt + 1) & 1);
-      cp_async_wait<1>();
-    } else {
-      cp_async_wait<0>();
+    for (int j = 0; j < 4; ++j) {
+      const uint32_t x0 = tile[8 * c + 2 * j][d >> 1], x1 = tile[8 * c + 2 * j + 1][d >> 1];
+      const uint32_t lo = (d & 1) ? (x0 >> 16) : (x0 & 0xffffu);
+      const uint32_t hi = (d & 1) ? (x1 >> 16) : (x1 & 0xffffu);
+      w[j] = lo | (hi << 16);
     }
-    __syncthreads();
-    const uint32_t ks = smem_u32(base + (kt & 1) * 2 * kTile), vs = ks + kTile;
-
-    // S = Q K^T: 16 rows x 64 keys (8 n-tiles)
-    float s[8][4];
-#pragma unroll
-    for (int nt = 0; nt < 8; ++nt) s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
-#pragma unroll
-    for (int c = 0; c < KC; ++c) {
-#pragma unroll
-      for (int np = 0; np < 4; ++np) {
-        const int key = np * 16 + (lane & 7) + ((lane >> 4) << 3);
-        const int c16 = 2 * c + ((lane >> 3) & 1);
-        uint32_t b0, b1, b2, b3;
-        ldsm_x4(ks + pf_sw(key, c16), b0, b1, b2, b3);
-        mma_bf16(s[2 * np], qa[c], b0, b1);
-        mma_bf16(s[2 * np + 1], qa[c], b2, b3);
-      }
-    }
-    // scale to log2 units; causal mask (key > row) and keys past the end
-    float mx0 = -INFINITY, mx1 = -INFINITY;
-#pragma unroll
-    for (int nt = 0; nt < 8; ++nt)
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int key = kt * kPfKeys + nt * 8 + 2 * qc + (e & 1);
-        const int row = e < 2 ? r0 : r1;
-        const bool keep = key <= row && key < len;
-        s[nt][e] = keep ? s[nt][e] * a.scale_log2 : -INFINITY;
-        if (e < 2) mx0 = fmaxf(mx0, s[nt][e]);
-        else mx1 = fmaxf(mx1, s[nt][e]);
-      }
-    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
-    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
-    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
-    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
-    const float n0 = fmaxf(m0, mx0), n1 = fmaxf(m1, mx1);
-    // rows whose keys are all masked so far keep m = -inf: use 0 as the reference
-    const float e0 = n0 == -INFINITY ? 0.f : n0, e1 = n1 == -INFINITY ? 0.f : n1;
-    const float c0 = exp2f(m0 - e0), c1 = exp2f(m1 - e1);
-    m0 = n0;
-    m1 = n1;
-    float rs0 = 0.f, rs1 = 0.f;
-#pragma unroll
-    for (int nt = 0; nt < 8; ++nt) {
-      s[nt][0] = exp2f(s[nt][0] - e0);
-      s[nt][1] = exp2f(s[nt][1] - e0);
-      s[nt][2] = exp2f(s[nt][2] - e1);
-      s[nt][3] = exp2f(s[nt][3] - e1);
-      rs0 += s[nt][0] + s[nt][1];
-      rs1 += s[nt][2] + s[nt][3];
-    }
-    l0 = l0 * c0 + rs0;
-    l1 = l1 * c1 + rs1;
-#pragma unroll
-    for (int j = 0; j < NT; ++j) {
-      acc[j][0] *= c0;
-      acc[j][1] *= c0;
-      acc[j][2] *= c1;
-      acc[j][3] *= c1;
-    }
-    // O += P V over the tile's 4 groups of 16 keys
-#pragma unroll
-    for (int kc = 0; kc < 4; ++kc) {
-      uint32_t ph[4], pl[4];
-      const float v4[4][2] = {{s[2 * kc][0], s[2 * kc][1]}, {s[2 * kc][2], s[2 * kc][3]},
-                              {s[2 * kc + 1][0], s[2 * kc + 1][1]}, {s[2 * kc + 1][2], s[2 * kc + 1][3]}};
-#pragma unroll
-      for (int r = 0; r < 4; ++r) {
-        const __nv_bfloat162 hh = __floats2bfloat162_rn(v4[r][0], v4[r][1]);
-        ph[r] = *reinterpret_cast<const uint32_t *>(&hh);
-        pl[r] = pack_bf16(v4[r][0] - __low2float(hh), v4[r][1] - __high2float(hh));
-      }
-#pragma unroll
-      for (int j = 0; j < D / 16; ++j) {
-        const int key = kc * 16 + (lane & 7) + (((lane >> 3) & 1) << 3);
-        const int c16 = 2 * j + (lane >> 4);
-        uint32_t b0, b1, b2, b3;
-        ldsm_x4_t(vs + pf_sw(key, c16), b0, b1, b2, b3);
-        mma_bf16(acc[2 * j], ph, b0, b1);
-        mma_bf16(acc[2 * j + 1], ph, b2, b3);
-        mma_bf16(acc[2 * j], pl, b0, b1);
-        mma_bf16(acc[2 * j + 1], pl, b2, b3);
-      }
-    }
-    __syncthreads();   // this buffer is refilled two tiles later
-  }
-
-  // normalise and store
-  l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
-  l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
-  l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
-  l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
-  const float i0 = l0 > 0.f ? 1.f / l0 : 0.f, i1 = l1 > 0.f ? 1.f / l1 : 0.f;
-  __nv_bfloat16 *o0 = a.out + (((int64_t)s0 + r0) * a.Hq + h) * D;
-  __nv_bfloat16 *o1 = a.out + (((int64_t)s0 + r1) * a.Hq + h) * D;
-#pragma unroll
-  for (int j = 0; j < NT; ++j) {
-    const int col = j * 8 + 2 * qc;
-    if (r0 < len) *reinterpret_cast<uint32_t *>(o0 + col) = pack_bf16(acc[j][0] * i0, acc[j][1] * i0);
-    if (r1 < len) *reinterpret_cast<uint32_t *>(o1 + col) = pack_bf16(acc[j][2] * i1, acc[j][3] * i1);
+    *reinterpret_cast<uint4 *>(a.vt + ((int64_t)g * D + d) * a.Tp + k0 + 8 * c) = make_uint4(w[0], w[1], w[2], w[3]);
   }
 }
+
+__device__ __forceinline__ void tma_load_3d(void *dst, const CUtensorMap *map, uint64_t *bar, int c0, int c1, int c2,
+                                            uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%2, %3, %4}], [%5], %6;" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(smem_u32(bar)), "l"(policy)
+      : "memory");
+}
+
+// 32 lanes x 32 consecutive fp32 columns back into tensor memory (thread i: row lane base + i)
+__device__ __forceinline__ void tmem_st_32x32b_x32(uint32_t taddr, const float (&v)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
+      "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, "
+      "%17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(taddr),
+      "f"(v[0]), "f"(v[1]), "f"(v[2]), "f"(v[3]), "f"(v[4]), "f"(v[5]), "f"(v[6]), "f"(v[7]), "f"(v[8]), "f"(v[9]),
+      "f"(v[10]), "f"(v[11]), "f"(v[12]), "f"(v[13]), "f"(v[14]), "f"(v[15]), "f"(v[16]), "f"(v[17]), "f"(v[18]),
+      "f"(v[19]), "f"(v[20]), "f"(v[21]), "f"(v[22]), "f"(v[23]), "f"(v[24]), "f"(v[25]), "f"(v[26]), "f"(v[27]),
+      "f"(v[28]), "f"(v[29]), "f"(v[30]), "f"(v[31])
+      : "memory");
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  __nv_bfloat162 p = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t *>(&p);
+}
+
+// shared-memory layout of the attention kernel (bytes, every piece 1024-aligned)
+template <int D>
+struct PfSmem {
+  static constexpr int kQ = kPfRows * D * 2;              // Q: D/64 atoms of [128 rows][128 B]
+  static constexpr int kK = kPfKeys * D * 2;              // K tile: D/64 atoms of [64 keys][128 B]
+  static constexpr int kV = D * kPfKeys * 2;              // V^T tile: [D rows][128 B]
+  static constexpr int kStage = kK + kV;
+  static constexpr int kP = kPfRows * kPfKeys * 2;        // one P part: [128 rows][128 B]
+  static constexpr int kStages = kQ;                      // offsets
+  static constexpr int kPbuf = kStages + kPfStages * kStage;
+  static constexpr int kTotal = kPbuf + 2 * 2 * kP;       // two buffers of (high, remainder)
+};
+
+template <int D>
+__global__ void __launch_bounds__(kPfThreads, 1)
+    prefill_tc_kernel(const __grid_constant__ CUtensorMap q_map, const __grid_constant__ CUtensorMap k_map,
+                      const __grid_constant__ CUtensorMap vt_map, PfArgs a) {
+  using L = PfSmem<D>;
+  constexpr int DA = D / 64;   // 64-wide atoms along the head dimension
+  extern __shared__ __align__(1024) uint8_t pf_raw[];
+  __shared__ __align__(8) uint64_t q_full, kv_full[kPfStages], kv_empty[kPfStages], s_full[2], s_empty[2], p_full[2],
+      p_empty[2], mma_done;
+  __shared__ uint32_t tmem_base;
+  uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(pf_raw) + 1023) & ~uintptr_t(1023));
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    mbar_init(&q_full, 1);
+    for (int s = 0; s < kPfStages; ++s) {
+      mbar_init(&kv_full[s], 1);
+      mbar_init(&kv_empty[s], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&s_full[i], 1);
+      mbar_init(&s_empty[i], 4);   // one arrival per softmax warp
+      mbar_init(&p_full[i], 4);
+      mbar_init(&p_empty[i], 1);
+    }
+    mbar_init(&mma_done, 1);
+    fence_mbar_init();
+    prefetch_tensormap(&q_map);
+    prefetch_tensormap(&k_map);
+    prefetch_tensormap(&vt_map);
+  }
+  if (warp == 1) {
+    tmem_alloc(&tmem_base, kPfTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tmem_base;
+  griddep_wait();
+
+  // the work unit: query tile qt of sequence b, query head h
+  const int total = a.cu_tiles[a.B];
+  bool active = (int)blockIdx.x < total;
+  int b = 0, qt = 0;
+  if (active) {
+    const int t = total - 1 - (int)blockIdx.x;   // a sequence's last (heaviest) tiles first
+    b = pf_find(a.cu_tiles, a.B, t);
+    qt = t - a.cu_tiles[b];
+  }
+  const int s0 = active ? a.cu[b] : 0, len = active ? a.cu[b + 1] - s0 : 0;
+  const int q0 = qt * kPfRows;
+  const int h = blockIdx.y, g = h / a.G;
+  const int n_kv = active ? (min(q0 + kPfRows, len) + kPfKeys - 1) / kPfKeys : 0;   // causal key tiles
+  const int kbase = active ? a.pcu[b] : 0;
+
+  if (warp == 0) {
+    if (lane == 0 && n_kv > 0) {
+      const uint64_t pol_q = policy_evict_first(), pol_kv = policy_evict_last();
+      mbar_arrive_expect_tx(&q_full, L::kQ);
+#pragma unroll
+      for (int d = 0; d < DA; ++d) tma_load_3d(smem + d * (kPfRows * 128), &q_map, &q_full, d * 64, h, s0 + q0, pol_q);
+      int j = 0;
+      for (; j < n_kv; ++j) {
+        const int s = j % kPfStages;
+        if (!mbar_wait(&kv_empty[s], ((j / kPfStages) & 1) ^ 1)) {
+          set_error(a.status, UMIM_ERR_TIMEOUT);
+          break;
+        }
+        uint8_t *st = smem + L::kStages + s * L::kStage;
+        mbar_arrive_expect_tx(&kv_full[s], L::kStage);
+#pragma unroll
+        for (int d = 0; d < DA; ++d)
+          tma_load_3d(st + d * (kPfKeys * 128), &k_map, &kv_full[s], d * 64, g, s0 + j * kPfKeys, pol_kv);
+        tma_load_3d(st + L::kK, &vt_map, &kv_full[s], kbase + j * kPfKeys, 0, g, pol_kv);
+      }
+      // copies still in flight when a consumer gave up: wait for them (bounded)
+      for (int i = max(0, j - kPfStages); i < j; ++i)
+        mbar_wait_for(&kv_full[i % kPfStages], (i / kPfStages) & 1, kWaitLimitNs);
+      mbar_wait_for(&q_full, 0, kWaitLimitNs);
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && n_kv > 0) {
+      constexpr uint32_t idesc_s = idesc_f32acc(kPfRows, kPfKeys, false);
+      constexpr uint32_t idesc_o = idesc_f32acc(kPfRows, D, false);
+      const uint32_t q_base = smem_u32(smem);
+      const uint32_t o_tmem = tmem + 128;
+      bool ok = mbar_wait(&q_full, 0);
+      tc_fence_after();
+      // O += P_i V_i for key tile i (high part, then remainder)
+      auto pv = [&](int i) {
+        const int pb = i & 1;
+        if (!mbar_wait(&p_full[pb], (i >> 1) & 1)) return false;
+        if (!mbar_wait(&kv_full[i % kPfStages], (i / kPfStages) & 1)) return false;
+        tc_fence_after();
+        const uint32_t v_base = smem_u32(smem + L::kStages + (i % kPfStages) * L::kStage + L::kK);
+#pragma unroll
+        for (int part = 0; part < 2; ++part) {
+          const uint32_t p_base = smem_u32(smem + L::kPbuf + (pb * 2 + part) * L::kP);
+#pragma unroll
+          for (int kk = 0; kk < kPfKeys / 16; ++kk)
+            tc_mma_bf16(o_tmem, sw128_kmajor_desc(p_base + kk * 32), sw128_kmajor_desc(v_base + kk * 32), idesc_o,
+                        (i | part | kk) != 0 ? 1u : 0u);
+        }
+        tc_commit(&p_empty[pb]);
+        tc_commit(&kv_empty[i % kPfStages]);
+        return true;
+      };
+      for (int j = 0; j < n_kv && ok; ++j) {
+        const int s = j % kPfStages, sb = j & 1;
+        if (!mbar_wait(&kv_full[s], (j / kPfStages) & 1) || !mbar_wait(&s_empty[sb], ((j >> 1) & 1) ^ 1)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t k_base = smem_u32(smem + L::kStages + s * L::kStage);
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {
+          const uint32_t off = (kk & 3) * 32;
+          const uint64_t ad = sw128_kmajor_desc(q_base + (kk >> 2) * (kPfRows * 128) + off);
+          const uint64_t bd = sw128_kmajor_desc(k_base + (kk >> 2) * (kPfKeys * 128) + off);
+          tc_mma_bf16(tmem + sb * kPfKeys, ad, bd, idesc_s, kk != 0 ? 1u : 0u);
+        }
+        tc_commit(&s_full[sb]);
+        if (j >= 1 && !pv(j - 1)) ok = false;
+      }
+      if (ok && !pv(n_kv - 1)) ok = false;
+      if (!ok) set_error(a.status, UMIM_ERR_TIMEOUT);
+      // every MMA issued has finished before tensor memory is released
+      tc_commit(&mma_done);
+      mbar_wait_for(&mma_done, 0, kWaitLimitNs);
+    }
+  } else {
+    // ---- softmax and epilogue: warps 2-5, thread = query row ----
+    const int quad = warp & 3;                 // tensor-memory lanes this warp may access
+    const int r = quad * 32 + lane;            // query row within the tile
+    const int qpos = q0 + r;                   // position within the sequence
+    const int kmax = min(qpos, len - 1);       // last key this row sees (< 0: a row past the sequence)
+    const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
+    const float sl2 = a.scale_log2;
+    float m_run = -INFINITY, l_run = 0.f;      // running max (log2 units, moved in steps > 8) and row sum
+    bool ok = true;
+    // every lane waits (each needs the acquire), the warp goes on only if all saw the phase:
+    // the .sync.aligned tensor-memory instructions below need the whole warp
+    auto wwait = [&](uint64_t *m, uint32_t parity) { return __all_sync(0xffffffffu, mbar_wait(m, parity)) != 0; };
+    for (int j = 0; j < n_kv && ok; ++j) {
+      const int sb = j & 1;
+      if (!wwait(&s_full[sb], (j >> 1) & 1)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      float x[kPfKeys];
+      tmem_ld_32x32b_x32(tmem + lane_addr + sb * kPfKeys, *reinterpret_cast<float(*)[32]>(x));
+      tmem_ld_32x32b_x32(tmem + lane_addr + sb * kPfKeys + 32, *reinterpret_cast<float(*)[32]>(x + 32));
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&s_empty[sb]);   // the S buffer may be overwritten
+      const int k0 = j * kPfKeys;
+      float mx = -INFINITY;
+#pragma unroll
+      for (int c = 0; c < kPfKeys; ++c) {
+        x[c] = (k0 + c <= kmax) ? x[c] * sl2 : -INFINITY;
+        mx = fmaxf(mx, x[c]);
+      }
+      // move the running max only when it grows by more than 2^8
+      const bool grow = mx > m_run + 8.f;
+      float alpha = 1.f;
+      if (grow) {
+        alpha = (m_run == -INFINITY) ? 0.f : exp2f(m_run - mx);
+        m_run = mx;
+        l_run *= alpha;
+      }
+      if (j > 0 && __any_sync(0xffffffffu, grow && alpha != 1.f)) {
+        // rescale this warp's rows of O once the product of tile j - 1 has landed
+        if (!wwait(&p_empty[(j - 1) & 1], ((j - 1) >> 1) & 1)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+#pragma unroll 1
+        for (int c = 0; c < D / 32; ++c) {
+          float o[32];
+          tmem_ld_32x32b_x32(tmem + lane_addr + 128 + c * 32, o);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) o[i] *= alpha;
+          tmem_st_32x32b_x32(tmem + lane_addr + 128 + c * 32, o);
+        }
+        tc_fence_before();
+      }
+      const float mb = (m_run == -INFINITY) ? 0.f : m_run;
+      float sum = 0.f;
+#pragma unroll
+      for (int c = 0; c < kPfKeys; ++c) {
+        x[c] = exp2f(x[c] - mb);   // masked: 0
+        sum += x[c];
+      }
+      l_run += sum;
+      // P of tile j into buffer j & 1 once the product of tile j - 2 has read it
+      const int pb = j & 1;
+      if (j >= 2 && !wwait(&p_empty[pb], ((j >> 1) & 1) ^ 1)) {
+        ok = false;
+        break;
+      }
+      uint8_t *ph = smem + L::kPbuf + (pb * 2) * L::kP + r * 128;
+      uint8_t *pl = ph + L::kP;
+#pragma unroll
+      for (int c = 0; c < kPfKeys / 8; ++c) {
+        uint32_t hw[4], lw[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float p0 = x[8 * c + 2 * e], p1 = x[8 * c + 2 * e + 1];
+          const __nv_bfloat162 hh = __floats2bfloat162_rn(p0, p1);
+          hw[e] = *reinterpret_cast<const uint32_t *>(&hh);
+          lw[e] = pack_bf16x2(p0 - __low2float(hh), p1 - __high2float(hh));
+        }
+        const int pos = (c ^ (r & 7)) << 4;   // 128-byte swizzle of a K-major operand
+        *reinterpret_cast<uint4 *>(ph + pos) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+        *reinterpret_cast<uint4 *>(pl + pos) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+      }
+      fence_proxy_async_smem();   // visible to the tensor cores
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&p_full[pb]);
+    }
+    if (!ok) set_error(a.status, UMIM_ERR_TIMEOUT);
+    // epilogue: O / l once the last product has landed
+    if (ok && n_kv > 0 && wwait(&p_empty[(n_kv - 1) & 1], ((n_kv - 1) >> 1) & 1)) {
+      tc_fence_after();
+      const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
+      __nv_bfloat16 *orow = a.out + (((int64_t)s0 + qpos) * a.Hq + h) * D;
+#pragma unroll 1
+      for (int c = 0; c < D / 32; ++c) {
+        float o[32];
+        tmem_ld_32x32b_x32(tmem + lane_addr + 128 + c * 32, o);
+        if (qpos < len) {
+          uint4 *dst = reinterpret_cast<uint4 *>(orow + c * 32);
+#pragma unroll
+          for (int e = 0; e < 4; ++e)
+            dst[e] = make_uint4(pack_bf16x2(o[8 * e] * inv, o[8 * e + 1] * inv),
+                                pack_bf16x2(o[8 * e + 2] * inv, o[8 * e + 3] * inv),
+                                pack_bf16x2(o[8 * e + 4] * inv, o[8 * e + 5] * inv),
+                                pack_bf16x2(o[8 * e + 6] * inv, o[8 * e + 7] * inv));
+        }
+      }
+    } else if (n_kv > 0 && ok) {
+      set_error(a.status, UMIM_ERR_TIMEOUT);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kPfTmemCols);
+  }
+}
+
+bool encode_3d(EncodeTiledFn enc, CUtensorMap *map, const void *base, uint64_t d0, uint64_t d1, uint64_t d2,
+               uint64_t stride1, uint64_t stride2, uint32_t b0, uint32_t b1, uint32_t b2) {
+  const cuuint64_t dims[3] = {d0, d1, d2};
+  const cuuint64_t strides[2] = {stride1, stride2};
+  const cuuint32_t box[3] = {b0, b1, b2};
+  const cuuint32_t es[3] = {1, 1, 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims, strides, box, es,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// row length of V^T: room for every sequence padded to 64 keys
+int64_t vt_row(int B, int T) { return ((int64_t)T + 63LL * B + 63) / 64 * 64; }
 
 }  // namespace
 
-size_t prefill_attention_workspace_bytes(int B) { return ((size_t)(B + 1) * sizeof(int32_t) + 255) & ~size_t(255); }
+size_t prefill_attention_workspace_bytes(int B, int T, int Hkv, int D) {
+  const size_t plan = ((size_t)2 * (B + 1) * sizeof(int32_t) + 1023) & ~size_t(1023);
+  return plan + (size_t)Hkv * D * vt_row(B, T) * 2;
+}
 
 umim_status prefill_attention(const void *q, const void *k, const void *v, int T, int Hq, int Hkv, int D,
                               const int32_t *cu_seqlens, int B, float scale, void *out, void *ws, int32_t *status,
-                              cudaStream_t stream) {
+                              cudaStream_t stream, int num_sms) {
+  (void)num_sms;
+  EncodeTiledFn enc = get_encode_tiled();
+  if (!enc) return UMIM_ERR_CUDA;
   PfArgs a{};
-  a.q = static_cast<const __nv_bfloat16 *>(q);
-  a.k = static_cast<const __nv_bfloat16 *>(k);
-  a.v = static_cast<const __nv_bfloat16 *>(v);
   a.out = static_cast<__nv_bfloat16 *>(out);
   a.cu = cu_seqlens;
   a.cu_tiles = static_cast<int32_t *>(ws);
+  a.pcu = a.cu_tiles + (B + 1);
+  a.v = static_cast<const __nv_bfloat16 *>(v);
+  a.vt = reinterpret_cast<__nv_bfloat16 *>(static_cast<char *>(ws) +
+                                           (((size_t)2 * (B + 1) * sizeof(int32_t) + 1023) & ~size_t(1023)));
+  a.Tp = vt_row(B, T);
   a.B = B;
   a.T = T;
   a.Hq = Hq;
@@ -285,17 +501,26 @@ umim_status prefill_attention(const void *q, const void *k, const void *v, int T
   a.G = Hq / Hkv;
   a.scale_log2 = (scale > 0.f ? scale : 1.0f / sqrtf((float)D)) * 1.4426950408889634f;
   a.status = status;
+  CUtensorMap qm, km, vm;
+  if (!encode_3d(enc, &qm, q, D, Hq, T, (uint64_t)D * 2, (uint64_t)Hq * D * 2, 64, 1, kPfRows) ||
+      !encode_3d(enc, &km, k, D, Hkv, T, (uint64_t)D * 2, (uint64_t)Hkv * D * 2, 64, 1, kPfKeys) ||
+      !encode_3d(enc, &vm, a.vt, a.Tp, D, Hkv, (uint64_t)a.Tp * 2, (uint64_t)D * a.Tp * 2, kPfKeys, D, 1))
+    return UMIM_ERR_CUDA;
   trace_mark(stream, "prefill.plan");
   if (launch_pdl(prefill_plan_kernel, dim3(1), dim3(kPfPlanThreads), 0, stream, a) != cudaSuccess)
     return UMIM_ERR_CUDA;
-  auto kern = D == 128 ? prefill_attn_kernel<128> : prefill_attn_kernel<64>;
-  const size_t smem = (size_t)2 * 2 * kPfKeys * D * 2 + 1024;
+  trace_mark(stream, "prefill.v_transpose");
+  auto vk = D == 128 ? vt_kernel<128> : vt_kernel<64>;
+  if (launch_pdl(vk, dim3((unsigned)(a.Tp / kPfKeys), (unsigned)Hkv), dim3(256), 0, stream, a) != cudaSuccess)
+    return UMIM_ERR_CUDA;
+  auto kern = D == 128 ? prefill_tc_kernel<128> : prefill_tc_kernel<64>;
+  const size_t smem = (size_t)(D == 128 ? PfSmem<128>::kTotal : PfSmem<64>::kTotal) + 1024;
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
     return UMIM_ERR_CUDA;
   // an upper bound of the query tiles: each sequence wastes less than one
   const unsigned gx = (unsigned)((T + kPfRows - 1) / kPfRows + B);
   trace_mark(stream, "prefill.attention");
-  if (launch_pdl(kern, dim3(gx, (unsigned)Hq), dim3(kPfWarps * 32), smem, stream, a) != cudaSuccess)
+  if (launch_pdl(kern, dim3(gx, (unsigned)Hq), dim3(kPfThreads), smem, stream, qm, km, vm, a) != cudaSuccess)
     return UMIM_ERR_CUDA;
   trace_mark(stream, nullptr);
   return UMIM_OK;
