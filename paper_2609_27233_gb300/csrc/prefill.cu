@@ -8,8 +8,8 @@
 // sequence and one query head.  Warp 0 loads tiles with TMA (Q once; K and
 // V^T tiles of 64 keys into a 3-stage ring), warp 1 issues tcgen05.mma
 // (S = Q K^T into one of two tensor-memory buffers, then O += P V into a
-// tensor-memory accumulator), warps 2-5 run the online softmax, one thread
-// per query row: S from tensor memory (tcgen05.ld), causal mask, running max,
+// tensor-memory accumulator), warps 2-9 run the online softmax, two warps
+// per 32 query rows (32 of a tile's 64 keys each): S from tensor memory (tcgen05.ld), causal mask, running max,
 // P = exp2(S - max) written to shared memory as a bf16 high part and a bf16
 // remainder (two MMAs per P V product keep P's rounding out of the error
 // budget), row sums.  The running max is only moved when it grows by more
@@ -36,10 +36,10 @@ namespace {
 
 constexpr int kPfRows = 128;             // query rows per CTA (the MMA's M)
 constexpr int kPfKeys = 64;              // keys per K / V tile (the S MMA's N)
-constexpr int kPfStages = 3;             // K / V^T ring
-constexpr int kPfThreads = 192;          // warp 0 TMA, warp 1 MMA + tensor memory, warps 2-5 softmax
+constexpr int kPfStages = 2;             // K and V^T rings
+constexpr int kPfThreads = 320;          // warp 0 TMA, warp 1 MMA + tensor memory, warps 2-5 / 6-9 softmax of head 0 / 1
 constexpr int kPfPlanThreads = 1024;
-constexpr uint32_t kPfTmemCols = 256;    // S buffers at columns 0 and 64, O at 128
+constexpr uint32_t kPfTmemCols = 512;    // per head x: S buffers at 256x + 0 and + 64, O at 256x + 128
 
 struct PfArgs {
   __nv_bfloat16 *out;               // [T][Hq][D]
@@ -170,6 +170,21 @@ __device__ __forceinline__ void tma_load_3d(void *dst, const CUtensorMap *map, u
       : "memory");
 }
 
+// 32 lanes x 64 consecutive fp32 columns from tensor memory in one load
+// (thread i: row lane base + i), waited for inside the same statement so no
+// register is read before it has landed
+__device__ __forceinline__ void tmem_ld_32x32b_x64(uint32_t taddr, float (&v)[64]) {
+  uint32_t r[64];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x64.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32, %33, %34, %35, %36, %37, %38, %39, %40, %41, %42, %43, %44, %45, %46, %47, %48, %49, %50, %51, %52, %53, %54, %55, %56, %57, %58, %59, %60, %61, %62, %63}, [%64];\n\t"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31]), "=r"(r[32]), "=r"(r[33]), "=r"(r[34]), "=r"(r[35]), "=r"(r[36]), "=r"(r[37]), "=r"(r[38]), "=r"(r[39]), "=r"(r[40]), "=r"(r[41]), "=r"(r[42]), "=r"(r[43]), "=r"(r[44]), "=r"(r[45]), "=r"(r[46]), "=r"(r[47]), "=r"(r[48]), "=r"(r[49]), "=r"(r[50]), "=r"(r[51]), "=r"(r[52]), "=r"(r[53]), "=r"(r[54]), "=r"(r[55]), "=r"(r[56]), "=r"(r[57]), "=r"(r[58]), "=r"(r[59]), "=r"(r[60]), "=r"(r[61]), "=r"(r[62]), "=r"(r[63])
+      : "r"(taddr)
+      : "memory");
+#pragma unroll
+  for (int i = 0; i < 64; ++i) v[i] = __uint_as_float(r[i]);
+}
+
 // 32 lanes x 32 consecutive fp32 columns back into tensor memory (thread i: row lane base + i)
 __device__ __forceinline__ void tmem_st_32x32b_x32(uint32_t taddr, const float (&v)[32]) {
   asm volatile(
@@ -184,6 +199,14 @@ __device__ __forceinline__ void tmem_st_32x32b_x32(uint32_t taddr, const float (
   asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
 
+// the hardware's approximate base-2 exponential (PTX ex2.approx.ftz: relative
+// error about 2^-22, -inf -> 0)
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   __nv_bfloat162 p = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t *>(&p);
@@ -192,14 +215,14 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 // shared-memory layout of the attention kernel (bytes, every piece 1024-aligned)
 template <int D>
 struct PfSmem {
-  static constexpr int kQ = kPfRows * D * 2;              // Q: D/64 atoms of [128 rows][128 B]
+  static constexpr int kQ = kPfRows * D * 2;              // Q of one head: D/64 atoms of [128 rows][128 B]
   static constexpr int kK = kPfKeys * D * 2;              // K tile: D/64 atoms of [64 keys][128 B]
   static constexpr int kV = D * kPfKeys * 2;              // V^T tile: [D rows][128 B]
-  static constexpr int kStage = kK + kV;
-  static constexpr int kP = kPfRows * kPfKeys * 2;        // one P part: [128 rows][128 B]
-  static constexpr int kStages = kQ;                      // offsets
-  static constexpr int kPbuf = kStages + kPfStages * kStage;
-  static constexpr int kTotal = kPbuf + 2 * 2 * kP;       // two buffers of (high, remainder)
+  static constexpr int kP = kPfRows * kPfKeys * 2;        // one P part of one head: [128 rows][128 B]
+  static constexpr int kKoff = 2 * kQ;
+  static constexpr int kVoff = kKoff + kPfStages * kK;
+  static constexpr int kPoff = kVoff + kPfStages * kV;
+  static constexpr int kTotal = kPoff + 2 * 2 * kP;       // [head][high, remainder]
 };
 
 template <int D>
@@ -209,8 +232,8 @@ __global__ void __launch_bounds__(kPfThreads, 1)
   using L = PfSmem<D>;
   constexpr int DA = D / 64;   // 64-wide atoms along the head dimension
   extern __shared__ __align__(1024) uint8_t pf_raw[];
-  __shared__ __align__(8) uint64_t q_full, kv_full[kPfStages], kv_empty[kPfStages], s_full[2], s_empty[2], p_full[2],
-      p_empty[2], mma_done;
+  __shared__ __align__(8) uint64_t q_full, k_full[kPfStages], k_empty[kPfStages], v_full[kPfStages],
+      v_empty[kPfStages], s_full[2][2], s_empty[2][2], p_full[2], p_empty[2], mma_done;
   __shared__ uint32_t tmem_base;
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(pf_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -218,14 +241,18 @@ __global__ void __launch_bounds__(kPfThreads, 1)
   if (threadIdx.x == 0) {
     mbar_init(&q_full, 1);
     for (int s = 0; s < kPfStages; ++s) {
-      mbar_init(&kv_full[s], 1);
-      mbar_init(&kv_empty[s], 1);
+      mbar_init(&k_full[s], 1);
+      mbar_init(&k_empty[s], 1);
+      mbar_init(&v_full[s], 1);
+      mbar_init(&v_empty[s], 1);
     }
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(&s_full[i], 1);
-      mbar_init(&s_empty[i], 4);   // one arrival per softmax warp
-      mbar_init(&p_full[i], 4);
-      mbar_init(&p_empty[i], 1);
+    for (int x = 0; x < 2; ++x) {
+      for (int i = 0; i < 2; ++i) {
+        mbar_init(&s_full[x][i], 1);
+        mbar_init(&s_empty[x][i], 4);   // one arrival per softmax warp of the head
+      }
+      mbar_init(&p_full[x], 4);
+      mbar_init(&p_empty[x], 1);
     }
     mbar_init(&mma_done, 1);
     fence_mbar_init();
@@ -243,9 +270,9 @@ __global__ void __launch_bounds__(kPfThreads, 1)
   const uint32_t tmem = tmem_base;
   griddep_wait();
 
-  // the work unit: query tile qt of sequence b, query head h
+  // the work unit: query tile qt of sequence b for the query heads h0 (and h0 + 1)
   const int total = a.cu_tiles[a.B];
-  bool active = (int)blockIdx.x < total;
+  const bool active = (int)blockIdx.x < total;
   int b = 0, qt = 0;
   if (active) {
     const int t = total - 1 - (int)blockIdx.x;   // a sequence's last (heaviest) tiles first
@@ -254,78 +281,103 @@ __global__ void __launch_bounds__(kPfThreads, 1)
   }
   const int s0 = active ? a.cu[b] : 0, len = active ? a.cu[b + 1] - s0 : 0;
   const int q0 = qt * kPfRows;
-  const int h = blockIdx.y, g = h / a.G;
+  const int pairs = (a.G + 1) >> 1;                        // head pairs per KV head
+  const int g = (int)blockIdx.y / pairs, pr = (int)blockIdx.y % pairs;
+  const int h0 = g * a.G + 2 * pr;
+  const int nh = min(2, a.G - 2 * pr);                     // query heads of this CTA (1 or 2)
   const int n_kv = active ? (min(q0 + kPfRows, len) + kPfKeys - 1) / kPfKeys : 0;   // causal key tiles
   const int kbase = active ? a.pcu[b] : 0;
 
   if (warp == 0) {
     if (lane == 0 && n_kv > 0) {
       const uint64_t pol_q = policy_evict_first(), pol_kv = policy_evict_last();
-      mbar_arrive_expect_tx(&q_full, L::kQ);
-#pragma unroll
-      for (int d = 0; d < DA; ++d) tma_load_3d(smem + d * (kPfRows * 128), &q_map, &q_full, d * 64, h, s0 + q0, pol_q);
-      int j = 0;
-      for (; j < n_kv; ++j) {
-        const int s = j % kPfStages;
-        if (!mbar_wait(&kv_empty[s], ((j / kPfStages) & 1) ^ 1)) {
-          set_error(a.status, UMIM_ERR_TIMEOUT);
-          break;
-        }
-        uint8_t *st = smem + L::kStages + s * L::kStage;
-        mbar_arrive_expect_tx(&kv_full[s], L::kStage);
+      mbar_arrive_expect_tx(&q_full, nh * L::kQ);
+      for (int x = 0; x < nh; ++x)
 #pragma unroll
         for (int d = 0; d < DA; ++d)
-          tma_load_3d(st + d * (kPfKeys * 128), &k_map, &kv_full[s], d * 64, g, s0 + j * kPfKeys, pol_kv);
-        tma_load_3d(st + L::kK, &vt_map, &kv_full[s], kbase + j * kPfKeys, 0, g, pol_kv);
+          tma_load_3d(smem + x * L::kQ + d * (kPfRows * 128), &q_map, &q_full, d * 64, h0 + x, s0 + q0, pol_q);
+      int jk = 0, jv = 0;
+      bool ok = true;
+      for (int j = 0; j < n_kv && ok; ++j) {
+        const int s = j % kPfStages;
+        const uint32_t ph = ((j / kPfStages) & 1) ^ 1;
+        if (!mbar_wait(&k_empty[s], ph)) {
+          ok = false;
+          break;
+        }
+        mbar_arrive_expect_tx(&k_full[s], L::kK);
+#pragma unroll
+        for (int d = 0; d < DA; ++d)
+          tma_load_3d(smem + L::kKoff + s * L::kK + d * (kPfKeys * 128), &k_map, &k_full[s], d * 64, g,
+                      s0 + j * kPfKeys, pol_kv);
+        jk = j + 1;
+        if (!mbar_wait(&v_empty[s], ph)) {
+          ok = false;
+          break;
+        }
+        mbar_arrive_expect_tx(&v_full[s], L::kV);
+        tma_load_3d(smem + L::kVoff + s * L::kV, &vt_map, &v_full[s], kbase + j * kPfKeys, 0, g, pol_kv);
+        jv = j + 1;
       }
+      if (!ok) set_error(a.status, UMIM_ERR_TIMEOUT);
       // copies still in flight when a consumer gave up: wait for them (bounded)
-      for (int i = max(0, j - kPfStages); i < j; ++i)
-        mbar_wait_for(&kv_full[i % kPfStages], (i / kPfStages) & 1, kWaitLimitNs);
+      for (int i = max(0, jk - kPfStages); i < jk; ++i)
+        mbar_wait_for(&k_full[i % kPfStages], (i / kPfStages) & 1, kWaitLimitNs);
+      for (int i = max(0, jv - kPfStages); i < jv; ++i)
+        mbar_wait_for(&v_full[i % kPfStages], (i / kPfStages) & 1, kWaitLimitNs);
       mbar_wait_for(&q_full, 0, kWaitLimitNs);
     }
   } else if (warp == 1) {
     if (lane == 0 && n_kv > 0) {
       constexpr uint32_t idesc_s = idesc_f32acc(kPfRows, kPfKeys, false);
       constexpr uint32_t idesc_o = idesc_f32acc(kPfRows, D, false);
-      const uint32_t q_base = smem_u32(smem);
-      const uint32_t o_tmem = tmem + 128;
       bool ok = mbar_wait(&q_full, 0);
       tc_fence_after();
-      // O += P_i V_i for key tile i (high part, then remainder)
+      // O_x += P_x(i) V(i) for both heads (high part, then remainder); frees V(i)
       auto pv = [&](int i) {
-        const int pb = i & 1;
-        if (!mbar_wait(&p_full[pb], (i >> 1) & 1)) return false;
-        if (!mbar_wait(&kv_full[i % kPfStages], (i / kPfStages) & 1)) return false;
-        tc_fence_after();
-        const uint32_t v_base = smem_u32(smem + L::kStages + (i % kPfStages) * L::kStage + L::kK);
+        const int s = i % kPfStages;
+        if (!mbar_wait(&v_full[s], (i / kPfStages) & 1)) return false;
+        const uint32_t v_base = smem_u32(smem + L::kVoff + s * L::kV);
+        for (int x = 0; x < nh; ++x) {
+          if (!mbar_wait(&p_full[x], i & 1)) return false;
+          tc_fence_after();
 #pragma unroll
-        for (int part = 0; part < 2; ++part) {
-          const uint32_t p_base = smem_u32(smem + L::kPbuf + (pb * 2 + part) * L::kP);
+          for (int part = 0; part < 2; ++part) {
+            const uint32_t p_base = smem_u32(smem + L::kPoff + (x * 2 + part) * L::kP);
 #pragma unroll
-          for (int kk = 0; kk < kPfKeys / 16; ++kk)
-            tc_mma_bf16(o_tmem, sw128_kmajor_desc(p_base + kk * 32), sw128_kmajor_desc(v_base + kk * 32), idesc_o,
-                        (i | part | kk) != 0 ? 1u : 0u);
+            for (int kk = 0; kk < kPfKeys / 16; ++kk)
+              tc_mma_bf16(tmem + x * 256 + 128, sw128_kmajor_desc(p_base + kk * 32),
+                          sw128_kmajor_desc(v_base + kk * 32), idesc_o, (i | part | kk) != 0 ? 1u : 0u);
+          }
+          tc_commit(&p_empty[x]);
         }
-        tc_commit(&p_empty[pb]);
-        tc_commit(&kv_empty[i % kPfStages]);
+        tc_commit(&v_empty[s]);
         return true;
       };
       for (int j = 0; j < n_kv && ok; ++j) {
         const int s = j % kPfStages, sb = j & 1;
-        if (!mbar_wait(&kv_full[s], (j / kPfStages) & 1) || !mbar_wait(&s_empty[sb], ((j >> 1) & 1) ^ 1)) {
+        if (!mbar_wait(&k_full[s], (j / kPfStages) & 1)) {
           ok = false;
           break;
         }
-        tc_fence_after();
-        const uint32_t k_base = smem_u32(smem + L::kStages + s * L::kStage);
+        const uint32_t k_base = smem_u32(smem + L::kKoff + s * L::kK);
+        for (int x = 0; x < nh && ok; ++x) {
+          if (!mbar_wait(&s_empty[x][sb], ((j >> 1) & 1) ^ 1)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t q_base = smem_u32(smem + x * L::kQ);
 #pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) {
-          const uint32_t off = (kk & 3) * 32;
-          const uint64_t ad = sw128_kmajor_desc(q_base + (kk >> 2) * (kPfRows * 128) + off);
-          const uint64_t bd = sw128_kmajor_desc(k_base + (kk >> 2) * (kPfKeys * 128) + off);
-          tc_mma_bf16(tmem + sb * kPfKeys, ad, bd, idesc_s, kk != 0 ? 1u : 0u);
+          for (int kk = 0; kk < D / 16; ++kk) {
+            const uint32_t off = (kk & 3) * 32;
+            tc_mma_bf16(tmem + x * 256 + sb * kPfKeys, sw128_kmajor_desc(q_base + (kk >> 2) * (kPfRows * 128) + off),
+                        sw128_kmajor_desc(k_base + (kk >> 2) * (kPfKeys * 128) + off), idesc_s, kk != 0 ? 1u : 0u);
+          }
+          tc_commit(&s_full[x][sb]);
         }
-        tc_commit(&s_full[sb]);
+        if (!ok) break;
+        tc_commit(&k_empty[s]);
         if (j >= 1 && !pv(j - 1)) ok = false;
       }
       if (ok && !pv(n_kv - 1)) ok = false;
@@ -334,86 +386,84 @@ __global__ void __launch_bounds__(kPfThreads, 1)
       tc_commit(&mma_done);
       mbar_wait_for(&mma_done, 0, kWaitLimitNs);
     }
-  } else {
-    // ---- softmax and epilogue: warps 2-5, thread = query row ----
+  } else if ((warp - 2) / 4 < nh) {
+    // ---- softmax and epilogue of head x: four warps, thread = query row ----
+    const int x = (warp - 2) >> 2;
     const int quad = warp & 3;                 // tensor-memory lanes this warp may access
     const int r = quad * 32 + lane;            // query row within the tile
     const int qpos = q0 + r;                   // position within the sequence
-    const int kmax = min(qpos, len - 1);       // last key this row sees (< 0: a row past the sequence)
-    const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
+    const int kmax = min(qpos, len - 1);       // last key this row sees
+    const uint32_t t_s = tmem + ((uint32_t)(quad * 32) << 16) + x * 256;   // this row's S buffers
+    const uint32_t t_o = t_s + 128;                                         // and O
     const float sl2 = a.scale_log2;
     float m_run = -INFINITY, l_run = 0.f;      // running max (log2 units, moved in steps > 8) and row sum
     bool ok = true;
     // every lane waits (each needs the acquire), the warp goes on only if all saw the phase:
     // the .sync.aligned tensor-memory instructions below need the whole warp
     auto wwait = [&](uint64_t *m, uint32_t parity) { return __all_sync(0xffffffffu, mbar_wait(m, parity)) != 0; };
+    uint8_t *ph = smem + L::kPoff + (x * 2) * L::kP + r * 128;
+    uint8_t *pl = ph + L::kP;
     for (int j = 0; j < n_kv && ok; ++j) {
       const int sb = j & 1;
-      if (!wwait(&s_full[sb], (j >> 1) & 1)) {
+      if (!wwait(&s_full[x][sb], (j >> 1) & 1)) {
         ok = false;
         break;
       }
       tc_fence_after();
-      float x[kPfKeys];
-      tmem_ld_32x32b_x32(tmem + lane_addr + sb * kPfKeys, *reinterpret_cast<float(*)[32]>(x));
-      tmem_ld_32x32b_x32(tmem + lane_addr + sb * kPfKeys + 32, *reinterpret_cast<float(*)[32]>(x + 32));
+      float s[kPfKeys];
+      tmem_ld_32x32b_x64(t_s + sb * kPfKeys, s);
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&s_empty[sb]);   // the S buffer may be overwritten
+      if (lane == 0) mbar_arrive(&s_empty[x][sb]);   // the S buffer may be overwritten
       const int k0 = j * kPfKeys;
-      float mx = -INFINITY;
+      if (k0 + kPfKeys - 1 > kmax) {   // the diagonal tile (or a row past the sequence)
 #pragma unroll
-      for (int c = 0; c < kPfKeys; ++c) {
-        x[c] = (k0 + c <= kmax) ? x[c] * sl2 : -INFINITY;
-        mx = fmaxf(mx, x[c]);
+        for (int c = 0; c < kPfKeys; ++c) s[c] = (k0 + c <= kmax) ? s[c] : -INFINITY;
       }
+      float m4[4] = {s[0], s[1], s[2], s[3]};
+#pragma unroll
+      for (int c = 4; c < kPfKeys; ++c) m4[c & 3] = fmaxf(m4[c & 3], s[c]);
+      const float mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])) * sl2;
       // move the running max only when it grows by more than 2^8
       const bool grow = mx > m_run + 8.f;
       float alpha = 1.f;
       if (grow) {
-        alpha = (m_run == -INFINITY) ? 0.f : exp2f(m_run - mx);
+        alpha = (m_run == -INFINITY) ? 0.f : ex2_approx(m_run - mx);
         m_run = mx;
         l_run *= alpha;
       }
-      if (j > 0 && __any_sync(0xffffffffu, grow && alpha != 1.f)) {
-        // rescale this warp's rows of O once the product of tile j - 1 has landed
-        if (!wwait(&p_empty[(j - 1) & 1], ((j - 1) >> 1) & 1)) {
-          ok = false;
-          break;
-        }
+      const float nm = (m_run == -INFINITY) ? 0.f : -m_run;
+      float l4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int c = 0; c < kPfKeys; ++c) {
+        s[c] = ex2_approx(fmaf(s[c], sl2, nm));   // masked (-inf): 0
+        l4[c & 3] += s[c];
+      }
+      l_run += (l4[0] + l4[1]) + (l4[2] + l4[3]);
+      // P(j) goes where P(j - 1) was, and O may be rescaled: the product of
+      // tile j - 1 must have landed (waited for only now, after the exponentials)
+      if (j >= 1 && !wwait(&p_empty[x], (j - 1) & 1)) {
+        ok = false;
+        break;
+      }
+      if (j > 0 && __any_sync(0xffffffffu, grow)) {
         tc_fence_after();
 #pragma unroll 1
         for (int c = 0; c < D / 32; ++c) {
           float o[32];
-          tmem_ld_32x32b_x32(tmem + lane_addr + 128 + c * 32, o);
+          tmem_ld_32x32b_x32(t_o + c * 32, o);
 #pragma unroll
           for (int i = 0; i < 32; ++i) o[i] *= alpha;
-          tmem_st_32x32b_x32(tmem + lane_addr + 128 + c * 32, o);
+          tmem_st_32x32b_x32(t_o + c * 32, o);
         }
         tc_fence_before();
       }
-      const float mb = (m_run == -INFINITY) ? 0.f : m_run;
-      float sum = 0.f;
-#pragma unroll
-      for (int c = 0; c < kPfKeys; ++c) {
-        x[c] = exp2f(x[c] - mb);   // masked: 0
-        sum += x[c];
-      }
-      l_run += sum;
-      // P of tile j into buffer j & 1 once the product of tile j - 2 has read it
-      const int pb = j & 1;
-      if (j >= 2 && !wwait(&p_empty[pb], ((j >> 1) & 1) ^ 1)) {
-        ok = false;
-        break;
-      }
-      uint8_t *ph = smem + L::kPbuf + (pb * 2) * L::kP + r * 128;
-      uint8_t *pl = ph + L::kP;
 #pragma unroll
       for (int c = 0; c < kPfKeys / 8; ++c) {
         uint32_t hw[4], lw[4];
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
-          const float p0 = x[8 * c + 2 * e], p1 = x[8 * c + 2 * e + 1];
+          const float p0 = s[8 * c + 2 * e], p1 = s[8 * c + 2 * e + 1];
           const __nv_bfloat162 hh = __floats2bfloat162_rn(p0, p1);
           hw[e] = *reinterpret_cast<const uint32_t *>(&hh);
           lw[e] = pack_bf16x2(p0 - __low2float(hh), p1 - __high2float(hh));
@@ -424,18 +474,18 @@ __global__ void __launch_bounds__(kPfThreads, 1)
       }
       fence_proxy_async_smem();   // visible to the tensor cores
       __syncwarp();
-      if (lane == 0) mbar_arrive(&p_full[pb]);
+      if (lane == 0) mbar_arrive(&p_full[x]);
     }
     if (!ok) set_error(a.status, UMIM_ERR_TIMEOUT);
     // epilogue: O / l once the last product has landed
-    if (ok && n_kv > 0 && wwait(&p_empty[(n_kv - 1) & 1], ((n_kv - 1) >> 1) & 1)) {
+    if (ok && n_kv > 0 && wwait(&p_empty[x], (n_kv - 1) & 1)) {
       tc_fence_after();
       const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
-      __nv_bfloat16 *orow = a.out + (((int64_t)s0 + qpos) * a.Hq + h) * D;
+      __nv_bfloat16 *orow = a.out + (((int64_t)s0 + qpos) * a.Hq + h0 + x) * D;
 #pragma unroll 1
       for (int c = 0; c < D / 32; ++c) {
         float o[32];
-        tmem_ld_32x32b_x32(tmem + lane_addr + 128 + c * 32, o);
+        tmem_ld_32x32b_x32(t_o + c * 32, o);
         if (qpos < len) {
           uint4 *dst = reinterpret_cast<uint4 *>(orow + c * 32);
 #pragma unroll
@@ -520,7 +570,8 @@ umim_status prefill_attention(const void *q, const void *k, const void *v, int T
   // an upper bound of the query tiles: each sequence wastes less than one
   const unsigned gx = (unsigned)((T + kPfRows - 1) / kPfRows + B);
   trace_mark(stream, "prefill.attention");
-  if (launch_pdl(kern, dim3(gx, (unsigned)Hq), dim3(kPfThreads), smem, stream, qm, km, vm, a) != cudaSuccess)
+  const unsigned gy = (unsigned)(Hkv * ((a.G + 1) / 2));   // query-head pairs sharing a KV head
+  if (launch_pdl(kern, dim3(gx, gy), dim3(kPfThreads), smem, stream, qm, km, vm, a) != cudaSuccess)
     return UMIM_ERR_CUDA;
   trace_mark(stream, nullptr);
   return UMIM_OK;
