@@ -5,23 +5,29 @@
 // cu_seqlens[b] .. cu_seqlens[b+1]-1 of q [T][Hq][D], k, v [T][Hkv][D].
 //
 // On the 5th-generation tensor cores: one CTA takes 128 query rows of one
-// sequence and one query head.  Warp 0 loads tiles with TMA (Q once; K and
-// V^T tiles of 64 keys into a 3-stage ring), warp 1 issues tcgen05.mma
-// (S = Q K^T into one of two tensor-memory buffers, then O += P V into a
-// tensor-memory accumulator), warps 2-9 run the online softmax, two warps
-// per 32 query rows (32 of a tile's 64 keys each): S from tensor memory (tcgen05.ld), causal mask, running max,
-// P = exp2(S - max) written to shared memory as a bf16 high part and a bf16
-// remainder (two MMAs per P V product keep P's rounding out of the error
-// budget), row sums.  The running max is only moved when it grows by more
-// than 2^8, so the accumulator in tensor memory is rescaled rarely (the
-// result is the same: P and the row sum use the same stale max).  The S MMA
-// of the next tile runs while the softmax works on the current one.
+// sequence for two query heads that share a KV head (one when the group has
+// an odd head left over), so every K and V tile serves both.  Warp 0 loads
+// tiles with TMA (Q once; 64-key K tiles into a 3-stage ring running two
+// tiles ahead of the V^T tiles' 2-stage ring), warp 1 issues tcgen05.mma
+// (per head, S = Q K^T into one of two tensor-memory buffers and O += P V into
+// a tensor-memory accumulator), and warps 2-5 / 6-9 run the online softmax of
+// head 0 / 1, one thread per query row: S from tensor memory (tcgen05.ld),
+// causal mask, running max, P = exp2(S - max) written to shared memory in
+// fp16, row sums.  P V runs on fp16 operands (V^T is converted when it is
+// transposed): fp16's 11-bit significand keeps P's and V's rounding near
+// 3e-4 relative, where bf16 P would cost 1e-3 of the output's error budget;
+// P <= 2^8 by construction and |v| < 65504 is checked (UMIM_ERR_UNSUPPORTED
+// otherwise).  One head's softmax overlaps the other head's products.  The running max is only moved when it grows by
+// more than 2^8, so the accumulator in tensor memory is rescaled rarely (the
+// result is the same: P and the row sum use the same stale max).
 //
 // V is transposed first (per sequence, padded to a multiple of 64 keys) so
 // that both products read K-major operands and every TMA copy starts on a
 // 16-byte boundary.  A plan kernel turns cu_seqlens into per-sequence tile
 // offsets and padded key offsets (and validates them); tiles run heaviest
 // (last in their sequence) first.
+#include <cuda_fp16.h>
+
 #include "common.cuh"
 
 namespace umim {
@@ -36,7 +42,8 @@ namespace {
 
 constexpr int kPfRows = 128;             // query rows per CTA (the MMA's M)
 constexpr int kPfKeys = 64;              // keys per K / V tile (the S MMA's N)
-constexpr int kPfStages = 2;             // K and V^T rings
+constexpr int kPfKStages = 3;            // K ring (K runs kPfKStages - 1 tiles ahead of V^T)
+constexpr int kPfVStages = 2;            // V^T ring
 constexpr int kPfThreads = 320;          // warp 0 TMA, warp 1 MMA + tensor memory, warps 2-5 / 6-9 softmax of head 0 / 1
 constexpr int kPfPlanThreads = 1024;
 constexpr uint32_t kPfTmemCols = 512;    // per head x: S buffers at 256x + 0 and + 64, O at 256x + 128
@@ -47,7 +54,7 @@ struct PfArgs {
   int32_t *cu_tiles;                // [B + 1] workspace: query-tile offsets
   int32_t *pcu;                     // [B + 1] workspace: key offsets padded to 64 in V^T
   const __nv_bfloat16 *v;           // [T][Hkv][D]
-  __nv_bfloat16 *vt;                // [Hkv][D][Tp] workspace
+  __half *vt;                       // [Hkv][D][Tp] workspace, fp16
   int64_t Tp;                       // row length of V^T (a multiple of 64)
   int32_t B, T, Hq, Hkv, G;
   float scale_log2;
@@ -146,19 +153,23 @@ __global__ void __launch_bounds__(256) vt_kernel(PfArgs a) {
     tile[r][4 * c + 3] = u.w;
   }
   __syncthreads();
-  // each thread writes 8 keys of one d row (16 bytes)
+  // each thread writes 8 keys of one d row (16 bytes), converted to fp16
+  bool too_big = false;
   for (int i = threadIdx.x; i < D * (kPfKeys / 8); i += blockDim.x) {
     const int d = i / (kPfKeys / 8), c = i % (kPfKeys / 8);
     uint32_t w[4];
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
       const uint32_t x0 = tile[8 * c + 2 * j][d >> 1], x1 = tile[8 * c + 2 * j + 1][d >> 1];
-      const uint32_t lo = (d & 1) ? (x0 >> 16) : (x0 & 0xffffu);
-      const uint32_t hi = (d & 1) ? (x1 >> 16) : (x1 & 0xffffu);
-      w[j] = lo | (hi << 16);
+      const float f0 = __uint_as_float((d & 1) ? (x0 & 0xffff0000u) : (x0 << 16));
+      const float f1 = __uint_as_float((d & 1) ? (x1 & 0xffff0000u) : (x1 << 16));
+      too_big |= !(fabsf(f0) < 65504.f) || !(fabsf(f1) < 65504.f);
+      const __half2 hh = __floats2half2_rn(f0, f1);
+      w[j] = *reinterpret_cast<const uint32_t *>(&hh);
     }
     *reinterpret_cast<uint4 *>(a.vt + ((int64_t)g * D + d) * a.Tp + k0 + 8 * c) = make_uint4(w[0], w[1], w[2], w[3]);
   }
+  if (too_big) set_error(a.status, UMIM_ERR_UNSUPPORTED);   // |v| outside fp16's range (or not finite)
 }
 
 __device__ __forceinline__ void tma_load_3d(void *dst, const CUtensorMap *map, uint64_t *bar, int c0, int c1, int c2,
@@ -218,11 +229,11 @@ struct PfSmem {
   static constexpr int kQ = kPfRows * D * 2;              // Q of one head: D/64 atoms of [128 rows][128 B]
   static constexpr int kK = kPfKeys * D * 2;              // K tile: D/64 atoms of [64 keys][128 B]
   static constexpr int kV = D * kPfKeys * 2;              // V^T tile: [D rows][128 B]
-  static constexpr int kP = kPfRows * kPfKeys * 2;        // one P part of one head: [128 rows][128 B]
+  static constexpr int kP = kPfRows * kPfKeys * 2;        // P of one head, fp16: [128 rows][128 B]
   static constexpr int kKoff = 2 * kQ;
-  static constexpr int kVoff = kKoff + kPfStages * kK;
-  static constexpr int kPoff = kVoff + kPfStages * kV;
-  static constexpr int kTotal = kPoff + 2 * 2 * kP;       // [head][high, remainder]
+  static constexpr int kVoff = kKoff + kPfKStages * kK;
+  static constexpr int kPoff = kVoff + kPfVStages * kV;
+  static constexpr int kTotal = kPoff + 2 * kP;           // [head]
 };
 
 template <int D>
@@ -232,17 +243,19 @@ __global__ void __launch_bounds__(kPfThreads, 1)
   using L = PfSmem<D>;
   constexpr int DA = D / 64;   // 64-wide atoms along the head dimension
   extern __shared__ __align__(1024) uint8_t pf_raw[];
-  __shared__ __align__(8) uint64_t q_full, k_full[kPfStages], k_empty[kPfStages], v_full[kPfStages],
-      v_empty[kPfStages], s_full[2][2], s_empty[2][2], p_full[2], p_empty[2], mma_done;
+  __shared__ __align__(8) uint64_t q_full, k_full[kPfKStages], k_empty[kPfKStages], v_full[kPfVStages],
+      v_empty[kPfVStages], s_full[2][2], s_empty[2][2], p_full[2], p_empty[2], mma_done;
   __shared__ uint32_t tmem_base;
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(pf_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) {
     mbar_init(&q_full, 1);
-    for (int s = 0; s < kPfStages; ++s) {
+    for (int s = 0; s < kPfKStages; ++s) {
       mbar_init(&k_full[s], 1);
       mbar_init(&k_empty[s], 1);
+    }
+    for (int s = 0; s < kPfVStages; ++s) {
       mbar_init(&v_full[s], 1);
       mbar_init(&v_empty[s], 1);
     }
@@ -296,67 +309,72 @@ __global__ void __launch_bounds__(kPfThreads, 1)
 #pragma unroll
         for (int d = 0; d < DA; ++d)
           tma_load_3d(smem + x * L::kQ + d * (kPfRows * 128), &q_map, &q_full, d * 64, h0 + x, s0 + q0, pol_q);
+      // K runs kPfKStages - 1 tiles ahead of V^T: a K load never waits behind
+      // the P V product that frees a V^T stage
+      constexpr int kLead = kPfKStages - 1;
       int jk = 0, jv = 0;
       bool ok = true;
-      for (int j = 0; j < n_kv && ok; ++j) {
-        const int s = j % kPfStages;
-        const uint32_t ph = ((j / kPfStages) & 1) ^ 1;
-        if (!mbar_wait(&k_empty[s], ph)) {
-          ok = false;
-          break;
-        }
-        mbar_arrive_expect_tx(&k_full[s], L::kK);
+      for (int i = 0; i < n_kv + kLead && ok; ++i) {
+        if (i < n_kv) {
+          const int s = i % kPfKStages;
+          if (!mbar_wait(&k_empty[s], ((i / kPfKStages) & 1) ^ 1)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(&k_full[s], L::kK);
 #pragma unroll
-        for (int d = 0; d < DA; ++d)
-          tma_load_3d(smem + L::kKoff + s * L::kK + d * (kPfKeys * 128), &k_map, &k_full[s], d * 64, g,
-                      s0 + j * kPfKeys, pol_kv);
-        jk = j + 1;
-        if (!mbar_wait(&v_empty[s], ph)) {
-          ok = false;
-          break;
+          for (int d = 0; d < DA; ++d)
+            tma_load_3d(smem + L::kKoff + s * L::kK + d * (kPfKeys * 128), &k_map, &k_full[s], d * 64, g,
+                        s0 + i * kPfKeys, pol_kv);
+          jk = i + 1;
         }
-        mbar_arrive_expect_tx(&v_full[s], L::kV);
-        tma_load_3d(smem + L::kVoff + s * L::kV, &vt_map, &v_full[s], kbase + j * kPfKeys, 0, g, pol_kv);
-        jv = j + 1;
+        const int j = i - kLead;
+        if (j >= 0 && j < n_kv) {
+          const int s = j % kPfVStages;
+          if (!mbar_wait(&v_empty[s], ((j / kPfVStages) & 1) ^ 1)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(&v_full[s], L::kV);
+          tma_load_3d(smem + L::kVoff + s * L::kV, &vt_map, &v_full[s], kbase + j * kPfKeys, 0, g, pol_kv);
+          jv = j + 1;
+        }
       }
       if (!ok) set_error(a.status, UMIM_ERR_TIMEOUT);
       // copies still in flight when a consumer gave up: wait for them (bounded)
-      for (int i = max(0, jk - kPfStages); i < jk; ++i)
-        mbar_wait_for(&k_full[i % kPfStages], (i / kPfStages) & 1, kWaitLimitNs);
-      for (int i = max(0, jv - kPfStages); i < jv; ++i)
-        mbar_wait_for(&v_full[i % kPfStages], (i / kPfStages) & 1, kWaitLimitNs);
+      for (int i = max(0, jk - kPfKStages); i < jk; ++i)
+        mbar_wait_for(&k_full[i % kPfKStages], (i / kPfKStages) & 1, kWaitLimitNs);
+      for (int i = max(0, jv - kPfVStages); i < jv; ++i)
+        mbar_wait_for(&v_full[i % kPfVStages], (i / kPfVStages) & 1, kWaitLimitNs);
       mbar_wait_for(&q_full, 0, kWaitLimitNs);
     }
   } else if (warp == 1) {
     if (lane == 0 && n_kv > 0) {
       constexpr uint32_t idesc_s = idesc_f32acc(kPfRows, kPfKeys, false);
-      constexpr uint32_t idesc_o = idesc_f32acc(kPfRows, D, false);
+      constexpr uint32_t idesc_o = idesc_f32acc(kPfRows, D, true);   // P and V^T in fp16
       bool ok = mbar_wait(&q_full, 0);
       tc_fence_after();
-      // O_x += P_x(i) V(i) for both heads (high part, then remainder); frees V(i)
+      // O_x += P_x(i) V(i) for both heads (fp16 operands); frees V(i)
       auto pv = [&](int i) {
-        const int s = i % kPfStages;
-        if (!mbar_wait(&v_full[s], (i / kPfStages) & 1)) return false;
+        const int s = i % kPfVStages;
+        if (!mbar_wait(&v_full[s], (i / kPfVStages) & 1)) return false;
         const uint32_t v_base = smem_u32(smem + L::kVoff + s * L::kV);
         for (int x = 0; x < nh; ++x) {
           if (!mbar_wait(&p_full[x], i & 1)) return false;
           tc_fence_after();
+          const uint32_t p_base = smem_u32(smem + L::kPoff + x * L::kP);
 #pragma unroll
-          for (int part = 0; part < 2; ++part) {
-            const uint32_t p_base = smem_u32(smem + L::kPoff + (x * 2 + part) * L::kP);
-#pragma unroll
-            for (int kk = 0; kk < kPfKeys / 16; ++kk)
-              tc_mma_bf16(tmem + x * 256 + 128, sw128_kmajor_desc(p_base + kk * 32),
-                          sw128_kmajor_desc(v_base + kk * 32), idesc_o, (i | part | kk) != 0 ? 1u : 0u);
-          }
+          for (int kk = 0; kk < kPfKeys / 16; ++kk)
+            tc_mma_bf16(tmem + x * 256 + 128, sw128_kmajor_desc(p_base + kk * 32), sw128_kmajor_desc(v_base + kk * 32),
+                        idesc_o, (i | kk) != 0 ? 1u : 0u);
           tc_commit(&p_empty[x]);
         }
         tc_commit(&v_empty[s]);
         return true;
       };
       for (int j = 0; j < n_kv && ok; ++j) {
-        const int s = j % kPfStages, sb = j & 1;
-        if (!mbar_wait(&k_full[s], (j / kPfStages) & 1)) {
+        const int s = j % kPfKStages, sb = j & 1;
+        if (!mbar_wait(&k_full[s], (j / kPfKStages) & 1)) {
           ok = false;
           break;
         }
@@ -401,8 +419,7 @@ __global__ void __launch_bounds__(kPfThreads, 1)
     // every lane waits (each needs the acquire), the warp goes on only if all saw the phase:
     // the .sync.aligned tensor-memory instructions below need the whole warp
     auto wwait = [&](uint64_t *m, uint32_t parity) { return __all_sync(0xffffffffu, mbar_wait(m, parity)) != 0; };
-    uint8_t *ph = smem + L::kPoff + (x * 2) * L::kP + r * 128;
-    uint8_t *pl = ph + L::kP;
+    uint8_t *prow = smem + L::kPoff + x * L::kP + r * 128;
     for (int j = 0; j < n_kv && ok; ++j) {
       const int sb = j & 1;
       if (!wwait(&s_full[x][sb], (j >> 1) & 1)) {
@@ -460,17 +477,14 @@ __global__ void __launch_bounds__(kPfThreads, 1)
       }
 #pragma unroll
       for (int c = 0; c < kPfKeys / 8; ++c) {
-        uint32_t hw[4], lw[4];
+        uint32_t hw[4];
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
-          const float p0 = s[8 * c + 2 * e], p1 = s[8 * c + 2 * e + 1];
-          const __nv_bfloat162 hh = __floats2bfloat162_rn(p0, p1);
+          const __half2 hh = __floats2half2_rn(s[8 * c + 2 * e], s[8 * c + 2 * e + 1]);   // P <= 2^8
           hw[e] = *reinterpret_cast<const uint32_t *>(&hh);
-          lw[e] = pack_bf16x2(p0 - __low2float(hh), p1 - __high2float(hh));
         }
         const int pos = (c ^ (r & 7)) << 4;   // 128-byte swizzle of a K-major operand
-        *reinterpret_cast<uint4 *>(ph + pos) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
-        *reinterpret_cast<uint4 *>(pl + pos) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+        *reinterpret_cast<uint4 *>(prow + pos) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
       }
       fence_proxy_async_smem();   // visible to the tensor cores
       __syncwarp();
@@ -509,12 +523,13 @@ __global__ void __launch_bounds__(kPfThreads, 1)
 }
 
 bool encode_3d(EncodeTiledFn enc, CUtensorMap *map, const void *base, uint64_t d0, uint64_t d1, uint64_t d2,
-               uint64_t stride1, uint64_t stride2, uint32_t b0, uint32_t b1, uint32_t b2) {
+               uint64_t stride1, uint64_t stride2, uint32_t b0, uint32_t b1, uint32_t b2, bool fp16 = false) {
   const cuuint64_t dims[3] = {d0, d1, d2};
   const cuuint64_t strides[2] = {stride1, stride2};
   const cuuint32_t box[3] = {b0, b1, b2};
   const cuuint32_t es[3] = {1, 1, 1};
-  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims, strides, box, es,
+  return enc(map, fp16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3,
+             const_cast<void *>(base), dims, strides, box, es,
              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
@@ -541,7 +556,7 @@ umim_status prefill_attention(const void *q, const void *k, const void *v, int T
   a.cu_tiles = static_cast<int32_t *>(ws);
   a.pcu = a.cu_tiles + (B + 1);
   a.v = static_cast<const __nv_bfloat16 *>(v);
-  a.vt = reinterpret_cast<__nv_bfloat16 *>(static_cast<char *>(ws) +
+  a.vt = reinterpret_cast<__half *>(static_cast<char *>(ws) +
                                            (((size_t)2 * (B + 1) * sizeof(int32_t) + 1023) & ~size_t(1023)));
   a.Tp = vt_row(B, T);
   a.B = B;
@@ -554,7 +569,7 @@ umim_status prefill_attention(const void *q, const void *k, const void *v, int T
   CUtensorMap qm, km, vm;
   if (!encode_3d(enc, &qm, q, D, Hq, T, (uint64_t)D * 2, (uint64_t)Hq * D * 2, 64, 1, kPfRows) ||
       !encode_3d(enc, &km, k, D, Hkv, T, (uint64_t)D * 2, (uint64_t)Hkv * D * 2, 64, 1, kPfKeys) ||
-      !encode_3d(enc, &vm, a.vt, a.Tp, D, Hkv, (uint64_t)a.Tp * 2, (uint64_t)D * a.Tp * 2, kPfKeys, D, 1))
+      !encode_3d(enc, &vm, a.vt, a.Tp, D, Hkv, (uint64_t)a.Tp * 2, (uint64_t)D * a.Tp * 2, kPfKeys, D, 1, true))
     return UMIM_ERR_CUDA;
   trace_mark(stream, "prefill.plan");
   if (launch_pdl(prefill_plan_kernel, dim3(1), dim3(kPfPlanThreads), 0, stream, a) != cudaSuccess)
