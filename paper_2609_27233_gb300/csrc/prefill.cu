@@ -10,10 +10,12 @@
 // tiles with TMA (Q once; 64-key K tiles into a 3-stage ring running two
 // tiles ahead of the V^T tiles' 2-stage ring), warp 1 issues tcgen05.mma
 // (per head, S = Q K^T into one of two tensor-memory buffers and O += P V into
-// a tensor-memory accumulator), and warps 2-5 / 6-9 run the online softmax of
+// a tensor-memory accumulator; an S buffer is reused once the P V product
+// that read it is done), and warps 2-5 / 6-9 run the online softmax of
 // head 0 / 1, one thread per query row: S from tensor memory (tcgen05.ld),
-// causal mask, running max, P = exp2(S - max) written to shared memory in
-// fp16, row sums.  P V runs on fp16 operands (V^T is converted when it is
+// causal mask, running max, P = exp2(S - max) written back in fp16 over the
+// S columns it came from (tcgen05.st; the P V product reads its A operand
+// from tensor memory, so P never touches shared memory), row sums.  P V runs on fp16 operands (V^T is converted when it is
 // transposed): fp16's 11-bit significand keeps P's and V's rounding near
 // 3e-4 relative, where bf16 P would cost 1e-3 of the output's error budget;
 // P <= 2^8 by construction and |v| < 65504 is checked (UMIM_ERR_UNSUPPORTED
@@ -223,17 +225,27 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return *reinterpret_cast<uint32_t *>(&p);
 }
 
+// D[tmem] (+)= A[tmem] * B[smem]^T (kind::f16): A's rows in the 128 lanes,
+// two 16-bit values of consecutive K per 32-bit column
+__device__ __forceinline__ void tc_mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
+                                          uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
 // shared-memory layout of the attention kernel (bytes, every piece 1024-aligned)
 template <int D>
 struct PfSmem {
   static constexpr int kQ = kPfRows * D * 2;              // Q of one head: D/64 atoms of [128 rows][128 B]
   static constexpr int kK = kPfKeys * D * 2;              // K tile: D/64 atoms of [64 keys][128 B]
   static constexpr int kV = D * kPfKeys * 2;              // V^T tile: [D rows][128 B]
-  static constexpr int kP = kPfRows * kPfKeys * 2;        // P of one head, fp16: [128 rows][128 B]
   static constexpr int kKoff = 2 * kQ;
   static constexpr int kVoff = kKoff + kPfKStages * kK;
-  static constexpr int kPoff = kVoff + kPfVStages * kV;
-  static constexpr int kTotal = kPoff + 2 * kP;           // [head]
+  static constexpr int kTotal = kVoff + kPfVStages * kV;
 };
 
 template <int D>
@@ -244,7 +256,7 @@ __global__ void __launch_bounds__(kPfThreads, 1)
   constexpr int DA = D / 64;   // 64-wide atoms along the head dimension
   extern __shared__ __align__(1024) uint8_t pf_raw[];
   __shared__ __align__(8) uint64_t q_full, k_full[kPfKStages], k_empty[kPfKStages], v_full[kPfVStages],
-      v_empty[kPfVStages], s_full[2][2], s_empty[2][2], p_full[2], p_empty[2], mma_done;
+      v_empty[kPfVStages], s_full[2][2], s_empty[2][2], p_full[2][2], p_empty[2], o_done[2], mma_done;
   __shared__ uint32_t tmem_base;
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(pf_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -262,10 +274,13 @@ __global__ void __launch_bounds__(kPfThreads, 1)
     for (int x = 0; x < 2; ++x) {
       for (int i = 0; i < 2; ++i) {
         mbar_init(&s_full[x][i], 1);
-        mbar_init(&s_empty[x][i], 4);   // one arrival per softmax warp of the head
+        mbar_init(&s_empty[x][i], 1);   // committed once the P V product that read P from it is done
       }
-      mbar_init(&p_full[x], 4);
+      // P(j) ready, by tile parity: the softmax can run a tile ahead of the MMA warp's wait
+      mbar_init(&p_full[x][0], 4);
+      mbar_init(&p_full[x][1], 4);
       mbar_init(&p_empty[x], 1);
+      mbar_init(&o_done[x], 1);   // one phase: every product of the CTA has landed
     }
     mbar_init(&mma_done, 1);
     fence_mbar_init();
@@ -354,20 +369,21 @@ __global__ void __launch_bounds__(kPfThreads, 1)
       constexpr uint32_t idesc_o = idesc_f32acc(kPfRows, D, true);   // P and V^T in fp16
       bool ok = mbar_wait(&q_full, 0);
       tc_fence_after();
-      // O_x += P_x(i) V(i) for both heads (fp16 operands); frees V(i)
+      // O_x += P_x(i) V(i) for both heads (fp16 operands, P from tensor memory); frees V(i) and S(i)'s buffer
       auto pv = [&](int i) {
         const int s = i % kPfVStages;
         if (!mbar_wait(&v_full[s], (i / kPfVStages) & 1)) return false;
         const uint32_t v_base = smem_u32(smem + L::kVoff + s * L::kV);
         for (int x = 0; x < nh; ++x) {
-          if (!mbar_wait(&p_full[x], i & 1)) return false;
+          if (!mbar_wait(&p_full[x][i & 1], (i >> 1) & 1)) return false;
           tc_fence_after();
-          const uint32_t p_base = smem_u32(smem + L::kPoff + x * L::kP);
+          const uint32_t p_tmem = tmem + x * 256 + (i & 1) * kPfKeys;   // P(i) sits where S(i) was
 #pragma unroll
           for (int kk = 0; kk < kPfKeys / 16; ++kk)
-            tc_mma_bf16(tmem + x * 256 + 128, sw128_kmajor_desc(p_base + kk * 32), sw128_kmajor_desc(v_base + kk * 32),
-                        idesc_o, (i | kk) != 0 ? 1u : 0u);
+            tc_mma_ts(tmem + x * 256 + 128, p_tmem + kk * 8, sw128_kmajor_desc(v_base + kk * 32), idesc_o,
+                      (i | kk) != 0 ? 1u : 0u);
           tc_commit(&p_empty[x]);
+          tc_commit(&s_empty[x][i & 1]);
         }
         tc_commit(&v_empty[s]);
         return true;
@@ -399,6 +415,8 @@ __global__ void __launch_bounds__(kPfThreads, 1)
         if (j >= 1 && !pv(j - 1)) ok = false;
       }
       if (ok && !pv(n_kv - 1)) ok = false;
+      if (ok)
+        for (int x = 0; x < nh; ++x) tc_commit(&o_done[x]);
       if (!ok) set_error(a.status, UMIM_ERR_TIMEOUT);
       // every MMA issued has finished before tensor memory is released
       tc_commit(&mma_done);
@@ -419,7 +437,6 @@ __global__ void __launch_bounds__(kPfThreads, 1)
     // every lane waits (each needs the acquire), the warp goes on only if all saw the phase:
     // the .sync.aligned tensor-memory instructions below need the whole warp
     auto wwait = [&](uint64_t *m, uint32_t parity) { return __all_sync(0xffffffffu, mbar_wait(m, parity)) != 0; };
-    uint8_t *prow = smem + L::kPoff + x * L::kP + r * 128;
     for (int j = 0; j < n_kv && ok; ++j) {
       const int sb = j & 1;
       if (!wwait(&s_full[x][sb], (j >> 1) & 1)) {
@@ -429,9 +446,6 @@ __global__ void __launch_bounds__(kPfThreads, 1)
       tc_fence_after();
       float s[kPfKeys];
       tmem_ld_32x32b_x64(t_s + sb * kPfKeys, s);
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&s_empty[x][sb]);   // the S buffer may be overwritten
       const int k0 = j * kPfKeys;
       if (k0 + kPfKeys - 1 > kmax) {   // the diagonal tile (or a row past the sequence)
 #pragma unroll
@@ -457,13 +471,12 @@ __global__ void __launch_bounds__(kPfThreads, 1)
         l4[c & 3] += s[c];
       }
       l_run += (l4[0] + l4[1]) + (l4[2] + l4[3]);
-      // P(j) goes where P(j - 1) was, and O may be rescaled: the product of
-      // tile j - 1 must have landed (waited for only now, after the exponentials)
-      if (j >= 1 && !wwait(&p_empty[x], (j - 1) & 1)) {
-        ok = false;
-        break;
-      }
+      // O is rescaled only once the product of tile j - 1 has landed
       if (j > 0 && __any_sync(0xffffffffu, grow)) {
+        if (!wwait(&p_empty[x], (j - 1) & 1)) {
+          ok = false;
+          break;
+        }
         tc_fence_after();
 #pragma unroll 1
         for (int c = 0; c < D / 32; ++c) {
@@ -475,24 +488,23 @@ __global__ void __launch_bounds__(kPfThreads, 1)
         }
         tc_fence_before();
       }
+      // P(j) in fp16 over S(j)'s columns (this thread has read them), for the P V product
+      {
+        float pk[32];
 #pragma unroll
-      for (int c = 0; c < kPfKeys / 8; ++c) {
-        uint32_t hw[4];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const __half2 hh = __floats2half2_rn(s[8 * c + 2 * e], s[8 * c + 2 * e + 1]);   // P <= 2^8
-          hw[e] = *reinterpret_cast<const uint32_t *>(&hh);
+        for (int c = 0; c < 32; ++c) {
+          const __half2 hh = __floats2half2_rn(s[2 * c], s[2 * c + 1]);   // P <= 2^8
+          pk[c] = __uint_as_float(*reinterpret_cast<const uint32_t *>(&hh));
         }
-        const int pos = (c ^ (r & 7)) << 4;   // 128-byte swizzle of a K-major operand
-        *reinterpret_cast<uint4 *>(prow + pos) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+        tmem_st_32x32b_x32(t_s + sb * kPfKeys, pk);
       }
-      fence_proxy_async_smem();   // visible to the tensor cores
+      tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&p_full[x]);
+      if (lane == 0) mbar_arrive(&p_full[x][sb]);
     }
     if (!ok) set_error(a.status, UMIM_ERR_TIMEOUT);
     // epilogue: O / l once the last product has landed
-    if (ok && n_kv > 0 && wwait(&p_empty[x], (n_kv - 1) & 1)) {
+    if (ok && n_kv > 0 && wwait(&o_done[x], 0)) {
       tc_fence_after();
       const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
       __nv_bfloat16 *orow = a.out + (((int64_t)s0 + qpos) * a.Hq + h0 + x) * D;
