@@ -348,7 +348,9 @@ umim_status umim_decode_attention(const void *q, int32_t n_q_heads, const umim_p
  *              n_kv_heads * head_dim * (n_rows + 64 * batch) * 2 bytes)
  * head_dim 64 or 128; n_q_heads a multiple of n_kv_heads (else
  * UMIM_ERR_UNSUPPORTED).  Device-side errors: UMIM_ERR_INVALID_ARG for
- * offsets that break the rules above (nothing is written).
+ * offsets that break the rules above (nothing is written);
+ * UMIM_ERR_UNSUPPORTED when some |v| >= 65504 or is not finite (the P V
+ * product runs on fp16 operands; the output is then not valid).
  * ------------------------------------------------------------------------ */
 size_t umim_prefill_attention_workspace_size(int32_t batch, int32_t n_rows, int32_t n_kv_heads, int32_t head_dim);
 
