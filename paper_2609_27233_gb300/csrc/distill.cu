@@ -388,6 +388,31 @@ __device__ __forceinline__ void warp_lse(float &m, float &z) {
   z = w;
 }
 
+// mbarrier wait that sleeps instead of spinning: try_wait with a suspend-time
+// hint (the thread is woken when the phase completes, or after 1 ms), so a
+// warp waiting for the cluster takes no issue slots from warps still
+// computing; bounded by kWaitLimitNs like every wait of the library
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity), "r"(1000000u)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ bool mbar_wait_sleep(uint64_t *bar, uint32_t parity) {
+  const uint32_t a = smem_u32(bar);
+  if (mbar_try_wait_sleep(a, parity)) return true;
+  const uint64_t t0 = globaltimer();
+  while (true) {
+    if (mbar_try_wait_sleep(a, parity)) return true;
+    if (globaltimer() - t0 > kWaitLimitNs) return false;
+  }
+}
+
 __device__ __forceinline__ float warp_sum(float x) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
@@ -512,7 +537,7 @@ __global__ void __launch_bounds__(T, 512 / T) ce_kernel(CeArgs a) {
 
   // wait for phase `parity` of mbarrier m; a wait that gives up marks the CTA failed
   auto xwait = [&](uint64_t *m, uint32_t parity) {
-    if (!failed && !mbar_wait(m, parity)) {
+    if (!failed && !mbar_wait_sleep(m, parity)) {
       failed = true;
       set_error(a.status, UMIM_ERR_TIMEOUT);
     }
@@ -616,20 +641,35 @@ __global__ void __launch_bounds__(T, 512 / T) ce_kernel(CeArgs a) {
     Zt = warp_sum(Zt);
     Zs = warp_sum(Zs);
     // P(v) = exp(x - m_thread) * exp(m_thread - M) / Z
-    const float ct = (mt == -INFINITY) ? 0.f : ex2_approx(fmaf(mt, kLog2e, nMt)) * rcp_approx(Zt);
+    // (P^T carries the 1/N of the loss from here on: the loss terms, a and A
+    // come out divided by N, and the gradient is one FMA per element)
+    const float ct = (mt == -INFINITY) ? 0.f : ex2_approx(fmaf(mt, kLog2e, nMt)) * rcp_approx(Zt) * invN;
     const float cs = (ms == -INFINITY) ? 0.f : ex2_approx(fmaf(ms, kLog2e, nMs)) * rcp_approx(Zs);
 
-    // ---- pass 2: P^T, P^S, the loss terms and a ----
+    // ---- pass 2: P^T / N, P^S, the loss terms and a / N ----
     float lsum = 0.f, asum = 0.f;
+    if (eps > 0.f) {
 #pragma unroll
-    for (int i = 0; i < KV * 8; ++i) {
-      const float pt = xt[i] * ct, ps = xs[i] * cs;
-      const float q = fmaxf(ps + eps, 1.17549435e-38f);   // log2 stays finite when eps = 0
-      lsum = fmaf(pt, lg2_approx(q), lsum);
-      const float av = pt * (ps * rcp_approx(q));
-      asum += av;
-      xt[i] = av;
-      xs[i] = ps;
+      for (int i = 0; i < KV * 8; ++i) {
+        const float pt = xt[i] * ct, ps = xs[i] * cs;
+        const float q = ps + eps;
+        lsum = fmaf(pt, lg2_approx(q), lsum);
+        const float av = pt * (ps * rcp_approx(q));
+        asum += av;
+        xt[i] = av;
+        xs[i] = ps;
+      }
+    } else {
+#pragma unroll
+      for (int i = 0; i < KV * 8; ++i) {
+        const float pt = xt[i] * ct, ps = xs[i] * cs;
+        const float q = fmaxf(ps, 1.17549435e-38f);   // log2 stays finite when eps = 0
+        lsum = fmaf(pt, lg2_approx(q), lsum);
+        const float av = pt * (ps * rcp_approx(q));
+        asum += av;
+        xt[i] = av;
+        xs[i] = ps;
+      }
     }
     lsum = warp_sum(lsum);
     asum = warp_sum(asum);
@@ -646,9 +686,9 @@ __global__ void __launch_bounds__(T, 512 / T) ce_kernel(CeArgs a) {
     }
     Lp = warp_sum(Lp);
     A = warp_sum(A);
-    if (rank == 0 && tid == 0) a.pair_loss[p] = -Lp * kLn2;
+    if (rank == 0 && tid == 0) a.pair_loss[p] = -Lp * kLn2 * (float)N;   // Lp is the sum / N
 
-    // ---- pass 3: gradient -(1/N) (a_v - P^S(v) A) ----
+    // ---- pass 3: gradient -(1/N) (a_v - P^S(v) A) = P^S(v) (A/N) - a_v/N ----
     if (grow) {
 #pragma unroll
       for (int k = 0; k < KV; ++k) {
@@ -656,7 +696,7 @@ __global__ void __launch_bounds__(T, 512 / T) ce_kernel(CeArgs a) {
         if (vi < vcnt) {
           float gr[8];
 #pragma unroll
-          for (int j = 0; j < 8; ++j) gr[j] = (xs[8 * k + j] * A - xt[8 * k + j]) * invN;
+          for (int j = 0; j < 8; ++j) gr[j] = fmaf(xs[8 * k + j], A, -xt[8 * k + j]);   // A and a already / N
           store8(grow, (int64_t)(vbeg + vi) * 8, a.V, gr);
         }
       }
