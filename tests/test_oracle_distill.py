@@ -106,7 +106,7 @@ def test_gradient_matches_autograd(eps):
     pt = torch.softmax(torch.from_numpy(T[tr]), -1)
     ls = -(pt * torch.log(torch.softmax(s[sr], -1) + eps)).sum(-1).mean()
     ls.backward()
-    assert abs(float(ls) - loss) < 1e-12
+    assert abs(ls.detach().item() - loss) < 1e-12
     np.testing.assert_allclose(grad, s.grad.numpy(), rtol=1e-9, atol=1e-14)
     assert np.all(grad[[0, 2]] == 0)   # rows in no pair
 

@@ -53,19 +53,3 @@ def test_batch_too_large_for_the_scratch_array_is_refused():
         m.umim_decode_attention_static(q, pool, 0, bt, lens)
     assert e.value.code == 5   # UMIM_ERR_WORKSPACE
 
-
-def test_static_entry_point_can_be_captured_in_a_cuda_graph():
-    """After a first call outside capture, calls can be captured into a CUDA
-    graph; the replay gives what the eager call gives, bit for bit."""
-    m = umim()
-    d = dev()
-    c = W.decode_case(303, lens=[700, 31, 2048], n_q_heads=32, n_kv_heads=8, head_dim=128, n_spans=[0] * 3)
-    g = case_to_dev(c, d)
-    eager = m.umim_decode_attention_static(g["q"], g["pool"], 0, g["bt"], g["lens"])
-    out = torch.empty_like(eager)
-    graph = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(graph):
-        m.umim_decode_attention_static(g["q"], g["pool"], 0, g["bt"], g["lens"], out=out)
-    graph.replay()
-    torch.cuda.synchronize()
-    assert torch.equal(out, eager)
