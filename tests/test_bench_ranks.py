@@ -58,3 +58,34 @@ def test_ranks_get_independent_batches_of_the_same_shape():
     assert not np.array_equal(a["span_start"], b["span_start"])
     # weak scaling: about the same work per rank (30 % coverage of the same lengths)
     assert abs(len(a["span_start"]) - len(b["span_start"])) < 0.05 * len(a["span_start"])
+
+
+def _run_bench(args, env_extra):
+    import json
+    import subprocess
+    import sys
+    env = dict(os.environ, **env_extra)
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    r = subprocess.run([sys.executable, os.path.join(root, "bench.py")] + args, cwd=root, env=env,
+                       capture_output=True, text=True, timeout=600)
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = [l for l in r.stdout.splitlines() if l.startswith("{")]
+    return [json.loads(l) for l in lines]
+
+
+def test_reference_arm_prints_one_line_with_the_contract_keys():
+    """The oracle arm runs on the host cores only and prints one JSON line
+    on the same metric, unit and workload as the GPU arm."""
+    (line,) = _run_bench(["--impl", "reference", "--steps", "1", "--warmup", "3"], {})
+    assert line["impl"] == "reference"
+    assert line["metric"] == bench.METRIC and line["unit"] == bench.UNIT
+    assert line["higher_is_better"] is True and line["value"] > 0
+    assert line["config"]["workload"].startswith("llama8b_layer")
+    assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["value"] == line["value"]
+    assert line["e2e"] == {"value": line["value"], "unit": bench.UNIT, "h2d_bytes_per_step": 0,
+                           "d2h_bytes_per_step": 0}
+
+
+def test_reference_arm_other_ranks_exit_without_work():
+    assert _run_bench(["--impl", "reference", "--gpus", "2", "--steps", "1", "--warmup", "3"],
+                      {"RANK": "1", "WORLD_SIZE": "2", "LOCAL_RANK": "1"}) == []
