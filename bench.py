@@ -304,7 +304,7 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--workload", default="llama8b_layer",
                     choices=["llama8b_layer", "serving", "prompt_compression", "long_context", "rule_matching",
-                             "prefill", "distill"])
+                             "prefill", "distill", "tiny"])
     ap.add_argument("--coverage", type=float, default=0.4, help="long_context span coverage")
     ap.add_argument("--rope", action="store_true",
                     help="llama8b_layer / long_context: re-rotate moved keys to their compressed positions "
@@ -315,6 +315,8 @@ def main():
     args = ap.parse_args()
     if args.workload == "serving" and args.impl == "umim":
         return serving_bench(args)
+    if args.workload == "tiny" and args.impl == "umim":
+        return tiny_bench(args)
     if args.workload in ("prompt_compression", "long_context", "rule_matching", "prefill", "distill") and \
             args.impl == "umim":
         return side_bench(args)
@@ -1191,6 +1193,114 @@ def side_bench(args):
             "clocks": clk.summary(w0, w1),
             "traced_ms_per_step": tms / K, "peaks": {"hbm_gbs": peaks["hbm"], "bf16_tflops": peaks["bf16"],
                                                      "source": peaks["src"]}}
+    print(json.dumps(line))
+    return 0
+
+
+def tiny_bench(args):
+    """The tiny workload, a latency case: one sequence of 512 cached tokens
+    (8/2 heads, head_dim 64, page 16) with 40 spans of 2..4 tokens; the merge
+    module (d_model 512, 4 heads, 32000-row table) maps the spans' tokens to
+    surrogates, the spans are rolled back to one surrogate KV entry each, then
+    decode attention runs over the compacted cache.  Each step is timed alone
+    with CUDA events; before each step the cache is restored and L2 is flushed
+    (a 256 MB write), both outside the timed interval."""
+    import torch
+    import paper_2609_27233_gb300 as umim
+    import workloads as W
+
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    umim.lib()
+    peaks = load_peaks()
+    K, Wm = args.steps, max(3, args.warmup)
+    status = umim.new_status(dev)
+    seed = W.SEEDS["tiny"]
+    V, d, h, L, Hq, Hkv, D = 32000, 512, 4, 512, 8, 2, 64
+    c = W.decode_case(seed, lens=[L], n_q_heads=Hq, n_kv_heads=Hkv, head_dim=D, n_spans=[40], device=dev)
+    S = c.span_start.numel()
+    st_np, ln_np = c.span_start.cpu().numpy(), c.span_len.cpu().numpy()
+    ids = W.rng(seed + 7).integers(0, V, size=L).astype(np.int32)
+    span_ids = np.concatenate([ids[s:s + k] for s, k in zip(st_np, ln_np)]).astype(np.int32)
+    span_offs = np.concatenate([[0], np.cumsum(ln_np)]).astype(np.int32)
+    T = len(span_ids)
+    tok, toffs = torch.from_numpy(span_ids).to(dev), torch.from_numpy(span_offs).to(dev)
+    table = W.bf16_normal((V, d), 0.02, seed + 101, dev)
+    weights = W.merge_weights(d, h, seed + 202, dev)
+    z = torch.empty((S, d), dtype=torch.float32, device=dev)
+    pool, bt, lens = torch.empty_like(c.pool), torch.empty_like(c.block_table), torch.empty_like(c.seq_lens)
+    freed = torch.empty(c.max_pages, dtype=torch.int32, device=dev)
+    out = torch.empty_like(c.q)
+    ws_m = umim.workspace(umim.umim_merge_spans_workspace_size(T, S, d), dev)
+    ws_r = umim.workspace(umim.umim_kv_rollback_workspace_size(1, S, c.max_pages, 1, Hkv, D), dev)
+    ws_a = umim.workspace(umim.umim_decode_attention_workspace_size(1, Hq, Hkv, D), dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+
+    def step():
+        umim.umim_merge_spans(table, tok, toffs, weights, surrogates=z, workspace_buf=ws_m, dev_status=status)
+        umim.umim_kv_rollback(pool, bt, lens, c.span_offsets, c.span_start, c.span_len, c.surrogate_k,
+                              c.surrogate_v, freed_pages=freed, workspace_buf=ws_r, dev_status=status)
+        umim.umim_decode_attention(c.q, pool, 0, bt, lens, out=out, workspace_buf=ws_a, dev_status=status)
+
+    def run(n):
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n)]
+        for e0, e1 in ev:
+            pool.copy_(c.pool)
+            bt.copy_(c.block_table)
+            lens.copy_(c.seq_lens)
+            flush.zero_()
+            e0.record()
+            step()
+            e1.record()
+        torch.cuda.synchronize()
+        return [e0.elapsed_time(e1) for e0, e1 in ev]
+
+    run(Wm)
+    umim.check_status(status, "warm-up")
+    Lp = L - int((ln_np - 1).sum())
+    entry = 2 * Hkv * D * 2
+    moved, r, prev = 0, 0, 0
+    for s_, k_ in zip(st_np, ln_np):
+        if r > 0:
+            moved += int(s_) - prev
+        r += int(k_) - 1
+        prev = int(s_ + k_)
+    if r > 0:
+        moved += L - prev
+    work_of = {"merge.gemm1": ("tensor", 2.0 * T * d * d / 1e12, "TFLOP/s", peaks["bf16"]),
+               "merge.gemm2": ("tensor", 2.0 * S * d * d / 1e12, "TFLOP/s", peaks["bf16"]),
+               "rollback.move": ("hbm", (moved + S) * entry * 2 / 1e9, "GB/s", peaks["hbm"]),
+               "attention.decode": ("hbm", (Lp * entry + 2 * Hq * D * 2) / 1e9, "GB/s", peaks["hbm"])}
+    clk = ClockSampler(0)
+    time.sleep(0.3)
+    w0 = time.time()
+    per = run(K)
+    w1 = time.time()
+    time.sleep(0.1)
+    clk.stop()
+    umim.check_status(status, "timed steps")
+    umim.trace_start(64 * (K + 2))
+    run(K)
+    umim.trace_stop()
+    recs = umim.trace_read(64 * (K + 2))
+    kernels = kernel_table(recs, K, work_of)
+    calls = {}
+    for lab, v in recs:
+        calls[lab.split(".")[0]] = calls.get(lab.split(".")[0], 0.0) + v
+    ms = float(np.sum(per))
+    line = {"metric": "tiny merged-context decode step (latency): merged spans/s", "value": S * K / (ms / 1000.0),
+            "unit": "spans/s", "n_gpus": 1, "steps": K, "warmup": Wm, "ms_per_step": ms / K,
+            "higher_is_better": True, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": "tiny: 1 sequence x 512 cached tokens, 8/2 heads, head_dim 64, bf16 paged KV "
+                                   "(page 16), 40 spans of 2..4 tokens merged (merge module d_model 512, 4 heads, "
+                                   "32000 x 512 table), rolled back, then decode attention",
+                       "spans": S, "span_tokens": T, "compacted_length": Lp,
+                       "us_per_step": {"median": round(1000 * float(np.median(per)), 2),
+                                       "mean": round(1000 * ms / K, 2), "min": round(1000 * float(np.min(per)), 2)},
+                       "traced_kernel_us_per_call": {k: round(1000 * v / K, 2) for k, v in calls.items()},
+                       "l2": "flushed before every timed step (256 MB write outside the timed interval)"},
+            "kernels": kernels, "gpu_launches": len(recs), "clocks": clk.summary(w0, w1),
+            "traced_ms_per_step": float(np.sum([v for _, v in recs])) / K}
     print(json.dumps(line))
     return 0
 
