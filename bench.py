@@ -191,8 +191,8 @@ class ClockSampler:
 # CPU oracle on a bounded sample (the cpu_baseline and the reference arm)
 # ---------------------------------------------------------------------------
 class OracleSampler:
-    """Times the oracle on part of one step and scales it to spans/s of a
-    whole step.  The merge-module weights are built once; each sample draws
+    """Times the oracle on a sample of one step (or on the whole step) and
+    scales it to spans/s of a whole step.  The merge-module weights are built once; each sample draws
     its own spans and sequences."""
 
     def __init__(self, st, seed):
@@ -1038,8 +1038,8 @@ def side_bench(args):
                "compressed_rows": Tc, "uncompressed_rows": Tu, "mean_compressed_length": round(Tc / B, 1),
                "uncompressed_ms": round(unc_ms, 4),
                "uncompressed_tflops": round(causal_flops([L] * B) / unc_ms / 1e9, 1),
-               "kernel": "tcgen05.mma (S and O in tensor memory; P from shared memory as bf16 high + remainder), "
-                         "TMA-fed K / V^T ring, V transposed per call",
+               "kernel": "tcgen05.mma (S, P and O in tensor memory; P V on fp16 operands), "
+                         "TMA-fed K / V^T rings, V transposed per call",
                "l2": "q/k/v of one layer are 0.96 GB (compressed) / 1.34 GB (uncompressed): larger than L2"}
     elif args.workload == "distill":
         seed = W.SEEDS["distillation"]

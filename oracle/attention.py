@@ -1,8 +1,9 @@
 """Decode attention over the compacted paged cache, oracle (test infrastructure only).
 
 After rollback the frozen backbone attends over the shorter cache in the usual
-way (App. I.1: each decode step "attends to the accumulated KV cache"; App. E:
-the surrogate's KV state is one ordinary cache entry).  The paper gives no
+way (App. I.1: every decode step attends over whatever KV entries the cache
+holds at that point; App. E: the surrogate's KV state is one ordinary cache
+entry).  The paper gives no
 formula of its own, so this is the standard grouped-query scaled dot-product
 attention of a Llama-style decoder for one new query token:
 

@@ -3,8 +3,8 @@
 App. E ("Decoding-Time Merging and KV-Cache Update") and App. C.6: when a span
 is merged, the KV entries stored for its tokens are cropped and a single KV
 state computed from the surrogate takes their place, so the cache length goes
-from L_C to L_C - (n - 1) + 1 (Fig. 2 caption: "replaces its multiple KV
-entries with a single merged KV cache").
+from L_C to L_C - (n - 1) + 1 (Fig. 2 caption: the span's several KV
+entries give way to one merged entry).
 
 This restates that operation for a paged cache and for any number of sorted,
 non-overlapping spans per sequence (the paper crops a suffix; spans placed
