@@ -1287,6 +1287,29 @@ def tiny_bench(args):
     calls = {}
     for lab, v in recs:
         calls[lab.split(".")[0]] = calls.get(lab.split(".")[0], 0.0) + v
+    # the same three calls captured once as a CUDA graph and replayed (launch gaps removed)
+    graph = None
+    try:
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            step()
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+        for e0, e1 in ev:
+            pool.copy_(c.pool)
+            bt.copy_(c.block_table)
+            lens.copy_(c.seq_lens)
+            flush.zero_()
+            e0.record()
+            g.replay()
+            e1.record()
+        torch.cuda.synchronize()
+        umim.check_status(status, "graph replays")
+        gper = [e0.elapsed_time(e1) for e0, e1 in ev]
+        graph = {"us_per_step": {"median": round(1000 * float(np.median(gper)), 2),
+                                 "mean": round(1000 * float(np.mean(gper)), 2)},
+                 "spans_per_s": S * K / (float(np.sum(gper)) / 1000.0)}
+    except Exception as ex:   # capture refused: report it, the eager numbers stand
+        graph = {"error": str(ex)[:200]}
     ms = float(np.sum(per))
     line = {"metric": "tiny merged-context decode step (latency): merged spans/s", "value": S * K / (ms / 1000.0),
             "unit": "spans/s", "n_gpus": 1, "steps": K, "warmup": Wm, "ms_per_step": ms / K,
@@ -1298,6 +1321,7 @@ def tiny_bench(args):
                        "us_per_step": {"median": round(1000 * float(np.median(per)), 2),
                                        "mean": round(1000 * ms / K, 2), "min": round(1000 * float(np.min(per)), 2)},
                        "traced_kernel_us_per_call": {k: round(1000 * v / K, 2) for k, v in calls.items()},
+                       "cuda_graph": graph,
                        "l2": "flushed before every timed step (256 MB write outside the timed interval)"},
             "kernels": kernels, "gpu_launches": len(recs), "clocks": clk.summary(w0, w1),
             "traced_ms_per_step": float(np.sum([v for _, v in recs])) / K}
