@@ -1,5 +1,6 @@
 // C ABI of libumim: host-side argument checks, then the kernels of each part.
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <cstring>
 #include <mutex>
@@ -83,14 +84,16 @@ int prepare_device(cudaStream_t stream) {
     cudaSetDevice(dev);
   else
     cudaGetDevice(&dev);
-  static int cached_dev = -1, cached_sms = 0;
-  if (dev != cached_dev) {
-    int sms = 0;
+  // SM count per device, looked up once; atomics, since calls for different
+  // devices may come from different host threads
+  static std::atomic<int> sms_of[64];
+  int sms = 0;
+  if (dev >= 0 && dev < 64) sms = sms_of[dev].load(std::memory_order_relaxed);
+  if (sms == 0) {
     if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) sms = 0;
-    cached_sms = sms;
-    cached_dev = dev;
+    if (sms > 0 && dev >= 0 && dev < 64) sms_of[dev].store(sms, std::memory_order_relaxed);
   }
-  return cached_sms;
+  return sms;
 }
 
 int current_sms() {
