@@ -102,3 +102,20 @@ def test_distillation_host_checks(lib):
                                   null) == 1     # spans but no span arrays
     assert lib.umim_distill_align(fake, 2, fake, fake, fake, 3, fake, fake, fake, 10, null, null, 0, null,
                                   null) == 5     # no workspace
+
+
+def test_product_path_and_oracle_share_nothing():
+    """The library, its binding and its header never name the oracle, and the
+    oracle never imports the library: the two sides meet only in the tests."""
+    pkg = os.path.join(ROOT, "paper_2609_27233_gb300")
+    product = [os.path.join(pkg, f) for f in os.listdir(pkg) if f.endswith(".py")]
+    product += [os.path.join(pkg, "csrc", f) for f in os.listdir(os.path.join(pkg, "csrc"))]
+    product += HEADERS
+    for p in product:
+        assert "oracle" not in open(p, errors="ignore").read(), p
+    odir = os.path.join(ROOT, "oracle")
+    for f in os.listdir(odir):
+        if f.endswith(".py"):
+            text = open(os.path.join(odir, f)).read()
+            for bad in ("import paper_2609_27233_gb300", "from paper_2609_27233_gb300", "ctypes", "libumim"):
+                assert bad not in text, (f, bad)
