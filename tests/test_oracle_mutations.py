@@ -20,9 +20,13 @@ from oracle import distill as D
 from oracle import merge as M
 from oracle import rollback as R
 import test_oracle_attention as TA
+import test_oracle_compaction as TC
 import test_oracle_distill as TD
 import test_oracle_merge as TM
+import test_oracle_prefill as TP
 import test_oracle_rollback as TR
+from oracle import bf16 as OB
+from oracle import compaction as C
 
 
 def _failures(pins):
@@ -290,5 +294,113 @@ def test_distill_pins_catch(name):
         assert _failures(DISTILL_PINS) >= 1, name
 
 
+# ---------------------------------------------------------------------------
+# compressed prompts (App. C.5, App. E "Prompt Merging", App. J.4)
+# ---------------------------------------------------------------------------
+COMPACTION_PINS = [
+    (TC.test_worked_example, ()),
+    (TC.test_compressed_length_formula, ()),
+    (TC.test_no_spans_is_embedding_lookup, ()),
+    (TC.test_bf16_rounding_matches_torch, ()),
+]
+_build = C.build_compressed
+
+
+def _positions_kept_from_the_original(table_bits, token_ids, span_offsets, span_start, span_len, surrogates):
+    """Position ids that keep each unit's original index (t) instead of
+    renumbering the compressed sequence 0 .. L'-1."""
+    out, pos, cu = _build(table_bits, token_ids, span_offsets, span_start, span_len, surrogates)
+    B, L = np.asarray(token_ids).shape
+    orig = []
+    for b in range(B):
+        lo, hi = int(span_offsets[b]), int(span_offsets[b + 1])
+        t, i = 0, lo
+        while t < L:
+            orig.append(t)
+            if i < hi and t == int(span_start[i]):
+                t += int(span_len[i])
+                i += 1
+            else:
+                t += 1
+    return out, np.asarray(orig, np.int32), cu
+
+
+class _TruncatingBf16:
+    """bf16 conversions with the rounding replaced by truncation."""
+    to_f64 = staticmethod(OB.to_f64)
+
+    @staticmethod
+    def from_f32(x):
+        return (np.asarray(x, np.float32).view(np.uint32) >> 16).astype(np.uint16)
+
+    from_f64 = staticmethod(OB.from_f64)
+
+
+COMPACTION_MUTATIONS = {
+    "original positions kept": ("build_compressed", _positions_kept_from_the_original),
+    "surrogates rounded to bf16 by truncation": ("bf16", _TruncatingBf16),
+}
+
+
+@pytest.mark.parametrize("name", sorted(COMPACTION_MUTATIONS))
+def test_compaction_pins_catch(name):
+    attr, fn = COMPACTION_MUTATIONS[name]
+    with pytest.MonkeyPatch.context() as mp:
+        mp.setattr(C, attr, fn)
+        if attr == "build_compressed":
+            mp.setattr(oracle, attr, fn)
+        else:   # the pins convert through the same module
+            mp.setattr(TC, "bf16", fn)
+        assert _failures(COMPACTION_PINS) >= 1, name
+
+
+# ---------------------------------------------------------------------------
+# prefill attention over packed compressed prompts
+# ---------------------------------------------------------------------------
+PREFILL_PINS = [
+    (TP.test_matches_library_causal_sdpa, (8, 2, 32)),
+    (TP.test_closed_forms, ()),
+    (TP.test_packing_is_per_sequence, ()),
+    (TP.test_last_row_is_decode_attention, ()),
+]
+
+
+def _prefill_variant(keys_to=lambda lo, hi, i: i + 1, first_key=lambda lo, i: lo):
+    def prefill_attention(q_bits, k_bits, v_bits, cu_seqlens, scale=None, rows=None):
+        q, k, v = OB.to_f64(q_bits), OB.to_f64(k_bits), OB.to_f64(v_bits)
+        T, Hq, D = q.shape
+        G = Hq // k.shape[1]
+        scale = 1.0 / math.sqrt(D) if not scale else scale
+        cu = np.asarray(cu_seqlens)
+        out = np.zeros((T, Hq, D))
+        for b in range(len(cu) - 1):
+            lo, hi = int(cu[b]), int(cu[b + 1])
+            for i in range(lo, hi):
+                a, z = first_key(lo, i), keys_to(lo, hi, i)
+                if z <= a:
+                    continue
+                for h in range(Hq):
+                    s = (k[a:z, h // G, :] @ q[i, h]) * scale
+                    e = np.exp(s - s.max())
+                    out[i, h] = (e / e.sum()) @ v[a:z, h // G, :]
+        return out
+    return prefill_attention
+
+
+PREFILL_MUTATIONS = {
+    "no causal mask": _prefill_variant(keys_to=lambda lo, hi, i: hi),
+    "diagonal masked out": _prefill_variant(keys_to=lambda lo, hi, i: i if i > lo else i + 1),
+    "keys of earlier sequences visible": _prefill_variant(first_key=lambda lo, i: 0),
+}
+
+
+@pytest.mark.parametrize("name", sorted(PREFILL_MUTATIONS))
+def test_prefill_pins_catch(name):
+    with pytest.MonkeyPatch.context() as mp:
+        mp.setattr(TP, "prefill_attention", PREFILL_MUTATIONS[name])
+        assert _failures(PREFILL_PINS) >= 1, name
+
+
 def test_unmodified_oracle_passes_the_same_pins():
-    assert _failures(MERGE_PINS + ATTENTION_PINS + ROLLBACK_PINS + DISTILL_PINS) == 0
+    assert _failures(MERGE_PINS + ATTENTION_PINS + ROLLBACK_PINS + DISTILL_PINS + COMPACTION_PINS +
+                     PREFILL_PINS) == 0
