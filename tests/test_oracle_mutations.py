@@ -15,10 +15,12 @@ import pytest
 import torch
 
 import oracle
+from oracle import append as AP
 from oracle import attention as A
 from oracle import distill as D
 from oracle import merge as M
 from oracle import rollback as R
+import test_oracle_append as TAP
 import test_oracle_attention as TA
 import test_oracle_compaction as TC
 import test_oracle_distill as TD
@@ -30,11 +32,13 @@ from oracle import compaction as C
 
 
 def _failures(pins):
+    """How many pins fail: an assertion, or the oracle's own input checks
+    refusing the state the planted mistake left behind."""
     n = 0
     for fn, args in pins:
         try:
             fn(*args)
-        except AssertionError:
+        except (AssertionError, ValueError):
             n += 1
     return n
 
@@ -401,6 +405,61 @@ def test_prefill_pins_catch(name):
         assert _failures(PREFILL_PINS) >= 1, name
 
 
+# ---------------------------------------------------------------------------
+# decode-step append (App. E, Fig. 2 step (2))
+# ---------------------------------------------------------------------------
+APPEND_PINS = [
+    (TAP.test_append_matches_logical_list_model, ()),
+    (TAP.test_page_opened_only_at_boundary, ()),
+    (TAP.test_append_then_replace_by_one_entry_is_appending_that_entry, ()),
+    (TAP.test_appending_n_then_merging_them_is_appending_the_surrogate, (3,)),
+    (TAP.test_appending_n_then_merging_them_is_appending_the_surrogate, (17,)),
+    (TAP.test_rejected_sequences_are_left_unchanged, ()),
+]
+_append = AP.kv_append
+
+
+def _append_variant(slot_shift=0, page_every_call=False, k_into_v=False):
+    def kv_append(pool, block_table, seq_lens, new_k, new_v, new_pages=None, page_size=16):
+        P = page_size
+        pool = np.array(pool, copy=True)
+        bt = np.array(block_table, dtype=np.int32, copy=True)
+        lens = np.array(seq_lens, dtype=np.int32, copy=True)
+        rejected = []
+        for b in range(bt.shape[0]):
+            L = int(lens[b])
+            t = L + slot_shift
+            if L < 0 or t >= bt.shape[1] * P:
+                rejected.append(b)
+                continue
+            opens = page_every_call or t % P == 0
+            page = (-1 if new_pages is None else int(new_pages[b])) if opens else int(bt[b, t // P])
+            if page < 0 or page >= pool.shape[1]:
+                rejected.append(b)
+                continue
+            bt[b, t // P] = page
+            pool[:, page, 0, :, t % P, :] = new_k[b]
+            pool[:, page, 1, :, t % P, :] = new_k[b] if k_into_v else new_v[b]
+            lens[b] = L + 1
+        return pool, bt, lens, rejected
+    return kv_append
+
+
+APPEND_MUTATIONS = {
+    "written one slot too far": _append_variant(slot_shift=1),
+    "a new page taken on every append": _append_variant(page_every_call=True),
+    "K written into the V slot too": _append_variant(k_into_v=True),
+}
+
+
+@pytest.mark.parametrize("name", sorted(APPEND_MUTATIONS))
+def test_append_pins_catch(name):
+    with pytest.MonkeyPatch.context() as mp:
+        mp.setattr(AP, "kv_append", APPEND_MUTATIONS[name])
+        mp.setattr(oracle, "kv_append", APPEND_MUTATIONS[name])
+        assert _failures(APPEND_PINS) >= 1, name
+
+
 def test_unmodified_oracle_passes_the_same_pins():
     assert _failures(MERGE_PINS + ATTENTION_PINS + ROLLBACK_PINS + DISTILL_PINS + COMPACTION_PINS +
-                     PREFILL_PINS) == 0
+                     PREFILL_PINS + APPEND_PINS) == 0
