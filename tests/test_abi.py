@@ -119,3 +119,25 @@ def test_product_path_and_oracle_share_nothing():
             text = open(os.path.join(odir, f)).read()
             for bad in ("import paper_2609_27233_gb300", "from paper_2609_27233_gb300", "ctypes", "libumim"):
                 assert bad not in text, (f, bad)
+
+
+def test_allocation_free_attention_host_checks(lib):
+    """Shapes and arguments are refused on the host, before the first CUDA call."""
+    from paper_2609_27233_gb300._lib import PagedKVC
+    null = ctypes.c_void_p(0)
+    fake = ctypes.c_void_p(1 << 20)      # never dereferenced: every call below stops at a host check
+
+    def call(kv, hq=8, layer=0, batch=2, q=fake, out=fake):
+        return lib.umim_decode_attention_static(q, hq, ctypes.byref(kv), layer, fake, 4, fake, batch, 0.0, out,
+                                                null, null)
+
+    assert call(PagedKVC(0, 1, 4, 2, 16, 128)) == 1          # no pool
+    assert call(PagedKVC(4096 + 8, 1, 4, 2, 16, 128)) == 1   # pool not 16-byte aligned
+    assert call(PagedKVC(4096, 1, 4, 2, 8, 128)) == 2        # page size 8
+    assert call(PagedKVC(4096, 1, 4, 2, 16, 96)) == 2        # head_dim 96
+    assert call(PagedKVC(4096, 1, 4, 2, 16, 128), hq=34) == 2   # 17 query heads per KV head
+    assert call(PagedKVC(4096, 1, 4, 2, 16, 128), hq=7) == 2    # not a multiple of the KV heads
+    assert call(PagedKVC(4096, 2, 4, 2, 16, 128), layer=2) == 1
+    assert call(PagedKVC(4096, 1, 4, 2, 16, 128), q=null) == 1
+    assert call(PagedKVC(4096, 1, 4, 2, 16, 128), out=ctypes.c_void_p((1 << 20) + 1)) == 1
+    assert call(PagedKVC(4096, 1, 4, 2, 16, 128), batch=0) == 0   # nothing to do
