@@ -141,3 +141,48 @@ def test_allocation_free_attention_host_checks(lib):
     assert call(PagedKVC(4096, 1, 4, 2, 16, 128), q=null) == 1
     assert call(PagedKVC(4096, 1, 4, 2, 16, 128), out=ctypes.c_void_p((1 << 20) + 1)) == 1
     assert call(PagedKVC(4096, 1, 4, 2, 16, 128), batch=0) == 0   # nothing to do
+
+
+def test_other_entry_points_host_checks(lib):
+    """Compressed prompts, append, surrogate lookup, prefill and the wait
+    self-test refuse bad arguments on the host (no CUDA call is reached)."""
+    from paper_2609_27233_gb300._lib import PagedKVC
+    null = ctypes.c_void_p(0)
+    fake = ctypes.c_void_p(1 << 20)
+    odd = ctypes.c_void_p((1 << 20) + 4)
+
+    def compressed(d=512, batch=2, emb=fake, ws=fake, wsb=1 << 24):
+        return lib.umim_build_compressed(emb, 1000, d, fake, batch, 64, fake, fake, fake, 3, fake, fake, 1000,
+                                         fake, fake, ws, wsb, null, null)
+    assert compressed(d=500) == 2                # d_model not a multiple of 8
+    assert compressed(batch=-1) == 1
+    assert compressed(batch=0) == 0
+    assert compressed(emb=null) == 1
+    assert compressed(emb=odd) == 1              # table not 16-byte aligned
+    assert compressed(ws=null) == 5
+    assert compressed(wsb=16) == 5
+
+    kv = PagedKVC(4096, 1, 4, 2, 16, 128)
+    assert lib.umim_kv_append(ctypes.byref(kv), fake, 4, fake, 2, odd, fake, fake, null, null) == 1
+    assert lib.umim_kv_append(ctypes.byref(kv), null, 4, fake, 2, fake, fake, fake, null, null) == 1
+    assert lib.umim_kv_append(ctypes.byref(kv), fake, 4, fake, 0, fake, fake, fake, null, null) == 0
+    kv64 = PagedKVC(4096, 1, 4, 2, 16, 96)
+    assert lib.umim_kv_append(ctypes.byref(kv64), fake, 4, fake, 2, fake, fake, fake, null, null) == 2
+
+    assert lib.umim_lookup_surrogates(fake, 10, 6, fake, 4, null, fake, null, null) == 1   # d % 4 != 0
+    assert lib.umim_lookup_surrogates(odd, 10, 8, fake, 4, null, fake, null, null) == 1
+    assert lib.umim_lookup_surrogates(fake, 10, 8, fake, 0, null, fake, null, null) == 0
+
+    def prefill(hd=128, hq=32, hkv=8, q=fake, ws=fake, batch=2):
+        return lib.umim_prefill_attention(q, fake, fake, 100, hq, hkv, hd, fake, batch, 0.0, fake, ws, 1 << 30,
+                                          null, null)
+    assert prefill(hd=96) == 2
+    assert prefill(hq=30) == 2                   # not a multiple of the KV heads
+    assert prefill(batch=0) == 0
+    assert prefill(q=odd) == 1
+    assert prefill(ws=null) == 5
+
+    assert lib.umim_selftest_bounded_wait(2, 1000, null, null, null, null) == 1
+    assert lib.umim_selftest_bounded_wait(0, 0, null, null, null, null) == 1
+    assert lib.umim_selftest_bounded_wait(0, 2000000, null, null, null, null) == 1
+    assert lib.umim_selftest_bounded_wait(1, 1000, null, null, null, null) == 1   # flags needed
