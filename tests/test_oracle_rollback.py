@@ -186,3 +186,29 @@ def test_page_aligned_lengths(L, spans, exp_len, exp_pages):
     assert freed == [int(x) for x in c["bt"][0, exp_pages:n_before]]
     assert np.all(bt[0, exp_pages:] == -1)
     np.testing.assert_array_equal(bt[0, :exp_pages], c["bt"][0, :exp_pages])
+
+
+@pytest.mark.parametrize("seed,lens,cov", [(21, [300, 64, 0, 17], 0.4), (22, [1000], 0.6)])
+def test_one_span_at_a_time_right_to_left_equals_the_batched_call(seed, lens, cov):
+    """Rolling back the spans one call at a time, rightmost first (so every
+    start is still valid), ends in the state of the one batched call: same
+    lengths, same block tables, same logical entries, same set of pages
+    released."""
+    case = W.decode_case(seed, lens=lens, n_q_heads=4, n_kv_heads=2, head_dim=8, n_layers=2, coverage=cov)
+    c = _np(case)
+    pool, bt, nl, freed = _run(c)
+    B = len(lens)
+    p1, b1, l1, f1 = c["pool"], c["bt"], c["lens"], []
+    for b in range(B):
+        for i in reversed(range(int(c["offs"][b]), int(c["offs"][b + 1]))):
+            o = np.zeros(B + 1, np.int32)
+            o[b + 1:] = 1
+            p1, b1, l1, f = oracle.kv_rollback(p1, b1, l1, o, c["st"][i:i + 1], c["ln"][i:i + 1],
+                                               c["sk"][i:i + 1], c["sv"][i:i + 1])
+            f1 += f
+    np.testing.assert_array_equal(l1, nl)
+    np.testing.assert_array_equal(b1, bt)
+    assert sorted(f1) == sorted(freed)
+    for layer in range(2):
+        for b in range(B):
+            assert _logical(p1, b1[b], int(l1[b]), layer) == _logical(pool, bt[b], int(nl[b]), layer)
