@@ -97,3 +97,31 @@ def test_after_rollback_equals_rebuilt_cache():
             s_ = Kr[:, h // 4] @ q[b, h] / math.sqrt(32)
             e = np.exp(s_ - s_.max())
             np.testing.assert_allclose(out[b, h], (e / e.sum()) @ Vr[:, h // 4], atol=1e-12)
+
+
+@pytest.mark.parametrize("pieces", [1, 2, 5, 40])
+def test_split_keys_merged_by_log_sum_exp_equal_the_whole(pieces):
+    """The split-K form: softmax statistics (max, sum, weighted values) of
+    separate key ranges, merged with log-sum-exp weights, give the same
+    output as attention over all keys at once (float64, any split)."""
+    case = W.decode_case(15, lens=[333, 40], n_q_heads=8, n_kv_heads=2, head_dim=32, n_spans=[0, 0])
+    pool, bt, lens = W.bits(case.pool), case.block_table.numpy(), case.seq_lens.numpy()
+    qb = W.bits(case.q)
+    out = oracle.decode_attention(qb, pool, 0, bt, lens)
+    q = bf16.to_f64(qb)
+    for b in range(2):
+        K, V = _contig(pool, bt[b], int(lens[b]), 0)
+        bounds = np.linspace(0, int(lens[b]), pieces + 1).astype(int)
+        for h in range(8):
+            parts = []
+            for lo, hi in zip(bounds[:-1], bounds[1:]):
+                if hi == lo:
+                    continue
+                s = K[lo:hi, h // 4] @ q[b, h] / math.sqrt(32)
+                m = s.max()
+                e = np.exp(s - m)
+                parts.append((m, e.sum(), e @ V[lo:hi, h // 4]))
+            M = max(p[0] for p in parts)
+            l = sum(p[1] * math.exp(p[0] - M) for p in parts)
+            acc = sum(p[2] * math.exp(p[0] - M) for p in parts)
+            np.testing.assert_allclose(acc / l, out[b, h], rtol=0, atol=1e-12)
