@@ -23,6 +23,10 @@
  *  - Pointers named *device* point to GPU memory of the current device; the
  *    caller allocates and owns every buffer, including the workspace.  The
  *    library never allocates GPU memory.
+ *  - Each call runs on the device of `stream` and restores the caller's
+ *    current device before returning.  While `stream` is being captured
+ *    into a CUDA graph its device cannot be queried: the current device must
+ *    then be the stream's device.
  *  - Every call is asynchronous on `stream`.  The returned umim_status only
  *    reports what the host can check (null pointers, unsupported shapes, a
  *    workspace that is too small, a failed launch).  Checks that need device
@@ -553,16 +557,25 @@ umim_status umim_distill_soft_ce(const void *teacher_logits, int32_t n_teacher_r
  * forbids allocations outside its arena, may be unable to provide the
  * workspace that umim_decode_attention needs.  This variant computes exactly
  * the same result but takes its scratch (split-K plan and fp32 partials)
- * from an array of UMIM_STATIC_SCRATCH_BYTES compiled into the library; every
- * GPU that loads the library holds that array until the process exits.
+ * from an array of UMIM_STATIC_SCRATCH_BYTES compiled into the library.
  *  - Arguments and results are those of umim_decode_attention, without the
- *    workspace.  It allocates nothing and calls no allocating routine.
+ *    workspace.  It calls no cudaMalloc, cudaFree or allocating library
+ *    routine.
  *  - A batch whose scratch would exceed the array (about
  *    (batch * n_kv_heads + 12 * SMs) * 16 * (head_dim + 2) * 4 bytes) is
  *    rejected with UMIM_ERR_WORKSPACE before anything is launched.
- *  - The first call on a device looks up the array's device address
- *    (cudaGetSymbolAddress) and the SM count; make that first call before
- *    any stream capture begins.
+ *  - The first call on a device does the set-up: it looks up the array's
+ *    device address (cudaGetSymbolAddress) and the SM count.  Under CUDA's
+ *    default lazy module loading, that lookup is also when the driver loads
+ *    the array onto the device and reserves its UMIM_STATIC_SCRATCH_BYTES,
+ *    which then stay reserved until the process exits.  So make the first
+ *    call on each device early: before the caller's own allocator takes the
+ *    device's free memory (otherwise the set-up fails with UMIM_ERR_CUDA),
+ *    and before any stream capture begins.  Later calls reserve nothing.
+ *  - The stream's device is made current for the call and the caller's
+ *    current device is restored before it returns.  While the stream is
+ *    being captured into a CUDA graph its device cannot be queried, so the
+ *    current device must then be the stream's device.
  *  - All calls share the one array.  Nothing in it has to start at zero
  *    (each call rewrites every field it reads), but calls whose kernels
  *    overlap on the GPU (different streams, no ordering between them) race

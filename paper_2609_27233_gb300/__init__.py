@@ -31,6 +31,7 @@ UMIM_OK = 0
 STATUS = {0: "UMIM_OK", 1: "UMIM_ERR_INVALID_ARG", 2: "UMIM_ERR_UNSUPPORTED", 3: "UMIM_ERR_CUDA",
           4: "UMIM_ERR_TIMEOUT", 5: "UMIM_ERR_WORKSPACE"}
 PAGE_SIZE = 16
+STATIC_SCRATCH_BYTES = 32 << 20   # UMIM_STATIC_SCRATCH_BYTES of include/umim.h
 
 
 class UmimError(RuntimeError):
@@ -266,7 +267,7 @@ def umim_decode_attention_static(q, pool, layer, block_table, seq_lens, scale=0.
 
 
 # ---------------------------------------------------------------------------
-# kernel tracing (profiling aid)
+# prefill attention and the bounded-wait self-test
 # ---------------------------------------------------------------------------
 def umim_prefill_attention(q, k, v, cu_seqlens, scale=0.0, out=None, workspace_buf=None, dev_status=None,
                            stream=None):
@@ -443,6 +444,9 @@ def umim_distill_soft_ce(teacher_logits, student_logits, teacher_rows, student_r
     return loss, pair_loss, (grad if with_grad else None)
 
 
+# ---------------------------------------------------------------------------
+# kernel tracing (profiling aid)
+# ---------------------------------------------------------------------------
 def trace_start(capacity=4096):
     _check(lib().umim_trace_start(capacity), "umim_trace_start")
 

@@ -73,29 +73,6 @@ umim_status decode_attention(const void *, int, const umim_paged_kv *, int, cons
 
 namespace {
 
-// Make the stream's device current for this runtime instance; return its SM count.
-// A stream being captured into a CUDA graph refuses cudaStreamGetDevice (and the
-// refusal invalidates the capture), so there the current device is taken.
-int prepare_device(cudaStream_t stream) {
-  int dev = 0;
-  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
-  if (stream != nullptr && cudaStreamIsCapturing(stream, &cs) == cudaSuccess && cs == cudaStreamCaptureStatusNone &&
-      cudaStreamGetDevice(stream, &dev) == cudaSuccess)
-    cudaSetDevice(dev);
-  else
-    cudaGetDevice(&dev);
-  // SM count per device, looked up once; atomics, since calls for different
-  // devices may come from different host threads
-  static std::atomic<int> sms_of[64];
-  int sms = 0;
-  if (dev >= 0 && dev < 64) sms = sms_of[dev].load(std::memory_order_relaxed);
-  if (sms == 0) {
-    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) sms = 0;
-    if (sms > 0 && dev >= 0 && dev < 64) sms_of[dev].store(sms, std::memory_order_relaxed);
-  }
-  return sms;
-}
-
 int current_sms() {
   int dev = 0, sms = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return 0;
@@ -171,7 +148,8 @@ umim_status umim_merge_spans(const void *embeddings, int64_t vocab, const int32_
   if (!workspace || !aligned(workspace, 256) ||
       workspace_bytes < merge_spans_workspace_bytes(n_tokens, n_spans, w->d_model))
     return UMIM_ERR_WORKSPACE;
-  const int sms = prepare_device(stream);
+  const DeviceScope scope(stream);
+  const int sms = scope.sms();
   return merge_spans(embeddings, vocab, token_ids, n_tokens, span_offsets, n_spans, w, surrogates, workspace,
                      dev_status, stream, sms);
 }
@@ -199,7 +177,8 @@ umim_status umim_build_compressed(const void *embeddings, int64_t vocab, int32_t
     return UMIM_ERR_INVALID_ARG;
   if (!workspace || !aligned(workspace, 256) || workspace_bytes < build_compressed_workspace_bytes(batch, n_spans))
     return UMIM_ERR_WORKSPACE;
-  const int sms = prepare_device(stream);
+  const DeviceScope scope(stream);
+  const int sms = scope.sms();
   return build_compressed(embeddings, vocab, d_model, token_ids, batch, prompt_len, span_offsets, span_start,
                           span_len, n_spans, surrogates, out_embeds, out_capacity_rows, position_ids, cu_seqlens,
                           workspace, dev_status, stream, sms);
@@ -235,7 +214,8 @@ umim_status rollback_checked(const umim_paged_kv *kv, int32_t *block_table, int3
       workspace_bytes < kv_rollback_workspace_bytes(batch, n_spans, max_pages, kv->n_layers, kv->n_kv_heads,
                                                     kv->head_dim))
     return UMIM_ERR_WORKSPACE;
-  const int sms = prepare_device(stream);
+  const DeviceScope scope(stream);
+  const int sms = scope.sms();
   return kv_rollback(kv, block_table, max_pages, seq_lens, batch, span_offsets, span_start, span_len, n_spans,
                      surrogate_k, surrogate_v, freed_pages, workspace, workspace_bytes, dev_status, stream, sms,
                      rope_inv_freq, rotary_dim);
@@ -273,7 +253,7 @@ umim_status umim_kv_append(const umim_paged_kv *kv, int32_t *block_table, int32_
   if (batch == 0) return UMIM_OK;
   if (!block_table || !seq_lens || !new_k || !new_v) return UMIM_ERR_INVALID_ARG;
   if (!aligned(new_k, 16) || !aligned(new_v, 16)) return UMIM_ERR_INVALID_ARG;
-  prepare_device(stream);
+  const DeviceScope scope(stream);
   return kv_append(kv, block_table, max_pages, seq_lens, batch, new_k, new_v, new_pages, dev_status, stream);
 }
 
@@ -290,7 +270,7 @@ umim_status umim_decode_append_merge(const umim_paged_kv *kv, int32_t *block_tab
   if (!aligned(new_k, 16) || !aligned(new_v, 16)) return UMIM_ERR_INVALID_ARG;
   if (merge_k && n_merge_rows > 0 && (!merge_row || !surrogate_k || !surrogate_v)) return UMIM_ERR_INVALID_ARG;
   if (n_merge_rows > 0 && (!aligned(surrogate_k, 16) || !aligned(surrogate_v, 16))) return UMIM_ERR_INVALID_ARG;
-  prepare_device(stream);
+  const DeviceScope scope(stream);
   return decode_append_merge(kv, block_table, max_pages, seq_lens, batch, new_k, new_v, new_pages, merge_k,
                              merge_row, n_merge_rows, surrogate_k, surrogate_v, released_pages, dev_status, stream);
 }
@@ -305,7 +285,8 @@ umim_status umim_rules_build(void *table, size_t table_bytes, const int32_t *rul
   if (n_rules < 0 || n_rules > kMaxRules || !table_ok(table, table_bytes)) return UMIM_ERR_INVALID_ARG;
   if ((uint64_t)table_bytes < 24ull * (uint64_t)n_rules) return UMIM_ERR_WORKSPACE;
   if (n_rules > 0 && (!rule_tokens || !aligned(rule_tokens, 16))) return UMIM_ERR_INVALID_ARG;
-  const int sms = prepare_device(stream);
+  const DeviceScope scope(stream);
+  const int sms = scope.sms();
   return rules_build(table, table_bytes, rule_tokens, n_rules, dev_status, stream, sms);
 }
 
@@ -322,7 +303,8 @@ umim_status umim_match_prompts(const void *table, size_t table_bytes, const int3
   if (!table_ok(table, table_bytes) || batch < 0 || max_len < 0 || !span_offsets) return UMIM_ERR_INVALID_ARG;
   if ((int64_t)batch * max_len >= INT32_MAX) return UMIM_ERR_UNSUPPORTED;
   if ((merge_token_ids == nullptr) != (merge_offsets == nullptr)) return UMIM_ERR_INVALID_ARG;
-  const int sms = prepare_device(stream);
+  const DeviceScope scope(stream);
+  const int sms = scope.sms();
   if (batch == 0) {
     if (cudaMemsetAsync(span_offsets, 0, sizeof(int32_t), stream) != cudaSuccess) return UMIM_ERR_CUDA;
     if (merge_offsets && cudaMemsetAsync(merge_offsets, 0, sizeof(int32_t), stream) != cudaSuccess)
@@ -342,7 +324,7 @@ umim_status umim_match_suffix(const void *table, size_t table_bytes, umim_suffix
                               cudaStream_t stream) {
   static_assert(sizeof(umim_suffix_state) == 16, "suffix state is one 16-byte vector");
   if (!table_ok(table, table_bytes) || batch < 0) return UMIM_ERR_INVALID_ARG;
-  prepare_device(stream);
+  const DeviceScope scope(stream);
   if (batch == 0) {
     if (n_merges && cudaMemsetAsync(n_merges, 0, sizeof(int32_t), stream) != cudaSuccess) return UMIM_ERR_CUDA;
     return UMIM_OK;
@@ -359,7 +341,8 @@ umim_status umim_lookup_surrogates(const float *lut, int64_t n_rules, int32_t d,
   if (n_rules < 0 || d <= 0 || d % 4 != 0 || n_max < 0) return UMIM_ERR_INVALID_ARG;
   if (n_max == 0) return UMIM_OK;
   if (!lut || !aligned(lut, 16) || !rule_ids || !out || !aligned(out, 16)) return UMIM_ERR_INVALID_ARG;
-  const int sms = prepare_device(stream);
+  const DeviceScope scope(stream);
+  const int sms = scope.sms();
   return lookup_surrogates(lut, n_rules, d, rule_ids, n_max, n_dev, out, dev_status, stream, sms);
 }
 
@@ -367,7 +350,7 @@ umim_status umim_selftest_bounded_wait(int32_t which, uint32_t limit_us, const i
                                        uint64_t *elapsed_ns, int32_t *dev_status, cudaStream_t stream) {
   if ((which != 0 && which != 1) || limit_us == 0 || limit_us > 1000000u) return UMIM_ERR_INVALID_ARG;
   if (which == 1 && !flags) return UMIM_ERR_INVALID_ARG;
-  prepare_device(stream);
+  const DeviceScope scope(stream);
   return selftest_bounded_wait(which, limit_us, flags, elapsed_ns, dev_status, stream);
 }
 
@@ -389,7 +372,8 @@ umim_status umim_prefill_attention(const void *q, const void *k, const void *v, 
   if (!workspace || !aligned(workspace, 256) ||
       workspace_bytes < prefill_attention_workspace_bytes(batch, n_rows, n_kv_heads, head_dim))
     return UMIM_ERR_WORKSPACE;
-  const int sms = prepare_device(stream);
+  const DeviceScope scope(stream);
+  const int sms = scope.sms();
   return prefill_attention(q, k, v, n_rows, n_q_heads, n_kv_heads, head_dim, cu_seqlens, batch, scale, out,
                            workspace, dev_status, stream, sms);
 }
@@ -405,7 +389,7 @@ umim_status umim_distill_align(const int32_t *seq_lens, int32_t batch, const int
                                int32_t capacity, int32_t *student_cu, void *workspace, size_t workspace_bytes,
                                int32_t *dev_status, cudaStream_t stream) {
   if (batch < 0 || n_spans < 0 || capacity < 0 || !pair_offsets) return UMIM_ERR_INVALID_ARG;
-  prepare_device(stream);
+  const DeviceScope scope(stream);
   if (batch == 0) {
     if (cudaMemsetAsync(pair_offsets, 0, sizeof(int32_t), stream) != cudaSuccess) return UMIM_ERR_CUDA;
     if (student_cu && cudaMemsetAsync(student_cu, 0, sizeof(int32_t), stream) != cudaSuccess) return UMIM_ERR_CUDA;
@@ -440,7 +424,8 @@ umim_status umim_distill_soft_ce(const void *teacher_logits, int32_t n_teacher_r
   if (!workspace || !aligned(workspace, 256) ||
       workspace_bytes < distill_soft_ce_workspace_bytes(n_student_rows, max_pairs))
     return UMIM_ERR_WORKSPACE;
-  const int sms = prepare_device(stream);
+  const DeviceScope scope(stream);
+  const int sms = scope.sms();
   return distill_soft_ce(teacher_logits, n_teacher_rows, student_logits, n_student_rows, vocab, ld, teacher_rows,
                          student_rows, max_pairs, n_pairs, eps, loss, pair_loss, grad, workspace, dev_status,
                          stream, sms);
@@ -466,7 +451,8 @@ umim_status umim_decode_attention(const void *q, int32_t n_q_heads, const umim_p
   if (batch == 0) return UMIM_OK;
   if (!q || !block_table || !seq_lens || !out) return UMIM_ERR_INVALID_ARG;
   if (!aligned(q, 4) || !aligned(out, 2)) return UMIM_ERR_INVALID_ARG;
-  const int sms = prepare_device(stream);
+  const DeviceScope scope(stream);
+  const int sms = scope.sms();
   if (!workspace || !aligned(workspace, 256) ||
       workspace_bytes < decode_attention_workspace_bytes(batch, n_q_heads, kv->n_kv_heads, kv->head_dim, sms))
     return UMIM_ERR_WORKSPACE;

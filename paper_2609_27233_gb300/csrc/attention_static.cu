@@ -70,14 +70,10 @@ umim_status umim_decode_attention_static(const void *q, int32_t n_q_heads, const
   if (!q || !block_table || !seq_lens || !out) return UMIM_ERR_INVALID_ARG;
   if ((reinterpret_cast<uintptr_t>(q) % 4) != 0 || (reinterpret_cast<uintptr_t>(out) % 2) != 0)
     return UMIM_ERR_INVALID_ARG;
-  // a stream being captured into a CUDA graph refuses cudaStreamGetDevice (the refusal would
-  // invalidate the capture): there the current device is the stream's
-  int dev = 0;
-  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
-  if (stream != nullptr && cudaStreamIsCapturing(stream, &cs) == cudaSuccess && cs == cudaStreamCaptureStatusNone &&
-      cudaStreamGetDevice(stream, &dev) == cudaSuccess) {
-    if (cudaSetDevice(dev) != cudaSuccess) return UMIM_ERR_CUDA;
-  }
+  // the stream's device is current until this call returns (the caller's current
+  // device is put back then); during a stream capture the current device is taken
+  // as the stream's
+  const DeviceScope scope(stream);
   void *scratch = nullptr;
   int sms = 0;
   const umim_status st = scratch_for_current_device(&scratch, &sms);

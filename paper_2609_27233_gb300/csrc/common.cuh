@@ -2,6 +2,7 @@
 // TMA (cp.async.bulk.tensor) and tcgen05 wrappers as inline PTX for sm_103a.
 #pragma once
 
+#include <atomic>
 #include <cstdint>
 #include <cuda.h>
 #include <cuda_runtime.h>
@@ -269,6 +270,51 @@ inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, siz
   cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
 }
+
+// SM count of a device, looked up once per device; atomics, since calls for
+// different devices may come from different host threads.
+inline int sm_count(int dev) {
+  static std::atomic<int> sms_of[64];
+  int sms = 0;
+  if (dev >= 0 && dev < 64) sms = sms_of[dev].load(std::memory_order_relaxed);
+  if (sms == 0) {
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) sms = 0;
+    if (sms > 0 && dev >= 0 && dev < 64) sms_of[dev].store(sms, std::memory_order_relaxed);
+  }
+  return sms;
+}
+
+// For the duration of one library call: makes the stream's device current and
+// puts the caller's current device back when the call returns.  A stream being
+// captured into a CUDA graph refuses cudaStreamGetDevice (and the refusal would
+// invalidate the capture), so during a capture the current device is taken as
+// the stream's.
+class DeviceScope {
+ public:
+  explicit DeviceScope(cudaStream_t stream) {
+    int cur = -1;
+    if (cudaGetDevice(&cur) != cudaSuccess) cur = -1;
+    dev_ = cur;
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    int sdev = -1;
+    if (stream != nullptr && cudaStreamIsCapturing(stream, &cs) == cudaSuccess && cs == cudaStreamCaptureStatusNone &&
+        cudaStreamGetDevice(stream, &sdev) == cudaSuccess && sdev != cur && cudaSetDevice(sdev) == cudaSuccess) {
+      prev_ = cur;
+      dev_ = sdev;
+    }
+    sms_ = dev_ >= 0 ? sm_count(dev_) : 0;
+  }
+  ~DeviceScope() {
+    if (prev_ >= 0) cudaSetDevice(prev_);
+  }
+  DeviceScope(const DeviceScope &) = delete;
+  DeviceScope &operator=(const DeviceScope &) = delete;
+  int device() const { return dev_; }
+  int sms() const { return sms_; }
+
+ private:
+  int dev_ = -1, prev_ = -1, sms_ = 0;
+};
 
 // Kernel tracing (trace.cu): records an event labelled with the next kernel,
 // or, with a null label, the end of a call.  No-op unless a trace is active.

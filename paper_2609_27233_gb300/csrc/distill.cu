@@ -833,20 +833,7 @@ bool ce_try_layout(int64_t V, int T, int C, int num_sms, CeLayout &L) {
 // the one with more threads resident wins -- cluster placement within a GPC
 // can leave SMs idle (on a GB300 at the Llama-3 vocabulary: 14 clusters of
 // 16 x 256 threads on 112 SMs, 15 clusters of 8 x 512 on 120).
-// UMIM_SOFT_CE_LAYOUT="T,C" picks a layout (for measurements).
 bool ce_layout(int64_t V, int num_sms, CeLayout &L) {
-  static int env_T = -1, env_C = -1;
-  static std::once_flag once;
-  std::call_once(once, [] {
-    const char *e = getenv("UMIM_SOFT_CE_LAYOUT");
-    int t = 0, c = 0;
-    if (e && sscanf(e, "%d,%d", &t, &c) == 2 && (t == 256 || t == 512) && c >= 1 && c <= kCeMaxCluster &&
-        (c & (c - 1)) == 0) {
-      env_T = t;
-      env_C = c;
-    }
-  });
-  if (env_T > 0 && ce_try_layout(V, env_T, env_C, num_sms, L)) return true;
   // per thread count, the fewest CTAs per row with <= 4 vectors per thread (5 at the largest cluster)
   CeLayout best{};
   bool found = false;

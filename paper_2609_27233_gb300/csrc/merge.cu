@@ -656,13 +656,11 @@ static umim_status launch_gemm(EncodeTiledFn enc, const void *A, int64_t M, cons
   g.cvt_out = static_cast<uint4 *>(cvt_out);
   g.cvt_n = cvt_n;
   g.status = status;
-  static bool attr_done = false;
-  if (!attr_done) {
-    if (cudaFuncSetAttribute(gemm_bias_gelu_kernel<OutT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             kGemmSmem) != cudaSuccess)
-      return UMIM_ERR_CUDA;
-    attr_done = true;
-  }
+  // set on every call: the attribute belongs to the current device, and calls may
+  // come for several devices and from several threads
+  if (cudaFuncSetAttribute(gemm_bias_gelu_kernel<OutT>, cudaFuncAttributeMaxDynamicSharedMemorySize, kGemmSmem) !=
+      cudaSuccess)
+    return UMIM_ERR_CUDA;
   const int64_t tiles = (int64_t)(d / BN) * ((M + BM - 1) / BM);
   const int grid = (int)std::min<int64_t>(tiles, std::max(1, num_sms));
   trace_mark(st, label);

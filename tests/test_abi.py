@@ -186,3 +186,11 @@ def test_other_entry_points_host_checks(lib):
     assert lib.umim_selftest_bounded_wait(0, 0, null, null, null, null) == 1
     assert lib.umim_selftest_bounded_wait(0, 2000000, null, null, null, null) == 1
     assert lib.umim_selftest_bounded_wait(1, 1000, null, null, null, null) == 1   # flags needed
+
+
+def test_binding_scratch_size_matches_the_header():
+    text = open(os.path.join(ROOT, "include", "umim.h")).read()
+    m = re.search(r"#define UMIM_STATIC_SCRATCH_BYTES \((\d+)u << (\d+)\)", text)
+    assert m
+    import paper_2609_27233_gb300 as umim
+    assert umim.STATIC_SCRATCH_BYTES == int(m.group(1)) << int(m.group(2))

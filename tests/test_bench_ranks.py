@@ -76,8 +76,10 @@ def _run_bench(args, env_extra):
 def test_reference_arm_prints_one_line_with_the_contract_keys():
     """The oracle arm runs on the host cores only and prints one JSON line
     on the same metric, unit and workload as the GPU arm."""
-    (line,) = _run_bench(["--impl", "reference", "--steps", "1", "--warmup", "3"], {})
+    (line,) = _run_bench(["--impl", "reference", "--steps", "2", "--warmup", "3"], {})
     assert line["impl"] == "reference"
+    # the steps it reports were timed, not extrapolated: they fit in the run's own wall time
+    assert line["steps"] == 2 and line["ms_per_step"] * line["steps"] <= 1000.0 * line["wall_s"] + 1.0
     assert line["metric"] == bench.METRIC and line["unit"] == bench.UNIT
     assert line["higher_is_better"] is True and line["value"] > 0
     assert line["config"]["workload"].startswith("llama8b_layer")

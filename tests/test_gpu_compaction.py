@@ -61,8 +61,9 @@ def test_capacity_too_small_writes_nothing():
 
 
 def test_prompt_compression_full_size():
-    """64 x 2048 prompts, 128256 x 4096 table, 40 % coverage: every index
-    output compared, embedding rows of prompts 0, 31 and 63 compared."""
+    """64 x 2048 prompts, 128256 x 4096 table, 40 % coverage: position ids
+    and cu_seqlens of all 64 prompts compared with the oracle, embedding rows
+    of prompts 0, 31 and 63 compared."""
     seed = W.SEEDS["prompt_compression"]
     d = dev()
     table = W.bf16_normal((128256, 4096), 0.02, seed + 101, d)
@@ -88,7 +89,13 @@ def test_prompt_compression_full_size():
         assert cu_h[b + 1] - cu_h[b] == rcu[-1]
         np.testing.assert_array_equal(pos[cu_h[b]:cu_h[b + 1]].cpu().numpy(), rpos)
         np.testing.assert_array_equal(W.bits(emb[cu_h[b]:cu_h[b + 1]].cpu()), re)
-    # lengths of every prompt
+    # position ids and cu_seqlens of every prompt: they do not depend on the
+    # embedding width, so the oracle runs on a one-column table
+    narrow = np.zeros((128256, 1), dtype=np.uint16)
+    _, rpos_all, rcu_all = oracle.build_compressed(narrow, ids, offs, st_, ln_,
+                                                   np.zeros((len(st_), 1), np.float32))
+    np.testing.assert_array_equal(cu_h, rcu_all)
+    np.testing.assert_array_equal(pos[:cu_h[-1]].cpu().numpy(), rpos_all)
     for b in range(64):
         lo, hi = offs[b], offs[b + 1]
         assert cu_h[b + 1] - cu_h[b] == 2048 - int((ln_[lo:hi] - 1).sum())

@@ -53,3 +53,68 @@ def test_batch_too_large_for_the_scratch_array_is_refused():
         m.umim_decode_attention_static(q, pool, 0, bt, lens)
     assert e.value.code == 5   # UMIM_ERR_WORKSPACE
 
+
+
+def _largest_batch_that_fits(m, Hq, Hkv, D):
+    """The largest batch whose scratch, sized like the workspace of
+    umim_decode_attention on this device, fits in the library's array."""
+    lo, hi = 1, 1
+    while m.umim_decode_attention_workspace_size(hi, Hq, Hkv, D) <= m.STATIC_SCRATCH_BYTES:
+        lo, hi = hi, 2 * hi
+    while hi - lo > 1:
+        mid = (lo + hi) // 2
+        if m.umim_decode_attention_workspace_size(mid, Hq, Hkv, D) <= m.STATIC_SCRATCH_BYTES:
+            lo = mid
+        else:
+            hi = mid
+    return lo
+
+
+def test_batch_just_under_the_array_limit_matches_the_oracle():
+    """A batch whose plan and partials nearly fill the array (computed from the
+    workspace size at this device's SM count) still runs and matches the
+    oracle; one more sequence is refused."""
+    import numpy as np
+    import oracle
+    m = umim()
+    d = dev()
+    Hq, Hkv, D = 32, 8, 128
+    B = _largest_batch_that_fits(m, Hq, Hkv, D)
+    assert m.umim_decode_attention_workspace_size(B + 1, Hq, Hkv, D) > m.STATIC_SCRATCH_BYTES
+    lens = W.rng(303).integers(0, 70, size=B).tolist()
+    c = W.decode_case(303, lens=lens, n_q_heads=Hq, n_kv_heads=Hkv, head_dim=D, n_spans=[0] * B)
+    g = case_to_dev(c, d)
+    status = m.new_status(d)
+    got = m.umim_decode_attention_static(g["q"], g["pool"], 0, g["bt"], g["lens"], dev_status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    want = oracle.decode_attention(W.bits(c.q), W.bits(c.pool), 0, c.block_table.numpy(), c.seq_lens.numpy())
+    float_close(got.cpu().double().numpy(), want, "batch at the array limit")
+    q1 = torch.zeros((B + 1, Hq, D), dtype=torch.bfloat16, device=d)
+    bt1 = torch.zeros((B + 1, g["bt"].shape[1]), dtype=torch.int32, device=d)
+    l1 = torch.zeros(B + 1, dtype=torch.int32, device=d)
+    with pytest.raises(m.UmimError) as e:
+        m.umim_decode_attention_static(q1, g["pool"], 0, bt1, l1)
+    assert e.value.code == 5   # UMIM_ERR_WORKSPACE
+
+
+def test_warm_calls_reserve_no_device_memory_and_keep_the_current_device():
+    """After the first call on the device (the set-up), further calls leave the
+    device's free memory unchanged, and the caller's current device is the
+    same after each call."""
+    m = umim()
+    d = dev()
+    c = W.decode_case(304, lens=[300, 5, 1200], n_q_heads=16, n_kv_heads=4, head_dim=64, n_spans=[0] * 3)
+    g = case_to_dev(c, d)
+    out = torch.empty_like(g["q"])
+    status = m.new_status(d)
+    m.umim_decode_attention_static(g["q"], g["pool"], 0, g["bt"], g["lens"], out=out, dev_status=status)
+    torch.cuda.synchronize()
+    before_dev = torch.cuda.current_device()
+    free0 = torch.cuda.mem_get_info(d)[0]
+    for _ in range(3):
+        m.umim_decode_attention_static(g["q"], g["pool"], 0, g["bt"], g["lens"], out=out, dev_status=status)
+        assert torch.cuda.current_device() == before_dev
+    torch.cuda.synchronize()
+    assert torch.cuda.mem_get_info(d)[0] == free0
+    assert int(status.item()) == 0
