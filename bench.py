@@ -343,14 +343,15 @@ def main():
     ap.add_argument("--lut-rows", type=int, default=0,
                     help="rule_matching: keep only this many lookup-table rows (rule id mod rows), to bound "
                          "device memory under a profiler; 0 = one row per rule")
+    ap.add_argument("--serving-steps", type=int, default=256, help="serving: decode steps of the loop")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="default workload: skip the sub-runs of the other configurations")
     args = ap.parse_args()
-    if args.workload == "serving" and args.impl == "umim":
-        return serving_bench(args)
-    if args.workload == "tiny" and args.impl == "umim":
-        return tiny_bench(args)
-    if args.workload in ("prompt_compression", "long_context", "rule_matching", "prefill", "distill") and \
-            args.impl == "umim":
-        return side_bench(args)
+    side = {"serving": serving_bench, "tiny": tiny_bench, "prompt_compression": side_bench,
+            "long_context": side_bench, "rule_matching": side_bench, "prefill": side_bench, "distill": side_bench}
+    if args.workload in side and args.impl == "umim":
+        print(json.dumps(side[args.workload](args)))
+        return 0
     K, Wm = args.steps, max(3, args.warmup)
 
     rank = int(os.environ.get("RANK", "0"))
@@ -384,6 +385,22 @@ def main():
         print(json.dumps(line))
         return 0
 
+    line = headline(args, K, Wm, rank, world, local, peaks)
+    if rank == 0:
+        if world == 1 and not args.no_configs:
+            import torch
+            torch.cuda.empty_cache()
+            line["configs"] = config_runs(args)
+        print(json.dumps(line))
+    if world > 1:
+        import torch
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+def headline(args, K, Wm, rank, world, local, peaks):
+    """The default step (merge -> rollback -> attention on the Llama-8B layer),
+    timed on this rank; rank 0 gets the contract line, other ranks None."""
     import torch
     import paper_2609_27233_gb300 as umim
     import workloads as W
@@ -633,13 +650,74 @@ def main():
                               "frac_of_8tbs_nominal": round(att_gbs / 7900.0, 4)},
                 "roofline": roof, "kernels": kernels, "cpu_baseline": cpu, "e2e": e2e,
                 "gpu_launches": int(round(launches_per_step * K)), "clocks": clocks,
-                "traced_ms_per_step": tms / K}
+                "traced_ms_per_step": tms / K, "targets": _targets(kernels)}
         if args.rope:
             line["config"]["rope"] = "moved keys re-rotated to their compressed positions (umim_kv_rollback_rope)"
-        print(json.dumps(line))
-    if world > 1:
-        torch.distributed.destroy_process_group()
-    return 0
+        return line
+    return None
+
+
+def _targets(kernels, att_key="attention.decode", rb_key="rollback.move"):
+    t = {}
+    if att_key in kernels and "frac" in kernels[att_key]:
+        t["attention_frac_of_hbm"] = kernels[att_key]["frac"]
+        t["attention_target"] = 0.70
+        t["attention_met"] = kernels[att_key]["frac"] >= 0.70
+    if rb_key in kernels and "frac" in kernels[rb_key]:
+        t["rollback_frac_of_hbm"] = kernels[rb_key]["frac"]
+        t["rollback_target"] = 0.60
+        t["rollback_met"] = kernels[rb_key]["frac"] >= 0.60
+    return t
+
+
+def config_runs(args):
+    """Sub-runs of the other configurations, each timed like its own
+    --workload run (CUDA events around the timed steps, clocks sampled
+    during them, per-kernel times from a traced repeat), bounded so that the
+    default bench stays within a couple of minutes.  Returns one record per
+    configuration; a sub-run that fails records its error instead."""
+    import copy
+    import gc
+    import torch
+    runs = [
+        ("tiny", dict(workload="tiny", steps=50, warmup=5)),
+        ("prompt_compression", dict(workload="prompt_compression", steps=10, warmup=3)),
+        ("long_context_cov40", dict(workload="long_context", coverage=0.4, steps=20, warmup=3)),
+        ("long_context_cov60", dict(workload="long_context", coverage=0.6, steps=20, warmup=3)),
+        ("serving", dict(workload="serving", serving_steps=32, warmup=3)),
+    ]
+    out = {}
+    for name, kw in runs:
+        ns = copy.copy(args)
+        ns.rope = False
+        for k, v in kw.items():
+            setattr(ns, k, v)
+        t0 = time.time()
+        try:
+            fn = {"tiny": tiny_bench, "serving": serving_bench}.get(ns.workload, side_bench)
+            line = fn(ns)
+            rec = {k: line[k] for k in ("metric", "value", "unit", "steps", "warmup", "ms_per_step", "clocks",
+                                        "roofline", "gpu_launches", "config", "kernels", "attention")
+                   if k in line}
+            if ns.workload == "serving":
+                rec["targets"] = {"attention_frac_of_hbm_averaged": line["attention"]["frac_of_hbm"],
+                                  "attention_target": 0.70,
+                                  "attention_met": line["attention"]["frac_of_hbm"] >= 0.70}
+                for k in ("rollbacks", "rollbacks_per_s", "fused_append_merge", "fused_graph", "per_layer_fused"):
+                    if k in line:
+                        rec[k] = line[k]
+            elif ns.workload == "tiny":
+                rec["targets"] = {"note": "latency case (one 512-token sequence): parity and microseconds per "
+                                          "step; no kernel is large enough to approach a roofline"}
+            else:
+                rec["targets"] = _targets(line.get("kernels", {}))
+        except Exception as ex:   # keep the headline and the other records
+            rec = {"error": f"{type(ex).__name__}: {str(ex)[:300]}"}
+        rec["wall_s"] = round(time.time() - t0, 1)
+        out[name] = rec
+        gc.collect()
+        torch.cuda.empty_cache()
+    return out
 
 
 def serving_plan(sl):
@@ -691,7 +769,7 @@ def serving_bench(args):
     umim.lib()
     peaks = load_peaks()
     sl = W.serving_loop(W.SEEDS["serving"], B=128, n_layers=32, n_q_heads=32, n_kv_heads=8, head_dim=128,
-                        steps=256, p=0.1)
+                        steps=args.serving_steps, p=0.1)
     plan = serving_plan(sl)
     B, NL = sl.B, sl.n_layers
     t = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev)
@@ -849,6 +927,13 @@ def serving_bench(args):
             "rollbacks": n_roll, "rollbacks_per_s": n_roll / (ms / 1000.0),
             "attention": {"gbs": round(att_gbs, 1), "frac_of_hbm": round(att_gbs / peaks["hbm"], 4),
                           "peak": peaks["hbm"], "peak_source": peaks["src"] + " HBM copy"},
+            "roofline": {"kernel": "attention.decode", "bound": "hbm", "achieved": round(att_gbs, 2),
+                         "peak": peaks["hbm"], "unit": "GB/s", "frac": round(att_gbs / peaks["hbm"], 4),
+                         "traffic": None, "algorithmic_per_launch": att_bytes / max(1, len(kern.get(
+                             "attention.decode", [1]))),
+                         "peak_source": peaks["src"] + " HBM copy",
+                         "what": "every attention launch of the loop: algorithmic bytes of all launches over "
+                                 "their summed traced time"},
             "kernels": {k: {"launches": len(v), "ms_total": round(float(np.sum(v)), 3),
                             "us_mean": round(1000 * float(np.mean(v)), 2)} for k, v in
                         sorted(kern.items(), key=lambda x: -np.sum(x[1]))},
@@ -863,8 +948,7 @@ def serving_bench(args):
                 "kernels": {k: {"launches": len(v), "ms_total": round(float(np.sum(v)), 3),
                                 "us_mean": round(1000 * float(np.mean(v)), 2)} for k, v in
                             sorted(f_kern.items(), key=lambda x: -np.sum(x[1]))}}}
-    print(json.dumps(line))
-    return 0
+    return line
 
 
 def kernel_table(recs, K, work_of):
@@ -1226,8 +1310,7 @@ def side_bench(args):
             "clocks": clk.summary(w0, w1),
             "traced_ms_per_step": tms / K, "peaks": {"hbm_gbs": peaks["hbm"], "bf16_tflops": peaks["bf16"],
                                                      "source": peaks["src"]}}
-    print(json.dumps(line))
-    return 0
+    return line
 
 
 def tiny_bench(args):
@@ -1358,8 +1441,7 @@ def tiny_bench(args):
                        "l2": "flushed before every timed step (256 MB write outside the timed interval)"},
             "kernels": kernels, "gpu_launches": len(recs), "clocks": clk.summary(w0, w1),
             "traced_ms_per_step": float(np.sum([v for _, v in recs])) / K}
-    print(json.dumps(line))
-    return 0
+    return line
 
 
 def llama3_inv_freq(D, dev):
