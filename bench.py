@@ -909,6 +909,44 @@ def serving_bench(args):
     umim.check_status(status, "graph loop")
     assert np.array_equal(lens.cpu().numpy(), plan[-1]["lens_after"]), "graph loop: lengths differ"
     fused[0] = False
+    # the per-layer decode step: one launch per layer writes that layer's new (or surrogate) entry and
+    # runs its attention over the updated cache; the last layer's launch commits tables and lengths
+    ws_s = umim.workspace(umim.umim_decode_layer_step_workspace_size(B, sl.n_kv_heads, sl.head_dim), dev)
+    sur_pl = [[(sk_[:, layer].contiguous(), sv_[:, layer].contiguous()) for layer in range(NL)]
+              for (sk_, sv_) in surs]
+
+    def layer_step(s):
+        nk, nv = entries[s]
+        dp = d_plan[s]
+        for layer in range(NL):
+            umim.umim_decode_layer_step(qs[layer], pool, layer, bt, lens, nk[:, layer], nv[:, layer],
+                                        dp["new_pages"], dp["merge_k"], dp["merge_row"], sur_pl[s][layer][0],
+                                        sur_pl[s][layer][1], commit=layer == NL - 1, released=released,
+                                        out=outs[layer], workspace_buf=ws_s, dev_status=status)
+
+    reset()
+    for s_ in range(max(3, args.warmup)):
+        layer_step(s_)
+    torch.cuda.synchronize()
+    umim.check_status(status, "per-layer warm-up")
+    reset()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for s_ in range(sl.steps):
+        layer_step(s_)
+    e1.record()
+    torch.cuda.synchronize()
+    pl_ms = e0.elapsed_time(e1)
+    umim.check_status(status, "per-layer loop")
+    assert np.array_equal(lens.cpu().numpy(), plan[-1]["lens_after"]), "per-layer loop: lengths differ"
+    reset()
+    umim.trace_start(200 * sl.steps)
+    for s_ in range(sl.steps):
+        layer_step(s_)
+    umim.trace_stop()
+    pl_kern = {}
+    for lab, v in umim.trace_read(200 * sl.steps):
+        pl_kern.setdefault(lab, []).append(v)
     entry = 2 * sl.n_kv_heads * sl.head_dim * 2
     att_bytes = sum(float(x["lens_after"].sum()) * entry + 2 * B * sl.n_q_heads * sl.head_dim * 2
                     for x in plan) * NL
@@ -943,6 +981,17 @@ def serving_bench(args):
                             "what": "the fused loop with each step replaying one captured CUDA graph (update + "
                                     "32 layers of attention, 97 kernels) after copying the step's inputs into "
                                     "its static buffers"},
+            "per_layer_fused": {
+                "value": B * sl.steps / (pl_ms / 1000.0), "unit": "tokens/s", "ms_per_step": pl_ms / sl.steps,
+                "what": "one umim_decode_layer_step launch per layer (the layer's new or surrogate entry written "
+                        "and its split-K attention over the updated cache, partial results merged in the same "
+                        "launch; the last layer's launch commits tables and lengths): 32 launches per step",
+                "attention_gbs": round((att_bytes + B * NL * entry * sl.steps) / 1e9 /
+                                       (float(np.sum(pl_kern.get("decode_step.layer", [0.0]) +
+                                                     pl_kern.get("decode_step.commit", [0.0]))) / 1000.0), 1),
+                "kernels": {k: {"launches": len(v), "ms_total": round(float(np.sum(v)), 3),
+                                "us_mean": round(1000 * float(np.mean(v)), 2)} for k, v in
+                            sorted(pl_kern.items(), key=lambda x: -np.sum(x[1]))}},
             "fused_append_merge": {
                 "value": B * sl.steps / (f_ms / 1000.0), "unit": "tokens/s", "ms_per_step": f_ms / sl.steps,
                 "kernels": {k: {"launches": len(v), "ms_total": round(float(np.sum(v)), 3),

@@ -305,6 +305,65 @@ umim_status umim_decode_append_merge(const umim_paged_kv *kv, int32_t *block_tab
                                      int32_t *released_pages, int32_t *dev_status, cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
+ * One layer of a decode step with decoding-time merging, in one launch
+ * (App. E "Decoding-Time Merging and KV-Cache Update"; Fig. 2 steps (2) and
+ * (3); App. I.1 on the overhead of many small kernel launches per step).
+ * A forward pass produces layer l's new K/V entry only after layer l - 1's
+ * attention, so a decode step calls this once per layer, in layer order,
+ * with that layer's new entries, query and (for merging sequences)
+ * surrogate entries.  Per sequence b, with L = seq_lens[b] as it was before
+ * the step and k = merge_k[b] (0 when merge_k is NULL):
+ *   k == 0      the new entry new_k/new_v[b] is written at slot s = L
+ *               (at a page boundary into page new_pages[b]);
+ *   k in 1..16  the forwarded token completes a merge of the last k tokens
+ *               (the k - 1 cached entries before it and itself): surrogate
+ *               row merge_row[b] is written at slot s = L + 1 - k;
+ * and out[b] is decode attention of q[b] over slots [0, s] of layer `layer`
+ * (the entry just written included).  Layer by layer this equals
+ * umim_decode_append_merge followed by umim_decode_attention.
+ * Block tables and lengths are read, not changed, by every call of the step
+ * except the one with `commit` != 0, which must be the step's last call (its
+ * last layer): once every CTA of that launch has finished reading them, it
+ * records new_pages[b] in the block table when L % 16 == 0, releases the
+ * page that no longer holds an entry (set to -1, reported in
+ * released_pages[b], -1 if none; at most one) and sets seq_lens[b] = s + 1.
+ *
+ * q                 device bf16 [batch][n_q_heads][head_dim] (this layer)
+ * new_k/new_v       device bf16: row b at new_k + b * new_row_stride elements,
+ *                   n_kv_heads * head_dim values (this layer), 16-B aligned;
+ *                   new_row_stride 0 means n_kv_heads * head_dim, otherwise a
+ *                   multiple of 8 not below it (rows inside a fused QKV
+ *                   projection output, or one layer of a [batch][layers][...]
+ *                   array)
+ * new_pages         device int32 [batch] or NULL (read at page boundaries)
+ * merge_k, merge_row  device int32 [batch] or NULL (no merges)
+ * surrogate_k/v     device bf16 [n_merge_rows][n_kv_heads][head_dim] (this layer)
+ * released_pages    device int32 [batch] out (commit call), or NULL
+ * out               device bf16 [batch][n_q_heads][head_dim], 4-B aligned
+ * workspace         device, umim_decode_layer_step_workspace_size() bytes,
+ *                   256-B aligned, ZEROED before its first use; each call
+ *                   leaves it ready for the next.  After a call that reported
+ *                   UMIM_ERR_TIMEOUT, zero it again.  Calls sharing one
+ *                   workspace must not overlap on the GPU.
+ * Host-side errors: UMIM_ERR_UNSUPPORTED for batch > 4096 or the shapes
+ * umim_decode_attention does not support.  Device-side errors:
+ * UMIM_ERR_INVALID_ARG when seq_lens[b] is outside [0, 16*max_pages), k is
+ * outside [0, min(16, L + 1)], merge_row[b] is outside [0, n_merge_rows), or
+ * a page to write is outside [0, n_pages): that sequence is left unchanged
+ * (nothing written, not committed) and its output is attention over its
+ * unchanged cache; UMIM_ERR_TIMEOUT for a stalled copy.
+ * ------------------------------------------------------------------------ */
+size_t umim_decode_layer_step_workspace_size(int32_t batch, int32_t n_kv_heads, int32_t head_dim);
+
+umim_status umim_decode_layer_step(const void *q, int32_t n_q_heads, const umim_paged_kv *kv, int32_t layer,
+                                   int32_t *block_table, int32_t max_pages, int32_t *seq_lens, int32_t batch,
+                                   const void *new_k, const void *new_v, int64_t new_row_stride,
+                                   const int32_t *new_pages, const int32_t *merge_k, const int32_t *merge_row,
+                                   int32_t n_merge_rows, const void *surrogate_k, const void *surrogate_v,
+                                   int32_t commit, int32_t *released_pages, float scale, void *out, void *workspace,
+                                   size_t workspace_bytes, int32_t *dev_status, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
  * Grouped-query decode attention over the (compacted) paged cache, one
  * query token per sequence (App. I.1; the backbone's ordinary attention):
  *   out[b][h] = sum_{j < seq_lens[b]} softmax_j(scale <q[b][h], K[b][g][j]>) V[b][g][j]

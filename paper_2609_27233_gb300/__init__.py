@@ -11,6 +11,8 @@ points keep the C names:
   umim_kv_append          decode-step append of one KV entry per layer (App. E, Fig. 2)
   umim_decode_append_merge  append or suffix merge per sequence in one call (App. E decoding loop)
   umim_decode_attention   GQA decode attention over the compacted paged cache (App. I.1)
+  umim_decode_layer_step  one layer of a decode step: its new or surrogate entry written and
+                          attention over the updated cache in one launch (App. E, App. I.1)
   umim_prefill_attention  causal GQA attention over the packed compressed prompts (App. E, App. C.5)
   umim_rules_build, umim_match_prompts, umim_match_suffix, umim_lookup_surrogates
                           merge-rule table, longest-first span selection for prompts
@@ -246,6 +248,43 @@ def umim_decode_attention(q, pool, layer, block_table, seq_lens, scale=0.0, out=
                                        _p(seq_lens), B, float(scale), _p(out), _p(workspace_buf),
                                        workspace_buf.numel(), _p(dev_status), _stream(stream))
     _check(code, "umim_decode_attention")
+    return out
+
+
+def umim_decode_layer_step_workspace_size(batch, n_kv_heads, head_dim):
+    return lib().umim_decode_layer_step_workspace_size(batch, n_kv_heads, head_dim)
+
+
+def umim_decode_layer_step(q, pool, layer, block_table, seq_lens, new_k, new_v, new_pages=None, merge_k=None,
+                           merge_row=None, surrogate_k=None, surrogate_v=None, commit=False, released=None,
+                           scale=0.0, out=None, workspace_buf=None, dev_status=None, stream=None):
+    """One layer of a decode step: writes this layer's new (or, for a merging
+    sequence, surrogate) entry and returns out [B][Hq][D] bf16, attention of q
+    over the cache with that entry.  new_k / new_v are [B][Hkv][D] views whose
+    rows may be strided (e.g. one layer of [B][layers][Hkv][D]); surrogate_k /
+    surrogate_v are [rows][Hkv][D].  commit=True on the step's last layer
+    records the new lengths, opened pages and released pages.  workspace_buf
+    must be zeroed before its first use (workspace() zeroes it)."""
+    dev = _dev(q)
+    kv = paged_kv(pool)
+    B, Hq, D = q.shape
+    for t in (new_k, new_v):
+        if t.dtype != torch.bfloat16 or t.dim() != 3 or t.shape[0] != B or t.stride(2) != 1 or \
+                t.stride(1) != t.shape[2]:
+            raise ValueError("new_k / new_v must be bf16 [B][Hkv][D] with contiguous rows")
+    if new_k.stride(0) != new_v.stride(0):
+        raise ValueError("new_k and new_v must have the same row stride")
+    if out is None:
+        out = torch.empty_like(q)
+    if workspace_buf is None:
+        workspace_buf = workspace(umim_decode_layer_step_workspace_size(B, kv.n_kv_heads, D), dev)
+    n_rows = 0 if surrogate_k is None else surrogate_k.shape[0]
+    code = lib().umim_decode_layer_step(_p(q), Hq, ctypes.byref(kv), layer, _p(block_table), block_table.shape[1],
+                                        _p(seq_lens), B, _p(new_k), _p(new_v), new_k.stride(0), _p(new_pages),
+                                        _p(merge_k), _p(merge_row), n_rows, _p(surrogate_k), _p(surrogate_v),
+                                        1 if commit else 0, _p(released), float(scale), _p(out), _p(workspace_buf),
+                                        workspace_buf.numel(), _p(dev_status), _stream(stream))
+    _check(code, "umim_decode_layer_step")
     return out
 
 

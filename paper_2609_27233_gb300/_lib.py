@@ -51,6 +51,10 @@ SIGNATURES = {
                                       c_ptr, c_ptr]),
     "umim_decode_append_merge": (ctypes.c_int, [ctypes.POINTER(PagedKVC), c_ptr, c_i32, c_ptr, c_i32, c_ptr, c_ptr,
                                                 c_ptr, c_ptr, c_ptr, c_i32, c_ptr, c_ptr, c_ptr, c_ptr, c_ptr]),
+    "umim_decode_layer_step_workspace_size": (c_size, [c_i32, c_i32, c_i32]),
+    "umim_decode_layer_step": (ctypes.c_int, [c_ptr, c_i32, ctypes.POINTER(PagedKVC), c_i32, c_ptr, c_i32, c_ptr,
+                                              c_i32, c_ptr, c_ptr, c_i64, c_ptr, c_ptr, c_ptr, c_i32, c_ptr, c_ptr,
+                                              c_i32, c_ptr, ctypes.c_float, c_ptr, c_ptr, c_size, c_ptr, c_ptr]),
     "umim_selftest_bounded_wait": (ctypes.c_int, [c_i32, ctypes.c_uint32, c_ptr, c_ptr, c_ptr, c_ptr]),
     "umim_prefill_attention_workspace_size": (c_size, [c_i32, c_i32, c_i32, c_i32]),
     "umim_prefill_attention": (ctypes.c_int, [c_ptr, c_ptr, c_ptr, c_i32, c_i32, c_i32, c_i32, c_ptr, c_i32,

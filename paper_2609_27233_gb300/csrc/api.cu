@@ -67,6 +67,12 @@ int distill_soft_ce_vecs(int64_t V);
 umim_status distill_soft_ce(const void *, int32_t, const void *, int32_t, int32_t, int64_t, const int32_t *,
                             const int32_t *, int32_t, const int32_t *, float, float *, float *, void *, void *,
                             int32_t *, cudaStream_t, int);
+int decode_step_max_batch();
+size_t decode_step_workspace_bytes(int B, int Hkv, int D, int num_sms);
+umim_status decode_layer_step(const void *, int, const umim_paged_kv *, int, int32_t *, int, int32_t *, int,
+                              const void *, const void *, int64_t, const int32_t *, const int32_t *, const int32_t *,
+                              int, const void *, const void *, int, int32_t *, float, void *, void *, int32_t *,
+                              cudaStream_t, int);
 size_t decode_attention_workspace_bytes(int B, int Hq, int Hkv, int D, int num_sms);
 umim_status decode_attention(const void *, int, const umim_paged_kv *, int, const int32_t *, int, const int32_t *,
                              int, float, void *, void *, int32_t *, cudaStream_t, int);
@@ -460,6 +466,45 @@ umim_status umim_decode_attention(const void *q, int32_t n_q_heads, const umim_p
   int32_t *status = dev_status;
   return decode_attention(q, n_q_heads, kv, layer, block_table, max_pages, seq_lens, batch, scale, out, workspace,
                           status, stream, sms);
+}
+
+size_t umim_decode_layer_step_workspace_size(int32_t batch, int32_t n_kv_heads, int32_t head_dim) {
+  if (batch < 0 || n_kv_heads <= 0 || (head_dim != 64 && head_dim != 128)) return 0;
+  int sms = current_sms();
+  if (sms <= 0) sms = 256;   // no device yet: size for the largest grid this library launches
+  return decode_step_workspace_bytes(batch, n_kv_heads, head_dim, sms);
+}
+
+umim_status umim_decode_layer_step(const void *q, int32_t n_q_heads, const umim_paged_kv *kv, int32_t layer,
+                                   int32_t *block_table, int32_t max_pages, int32_t *seq_lens, int32_t batch,
+                                   const void *new_k, const void *new_v, int64_t new_row_stride,
+                                   const int32_t *new_pages, const int32_t *merge_k, const int32_t *merge_row,
+                                   int32_t n_merge_rows, const void *surrogate_k, const void *surrogate_v,
+                                   int32_t commit, int32_t *released_pages, float scale, void *out, void *workspace,
+                                   size_t workspace_bytes, int32_t *dev_status, cudaStream_t stream) {
+  if (!kv_ok(kv) || batch < 0 || max_pages < 0 || n_q_heads <= 0 || n_merge_rows < 0 || new_row_stride < 0)
+    return UMIM_ERR_INVALID_ARG;
+  if (!kv_supported(kv)) return UMIM_ERR_UNSUPPORTED;
+  if (n_q_heads % kv->n_kv_heads != 0 || n_q_heads / kv->n_kv_heads > 16) return UMIM_ERR_UNSUPPORTED;
+  if (batch > decode_step_max_batch() || (int64_t)batch * max_pages > INT32_MAX / 16) return UMIM_ERR_UNSUPPORTED;
+  if (layer < 0 || layer >= kv->n_layers) return UMIM_ERR_INVALID_ARG;
+  if (batch == 0) return UMIM_OK;
+  const int64_t row = (int64_t)kv->n_kv_heads * kv->head_dim;
+  if (new_row_stride == 0) new_row_stride = row;
+  if (new_row_stride < row || new_row_stride % 8 != 0) return UMIM_ERR_INVALID_ARG;
+  if (!q || !block_table || !seq_lens || !out || !new_k || !new_v) return UMIM_ERR_INVALID_ARG;
+  if (!aligned(q, 4) || !aligned(out, 4) || !aligned(new_k, 16) || !aligned(new_v, 16)) return UMIM_ERR_INVALID_ARG;
+  if (merge_k && n_merge_rows > 0 && (!merge_row || !surrogate_k || !surrogate_v)) return UMIM_ERR_INVALID_ARG;
+  if (n_merge_rows > 0 && (!aligned(surrogate_k, 16) || !aligned(surrogate_v, 16))) return UMIM_ERR_INVALID_ARG;
+  const DeviceScope scope(stream);
+  const int sms = scope.sms();
+  if (!workspace || !aligned(workspace, 256) ||
+      workspace_bytes < decode_step_workspace_bytes(batch, kv->n_kv_heads, kv->head_dim, sms))
+    return UMIM_ERR_WORKSPACE;
+  if (!(scale > 0.f)) scale = 1.0f / sqrtf((float)kv->head_dim);
+  return decode_layer_step(q, n_q_heads, kv, layer, block_table, max_pages, seq_lens, batch, new_k, new_v,
+                           new_row_stride, new_pages, merge_k, merge_row, n_merge_rows, surrogate_k, surrogate_v,
+                           commit != 0, released_pages, scale, out, workspace, dev_status, stream, sms);
 }
 
 }  // extern "C"

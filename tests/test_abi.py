@@ -194,3 +194,31 @@ def test_binding_scratch_size_matches_the_header():
     assert m
     import paper_2609_27233_gb300 as umim
     assert umim.STATIC_SCRATCH_BYTES == int(m.group(1)) << int(m.group(2))
+
+
+def test_layer_step_host_checks(lib):
+    """The per-layer decode step refuses bad shapes and arguments on the host,
+    before the first CUDA call."""
+    from paper_2609_27233_gb300._lib import PagedKVC
+    null = ctypes.c_void_p(0)
+    fake = ctypes.c_void_p(1 << 20)      # never dereferenced: every call below stops at a host check
+    kv = PagedKVC(4096, 2, 4, 2, 16, 128)
+
+    def call(kv=kv, hq=8, layer=0, batch=2, stride=0, q=fake, out=fake, nk=fake, rows=0, mk=null):
+        return lib.umim_decode_layer_step(q, hq, ctypes.byref(kv), layer, fake, 4, fake, batch, nk, fake, stride,
+                                          null, mk, null, rows, null, null, 0, null, 0.0, out, null, 0, null, null)
+
+    assert lib.umim_decode_layer_step_workspace_size(128, 8, 128) > 0
+    assert lib.umim_decode_layer_step_workspace_size(128, 8, 96) == 0
+    assert call(kv=PagedKVC(0, 2, 4, 2, 16, 128)) == 1       # no pool
+    assert call(kv=PagedKVC(4096, 2, 4, 2, 16, 96)) == 2     # head_dim 96
+    assert call(hq=34) == 2                                  # 17 query heads per KV head
+    assert call(batch=4097) == 2                             # above the largest batch
+    assert call(layer=2) == 1                                # no such layer
+    assert call(stride=100) == 1                             # row stride below n_kv_heads * head_dim
+    assert call(stride=260) == 1                             # not a multiple of 8 elements
+    assert call(nk=null) == 1                                # no new entries
+    assert call(nk=ctypes.c_void_p((1 << 20) + 8)) == 1      # new entries not 16-byte aligned
+    assert call(out=ctypes.c_void_p((1 << 20) + 2)) == 1     # output not 4-byte aligned
+    assert call(rows=3, mk=fake) == 1                        # merges without surrogate arrays
+    assert call(batch=0) == 0                                # an empty batch is a no-op
