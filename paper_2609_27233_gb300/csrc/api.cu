@@ -142,6 +142,7 @@ umim_status umim_merge_spans(const void *embeddings, int64_t vocab, const int32_
   if (!w || n_spans < 0 || n_tokens < 0 || vocab <= 0) return UMIM_ERR_INVALID_ARG;
   if (!merge_supported(w->d_model, w->n_heads)) return UMIM_ERR_UNSUPPORTED;
   if (n_tokens > (int64_t)n_spans * UMIM_MAX_SPAN_TOKENS || n_tokens > INT32_MAX) return UMIM_ERR_INVALID_ARG;
+  if (n_tokens < n_spans) return UMIM_ERR_INVALID_ARG;   // every span has at least one token
   if (n_spans == 0) return UMIM_OK;
   if (!embeddings || !span_offsets || !surrogates || (n_tokens > 0 && !token_ids)) return UMIM_ERR_INVALID_ARG;
   if (!w->w_kv || !w->b_kv || !w->ln_kv_gamma || !w->ln_kv_beta || !w->query || !w->w_o || !w->b_o ||

@@ -48,8 +48,26 @@ struct GemmArgs {
   const uint4 *cvt_in;
   uint4 *cvt_out;
   int64_t cvt_n;
+  float cvt_scale;             // applied before the fp16 rounding of the side job
+  float acc_scale;             // applied to the accumulator before the bias (undoes an operand scaling)
+  int32_t *range_flag;         // set (with UMIM_ERR_UNSUPPORTED) when a value does not fit fp16
   int32_t *status;
 };
+
+// fp16's largest finite value is 65504; a value at or above it (or not
+// finite) cannot be stored in the fp16 intermediates of the merge module.
+constexpr float kF16Limit = 65504.f;
+
+// W_o is staged in fp16 multiplied by this power of two (GEMM2's accumulator is
+// multiplied back by its inverse, both exact): entries from 2^-22 up to
+// 65504 / 2^8 = 255.875 in magnitude keep a normal fp16 form, so bf16 weights
+// of that range are represented exactly.
+constexpr float kWoScale = 256.f;
+
+__device__ __forceinline__ void flag_range(int32_t *flag, int32_t *status) {
+  set_error(status, UMIM_ERR_UNSUPPORTED);
+  if (flag) *reinterpret_cast<volatile int32_t *>(flag) = 1;
+}
 
 // Persistent: each CTA walks tiles blockIdx.x, blockIdx.x + gridDim.x, ...
 // (n fastest, so CTAs running at the same time share the A block in L2).
@@ -182,6 +200,13 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           bf16x8_to_float(u[k], f);
           uint4 o;
           __half2 *hh = reinterpret_cast<__half2 *>(&o);
+          bool bad = false;
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            f[e] *= g.cvt_scale;
+            bad |= !(fabsf(f[e]) < kF16Limit);
+          }
+          if (bad) flag_range(g.range_flag, g.status);
 #pragma unroll
           for (int e = 0; e < 4; ++e) hh[e] = __floats2half2_rn(f[2 * e], f[2 * e + 1]);
           g.cvt_out[i] = o;
@@ -201,6 +226,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       }
       tc_fence_after();
       float mean = 0.f, m2 = 0.f, cnt = 0.f;
+      bool bad = false;
 #pragma unroll 1
       for (int c = 0; c < BN / 32; ++c) {
         float v[32];
@@ -213,8 +239,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           bf16x8_to_float(__ldg(bp + i), bb);
 #pragma unroll
           for (int e = 0; e < 8; ++e) {
-            v[8 * i + e] = gelu_erf(v[8 * i + e] + bb[e]);
+            v[8 * i + e] = gelu_erf(fmaf(v[8 * i + e], g.acc_scale, bb[e]));
             sum += v[8 * i + e];
+            bad |= !(fabsf(v[8 * i + e]) < kF16Limit);
           }
         }
         const float cm = sum * (1.f / 32.f);
@@ -232,6 +259,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         if (row < g.M) store32(g.out + (int64_t)row * g.N + n0 + c * 32, v);
       }
       if (row < g.M) g.stats[(int64_t)row * tiles_n + n0 / BN] = make_float2(mean, m2);
+      if (bad && row < g.M) flag_range(g.range_flag, g.status);   // this row's fp16 output overflowed
       // this warp's quarter of the accumulator has been read
       tc_fence_before();
       __syncwarp();
@@ -250,8 +278,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 // gather the static embeddings of the span tokens
 // ---------------------------------------------------------------------------
 __global__ void gather_rows_kernel(const uint4 *table, int64_t vocab, const int32_t *ids, int64_t T, int d,
-                                   uint4 *out, int32_t *status) {
+                                   uint4 *out, int32_t *range_flag, int32_t *status) {
   griddep_wait();
+  if (blockIdx.x == 0 && threadIdx.x == 0) *range_flag = 0;   // the first kernel of the call
   const int vec = d / 8;   // 16-byte vectors per row
   const int64_t warp = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const int64_t nwarps = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
@@ -333,7 +362,7 @@ template <int CH>
 __global__ void __launch_bounds__(kPoolConsumers + 32, CH <= 2 ? 2 : 1)
     pool_kernel(const __half *H, const float2 *stats, const int32_t *offs, int S, int64_t T, int d, int h,
                 const __nv_bfloat16 *gamma, const __nv_bfloat16 *beta, const __nv_bfloat16 *query, float eps,
-                __half *O, int32_t *status) {
+                __half *O, int32_t *range_flag, int32_t *status) {
   extern __shared__ __align__(128) uint8_t pool_smem[];
   __shared__ uint64_t full[kPoolRing], empty[kPoolRing];
   __shared__ int s_n[kPoolRing];
@@ -537,12 +566,15 @@ __global__ void __launch_bounds__(kPoolConsumers + 32, CH <= 2 ? 2 : 1)
         const float C = n > 0 ? s_C[head] : 0.f;
         uint4 packed;
         __half2 *hp = reinterpret_cast<__half2 *>(&packed);
+        bool bad = false;
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
           const float o0 = n > 0 ? fmaf(g[i][2 * e], x[2 * e] - C, b[i][2 * e]) : 0.f;
           const float o1 = n > 0 ? fmaf(g[i][2 * e + 1], x[2 * e + 1] - C, b[i][2 * e + 1]) : 0.f;
+          bad |= !(fabsf(o0) < kF16Limit) || !(fabsf(o1) < kF16Limit);
           hp[e] = __floats2half2_rn(o0, o1);
         }
+        if (bad) flag_range(range_flag, status);
         *reinterpret_cast<uint4 *>(O + (int64_t)s * d + cc * 8) = packed;
       }
     }
@@ -554,13 +586,291 @@ __global__ void __launch_bounds__(kPoolConsumers + 32, CH <= 2 ? 2 : 1)
 }
 
 // ---------------------------------------------------------------------------
+// LN_kv + attention pooling, one warp per (span, head) item: the default for
+// head widths up to 1024.  Warp w of the grid always takes head w mod h, so
+// its lanes keep that head's LayerNorm scale, shift and gamma*q in registers,
+// and walks the spans w / h, w / h + (warps / h), ...  Each warp owns two
+// shared-memory buffers: lane 0 bulk-copies the next item's rows of H (this
+// head's columns) and their per-tile statistics into one buffer while the
+// warp computes the current item from the other, so no CTA barrier is ever
+// taken.  The LayerNorm algebra is the one of pool_kernel above; a row's
+// (mean, M2) comes from its equal-count tiles as mean = avg(mean_t),
+// M2 = sum M2_t + 256 sum (mean_t - mean)^2.
+// ---------------------------------------------------------------------------
+constexpr int kHeadWarps = 12;
+constexpr int kHeadBufs = 2;
+
+// one buffer: [4][dh] fp16 rows, then [4][ntiles] float2 statistics; a multiple
+// of 128 bytes so that every buffer can take a tensor copy
+__host__ __device__ inline int head_buf_bytes(int dh, int ntiles) {
+  return (UMIM_MAX_SPAN_TOKENS * (dh * 2 + ntiles * 8) + 127) & ~127;
+}
+
+__device__ __forceinline__ void tma_load_3d(void *dst, const CUtensorMap *map, uint64_t *bar, int c0, int c1, int c2,
+                                            uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%2, %3, %4}], [%5], %6;" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(smem_u32(bar)), "l"(policy)
+      : "memory");
+}
+
+// H viewed as [T][d / inner][inner] fp16 with inner = 64, 128 or 256 dividing
+// the head width; map n - 1 copies n rows of one head (mid = dh / inner boxes
+// of inner columns each) in one operation, landing as [n][dh] in shared memory
+struct HeadMaps {
+  CUtensorMap m[UMIM_MAX_SPAN_TOKENS];
+};
+
+template <int CPL>
+__global__ void __launch_bounds__(kHeadWarps * 32, 1)
+    pool_head_kernel(const __grid_constant__ HeadMaps maps, int mid, const __half *H, const float2 *stats,
+                     const int32_t *offs, int S, int64_t T, int d, int h,
+                     const __nv_bfloat16 *gamma, const __nv_bfloat16 *beta, const __nv_bfloat16 *query, float eps,
+                     __half *O, int32_t *range_flag, int32_t *status) {
+  extern __shared__ __align__(128) uint8_t head_smem[];
+  __shared__ uint64_t bars[kHeadWarps][kHeadBufs];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int dh = d / h, Ch = dh / 8, ntiles = d / BN;
+  const int buf_bytes = head_buf_bytes(dh, ntiles);
+  uint8_t *wbuf = head_smem + (size_t)warp * kHeadBufs * buf_bytes;
+  const int gw = blockIdx.x * kHeadWarps + warp;
+  const int nw = gridDim.x * kHeadWarps;   // a multiple of h (the host sizes the grid so)
+  const int head = gw % h;
+  const int span_step = nw / h;
+
+  // this lane's columns of the head: chunk ci = k * 32 + lane
+  float2 gq[CPL][4];                 // gamma * q, column pairs
+  uint32_t gp[CPL][4], bp[CPL][4];   // gamma and beta as bf16 pairs
+  float A = 0.f, Bq = 0.f;            // sum over the head of gamma q and of beta q
+#pragma unroll
+  for (int k = 0; k < CPL; ++k) {
+    const int ci = k * 32 + lane;
+    float g[8], b[8], q[8];
+    uint4 g4 = make_uint4(0, 0, 0, 0), b4 = g4, q4 = g4;
+    if (ci < Ch) {
+      const int c = head * dh + ci * 8;
+      g4 = *reinterpret_cast<const uint4 *>(gamma + c);
+      b4 = *reinterpret_cast<const uint4 *>(beta + c);
+      q4 = *reinterpret_cast<const uint4 *>(query + c);   // query [h][dh]: d contiguous values
+    }
+    bf16x8_to_float(g4, g);
+    bf16x8_to_float(b4, b);
+    bf16x8_to_float(q4, q);
+    gp[k][0] = g4.x, gp[k][1] = g4.y, gp[k][2] = g4.z, gp[k][3] = g4.w;
+    bp[k][0] = b4.x, bp[k][1] = b4.y, bp[k][2] = b4.z, bp[k][3] = b4.w;
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      gq[k][e] = make_float2(g[2 * e] * q[2 * e], g[2 * e + 1] * q[2 * e + 1]);
+      A += gq[k][e].x + gq[k][e].y;
+      Bq = fmaf(b[2 * e], q[2 * e], Bq);
+      Bq = fmaf(b[2 * e + 1], q[2 * e + 1], Bq);
+    }
+  }
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) {
+    A += __shfl_xor_sync(0xffffffffu, A, o);
+    Bq += __shfl_xor_sync(0xffffffffu, Bq, o);
+  }
+  if (lane == 0) {
+    for (int i = 0; i < kHeadBufs; ++i) mbar_init(&bars[warp][i], 1);
+    fence_mbar_init();
+  }
+  __syncwarp();
+  griddep_wait();   // H and its statistics come from the projection kernel
+
+  const int n_items = (S - gw / h + span_step - 1) / span_step;   // spans gw/h, gw/h + step, ... below S
+  const uint64_t pol = policy_evict_first();
+  if (lane == 0) prefetch_tensormap(&maps.m[0]);
+  // lane 0 loads the span offsets one item ahead of the copies that need them
+  int pf_t0 = 0, pf_t1 = 0;
+  auto prefetch = [&](int item) {
+    if (item < n_items) {
+      const int sp = gw / h + item * span_step;
+      pf_t0 = offs[sp];
+      pf_t1 = offs[sp + 1];
+    }
+  };
+  // lane 0: issue the copies of the item-th span of this warp into buffer `b`
+  // (its offsets were prefetched); returns the span's row count (0 for an
+  // invalid span)
+  auto issue = [&](int b) -> int {
+    uint64_t *bar = &bars[warp][b];
+    const int t0 = pf_t0, t1 = pf_t1;
+    int n = t1 - t0;
+    if (t0 < 0 || n < 1 || n > UMIM_MAX_SPAN_TOKENS || t1 > T) {
+      if (head == 0) set_error(status, UMIM_ERR_INVALID_ARG);
+      n = 0;
+    }
+    if (n == 0) {
+      mbar_arrive(bar);
+      return 0;
+    }
+    uint8_t *dst = wbuf + b * buf_bytes;
+    mbar_arrive_expect_tx(bar, n * (dh * 2 + ntiles * 8));
+    // the span's rows of this head in one tensor copy, their statistics (consecutive) in one bulk copy
+    tma_load_3d(dst, &maps.m[n - 1], bar, 0, head * mid, t0, pol);
+    bulk_g2s(dst + UMIM_MAX_SPAN_TOKENS * dh * 2, stats + (int64_t)t0 * ntiles, n * ntiles * 8, bar);
+    return n;
+  };
+
+  static_assert(kHeadBufs == 2, "two buffers per warp");
+  int n_buf0 = 0, n_buf1 = 0;   // row counts of the items in flight (lane 0's view)
+  if (lane == 0) {
+    prefetch(0);
+    if (n_items > 0) {
+      n_buf0 = issue(0);
+      prefetch(1);
+    }
+    if (n_items > 1) {
+      n_buf1 = issue(1);
+      prefetch(2);
+    }
+  }
+  const float inv_sqrt_dh = rsqrtf((float)dh), inv_ntiles = 1.f / (float)ntiles, inv_d = 1.f / (float)d;
+  for (int item = 0; item < n_items; ++item) {
+    const int b = item % kHeadBufs;
+    const int sp = gw / h + item * span_step;
+    const int n = __shfl_sync(0xffffffffu, b ? n_buf1 : n_buf0, 0);
+    if (!__all_sync(0xffffffffu, mbar_wait(&bars[warp][b], (item / kHeadBufs) & 1))) {
+      set_error(status, UMIM_ERR_TIMEOUT);
+      // let the other buffer's copies land (bounded) before leaving
+      if (item + 1 < n_items) mbar_wait(&bars[warp][(item + 1) % kHeadBufs], ((item + 1) / kHeadBufs) & 1);
+      return;
+    }
+    const __half *hs = reinterpret_cast<const __half *>(wbuf + b * buf_bytes);
+    const float2 *ts = reinterpret_cast<const float2 *>(wbuf + b * buf_bytes + UMIM_MAX_SPAN_TOKENS * dh * 2);
+    // scores: per row sum_c H gamma q over the head (packed fp32 pairs, two
+    // accumulators per row), then the per-tile moments; rows interleaved so
+    // the shuffle reductions of the rows overlap
+    float2 pa[UMIM_MAX_SPAN_TOKENS], pb[UMIM_MAX_SPAN_TOKENS];
+    float2 tv[UMIM_MAX_SPAN_TOKENS];
+#pragma unroll
+    for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
+      pa[j] = make_float2(0.f, 0.f);
+      pb[j] = make_float2(0.f, 0.f);
+      tv[j] = make_float2(0.f, 0.f);
+      if (j < n) {
+#pragma unroll
+        for (int k = 0; k < CPL; ++k) {
+          const int ci = k * 32 + lane;
+          if (ci < Ch) {
+            const uint4 x = *reinterpret_cast<const uint4 *>(hs + j * dh + ci * 8);
+            const __half2 *h2 = reinterpret_cast<const __half2 *>(&x);
+            pa[j] = __ffma2_rn(__half22float2(h2[0]), gq[k][0], pa[j]);
+            pb[j] = __ffma2_rn(__half22float2(h2[1]), gq[k][1], pb[j]);
+            pa[j] = __ffma2_rn(__half22float2(h2[2]), gq[k][2], pa[j]);
+            pb[j] = __ffma2_rn(__half22float2(h2[3]), gq[k][3], pb[j]);
+          }
+        }
+        if (lane < ntiles) tv[j] = ts[j * ntiles + lane];
+      }
+    }
+    float p[UMIM_MAX_SPAN_TOKENS], sm[UMIM_MAX_SPAN_TOKENS], s2[UMIM_MAX_SPAN_TOKENS];
+#pragma unroll
+    for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
+      p[j] = (pa[j].x + pb[j].x) + (pa[j].y + pb[j].y);
+      sm[j] = tv[j].x;
+      s2[j] = tv[j].y;
+    }
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) {
+#pragma unroll
+      for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
+        p[j] += __shfl_xor_sync(0xffffffffu, p[j], o);
+        sm[j] += __shfl_xor_sync(0xffffffffu, sm[j], o);
+        s2[j] += __shfl_xor_sync(0xffffffffu, s2[j], o);
+      }
+    }
+    float mu[UMIM_MAX_SPAN_TOKENS], dv[UMIM_MAX_SPAN_TOKENS];
+#pragma unroll
+    for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
+      mu[j] = sm[j] * inv_ntiles;
+      dv[j] = lane < ntiles ? (tv[j].x - mu[j]) * (tv[j].x - mu[j]) : 0.f;
+    }
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) {
+#pragma unroll
+      for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) dv[j] += __shfl_xor_sync(0xffffffffu, dv[j], o);
+    }
+    float rs[UMIM_MAX_SPAN_TOKENS], w[UMIM_MAX_SPAN_TOKENS];
+    float mx = -INFINITY;
+#pragma unroll
+    for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
+      rs[j] = rsqrtf((s2[j] + (float)BN * dv[j]) * inv_d + eps);
+      w[j] = j < n ? (rs[j] * (p[j] - mu[j] * A) + Bq) * inv_sqrt_dh : -INFINITY;
+      mx = fmaxf(mx, w[j]);
+    }
+    // softmax over the span's rows; w_j = alpha_j r_j, C = sum_j w_j mu_j
+    float den = 0.f;
+#pragma unroll
+    for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
+      w[j] = j < n ? expf(w[j] - mx) : 0.f;
+      den += w[j];
+    }
+    const float inv_den = n > 0 ? 1.f / den : 0.f;
+    float C = 0.f;
+#pragma unroll
+    for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
+      w[j] = w[j] * inv_den * rs[j];
+      C = fmaf(w[j], mu[j], C);
+    }
+    // o_c = gamma_c (sum_j w_j H_jc - C) + beta_c  (0 for an invalid span); an
+    // fp16 rounding that is not finite (all exponent bits set) is flagged
+    uint32_t bad = 0;
+#pragma unroll
+    for (int k = 0; k < CPL; ++k) {
+      const int ci = k * 32 + lane;
+      if (ci < Ch) {
+        float2 x[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) x[e] = make_float2(-C, -C);
+#pragma unroll
+        for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
+          if (j < n) {
+            const uint4 hv = *reinterpret_cast<const uint4 *>(hs + j * dh + ci * 8);
+            const __half2 *h2 = reinterpret_cast<const __half2 *>(&hv);
+            const float2 w2 = make_float2(w[j], w[j]);
+#pragma unroll
+            for (int e = 0; e < 4; ++e) x[e] = __ffma2_rn(w2, __half22float2(h2[e]), x[e]);
+          }
+        }
+        uint4 packed;
+        uint32_t *pw = reinterpret_cast<uint32_t *>(&packed);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float2 g2 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&gp[k][e]));
+          const float2 b2 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&bp[k][e]));
+          const float2 o2 = n > 0 ? __ffma2_rn(g2, x[e], b2) : make_float2(0.f, 0.f);
+          const __half2 hh = __float22half2_rn(o2);
+          pw[e] = *reinterpret_cast<const uint32_t *>(&hh);
+          bad |= __vcmpeq2(pw[e] & 0x7C007C00u, 0x7C007C00u);
+        }
+        *reinterpret_cast<uint4 *>(O + (int64_t)sp * d + (int64_t)head * dh + ci * 8) = packed;
+      }
+    }
+    if (__any_sync(0xffffffffu, bad != 0) && lane == 0) flag_range(range_flag, status);
+    // every lane is done with this buffer: refill it with the item two ahead
+    __syncwarp();
+    if (lane == 0 && item + kHeadBufs < n_items) {
+      const int nn = issue(b);
+      prefetch(item + kHeadBufs + 1);
+      if (b) n_buf1 = nn;
+      else n_buf0 = nn;
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
 // LN_o over rows of Z (fp16, the GELU output of the projection; its row
 // statistics were taken from the fp32 values), one warp per row, z in fp32
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(256)
     ln_rows_kernel(const __half *Z, float *out, const float2 *stats, int S, int d, const __nv_bfloat16 *gamma,
-                   const __nv_bfloat16 *beta, float eps) {
+                   const __nv_bfloat16 *beta, float eps, const int32_t *range_flag) {
   griddep_wait();
+  // an intermediate did not fit fp16 (already reported): write no surrogate
+  if (*reinterpret_cast<const volatile int32_t *>(range_flag) != 0) return;
   const int r = blockIdx.x * 8 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (r >= S) return;
@@ -586,9 +896,11 @@ __global__ void __launch_bounds__(256)
   }
 }
 
-// W_o from bf16 to fp16 (exact for values in fp16's normal range)
-__global__ void bf16_to_f16_kernel(const uint4 *in, uint4 *out, int64_t n_vec) {
+// kWoScale * W_o from bf16 to fp16 (exact for |W_o| in [2^-22, 255.875])
+__global__ void bf16_to_f16_kernel(const uint4 *in, uint4 *out, int64_t n_vec, int32_t *range_flag,
+                                   int32_t *status) {
   griddep_wait();
+  bool bad = false;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n_vec; i += (int64_t)gridDim.x * blockDim.x) {
     const uint4 u = in[i];
     float f[8];
@@ -596,9 +908,15 @@ __global__ void bf16_to_f16_kernel(const uint4 *in, uint4 *out, int64_t n_vec) {
     uint4 o;
     __half2 *h = reinterpret_cast<__half2 *>(&o);
 #pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      f[e] *= kWoScale;
+      bad |= !(fabsf(f[e]) < kF16Limit);
+    }
+#pragma unroll
     for (int e = 0; e < 4; ++e) h[e] = __floats2half2_rn(f[2 * e], f[2 * e + 1]);
     out[i] = o;
   }
+  if (bad) flag_range(range_flag, status);
 }
 
 inline size_t al1k(size_t x) { return (x + 1023) & ~size_t(1023); }
@@ -620,6 +938,7 @@ size_t merge_spans_workspace_bytes(int64_t T, int S, int d) {
   b += al1k((size_t)std::max(S, 1) * d * 2);                   // o (fp16)
   b += al1k((size_t)d * d * 2);                                 // W_o (fp16)
   b += al1k((size_t)std::max(S, 1) * nt * 8);                  // stats of Z
+  b += al1k(sizeof(int32_t));                                   // fp16 range flag
   return b;
 }
 
@@ -638,9 +957,9 @@ static bool encode_kmajor(EncodeTiledFn enc, CUtensorMap *map, const void *base,
 // out[M][d] = GELU(A[M][d] B[d][d]^T + bias); A and B both bf16 or both fp16
 template <typename OutT>
 static umim_status launch_gemm(EncodeTiledFn enc, const void *A, int64_t M, const void *Bw, int d, bool fp16,
-                               const void *bias, OutT *out, float2 *stats, int32_t *status, cudaStream_t st,
-                               const char *label, int num_sms, const void *cvt_in = nullptr, void *cvt_out = nullptr,
-                               int64_t cvt_n = 0) {
+                               const void *bias, OutT *out, float2 *stats, int32_t *range_flag, float acc_scale,
+                               int32_t *status, cudaStream_t st, const char *label, int num_sms,
+                               const void *cvt_in = nullptr, void *cvt_out = nullptr, int64_t cvt_n = 0) {
   CUtensorMap am, bm;
   if (!encode_kmajor(enc, &am, A, M, d, BM, fp16) || !encode_kmajor(enc, &bm, Bw, d, d, BN, fp16))
     return UMIM_ERR_CUDA;
@@ -655,6 +974,9 @@ static umim_status launch_gemm(EncodeTiledFn enc, const void *A, int64_t M, cons
   g.cvt_in = static_cast<const uint4 *>(cvt_in);
   g.cvt_out = static_cast<uint4 *>(cvt_out);
   g.cvt_n = cvt_n;
+  g.cvt_scale = kWoScale;
+  g.acc_scale = acc_scale;
+  g.range_flag = range_flag;
   g.status = status;
   // set on every call: the attribute belongs to the current device, and calls may
   // come for several devices and from several threads
@@ -689,6 +1011,8 @@ umim_status merge_spans(const void *embeddings, int64_t vocab, const int32_t *to
   __half *Wo16 = reinterpret_cast<__half *>(p);
   p += al1k((size_t)d * d * 2);
   float2 *st2 = reinterpret_cast<float2 *>(p);
+  p += al1k((size_t)std::max(S, 1) * nt * 8);
+  int32_t *range_flag = reinterpret_cast<int32_t *>(p);
 
   if (S == 0) return UMIM_OK;
   bool wo_in_gemm1 = false;
@@ -696,7 +1020,7 @@ umim_status merge_spans(const void *embeddings, int64_t vocab, const int32_t *to
     const int blocks = std::max(1, std::min<int>((int)((T + 7) / 8), num_sms * 8));
     trace_mark(st, "merge.gather");
     if (launch_pdl(gather_rows_kernel, dim3(blocks), dim3(256), 0, st, static_cast<const uint4 *>(embeddings), vocab,
-                   token_ids, T, d, reinterpret_cast<uint4 *>(E), status) != cudaSuccess)
+                   token_ids, T, d, reinterpret_cast<uint4 *>(E), range_flag, status) != cudaSuccess)
       return UMIM_ERR_CUDA;
     // W_o -> fp16 rides along in a side warp of GEMM1 when its share is small
     // next to the tiles its CTA computes; else a kernel of its own
@@ -704,41 +1028,80 @@ umim_status merge_spans(const void *embeddings, int64_t vocab, const int32_t *to
     const int64_t grid1 = std::min<int64_t>(tiles1, std::max(1, num_sms));
     const int64_t n_vec = (int64_t)d * d / 8;
     wo_in_gemm1 = n_vec <= 128 * 32 * grid1 * (tiles1 / grid1);
-    umim_status r = launch_gemm(enc, E, T, w->w_kv, d, false, w->b_kv, H, st1, status, st, "merge.gemm1", num_sms,
-                                wo_in_gemm1 ? w->w_o : nullptr, wo_in_gemm1 ? Wo16 : nullptr,
+    umim_status r = launch_gemm(enc, E, T, w->w_kv, d, false, w->b_kv, H, st1, range_flag, 1.f, status, st,
+                                "merge.gemm1", num_sms, wo_in_gemm1 ? w->w_o : nullptr, wo_in_gemm1 ? Wo16 : nullptr,
                                 wo_in_gemm1 ? n_vec : 0);
     if (r != UMIM_OK) return r;
   }
   trace_mark(st, "merge.pool");
-  const int psmem = kPoolRing * pool_stage_bytes(d);
-  const int chunks = d / 8 / kPoolConsumers;   // 16-byte column chunks per consumer thread (d <= 8192)
-  auto pk = chunks <= 1 ? pool_kernel<1> : (chunks == 2 ? pool_kernel<2> : pool_kernel<4>);
-  if (cudaFuncSetAttribute(pk, cudaFuncAttributeMaxDynamicSharedMemorySize, psmem) != cudaSuccess)
-    return UMIM_ERR_CUDA;
-  int pool_per_sm = 1;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&pool_per_sm, pk, kPoolConsumers + 32, psmem) != cudaSuccess ||
-      pool_per_sm < 1)
-    pool_per_sm = 1;
-  const int pool_grid = std::max(1, std::min(S, std::max(1, num_sms) * pool_per_sm));
-  if (launch_pdl(pk, dim3(pool_grid), dim3(kPoolConsumers + 32), psmem, st, (const __half *)H, (const float2 *)st1,
-                 span_offsets, S, T, d, (int)w->n_heads, static_cast<const __nv_bfloat16 *>(w->ln_kv_gamma),
-                 static_cast<const __nv_bfloat16 *>(w->ln_kv_beta), static_cast<const __nv_bfloat16 *>(w->query),
-                 w->ln_eps, O, status) != cudaSuccess)
-    return UMIM_ERR_CUDA;
+  const int Ch = d / w->n_heads / 8;   // 16-byte chunks per head
+  if (Ch <= 128) {
+    // one warp per (span, head), double-buffered in shared memory
+    const int cpl = (Ch + 31) / 32;
+    auto pk = cpl == 1 ? pool_head_kernel<1> : cpl == 2 ? pool_head_kernel<2> : cpl == 3 ? pool_head_kernel<3>
+                                                                                  : pool_head_kernel<4>;
+    const int dh = d / w->n_heads;
+    const int inner = 64 * (((dh / 64) % 4 == 0) ? 4 : ((dh / 64) % 2 == 0) ? 2 : 1);
+    const int mid = dh / inner;
+    HeadMaps maps;
+    for (int n = 1; n <= UMIM_MAX_SPAN_TOKENS; ++n) {
+      const cuuint64_t dims[3] = {(cuuint64_t)inner, (cuuint64_t)(d / inner), (cuuint64_t)T};
+      const cuuint64_t strides[2] = {(cuuint64_t)inner * 2, (cuuint64_t)d * 2};
+      const cuuint32_t box[3] = {(cuuint32_t)inner, (cuuint32_t)mid, (cuuint32_t)n};
+      const cuuint32_t es[3] = {1, 1, 1};
+      if (enc(&maps.m[n - 1], CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 3, H, dims, strides, box, es,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+        return UMIM_ERR_CUDA;
+    }
+    const int psmem = kHeadWarps * kHeadBufs * head_buf_bytes(dh, nt);
+    if (cudaFuncSetAttribute(pk, cudaFuncAttributeMaxDynamicSharedMemorySize, psmem) != cudaSuccess)
+      return UMIM_ERR_CUDA;
+    // warps of the grid: a multiple of h, at most one CTA per SM and no more than the items
+    const int h = w->n_heads;
+    const int64_t items = (int64_t)S * h;
+    int grid = (int)std::min<int64_t>(std::max(1, num_sms), (items + kHeadWarps - 1) / kHeadWarps);
+    while (grid > 1 && (grid * kHeadWarps) % h != 0) --grid;
+    if ((grid * kHeadWarps) % h != 0) grid = h;   // 12 * h is a multiple of h
+    if (launch_pdl(pk, dim3(grid), dim3(kHeadWarps * 32), psmem, st, maps, mid, (const __half *)H,
+                   (const float2 *)st1, span_offsets, S, T, d, h, static_cast<const __nv_bfloat16 *>(w->ln_kv_gamma),
+                   static_cast<const __nv_bfloat16 *>(w->ln_kv_beta), static_cast<const __nv_bfloat16 *>(w->query),
+                   w->ln_eps, O, range_flag, status) != cudaSuccess)
+      return UMIM_ERR_CUDA;
+  } else {
+    // wider heads: the CTA-per-span kernel with a staged ring
+    const int psmem = kPoolRing * pool_stage_bytes(d);
+    const int chunks = d / 8 / kPoolConsumers;   // 16-byte column chunks per consumer thread (d <= 8192)
+    auto pk = chunks <= 1 ? pool_kernel<1> : (chunks == 2 ? pool_kernel<2> : pool_kernel<4>);
+    if (cudaFuncSetAttribute(pk, cudaFuncAttributeMaxDynamicSharedMemorySize, psmem) != cudaSuccess)
+      return UMIM_ERR_CUDA;
+    int pool_per_sm = 1;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&pool_per_sm, pk, kPoolConsumers + 32, psmem) != cudaSuccess ||
+        pool_per_sm < 1)
+      pool_per_sm = 1;
+    const int pool_grid = std::max(1, std::min(S, std::max(1, num_sms) * pool_per_sm));
+    if (launch_pdl(pk, dim3(pool_grid), dim3(kPoolConsumers + 32), psmem, st, (const __half *)H,
+                   (const float2 *)st1, span_offsets, S, T, d, (int)w->n_heads,
+                   static_cast<const __nv_bfloat16 *>(w->ln_kv_gamma),
+                   static_cast<const __nv_bfloat16 *>(w->ln_kv_beta), static_cast<const __nv_bfloat16 *>(w->query),
+                   w->ln_eps, O, range_flag, status) != cudaSuccess)
+      return UMIM_ERR_CUDA;
+  }
   if (!wo_in_gemm1) {
     trace_mark(st, "merge.wo_f16");
     if (launch_pdl(bf16_to_f16_kernel, dim3(std::max(1, num_sms) * 4), dim3(256), 0, st,
-                   static_cast<const uint4 *>(w->w_o), reinterpret_cast<uint4 *>(Wo16), (int64_t)d * d / 8) !=
-        cudaSuccess)
+                   static_cast<const uint4 *>(w->w_o), reinterpret_cast<uint4 *>(Wo16), (int64_t)d * d / 8,
+                   range_flag, status) != cudaSuccess)
       return UMIM_ERR_CUDA;
   }
-  umim_status r = launch_gemm(enc, O, S, Wo16, d, true, w->b_o, Z16, st2, status, st, "merge.gemm2", num_sms);
+  umim_status r = launch_gemm(enc, O, S, Wo16, d, true, w->b_o, Z16, st2, range_flag, 1.f / kWoScale, status, st,
+                              "merge.gemm2", num_sms);
   if (r != UMIM_OK) return r;
   trace_mark(st, "merge.ln_o");
   if (launch_pdl(ln_rows_kernel, dim3((S + 7) / 8), dim3(256), 0, st, (const __half *)Z16, surrogates,
                  (const float2 *)st2, S, d,
                  static_cast<const __nv_bfloat16 *>(w->ln_o_gamma), static_cast<const __nv_bfloat16 *>(w->ln_o_beta),
-                 w->ln_eps) != cudaSuccess)
+                 w->ln_eps, (const int32_t *)range_flag) != cudaSuccess)
     return UMIM_ERR_CUDA;
   trace_mark(st, nullptr);
   return UMIM_OK;

@@ -222,3 +222,10 @@ def test_layer_step_host_checks(lib):
     assert call(out=ctypes.c_void_p((1 << 20) + 2)) == 1     # output not 4-byte aligned
     assert call(rows=3, mk=fake) == 1                        # merges without surrogate arrays
     assert call(batch=0) == 0                                # an empty batch is a no-op
+
+
+def test_merge_needs_a_token_per_span(lib):
+    from paper_2609_27233_gb300._lib import MergeWeightsC
+    null = ctypes.c_void_p(0)
+    w = MergeWeightsC(*([1 << 20] * 9), 512, 4, 1e-5)
+    assert lib.umim_merge_spans(null, 10, null, 3, null, 4, ctypes.byref(w), null, null, 0, null, null) == 1
