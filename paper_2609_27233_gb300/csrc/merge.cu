@@ -622,6 +622,115 @@ struct HeadMaps {
   CUtensorMap m[UMIM_MAX_SPAN_TOKENS];
 };
 
+// One (span, head) item with N rows, staged in shared memory: hs [N][dh] fp16,
+// ts [N][ntiles] per-tile (mean, M2).  Writes the head's slice of o and
+// returns nonzero if some fp16 value of it is not finite.
+template <int CPL, int N>
+__device__ __forceinline__ uint32_t pool_item(const __half *hs, const float2 *ts, const float2 (&gq)[CPL][4],
+                                              const uint32_t (&gp)[CPL][4], const uint32_t (&bp)[CPL][4], float A,
+                                              float Bq, int lane, int Ch, int dh, int ntiles, float inv_ntiles,
+                                              float inv_d, float eps, float inv_sqrt_dh, __half *orow) {
+  // scores: per row sum_c H gamma q over the head (packed fp32 pairs, two
+  // accumulators per row), then the per-tile moments; the rows' shuffle
+  // reductions interleave
+  float p[N], sm[N], s2[N], tx[N];
+#pragma unroll
+  for (int j = 0; j < N; ++j) {
+    float2 pa = make_float2(0.f, 0.f), pb = make_float2(0.f, 0.f);
+#pragma unroll
+    for (int k = 0; k < CPL; ++k) {
+      const int ci = k * 32 + lane;
+      if (ci < Ch) {
+        const uint4 x = *reinterpret_cast<const uint4 *>(hs + j * dh + ci * 8);
+        const __half2 *h2 = reinterpret_cast<const __half2 *>(&x);
+        pa = __ffma2_rn(__half22float2(h2[0]), gq[k][0], pa);
+        pb = __ffma2_rn(__half22float2(h2[1]), gq[k][1], pb);
+        pa = __ffma2_rn(__half22float2(h2[2]), gq[k][2], pa);
+        pb = __ffma2_rn(__half22float2(h2[3]), gq[k][3], pb);
+      }
+    }
+    const float2 t = lane < ntiles ? ts[j * ntiles + lane] : make_float2(0.f, 0.f);
+    p[j] = (pa.x + pb.x) + (pa.y + pb.y);
+    tx[j] = t.x;
+    sm[j] = t.x;
+    s2[j] = t.y;
+  }
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) {
+#pragma unroll
+    for (int j = 0; j < N; ++j) {
+      p[j] += __shfl_xor_sync(0xffffffffu, p[j], o);
+      sm[j] += __shfl_xor_sync(0xffffffffu, sm[j], o);
+      s2[j] += __shfl_xor_sync(0xffffffffu, s2[j], o);
+    }
+  }
+  float mu[N], dv[N];
+#pragma unroll
+  for (int j = 0; j < N; ++j) {
+    mu[j] = sm[j] * inv_ntiles;
+    dv[j] = lane < ntiles ? (tx[j] - mu[j]) * (tx[j] - mu[j]) : 0.f;
+  }
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) {
+#pragma unroll
+    for (int j = 0; j < N; ++j) dv[j] += __shfl_xor_sync(0xffffffffu, dv[j], o);
+  }
+  // softmax over the rows; w_j = alpha_j r_j, C = sum_j w_j mu_j
+  float rs[N], w[N], mx = -INFINITY;
+#pragma unroll
+  for (int j = 0; j < N; ++j) {
+    rs[j] = rsqrtf((s2[j] + (float)BN * dv[j]) * inv_d + eps);
+    w[j] = (rs[j] * (p[j] - mu[j] * A) + Bq) * inv_sqrt_dh;
+    mx = fmaxf(mx, w[j]);
+  }
+  float den = 0.f;
+#pragma unroll
+  for (int j = 0; j < N; ++j) {
+    w[j] = expf(w[j] - mx);
+    den += w[j];
+  }
+  const float inv_den = 1.f / den;
+  float C = 0.f;
+#pragma unroll
+  for (int j = 0; j < N; ++j) {
+    w[j] = w[j] * inv_den * rs[j];
+    C = fmaf(w[j], mu[j], C);
+  }
+  // o_c = gamma_c (sum_j w_j H_jc - C) + beta_c; an fp16 result whose exponent
+  // bits are all set (inf or NaN) carries into bit 15 of its half when 0x0400
+  // is added to the masked exponent
+  uint32_t bad = 0;
+#pragma unroll
+  for (int k = 0; k < CPL; ++k) {
+    const int ci = k * 32 + lane;
+    if (ci < Ch) {
+      float2 x[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) x[e] = make_float2(-C, -C);
+#pragma unroll
+      for (int j = 0; j < N; ++j) {
+        const uint4 hv = *reinterpret_cast<const uint4 *>(hs + j * dh + ci * 8);
+        const __half2 *h2 = reinterpret_cast<const __half2 *>(&hv);
+        const float2 w2 = make_float2(w[j], w[j]);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) x[e] = __ffma2_rn(w2, __half22float2(h2[e]), x[e]);
+      }
+      uint4 packed;
+      uint32_t *pw = reinterpret_cast<uint32_t *>(&packed);
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float2 g2 = make_float2(__uint_as_float(gp[k][e] << 16), __uint_as_float(gp[k][e] & 0xFFFF0000u));
+        const float2 b2 = make_float2(__uint_as_float(bp[k][e] << 16), __uint_as_float(bp[k][e] & 0xFFFF0000u));
+        const __half2 hh = __float22half2_rn(__ffma2_rn(g2, x[e], b2));
+        pw[e] = *reinterpret_cast<const uint32_t *>(&hh);
+        bad |= (pw[e] & 0x7C007C00u) + 0x04000400u;
+      }
+      *reinterpret_cast<uint4 *>(orow + ci * 8) = packed;
+    }
+  }
+  return bad & 0x80008000u;
+}
+
 template <int CPL>
 __global__ void __launch_bounds__(kHeadWarps * 32, 1)
     pool_head_kernel(const __grid_constant__ HeadMaps maps, int mid, const __half *H, const float2 *stats,
@@ -740,114 +849,21 @@ __global__ void __launch_bounds__(kHeadWarps * 32, 1)
     }
     const __half *hs = reinterpret_cast<const __half *>(wbuf + b * buf_bytes);
     const float2 *ts = reinterpret_cast<const float2 *>(wbuf + b * buf_bytes + UMIM_MAX_SPAN_TOKENS * dh * 2);
-    // scores: per row sum_c H gamma q over the head (packed fp32 pairs, two
-    // accumulators per row), then the per-tile moments; rows interleaved so
-    // the shuffle reductions of the rows overlap
-    float2 pa[UMIM_MAX_SPAN_TOKENS], pb[UMIM_MAX_SPAN_TOKENS];
-    float2 tv[UMIM_MAX_SPAN_TOKENS];
-#pragma unroll
-    for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
-      pa[j] = make_float2(0.f, 0.f);
-      pb[j] = make_float2(0.f, 0.f);
-      tv[j] = make_float2(0.f, 0.f);
-      if (j < n) {
-#pragma unroll
-        for (int k = 0; k < CPL; ++k) {
-          const int ci = k * 32 + lane;
-          if (ci < Ch) {
-            const uint4 x = *reinterpret_cast<const uint4 *>(hs + j * dh + ci * 8);
-            const __half2 *h2 = reinterpret_cast<const __half2 *>(&x);
-            pa[j] = __ffma2_rn(__half22float2(h2[0]), gq[k][0], pa[j]);
-            pb[j] = __ffma2_rn(__half22float2(h2[1]), gq[k][1], pb[j]);
-            pa[j] = __ffma2_rn(__half22float2(h2[2]), gq[k][2], pa[j]);
-            pb[j] = __ffma2_rn(__half22float2(h2[3]), gq[k][3], pb[j]);
-          }
-        }
-        if (lane < ntiles) tv[j] = ts[j * ntiles + lane];
-      }
-    }
-    float p[UMIM_MAX_SPAN_TOKENS], sm[UMIM_MAX_SPAN_TOKENS], s2[UMIM_MAX_SPAN_TOKENS];
-#pragma unroll
-    for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
-      p[j] = (pa[j].x + pb[j].x) + (pa[j].y + pb[j].y);
-      sm[j] = tv[j].x;
-      s2[j] = tv[j].y;
-    }
-#pragma unroll
-    for (int o = 16; o >= 1; o >>= 1) {
-#pragma unroll
-      for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
-        p[j] += __shfl_xor_sync(0xffffffffu, p[j], o);
-        sm[j] += __shfl_xor_sync(0xffffffffu, sm[j], o);
-        s2[j] += __shfl_xor_sync(0xffffffffu, s2[j], o);
-      }
-    }
-    float mu[UMIM_MAX_SPAN_TOKENS], dv[UMIM_MAX_SPAN_TOKENS];
-#pragma unroll
-    for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
-      mu[j] = sm[j] * inv_ntiles;
-      dv[j] = lane < ntiles ? (tv[j].x - mu[j]) * (tv[j].x - mu[j]) : 0.f;
-    }
-#pragma unroll
-    for (int o = 16; o >= 1; o >>= 1) {
-#pragma unroll
-      for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) dv[j] += __shfl_xor_sync(0xffffffffu, dv[j], o);
-    }
-    float rs[UMIM_MAX_SPAN_TOKENS], w[UMIM_MAX_SPAN_TOKENS];
-    float mx = -INFINITY;
-#pragma unroll
-    for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
-      rs[j] = rsqrtf((s2[j] + (float)BN * dv[j]) * inv_d + eps);
-      w[j] = j < n ? (rs[j] * (p[j] - mu[j] * A) + Bq) * inv_sqrt_dh : -INFINITY;
-      mx = fmaxf(mx, w[j]);
-    }
-    // softmax over the span's rows; w_j = alpha_j r_j, C = sum_j w_j mu_j
-    float den = 0.f;
-#pragma unroll
-    for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
-      w[j] = j < n ? expf(w[j] - mx) : 0.f;
-      den += w[j];
-    }
-    const float inv_den = n > 0 ? 1.f / den : 0.f;
-    float C = 0.f;
-#pragma unroll
-    for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
-      w[j] = w[j] * inv_den * rs[j];
-      C = fmaf(w[j], mu[j], C);
-    }
-    // o_c = gamma_c (sum_j w_j H_jc - C) + beta_c  (0 for an invalid span); an
-    // fp16 rounding that is not finite (all exponent bits set) is flagged
     uint32_t bad = 0;
+    __half *orow = O + (int64_t)sp * d + (int64_t)head * dh;
+    switch (n) {
+      case 1: bad = pool_item<CPL, 1>(hs, ts, gq, gp, bp, A, Bq, lane, Ch, dh, ntiles, inv_ntiles, inv_d, eps,
+                                      inv_sqrt_dh, orow); break;
+      case 2: bad = pool_item<CPL, 2>(hs, ts, gq, gp, bp, A, Bq, lane, Ch, dh, ntiles, inv_ntiles, inv_d, eps,
+                                      inv_sqrt_dh, orow); break;
+      case 3: bad = pool_item<CPL, 3>(hs, ts, gq, gp, bp, A, Bq, lane, Ch, dh, ntiles, inv_ntiles, inv_d, eps,
+                                      inv_sqrt_dh, orow); break;
+      case 4: bad = pool_item<CPL, 4>(hs, ts, gq, gp, bp, A, Bq, lane, Ch, dh, ntiles, inv_ntiles, inv_d, eps,
+                                      inv_sqrt_dh, orow); break;
+      default:   // an invalid span: o = 0
 #pragma unroll
-    for (int k = 0; k < CPL; ++k) {
-      const int ci = k * 32 + lane;
-      if (ci < Ch) {
-        float2 x[4];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) x[e] = make_float2(-C, -C);
-#pragma unroll
-        for (int j = 0; j < UMIM_MAX_SPAN_TOKENS; ++j) {
-          if (j < n) {
-            const uint4 hv = *reinterpret_cast<const uint4 *>(hs + j * dh + ci * 8);
-            const __half2 *h2 = reinterpret_cast<const __half2 *>(&hv);
-            const float2 w2 = make_float2(w[j], w[j]);
-#pragma unroll
-            for (int e = 0; e < 4; ++e) x[e] = __ffma2_rn(w2, __half22float2(h2[e]), x[e]);
-          }
-        }
-        uint4 packed;
-        uint32_t *pw = reinterpret_cast<uint32_t *>(&packed);
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float2 g2 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&gp[k][e]));
-          const float2 b2 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&bp[k][e]));
-          const float2 o2 = n > 0 ? __ffma2_rn(g2, x[e], b2) : make_float2(0.f, 0.f);
-          const __half2 hh = __float22half2_rn(o2);
-          pw[e] = *reinterpret_cast<const uint32_t *>(&hh);
-          bad |= __vcmpeq2(pw[e] & 0x7C007C00u, 0x7C007C00u);
-        }
-        *reinterpret_cast<uint4 *>(O + (int64_t)sp * d + (int64_t)head * dh + ci * 8) = packed;
-      }
+        for (int k = 0; k < CPL; ++k)
+          if (k * 32 + lane < Ch) *reinterpret_cast<uint4 *>(orow + (k * 32 + lane) * 8) = make_uint4(0, 0, 0, 0);
     }
     if (__any_sync(0xffffffffu, bad != 0) && lane == 0) flag_range(range_flag, status);
     // every lane is done with this buffer: refill it with the item two ahead
