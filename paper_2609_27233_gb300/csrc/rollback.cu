@@ -46,6 +46,7 @@ struct MoveArgs {
   int32_t *status;
   const float *rope_inv_freq;   // [rotary_dim / 2] or nullptr: keys move verbatim
   int32_t rotary_dim;
+  uint32_t zero;                // always 0 (see red_add_after)
 };
 
 // largest i in [lo, hi) with key(i) <= x, or lo - 1
@@ -72,8 +73,16 @@ __device__ __forceinline__ void st_v4(uint16_t *p, uint4 v) {
                : "memory");
 }
 
-__device__ __forceinline__ void red_release_add(int32_t *p, int32_t v) {
-  asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+// Adds 1 + (dep & zero) to *p, zero being 0 at run time (a kernel argument,
+// so the compiler cannot drop the term): the add depends on `dep`, a fold of
+// the unit's loaded data, so it cannot issue before those loads have returned
+// their values, and a load that has returned cannot be changed by a store that
+// follows the add -- which is all the page's writer relies on.  No release
+// fence: this thread's earlier stores (of another unit) need not be visible to
+// the waiter, and a fence would stall the warp until they are.
+__device__ __forceinline__ void red_add_after(int32_t *p, uint32_t dep, uint32_t zero) {
+  const int32_t v = 1 + (int32_t)(dep & zero);
+  asm volatile("red.relaxed.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
 }
 
 // Per compacted row (global row index over the active sequences).
@@ -278,9 +287,10 @@ __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs
     uint32_t fold = 0;
 #pragma unroll
     for (int it = 0; it < PER_LANE; ++it) fold ^= t.v[it].x ^ t.v[it].y ^ t.v[it].z ^ t.v[it].w;
-    asm volatile("" ::"r"(fold) : "memory");
-    __syncwarp();
-    if (t.valid && lane == 0) red_release_add(&pd.dep[t.row].landed, 1);
+    // every lane's loads have returned once lane 0 holds the fold of all of them
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) fold ^= __shfl_xor_sync(0xffffffffu, fold, o);
+    if (t.valid && lane == 0) red_add_after(&pd.dep[t.row].landed, fold, a.zero);
   };
   // RoPE: a moved key (shift r) is rotated by -r w_m on the pairs (m, m + rotary_dim/2):
   // x' = x cos + y sin, y' = y cos - x sin.  The lane holding chunk c of a slot's
@@ -488,6 +498,7 @@ umim_status kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t m
   ma.status = status;
   ma.rope_inv_freq = rope_inv_freq;
   ma.rotary_dim = rope_inv_freq ? rotary_dim : 0;
+  ma.zero = 0;
   const bool rope = rope_inv_freq != nullptr;
   auto kern = D == 128 ? (rope ? rollback_move_kernel<128, true> : rollback_move_kernel<128, false>)
                        : (rope ? rollback_move_kernel<64, true> : rollback_move_kernel<64, false>);
