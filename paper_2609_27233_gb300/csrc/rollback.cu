@@ -85,6 +85,12 @@ __device__ __forceinline__ void red_add_after(int32_t *p, uint32_t dep, uint32_t
   asm volatile("red.relaxed.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
 }
 
+__device__ __forceinline__ int32_t ld_relaxed(const int32_t *p) {
+  int32_t v;
+  asm volatile("ld.relaxed.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
 // Per compacted row (global row index over the active sequences).
 struct RowDep {
   int32_t lo, hi;   // reader rows of this row's old page that precede it (lo > hi: none)
@@ -229,6 +235,7 @@ __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs
     int valid, rot;     // rot: a K tile whose moved entries get re-rotated
     int64_t dst;
     int32_t row, dlo, dhi;
+    int32_t seen;       // the reader rows' smallest landed count when the unit was loaded
     int32_t shift;      // lanes < 16: the shift of slot `lane`
   };
   // slot i = kk * row_size + pos, kk the compacted page row
@@ -241,6 +248,7 @@ __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs
     t.row = 0;
     t.dlo = 1;
     t.dhi = 0;
+    t.seen = a.n_lanes;
 #pragma unroll
     for (int it = 0; it < PER_LANE; ++it) t.v[it] = make_uint4(0, 0, 0, 0);
     if (kk >= max_dest) return;
@@ -272,8 +280,9 @@ __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs
         t.v[it] = ld_v4(sur + ((si * a.n_layers + layer) * Hkv + h) * D + my_col * 8);
       }
     }
-    t.dlo = pd.dep[idx].lo;
-    t.dhi = pd.dep[idx].hi;
+    const RowDep dep = pd.dep[idx];
+    t.dlo = dep.lo;
+    t.dhi = dep.hi;
   };
   auto store = [&](const Tile &t) {
 #pragma unroll
@@ -283,7 +292,7 @@ __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs
     }
   };
   // the unit's loads have arrived; count it into its row
-  auto land_and_count = [&](const Tile &t) {
+  auto land_and_count = [&](Tile &t) {
     uint32_t fold = 0;
 #pragma unroll
     for (int it = 0; it < PER_LANE; ++it) fold ^= t.v[it].x ^ t.v[it].y ^ t.v[it].z ^ t.v[it].w;
@@ -291,6 +300,10 @@ __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs
 #pragma unroll
     for (int o = 16; o >= 1; o >>= 1) fold ^= __shfl_xor_sync(0xffffffffu, fold, o);
     if (t.valid && lane == 0) red_add_after(&pd.dep[t.row].landed, fold, a.zero);
+    // the reader rows' counts, read a step before the store so that their
+    // latency overlaps this step; a complete count then needs no further wait
+    t.seen = a.n_lanes;
+    for (int rw = t.dlo; rw <= t.dhi; ++rw) t.seen = min(t.seen, ld_relaxed(&pd.dep[rw].landed));
   };
   // RoPE: a moved key (shift r) is rotated by -r w_m on the pairs (m, m + rotary_dim/2):
   // x' = x cos + y sin, y' = y cos - x sin.  The lane holding chunk c of a slot's
@@ -354,6 +367,9 @@ __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs
   };
   // every reader of the unit's old page has its loads landed
   auto readers_done = [&](const Tile &t) -> bool {
+    // counts only grow: if every reader had landed when the unit was loaded,
+    // the store may go ahead (it is issued only after that read returned)
+    if (t.seen >= a.n_lanes) return true;
     for (int rw = t.dlo; rw <= t.dhi; ++rw)
       if (!wait_landed(&pd.dep[rw].landed, a.n_lanes, abort_flag)) return false;
     return true;
