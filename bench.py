@@ -344,6 +344,8 @@ def main():
                     help="rule_matching: keep only this many lookup-table rows (rule id mod rows), to bound "
                          "device memory under a profiler; 0 = one row per rule")
     ap.add_argument("--serving-steps", type=int, default=256, help="serving: decode steps of the loop")
+    ap.add_argument("--serving-batch", type=int, default=128,
+                    help="serving: sequences in the loop (fewer bound device memory under a profiler)")
     ap.add_argument("--no-configs", action="store_true",
                     help="default workload: skip the sub-runs of the other configurations")
     args = ap.parse_args()
@@ -768,8 +770,8 @@ def serving_bench(args):
     dev = torch.device("cuda", 0)
     umim.lib()
     peaks = load_peaks()
-    sl = W.serving_loop(W.SEEDS["serving"], B=128, n_layers=32, n_q_heads=32, n_kv_heads=8, head_dim=128,
-                        steps=args.serving_steps, p=0.1)
+    sl = W.serving_loop(W.SEEDS["serving"], B=args.serving_batch, n_layers=32, n_q_heads=32, n_kv_heads=8,
+                        head_dim=128, steps=args.serving_steps, p=0.1)
     plan = serving_plan(sl)
     B, NL = sl.B, sl.n_layers
     t = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev)
@@ -957,9 +959,9 @@ def serving_bench(args):
             "value": B * sl.steps / (ms / 1000.0), "unit": "tokens/s", "n_gpus": 1, "steps": sl.steps,
             "warmup": max(3, args.warmup), "ms_per_step": ms / sl.steps, "higher_is_better": True,
             "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": "serving decode loop: 128 seqs, lognormal(ln 1024, 1) lengths in [256, 8192], "
-                                   "32 layers x 32/8 heads, head_dim 128, bf16 paged KV (page 16), 256 steps of "
-                                   "append + p=0.1 merge of the last 2..4 entries + attention per layer",
+            "config": {"workload": f"serving decode loop: {B} seqs, lognormal(ln 1024, 1) lengths in [256, 8192], "
+                                   f"32 layers x 32/8 heads, head_dim 128, bf16 paged KV (page 16), {sl.steps} steps "
+                                   "of append + p=0.1 merge of the last 2..4 entries + attention per layer",
                        "kv_cache_gb": round(pool.numel() * 2 / 1e9, 1),
                        "l2": "inputs larger than L2: every attention launch reads about 1 GB of cache"},
             "rollbacks": n_roll, "rollbacks_per_s": n_roll / (ms / 1000.0),

@@ -371,30 +371,64 @@ __global__ void __launch_bounds__(kStepThreads, 1)
       const int w0 = o / W, w1 = (o + n - 1) / W;
       if (old != w1 - w0) return;   // another warp of the segment is still running
       // last to finish: merge the segment's partials (warp w0 used slot 1
-      // unless the segment starts its range; every later warp used slot 0)
+      // unless the segment starts its range; every later warp used slot 0),
+      // several pieces' loads in flight at a time
       __threadfence();
+      constexpr int U = E == 4 ? 4 : 8;
       for (int r = 0; r < G; ++r) {
         float M = -INFINITY, l = 0.f, ov[E];
 #pragma unroll
         for (int e = 0; e < E; ++e) ov[e] = 0.f;
-        for (int w = w0; w <= w1; ++w) {
-          const int sl = (w == w0 && o != w0 * W) ? 1 : 0;
-          const int64_t pc = ((int64_t)w * 2 + sl) * 16 + r;
-          const float2 pm = __ldcg(ws.part_ml + pc);
-          float av[E];
+        for (int w = w0; w <= w1; w += U) {
+          float2 pm[U];
+          float av[U][E];
 #pragma unroll
-          for (int e = 0; e < E; ++e) av[e] = __ldcg(ws.part_acc + pc * D + lane * E + e);
-          const float nm = fmaxf(M, pm.x);
+          for (int u = 0; u < U; ++u) {
+            pm[u] = make_float2(-INFINITY, 0.f);
+#pragma unroll
+            for (int e = 0; e < E; ++e) av[u][e] = 0.f;
+            if (w + u <= w1) {
+              const int sl = (w + u == w0 && o != w0 * W) ? 1 : 0;
+              const int64_t pc = ((int64_t)(w + u) * 2 + sl) * 16 + r;
+              pm[u] = __ldcg(ws.part_ml + pc);
+              if constexpr (E == 4) {
+                const float4 f = __ldcg(reinterpret_cast<const float4 *>(ws.part_acc + pc * D + lane * E));
+                av[u][0] = f.x, av[u][1] = f.y, av[u][2] = f.z, av[u][3] = f.w;
+              } else {
+                const float2 f = __ldcg(reinterpret_cast<const float2 *>(ws.part_acc + pc * D + lane * E));
+                av[u][0] = f.x, av[u][1] = f.y;
+              }
+            }
+          }
+          float nm = M;
+#pragma unroll
+          for (int u = 0; u < U; ++u) nm = fmaxf(nm, pm[u].x);
           if (nm == -INFINITY) continue;
-          const float c_old = exp2f(M - nm), c_new = exp2f(pm.x - nm);
-          l = l * c_old + pm.y * c_new;
+          const float c_old = exp2f(M - nm);
+          l *= c_old;
 #pragma unroll
-          for (int e = 0; e < E; ++e) ov[e] = ov[e] * c_old + av[e] * c_new;
+          for (int e = 0; e < E; ++e) ov[e] *= c_old;
+#pragma unroll
+          for (int u = 0; u < U; ++u) {
+            const float c = exp2f(pm[u].x - nm);   // 0 for an absent or empty piece
+            l = fmaf(pm[u].y, c, l);
+#pragma unroll
+            for (int e = 0; e < E; ++e) ov[e] = fmaf(av[u][e], c, ov[e]);
+          }
           M = nm;
         }
         const float inv = l > 0.f ? 1.f / l : 0.f;
-#pragma unroll
-        for (int e = 0; e < E; ++e) obase[(int64_t)r * D + lane * E + e] = __float2bfloat16_rn(ov[e] * inv);
+        if constexpr (E == 4) {
+          __nv_bfloat162 lo = __floats2bfloat162_rn(ov[0] * inv, ov[1] * inv);
+          __nv_bfloat162 hi = __floats2bfloat162_rn(ov[2] * inv, ov[3] * inv);
+          uint2 pk;
+          pk.x = *reinterpret_cast<uint32_t *>(&lo);
+          pk.y = *reinterpret_cast<uint32_t *>(&hi);
+          *reinterpret_cast<uint2 *>(obase + (int64_t)r * D + lane * E) = pk;
+        } else {
+          *reinterpret_cast<__nv_bfloat162 *>(obase + (int64_t)r * D + lane * E) =
+              __floats2bfloat162_rn(ov[0] * inv, ov[1] * inv);
+        }
       }
       if (lane == 0) ws.cnt[seg] = 0;   // ready for the next call
     };
