@@ -133,3 +133,22 @@ def test_serving_shape_sampled_layers():
     for layer, out in outs.items():
         ref = oracle.decode_attention(W.bits(c.q), rp, layer, rbt, rl)
         float_close(out.cpu().double().numpy(), ref, f"layer {layer}")
+
+
+def test_calls_leave_the_callers_current_device_unchanged():
+    """Every call makes its stream's device current only while it runs: the
+    caller's current device is the same afterwards (on a side stream too)."""
+    m = umim()
+    d = dev()
+    c = W.decode_case(71, lens=[100, 37], n_q_heads=8, n_kv_heads=2, head_dim=64, n_spans=[0, 0])
+    g = case_to_dev(c, d)
+    before = torch.cuda.current_device()
+    side = torch.cuda.Stream(d)
+    status = m.new_status(d)
+    with torch.cuda.stream(side):
+        m.umim_decode_attention(g["q"], g["pool"], 0, g["bt"], g["lens"], dev_status=status, stream=side)
+    assert torch.cuda.current_device() == before
+    m.umim_decode_attention(g["q"], g["pool"], 0, g["bt"], g["lens"], dev_status=status)
+    assert torch.cuda.current_device() == before
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
