@@ -238,8 +238,30 @@ __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs
     int32_t seen;       // the reader rows' smallest landed count when the unit was loaded
     int32_t shift;      // lanes < 16: the shift of slot `lane`
   };
+  // A unit's descriptors (its 16 sources, its page, its reader rows), read
+  // one unit ahead of its data loads so that the two round trips overlap.
+  struct Meta {
+    int64_t my_src;   // lanes < 16: the source of slot `lane`
+    int32_t valid, idx, page, tl;
+    int32_t shift;
+    RowDep dep;
+  };
   // slot i = kk * row_size + pos, kk the compacted page row
-  auto load = [&](int kk, int pos, Tile &t) {
+  auto fetch = [&](int kk, int pos, Meta &m) {
+    m.valid = 0;
+    if (kk >= max_dest) return;
+    const int j = pos / a.n_lanes;
+    if (kk >= nd_of(j)) return;
+    const int b = seq_of(j);
+    m.valid = 1;
+    m.tl = pos - j * a.n_lanes;
+    m.idx = ub_of(j) / a.n_lanes + kk;
+    m.my_src = lane < kPageSize ? pd.src[(int64_t)m.idx * kPageSize + lane] : kNoWrite;
+    m.page = a.block_table[(int64_t)b * a.max_pages + fp_of(j) + kk];
+    m.shift = (ROPE && lane < kPageSize) ? pd.shift[(int64_t)m.idx * kPageSize + lane] : 0;
+    m.dep = pd.dep[m.idx];
+  };
+  auto load = [&](const Meta &m, Tile &t) {
     t.mask = 0;
     t.valid = 0;
     t.rot = 0;
@@ -251,27 +273,22 @@ __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs
     t.seen = a.n_lanes;
 #pragma unroll
     for (int it = 0; it < PER_LANE; ++it) t.v[it] = make_uint4(0, 0, 0, 0);
-    if (kk >= max_dest) return;
-    const int j = pos / a.n_lanes, tl = pos - j * a.n_lanes;
-    if (kk >= nd_of(j)) return;
-    const int b = seq_of(j);
-    const int idx = ub_of(j) / a.n_lanes + kk;
-    const int64_t my_src = lane < kPageSize ? pd.src[(int64_t)idx * kPageSize + lane] : kNoWrite;
-    const int page = a.block_table[(int64_t)b * a.max_pages + fp_of(j) + kk];
+    if (!m.valid) return;
+    const int tl = m.tl;
     const int layer = tl / (2 * Hkv), kv = (tl / Hkv) & 1, h = tl % Hkv;
     const int64_t tile = layer * layer_stride + (int)(kv * kv_stride32 + h * kHead + my_col * 8);
     const uint16_t *sur = kv ? a.sur_v : a.sur_k;
     t.valid = 1;
-    t.row = idx;
-    t.dst = tile + (int64_t)page * page_stride32;
+    t.row = m.idx;
+    t.dst = tile + (int64_t)m.page * page_stride32;
     if (ROPE) {
       t.rot = kv == 0;
-      t.shift = lane < kPageSize ? pd.shift[(int64_t)idx * kPageSize + lane] : 0;
+      t.shift = m.shift;
     }
 #pragma unroll
     for (int it = 0; it < PER_LANE; ++it) {
       const int slot = my_slot0 + it * SLOT_STEP;
-      const int64_t src = __shfl_sync(0xffffffffu, my_src, slot);
+      const int64_t src = __shfl_sync(0xffffffffu, m.my_src, slot);
       if (src != kNoWrite) t.mask |= 1u << it;
       if (src >= 0) {
         t.v[it] = ld_v4(a.pool + tile + src);
@@ -280,9 +297,8 @@ __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs
         t.v[it] = ld_v4(sur + ((si * a.n_layers + layer) * Hkv + h) * D + my_col * 8);
       }
     }
-    const RowDep dep = pd.dep[idx];
-    t.dlo = dep.lo;
-    t.dhi = dep.hi;
+    t.dlo = m.dep.lo;
+    t.dhi = m.dep.hi;
   };
   auto store = [&](const Tile &t) {
 #pragma unroll
@@ -388,21 +404,30 @@ __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs
     }
   };
   Tile A, B;
+  Meta M;   // the descriptors of the next unit to load
   if (my_units > 0) {
-    load(kk, pos, A);
+    fetch(kk, pos, M);
     advance();
-    load(kk, pos, B);
+    load(M, A);
+    fetch(kk, pos, M);
+    advance();
+    load(M, B);
+    fetch(kk, pos, M);
     advance();
     land_and_count(A);
     rotate(A);
-    // unit u in `cur` (landed, counted, rotated), unit u + 1 in flight in `next`;
-    // the next unit is rotated while unit u + 2's loads are in flight
+    // unit u in `cur` (landed, counted, rotated), unit u + 1 in flight in `next`:
+    // u is stored and u + 2's loads are issued before waiting for u + 1's, so
+    // two units' loads are in flight during that wait.  Every unit is still
+    // counted before it is stored, so the lowest-numbered unstored unit can
+    // always proceed.
     auto step = [&](Tile &cur, Tile &next) -> bool {
-      land_and_count(next);
       if (!readers_done(cur)) return false;
       store(cur);
-      load(kk, pos, cur);   // unit u + 2
+      load(M, cur);   // unit u + 2
+      fetch(kk, pos, M);
       advance();
+      land_and_count(next);
       rotate(next);
       return true;
     };
