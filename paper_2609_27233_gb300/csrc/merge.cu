@@ -309,21 +309,22 @@ __device__ __forceinline__ Moments merge_moments(Moments a, Moments b) {
 }
 
 // One warp merges the per-tile (mean, M2) of a row; every lane gets
-// (mean, 1/sqrt(var + eps)).
+// (mean, 1/sqrt(var + eps)).  Every tile holds BN values, so the row's mean is
+// the tiles' average mean and M2 = sum M2_t + BN sum (mean_t - mean)^2.
 __device__ __forceinline__ float2 row_moments_warp(const float2 *st, int ntiles, int d, float eps) {
   const int lane = threadIdx.x & 31;
-  Moments m{0.f, 0.f, 0.f};
-  for (int t = lane; t < ntiles; t += 32) {
-    const float2 v = st[t];
-    m = merge_moments(m, Moments{(float)BN, v.x, v.y});
-  }
+  const float2 v = lane < ntiles ? st[lane] : make_float2(0.f, 0.f);   // ntiles <= 32 (d <= 8192)
+  float sm = v.x, s2 = v.y;
 #pragma unroll
   for (int o = 16; o >= 1; o >>= 1) {
-    Moments x{__shfl_xor_sync(0xffffffffu, m.n, o), __shfl_xor_sync(0xffffffffu, m.mean, o),
-              __shfl_xor_sync(0xffffffffu, m.m2, o)};
-    m = merge_moments(m, x);
+    sm += __shfl_xor_sync(0xffffffffu, sm, o);
+    s2 += __shfl_xor_sync(0xffffffffu, s2, o);
   }
-  return make_float2(m.mean, rsqrtf(m.m2 / (float)d + eps));
+  const float mean = sm / (float)ntiles;
+  float dv = lane < ntiles ? (v.x - mean) * (v.x - mean) : 0.f;
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) dv += __shfl_xor_sync(0xffffffffu, dv, o);
+  return make_float2(mean, rsqrtf((s2 + (float)BN * dv) / (float)d + eps));
 }
 
 // ---------------------------------------------------------------------------
