@@ -7,24 +7,22 @@
 // On the 5th-generation tensor cores: one CTA takes 128 query rows of one
 // sequence for one query head, and two CTAs share an SM (each allocates half
 // of the tensor memory), so one CTA's products fill the tensor cores while
-// the other's softmax runs.  The softmax threads (one per query row) copy
-// their row of Q into tensor memory, so the product S = Q K^T takes Q from
-// tensor memory and reads only the 64-key K tile from shared memory (at
-// N = 64, products with both operands in shared memory are bound by its
-// bandwidth).  Warp 0 loads K tiles (3-stage ring, two tiles ahead of the
-// V^T tiles' 2-stage ring) with TMA; warp 1 issues tcgen05.mma: S(j) into
-// the S columns, then, once the softmax has turned S(j) into P(j), O += P(j)
-// V(j) (fp16 operands, P read from tensor memory), and S(j + 1) only after
-// that product has finished reading P(j).  Warps 2-5 run the online softmax:
-// S from tensor memory (tcgen05.ld), causal mask, running max, P =
-// exp2(S - max) written back in fp16 over the S columns (tcgen05.st), row
-// sums.  P V runs on fp16 operands (V^T is converted when it is transposed):
-// fp16's 11-bit significand keeps P's and V's rounding near 3e-4 relative,
-// where bf16 P would cost 1e-3 of the output's error budget; P <= 2^8 by
-// construction and |v| < 65504 is checked (UMIM_ERR_UNSUPPORTED otherwise).
-// The running max is only moved when it grows by more than 2^8, so the
-// accumulator in tensor memory is rescaled rarely (the result is the same: P
-// and the row sum use the same stale max).
+// the other's softmax runs.  Warp 0 loads tiles with TMA (Q once; 64-key K
+// tiles into a 2-stage ring running a tile ahead of the V^T tiles' 2-stage
+// ring), warp 1 issues tcgen05.mma (S = Q K^T into one of two tensor-memory
+// buffers, O += P V into a tensor-memory accumulator; an S buffer is reused
+// once the P V product that read it is done), and warps 2-5 run the online
+// softmax, one thread per query row: S from tensor memory (tcgen05.ld),
+// causal mask, running max, P = exp2(S - max) written back in fp16 over the
+// S columns it came from (tcgen05.st; the P V product reads its A operand
+// from tensor memory, so P never touches shared memory), row sums.  P V runs
+// on fp16 operands (V^T is converted when it is transposed): fp16's 11-bit
+// significand keeps P's and V's rounding near 3e-4 relative, where bf16 P
+// would cost 1e-3 of the output's error budget; P <= 2^8 by construction and
+// |v| < 65504 is checked (UMIM_ERR_UNSUPPORTED otherwise).  The running max
+// is only moved when it grows by more than 2^8, so the accumulator in tensor
+// memory is rescaled rarely (the result is the same: P and the row sum use
+// the same stale max).
 //
 // V is transposed first (per sequence, padded to a multiple of 64 keys) so
 // that both products read K-major operands and every TMA copy starts on a
@@ -47,15 +45,13 @@ namespace {
 
 constexpr int kPfRows = 128;             // query rows per CTA (the MMA's M)
 constexpr int kPfKeys = 64;              // keys per K / V tile (the S MMA's N)
-constexpr int kPfKStages = 3;            // K ring (K runs kPfKStages - 1 tiles ahead of V^T)
+constexpr int kPfKStages = 2;            // K ring (K runs kPfKStages - 1 tiles ahead of V^T)
 constexpr int kPfVStages = 2;            // V^T ring
 constexpr int kPfThreads = 192;          // warp 0 TMA, warp 1 MMA + tensor memory, warps 2-5 softmax (thread = query row)
 constexpr int kPfPlanThreads = 1024;
-constexpr uint32_t kPfTmemCols = 256;    // Q at 0 (D/2 columns), S / P at 64, O at 128: two CTAs per SM
-constexpr uint32_t kPfColS = 64, kPfColO = 128;
+constexpr uint32_t kPfTmemCols = 256;    // S buffers at 0 and 64, O at 128: two CTAs per SM
 
 struct PfArgs {
-  const __nv_bfloat16 *q;           // [T][Hq][D]
   __nv_bfloat16 *out;               // [T][Hq][D]
   const int32_t *cu;                // [B + 1]
   int32_t *cu_tiles;                // [B + 1] workspace: query-tile offsets
@@ -245,27 +241,29 @@ __device__ __forceinline__ void tc_mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint
 // shared-memory layout of the attention kernel (bytes, every piece 1024-aligned)
 template <int D>
 struct PfSmem {
+  static constexpr int kQ = kPfRows * D * 2;              // Q of one head: D/64 atoms of [128 rows][128 B]
   static constexpr int kK = kPfKeys * D * 2;              // K tile: D/64 atoms of [64 keys][128 B]
   static constexpr int kV = D * kPfKeys * 2;              // V^T tile: [D rows][128 B]
-  static constexpr int kKoff = 0;
+  static constexpr int kKoff = kQ;
   static constexpr int kVoff = kKoff + kPfKStages * kK;
   static constexpr int kTotal = kVoff + kPfVStages * kV;
 };
 
 template <int D>
 __global__ void __launch_bounds__(kPfThreads, 2)
-    prefill_tc_kernel(const __grid_constant__ CUtensorMap k_map, const __grid_constant__ CUtensorMap vt_map, PfArgs a) {
+    prefill_tc_kernel(const __grid_constant__ CUtensorMap q_map, const __grid_constant__ CUtensorMap k_map,
+                      const __grid_constant__ CUtensorMap vt_map, PfArgs a) {
   using L = PfSmem<D>;
   constexpr int DA = D / 64;   // 64-wide atoms along the head dimension
   extern __shared__ __align__(1024) uint8_t pf_raw[];
   __shared__ __align__(8) uint64_t q_full, k_full[kPfKStages], k_empty[kPfKStages], v_full[kPfVStages],
-      v_empty[kPfVStages], s_full, p_full, pv_done, o_done, mma_done;
+      v_empty[kPfVStages], s_full[2][2], s_empty[2][2], p_full[2][2], p_empty[2], o_done[2], mma_done;
   __shared__ uint32_t tmem_base;
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(pf_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) {
-    mbar_init(&q_full, 4);   // one arrival per softmax warp (its rows of Q are in tensor memory)
+    mbar_init(&q_full, 1);
     for (int s = 0; s < kPfKStages; ++s) {
       mbar_init(&k_full[s], 1);
       mbar_init(&k_empty[s], 1);
@@ -274,12 +272,20 @@ __global__ void __launch_bounds__(kPfThreads, 2)
       mbar_init(&v_full[s], 1);
       mbar_init(&v_empty[s], 1);
     }
-    mbar_init(&s_full, 1);    // S(j) landed: phase j
-    mbar_init(&p_full, 4);    // P(j) written: phase j, one arrival per softmax warp
-    mbar_init(&pv_done, 1);   // P(j) V(j) finished (P(j)'s columns and O free): phase j
-    mbar_init(&o_done, 1);    // one phase: every product of the CTA has landed
+    for (int x = 0; x < 2; ++x) {
+      for (int i = 0; i < 2; ++i) {
+        mbar_init(&s_full[x][i], 1);
+        mbar_init(&s_empty[x][i], 1);   // committed once the P V product that read P from it is done
+      }
+      // P(j) ready, by tile parity: the softmax can run a tile ahead of the MMA warp's wait
+      mbar_init(&p_full[x][0], 4);
+      mbar_init(&p_full[x][1], 4);
+      mbar_init(&p_empty[x], 1);
+      mbar_init(&o_done[x], 1);   // one phase: every product of the CTA has landed
+    }
     mbar_init(&mma_done, 1);
     fence_mbar_init();
+    prefetch_tensormap(&q_map);
     prefetch_tensormap(&k_map);
     prefetch_tensormap(&vt_map);
   }
@@ -293,7 +299,7 @@ __global__ void __launch_bounds__(kPfThreads, 2)
   const uint32_t tmem = tmem_base;
   griddep_wait();
 
-  // the work unit: query tile qt of sequence b for query head h
+  // the work unit: query tile qt of sequence b for the query heads h0 (and h0 + 1)
   const int total = a.cu_tiles[a.B];
   const bool active = (int)blockIdx.x < total;
   int b = 0, qt = 0;
@@ -304,13 +310,19 @@ __global__ void __launch_bounds__(kPfThreads, 2)
   }
   const int s0 = active ? a.cu[b] : 0, len = active ? a.cu[b + 1] - s0 : 0;
   const int q0 = qt * kPfRows;
-  const int h = (int)blockIdx.y, g = h / a.G;
+  const int h0 = (int)blockIdx.y, g = h0 / a.G;          // one query head per CTA
+  const int nh = 1;
   const int n_kv = active ? (min(q0 + kPfRows, len) + kPfKeys - 1) / kPfKeys : 0;   // causal key tiles
   const int kbase = active ? a.pcu[b] : 0;
 
   if (warp == 0) {
     if (lane == 0 && n_kv > 0) {
-      const uint64_t pol_kv = policy_evict_last();
+      const uint64_t pol_q = policy_evict_first(), pol_kv = policy_evict_last();
+      mbar_arrive_expect_tx(&q_full, nh * L::kQ);
+      for (int x = 0; x < nh; ++x)
+#pragma unroll
+        for (int d = 0; d < DA; ++d)
+          tma_load_3d(smem + x * L::kQ + d * (kPfRows * 128), &q_map, &q_full, d * 64, h0 + x, s0 + q0, pol_q);
       // K runs kPfKStages - 1 tiles ahead of V^T: a K load never waits behind
       // the P V product that frees a V^T stage
       constexpr int kLead = kPfKStages - 1;
@@ -348,91 +360,91 @@ __global__ void __launch_bounds__(kPfThreads, 2)
         mbar_wait_for(&k_full[i % kPfKStages], (i / kPfKStages) & 1, kWaitLimitNs);
       for (int i = max(0, jv - kPfVStages); i < jv; ++i)
         mbar_wait_for(&v_full[i % kPfVStages], (i / kPfVStages) & 1, kWaitLimitNs);
+      mbar_wait_for(&q_full, 0, kWaitLimitNs);
     }
   } else if (warp == 1) {
     if (lane == 0 && n_kv > 0) {
-      constexpr uint32_t idesc_s = idesc_f32acc(kPfRows, kPfKeys, false);   // Q (tensor memory) and K in bf16
-      constexpr uint32_t idesc_o = idesc_f32acc(kPfRows, D, true);          // P and V^T in fp16
+      constexpr uint32_t idesc_s = idesc_f32acc(kPfRows, kPfKeys, false);
+      constexpr uint32_t idesc_o = idesc_f32acc(kPfRows, D, true);   // P and V^T in fp16
       bool ok = mbar_wait(&q_full, 0);
+      tc_fence_after();
+      // O_x += P_x(i) V(i) for both heads (fp16 operands, P from tensor memory); frees V(i) and S(i)'s buffer
+      auto pv = [&](int i) {
+        const int s = i % kPfVStages;
+        if (!mbar_wait(&v_full[s], (i / kPfVStages) & 1)) return false;
+        const uint32_t v_base = smem_u32(smem + L::kVoff + s * L::kV);
+        for (int x = 0; x < nh; ++x) {
+          if (!mbar_wait(&p_full[x][i & 1], (i >> 1) & 1)) return false;
+          tc_fence_after();
+          const uint32_t p_tmem = tmem + x * 256 + (i & 1) * kPfKeys;   // P(i) sits where S(i) was
+#pragma unroll
+          for (int kk = 0; kk < kPfKeys / 16; ++kk)
+            tc_mma_ts(tmem + x * 256 + 128, p_tmem + kk * 8, sw128_kmajor_desc(v_base + kk * 32), idesc_o,
+                      (i | kk) != 0 ? 1u : 0u);
+          tc_commit(&p_empty[x]);
+          tc_commit(&s_empty[x][i & 1]);
+        }
+        tc_commit(&v_empty[s]);
+        return true;
+      };
       for (int j = 0; j < n_kv && ok; ++j) {
-        const int s = j % kPfKStages;
-        // K(j) has landed, and the product of tile j - 1 no longer reads P(j - 1)'s columns
-        if (!mbar_wait(&k_full[s], (j / kPfKStages) & 1) || (j > 0 && !mbar_wait(&pv_done, (j - 1) & 1))) {
+        const int s = j % kPfKStages, sb = j & 1;
+        if (!mbar_wait(&k_full[s], (j / kPfKStages) & 1)) {
           ok = false;
           break;
         }
-        tc_fence_after();
         const uint32_t k_base = smem_u32(smem + L::kKoff + s * L::kK);
+        for (int x = 0; x < nh && ok; ++x) {
+          if (!mbar_wait(&s_empty[x][sb], ((j >> 1) & 1) ^ 1)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t q_base = smem_u32(smem + x * L::kQ);
 #pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk)
-          tc_mma_ts(tmem + kPfColS, tmem + kk * 8,
-                    sw128_kmajor_desc(k_base + (kk >> 2) * (kPfKeys * 128) + (kk & 3) * 32), idesc_s,
-                    kk != 0 ? 1u : 0u);
-        tc_commit(&s_full);
-        tc_commit(&k_empty[s]);
-        // O += P(j) V(j) once the softmax has written P(j)
-        const int sv = j % kPfVStages;
-        if (!mbar_wait(&p_full, j & 1) || !mbar_wait(&v_full[sv], (j / kPfVStages) & 1)) {
-          ok = false;
-          break;
+          for (int kk = 0; kk < D / 16; ++kk) {
+            const uint32_t off = (kk & 3) * 32;
+            tc_mma_bf16(tmem + x * 256 + sb * kPfKeys, sw128_kmajor_desc(q_base + (kk >> 2) * (kPfRows * 128) + off),
+                        sw128_kmajor_desc(k_base + (kk >> 2) * (kPfKeys * 128) + off), idesc_s, kk != 0 ? 1u : 0u);
+          }
+          tc_commit(&s_full[x][sb]);
         }
-        tc_fence_after();
-        const uint32_t v_base = smem_u32(smem + L::kVoff + sv * L::kV);
-#pragma unroll
-        for (int kk = 0; kk < kPfKeys / 16; ++kk)
-          tc_mma_ts(tmem + kPfColO, tmem + kPfColS + kk * 8, sw128_kmajor_desc(v_base + kk * 32), idesc_o,
-                    (j | kk) != 0 ? 1u : 0u);
-        tc_commit(&pv_done);
-        tc_commit(&v_empty[sv]);
+        if (!ok) break;
+        tc_commit(&k_empty[s]);
+        if (j >= 1 && !pv(j - 1)) ok = false;
       }
-      if (ok) tc_commit(&o_done);
+      if (ok && !pv(n_kv - 1)) ok = false;
+      if (ok)
+        for (int x = 0; x < nh; ++x) tc_commit(&o_done[x]);
       if (!ok) set_error(a.status, UMIM_ERR_TIMEOUT);
       // every MMA issued has finished before tensor memory is released
       tc_commit(&mma_done);
       mbar_wait_for(&mma_done, 0, kWaitLimitNs);
     }
-  } else {
-    // ---- softmax and epilogue: four warps, thread = query row ----
+  } else if ((warp - 2) / 4 < nh) {
+    // ---- softmax and epilogue of head x: four warps, thread = query row ----
+    const int x = (warp - 2) >> 2;
     const int quad = warp & 3;                 // tensor-memory lanes this warp may access
     const int r = quad * 32 + lane;            // query row within the tile
     const int qpos = q0 + r;                   // position within the sequence
     const int kmax = min(qpos, len - 1);       // last key this row sees
-    const uint32_t t_row = tmem + ((uint32_t)(quad * 32) << 16);
-    const uint32_t t_s = t_row + kPfColS, t_o = t_row + kPfColO;
+    const uint32_t t_s = tmem + ((uint32_t)(quad * 32) << 16) + x * 256;   // this row's S buffers
+    const uint32_t t_o = t_s + 128;                                         // and O
     const float sl2 = a.scale_log2;
     float m_run = -INFINITY, l_run = 0.f;      // running max (log2 units, moved in steps > 8) and row sum
     bool ok = true;
     // every lane waits (each needs the acquire), the warp goes on only if all saw the phase:
     // the .sync.aligned tensor-memory instructions below need the whole warp
     auto wwait = [&](uint64_t *m, uint32_t parity) { return __all_sync(0xffffffffu, mbar_wait(m, parity)) != 0; };
-    if (n_kv > 0) {
-      // this row of Q into tensor memory (bf16 pairs, column c = elements 2c and 2c + 1): the A operand of S
-      const uint4 *qrow = reinterpret_cast<const uint4 *>(a.q + (((int64_t)s0 + qpos) * a.Hq + h) * D);
-#pragma unroll
-      for (int half = 0; half < D / 64; ++half) {
-        float qv[32];
-#pragma unroll
-        for (int c = 0; c < 8; ++c) {
-          const uint4 u = qpos < len ? __ldg(qrow + half * 8 + c) : make_uint4(0, 0, 0, 0);
-          qv[4 * c] = __uint_as_float(u.x);
-          qv[4 * c + 1] = __uint_as_float(u.y);
-          qv[4 * c + 2] = __uint_as_float(u.z);
-          qv[4 * c + 3] = __uint_as_float(u.w);
-        }
-        tmem_st_32x32b_x32(t_row + half * 32, qv);
-      }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&q_full);
-    }
     for (int j = 0; j < n_kv && ok; ++j) {
-      if (!wwait(&s_full, j & 1)) {
+      const int sb = j & 1;
+      if (!wwait(&s_full[x][sb], (j >> 1) & 1)) {
         ok = false;
         break;
       }
       tc_fence_after();
       float s[kPfKeys];
-      tmem_ld_32x32b_x64(t_s, s);
+      tmem_ld_32x32b_x64(t_s + sb * kPfKeys, s);
       const int k0 = j * kPfKeys;
       if (k0 + kPfKeys - 1 > kmax) {   // the diagonal tile (or a row past the sequence)
 #pragma unroll
@@ -458,10 +470,9 @@ __global__ void __launch_bounds__(kPfThreads, 2)
         l4[c & 3] += s[c];
       }
       l_run += (l4[0] + l4[1]) + (l4[2] + l4[3]);
-      // P(j) in fp16 over S(j)'s columns (this thread has read them), for the P V product; O is
-      // rescaled first, once the product of tile j - 1 has landed
+      // O is rescaled only once the product of tile j - 1 has landed
       if (j > 0 && __any_sync(0xffffffffu, grow)) {
-        if (!wwait(&pv_done, (j - 1) & 1)) {
+        if (!wwait(&p_empty[x], (j - 1) & 1)) {
           ok = false;
           break;
         }
@@ -474,7 +485,9 @@ __global__ void __launch_bounds__(kPfThreads, 2)
           for (int i = 0; i < 32; ++i) o[i] *= alpha;
           tmem_st_32x32b_x32(t_o + c * 32, o);
         }
+        tc_fence_before();
       }
+      // P(j) in fp16 over S(j)'s columns (this thread has read them), for the P V product
       {
         float pk[32];
 #pragma unroll
@@ -482,18 +495,18 @@ __global__ void __launch_bounds__(kPfThreads, 2)
           const __half2 hh = __floats2half2_rn(s[2 * c], s[2 * c + 1]);   // P <= 2^8
           pk[c] = __uint_as_float(*reinterpret_cast<const uint32_t *>(&hh));
         }
-        tmem_st_32x32b_x32(t_s, pk);
+        tmem_st_32x32b_x32(t_s + sb * kPfKeys, pk);
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&p_full);
+      if (lane == 0) mbar_arrive(&p_full[x][sb]);
     }
     if (!ok) set_error(a.status, UMIM_ERR_TIMEOUT);
     // epilogue: O / l once the last product has landed
-    if (ok && n_kv > 0 && wwait(&o_done, 0)) {
+    if (ok && n_kv > 0 && wwait(&o_done[x], 0)) {
       tc_fence_after();
       const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
-      __nv_bfloat16 *orow = a.out + (((int64_t)s0 + qpos) * a.Hq + h) * D;
+      __nv_bfloat16 *orow = a.out + (((int64_t)s0 + qpos) * a.Hq + h0 + x) * D;
 #pragma unroll 1
       for (int c = 0; c < D / 32; ++c) {
         float o[32];
@@ -549,7 +562,6 @@ umim_status prefill_attention(const void *q, const void *k, const void *v, int T
   EncodeTiledFn enc = get_encode_tiled();
   if (!enc) return UMIM_ERR_CUDA;
   PfArgs a{};
-  a.q = static_cast<const __nv_bfloat16 *>(q);
   a.out = static_cast<__nv_bfloat16 *>(out);
   a.cu = cu_seqlens;
   a.cu_tiles = static_cast<int32_t *>(ws);
@@ -565,8 +577,9 @@ umim_status prefill_attention(const void *q, const void *k, const void *v, int T
   a.G = Hq / Hkv;
   a.scale_log2 = (scale > 0.f ? scale : 1.0f / sqrtf((float)D)) * 1.4426950408889634f;
   a.status = status;
-  CUtensorMap km, vm;
-  if (!encode_3d(enc, &km, k, D, Hkv, T, (uint64_t)D * 2, (uint64_t)Hkv * D * 2, 64, 1, kPfKeys) ||
+  CUtensorMap qm, km, vm;
+  if (!encode_3d(enc, &qm, q, D, Hq, T, (uint64_t)D * 2, (uint64_t)Hq * D * 2, 64, 1, kPfRows) ||
+      !encode_3d(enc, &km, k, D, Hkv, T, (uint64_t)D * 2, (uint64_t)Hkv * D * 2, 64, 1, kPfKeys) ||
       !encode_3d(enc, &vm, a.vt, a.Tp, D, Hkv, (uint64_t)a.Tp * 2, (uint64_t)D * a.Tp * 2, kPfKeys, D, 1, true))
     return UMIM_ERR_CUDA;
   trace_mark(stream, "prefill.plan");
@@ -584,7 +597,7 @@ umim_status prefill_attention(const void *q, const void *k, const void *v, int T
   const unsigned gx = (unsigned)((T + kPfRows - 1) / kPfRows + B);
   trace_mark(stream, "prefill.attention");
   const unsigned gy = (unsigned)Hq;   // one query head per CTA
-  if (launch_pdl(kern, dim3(gx, gy), dim3(kPfThreads), smem, stream, km, vm, a) != cudaSuccess)
+  if (launch_pdl(kern, dim3(gx, gy), dim3(kPfThreads), smem, stream, qm, km, vm, a) != cudaSuccess)
     return UMIM_ERR_CUDA;
   trace_mark(stream, nullptr);
   return UMIM_OK;
