@@ -29,6 +29,9 @@
 #include <cstdio>
 #include <cstdlib>
 #include <mutex>
+#include <type_traits>
+
+#include <cuda_fp16.h>
 
 #include "common.cuh"
 
@@ -277,7 +280,7 @@ struct CeHeader {
 static_assert(sizeof(CeHeader) == 256, "ce header size");
 
 size_t ce_ws_bytes(int R_S, int max_pairs) {
-  return a256(sizeof(CeHeader)) + a256(sizeof(int32_t) * (size_t)std::max(R_S, 1)) +
+  return a256(sizeof(CeHeader)) + 2 * a256(sizeof(int32_t) * (size_t)std::max(R_S, 1)) +
          a256(sizeof(float) * (size_t)std::max(max_pairs, 1));
 }
 
@@ -293,6 +296,7 @@ struct CeArgs {
   float *pair_loss;
   uint16_t *grad;                      // bf16 [R_S][ld] or nullptr
   int32_t *row_pair;                   // [R_S] pair of each student row, -1 if none
+  int32_t *row_teacher;                // [R_S] teacher row paired with each student row, -1 if none
   CeHeader *hdr;
   int32_t *status;
   int32_t chunk_vecs;                  // 16-byte vectors of a row per CTA
@@ -314,6 +318,7 @@ __global__ void ce_prep_kernel(CeArgs a) {
     const int t = a.teacher_rows[p], s = a.student_rows[p];
     bool ok = t >= 0 && t < a.R_T && s >= 0 && s < a.R_S;
     if (ok && atomicCAS(&a.row_pair[s], -1, p) != -1) ok = false;   // a student row in two pairs
+    if (ok) a.row_teacher[s] = t;
     if (!ok) {
       atomicOr(&a.hdr->error, 1);
       set_error(a.status, UMIM_ERR_INVALID_ARG);
@@ -373,19 +378,52 @@ __device__ __forceinline__ float rcp_approx(float x) {
   return y;
 }
 
-// Softmax statistics over a warp: from each lane's (m, z) with
-// z = sum exp(x - m) over its values (m = -inf: no values), every lane gets
-// the warp's max and its sum exp(x - max).  The max first, then one rescale
-// per lane, then a plain sum: xor butterflies give every lane the same bits.
-__device__ __forceinline__ void warp_lse(float &m, float &z) {
-  float M = m;
+// 32 lanes x 16 consecutive 32-bit columns of tensor memory from / to 16
+// registers of each thread of the warp (thread i: lane base + i)
+__device__ __forceinline__ void tmem_st_x16(uint32_t taddr, const uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+      "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]),
+      "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
+      : "memory");
+}
+__device__ __forceinline__ void tmem_ld_x16(uint32_t taddr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr)
+      : "memory");
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+
+// bf16x2 -inf, and the packed maximum of two bf16 pairs
+constexpr uint32_t kNegInfBf16x2 = 0xff80ff80u;
+__device__ __forceinline__ uint32_t max_bf16x2(uint32_t x, uint32_t y) {
+  uint32_t d;
+  asm("max.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(x), "r"(y));
+  return d;
+}
+// a bf16 pair (element 0 in the low half) as two floats
+__device__ __forceinline__ float2 bf16x2_to_float2(uint32_t w) {
+  return make_float2(__uint_as_float(w << 16), __uint_as_float(w & 0xffff0000u));
+}
+// the maximum over the warp, one instruction
+__device__ __forceinline__ float redux_max_f32(float x) {
+  float r;
+  asm volatile("redux.sync.max.f32 %0, %1, 0xffffffff;" : "=f"(r) : "f"(x));
+  return r;
+}
+// sum over the warp of a pair of floats: xor butterflies, so every lane gets
+// the same bits
+__device__ __forceinline__ float2 warp_sum2(float2 v) {
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-  float w = (m == -INFINITY) ? 0.f : z * ex2_approx((m - M) * kLog2e);
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) w += __shfl_xor_sync(0xffffffffu, w, o);
-  m = M;
-  z = w;
+  for (int o = 16; o > 0; o >>= 1)
+    v = __fadd2_rn(v, make_float2(__shfl_xor_sync(0xffffffffu, v.x, o), __shfl_xor_sync(0xffffffffu, v.y, o)));
+  return v;
 }
 
 // mbarrier wait that sleeps instead of spinning: try_wait with a suspend-time
@@ -403,28 +441,25 @@ __device__ __forceinline__ bool mbar_try_wait_sleep(uint32_t bar, uint32_t parit
       : "memory");
   return ok != 0;
 }
+__device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
 __device__ __forceinline__ bool mbar_wait_sleep(uint64_t *bar, uint32_t parity) {
   const uint32_t a = smem_u32(bar);
+  if (mbar_test_wait(a, parity)) return true;   // a phase already complete costs no suspension
   if (mbar_try_wait_sleep(a, parity)) return true;
   const uint64_t t0 = globaltimer();
   while (true) {
     if (mbar_try_wait_sleep(a, parity)) return true;
     if (globaltimer() - t0 > kWaitLimitNs) return false;
-  }
-}
-
-__device__ __forceinline__ float warp_sum(float x) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
-  return x;
-}
-
-__device__ __forceinline__ void unpack8(const uint4 u, float *f) {
-  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
-#pragma unroll
-  for (int j = 0; j < 4; ++j) {
-    f[2 * j] = __uint_as_float(w[j] << 16);
-    f[2 * j + 1] = __uint_as_float(w[j] & 0xffff0000u);
   }
 }
 
@@ -443,10 +478,12 @@ __device__ __forceinline__ void store8(uint16_t *row, int64_t e, int V, const fl
     o.w = pack_bf16x2(g[6], g[7]);
     *reinterpret_cast<uint4 *>(row + e) = o;
   } else {
-    for (int j = 0; j < 8 && e + j < V; ++j) {
-      __nv_bfloat16 h = __float2bfloat16_rn(g[j]);
-      row[e + j] = *reinterpret_cast<uint16_t *>(&h);
-    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+      if (e + j < V) {
+        __nv_bfloat16 h = __float2bfloat16_rn(g[j]);
+        row[e + j] = *reinterpret_cast<uint16_t *>(&h);
+      }
   }
 }
 
@@ -471,14 +508,39 @@ __device__ __forceinline__ void st_async_f4(uint32_t raddr, float4 v, uint32_t r
                : "memory");
 }
 
+// One cluster of C CTAs per student row; CTA `rank` owns vectors
+// [rank * chunk_vecs, ...) of the row.  T compute threads (NW warps) hold
+// KV vectors of the teacher and student row each, and one more warp issues
+// the copies: lane 0 walks the CTA's paired rows, waits for a stage of the
+// ring to be released by every compute warp, and loads the teacher and
+// student chunk into it with two bulk copies.
+//
+// The compute warps run two rows at once.  For row c they take the logits
+// from the stage, the thread's max, exp(x - max) and the sums (pass 1) and
+// push the warp's softmax statistics to every CTA of the cluster; then they
+// wait for the loss sums of row c - 1 and write its gradient; then they wait
+// for row c's statistics, form P^T and P^S, the loss terms and
+// a_v = P^T P^S / (P^S + eps) (pass 2) and push the warp's sums.  Each
+// exchange is thus waited for one compute phase after it was pushed.
+// Between the phases a row is held in registers as fp32 exp(x - max)
+// (pass 1 -> 2), then in tensor memory (which this kernel has no other use
+// for) as fp32 P^S and -a_v / N (pass 2 -> gradient): each warp owns 16 x KV
+// columns of its lane quarter, 16 per vector.
 template <int KV, int T>
-__global__ void __launch_bounds__(T, 512 / T) ce_kernel(CeArgs a) {
-  constexpr int NW = T / 32;
+__global__ void __launch_bounds__(T + 32, 1) ce_kernel(CeArgs a) {
+  constexpr int NW = T / 32;               // compute warps; warp NW issues the copies
   constexpr int NX = kCeMaxCluster * NW;   // partial slots per buffer
+  constexpr int NP = 4 * KV;               // element pairs (one 32-bit word of each row) per thread
+  constexpr int NPX = (NX + 31) / 32;      // partials per lane, at most
+  // tensor-memory columns: 16 per vector for each warp of a lane quarter
+  constexpr uint32_t kTmemNeed = (uint32_t)((NW + 3) / 4) * 16u * KV;
+  constexpr uint32_t kTmemCols = kTmemNeed <= 32 ? 32 : kTmemNeed <= 64 ? 64 : kTmemNeed <= 128 ? 128 : 256;
+  static_assert(kTmemNeed <= 256, "tensor memory");
   extern __shared__ __align__(128) uint8_t ce_smem[];
-  __shared__ __align__(8) uint64_t full_bar[kCeMaxStages];
+  __shared__ __align__(8) uint64_t full_bar[kCeMaxStages], empty_bar[kCeMaxStages];
   __shared__ __align__(8) uint64_t xbar[2][2];        // [stats | sums][row parity]
   __shared__ __align__(16) float4 xbuf[2][2][NX];     // [stats | sums][row parity][rank * NW + warp]
+  __shared__ uint32_t s_tmem;
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const uint32_t rank = cluster_ctarank();
@@ -487,6 +549,8 @@ __global__ void __launch_bounds__(T, 512 / T) ce_kernel(CeArgs a) {
   const int nvec = (a.V + 7) >> 3;
   const int vbeg = (int)rank * a.chunk_vecs;
   const int vcnt = max(0, min(a.chunk_vecs, nvec - vbeg));
+  // vectors of the chunk that lie wholly below V; a vector cut by V is stored element-wise
+  const int vfull = max(0, min(vcnt, a.V / 8 - vbeg));
   const int S = a.stages;
   uint4 *stage_base = reinterpret_cast<uint4 *>(ce_smem);   // [S][2][chunk_vecs]
   const uint32_t tx_bytes = 2u * (uint32_t)vcnt * 16u;
@@ -494,48 +558,31 @@ __global__ void __launch_bounds__(T, 512 / T) ce_kernel(CeArgs a) {
 
   if (a.hdr->error) return;   // the prep kernel rejected the pairs: write nothing (every CTA alike)
   if (tid == 0) {
-    for (int s = 0; s < S; ++s) mbar_init(&full_bar[s], 1);
+    for (int s = 0; s < S; ++s) {
+      mbar_init(&full_bar[s], 1);
+      mbar_init(&empty_bar[s], NW);
+    }
     for (int k = 0; k < 2; ++k)
       for (int b = 0; b < 2; ++b) mbar_init(&xbar[k][b], 1);
     fence_mbar_init();
     for (int k = 0; k < 2; ++k)
       for (int b = 0; b < 2; ++b) mbar_arrive_expect_tx(&xbar[k][b], x_bytes);   // rows 0 and 1
   }
+  if (warp == 0) {
+    tmem_alloc(&s_tmem, kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
   cluster_sync_all();   // every CTA's mbarriers exist before anyone pushes to them
+  tc_fence_after();
+  // this warp's columns in its lane quarter
+  const uint32_t t_hold = s_tmem + ((uint32_t)((warp & 3) * 32) << 16) + (uint32_t)(warp >> 2) * 16u * KV;
   const int N = a.hdr->n_pairs;
   const float invN = N > 0 ? 1.0f / (float)N : 0.f;
   const float eps = a.eps;
-
-  // producer state (thread 0): next item to consider, copies issued
-  int issue_w = cid, issued = 0;
-  uint32_t pending = 0;     // stages with a copy in flight that thread 0 has not seen land
+  const float2 kL2 = make_float2(kLog2e, kLog2e);
   bool failed = false;
-  const uint64_t pol = policy_evict_first();
-  auto issue_next = [&]() {
-    while (issue_w < a.R_S) {
-      const int w = issue_w;
-      issue_w += ncl;
-      const int p = a.row_pair[w];
-      if (p < 0) continue;
-      const int s = issued % S;
-      ++issued;
-      uint4 *dst = stage_base + (size_t)s * 2 * a.chunk_vecs;
-      mbar_arrive_expect_tx(&full_bar[s], tx_bytes);
-      pending |= 1u << s;
-      if (vcnt > 0) {
-        const int t = a.teacher_rows[p];
-        const uint16_t *src_t = a.teacher + (int64_t)t * a.ld + (int64_t)vbeg * 8;
-        const uint16_t *src_s = a.student + (int64_t)w * a.ld + (int64_t)vbeg * 8;
-        bulk_load(dst, src_t, (uint32_t)vcnt * 16u, &full_bar[s], pol);
-        bulk_load(dst + a.chunk_vecs, src_s, (uint32_t)vcnt * 16u, &full_bar[s], pol);
-      }
-      return;
-    }
-  };
-  if (tid == 0)
-    for (int s = 0; s < S; ++s) issue_next();
-
-  // wait for phase `parity` of mbarrier m; a wait that gives up marks the CTA failed
+  // wait for phase `parity` of mbarrier m; a wait that gives up marks the thread failed
   auto xwait = [&](uint64_t *m, uint32_t parity) {
     if (!failed && !mbar_wait_sleep(m, parity)) {
       failed = true;
@@ -543,179 +590,274 @@ __global__ void __launch_bounds__(T, 512 / T) ce_kernel(CeArgs a) {
     }
   };
 
-  int consumed = 0;
-  int p_next = cid < a.R_S ? a.row_pair[cid] : -1;
-  for (int w = cid; w < a.R_S; w += ncl) {
-    const int p = p_next;
-    if (w + ncl < a.R_S) p_next = a.row_pair[w + ncl];
-    uint16_t *grow = a.grad ? a.grad + (int64_t)w * a.ld : nullptr;
-    if (p < 0) {   // a student row in no pair: zero gradient
-      if (grow) {
-        float z[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-        for (int vi = tid; vi < vcnt; vi += T) store8(grow, (int64_t)(vbeg + vi) * 8, a.V, z);
+  if (warp == NW) {
+    // ---- the copies ----
+    if (lane == 0) {
+      const uint64_t pol = policy_evict_first();
+      int issued = 0;
+      int w = cid, t = cid < a.R_S ? a.row_teacher[cid] : -1;
+      while (w < a.R_S && !failed) {
+        const int cw = w, ct = t;
+        w += ncl;
+        t = w < a.R_S ? a.row_teacher[w] : -1;   // the next row's teacher, loaded ahead
+        if (ct < 0) continue;                     // a student row in no pair
+        const int s = issued % S;
+        if (issued >= S) xwait(&empty_bar[s], (uint32_t)(issued / S - 1) & 1u);
+        if (failed) break;
+        mbar_arrive_expect_tx(&full_bar[s], tx_bytes);
+        if (vcnt > 0) {
+          uint4 *dst = stage_base + (size_t)s * 2 * a.chunk_vecs;
+          bulk_load(dst, a.teacher + (int64_t)ct * a.ld + (int64_t)vbeg * 8, (uint32_t)vcnt * 16u, &full_bar[s], pol);
+          bulk_load(dst + a.chunk_vecs, a.student + (int64_t)cw * a.ld + (int64_t)vbeg * 8, (uint32_t)vcnt * 16u,
+                    &full_bar[s], pol);
+        }
+        ++issued;
       }
-      continue;
+      // every copy has landed before the CTA's shared memory goes away (bounded)
+      for (int s = 0; s < S && s < issued; ++s) {
+        const int last = ((issued - 1 - s) / S) * S + s;   // the last copy issued to stage s
+        mbar_wait_for(&full_bar[s], (uint32_t)(last / S) & 1u, kWaitLimitNs);
+      }
     }
-    const int c = consumed++;
-    const int s = c % S;
-    const int xb = c & 1;
-    const uint32_t xpar = (uint32_t)(c >> 1) & 1u;
-    xwait(&full_bar[s], (uint32_t)(c / S) & 1u);
-    if (tid == 0 && !failed) pending &= ~(1u << s);
-    const uint4 *st = stage_base + (size_t)s * 2 * a.chunk_vecs;
+  } else {
+    // ---- the compute warps ----
+    int prev_c = -1, prev_p = -1;
+    uint16_t *prev_grow = nullptr;
 
-    // ---- pass 1: logits into registers, this thread's max, then exp(x - max) and its sum ----
-    float xt[KV * 8], xs[KV * 8];
-    float mt = -INFINITY, ms = -INFINITY;
+    // loss sums of row prev_c, then its gradient -(1/N) (a_v - P^S(v) A) = P^S(v) (A/N) - a_v/N
+    auto finish_prev = [&]() {
+      const int xb = prev_c & 1;
+      xwait(&xbar[1][xb], (uint32_t)(prev_c >> 1) & 1u);
+      if (tid == 0 && !failed) mbar_arrive_expect_tx(&xbar[1][xb], x_bytes);   // row prev_c + 2
+      const int nx = C * NW;
+      float2 LA = make_float2(0.f, 0.f);
 #pragma unroll
-    for (int k = 0; k < KV; ++k) {
-      const int vi = tid + k * T;
-      if (vi < vcnt) {
-        unpack8(st[vi], xt + 8 * k);
-        unpack8(st[a.chunk_vecs + vi], xs + 8 * k);
-        const int e0 = (vbeg + vi) * 8;
-        if (e0 + 8 > a.V) {
+      for (int i = 0; i < NPX; ++i)
+        if (32 * i < nx) {
+          const int j = lane + 32 * i;
+          if (j < nx) LA = __fadd2_rn(LA, *reinterpret_cast<const float2 *>(&xbuf[1][xb][j]));
+        }
+      LA = warp_sum2(LA);   // (-sum P^T log2(P^S + eps), -A), both / N
+      if (rank == 0 && tid == 0) a.pair_loss[prev_p] = LA.x * kLn2 * (float)N;
+      if (prev_grow) {
+        const float2 A2 = make_float2(-LA.y, -LA.y);
+        tmem_wait_st();
 #pragma unroll
-          for (int j = 0; j < 8; ++j)
-            if (e0 + j >= a.V) {
-              xt[8 * k + j] = -INFINITY;
-              xs[8 * k + j] = -INFINITY;
+        for (int k = 0; k < KV; ++k) {
+          const int vi = tid + k * T;
+          uint32_t hold[16];
+          tmem_ld_x16(t_hold + 16u * k, hold);   // P^S (8 values), then -a_v / N (8 values)
+          if (vi < vcnt) {
+            uint32_t g[4];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+              const float2 pS = make_float2(__uint_as_float(hold[2 * j]), __uint_as_float(hold[2 * j + 1]));
+              const float2 nav = make_float2(__uint_as_float(hold[8 + 2 * j]), __uint_as_float(hold[9 + 2 * j]));
+              const float2 gr = __ffma2_rn(pS, A2, nav);
+              g[j] = pack_bf16x2(gr.x, gr.y);
             }
+            const int64_t e0 = (int64_t)(vbeg + vi) * 8;
+            if (vi < vfull) {
+              *reinterpret_cast<uint4 *>(prev_grow + e0) = make_uint4(g[0], g[1], g[2], g[3]);
+            } else {   // the vector cut by V: only the elements below V
+#pragma unroll
+              for (int j = 0; j < 8; ++j)
+                if (e0 + j < a.V) prev_grow[e0 + j] = (uint16_t)((j & 1) ? (g[j / 2] >> 16) : (g[j / 2] & 0xffffu));
+            }
+          }
         }
-      } else {
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          xt[8 * k + j] = -INFINITY;
-          xs[8 * k + j] = -INFINITY;
+      }
+    };
+
+    int consumed = 0;
+    int p_next = cid < a.R_S ? a.row_pair[cid] : -1;
+    for (int w = cid; w < a.R_S; w += ncl) {
+      const int p = p_next;
+      if (w + ncl < a.R_S) p_next = a.row_pair[w + ncl];
+      uint16_t *grow = a.grad ? a.grad + (int64_t)w * a.ld : nullptr;
+      if (p < 0) {   // a student row in no pair: zero gradient
+        if (grow) {
+          float z[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+          for (int vi = tid; vi < vcnt; vi += T) store8(grow, (int64_t)(vbeg + vi) * 8, a.V, z);
         }
+        continue;
       }
-#pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        mt = fmaxf(mt, xt[8 * k + j]);
-        ms = fmaxf(ms, xs[8 * k + j]);
-      }
-    }
-    const float bt = (mt == -INFINITY) ? 0.f : -mt * kLog2e;
-    const float bs = (ms == -INFINITY) ? 0.f : -ms * kLog2e;
-    float zt = 0.f, zs = 0.f;
-#pragma unroll
-    for (int i = 0; i < KV * 8; ++i) {
-      xt[i] = ex2_approx(fmaf(xt[i], kLog2e, bt));   // -inf -> 0
-      xs[i] = ex2_approx(fmaf(xs[i], kLog2e, bs));
-      zt += xt[i];
-      zs += xs[i];
-    }
-    // ---- softmax statistics of the whole row ----
-    {
-      float m1 = mt, z1 = zt, m2 = ms, z2 = zs;
-      warp_lse(m1, z1);
-      warp_lse(m2, z2);
-      if (lane < C)
-        st_async_f4(peer_addr(&xbuf[0][xb][rank * NW + warp], (uint32_t)lane), make_float4(m1, z1, m2, z2),
-                    peer_addr(&xbar[0][xb], (uint32_t)lane));
-    }
-    xwait(&xbar[0][xb], xpar);
-    if (tid == 0) {
-      if (!failed) mbar_arrive_expect_tx(&xbar[0][xb], x_bytes);   // row c + 2
-      if (!failed) issue_next();                                     // every warp is past stage s
-    }
-    // the row's max over the C x NW partials, then one rescale per partial
-    float Mt = -INFINITY, Ms = -INFINITY;
-    for (int j = lane; j < C * NW; j += 32) {
-      const float4 v = xbuf[0][xb][j];
-      Mt = fmaxf(Mt, v.x);
-      Ms = fmaxf(Ms, v.z);
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      Mt = fmaxf(Mt, __shfl_xor_sync(0xffffffffu, Mt, o));
-      Ms = fmaxf(Ms, __shfl_xor_sync(0xffffffffu, Ms, o));
-    }
-    const float nMt = (Mt == -INFINITY) ? 0.f : -Mt * kLog2e, nMs = (Ms == -INFINITY) ? 0.f : -Ms * kLog2e;
-    float Zt = 0.f, Zs = 0.f;
-    for (int j = lane; j < C * NW; j += 32) {
-      const float4 v = xbuf[0][xb][j];
-      Zt = fmaf(v.y, ex2_approx(fmaf(v.x, kLog2e, nMt)), Zt);   // empty partials: z = 0
-      Zs = fmaf(v.w, ex2_approx(fmaf(v.z, kLog2e, nMs)), Zs);
-    }
-    Zt = warp_sum(Zt);
-    Zs = warp_sum(Zs);
-    // P(v) = exp(x - m_thread) * exp(m_thread - M) / Z
-    // (P^T carries the 1/N of the loss from here on: the loss terms, a and A
-    // come out divided by N, and the gradient is one FMA per element)
-    const float ct = (mt == -INFINITY) ? 0.f : ex2_approx(fmaf(mt, kLog2e, nMt)) * rcp_approx(Zt) * invN;
-    const float cs = (ms == -INFINITY) ? 0.f : ex2_approx(fmaf(ms, kLog2e, nMs)) * rcp_approx(Zs);
+      const int c = consumed++;
+      const int s = c % S;
+      const int xb = c & 1;
+      const uint32_t xpar = (uint32_t)(c >> 1) & 1u;
 
-    // ---- pass 2: P^T / N, P^S, the loss terms and a / N ----
-    float lsum = 0.f, asum = 0.f;
-    if (eps > 0.f) {
-#pragma unroll
-      for (int i = 0; i < KV * 8; ++i) {
-        const float pt = xt[i] * ct, ps = xs[i] * cs;
-        const float q = ps + eps;
-        lsum = fmaf(pt, lg2_approx(q), lsum);
-        const float av = pt * (ps * rcp_approx(q));
-        asum += av;
-        xt[i] = av;
-        xs[i] = ps;
-      }
-    } else {
-#pragma unroll
-      for (int i = 0; i < KV * 8; ++i) {
-        const float pt = xt[i] * ct, ps = xs[i] * cs;
-        const float q = fmaxf(ps, 1.17549435e-38f);   // log2 stays finite when eps = 0
-        lsum = fmaf(pt, lg2_approx(q), lsum);
-        const float av = pt * (ps * rcp_approx(q));
-        asum += av;
-        xt[i] = av;
-        xs[i] = ps;
-      }
-    }
-    lsum = warp_sum(lsum);
-    asum = warp_sum(asum);
-    if (lane < C)
-      st_async_f4(peer_addr(&xbuf[1][xb][rank * NW + warp], (uint32_t)lane), make_float4(lsum, asum, 0.f, 0.f),
-                  peer_addr(&xbar[1][xb], (uint32_t)lane));
-    xwait(&xbar[1][xb], xpar);
-    if (tid == 0 && !failed) mbar_arrive_expect_tx(&xbar[1][xb], x_bytes);   // row c + 2
-    float Lp = 0.f, A = 0.f;
-    for (int j = lane; j < C * NW; j += 32) {
-      const float4 v = xbuf[1][xb][j];
-      Lp += v.x;
-      A += v.y;
-    }
-    Lp = warp_sum(Lp);
-    A = warp_sum(A);
-    if (rank == 0 && tid == 0) a.pair_loss[p] = -Lp * kLn2 * (float)N;   // Lp is the sum / N
-
-    // ---- pass 3: gradient -(1/N) (a_v - P^S(v) A) = P^S(v) (A/N) - a_v/N ----
-    if (grow) {
+      // ---- pass 1: the logits as bf16 pairs, this thread's max over the
+      // packed pairs, then exp(x - max) and its sum, two elements per instruction ----
+      xwait(&full_bar[s], (uint32_t)(c / S) & 1u);
+      const uint4 *st = stage_base + (size_t)s * 2 * a.chunk_vecs;
+      uint32_t wt[NP], ws[NP];
 #pragma unroll
       for (int k = 0; k < KV; ++k) {
         const int vi = tid + k * T;
+        uint4 ut = make_uint4(kNegInfBf16x2, kNegInfBf16x2, kNegInfBf16x2, kNegInfBf16x2), us = ut;
         if (vi < vcnt) {
-          float gr[8];
+          ut = st[vi];
+          us = st[a.chunk_vecs + vi];
+        }
+        wt[4 * k] = ut.x, wt[4 * k + 1] = ut.y, wt[4 * k + 2] = ut.z, wt[4 * k + 3] = ut.w;
+        ws[4 * k] = us.x, ws[4 * k + 1] = us.y, ws[4 * k + 2] = us.z, ws[4 * k + 3] = us.w;
+        const int e0 = (vbeg + vi) * 8;
+        if (vi < vcnt && e0 + 8 > a.V) {   // the row's last vector: elements past V become -inf
 #pragma unroll
-          for (int j = 0; j < 8; ++j) gr[j] = fmaf(xs[8 * k + j], A, -xt[8 * k + j]);   // A and a already / N
-          store8(grow, (int64_t)(vbeg + vi) * 8, a.V, gr);
+          for (int j = 0; j < 8; ++j)
+            if (e0 + j >= a.V) {
+              const uint32_t keep = (j & 1) ? 0x0000ffffu : 0xffff0000u;
+              wt[4 * k + j / 2] = (wt[4 * k + j / 2] & keep) | (kNegInfBf16x2 & ~keep);
+              ws[4 * k + j / 2] = (ws[4 * k + j / 2] & keep) | (kNegInfBf16x2 & ~keep);
+            }
         }
       }
+      float mt, ms;
+      {
+        uint32_t m2t = wt[0], m2s = ws[0];
+#pragma unroll
+        for (int i = 1; i < NP; ++i) {
+          m2t = max_bf16x2(m2t, wt[i]);
+          m2s = max_bf16x2(m2s, ws[i]);
+        }
+        const float2 ft = bf16x2_to_float2(m2t), fs = bf16x2_to_float2(m2s);
+        mt = fmaxf(ft.x, ft.y);
+        ms = fmaxf(fs.x, fs.y);
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty_bar[s]);   // this warp is done with the stage
+      const float bt = (mt == -INFINITY) ? 0.f : -mt * kLog2e;
+      const float bs = (ms == -INFINITY) ? 0.f : -ms * kLog2e;
+      const float2 bt2 = make_float2(bt, bt), bs2 = make_float2(bs, bs);
+      float2 zt0 = make_float2(0.f, 0.f), zt1 = zt0, zs0 = zt0, zs1 = zt0;
+      float2 et[NP], es[NP];
+#pragma unroll
+      for (int i = 0; i < NP; ++i) {
+        const float2 at = __ffma2_rn(bf16x2_to_float2(wt[i]), kL2, bt2);   // -inf -> exp 0
+        const float2 as = __ffma2_rn(bf16x2_to_float2(ws[i]), kL2, bs2);
+        et[i] = make_float2(ex2_approx(at.x), ex2_approx(at.y));
+        es[i] = make_float2(ex2_approx(as.x), ex2_approx(as.y));
+        if (i & 1) {
+          zt1 = __fadd2_rn(zt1, et[i]);
+          zs1 = __fadd2_rn(zs1, es[i]);
+        } else {
+          zt0 = __fadd2_rn(zt0, et[i]);
+          zs0 = __fadd2_rn(zs0, es[i]);
+        }
+      }
+      // ---- softmax statistics of this thread's warp, to every CTA of the cluster ----
+      {
+        const float2 zt2 = __fadd2_rn(zt0, zt1), zs2 = __fadd2_rn(zs0, zs1);
+        const float Mwt = redux_max_f32(mt), Mws = redux_max_f32(ms);
+        float2 z = make_float2((mt == -INFINITY) ? 0.f : (zt2.x + zt2.y) * ex2_approx((mt - Mwt) * kLog2e),
+                               (ms == -INFINITY) ? 0.f : (zs2.x + zs2.y) * ex2_approx((ms - Mws) * kLog2e));
+        z = warp_sum2(z);
+        if (lane < C)
+          st_async_f4(peer_addr(&xbuf[0][xb][rank * NW + warp], (uint32_t)lane), make_float4(Mwt, Mws, z.x, z.y),
+                      peer_addr(&xbar[0][xb], (uint32_t)lane));
+      }
+
+      // ---- the previous row, while this row's statistics travel ----
+      if (prev_c >= 0) finish_prev();
+
+      // ---- the row's max over the C x NW partials, then one rescale per partial ----
+      xwait(&xbar[0][xb], xpar);
+      if (tid == 0 && !failed) mbar_arrive_expect_tx(&xbar[0][xb], x_bytes);   // row c + 2
+      const int nx = C * NW;
+      float Mt = -INFINITY, Ms = -INFINITY;
+#pragma unroll
+      for (int i = 0; i < NPX; ++i)
+        if (32 * i < nx) {
+          const int j = lane + 32 * i;
+          if (j < nx) {
+            const float2 m = *reinterpret_cast<const float2 *>(&xbuf[0][xb][j]);
+            Mt = fmaxf(Mt, m.x);
+            Ms = fmaxf(Ms, m.y);
+          }
+        }
+      Mt = redux_max_f32(Mt);
+      Ms = redux_max_f32(Ms);
+      const float nMt = (Mt == -INFINITY) ? 0.f : -Mt * kLog2e, nMs = (Ms == -INFINITY) ? 0.f : -Ms * kLog2e;
+      const float2 nM2 = make_float2(nMt, nMs);
+      float2 Z = make_float2(0.f, 0.f);
+#pragma unroll
+      for (int i = 0; i < NPX; ++i)
+        if (32 * i < nx) {
+          const int j = lane + 32 * i;
+          if (j < nx) {
+            const float4 v = xbuf[0][xb][j];
+            const float2 x = __ffma2_rn(make_float2(v.x, v.y), kL2, nM2);   // empty partials: z = 0
+            Z = __ffma2_rn(make_float2(v.z, v.w), make_float2(ex2_approx(x.x), ex2_approx(x.y)), Z);
+          }
+        }
+      Z = warp_sum2(Z);
+      // P(v) = exp(x - m_thread) * exp(m_thread - M) / Z.  The teacher's
+      // factor carries -1/N: the loss terms, a and A come out as -(.)/N and
+      // the gradient P^S(v) (A/N) - a_v/N is one FMA per element.
+      const float nct = (mt == -INFINITY) ? 0.f : -ex2_approx(fmaf(mt, kLog2e, nMt)) * rcp_approx(Z.x) * invN;
+      const float cs = (ms == -INFINITY) ? 0.f : ex2_approx(fmaf(ms, kLog2e, nMs)) * rcp_approx(Z.y);
+      const float2 nct2 = make_float2(nct, nct), cs2 = make_float2(cs, cs);
+
+      // ---- pass 2: -P^T / N, P^S, -(loss terms) / N and -a / N; P^S and -a / N to tensor memory ----
+      float2 l0 = make_float2(0.f, 0.f), l1 = l0, s0 = l0, s1 = l0;
+      auto pass2 = [&](auto clamp) {
+        const float2 eps2 = make_float2(eps, eps);
+        uint32_t hold[16];
+#pragma unroll
+        for (int i = 0; i < NP; ++i) {
+          const float2 pt = __fmul2_rn(et[i], nct2);
+          const float2 pS = __fmul2_rn(es[i], cs2);
+          float2 q = __fadd2_rn(pS, eps2);
+          if constexpr (decltype(clamp)::value)   // eps = 0: log2 stays finite
+            q = make_float2(fmaxf(q.x, 1.17549435e-38f), fmaxf(q.y, 1.17549435e-38f));
+          const float2 lg = make_float2(lg2_approx(q.x), lg2_approx(q.y));
+          const float2 rq = make_float2(ex2_approx(-lg.x), ex2_approx(-lg.y));   // 1 / q
+          const float2 av = __fmul2_rn(pt, __fmul2_rn(pS, rq));
+          if (i & 1) {
+            l1 = __ffma2_rn(pt, lg, l1);
+            s1 = __fadd2_rn(s1, av);
+          } else {
+            l0 = __ffma2_rn(pt, lg, l0);
+            s0 = __fadd2_rn(s0, av);
+          }
+          const int j = i & 3;
+          hold[2 * j] = __float_as_uint(pS.x);
+          hold[2 * j + 1] = __float_as_uint(pS.y);
+          hold[8 + 2 * j] = __float_as_uint(av.x);
+          hold[9 + 2 * j] = __float_as_uint(av.y);
+          if (j == 3) tmem_st_x16(t_hold + 16u * (i / 4), hold);
+        }
+      };
+      if (eps > 0.f)
+        pass2(std::false_type{});
+      else
+        pass2(std::true_type{});
+      {
+        const float2 l2 = __fadd2_rn(l0, l1), s2 = __fadd2_rn(s0, s1);
+        const float2 r = warp_sum2(make_float2(l2.x + l2.y, s2.x + s2.y));
+        if (lane < C)
+          st_async_f4(peer_addr(&xbuf[1][xb][rank * NW + warp], (uint32_t)lane), make_float4(r.x, r.y, 0.f, 0.f),
+                      peer_addr(&xbar[1][xb], (uint32_t)lane));
+      }
+      prev_c = c;
+      prev_p = p;
+      prev_grow = grow;
     }
+    if (prev_c >= 0) finish_prev();
+    tmem_wait_st();   // the last row's stores, when no gradient read them back
   }
 
   // no CTA leaves while a peer may still push to or read its shared memory
+  tc_fence_before();
   cluster_sync_all();
-
-  // a copy whose wait gave up may still be in flight: wait for it, bounded
-  if (tid == 0 && failed) {
-    for (int s = 0; s < S; ++s)
-      if (pending & (1u << s)) {
-        const int last = ((issued - 1 - s) / S) * S + s;   // the last copy issued to stage s
-        if (last >= 0) mbar_wait_for(&full_bar[s], (uint32_t)(last / S) & 1u, kWaitLimitNs);
-      }
+  if (warp == 0) {
+    tc_fence_after();
+    tmem_dealloc(s_tmem, kTmemCols);
   }
 
   // ---- the loss: the last CTA sums the per-pair losses in pair order ----
+  constexpr int NT = T + 32;
   __shared__ int s_last;
   __syncthreads();
   if (tid == 0) {
@@ -725,8 +867,8 @@ __global__ void __launch_bounds__(T, 512 / T) ce_kernel(CeArgs a) {
   __syncthreads();
   if (!s_last) return;
   __threadfence();
-  __shared__ double dpart[NW];
-  const int per = (N + T - 1) / T;
+  __shared__ double dpart[NW + 1];
+  const int per = (N + NT - 1) / NT;
   double acc = 0.0;
   for (int i = 0; i < per; ++i) {
     const int q = tid * per + i;
@@ -738,7 +880,7 @@ __global__ void __launch_bounds__(T, 512 / T) ce_kernel(CeArgs a) {
   __syncthreads();
   if (tid == 0) {
     double t = 0.0;
-    for (int w2 = 0; w2 < NW; ++w2) t += dpart[w2];
+    for (int w2 = 0; w2 <= NW; ++w2) t += dpart[w2];
     a.loss[0] = N > 0 ? (float)(t / (double)N) : 0.f;
   }
 }
@@ -748,9 +890,8 @@ using CeKernel = void (*)(CeArgs);
 CeKernel ce_kernel_for(int kv, int T) {
   static const CeKernel k256[kCeMaxVecs] = {ce_kernel<1, 256>, ce_kernel<2, 256>, ce_kernel<3, 256>,
                                             ce_kernel<4, 256>, ce_kernel<5, 256>};
-  static const CeKernel k512[kCeMaxVecs] = {ce_kernel<1, 512>, ce_kernel<2, 512>, ce_kernel<3, 512>,
-                                            ce_kernel<4, 512>, ce_kernel<5, 512>};
-  return (T == 256 ? k256 : k512)[kv - 1];
+  static const CeKernel k448[4] = {ce_kernel<1, 448>, ce_kernel<2, 448>, ce_kernel<3, 448>, ce_kernel<4, 448>};
+  return T == 256 ? k256[kv - 1] : k448[kv - 1];
 }
 
 // 16-byte vectors per thread per row with T threads per CTA and C CTAs per row
@@ -775,7 +916,7 @@ int ce_resident_clusters(int kv, int T, int C, size_t smem, int num_sms) {
     size_t smem;
     int n;
   };
-  static Entry cache[32];
+  static Entry cache[64];
   static int n_cache = 0;
   static std::mutex mu;
   int dev = 0;
@@ -790,8 +931,8 @@ int ce_resident_clusters(int kv, int T, int C, size_t smem, int num_sms) {
   cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kCeSmemLimit);
   if (C > 8) cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((unsigned)(C * std::max(1, 2 * num_sms / C)));
-  cfg.blockDim = dim3((unsigned)T);
+  cfg.gridDim = dim3((unsigned)(C * std::max(1, num_sms / C)));
+  cfg.blockDim = dim3((unsigned)(T + 32));
   cfg.dynamicSmemBytes = smem;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -805,7 +946,7 @@ int ce_resident_clusters(int kv, int T, int C, size_t smem, int num_sms) {
     cudaGetLastError();
     n = 0;
   }
-  if (n_cache < 32) cache[n_cache++] = Entry{dev, kv, T, C, smem, n};
+  if (n_cache < 64) cache[n_cache++] = Entry{dev, kv, T, C, smem, n};
   return n;
 }
 
@@ -818,40 +959,47 @@ bool ce_try_layout(int64_t V, int T, int C, int num_sms, CeLayout &L) {
   L.kv = kv;
   L.chunk_vecs = (nvec + C - 1) / C;
   const size_t stage_bytes = (size_t)2 * L.chunk_vecs * 16;
-  // 256-thread CTAs run two to an SM: each keeps to half of the shared memory
-  const size_t limit = T == 256 ? kCeSmemLimit / 2 : kCeSmemLimit;
-  L.stages = (int)std::min<size_t>(kCeMaxStages, limit / stage_bytes);
+  L.stages = (int)std::min<size_t>(kCeMaxStages, kCeSmemLimit / stage_bytes);
   if (L.stages < 2) return false;
   L.smem = stage_bytes * L.stages;
   L.resident = ce_resident_clusters(kv, T, C, L.smem, num_sms);
   return L.resident > 0;
 }
 
-// Two candidates: 256-thread CTAs (two per SM, one computing while the other
-// waits for its exchange) and 512-thread CTAs, each with the fewest CTAs per
-// row that keep a thread at <= 4 vectors per row (5 at the largest cluster);
-// the one with more threads resident wins -- cluster placement within a GPC
-// can leave SMs idle (on a GB300 at the Llama-3 vocabulary: 14 clusters of
-// 16 x 256 threads on 112 SMs, 15 clusters of 8 x 512 on 120).
+// Candidates: 256 and 448 compute threads per CTA (one CTA per SM), each
+// with the three smallest cluster sizes whose threads hold at most 4 vectors
+// of a row (5 at 256 threads and the largest cluster).  The score is the SMs
+// the resident clusters occupy times the share of the threads' vector slots
+// that hold data: cluster placement within a GPC can leave SMs idle (on a
+// GB300 at the Llama-3 vocabulary, 15 clusters of 9 x 448 threads occupy
+// 135 SMs, 7 clusters of 16 x 256 threads 112).
 bool ce_layout(int64_t V, int num_sms, CeLayout &L) {
-  // per thread count, the fewest CTAs per row with <= 4 vectors per thread (5 at the largest cluster)
+  const int64_t nvec = (V + 7) / 8;
   CeLayout best{};
-  bool found = false;
-  for (const int T : {256, 512}) {
-    const int Cmax = T == 256 ? kCeMaxCluster : 8;
-    for (int C = 1; C <= Cmax; C *= 2) {
-      if (ce_vecs(V, T, C) > 4 && C < Cmax) continue;
+  double best_score = -1.0;
+  for (const int T : {256, 448}) {
+    const int Cmax = kCeMaxCluster;
+    const int kv_max = T == 256 ? kCeMaxVecs : 4;
+    int tried = 0;
+    for (int C = 1; C <= Cmax && tried < 3; ++C) {   // the three smallest admissible cluster sizes
+      const int kv = ce_vecs(V, T, C);
+      if (kv > 4 && !(C == Cmax && kv <= kv_max)) continue;
+      ++tried;
       CeLayout cand;
-      if (ce_try_layout(V, T, C, num_sms, cand)) {
-        // more resident threads wins (a cluster size that leaves SMs of a GPC idle loses)
-        if (!found || (int64_t)cand.resident * cand.C * cand.T > (int64_t)best.resident * best.C * best.T) best = cand;
-        found = true;
+      if (!ce_try_layout(V, T, C, num_sms, cand)) continue;
+      const double sms_used = (double)cand.resident * C;
+      const double fill = (double)nvec / ((double)C * T * kv);
+      const double score = sms_used * fill;
+      if (score > best_score * 1.001) {   // ties: the smaller cluster, found first
+        best = cand;
+        best_score = score;
       }
-      break;
+      if (kv == 1) break;   // more CTAs per row only adds empty slots
     }
   }
-  if (found) L = best;
-  return found;
+  if (best_score < 0) return false;
+  L = best;
+  return true;
 }
 
 }  // namespace
@@ -906,6 +1054,8 @@ umim_status distill_soft_ce(const void *teacher, int32_t R_T, const void *studen
   p += a256(sizeof(CeHeader));
   int32_t *row_pair = reinterpret_cast<int32_t *>(p);
   p += a256(sizeof(int32_t) * (size_t)std::max(R_S, 1));
+  int32_t *row_teacher = reinterpret_cast<int32_t *>(p);
+  p += a256(sizeof(int32_t) * (size_t)std::max(R_S, 1));
   float *ws_pair_loss = reinterpret_cast<float *>(p);
 
   CeArgs a;
@@ -924,6 +1074,7 @@ umim_status distill_soft_ce(const void *teacher, int32_t R_T, const void *studen
   a.pair_loss = pair_loss ? pair_loss : ws_pair_loss;
   a.grad = static_cast<uint16_t *>(grad);
   a.row_pair = row_pair;
+  a.row_teacher = row_teacher;
   a.hdr = hdr;
   a.status = dev_status ? dev_status : &hdr->status;
   a.chunk_vecs = lay.chunk_vecs;
@@ -931,6 +1082,8 @@ umim_status distill_soft_ce(const void *teacher, int32_t R_T, const void *studen
 
   if (cudaMemsetAsync(hdr, 0, sizeof(CeHeader), stream) != cudaSuccess) return UMIM_ERR_CUDA;
   if (R_S > 0 && cudaMemsetAsync(row_pair, 0xFF, sizeof(int32_t) * (size_t)R_S, stream) != cudaSuccess)
+    return UMIM_ERR_CUDA;
+  if (R_S > 0 && cudaMemsetAsync(row_teacher, 0xFF, sizeof(int32_t) * (size_t)R_S, stream) != cudaSuccess)
     return UMIM_ERR_CUDA;
   const int prep_blocks = std::max(1, std::min((max_pairs + 255) / 256, num_sms * 4));
   trace_mark(stream, "distill.ce_prep");
@@ -940,7 +1093,7 @@ umim_status distill_soft_ce(const void *teacher, int32_t R_T, const void *studen
   const int n_cl = std::max(1, std::min(R_S, lay.resident));
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)(n_cl * lay.C));
-  cfg.blockDim = dim3((unsigned)lay.T);
+  cfg.blockDim = dim3((unsigned)(lay.T + 32));
   cfg.dynamicSmemBytes = lay.smem;
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];
