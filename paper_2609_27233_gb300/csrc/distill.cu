@@ -300,6 +300,7 @@ struct CeArgs {
   CeHeader *hdr;
   int32_t *status;
   int32_t chunk_vecs;                  // 16-byte vectors of a row per CTA
+  int32_t stage_vecs;                  // vectors per row in a stage: chunk_vecs, padded with -inf to KV x T
   int32_t stages;
 };
 
@@ -526,12 +527,11 @@ __device__ __forceinline__ void st_async_f4(uint32_t raddr, float4 v, uint32_t r
 // (pass 1 -> 2), then in tensor memory (which this kernel has no other use
 // for) as fp32 P^S and -a_v / N (pass 2 -> gradient): each warp owns 16 x KV
 // columns of its lane quarter, 16 per vector.
-template <int KV, int T>
+template <int KV, int T, bool TAIL>   // TAIL: V is not a multiple of 8 (a vector is cut by V)
 __global__ void __launch_bounds__(T + 32, 1) ce_kernel(CeArgs a) {
   constexpr int NW = T / 32;               // compute warps; warp NW issues the copies
   constexpr int NX = kCeMaxCluster * NW;   // partial slots per buffer
   constexpr int NP = 4 * KV;               // element pairs (one 32-bit word of each row) per thread
-  constexpr int NPX = (NX + 31) / 32;      // partials per lane, at most
   // tensor-memory columns: 16 per vector for each warp of a lane quarter
   constexpr uint32_t kTmemNeed = (uint32_t)((NW + 3) / 4) * 16u * KV;
   constexpr uint32_t kTmemCols = kTmemNeed <= 32 ? 32 : kTmemNeed <= 64 ? 64 : kTmemNeed <= 128 ? 128 : 256;
@@ -550,9 +550,10 @@ __global__ void __launch_bounds__(T + 32, 1) ce_kernel(CeArgs a) {
   const int vbeg = (int)rank * a.chunk_vecs;
   const int vcnt = max(0, min(a.chunk_vecs, nvec - vbeg));
   // vectors of the chunk that lie wholly below V; a vector cut by V is stored element-wise
-  const int vfull = max(0, min(vcnt, a.V / 8 - vbeg));
+  const int vfull = TAIL ? max(0, min(vcnt, a.V / 8 - vbeg)) : vcnt;
   const int S = a.stages;
-  uint4 *stage_base = reinterpret_cast<uint4 *>(ce_smem);   // [S][2][chunk_vecs]
+  uint4 *stage_base = reinterpret_cast<uint4 *>(ce_smem);   // [S][2][stage_vecs]
+  const int SV = a.stage_vecs;
   const uint32_t tx_bytes = 2u * (uint32_t)vcnt * 16u;
   const uint32_t x_bytes = (uint32_t)(C * NW * 16);
 
@@ -567,6 +568,13 @@ __global__ void __launch_bounds__(T + 32, 1) ce_kernel(CeArgs a) {
     fence_mbar_init();
     for (int k = 0; k < 2; ++k)
       for (int b = 0; b < 2; ++b) mbar_arrive_expect_tx(&xbar[k][b], x_bytes);   // rows 0 and 1
+  }
+  // vectors [vcnt, stage_vecs) of every stage hold -inf (no copy writes them), so every
+  // thread reads its KV vectors of a row without a bounds check
+  for (int i = tid; i < S * 2 * (SV - vcnt); i += T + 32) {
+    const int h = i / (SV - vcnt);
+    stage_base[(size_t)h * SV + vcnt + i % (SV - vcnt)] =
+        make_uint4(kNegInfBf16x2, kNegInfBf16x2, kNegInfBf16x2, kNegInfBf16x2);
   }
   if (warp == 0) {
     tmem_alloc(&s_tmem, kTmemCols);
@@ -594,24 +602,28 @@ __global__ void __launch_bounds__(T + 32, 1) ce_kernel(CeArgs a) {
     // ---- the copies ----
     if (lane == 0) {
       const uint64_t pol = policy_evict_first();
-      int issued = 0;
+      int issued = 0, s = 0;
+      uint32_t phase = 0;   // of stage s's full barrier for the copy about to be issued
       int w = cid, t = cid < a.R_S ? a.row_teacher[cid] : -1;
       while (w < a.R_S && !failed) {
         const int cw = w, ct = t;
         w += ncl;
         t = w < a.R_S ? a.row_teacher[w] : -1;   // the next row's teacher, loaded ahead
         if (ct < 0) continue;                     // a student row in no pair
-        const int s = issued % S;
-        if (issued >= S) xwait(&empty_bar[s], (uint32_t)(issued / S - 1) & 1u);
+        if (issued >= S) xwait(&empty_bar[s], phase ^ 1u);   // the stage's previous row is consumed
         if (failed) break;
         mbar_arrive_expect_tx(&full_bar[s], tx_bytes);
         if (vcnt > 0) {
-          uint4 *dst = stage_base + (size_t)s * 2 * a.chunk_vecs;
+          uint4 *dst = stage_base + (size_t)s * 2 * SV;
           bulk_load(dst, a.teacher + (int64_t)ct * a.ld + (int64_t)vbeg * 8, (uint32_t)vcnt * 16u, &full_bar[s], pol);
-          bulk_load(dst + a.chunk_vecs, a.student + (int64_t)cw * a.ld + (int64_t)vbeg * 8, (uint32_t)vcnt * 16u,
-                    &full_bar[s], pol);
+          bulk_load(dst + SV, a.student + (int64_t)cw * a.ld + (int64_t)vbeg * 8, (uint32_t)vcnt * 16u, &full_bar[s],
+                    pol);
         }
         ++issued;
+        if (++s == S) {
+          s = 0;
+          phase ^= 1u;
+        }
       }
       // every copy has landed before the CTA's shared memory goes away (bounded)
       for (int s = 0; s < S && s < issued; ++s) {
@@ -622,6 +634,7 @@ __global__ void __launch_bounds__(T + 32, 1) ce_kernel(CeArgs a) {
   } else {
     // ---- the compute warps ----
     int prev_c = -1, prev_p = -1;
+    const int64_t goff = (int64_t)(vbeg + tid) * 8;   // this thread's first gradient element of a row
     uint16_t *prev_grow = nullptr;
 
     // loss sums of row prev_c, then its gradient -(1/N) (a_v - P^S(v) A) = P^S(v) (A/N) - a_v/N
@@ -632,11 +645,11 @@ __global__ void __launch_bounds__(T + 32, 1) ce_kernel(CeArgs a) {
       const int nx = C * NW;
       float2 LA = make_float2(0.f, 0.f);
 #pragma unroll
-      for (int i = 0; i < NPX; ++i)
-        if (32 * i < nx) {
-          const int j = lane + 32 * i;
-          if (j < nx) LA = __fadd2_rn(LA, *reinterpret_cast<const float2 *>(&xbuf[1][xb][j]));
-        }
+      for (int i = 0; i < 4; ++i) {
+        const int j = lane + 32 * i;
+        if (j < nx) LA = __fadd2_rn(LA, *reinterpret_cast<const float2 *>(&xbuf[1][xb][j]));
+      }
+      for (int j = lane + 128; j < nx; j += 32) LA = __fadd2_rn(LA, *reinterpret_cast<const float2 *>(&xbuf[1][xb][j]));
       LA = warp_sum2(LA);   // (-sum P^T log2(P^S + eps), -A), both / N
       if (rank == 0 && tid == 0) a.pair_loss[prev_p] = LA.x * kLn2 * (float)N;
       if (prev_grow) {
@@ -656,8 +669,8 @@ __global__ void __launch_bounds__(T + 32, 1) ce_kernel(CeArgs a) {
               const float2 gr = __ffma2_rn(pS, A2, nav);
               g[j] = pack_bf16x2(gr.x, gr.y);
             }
-            const int64_t e0 = (int64_t)(vbeg + vi) * 8;
-            if (vi < vfull) {
+            const int64_t e0 = goff + (int64_t)k * T * 8;
+            if (!TAIL || vi < vfull) {
               *reinterpret_cast<uint4 *>(prev_grow + e0) = make_uint4(g[0], g[1], g[2], g[3]);
             } else {   // the vector cut by V: only the elements below V
 #pragma unroll
@@ -669,7 +682,8 @@ __global__ void __launch_bounds__(T + 32, 1) ce_kernel(CeArgs a) {
       }
     };
 
-    int consumed = 0;
+    int consumed = 0, stage = 0;
+    uint32_t sphase = 0;   // of the stage's full barrier for the row about to be consumed
     int p_next = cid < a.R_S ? a.row_pair[cid] : -1;
     for (int w = cid; w < a.R_S; w += ncl) {
       const int p = p_next;
@@ -683,27 +697,28 @@ __global__ void __launch_bounds__(T + 32, 1) ce_kernel(CeArgs a) {
         continue;
       }
       const int c = consumed++;
-      const int s = c % S;
+      const int s = stage;
+      const uint32_t fpar = sphase;
+      if (++stage == S) {
+        stage = 0;
+        sphase ^= 1u;
+      }
       const int xb = c & 1;
       const uint32_t xpar = (uint32_t)(c >> 1) & 1u;
 
       // ---- pass 1: the logits as bf16 pairs, this thread's max over the
       // packed pairs, then exp(x - max) and its sum, two elements per instruction ----
-      xwait(&full_bar[s], (uint32_t)(c / S) & 1u);
-      const uint4 *st = stage_base + (size_t)s * 2 * a.chunk_vecs;
+      xwait(&full_bar[s], fpar);
+      const uint4 *st = stage_base + (size_t)s * 2 * SV;
       uint32_t wt[NP], ws[NP];
 #pragma unroll
       for (int k = 0; k < KV; ++k) {
         const int vi = tid + k * T;
-        uint4 ut = make_uint4(kNegInfBf16x2, kNegInfBf16x2, kNegInfBf16x2, kNegInfBf16x2), us = ut;
-        if (vi < vcnt) {
-          ut = st[vi];
-          us = st[a.chunk_vecs + vi];
-        }
+        const uint4 ut = st[vi], us = st[SV + vi];
         wt[4 * k] = ut.x, wt[4 * k + 1] = ut.y, wt[4 * k + 2] = ut.z, wt[4 * k + 3] = ut.w;
         ws[4 * k] = us.x, ws[4 * k + 1] = us.y, ws[4 * k + 2] = us.z, ws[4 * k + 3] = us.w;
         const int e0 = (vbeg + vi) * 8;
-        if (vi < vcnt && e0 + 8 > a.V) {   // the row's last vector: elements past V become -inf
+        if (TAIL && vi < vcnt && e0 + 8 > a.V) {   // the row's last vector: elements past V become -inf
 #pragma unroll
           for (int j = 0; j < 8; ++j)
             if (e0 + j >= a.V) {
@@ -766,31 +781,29 @@ __global__ void __launch_bounds__(T + 32, 1) ce_kernel(CeArgs a) {
       if (tid == 0 && !failed) mbar_arrive_expect_tx(&xbar[0][xb], x_bytes);   // row c + 2
       const int nx = C * NW;
       float Mt = -INFINITY, Ms = -INFINITY;
+      auto max_part = [&](int j) {
+        const float2 m = *reinterpret_cast<const float2 *>(&xbuf[0][xb][j]);
+        Mt = fmaxf(Mt, m.x);
+        Ms = fmaxf(Ms, m.y);
+      };
 #pragma unroll
-      for (int i = 0; i < NPX; ++i)
-        if (32 * i < nx) {
-          const int j = lane + 32 * i;
-          if (j < nx) {
-            const float2 m = *reinterpret_cast<const float2 *>(&xbuf[0][xb][j]);
-            Mt = fmaxf(Mt, m.x);
-            Ms = fmaxf(Ms, m.y);
-          }
-        }
+      for (int i = 0; i < 4; ++i)
+        if (lane + 32 * i < nx) max_part(lane + 32 * i);
+      for (int j = lane + 128; j < nx; j += 32) max_part(j);
       Mt = redux_max_f32(Mt);
       Ms = redux_max_f32(Ms);
       const float nMt = (Mt == -INFINITY) ? 0.f : -Mt * kLog2e, nMs = (Ms == -INFINITY) ? 0.f : -Ms * kLog2e;
       const float2 nM2 = make_float2(nMt, nMs);
       float2 Z = make_float2(0.f, 0.f);
+      auto sum_part = [&](int j) {
+        const float4 v = xbuf[0][xb][j];
+        const float2 x = __ffma2_rn(make_float2(v.x, v.y), kL2, nM2);   // empty partials: z = 0
+        Z = __ffma2_rn(make_float2(v.z, v.w), make_float2(ex2_approx(x.x), ex2_approx(x.y)), Z);
+      };
 #pragma unroll
-      for (int i = 0; i < NPX; ++i)
-        if (32 * i < nx) {
-          const int j = lane + 32 * i;
-          if (j < nx) {
-            const float4 v = xbuf[0][xb][j];
-            const float2 x = __ffma2_rn(make_float2(v.x, v.y), kL2, nM2);   // empty partials: z = 0
-            Z = __ffma2_rn(make_float2(v.z, v.w), make_float2(ex2_approx(x.x), ex2_approx(x.y)), Z);
-          }
-        }
+      for (int i = 0; i < 4; ++i)
+        if (lane + 32 * i < nx) sum_part(lane + 32 * i);
+      for (int j = lane + 128; j < nx; j += 32) sum_part(j);
       Z = warp_sum2(Z);
       // P(v) = exp(x - m_thread) * exp(m_thread - M) / Z.  The teacher's
       // factor carries -1/N: the loss terms, a and A come out as -(.)/N and
@@ -887,11 +900,16 @@ __global__ void __launch_bounds__(T + 32, 1) ce_kernel(CeArgs a) {
 
 using CeKernel = void (*)(CeArgs);
 
-CeKernel ce_kernel_for(int kv, int T) {
-  static const CeKernel k256[kCeMaxVecs] = {ce_kernel<1, 256>, ce_kernel<2, 256>, ce_kernel<3, 256>,
-                                            ce_kernel<4, 256>, ce_kernel<5, 256>};
-  static const CeKernel k448[4] = {ce_kernel<1, 448>, ce_kernel<2, 448>, ce_kernel<3, 448>, ce_kernel<4, 448>};
-  return T == 256 ? k256[kv - 1] : k448[kv - 1];
+CeKernel ce_kernel_for(int kv, int T, bool tail) {
+  static const CeKernel k256[2][kCeMaxVecs] = {
+      {ce_kernel<1, 256, false>, ce_kernel<2, 256, false>, ce_kernel<3, 256, false>, ce_kernel<4, 256, false>,
+       ce_kernel<5, 256, false>},
+      {ce_kernel<1, 256, true>, ce_kernel<2, 256, true>, ce_kernel<3, 256, true>, ce_kernel<4, 256, true>,
+       ce_kernel<5, 256, true>}};
+  static const CeKernel k448[2][4] = {
+      {ce_kernel<1, 448, false>, ce_kernel<2, 448, false>, ce_kernel<3, 448, false>, ce_kernel<4, 448, false>},
+      {ce_kernel<1, 448, true>, ce_kernel<2, 448, true>, ce_kernel<3, 448, true>, ce_kernel<4, 448, true>}};
+  return T == 256 ? k256[tail][kv - 1] : k448[tail][kv - 1];
 }
 
 // 16-byte vectors per thread per row with T threads per CTA and C CTAs per row
@@ -903,16 +921,16 @@ int ce_vecs(int64_t V, int T, int C) {
 
 // How a call runs: T threads per CTA, C CTAs (one cluster) per student row.
 struct CeLayout {
-  int T, C, kv, chunk_vecs, stages;
+  int T, C, kv, chunk_vecs, stage_vecs, stages;
   size_t smem;
   int resident;   // clusters that can be resident at once
 };
 
 // Clusters of a layout that can be resident at once (0: it cannot launch);
 // cached per device and layout.
-int ce_resident_clusters(int kv, int T, int C, size_t smem, int num_sms) {
+int ce_resident_clusters(int kv, int T, int C, size_t smem, int num_sms, bool tail) {
   struct Entry {
-    int dev, kv, T, C;
+    int dev, kv, T, C, tail;
     size_t smem;
     int n;
   };
@@ -924,9 +942,9 @@ int ce_resident_clusters(int kv, int T, int C, size_t smem, int num_sms) {
   std::lock_guard<std::mutex> lock(mu);
   for (int i = 0; i < n_cache; ++i) {
     const Entry &e = cache[i];
-    if (e.dev == dev && e.kv == kv && e.T == T && e.C == C && e.smem == smem) return e.n;
+    if (e.dev == dev && e.kv == kv && e.T == T && e.C == C && e.tail == (int)tail && e.smem == smem) return e.n;
   }
-  const CeKernel fn = ce_kernel_for(kv, T);
+  const CeKernel fn = ce_kernel_for(kv, T, tail);
   // the largest size any call may request, so that no later call finds a smaller limit
   cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kCeSmemLimit);
   if (C > 8) cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
@@ -946,7 +964,7 @@ int ce_resident_clusters(int kv, int T, int C, size_t smem, int num_sms) {
     cudaGetLastError();
     n = 0;
   }
-  if (n_cache < 64) cache[n_cache++] = Entry{dev, kv, T, C, smem, n};
+  if (n_cache < 64) cache[n_cache++] = Entry{dev, kv, T, C, (int)tail, smem, n};
   return n;
 }
 
@@ -958,11 +976,12 @@ bool ce_try_layout(int64_t V, int T, int C, int num_sms, CeLayout &L) {
   L.C = C;
   L.kv = kv;
   L.chunk_vecs = (nvec + C - 1) / C;
-  const size_t stage_bytes = (size_t)2 * L.chunk_vecs * 16;
+  L.stage_vecs = std::max(L.chunk_vecs, kv * T);
+  const size_t stage_bytes = (size_t)2 * L.stage_vecs * 16;
   L.stages = (int)std::min<size_t>(kCeMaxStages, kCeSmemLimit / stage_bytes);
   if (L.stages < 2) return false;
   L.smem = stage_bytes * L.stages;
-  L.resident = ce_resident_clusters(kv, T, C, L.smem, num_sms);
+  L.resident = ce_resident_clusters(kv, T, C, L.smem, num_sms, V % 8 != 0);
   return L.resident > 0;
 }
 
@@ -1078,6 +1097,7 @@ umim_status distill_soft_ce(const void *teacher, int32_t R_T, const void *studen
   a.hdr = hdr;
   a.status = dev_status ? dev_status : &hdr->status;
   a.chunk_vecs = lay.chunk_vecs;
+  a.stage_vecs = lay.stage_vecs;
   a.stages = lay.stages;
 
   if (cudaMemsetAsync(hdr, 0, sizeof(CeHeader), stream) != cudaSuccess) return UMIM_ERR_CUDA;
@@ -1104,7 +1124,7 @@ umim_status distill_soft_ce(const void *teacher, int32_t R_T, const void *studen
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   trace_mark(stream, "distill.soft_ce");
-  const cudaError_t e = cudaLaunchKernelEx(&cfg, ce_kernel_for(lay.kv, lay.T), a);
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, ce_kernel_for(lay.kv, lay.T, V % 8 != 0), a);
   trace_mark(stream, nullptr);
   return e == cudaSuccess ? UMIM_OK : UMIM_ERR_CUDA;
 }
