@@ -15,15 +15,17 @@
 //    respect to the student logits:
 //      L = -(1/N) sum_pairs sum_v P^T(v) log(P^S(v) + eps)
 //      dL/ds_v = -(1/N) (a_v - P^S(v) sum_u a_u),  a_u = P^T(u) P^S(u) / (P^S(u) + eps)
-//    One thread-block cluster of 8 CTAs per student row: each CTA holds one
-//    eighth of the vocabulary of the teacher and student rows in registers
-//    (fp32), so every logit byte is read once and every gradient byte written
-//    once.  Rows arrive by 1-D TMA bulk copies into a ring of shared-memory
-//    stages (the next rows load while the current one is computed); the
+//    One thread-block cluster of C CTAs per student row (9 at the Llama-3
+//    vocabulary): each CTA holds 1/C of the vocabulary of the teacher and
+//    student rows in registers (fp32), so every logit byte is read once and
+//    every gradient byte written once.  Rows arrive by 1-D TMA bulk copies
+//    into a ring of shared-memory stages that a copy warp refills; the
 //    softmax statistics and the two sums are exchanged between the cluster's
-//    CTAs through distributed shared memory.  Student rows that are in no
-//    pair get a zero gradient.  The loss is summed from the per-pair losses,
-//    in pair order, by the last CTA to finish.
+//    CTAs through distributed shared memory, and each warp keeps two rows in
+//    flight (the finished one in tensor memory) so that every exchange is
+//    waited for one compute phase after it was pushed.  Student rows that are
+//    in no pair get a zero gradient.  The loss is summed from the per-pair
+//    losses, in pair order, by the last CTA to finish.
 #include <algorithm>
 #include <cmath>
 #include <cstdio>
