@@ -169,6 +169,7 @@ __global__ void __launch_bounds__(256) rollback_map_kernel(MoveArgs a, PlanArray
 }
 
 constexpr int kSmemSeqs = 1024;   // active sequences whose plan values a CTA keeps in shared memory
+constexpr int kSmemLanes = 1024;  // tile lanes (layer, K|V, head) whose offsets a CTA keeps in shared memory
 
 // Waits until *cnt >= target; false when it gave up (time limit, or another
 // warp gave up: *abort != 0).
@@ -192,6 +193,9 @@ __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs
   const int my_slot0 = lane / CPR;
   __shared__ int s_last;
   __shared__ int s_sq[kSmemSeqs], s_nd[kSmemSeqs], s_ub[kSmemSeqs], s_fp[kSmemSeqs];
+  // per tile lane tl: its offset within a page (layer, K|V and head), and layer * Hkv + head | K|V << 31
+  __shared__ int64_t s_toff[kSmemLanes];
+  __shared__ int32_t s_tlh[kSmemLanes];
   __shared__ float s_w[ROPE ? D / 2 : 1];   // RoPE angular frequencies
 
   if (ROPE)
@@ -218,14 +222,22 @@ __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs
       const int b = arr.active[j];
       s_sq[j] = b;
       s_nd[j] = arr.n_dest[b];
-      s_ub[j] = arr.unit_base[b];
+      s_ub[j] = arr.unit_base[b] / a.n_lanes;   // the sequence's first row
       s_fp[j] = arr.first_page[b];
+    }
+  }
+  const bool lanes_in_smem = a.n_lanes <= kSmemLanes;
+  if (lanes_in_smem) {
+    for (int tl = threadIdx.x; tl < a.n_lanes; tl += blockDim.x) {
+      const int layer = tl / (2 * Hkv), kv = (tl / Hkv) & 1, h = tl % Hkv;
+      s_toff[tl] = layer * layer_stride + (int)(kv * kv_stride32 + h * kHead);
+      s_tlh[tl] = (int32_t)((uint32_t)(layer * Hkv + h) | ((uint32_t)kv << 31));
     }
   }
   __syncthreads();
   auto seq_of = [&](int j) { return seq_in_smem ? s_sq[j] : arr.active[j]; };
   auto nd_of = [&](int j) { return seq_in_smem ? s_nd[j] : arr.n_dest[arr.active[j]]; };
-  auto ub_of = [&](int j) { return seq_in_smem ? s_ub[j] : arr.unit_base[arr.active[j]]; };
+  auto row0_of = [&](int j) { return seq_in_smem ? s_ub[j] : arr.unit_base[arr.active[j]] / a.n_lanes; };
   auto fp_of = [&](int j) { return seq_in_smem ? s_fp[j] : arr.first_page[arr.active[j]]; };
 
   // a unit in registers, with where it goes and what it waits for
@@ -246,16 +258,16 @@ __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs
     int32_t shift;
     RowDep dep;
   };
-  // slot i = kk * row_size + pos, kk the compacted page row
-  auto fetch = [&](int kk, int pos, Meta &m) {
+  // slot i = kk * row_size + j * n_lanes + tl: kk the compacted page row, j the
+  // active sequence, tl the tile lane
+  auto fetch = [&](int kk, int j, int tl, Meta &m) {
     m.valid = 0;
     if (kk >= max_dest) return;
-    const int j = pos / a.n_lanes;
     if (kk >= nd_of(j)) return;
     const int b = seq_of(j);
     m.valid = 1;
-    m.tl = pos - j * a.n_lanes;
-    m.idx = ub_of(j) / a.n_lanes + kk;
+    m.tl = tl;
+    m.idx = row0_of(j) + kk;
     m.my_src = lane < kPageSize ? pd.src[(int64_t)m.idx * kPageSize + lane] : kNoWrite;
     m.page = a.block_table[(int64_t)b * a.max_pages + fp_of(j) + kk];
     m.shift = (ROPE && lane < kPageSize) ? pd.shift[(int64_t)m.idx * kPageSize + lane] : 0;
@@ -275,8 +287,19 @@ __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs
     for (int it = 0; it < PER_LANE; ++it) t.v[it] = make_uint4(0, 0, 0, 0);
     if (!m.valid) return;
     const int tl = m.tl;
-    const int layer = tl / (2 * Hkv), kv = (tl / Hkv) & 1, h = tl % Hkv;
-    const int64_t tile = layer * layer_stride + (int)(kv * kv_stride32 + h * kHead + my_col * 8);
+    int64_t tile;
+    int kv, lh;   // lh = layer * Hkv + head
+    if (lanes_in_smem) {
+      tile = s_toff[tl] + my_col * 8;
+      const int32_t e = s_tlh[tl];
+      kv = (int)((uint32_t)e >> 31);
+      lh = e & 0x7fffffff;
+    } else {
+      const int layer = tl / (2 * Hkv), h = tl % Hkv;
+      kv = (tl / Hkv) & 1;
+      lh = layer * Hkv + h;
+      tile = layer * layer_stride + (int)(kv * kv_stride32 + h * kHead + my_col * 8);
+    }
     const uint16_t *sur = kv ? a.sur_v : a.sur_k;
     t.valid = 1;
     t.row = m.idx;
@@ -294,7 +317,7 @@ __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs
         t.v[it] = ld_v4(a.pool + tile + src);
       } else if (src != kNoWrite) {
         const int64_t si = -src - 1;
-        t.v[it] = ld_v4(sur + ((si * a.n_layers + layer) * Hkv + h) * D + my_col * 8);
+        t.v[it] = ld_v4(sur + (si * a.n_layers * Hkv + lh) * D + my_col * 8);
       }
     }
     t.dlo = m.dep.lo;
@@ -393,26 +416,34 @@ __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs
 
   const int mover = blockIdx.x * kMovers + wid;
   const int my_units = mover < n_slots ? (n_slots - 1 - mover) / nm + 1 : 0;
+  // the unit's (kk, j, tl) advance by nm slots without a division
   const int step_kk = nm / row_size, step_pos = nm - step_kk * row_size;
+  const int step_j = step_pos / a.n_lanes, step_tl = step_pos - step_j * a.n_lanes;
   int kk = mover / row_size, pos = mover - kk * row_size;
+  int j = pos / a.n_lanes, tl = pos - j * a.n_lanes;
   auto advance = [&]() {
     kk += step_kk;
-    pos += step_pos;
-    if (pos >= row_size) {
-      pos -= row_size;
+    j += step_j;
+    tl += step_tl;
+    if (tl >= a.n_lanes) {
+      tl -= a.n_lanes;
+      ++j;
+    }
+    if (j >= n_active) {
+      j -= n_active;
       ++kk;
     }
   };
   Tile A, B;
   Meta M;   // the descriptors of the next unit to load
   if (my_units > 0) {
-    fetch(kk, pos, M);
+    fetch(kk, j, tl, M);
     advance();
     load(M, A);
-    fetch(kk, pos, M);
+    fetch(kk, j, tl, M);
     advance();
     load(M, B);
-    fetch(kk, pos, M);
+    fetch(kk, j, tl, M);
     advance();
     land_and_count(A);
     rotate(A);
@@ -425,7 +456,7 @@ __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs
       if (!readers_done(cur)) return false;
       store(cur);
       load(M, cur);   // unit u + 2
-      fetch(kk, pos, M);
+      fetch(kk, j, tl, M);
       advance();
       land_and_count(next);
       rotate(next);
