@@ -387,18 +387,13 @@ __global__ void __launch_bounds__(kPfThreads, 2)
         tc_commit(&v_empty[s]);
         return true;
       };
-      for (int j = 0; j < n_kv && ok; ++j) {
-        const int s = j % kPfKStages, sb = j & 1;
-        if (!mbar_wait(&k_full[s], (j / kPfKStages) & 1)) {
-          ok = false;
-          break;
-        }
+      // S_x(i) = Q_x K(i)^T into buffer i & 1, free once P V(i - 2) has read it
+      auto sq = [&](int i) {
+        const int s = i % kPfKStages, sb = i & 1;
+        if (!mbar_wait(&k_full[s], (i / kPfKStages) & 1)) return false;
         const uint32_t k_base = smem_u32(smem + L::kKoff + s * L::kK);
-        for (int x = 0; x < nh && ok; ++x) {
-          if (!mbar_wait(&s_empty[x][sb], ((j >> 1) & 1) ^ 1)) {
-            ok = false;
-            break;
-          }
+        for (int x = 0; x < nh; ++x) {
+          if (!mbar_wait(&s_empty[x][sb], ((i >> 1) & 1) ^ 1)) return false;
           tc_fence_after();
           const uint32_t q_base = smem_u32(smem + x * L::kQ);
 #pragma unroll
@@ -409,11 +404,17 @@ __global__ void __launch_bounds__(kPfThreads, 2)
           }
           tc_commit(&s_full[x][sb]);
         }
-        if (!ok) break;
         tc_commit(&k_empty[s]);
-        if (j >= 1 && !pv(j - 1)) ok = false;
+        return true;
+      };
+      // Order S(0), S(1), then P V(j) as soon as P(j) is ready and S(j + 2) as
+      // soon as that product has freed the buffer: the softmax of tile j + 1
+      // runs while P V(j) and S(j + 2) do.
+      ok = ok && sq(0) && (n_kv < 2 || sq(1));
+      for (int j = 0; j < n_kv && ok; ++j) {
+        if (!pv(j)) ok = false;
+        else if (j + 2 < n_kv && !sq(j + 2)) ok = false;
       }
-      if (ok && !pv(n_kv - 1)) ok = false;
       if (ok)
         for (int x = 0; x < nh; ++x) tc_commit(&o_done[x]);
       if (!ok) set_error(a.status, UMIM_ERR_TIMEOUT);
