@@ -9,9 +9,11 @@
 // of the tensor memory), so one CTA's products fill the tensor cores while
 // the other's softmax runs.  Warp 0 loads tiles with TMA (Q once; 64-key K
 // tiles into a 2-stage ring running a tile ahead of the V^T tiles' 2-stage
-// ring), warp 1 issues tcgen05.mma (S = Q K^T into one of two tensor-memory
-// buffers, O += P V into a tensor-memory accumulator; an S buffer is reused
-// once the P V product that read it is done), and warps 2-5 run the online
+// ring), warp 1 issues the S = Q K^T products (tcgen05.mma into one of two
+// tensor-memory buffers, reused once the P V product that read it is done),
+// warp 6 the O += P V products into a tensor-memory accumulator (a separate
+// issuing thread, so that a P V product never waits behind an S product that
+// waits for the previous P V), and warps 2-5 run the online
 // softmax, one thread per query row: S from tensor memory (tcgen05.ld),
 // causal mask, running max, P = exp2(S - max) written back in fp16 over the
 // S columns it came from (tcgen05.st; the P V product reads its A operand
@@ -47,7 +49,8 @@ constexpr int kPfRows = 128;             // query rows per CTA (the MMA's M)
 constexpr int kPfKeys = 64;              // keys per K / V tile (the S MMA's N)
 constexpr int kPfKStages = 2;            // K ring (K runs kPfKStages - 1 tiles ahead of V^T)
 constexpr int kPfVStages = 2;            // V^T ring
-constexpr int kPfThreads = 192;          // warp 0 TMA, warp 1 MMA + tensor memory, warps 2-5 softmax (thread = query row)
+constexpr int kPfThreads = 224;          // warp 0 TMA, warp 1 S products + tensor memory, warps 2-5 softmax
+                                         // (thread = query row), warp 6 P V products
 constexpr int kPfPlanThreads = 1024;
 constexpr uint32_t kPfTmemCols = 256;    // S buffers at 0 and 64, O at 128: two CTAs per SM
 
@@ -257,7 +260,7 @@ __global__ void __launch_bounds__(kPfThreads, 2)
   constexpr int DA = D / 64;   // 64-wide atoms along the head dimension
   extern __shared__ __align__(1024) uint8_t pf_raw[];
   __shared__ __align__(8) uint64_t q_full, k_full[kPfKStages], k_empty[kPfKStages], v_full[kPfVStages],
-      v_empty[kPfVStages], s_full[2][2], s_empty[2][2], p_full[2][2], p_empty[2], o_done[2], mma_done;
+      v_empty[kPfVStages], s_full[2][2], s_empty[2][2], p_full[2][2], p_empty[2], o_done[2], mma_done[2];
   __shared__ uint32_t tmem_base;
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(pf_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -283,7 +286,8 @@ __global__ void __launch_bounds__(kPfThreads, 2)
       mbar_init(&p_empty[x], 1);
       mbar_init(&o_done[x], 1);   // one phase: every product of the CTA has landed
     }
-    mbar_init(&mma_done, 1);
+    mbar_init(&mma_done[0], 1);
+    mbar_init(&mma_done[1], 1);
     fence_mbar_init();
     prefetch_tensormap(&q_map);
     prefetch_tensormap(&k_map);
@@ -363,37 +367,23 @@ __global__ void __launch_bounds__(kPfThreads, 2)
       mbar_wait_for(&q_full, 0, kWaitLimitNs);
     }
   } else if (warp == 1) {
+    // ---- S_x(i) = Q_x K(i)^T into S buffer i & 1, once P V(i - 2) has read that buffer ----
     if (lane == 0 && n_kv > 0) {
       constexpr uint32_t idesc_s = idesc_f32acc(kPfRows, kPfKeys, false);
-      constexpr uint32_t idesc_o = idesc_f32acc(kPfRows, D, true);   // P and V^T in fp16
       bool ok = mbar_wait(&q_full, 0);
       tc_fence_after();
-      // O_x += P_x(i) V(i) for both heads (fp16 operands, P from tensor memory); frees V(i) and S(i)'s buffer
-      auto pv = [&](int i) {
-        const int s = i % kPfVStages;
-        if (!mbar_wait(&v_full[s], (i / kPfVStages) & 1)) return false;
-        const uint32_t v_base = smem_u32(smem + L::kVoff + s * L::kV);
-        for (int x = 0; x < nh; ++x) {
-          if (!mbar_wait(&p_full[x][i & 1], (i >> 1) & 1)) return false;
-          tc_fence_after();
-          const uint32_t p_tmem = tmem + x * 256 + (i & 1) * kPfKeys;   // P(i) sits where S(i) was
-#pragma unroll
-          for (int kk = 0; kk < kPfKeys / 16; ++kk)
-            tc_mma_ts(tmem + x * 256 + 128, p_tmem + kk * 8, sw128_kmajor_desc(v_base + kk * 32), idesc_o,
-                      (i | kk) != 0 ? 1u : 0u);
-          tc_commit(&p_empty[x]);
-          tc_commit(&s_empty[x][i & 1]);
-        }
-        tc_commit(&v_empty[s]);
-        return true;
-      };
-      // S_x(i) = Q_x K(i)^T into buffer i & 1, free once P V(i - 2) has read it
-      auto sq = [&](int i) {
+      for (int i = 0; i < n_kv && ok; ++i) {
         const int s = i % kPfKStages, sb = i & 1;
-        if (!mbar_wait(&k_full[s], (i / kPfKStages) & 1)) return false;
+        if (!mbar_wait(&k_full[s], (i / kPfKStages) & 1)) {
+          ok = false;
+          break;
+        }
         const uint32_t k_base = smem_u32(smem + L::kKoff + s * L::kK);
-        for (int x = 0; x < nh; ++x) {
-          if (!mbar_wait(&s_empty[x][sb], ((i >> 1) & 1) ^ 1)) return false;
+        for (int x = 0; x < nh && ok; ++x) {
+          if (!mbar_wait(&s_empty[x][sb], ((i >> 1) & 1) ^ 1)) {
+            ok = false;
+            break;
+          }
           tc_fence_after();
           const uint32_t q_base = smem_u32(smem + x * L::kQ);
 #pragma unroll
@@ -404,23 +394,48 @@ __global__ void __launch_bounds__(kPfThreads, 2)
           }
           tc_commit(&s_full[x][sb]);
         }
-        tc_commit(&k_empty[s]);
-        return true;
-      };
-      // Order S(0), S(1), then P V(j) as soon as P(j) is ready and S(j + 2) as
-      // soon as that product has freed the buffer: the softmax of tile j + 1
-      // runs while P V(j) and S(j + 2) do.
-      ok = ok && sq(0) && (n_kv < 2 || sq(1));
-      for (int j = 0; j < n_kv && ok; ++j) {
-        if (!pv(j)) ok = false;
-        else if (j + 2 < n_kv && !sq(j + 2)) ok = false;
+        if (ok) tc_commit(&k_empty[s]);
+      }
+      if (!ok) set_error(a.status, UMIM_ERR_TIMEOUT);
+      // every product this thread issued has finished before tensor memory is released
+      tc_commit(&mma_done[0]);
+      mbar_wait_for(&mma_done[0], 0, kWaitLimitNs);
+    }
+  } else if (warp == 6) {
+    // ---- O_x += P_x(i) V(i) (fp16 operands, P from tensor memory), as soon as P(i) is ready;
+    // frees V(i)'s stage and S(i)'s buffer.  A separate issuing thread, so that a P V product
+    // never waits behind an S product that waits for the previous P V ----
+    if (lane == 0 && n_kv > 0) {
+      constexpr uint32_t idesc_o = idesc_f32acc(kPfRows, D, true);   // P and V^T in fp16
+      bool ok = true;
+      for (int i = 0; i < n_kv && ok; ++i) {
+        const int s = i % kPfVStages;
+        if (!mbar_wait(&v_full[s], (i / kPfVStages) & 1)) {
+          ok = false;
+          break;
+        }
+        const uint32_t v_base = smem_u32(smem + L::kVoff + s * L::kV);
+        for (int x = 0; x < nh && ok; ++x) {
+          if (!mbar_wait(&p_full[x][i & 1], (i >> 1) & 1)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t p_tmem = tmem + x * 256 + (i & 1) * kPfKeys;   // P(i) sits where S(i) was
+#pragma unroll
+          for (int kk = 0; kk < kPfKeys / 16; ++kk)
+            tc_mma_ts(tmem + x * 256 + 128, p_tmem + kk * 8, sw128_kmajor_desc(v_base + kk * 32), idesc_o,
+                      (i | kk) != 0 ? 1u : 0u);
+          tc_commit(&p_empty[x]);
+          tc_commit(&s_empty[x][i & 1]);
+        }
+        if (ok) tc_commit(&v_empty[s]);
       }
       if (ok)
         for (int x = 0; x < nh; ++x) tc_commit(&o_done[x]);
       if (!ok) set_error(a.status, UMIM_ERR_TIMEOUT);
-      // every MMA issued has finished before tensor memory is released
-      tc_commit(&mma_done);
-      mbar_wait_for(&mma_done, 0, kWaitLimitNs);
+      tc_commit(&mma_done[1]);
+      mbar_wait_for(&mma_done[1], 0, kWaitLimitNs);
     }
   } else if ((warp - 2) / 4 < nh) {
     // ---- softmax and epilogue of head x: four warps, thread = query row ----
