@@ -4,10 +4,12 @@
 // then runs over the shorter sequences).  Sequence b owns rows
 // cu_seqlens[b] .. cu_seqlens[b+1]-1 of q [T][Hq][D], k, v [T][Hkv][D].
 //
-// On the 5th-generation tensor cores: one CTA takes 128 query rows of one
-// sequence for one query head, and two CTAs share an SM (each allocates half
-// of the tensor memory), so one CTA's products fill the tensor cores while
-// the other's softmax runs.  Warp 0 loads tiles with TMA (Q once; 64-key K
+// On the 5th-generation tensor cores: a persistent kernel, two CTAs per SM
+// (each allocates half of the tensor memory, so one CTA's products fill the
+// tensor cores while the other's softmax runs), each walking work units of
+// 128 query rows of one sequence for one query head, heaviest first; the
+// next unit's Q and K loads and first S products overlap the current unit's
+// last tiles and epilogue.  Warp 0 loads tiles with TMA (Q once; 64-key K
 // tiles into a 2-stage ring running a tile ahead of the V^T tiles' 2-stage
 // ring), warp 1 issues the S = Q K^T products (tcgen05.mma into one of two
 // tensor-memory buffers, reused once the P V product that read it is done),
@@ -259,14 +261,17 @@ __global__ void __launch_bounds__(kPfThreads, 2)
   using L = PfSmem<D>;
   constexpr int DA = D / 64;   // 64-wide atoms along the head dimension
   extern __shared__ __align__(1024) uint8_t pf_raw[];
-  __shared__ __align__(8) uint64_t q_full, k_full[kPfKStages], k_empty[kPfKStages], v_full[kPfVStages],
-      v_empty[kPfVStages], s_full[2][2], s_empty[2][2], p_full[2][2], p_empty[2], o_done[2], mma_done[2];
+  __shared__ __align__(8) uint64_t q_full, q_empty, k_full[kPfKStages], k_empty[kPfKStages], v_full[kPfVStages],
+      v_empty[kPfVStages], s_full[2], s_empty[2], p_full[2], p_empty, o_done, o_free, mma_done[2];
   __shared__ uint32_t tmem_base;
+  __shared__ int s_abort;
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(pf_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) {
+    s_abort = 0;
     mbar_init(&q_full, 1);
+    mbar_init(&q_empty, 1);    // committed once a unit's S products have read Q
     for (int s = 0; s < kPfKStages; ++s) {
       mbar_init(&k_full[s], 1);
       mbar_init(&k_empty[s], 1);
@@ -275,17 +280,14 @@ __global__ void __launch_bounds__(kPfThreads, 2)
       mbar_init(&v_full[s], 1);
       mbar_init(&v_empty[s], 1);
     }
-    for (int x = 0; x < 2; ++x) {
-      for (int i = 0; i < 2; ++i) {
-        mbar_init(&s_full[x][i], 1);
-        mbar_init(&s_empty[x][i], 1);   // committed once the P V product that read P from it is done
-      }
-      // P(j) ready, by tile parity: the softmax can run a tile ahead of the MMA warp's wait
-      mbar_init(&p_full[x][0], 4);
-      mbar_init(&p_full[x][1], 4);
-      mbar_init(&p_empty[x], 1);
-      mbar_init(&o_done[x], 1);   // one phase: every product of the CTA has landed
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&s_full[i], 1);
+      mbar_init(&s_empty[i], 1);   // committed once the P V product that read P from it is done
+      mbar_init(&p_full[i], 4);    // P ready, by tile parity (the four softmax warps)
     }
+    mbar_init(&p_empty, 1);       // a P V product has landed
+    mbar_init(&o_done, 1);        // a unit's products have landed in O
+    mbar_init(&o_free, 4);        // a unit's epilogue has read O (the four softmax warps)
     mbar_init(&mma_done[0], 1);
     mbar_init(&mma_done[1], 1);
     fence_mbar_init();
@@ -303,231 +305,270 @@ __global__ void __launch_bounds__(kPfThreads, 2)
   const uint32_t tmem = tmem_base;
   griddep_wait();
 
-  // the work unit: query tile qt of sequence b for the query heads h0 (and h0 + 1)
+  // Work units: (query tile, query head), the tiles heaviest first (a
+  // sequence's last tiles) and the heads of a tile consecutive, so CTAs that
+  // run at the same time share K and V tiles in L2.  CTA c takes units c,
+  // c + G, c + 2G, ...; every barrier keeps counting across units (tile
+  // counters run over the CTA's units).
   const int total = a.cu_tiles[a.B];
-  const bool active = (int)blockIdx.x < total;
-  int b = 0, qt = 0;
-  if (active) {
-    const int t = total - 1 - (int)blockIdx.x;   // a sequence's last (heaviest) tiles first
-    b = pf_find(a.cu_tiles, a.B, t);
-    qt = t - a.cu_tiles[b];
-  }
-  const int s0 = active ? a.cu[b] : 0, len = active ? a.cu[b + 1] - s0 : 0;
-  const int q0 = qt * kPfRows;
-  const int h0 = (int)blockIdx.y, g = h0 / a.G;          // one query head per CTA
-  const int nh = 1;
-  const int n_kv = active ? (min(q0 + kPfRows, len) + kPfKeys - 1) / kPfKeys : 0;   // causal key tiles
-  const int kbase = active ? a.pcu[b] : 0;
+  const int n_units = total * a.Hq;
+  const int G = (int)gridDim.x;
+  struct Unit {
+    int s0, len, q0, h, g, n_kv, kbase;
+  };
+  auto unit_of = [&](int u) {
+    Unit w;
+    const int t = total - 1 - u / a.Hq;   // a sequence's last (heaviest) tiles first
+    const int b = pf_find(a.cu_tiles, a.B, t);
+    const int qt = t - a.cu_tiles[b];
+    w.s0 = a.cu[b];
+    w.len = a.cu[b + 1] - w.s0;
+    w.q0 = qt * kPfRows;
+    w.h = u % a.Hq;
+    w.g = w.h / a.G;
+    w.n_kv = (min(w.q0 + kPfRows, w.len) + kPfKeys - 1) / kPfKeys;   // causal key tiles
+    w.kbase = a.pcu[b];
+    return w;
+  };
+  // a warp that gave up tells the others, so that no wait is left to time out on its own
+  auto aborted = [&]() { return *reinterpret_cast<volatile int *>(&s_abort) != 0; };
+  auto give_up = [&]() {
+    set_error(a.status, UMIM_ERR_TIMEOUT);
+    *reinterpret_cast<volatile int *>(&s_abort) = 1;
+  };
 
   if (warp == 0) {
-    if (lane == 0 && n_kv > 0) {
+    if (lane == 0) {
       const uint64_t pol_q = policy_evict_first(), pol_kv = policy_evict_last();
-      mbar_arrive_expect_tx(&q_full, nh * L::kQ);
-      for (int x = 0; x < nh; ++x)
-#pragma unroll
-        for (int d = 0; d < DA; ++d)
-          tma_load_3d(smem + x * L::kQ + d * (kPfRows * 128), &q_map, &q_full, d * 64, h0 + x, s0 + q0, pol_q);
       // K runs kPfKStages - 1 tiles ahead of V^T: a K load never waits behind
       // the P V product that frees a V^T stage
       constexpr int kLead = kPfKStages - 1;
-      int jk = 0, jv = 0;
+      int nk = 0, nv = 0, nq = 0;   // K and V^T tiles (ring positions) and Q tiles loaded so far
       bool ok = true;
-      for (int i = 0; i < n_kv + kLead && ok; ++i) {
-        if (i < n_kv) {
-          const int s = i % kPfKStages;
-          if (!mbar_wait(&k_empty[s], ((i / kPfKStages) & 1) ^ 1)) {
-            ok = false;
-            break;
-          }
-          mbar_arrive_expect_tx(&k_full[s], L::kK);
-#pragma unroll
-          for (int d = 0; d < DA; ++d)
-            tma_load_3d(smem + L::kKoff + s * L::kK + d * (kPfKeys * 128), &k_map, &k_full[s], d * 64, g,
-                        s0 + i * kPfKeys, pol_kv);
-          jk = i + 1;
-        }
-        const int j = i - kLead;
-        if (j >= 0 && j < n_kv) {
-          const int s = j % kPfVStages;
-          if (!mbar_wait(&v_empty[s], ((j / kPfVStages) & 1) ^ 1)) {
-            ok = false;
-            break;
-          }
-          mbar_arrive_expect_tx(&v_full[s], L::kV);
-          tma_load_3d(smem + L::kVoff + s * L::kV, &vt_map, &v_full[s], kbase + j * kPfKeys, 0, g, pol_kv);
-          jv = j + 1;
-        }
-      }
-      if (!ok) set_error(a.status, UMIM_ERR_TIMEOUT);
-      // copies still in flight when a consumer gave up: wait for them (bounded)
-      for (int i = max(0, jk - kPfKStages); i < jk; ++i)
-        mbar_wait_for(&k_full[i % kPfKStages], (i / kPfKStages) & 1, kWaitLimitNs);
-      for (int i = max(0, jv - kPfVStages); i < jv; ++i)
-        mbar_wait_for(&v_full[i % kPfVStages], (i / kPfVStages) & 1, kWaitLimitNs);
-      mbar_wait_for(&q_full, 0, kWaitLimitNs);
-    }
-  } else if (warp == 1) {
-    // ---- S_x(i) = Q_x K(i)^T into S buffer i & 1, once P V(i - 2) has read that buffer ----
-    if (lane == 0 && n_kv > 0) {
-      constexpr uint32_t idesc_s = idesc_f32acc(kPfRows, kPfKeys, false);
-      bool ok = mbar_wait(&q_full, 0);
-      tc_fence_after();
-      for (int i = 0; i < n_kv && ok; ++i) {
-        const int s = i % kPfKStages, sb = i & 1;
-        if (!mbar_wait(&k_full[s], (i / kPfKStages) & 1)) {
+      int k_unit = 0;
+      for (int u = (int)blockIdx.x; u < n_units && ok; u += G, ++k_unit) {
+        const Unit w = unit_of(u);
+        // Q of the previous unit has been read by its last S product
+        if (k_unit > 0 && (aborted() || !mbar_wait(&q_empty, (uint32_t)(k_unit - 1) & 1u))) {
           ok = false;
           break;
         }
-        const uint32_t k_base = smem_u32(smem + L::kKoff + s * L::kK);
-        for (int x = 0; x < nh && ok; ++x) {
-          if (!mbar_wait(&s_empty[x][sb], ((i >> 1) & 1) ^ 1)) {
+        mbar_arrive_expect_tx(&q_full, L::kQ);
+#pragma unroll
+        for (int d = 0; d < DA; ++d)
+          tma_load_3d(smem + d * (kPfRows * 128), &q_map, &q_full, d * 64, w.h, w.s0 + w.q0, pol_q);
+        ++nq;
+        for (int i = 0; i < w.n_kv + kLead && ok; ++i) {
+          if (i < w.n_kv) {
+            const int s = nk % kPfKStages;
+            if (aborted() || !mbar_wait(&k_empty[s], ((nk / kPfKStages) & 1) ^ 1)) {
+              ok = false;
+              break;
+            }
+            mbar_arrive_expect_tx(&k_full[s], L::kK);
+#pragma unroll
+            for (int d = 0; d < DA; ++d)
+              tma_load_3d(smem + L::kKoff + s * L::kK + d * (kPfKeys * 128), &k_map, &k_full[s], d * 64, w.g,
+                          w.s0 + i * kPfKeys, pol_kv);
+            ++nk;
+          }
+          const int j = i - kLead;
+          if (j >= 0 && j < w.n_kv) {
+            const int s = nv % kPfVStages;
+            if (aborted() || !mbar_wait(&v_empty[s], ((nv / kPfVStages) & 1) ^ 1)) {
+              ok = false;
+              break;
+            }
+            mbar_arrive_expect_tx(&v_full[s], L::kV);
+            tma_load_3d(smem + L::kVoff + s * L::kV, &vt_map, &v_full[s], w.kbase + j * kPfKeys, 0, w.g, pol_kv);
+            ++nv;
+          }
+        }
+      }
+      if (!ok) give_up();
+      // copies still in flight when a consumer gave up: wait for them (bounded)
+      for (int i = max(0, nk - kPfKStages); i < nk; ++i)
+        mbar_wait_for(&k_full[i % kPfKStages], (i / kPfKStages) & 1, kWaitLimitNs);
+      for (int i = max(0, nv - kPfVStages); i < nv; ++i)
+        mbar_wait_for(&v_full[i % kPfVStages], (i / kPfVStages) & 1, kWaitLimitNs);
+      if (nq > 0) mbar_wait_for(&q_full, (uint32_t)(nq - 1) & 1u, kWaitLimitNs);
+    }
+  } else if (warp == 1) {
+    // ---- S = Q K(i)^T into S buffer (tile counter) & 1, once the P V product that read that buffer is done ----
+    if (lane == 0) {
+      constexpr uint32_t idesc_s = idesc_f32acc(kPfRows, kPfKeys, false);
+      bool ok = true;
+      int nt = 0, k_unit = 0;   // tiles and units so far
+      for (int u = (int)blockIdx.x; u < n_units && ok; u += G, ++k_unit) {
+        const Unit w = unit_of(u);
+        if (aborted() || !mbar_wait(&q_full, (uint32_t)k_unit & 1u)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t q_base = smem_u32(smem);
+        for (int i = 0; i < w.n_kv; ++i, ++nt) {
+          const int s = nt % kPfKStages, sb = nt & 1;
+          if (aborted() || !mbar_wait(&k_full[s], (nt / kPfKStages) & 1) ||
+              !mbar_wait(&s_empty[sb], ((nt >> 1) & 1) ^ 1)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t q_base = smem_u32(smem + x * L::kQ);
+          const uint32_t k_base = smem_u32(smem + L::kKoff + s * L::kK);
 #pragma unroll
           for (int kk = 0; kk < D / 16; ++kk) {
             const uint32_t off = (kk & 3) * 32;
-            tc_mma_bf16(tmem + x * 256 + sb * kPfKeys, sw128_kmajor_desc(q_base + (kk >> 2) * (kPfRows * 128) + off),
+            tc_mma_bf16(tmem + sb * kPfKeys, sw128_kmajor_desc(q_base + (kk >> 2) * (kPfRows * 128) + off),
                         sw128_kmajor_desc(k_base + (kk >> 2) * (kPfKeys * 128) + off), idesc_s, kk != 0 ? 1u : 0u);
           }
-          tc_commit(&s_full[x][sb]);
+          tc_commit(&s_full[sb]);
+          tc_commit(&k_empty[s]);
         }
-        if (ok) tc_commit(&k_empty[s]);
+        if (ok) tc_commit(&q_empty);   // the unit's S products have read Q
       }
-      if (!ok) set_error(a.status, UMIM_ERR_TIMEOUT);
+      if (!ok) give_up();
       // every product this thread issued has finished before tensor memory is released
       tc_commit(&mma_done[0]);
       mbar_wait_for(&mma_done[0], 0, kWaitLimitNs);
     }
   } else if (warp == 6) {
-    // ---- O_x += P_x(i) V(i) (fp16 operands, P from tensor memory), as soon as P(i) is ready;
-    // frees V(i)'s stage and S(i)'s buffer.  A separate issuing thread, so that a P V product
-    // never waits behind an S product that waits for the previous P V ----
-    if (lane == 0 && n_kv > 0) {
+    // ---- O += P V(i) (fp16 operands, P from tensor memory), as soon as P(i) is ready; frees V(i)'s
+    // stage and S(i)'s buffer.  A separate issuing thread, so that a P V product never waits behind
+    // an S product that waits for the previous P V.  A unit's first product overwrites O once the
+    // previous unit's epilogue has read it ----
+    if (lane == 0) {
       constexpr uint32_t idesc_o = idesc_f32acc(kPfRows, D, true);   // P and V^T in fp16
       bool ok = true;
-      for (int i = 0; i < n_kv && ok; ++i) {
-        const int s = i % kPfVStages;
-        if (!mbar_wait(&v_full[s], (i / kPfVStages) & 1)) {
+      int nt = 0, k_unit = 0;
+      for (int u = (int)blockIdx.x; u < n_units && ok; u += G, ++k_unit) {
+        const Unit w = unit_of(u);
+        if (k_unit > 0 && (aborted() || !mbar_wait(&o_free, (uint32_t)(k_unit - 1) & 1u))) {
           ok = false;
           break;
         }
-        const uint32_t v_base = smem_u32(smem + L::kVoff + s * L::kV);
-        for (int x = 0; x < nh && ok; ++x) {
-          if (!mbar_wait(&p_full[x][i & 1], (i >> 1) & 1)) {
+        for (int i = 0; i < w.n_kv; ++i, ++nt) {
+          const int s = nt % kPfVStages, sb = nt & 1;
+          if (aborted() || !mbar_wait(&v_full[s], (nt / kPfVStages) & 1) ||
+              !mbar_wait(&p_full[sb], (nt >> 1) & 1)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t p_tmem = tmem + x * 256 + (i & 1) * kPfKeys;   // P(i) sits where S(i) was
+          const uint32_t v_base = smem_u32(smem + L::kVoff + s * L::kV);
+          const uint32_t p_tmem = tmem + sb * kPfKeys;   // P(i) sits where S(i) was
 #pragma unroll
           for (int kk = 0; kk < kPfKeys / 16; ++kk)
-            tc_mma_ts(tmem + x * 256 + 128, p_tmem + kk * 8, sw128_kmajor_desc(v_base + kk * 32), idesc_o,
+            tc_mma_ts(tmem + 128, p_tmem + kk * 8, sw128_kmajor_desc(v_base + kk * 32), idesc_o,
                       (i | kk) != 0 ? 1u : 0u);
-          tc_commit(&p_empty[x]);
-          tc_commit(&s_empty[x][i & 1]);
+          tc_commit(&p_empty);
+          tc_commit(&s_empty[sb]);
+          tc_commit(&v_empty[s]);
         }
-        if (ok) tc_commit(&v_empty[s]);
+        if (ok) tc_commit(&o_done);   // the unit's products have landed in O
       }
-      if (ok)
-        for (int x = 0; x < nh; ++x) tc_commit(&o_done[x]);
-      if (!ok) set_error(a.status, UMIM_ERR_TIMEOUT);
+      if (!ok) give_up();
       tc_commit(&mma_done[1]);
       mbar_wait_for(&mma_done[1], 0, kWaitLimitNs);
     }
-  } else if ((warp - 2) / 4 < nh) {
-    // ---- softmax and epilogue of head x: four warps, thread = query row ----
-    const int x = (warp - 2) >> 2;
+  } else if (warp >= 2 && warp < 6) {
+    // ---- softmax and epilogue: four warps, thread = query row ----
     const int quad = warp & 3;                 // tensor-memory lanes this warp may access
     const int r = quad * 32 + lane;            // query row within the tile
-    const int qpos = q0 + r;                   // position within the sequence
-    const int kmax = min(qpos, len - 1);       // last key this row sees
-    const uint32_t t_s = tmem + ((uint32_t)(quad * 32) << 16) + x * 256;   // this row's S buffers
-    const uint32_t t_o = t_s + 128;                                         // and O
+    const uint32_t t_s = tmem + ((uint32_t)(quad * 32) << 16);   // this row's S buffers
+    const uint32_t t_o = t_s + 128;                                // and O
     const float sl2 = a.scale_log2;
-    float m_run = -INFINITY, l_run = 0.f;      // running max (log2 units, moved in steps > 8) and row sum
     bool ok = true;
     // every lane waits (each needs the acquire), the warp goes on only if all saw the phase:
     // the .sync.aligned tensor-memory instructions below need the whole warp
-    auto wwait = [&](uint64_t *m, uint32_t parity) { return __all_sync(0xffffffffu, mbar_wait(m, parity)) != 0; };
-    for (int j = 0; j < n_kv && ok; ++j) {
-      const int sb = j & 1;
-      if (!wwait(&s_full[x][sb], (j >> 1) & 1)) {
-        ok = false;
-        break;
-      }
-      tc_fence_after();
-      float s[kPfKeys];
-      tmem_ld_32x32b_x64(t_s + sb * kPfKeys, s);
-      const int k0 = j * kPfKeys;
-      if (k0 + kPfKeys - 1 > kmax) {   // the diagonal tile (or a row past the sequence)
-#pragma unroll
-        for (int c = 0; c < kPfKeys; ++c) s[c] = (k0 + c <= kmax) ? s[c] : -INFINITY;
-      }
-      float m4[4] = {s[0], s[1], s[2], s[3]};
-#pragma unroll
-      for (int c = 4; c < kPfKeys; ++c) m4[c & 3] = fmaxf(m4[c & 3], s[c]);
-      const float mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])) * sl2;
-      // move the running max only when it grows by more than 2^8
-      const bool grow = mx > m_run + 8.f;
-      float alpha = 1.f;
-      if (grow) {
-        alpha = (m_run == -INFINITY) ? 0.f : ex2_approx(m_run - mx);
-        m_run = mx;
-        l_run *= alpha;
-      }
-      const float nm = (m_run == -INFINITY) ? 0.f : -m_run;
-      float l4[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-      for (int c = 0; c < kPfKeys; ++c) {
-        s[c] = ex2_approx(fmaf(s[c], sl2, nm));   // masked (-inf): 0
-        l4[c & 3] += s[c];
-      }
-      l_run += (l4[0] + l4[1]) + (l4[2] + l4[3]);
-      // O is rescaled only once the product of tile j - 1 has landed
-      if (j > 0 && __any_sync(0xffffffffu, grow)) {
-        if (!wwait(&p_empty[x], (j - 1) & 1)) {
+    auto wwait = [&](uint64_t *m, uint32_t parity) {
+      return __all_sync(0xffffffffu, !aborted() && mbar_wait(m, parity)) != 0;
+    };
+    int nt = 0, k_unit = 0;
+    for (int u = (int)blockIdx.x; u < n_units && ok; u += G, ++k_unit) {
+      const Unit w = unit_of(u);
+      const int qpos = w.q0 + r;                  // position within the sequence
+      const int kmax = min(qpos, w.len - 1);      // last key this row sees
+      float m_run = -INFINITY, l_run = 0.f;       // running max (log2 units, moved in steps > 8) and row sum
+      for (int j = 0; j < w.n_kv; ++j, ++nt) {
+        const int sb = nt & 1;
+        if (!wwait(&s_full[sb], (nt >> 1) & 1)) {
           ok = false;
           break;
         }
         tc_fence_after();
-#pragma unroll 1
-        for (int c = 0; c < D / 32; ++c) {
-          float o[32];
-          tmem_ld_32x32b_x32(t_o + c * 32, o);
+        float s[kPfKeys];
+        tmem_ld_32x32b_x64(t_s + sb * kPfKeys, s);
+        const int k0 = j * kPfKeys;
+        if (k0 + kPfKeys - 1 > kmax) {   // the diagonal tile (or a row past the sequence)
 #pragma unroll
-          for (int i = 0; i < 32; ++i) o[i] *= alpha;
-          tmem_st_32x32b_x32(t_o + c * 32, o);
+          for (int c = 0; c < kPfKeys; ++c) s[c] = (k0 + c <= kmax) ? s[c] : -INFINITY;
+        }
+        float m4[4] = {s[0], s[1], s[2], s[3]};
+#pragma unroll
+        for (int c = 4; c < kPfKeys; ++c) m4[c & 3] = fmaxf(m4[c & 3], s[c]);
+        const float mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])) * sl2;
+        // move the running max only when it grows by more than 2^8
+        const bool grow = mx > m_run + 8.f;
+        float alpha = 1.f;
+        if (grow) {
+          alpha = (m_run == -INFINITY) ? 0.f : ex2_approx(m_run - mx);
+          m_run = mx;
+          l_run *= alpha;
+        }
+        const float nm = (m_run == -INFINITY) ? 0.f : -m_run;
+        float l4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int c = 0; c < kPfKeys; ++c) {
+          s[c] = ex2_approx(fmaf(s[c], sl2, nm));   // masked (-inf): 0
+          l4[c & 3] += s[c];
+        }
+        l_run += (l4[0] + l4[1]) + (l4[2] + l4[3]);
+        // O is rescaled only once the product of tile j - 1 has landed
+        if (j > 0 && __any_sync(0xffffffffu, grow)) {
+          if (!wwait(&p_empty, (uint32_t)(nt - 1) & 1u)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+#pragma unroll 1
+          for (int c = 0; c < D / 32; ++c) {
+            float o[32];
+            tmem_ld_32x32b_x32(t_o + c * 32, o);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) o[i] *= alpha;
+            tmem_st_32x32b_x32(t_o + c * 32, o);
+          }
+          tc_fence_before();
+        }
+        // P(j) in fp16 over S(j)'s columns (this thread has read them), for the P V product
+        {
+          float pk[32];
+#pragma unroll
+          for (int c = 0; c < 32; ++c) {
+            const __half2 hh = __floats2half2_rn(s[2 * c], s[2 * c + 1]);   // P <= 2^8
+            pk[c] = __uint_as_float(*reinterpret_cast<const uint32_t *>(&hh));
+          }
+          tmem_st_32x32b_x32(t_s + sb * kPfKeys, pk);
         }
         tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&p_full[sb]);
       }
-      // P(j) in fp16 over S(j)'s columns (this thread has read them), for the P V product
-      {
-        float pk[32];
-#pragma unroll
-        for (int c = 0; c < 32; ++c) {
-          const __half2 hh = __floats2half2_rn(s[2 * c], s[2 * c + 1]);   // P <= 2^8
-          pk[c] = __uint_as_float(*reinterpret_cast<const uint32_t *>(&hh));
-        }
-        tmem_st_32x32b_x32(t_s + sb * kPfKeys, pk);
+      if (!ok) break;
+      // epilogue: O / l once the unit's last product has landed, then O is free for the next unit
+      if (!wwait(&o_done, (uint32_t)k_unit & 1u)) {
+        ok = false;
+        break;
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&p_full[x][sb]);
-    }
-    if (!ok) set_error(a.status, UMIM_ERR_TIMEOUT);
-    // epilogue: O / l once the last product has landed
-    if (ok && n_kv > 0 && wwait(&o_done[x], 0)) {
       tc_fence_after();
       const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
-      __nv_bfloat16 *orow = a.out + (((int64_t)s0 + qpos) * a.Hq + h0 + x) * D;
+      __nv_bfloat16 *orow = a.out + (((int64_t)w.s0 + qpos) * a.Hq + w.h) * D;
 #pragma unroll 1
       for (int c = 0; c < D / 32; ++c) {
         float o[32];
         tmem_ld_32x32b_x32(t_o + c * 32, o);
-        if (qpos < len) {
+        if (qpos < w.len) {
           uint4 *dst = reinterpret_cast<uint4 *>(orow + c * 32);
 #pragma unroll
           for (int e = 0; e < 4; ++e)
@@ -537,9 +578,11 @@ __global__ void __launch_bounds__(kPfThreads, 2)
                                 pack_bf16x2(o[8 * e + 6] * inv, o[8 * e + 7] * inv));
         }
       }
-    } else if (n_kv > 0 && ok) {
-      set_error(a.status, UMIM_ERR_TIMEOUT);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&o_free);
     }
+    if (!ok) give_up();
   }
   tc_fence_before();
   __syncthreads();
@@ -574,7 +617,6 @@ size_t prefill_attention_workspace_bytes(int B, int T, int Hkv, int D) {
 umim_status prefill_attention(const void *q, const void *k, const void *v, int T, int Hq, int Hkv, int D,
                               const int32_t *cu_seqlens, int B, float scale, void *out, void *ws, int32_t *status,
                               cudaStream_t stream, int num_sms) {
-  (void)num_sms;
   EncodeTiledFn enc = get_encode_tiled();
   if (!enc) return UMIM_ERR_CUDA;
   PfArgs a{};
@@ -609,11 +651,12 @@ umim_status prefill_attention(const void *q, const void *k, const void *v, int T
   const size_t smem = (size_t)(D == 128 ? PfSmem<128>::kTotal : PfSmem<64>::kTotal) + 1024;
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
     return UMIM_ERR_CUDA;
-  // an upper bound of the query tiles: each sequence wastes less than one
-  const unsigned gx = (unsigned)((T + kPfRows - 1) / kPfRows + B);
+  // persistent: two CTAs per SM walk the (query tile, head) units; no more
+  // CTAs than an upper bound of the units (each sequence wastes less than one tile)
+  const int64_t units_max = ((int64_t)(T + kPfRows - 1) / kPfRows + B) * Hq;
+  const unsigned gx = (unsigned)std::max<int64_t>(1, std::min<int64_t>(2LL * std::max(num_sms, 1), units_max));
   trace_mark(stream, "prefill.attention");
-  const unsigned gy = (unsigned)Hq;   // one query head per CTA
-  if (launch_pdl(kern, dim3(gx, gy), dim3(kPfThreads), smem, stream, qm, km, vm, a) != cudaSuccess)
+  if (launch_pdl(kern, dim3(gx), dim3(kPfThreads), smem, stream, qm, km, vm, a) != cudaSuccess)
     return UMIM_ERR_CUDA;
   trace_mark(stream, nullptr);
   return UMIM_OK;
