@@ -517,13 +517,19 @@ __global__ void __launch_bounds__(kPfThreads, 2)
           l_run *= alpha;
         }
         const float nm = (m_run == -INFINITY) ? 0.f : -m_run;
-        float l4[4] = {0.f, 0.f, 0.f, 0.f};
+        // exp2(s * scale - max) and the row sum, two columns per packed instruction
+        const float2 sl2x2 = make_float2(sl2, sl2), nm2 = make_float2(nm, nm);
+        float2 la = make_float2(0.f, 0.f), lb = la;
 #pragma unroll
-        for (int c = 0; c < kPfKeys; ++c) {
-          s[c] = ex2_approx(fmaf(s[c], sl2, nm));   // masked (-inf): 0
-          l4[c & 3] += s[c];
+        for (int c = 0; c < kPfKeys; c += 2) {
+          const float2 x = __ffma2_rn(make_float2(s[c], s[c + 1]), sl2x2, nm2);
+          s[c] = ex2_approx(x.x);   // masked (-inf): 0
+          s[c + 1] = ex2_approx(x.y);
+          if (c & 2) lb = __fadd2_rn(lb, make_float2(s[c], s[c + 1]));
+          else la = __fadd2_rn(la, make_float2(s[c], s[c + 1]));
         }
-        l_run += (l4[0] + l4[1]) + (l4[2] + l4[3]);
+        const float2 lab = __fadd2_rn(la, lb);
+        l_run += lab.x + lab.y;
         // O is rescaled only once the product of tile j - 1 has landed
         if (j > 0 && __any_sync(0xffffffffu, grow)) {
           if (!wwait(&p_empty, (uint32_t)(nt - 1) & 1u)) {
