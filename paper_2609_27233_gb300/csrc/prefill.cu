@@ -220,6 +220,11 @@ __device__ __forceinline__ void tmem_st_32x32b_x32(uint32_t taddr, const float (
 
 // the hardware's approximate base-2 exponential (PTX ex2.approx.ftz: relative
 // error about 2^-22, -inf -> 0)
+__device__ __forceinline__ float max3f(float x, float y, float z) {   // max of three, one instruction
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(x), "f"(y), "f"(z));
+  return r;
+}
 __device__ __forceinline__ float ex2_approx(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
@@ -506,7 +511,7 @@ __global__ void __launch_bounds__(kPfThreads, 2)
         }
         float m4[4] = {s[0], s[1], s[2], s[3]};
 #pragma unroll
-        for (int c = 4; c < kPfKeys; ++c) m4[c & 3] = fmaxf(m4[c & 3], s[c]);
+        for (int c = 4; c < kPfKeys; c += 2) m4[(c >> 1) & 3] = max3f(m4[(c >> 1) & 3], s[c], s[c + 1]);
         const float mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])) * sl2;
         // move the running max only when it grows by more than 2^8
         const bool grow = mx > m_run + 8.f;
