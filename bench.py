@@ -308,14 +308,16 @@ def cpu_cores():
 
 
 # ---------------------------------------------------------------------------
-def traffic_from_profile(label):
-    """DRAM bytes per launch from the committed ncu summary, if the kernel's
-    source is unchanged since the capture."""
+def traffic_from_profile(label, workload="llama8b_layer"):
+    """DRAM bytes per launch from the committed ncu summary, if it was captured
+    on this workload and the kernel's source is unchanged since."""
     path = os.path.join(ROOT, "profiles", "ncu_traffic.json")
     try:
         with open(path) as f:
             prof = json.load(f)
         e = prof[label]
+        if e.get("workload") != workload:
+            return None
         src = os.path.join(ROOT, "paper_2609_27233_gb300", "csrc", e["source"])
         sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
         if sha != e["source_sha"]:
@@ -1031,6 +1033,7 @@ def side_bench(args):
     dev = torch.device("cuda", 0)
     umim.lib()
     peaks = load_peaks()
+    wl_name = args.workload   # the workload a committed DRAM capture must come from
     K, Wm = args.steps, max(3, args.warmup)
     status = umim.new_status(dev)
 
@@ -1352,7 +1355,7 @@ def side_bench(args):
         top = max(measured, key=lambda k: kernels[k]["share"])
         b, amount, unit_r, peak = work_of[top]
         roof = {"kernel": top, "bound": b, "achieved": kernels[top]["achieved"], "peak": peak, "unit": unit_r,
-                "frac": kernels[top]["frac"], "traffic": traffic_from_profile(top),
+                "frac": kernels[top]["frac"], "traffic": traffic_from_profile(top, wl_name),
                 "algorithmic_per_launch": amount * (1e12 if unit_r == "TFLOP/s" else 1e9),
                 "peak_source": peaks["src"] + (" bf16 burst" if b == "tensor" else " HBM copy")}
     line = {"metric": metric, "value": units * K / (ms / 1000.0), "unit": unit, "n_gpus": 1, "steps": K,

@@ -52,8 +52,10 @@ def test_traffic_is_reported_only_for_unchanged_sources():
     for label, e in prof.items():
         src = os.path.join(ROOT, "paper_2609_27233_gb300", "csrc", e["source"])
         same = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16] == e["source_sha"]
-        got = bench.traffic_from_profile(label)
+        got = bench.traffic_from_profile(label, e["workload"])
         assert (got == e["bytes_per_launch_full"]) if same else got is None, label
+        # a capture is never reported for another workload's launch of the kernel
+        assert bench.traffic_from_profile(label, "another_workload") is None, label
     assert bench.traffic_from_profile("no.such.kernel") is None
 
 
