@@ -22,6 +22,9 @@ def _qkv(seed, T, hq, hkv, d, dv):
     (82, [17, 129, 300], 8, 2, 64, 5),                  # head_dim 64, unused rows past the last sequence
     (83, [1000], 4, 4, 128, 0),                          # one long sequence, G = 1
     (84, [5, 77, 3, 250], 28, 4, 128, 0),                # G = 7 (the long-context model)
+    # 32 query tiles x 32 heads = 1024 work units over 2 CTAs per SM: every CTA runs
+    # several units, so barriers and rings count across units (checked on every row)
+    (85, [1000, 1000, 700, 513, 300, 65, 1], 32, 8, 128, 0),
 ])
 def test_prefill_matches_oracle(seed, lens, hq, hkv, d, pad):
     m, dv = umim(), dev()
