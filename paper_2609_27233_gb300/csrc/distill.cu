@@ -914,14 +914,15 @@ CeKernel ce_kernel_for(int kv, int T, bool tail) {
   return T == 256 ? k256[tail][kv - 1] : k448[tail][kv - 1];
 }
 
-// 16-byte vectors per thread per row with T threads per CTA and C CTAs per row
+// 16-byte vectors per thread per row with T compute threads per CTA and C CTAs per row
 int ce_vecs(int64_t V, int T, int C) {
   const int64_t nvec = (V + 7) / 8;
   const int64_t chunk = (nvec + C - 1) / C;
   return (int)std::max<int64_t>(1, (chunk + T - 1) / T);
 }
 
-// How a call runs: T threads per CTA, C CTAs (one cluster) per student row.
+// How a call runs: T compute threads (plus the copy warp) per CTA, C CTAs
+// (one cluster) per student row, KV vectors of each row per thread.
 struct CeLayout {
   int T, C, kv, chunk_vecs, stage_vecs, stages;
   size_t smem;
@@ -1059,8 +1060,8 @@ umim_status distill_align(const int32_t *seq_lens, int32_t B, const int32_t *spa
 
 size_t distill_soft_ce_workspace_bytes(int R_S, int max_pairs) { return ce_ws_bytes(R_S, max_pairs); }
 
-// vectors per thread per row for a vocabulary (0: unsupported)
-// nonzero when the vocabulary is supported (at most 16 CTAs x 256 threads x 5 vectors x 8 values)
+// nonzero when the vocabulary is supported (at most 16 CTAs x 256 threads x 5 vectors x 8 values;
+// the 448-thread layouts cover the same range with at most 4 vectors)
 int distill_soft_ce_vecs(int64_t V) { return (V >= 1 && ce_vecs(V, 256, kCeMaxCluster) <= kCeMaxVecs) ? 1 : 0; }
 
 umim_status distill_soft_ce(const void *teacher, int32_t R_T, const void *student, int32_t R_S, int32_t V, int64_t ld,
