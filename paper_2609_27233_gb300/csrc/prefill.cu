@@ -9,7 +9,7 @@
 // tensor cores while the other's softmax runs), each walking work units of
 // 128 query rows of one sequence for one query head, heaviest first; the
 // next unit's Q and K loads and first S products overlap the current unit's
-// last tiles and epilogue.  Warp 0 loads tiles with TMA (Q once; 64-key K
+// last tiles and epilogue.  Warp 0 loads tiles with TMA (a unit's Q; 64-key K
 // tiles into a 2-stage ring running a tile ahead of the V^T tiles' 2-stage
 // ring), warp 1 issues the S = Q K^T products (tcgen05.mma into one of two
 // tensor-memory buffers, reused once the P V product that read it is done),
