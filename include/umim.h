@@ -69,10 +69,13 @@ typedef enum umim_status {
   UMIM_ERR_UNSUPPORTED = 2, /* shape outside the supported set above     */
   UMIM_ERR_CUDA = 3,        /* a CUDA runtime / driver call failed       */
   UMIM_ERR_TIMEOUT = 4,     /* a bounded device-side wait gave up        */
-  UMIM_ERR_WORKSPACE = 5    /* workspace pointer or size insufficient    */
+  UMIM_ERR_WORKSPACE = 5,   /* workspace pointer or size insufficient    */
+  UMIM_ERR_BOUNDS = 6       /* debug build only: an access-site check    */
+                            /* failed; the word holds 6 | site << 8      */
 } umim_status;
 
-/* Human-readable name of a status code (static string). */
+/* Human-readable name of a status code (static string); a debug build's
+ * UMIM_ERR_BOUNDS | site << 8 reads as "UMIM_ERR_BOUNDS". */
 const char *umim_status_string(int status);
 
 /* Library version as 10000*major + 100*minor + patch. */
@@ -663,6 +666,37 @@ umim_status umim_decode_attention_static(const void *q, int32_t n_q_heads, const
  * ------------------------------------------------------------------------ */
 umim_status umim_selftest_bounded_wait(int32_t which, uint32_t limit_us, const int32_t *flags,
                                        uint64_t *elapsed_ns, int32_t *dev_status, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Debug build (not part of the method).  libumim_debug.so is this library
+ * compiled with UMIM_DEBUG defined: every kernel also checks, where it loads
+ * or stores, that each index it computed from device data (a page from a
+ * block table, a row or offset from one of its own plans, a partial-result
+ * slot) lies inside the buffer it addresses.  A failed check records
+ * UMIM_ERR_BOUNDS | site << 8 in dev_status (first error wins), skips that
+ * access (a store is dropped, a load reads zeros) and the kernel carries
+ * on; the call's outputs are then unspecified.  These are checks of the
+ * library's own invariants: inputs are validated the same way in both
+ * builds, so on valid and invalid inputs alike a correct library never
+ * records UMIM_ERR_BOUNDS.  The calls and their results are otherwise
+ * identical to libumim.so's.
+ *
+ * umim_debug_build       1 in libumim_debug.so, 0 in libumim.so
+ * umim_debug_site_name   the name of the access site in bits 8.. of a status
+ *                        word ("" when there is none)
+ * umim_selftest_bounds_check
+ *                        one check of the mechanism: a kernel stores 1 into
+ *                        buf[index] if 0 <= index < n, through the same
+ *                        check as the other kernels' access sites.  buf is
+ *                        a device int32 [n].  With an index outside [0, n)
+ *                        the expected outcome is UMIM_ERR_BOUNDS | 1 << 8 in
+ *                        dev_status and buf unchanged.  In libumim.so it
+ *                        returns UMIM_ERR_UNSUPPORTED and launches nothing.
+ * ------------------------------------------------------------------------ */
+int umim_debug_build(void);
+const char *umim_debug_site_name(int32_t status);
+umim_status umim_selftest_bounds_check(int32_t *buf, int64_t n, int64_t index, int32_t *dev_status,
+                                       cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
  * Kernel tracing, for profiling (not part of the method).  Between

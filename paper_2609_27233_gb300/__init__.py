@@ -31,7 +31,8 @@ from ._lib import MergeWeightsC, PagedKVC
 
 UMIM_OK = 0
 STATUS = {0: "UMIM_OK", 1: "UMIM_ERR_INVALID_ARG", 2: "UMIM_ERR_UNSUPPORTED", 3: "UMIM_ERR_CUDA",
-          4: "UMIM_ERR_TIMEOUT", 5: "UMIM_ERR_WORKSPACE"}
+          4: "UMIM_ERR_TIMEOUT", 5: "UMIM_ERR_WORKSPACE", 6: "UMIM_ERR_BOUNDS"}
+UMIM_ERR_BOUNDS = 6   # debug build: the status word holds 6 | site << 8
 PAGE_SIZE = 16
 STATIC_SCRATCH_BYTES = 32 << 20   # UMIM_STATIC_SCRATCH_BYTES of include/umim.h
 
@@ -39,7 +40,18 @@ STATIC_SCRATCH_BYTES = 32 << 20   # UMIM_STATIC_SCRATCH_BYTES of include/umim.h
 class UmimError(RuntimeError):
     def __init__(self, code, where=""):
         self.code = int(code)
-        super().__init__(f"{where}: {STATUS.get(self.code, self.code)}")
+        self.site = ""
+        msg = STATUS.get(self.code, self.code)
+        if self.code & 0xff == UMIM_ERR_BOUNDS:   # the debug build's access-site checks
+            self.site = lib().umim_debug_site_name(self.code).decode()
+            msg = f"UMIM_ERR_BOUNDS at {self.site}"
+        super().__init__(f"{where}: {msg}")
+
+
+def use_debug_library(flag: bool = True) -> None:
+    """Run every later call on libumim_debug.so, the build whose kernels check
+    each index they compute at their access sites (or back on libumim.so)."""
+    _lib.use_debug(flag)
 
 
 def lib():
@@ -336,6 +348,25 @@ def umim_selftest_bounded_wait(which, limit_us, device, dev_status=None, stream=
                                             _stream(stream))
     _check(code, "umim_selftest_bounded_wait")
     return status, elapsed
+
+
+def umim_debug_build():
+    """1 when the active library is libumim_debug.so, else 0."""
+    return int(lib().umim_debug_build())
+
+
+def umim_debug_site_name(code):
+    """The access site named in bits 8.. of a debug build's status word."""
+    return lib().umim_debug_site_name(int(code)).decode()
+
+
+def umim_selftest_bounds_check(buf, index, dev_status=None, stream=None):
+    """Debug build only: store 1 into buf[index] (buf a device int32 tensor)
+    through the kernels' access-site check; returns the status tensor."""
+    status = new_status(buf.device) if dev_status is None else dev_status
+    code = lib().umim_selftest_bounds_check(_p(buf), int(buf.numel()), int(index), _p(status), _stream(stream))
+    _check(code, "umim_selftest_bounds_check")
+    return status
 
 
 def umim_rule_table_bytes(n_rules):

@@ -8,6 +8,7 @@ import os
 
 HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(HERE, "libumim.so")
+DEBUG_LIB_PATH = os.path.join(HERE, "libumim_debug.so")   # the same calls built with UMIM_DEBUG
 
 c_i32 = ctypes.c_int32
 c_i64 = ctypes.c_int64
@@ -79,27 +80,40 @@ SIGNATURES = {
                                              c_ptr]),
     "umim_decode_attention_static": (ctypes.c_int, [c_ptr, c_i32, ctypes.POINTER(PagedKVC), c_i32, c_ptr, c_i32,
                                                     c_ptr, c_i32, ctypes.c_float, c_ptr, c_ptr, c_ptr]),
+    "umim_debug_build": (ctypes.c_int, []),
+    "umim_debug_site_name": (ctypes.c_char_p, [c_i32]),
+    "umim_selftest_bounds_check": (ctypes.c_int, [c_ptr, c_i64, c_i64, c_ptr, c_ptr]),
     "umim_trace_start": (ctypes.c_int, [c_i32]),
     "umim_trace_stop": (None, []),
     "umim_trace_read": (c_i32, [ctypes.POINTER(ctypes.c_float), ctypes.POINTER(ctypes.c_char_p), c_i32]),
 }
 
-_lib = None
+_libs = {}
+_active = LIB_PATH
 
 
-def load(path: str = LIB_PATH):
-    """Load libumim.so and declare every entry point; raises if it is missing."""
-    global _lib
-    if _lib is not None:
-        return _lib
+def use_debug(flag: bool) -> None:
+    """Route every later call of the binding through libumim_debug.so (True)
+    or libumim.so (False, the default).  Both may be loaded at once."""
+    global _active
+    _active = DEBUG_LIB_PATH if flag else LIB_PATH
+
+
+def load(path: str = None):
+    """Load the active library (or `path`) and declare every entry point;
+    raises if it is missing."""
+    path = path or _active
+    lib = _libs.get(path)
+    if lib is not None:
+        return lib
     if not os.path.exists(path):
         raise RuntimeError(
-            f"libumim.so not found at {path}: build it first "
+            f"{os.path.basename(path)} not found at {path}: build it first "
             "(python -c 'import __graft_entry__ as g; g.build()')")
     lib = ctypes.CDLL(path)
     for name, (res, args) in SIGNATURES.items():
         fn = getattr(lib, name)
         fn.restype = res
         fn.argtypes = args
-    _lib = lib
+    _libs[path] = lib
     return lib

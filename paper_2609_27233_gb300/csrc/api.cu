@@ -56,6 +56,7 @@ umim_status match_suffix(const void *, size_t, void *, const int32_t *, int, int
 umim_status lookup_surrogates(const float *, int64_t, int, const int32_t *, int, const int32_t *, float *, int32_t *,
                               cudaStream_t, int);
 umim_status selftest_bounded_wait(int, uint32_t, const int32_t *, uint64_t *, int32_t *, cudaStream_t);
+umim_status selftest_bounds_check(int32_t *, int64_t, int64_t, int32_t *, cudaStream_t);
 size_t prefill_attention_workspace_bytes(int B, int T, int Hkv, int D);
 umim_status prefill_attention(const void *, const void *, const void *, int, int, int, int, const int32_t *, int,
                               float, void *, void *, int32_t *, cudaStream_t, int);
@@ -117,6 +118,7 @@ using namespace umim;
 extern "C" {
 
 const char *umim_status_string(int s) {
+  if ((s & 0xff) == UMIM_ERR_BOUNDS) return "UMIM_ERR_BOUNDS";
   switch (s) {
     case UMIM_OK: return "UMIM_OK";
     case UMIM_ERR_INVALID_ARG: return "UMIM_ERR_INVALID_ARG";
@@ -359,6 +361,47 @@ umim_status umim_selftest_bounded_wait(int32_t which, uint32_t limit_us, const i
   if (which == 1 && !flags) return UMIM_ERR_INVALID_ARG;
   const DeviceScope scope(stream);
   return selftest_bounded_wait(which, limit_us, flags, elapsed_ns, dev_status, stream);
+}
+
+int umim_debug_build(void) { return kDebugChecks ? 1 : 0; }
+
+const char *umim_debug_site_name(int32_t status) {
+  static const char *const names[kSiteCount] = {
+      "",
+      "selftest",
+      "rollback_map.block_table",
+      "rollback_move.dst_page",
+      "rollback_move.src",
+      "rollback_move.surrogate",
+      "rollback_move.reader_row",
+      "append.dst",
+      "append.src_row",
+      "attention.block_table",
+      "attention.piece",
+      "decode_step.block_table",
+      "decode_step.cache_write",
+      "decode_step.partial",
+      "merge.pool_stats",
+      "merge.gemm_store",
+      "merge.pool_span",
+      "compaction.token",
+      "prefill.kv_row",
+      "prefill.out_row",
+      "distill.teacher_row",
+      "distill.pair",
+      "rules.span_slot",
+      "rules.span_token",
+  };
+  const int site = (status >> 8) & 0xffffff;
+  return site < kSiteCount ? names[site] : "";
+}
+
+umim_status umim_selftest_bounds_check(int32_t *buf, int64_t n, int64_t index, int32_t *dev_status,
+                                       cudaStream_t stream) {
+  if (!kDebugChecks) return UMIM_ERR_UNSUPPORTED;   // nothing would stop the store: launch nothing
+  if (!buf || n <= 0) return UMIM_ERR_INVALID_ARG;
+  const DeviceScope scope(stream);
+  return selftest_bounds_check(buf, n, index, dev_status, stream);
 }
 
 size_t umim_prefill_attention_workspace_size(int32_t batch, int32_t n_rows, int32_t n_kv_heads, int32_t head_dim) {

@@ -109,6 +109,10 @@ __global__ void __launch_bounds__(kAppendThreads) decode_update_kernel(AppendArg
   const uint16_t *src_k = k > 0 ? a.sur_k : a.new_k;
   const uint16_t *src_v = k > 0 ? a.sur_v : a.new_v;
   const int src_row = k > 0 ? row : b;
+  if (!in_bounds(src_row, k > 0 ? a.n_rows : (int)gridDim.x / C, rank == 0 ? a.status : nullptr,
+                 kSiteAppendSrcRow))
+    return;
+  const int64_t pool_elems = layer_stride * a.n_layers;   // debug checks
   const int stride = kAppendThreads * C;
   for (int c0 = rank * kAppendThreads + threadIdx.x; c0 < total; c0 += stride * kUnroll) {
     uint4 v[kUnroll];
@@ -128,8 +132,9 @@ __global__ void __launch_bounds__(kAppendThreads) decode_update_kernel(AppendArg
       if (c < total) {
         const int r = c / CPR, col = c % CPR;
         const int layer = r / (2 * Hkv), kv = (r / Hkv) & 1, h = r % Hkv;
-        *reinterpret_cast<uint4 *>(dst_base + layer * layer_stride + kv * kv_stride + h * head_stride + col * 8) =
-            v[u];
+        const int64_t off = layer * layer_stride + kv * kv_stride + h * head_stride + col * 8;
+        if (in_bounds((dst_base - a.pool) + off, pool_elems - 7, a.status, kSiteAppendDst))
+          *reinterpret_cast<uint4 *>(dst_base + off) = v[u];
       }
     }
   }

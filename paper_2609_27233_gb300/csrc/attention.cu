@@ -229,7 +229,8 @@ __global__ void __launch_bounds__(kAttnWarps * 32, 1)
     while (pos >= ws.seg_off[ld_seg + 1]) ++ld_seg;
     const int b = ld_seg / a.Hkv, g = ld_seg % a.Hkv;
     const int pi = pos - ws.seg_off[ld_seg];
-    const int page = a.block_table[(int64_t)b * a.max_pages + pi];
+    const int page = in_bounds(pi, a.max_pages, a.status, kSiteAttnTable)
+                         ? a.block_table[(int64_t)b * a.max_pages + pi] : -1;
     int c4 = a.layer * a.n_pages + page;
     if (page < 0 || page >= a.n_pages) {
       // a coordinate past the tensor's last page: the copy reads zeros
@@ -281,6 +282,7 @@ __global__ void __launch_bounds__(kAttnWarps * 32, 1)
     s1 += __shfl_xor_sync(0xffffffffu, s1, 1);
     s1 += __shfl_xor_sync(0xffffffffu, s1, 2);
     const int piece = ws.piece_base[cseg] + (gw - ws.seg_off[cseg] / W);
+    if (!in_bounds(piece, nseg + (int64_t)gridDim.x * kAttnWarps, a.status, kSiteAttnPiece)) return;
     float2 *ml = ws.part_ml + (int64_t)piece * 16;
     float *pacc = ws.part_acc + (int64_t)piece * 16 * D;
     if (qc == 0) {

@@ -30,6 +30,63 @@ __device__ __forceinline__ int32_t read_status(const int32_t *status) {
   return *reinterpret_cast<const volatile int32_t *>(status);
 }
 
+// ---------------------------------------------------------------------------
+// debug build
+// ---------------------------------------------------------------------------
+// Compiled with -DUMIM_DEBUG (libumim_debug.so), the kernels check at their
+// access sites that every index they computed from device data lies inside the
+// buffer it addresses.  A failed check records UMIM_ERR_BOUNDS | site << 8 in
+// the call's status word (the first error wins, as for every code) and the
+// access is skipped: a store is dropped, a load yields zeros or reads an
+// in-bounds stand-in (where a copy must still complete a barrier).  These are
+// checks of the kernels' own invariants (the inputs are validated in both
+// builds); in the normal build every check is the constant true and
+// compiles to nothing.
+#ifdef UMIM_DEBUG
+constexpr bool kDebugChecks = true;
+#else
+constexpr bool kDebugChecks = false;
+#endif
+
+// check sites; umim_debug_site_name() gives their names
+enum DebugSite : int32_t {
+  kSiteSelftest = 1,
+  kSiteRollbackMapTable = 2,
+  kSiteRollbackDstPage = 3,
+  kSiteRollbackSrc = 4,
+  kSiteRollbackSurrogate = 5,
+  kSiteRollbackReaderRow = 6,
+  kSiteAppendDst = 7,
+  kSiteAppendSrcRow = 8,
+  kSiteAttnTable = 9,
+  kSiteAttnPiece = 10,
+  kSiteStepTable = 11,
+  kSiteStepCacheWrite = 12,
+  kSiteStepPartial = 13,
+  kSiteMergePoolStats = 14,
+  kSiteMergeGemmStore = 15,
+  kSiteMergePoolSpan = 16,
+  kSiteCompactToken = 17,
+  kSitePrefillKvRow = 18,
+  kSitePrefillOutRow = 19,
+  kSiteDistillTeacherRow = 20,
+  kSiteDistillPair = 21,
+  kSiteRulesSpanSlot = 22,
+  kSiteRulesSpanToken = 23,
+  kSiteCount = 24
+};
+
+// true when 0 <= i < n; in the debug build a false result is recorded
+__device__ __forceinline__ bool in_bounds(int64_t i, int64_t n, int32_t *status, DebugSite site) {
+  if constexpr (!kDebugChecks) {
+    return true;
+  } else {
+    const bool ok = (uint64_t)i < (uint64_t)n;
+    if (!ok) set_error(status, UMIM_ERR_BOUNDS | ((int32_t)site << 8));
+    return ok;
+  }
+}
+
 __device__ __forceinline__ uint64_t globaltimer() {
   uint64_t t;
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));

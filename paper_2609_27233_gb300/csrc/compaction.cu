@@ -68,8 +68,9 @@ __global__ void __launch_bounds__(256) compact_kernel(CompactArgs a, PlanArrays 
       }
     } else {
       const int t = (i >= lo) ? j + arr.r_incl[i] : j;
-      const int id = a.token_ids[(int64_t)b * a.L + t];
-      const bool ok = id >= 0 && id < a.vocab;
+      const bool t_ok = in_bounds(t, a.L, lane == 0 ? a.status : nullptr, kSiteCompactToken);
+      const int id = t_ok ? a.token_ids[(int64_t)b * a.L + t] : 0;
+      const bool ok = id >= 0 && id < a.vocab && t_ok;
       if (!ok && lane == 0) set_error(a.status, UMIM_ERR_INVALID_ARG);
       const uint4 *src = a.table + (int64_t)(ok ? id : 0) * vec;
       for (int v = lane; v < vec; v += 32) dst[v] = ok ? __ldg(src + v) : make_uint4(0, 0, 0, 0);

@@ -265,7 +265,8 @@ __global__ void __launch_bounds__(kStepThreads, 1)
       if (lst.slot >= 0 && lpi == lst.slot / kPageSize && lst.slot % kPageSize == 0) {
         mbar_arrive(bar);   // only the new entry in this unit: nothing to copy
       } else {
-        const int page = a.block_table[(int64_t)lb * a.max_pages + lpi];
+        const int page = in_bounds(lpi, a.max_pages, a.status, kSiteStepTable)
+                             ? a.block_table[(int64_t)lb * a.max_pages + lpi] : -1;
         int c4 = a.layer * a.n_pages + page;
         if (page < 0 || page >= a.n_pages) {
           set_error(a.status, UMIM_ERR_INVALID_ARG);   // a coordinate past the last page reads zeros
@@ -370,6 +371,7 @@ __global__ void __launch_bounds__(kStepThreads, 1)
       old = __shfl_sync(0xffffffffu, old, 0);
       const int w0 = o / W, w1 = (o + n - 1) / W;
       if (old != w1 - w0) return;   // another warp of the segment is still running
+      if (!in_bounds(w1, (int64_t)gridDim.x * kStepWarps, a.status, kSiteStepPartial)) return;
       // last to finish: merge the segment's partials (warp w0 used slot 1
       // unless the segment starts its range; every later warp used slot 0),
       // several pieces' loads in flight at a time
@@ -463,9 +465,11 @@ __global__ void __launch_bounds__(kStepThreads, 1)
                            : (isv ? a.new_v : a.new_k) + (int64_t)cb * a.new_stride + (int64_t)cg * D;
           const uint4 v = ld_nc_v4(src + c * 8);
           *reinterpret_cast<uint4 *>((isv ? vt : kt) + sw_off(r, c)) = v;
-          uint16_t *dst = a.pool + ((((int64_t)a.layer * a.n_pages + cst.page) * 2 + isv) * Hkv + cg) * (16 * D) +
-                          (int64_t)r * D + c * 8;
-          *reinterpret_cast<uint4 *>(dst) = v;
+          const int64_t off = ((((int64_t)a.layer * a.n_pages + cst.page) * 2 + isv) * Hkv + cg) * (16 * D) +
+                              (int64_t)r * D + c * 8;
+          if (in_bounds(off, (int64_t)a.n_layers * a.n_pages * 2 * Hkv * 16 * D - 7, a.status,
+                        kSiteStepCacheWrite))
+            *reinterpret_cast<uint4 *>(a.pool + off) = v;
         }
       }
       if (nvalid < 16) {

@@ -617,7 +617,9 @@ __global__ void __launch_bounds__(T + 32, 1) ce_kernel(CeArgs a) {
         mbar_arrive_expect_tx(&full_bar[s], tx_bytes);
         if (vcnt > 0) {
           uint4 *dst = stage_base + (size_t)s * 2 * SV;
-          bulk_load(dst, a.teacher + (int64_t)ct * a.ld + (int64_t)vbeg * 8, (uint32_t)vcnt * 16u, &full_bar[s], pol);
+          const int ctl = in_bounds(ct, a.R_T, a.status, kSiteDistillTeacherRow) ? ct : 0;
+          bulk_load(dst, a.teacher + (int64_t)ctl * a.ld + (int64_t)vbeg * 8, (uint32_t)vcnt * 16u, &full_bar[s],
+                    pol);
           bulk_load(dst + SV, a.student + (int64_t)cw * a.ld + (int64_t)vbeg * 8, (uint32_t)vcnt * 16u, &full_bar[s],
                     pol);
         }
@@ -653,7 +655,8 @@ __global__ void __launch_bounds__(T + 32, 1) ce_kernel(CeArgs a) {
       }
       for (int j = lane + 128; j < nx; j += 32) LA = __fadd2_rn(LA, *reinterpret_cast<const float2 *>(&xbuf[1][xb][j]));
       LA = warp_sum2(LA);   // (-sum P^T log2(P^S + eps), -A), both / N
-      if (rank == 0 && tid == 0) a.pair_loss[prev_p] = LA.x * kLn2 * (float)N;
+      if (rank == 0 && tid == 0 && in_bounds(prev_p, N, a.status, kSiteDistillPair))
+        a.pair_loss[prev_p] = LA.x * kLn2 * (float)N;
       if (prev_grow) {
         const float2 A2 = make_float2(-LA.y, -LA.y);
         tmem_wait_st();

@@ -256,7 +256,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         mean += delta * (32.f / nt);
         m2 += cm2 + delta * delta * (cnt * 32.f / nt);
         cnt = nt;
-        if (row < g.M) store32(g.out + (int64_t)row * g.N + n0 + c * 32, v);
+        if (row < g.M && in_bounds(n0 + c * 32 + 31, g.N, g.status, kSiteMergeGemmStore))
+          store32(g.out + (int64_t)row * g.N + n0 + c * 32, v);
       }
       if (row < g.M) g.stats[(int64_t)row * tiles_n + n0 / BN] = make_float2(mean, m2);
       if (bad && row < g.M) flag_range(g.range_flag, g.status);   // this row's fp16 output overflowed
@@ -812,6 +813,7 @@ __global__ void __launch_bounds__(kHeadWarps * 32, 1)
       if (head == 0) set_error(status, UMIM_ERR_INVALID_ARG);
       n = 0;
     }
+    if (n > 0 && !in_bounds((int64_t)t1 * ntiles - 1, T * ntiles, status, kSiteMergePoolStats)) n = 0;
     if (n == 0) {
       mbar_arrive(bar);
       return 0;
@@ -852,7 +854,7 @@ __global__ void __launch_bounds__(kHeadWarps * 32, 1)
     const float2 *ts = reinterpret_cast<const float2 *>(wbuf + b * buf_bytes + UMIM_MAX_SPAN_TOKENS * dh * 2);
     uint32_t bad = 0;
     __half *orow = O + (int64_t)sp * d + (int64_t)head * dh;
-    switch (n) {
+    if (in_bounds(sp, S, status, kSiteMergePoolSpan)) switch (n) {
       case 1: bad = pool_item<CPL, 1>(hs, ts, gq, gp, bp, A, Bq, lane, Ch, dh, ntiles, inv_ntiles, inv_d, eps,
                                       inv_sqrt_dh, orow); break;
       case 2: bad = pool_item<CPL, 2>(hs, ts, gq, gp, bp, A, Bq, lane, Ch, dh, ntiles, inv_ntiles, inv_d, eps,

@@ -353,6 +353,10 @@ __global__ void __launch_bounds__(kPfThreads, 2)
       int k_unit = 0;
       for (int u = (int)blockIdx.x; u < n_units && ok; u += G, ++k_unit) {
         const Unit w = unit_of(u);
+        // the unit's last K row and V^T column (a TMA copy past the end of
+        // its tensor reads zeros, so these checks only record)
+        (void)in_bounds((int64_t)w.s0 + (w.n_kv - 1) * kPfKeys, a.T, a.status, kSitePrefillKvRow);
+        (void)in_bounds(w.kbase + (int64_t)(w.n_kv - 1) * kPfKeys, a.Tp, a.status, kSitePrefillKvRow);
         // Q of the previous unit has been read by its last S product
         if (k_unit > 0 && (aborted() || !mbar_wait(&q_empty, (uint32_t)(k_unit - 1) & 1u))) {
           ok = false;
@@ -579,7 +583,7 @@ __global__ void __launch_bounds__(kPfThreads, 2)
       for (int c = 0; c < D / 32; ++c) {
         float o[32];
         tmem_ld_32x32b_x32(t_o + c * 32, o);
-        if (qpos < w.len) {
+        if (qpos < w.len && in_bounds((int64_t)w.s0 + qpos, a.T, a.status, kSitePrefillOutRow)) {
           uint4 *dst = reinterpret_cast<uint4 *>(orow + c * 32);
 #pragma unroll
           for (int e = 0; e < 4; ++e)

@@ -134,7 +134,7 @@ __global__ void __launch_bounds__(256) rollback_map_kernel(MoveArgs a, PlanArray
           src = -(int64_t)i - 1;
         } else {
           const int t = j + arr.r_incl[i];
-          if (t != j) {
+          if (t != j && in_bounds(t / kPageSize, a.max_pages, a.status, kSiteRollbackMapTable)) {
             src = (int64_t)bt[t / kPageSize] * page_stride + (t % kPageSize) * D;
             shift = t - j;
           }
@@ -213,6 +213,7 @@ __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs
   // unit indices fit in 32 bits: batch x max_pages x tile lanes < 2^30 is checked on the host
   const int max_dest = total > 0 ? hdr->max_dest : 0;
   const int n_slots = max_dest * row_size;
+  const int n_rows = total / a.n_lanes;   // compacted rows of all sequences (debug checks)
 
   // plan values of the active sequences (row position order), from shared
   // memory when there are few enough of them
@@ -268,6 +269,10 @@ __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs
     m.valid = 1;
     m.tl = tl;
     m.idx = row0_of(j) + kk;
+    if (!in_bounds(m.idx, n_rows, a.status, kSiteRollbackReaderRow)) {
+      m.valid = 0;
+      return;
+    }
     m.my_src = lane < kPageSize ? pd.src[(int64_t)m.idx * kPageSize + lane] : kNoWrite;
     m.page = a.block_table[(int64_t)b * a.max_pages + fp_of(j) + kk];
     m.shift = (ROPE && lane < kPageSize) ? pd.shift[(int64_t)m.idx * kPageSize + lane] : 0;
@@ -314,14 +319,23 @@ __global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs
       const int64_t src = __shfl_sync(0xffffffffu, m.my_src, slot);
       if (src != kNoWrite) t.mask |= 1u << it;
       if (src >= 0) {
-        t.v[it] = ld_v4(a.pool + tile + src);
+        if (in_bounds(src, (int64_t)a.n_pages * page_stride32, a.status, kSiteRollbackSrc))
+          t.v[it] = ld_v4(a.pool + tile + src);
       } else if (src != kNoWrite) {
         const int64_t si = -src - 1;
-        t.v[it] = ld_v4(sur + (si * a.n_layers * Hkv + lh) * D + my_col * 8);
+        if (in_bounds(si, kDebugChecks ? a.span_offsets[a.B] : 0, a.status, kSiteRollbackSurrogate))
+          t.v[it] = ld_v4(sur + (si * a.n_layers * Hkv + lh) * D + my_col * 8);
       }
     }
     t.dlo = m.dep.lo;
     t.dhi = m.dep.hi;
+    if (!in_bounds(m.page, a.n_pages, a.status, kSiteRollbackDstPage)) t.mask = 0;
+    if (t.dlo <= t.dhi && !(in_bounds(t.dlo, n_rows, a.status, kSiteRollbackReaderRow) &&
+                            in_bounds(t.dhi, n_rows, a.status, kSiteRollbackReaderRow))) {
+      t.dlo = 1;   // no reader row to wait for, so nothing may be stored either
+      t.dhi = 0;
+      t.mask = 0;
+    }
   };
   auto store = [&](const Tile &t) {
 #pragma unroll

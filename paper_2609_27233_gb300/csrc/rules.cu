@@ -365,9 +365,12 @@ __global__ void __launch_bounds__(kWalkThreads) prompt_walk_kernel(MatchArgs a, 
       const int n = m[q];
       if (n >= 2) {
         const int p = base + tid * kSeg + q;
-        w.sp_start[sbase + out] = p;
-        w.sp_len[sbase + out] = n;
-        w.sp_rule[sbase + out] = w.mrule[row + p];
+        if (in_bounds(out, span_stride(a.L), a.status, kSiteRulesSpanSlot) &&
+            in_bounds(p, Lb, a.status, kSiteRulesSpanSlot)) {
+          w.sp_start[sbase + out] = p;
+          w.sp_len[sbase + out] = n;
+          w.sp_rule[sbase + out] = w.mrule[row + p];
+        }
         ++out;
         q += n;
       } else {
@@ -469,7 +472,8 @@ __global__ void __launch_bounds__(256) span_compact_kernel(MatchArgs a, MatchWs 
       if (i < n) {
         const int t0 = tcarry + before + incl - ln;
         a.merge_offsets[base + i] = t0;
-        for (int k = 0; k < ln; ++k) a.merge_tokens[t0 + k] = a.tokens[(int64_t)b * a.L + st + k];
+        if (ln > 0 && in_bounds(st + ln - 1, a.L, a.status, kSiteRulesSpanToken))
+          for (int k = 0; k < ln; ++k) a.merge_tokens[t0 + k] = a.tokens[(int64_t)b * a.L + st + k];
       }
       tcarry += total;
       __syncthreads();

@@ -26,7 +26,18 @@ __global__ void selftest_wait_kernel(int which, uint64_t limit_ns, const int32_t
   if (!ok) set_error(status, UMIM_ERR_TIMEOUT);
 }
 
+__global__ void selftest_bounds_kernel(int32_t *buf, int64_t n, int64_t index, int32_t *status) {
+  if (in_bounds(index, n, status, kSiteSelftest)) buf[index] = 1;
+}
+
 }  // namespace
+
+umim_status selftest_bounds_check(int32_t *buf, int64_t n, int64_t index, int32_t *status, cudaStream_t stream) {
+  // without the check the store would go wherever index points
+  if (!kDebugChecks) return UMIM_ERR_UNSUPPORTED;
+  selftest_bounds_kernel<<<1, 1, 0, stream>>>(buf, n, index, status);
+  return cudaGetLastError() == cudaSuccess ? UMIM_OK : UMIM_ERR_CUDA;
+}
 
 umim_status selftest_bounded_wait(int which, uint32_t limit_us, const int32_t *flags, uint64_t *elapsed,
                                   int32_t *status, cudaStream_t stream) {

@@ -20,12 +20,14 @@ def declared_functions():
     return names
 
 
-@pytest.fixture(scope="module")
-def lib():
+@pytest.fixture(scope="module", params=["release", "debug"])
+def lib(request):
+    """Each test below runs on libumim.so and on libumim_debug.so (UMIM_DEBUG)."""
     from paper_2609_27233_gb300 import build, _lib
-    if not os.path.exists(_lib.LIB_PATH):
-        build.build()
-    return _lib.load()
+    path = _lib.LIB_PATH if request.param == "release" else _lib.DEBUG_LIB_PATH
+    if not os.path.exists(path):
+        build.build(variants=(request.param,))
+    return _lib.load(path)
 
 
 def test_header_declares_the_four_calls():
@@ -47,6 +49,47 @@ def test_status_strings_and_version(lib):
     assert lib.umim_status_string(0) == b"UMIM_OK"
     assert lib.umim_status_string(4) == b"UMIM_ERR_TIMEOUT"
     assert lib.umim_version() >= 100
+
+
+def test_debug_build_flag_and_status_words(lib, request):
+    """The two builds say which they are; a debug build's UMIM_ERR_BOUNDS word
+    carries the access site in bits 8 and up, and the release build refuses
+    the bounds self-test without launching anything (no check would stop its
+    store there)."""
+    debug = request.node.callspec.params["lib"] == "debug"
+    assert lib.umim_debug_build() == (1 if debug else 0)
+    assert lib.umim_status_string(6) == b"UMIM_ERR_BOUNDS"
+    assert lib.umim_status_string(6 | (3 << 8)) == b"UMIM_ERR_BOUNDS"
+    assert lib.umim_debug_site_name(6 | (1 << 8)) == b"selftest"
+    assert lib.umim_debug_site_name(6 | (3 << 8)) == b"rollback_move.dst_page"
+    assert lib.umim_debug_site_name(6 | (23 << 8)) == b"rules.span_token"
+    assert lib.umim_debug_site_name(6) == b""
+    assert lib.umim_debug_site_name(6 | (999 << 8)) == b""
+    null = ctypes.c_void_p(0)
+    if debug:
+        assert lib.umim_selftest_bounds_check(null, 4, 0, null, null) == 1        # no buffer
+        assert lib.umim_selftest_bounds_check(ctypes.c_void_p(1 << 20), 0, 0, null, null) == 1   # empty
+    else:
+        assert lib.umim_selftest_bounds_check(ctypes.c_void_p(1 << 20), 4, 9, null, null) == 2
+
+
+def test_every_site_of_the_kernels_has_a_name():
+    """The site numbers the kernels record and the names the library gives
+    them come from one enumeration, each name used once."""
+    csrc = os.path.join(ROOT, "paper_2609_27233_gb300", "csrc")
+    common = open(os.path.join(csrc, "common.cuh")).read()
+    sites = dict((m.group(1), int(m.group(2))) for m in re.finditer(r"(kSite\w+) = (\d+)", common))
+    count = sites.pop("kSiteCount")
+    assert sorted(sites.values()) == list(range(1, count))
+    used = set()
+    for f in os.listdir(csrc):
+        if f.endswith(".cu"):
+            used |= set(re.findall(r"in_bounds\([^;]*?(kSite\w+)\)", open(os.path.join(csrc, f)).read(), flags=re.S))
+    assert used == set(sites), set(sites) ^ used
+    api = open(os.path.join(csrc, "api.cu")).read()
+    names = re.search(r"names\[kSiteCount\] = \{(.*?)\};", api, flags=re.S).group(1)
+    names = re.findall(r'"([^"]*)"', names)
+    assert len(names) == count and names[0] == "" and len(set(names)) == count
 
 
 def test_workspace_sizes_are_positive(lib):
