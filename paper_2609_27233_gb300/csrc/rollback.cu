@@ -7,9 +7,8 @@
 // from surrogate rows, and it is written to the same physical page that held
 // old page j / 16.  Units are numbered row by row (row = compacted page
 // index, over the sequences that have pages to write) and dealt round-robin
-// to the mover warps of a cooperative grid; each warp loads two units ahead
-// of its stores (through shared memory with the copy engine when keys move
-// verbatim, through registers when they are re-rotated).  A unit may overwrite its page once every unit that reads
+// to the mover warps of a cooperative grid; each warp copies two units ahead
+// of its stores, through shared memory with the copy engine.  A unit may overwrite its page once every unit that reads
 // that old page has its loads landed.  Because j <= t, the readers of old
 // page p are the units of the same sequence at compacted rows whose entries
 // come from p: at most two rows, both at or before p's own row (a unit reads
@@ -28,8 +27,6 @@
 namespace umim {
 namespace {
 
-constexpr int kMoveThreads = 256;   // 8 mover warps
-constexpr int kMovers = kMoveThreads / 32;
 constexpr int64_t kNoWrite = INT64_MIN;
 
 struct MoveArgs {
@@ -47,7 +44,6 @@ struct MoveArgs {
   int32_t *status;
   const float *rope_inv_freq;   // [rotary_dim / 2] or nullptr: keys move verbatim
   int32_t rotary_dim;
-  uint32_t zero;                // always 0 (see red_add_after)
 };
 
 // largest i in [lo, hi) with key(i) <= x, or lo - 1
@@ -59,31 +55,6 @@ __device__ __forceinline__ int upper_index(const int32_t *key, int lo, int hi, i
     else h = m;
   }
   return l - 1;
-}
-
-__device__ __forceinline__ uint4 ld_v4(const uint16_t *p) {
-  uint4 v;
-  asm volatile("ld.global.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
-               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-               : "l"(p));
-  return v;
-}
-
-__device__ __forceinline__ void st_v4(uint16_t *p, uint4 v) {
-  asm volatile("st.global.v4.u32 [%0], {%1, %2, %3, %4};" ::"l"(p), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
-               : "memory");
-}
-
-// Adds 1 + (dep & zero) to *p, zero being 0 at run time (a kernel argument,
-// so the compiler cannot drop the term): the add depends on `dep`, a fold of
-// the unit's loaded data, so it cannot issue before those loads have returned
-// their values, and a load that has returned cannot be changed by a store that
-// follows the add -- which is all the page's writer relies on.  No release
-// fence: this thread's earlier stores (of another unit) need not be visible to
-// the waiter, and a fence would stall the warp until they are.
-__device__ __forceinline__ void red_add_after(int32_t *p, uint32_t dep, uint32_t zero) {
-  const int32_t v = 1 + (int32_t)(dep & zero);
-  asm volatile("red.relaxed.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
 }
 
 __device__ __forceinline__ int32_t ld_relaxed(const int32_t *p) {
@@ -211,336 +182,20 @@ __device__ __forceinline__ bool wait_landed(const int32_t *cnt, int target, cons
   return wait_count_for(cnt, target, abort, kWaitLimitNs);
 }
 
-// Mover warps: lane l moves 16-byte chunks c = l + 32 it of a unit, row
-// (slot) c / CPR, column c % CPR.  Step: the next unit's loads land and it is
-// counted in; this unit waits for its page's readers and is stored; the unit
-// after next is loaded into its registers.
-template <int D, bool ROPE>
-__global__ void __launch_bounds__(kMoveThreads, 2) rollback_move_kernel(MoveArgs a, PlanArrays arr, PageDesc pd) {
-  constexpr int CPR = D / 8;                       // 16-byte chunks per row
-  constexpr int PER_LANE = kPageSize * CPR / 32;   // 8 (D=128) or 4 (D=64)
-  constexpr int SLOT_STEP = 32 / CPR;              // rows advanced per it
-  constexpr int kHead = kPageSize * D;             // elements of one (K|V, head) tile
-  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-  const int nm = gridDim.x * kMovers;
-  const int my_col = lane % CPR;
-  const int my_slot0 = lane / CPR;
-  __shared__ int s_last;
-  __shared__ int s_sq[kSmemSeqs], s_nd[kSmemSeqs], s_ub[kSmemSeqs], s_fp[kSmemSeqs];
-  // per tile lane tl: its offset within a page (layer, K|V and head), and layer * Hkv + head | K|V << 31
-  __shared__ int64_t s_toff[kSmemLanes];
-  __shared__ int32_t s_tlh[kSmemLanes];
-  __shared__ float s_w[ROPE ? D / 2 : 1];   // RoPE angular frequencies
-
-  if (ROPE)
-    for (int i = threadIdx.x; i < a.rotary_dim / 2; i += blockDim.x) s_w[i] = a.rope_inv_freq[i];
-  griddep_wait();
-  const PlanHeader *hdr = arr.hdr;
-  int32_t *abort_flag = &arr.hdr->ticket;
-  const int total = hdr->total_units;
-  const int Hkv = a.n_kv_heads;
-  const int64_t layer_stride = (int64_t)2 * kHead * Hkv * a.n_pages;
-  const int kv_stride32 = kHead * Hkv, page_stride32 = 2 * kHead * Hkv;
-  // a row holds the units of the sequences that have pages to write
-  const int n_active = total > 0 ? hdr->n_active : 0;
-  const int row_size = max(1, n_active * a.n_lanes);
-  // unit indices fit in 32 bits: batch x max_pages x tile lanes < 2^30 is checked on the host
-  const int max_dest = total > 0 ? hdr->max_dest : 0;
-  const int n_slots = max_dest * row_size;
-  const int n_rows = total / a.n_lanes;   // compacted rows of all sequences (debug checks)
-
-  // plan values of the active sequences (row position order), from shared
-  // memory when there are few enough of them
-  const bool seq_in_smem = n_active <= kSmemSeqs;
-  if (seq_in_smem) {
-    for (int j = threadIdx.x; j < n_active; j += blockDim.x) {
-      const int b = arr.active[j];
-      s_sq[j] = b;
-      s_nd[j] = arr.n_dest[b];
-      s_ub[j] = arr.unit_base[b] / a.n_lanes;   // the sequence's first row
-      s_fp[j] = arr.first_page[b];
-    }
-  }
-  const bool lanes_in_smem = a.n_lanes <= kSmemLanes;
-  if (lanes_in_smem) {
-    for (int tl = threadIdx.x; tl < a.n_lanes; tl += blockDim.x) {
-      const int layer = tl / (2 * Hkv), kv = (tl / Hkv) & 1, h = tl % Hkv;
-      s_toff[tl] = layer * layer_stride + (int)(kv * kv_stride32 + h * kHead);
-      s_tlh[tl] = (int32_t)((uint32_t)(layer * Hkv + h) | ((uint32_t)kv << 31));
-    }
-  }
-  __syncthreads();
-  auto seq_of = [&](int j) { return seq_in_smem ? s_sq[j] : arr.active[j]; };
-  auto nd_of = [&](int j) { return seq_in_smem ? s_nd[j] : arr.n_dest[arr.active[j]]; };
-  auto row0_of = [&](int j) { return seq_in_smem ? s_ub[j] : arr.unit_base[arr.active[j]] / a.n_lanes; };
-  auto fp_of = [&](int j) { return seq_in_smem ? s_fp[j] : arr.first_page[arr.active[j]]; };
-
-  // a unit in registers, with where it goes and what it waits for
-  struct Tile {
-    uint4 v[PER_LANE];
-    uint32_t mask;
-    int valid, rot;     // rot: a K tile whose moved entries get re-rotated
-    int64_t dst;
-    int32_t row, dlo, dhi;
-    int32_t seen;       // the reader rows' smallest landed count when the unit was loaded
-    int32_t shift;      // lanes < 16: the shift of slot `lane`
-  };
-  // A unit's descriptors (its 16 sources, its page, its reader rows), read
-  // one unit ahead of its data loads so that the two round trips overlap.
-  struct Meta {
-    int64_t my_src;   // lanes < 16: the source of slot `lane`
-    int32_t valid, idx, page, tl;
-    int32_t shift;
-    RowDep dep;
-  };
-  // slot i = kk * row_size + j * n_lanes + tl: kk the compacted page row, j the
-  // active sequence, tl the tile lane
-  auto fetch = [&](int kk, int j, int tl, Meta &m) {
-    m.valid = 0;
-    if (kk >= max_dest) return;
-    if (kk >= nd_of(j)) return;
-    const int b = seq_of(j);
-    m.valid = 1;
-    m.tl = tl;
-    m.idx = row0_of(j) + kk;
-    if (!in_bounds(m.idx, n_rows, a.status, kSiteRollbackReaderRow)) {
-      m.valid = 0;
-      return;
-    }
-    m.my_src = lane < kPageSize ? pd.src[(int64_t)m.idx * kPageSize + lane] : kNoWrite;
-    m.page = a.block_table[(int64_t)b * a.max_pages + fp_of(j) + kk];
-    m.shift = (ROPE && lane < kPageSize) ? pd.shift[(int64_t)m.idx * kPageSize + lane] : 0;
-    m.dep = pd.dep[m.idx];
-  };
-  auto load = [&](const Meta &m, Tile &t) {
-    t.mask = 0;
-    t.valid = 0;
-    t.rot = 0;
-    t.shift = 0;
-    t.dst = 0;
-    t.row = 0;
-    t.dlo = 1;
-    t.dhi = 0;
-    t.seen = a.n_lanes;
-#pragma unroll
-    for (int it = 0; it < PER_LANE; ++it) t.v[it] = make_uint4(0, 0, 0, 0);
-    if (!m.valid) return;
-    const int tl = m.tl;
-    int64_t tile;
-    int kv, lh;   // lh = layer * Hkv + head
-    if (lanes_in_smem) {
-      tile = s_toff[tl] + my_col * 8;
-      const int32_t e = s_tlh[tl];
-      kv = (int)((uint32_t)e >> 31);
-      lh = e & 0x7fffffff;
-    } else {
-      const int layer = tl / (2 * Hkv), h = tl % Hkv;
-      kv = (tl / Hkv) & 1;
-      lh = layer * Hkv + h;
-      tile = layer * layer_stride + (int)(kv * kv_stride32 + h * kHead + my_col * 8);
-    }
-    const uint16_t *sur = kv ? a.sur_v : a.sur_k;
-    t.valid = 1;
-    t.row = m.idx;
-    t.dst = tile + (int64_t)m.page * page_stride32;
-    if (ROPE) {
-      t.rot = kv == 0;
-      t.shift = m.shift;
-    }
-#pragma unroll
-    for (int it = 0; it < PER_LANE; ++it) {
-      const int slot = my_slot0 + it * SLOT_STEP;
-      const int64_t src = __shfl_sync(0xffffffffu, m.my_src, slot);
-      if (src != kNoWrite) t.mask |= 1u << it;
-      if (src >= 0) {
-        if (in_bounds(src, (int64_t)a.n_pages * page_stride32, a.status, kSiteRollbackSrc))
-          t.v[it] = ld_v4(a.pool + tile + src);
-      } else if (src != kNoWrite) {
-        const int64_t si = -src - 1;
-        if (in_bounds(si, kDebugChecks ? a.span_offsets[a.B] : 0, a.status, kSiteRollbackSurrogate))
-          t.v[it] = ld_v4(sur + (si * a.n_layers * Hkv + lh) * D + my_col * 8);
-      }
-    }
-    t.dlo = m.dep.lo;
-    t.dhi = m.dep.hi;
-    if (!in_bounds(m.page, a.n_pages, a.status, kSiteRollbackDstPage)) t.mask = 0;
-    if (t.dlo <= t.dhi && !(in_bounds(t.dlo, n_rows, a.status, kSiteRollbackReaderRow) &&
-                            in_bounds(t.dhi, n_rows, a.status, kSiteRollbackReaderRow))) {
-      t.dlo = 1;   // no reader row to wait for, so nothing may be stored either
-      t.dhi = 0;
-      t.mask = 0;
-    }
-  };
-  auto store = [&](const Tile &t) {
-#pragma unroll
-    for (int it = 0; it < PER_LANE; ++it) {
-      const int slot = my_slot0 + it * SLOT_STEP;
-      if (t.mask & (1u << it)) st_v4(a.pool + t.dst + slot * D, t.v[it]);
-    }
-  };
-  // the unit's loads have arrived; count it into its row
-  auto land_and_count = [&](Tile &t) {
-    uint32_t fold = 0;
-#pragma unroll
-    for (int it = 0; it < PER_LANE; ++it) fold ^= t.v[it].x ^ t.v[it].y ^ t.v[it].z ^ t.v[it].w;
-    // every lane's loads have returned once lane 0 holds the fold of all of them
-#pragma unroll
-    for (int o = 16; o >= 1; o >>= 1) fold ^= __shfl_xor_sync(0xffffffffu, fold, o);
-    if (t.valid && lane == 0) red_add_after(&pd.dep[t.row].landed, fold, a.zero);
-    // the reader rows' counts, read a step before the store so that their
-    // latency overlaps this step; a complete count then needs no further wait
-    t.seen = a.n_lanes;
-    for (int rw = t.dlo; rw <= t.dhi; ++rw) t.seen = min(t.seen, ld_relaxed(&pd.dep[rw].landed));
-  };
-  // RoPE: a moved key (shift r) is rotated by -r w_m on the pairs (m, m + rotary_dim/2):
-  // x' = x cos + y sin, y' = y cos - x sin.  The lane holding chunk c of a slot's
-  // row takes its partner chunk from the lane holding c +- rotary_dim/16.  The
-  // angle is r w rounded plus its exact rounding error (an fma), the error
-  // folded into the sine and cosine to first order; the rounded angle is
-  // reduced to [-pi, pi] (Cody and Waite's three-part reduction) for the
-  // hardware sine and cosine, whose error there (about 2^-21) is far below
-  // the bf16 result's resolution.
-  auto rotate = [&](Tile &t) {
-    if (!ROPE || !t.rot) return;
-    const int hc = a.rotary_dim / 16;   // 16-byte chunks in each half of the rotated columns
-    const bool in_x = my_col < hc, in_y = my_col >= hc && my_col < 2 * hc;
-    const int partner = lane - my_col + (in_x ? my_col + hc : (in_y ? my_col - hc : my_col));
-    const int m0 = (in_x || in_y) ? 8 * (in_x ? my_col : my_col - hc) : 0;   // lanes past rotary_dim: unused
-    const int mine = in_y ? 1 : 0;   // of each element pair (2q, 2q+1) this lane evaluates element 2q + mine
-#pragma unroll
-    for (int it = 0; it < PER_LANE; ++it) {
-      const int slot = my_slot0 + it * SLOT_STEP;
-      const float rf = (float)__shfl_sync(0xffffffffu, t.shift, slot);   // 0: the identity (same bytes)
-      uint4 pv;
-      pv.x = __shfl_sync(0xffffffffu, t.v[it].x, partner);
-      pv.y = __shfl_sync(0xffffffffu, t.v[it].y, partner);
-      pv.z = __shfl_sync(0xffffffffu, t.v[it].z, partner);
-      pv.w = __shfl_sync(0xffffffffu, t.v[it].w, partner);
-      // the x and y lanes of a pair need the same angles: each evaluates half and they swap
-      float sn_m[4], cs_m[4];
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const float w = s_w[m0 + 2 * q + mine];
-        const float ang = rf * w;
-        const float err = fmaf(rf, w, -ang);
-        const float kq = rintf(ang * 0.15915493667125702f);
-        float red = fmaf(-kq, 6.28125f, ang);
-        red = fmaf(-kq, 0.0019354820251464844f, red);
-        red = fmaf(-kq, -1.7484555314695172e-07f, red);
-        const float sn = __sinf(red), cs = __cosf(red);
-        sn_m[q] = fmaf(err, cs, sn);
-        cs_m[q] = fmaf(-err, sn, cs);
-      }
-      const uint32_t own[4] = {t.v[it].x, t.v[it].y, t.v[it].z, t.v[it].w};
-      const uint32_t oth[4] = {pv.x, pv.y, pv.z, pv.w};
-      uint32_t out[4];
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const float sn_o = __shfl_sync(0xffffffffu, sn_m[q], partner);
-        const float cs_o = __shfl_sync(0xffffffffu, cs_m[q], partner);
-        float res[2];
-#pragma unroll
-        for (int hlf = 0; hlf < 2; ++hlf) {
-          const float sn = hlf == mine ? sn_m[q] : sn_o, cs = hlf == mine ? cs_m[q] : cs_o;
-          const float x = __uint_as_float(hlf ? (own[q] & 0xFFFF0000u) : (own[q] << 16));
-          const float y = __uint_as_float(hlf ? (oth[q] & 0xFFFF0000u) : (oth[q] << 16));
-          res[hlf] = in_x ? fmaf(x, cs, y * sn) : fmaf(x, cs, -(y * sn));
-        }
-        const __nv_bfloat162 b2 = __floats2bfloat162_rn(res[0], res[1]);
-        out[q] = *reinterpret_cast<const uint32_t *>(&b2);
-      }
-      if (in_x || in_y) t.v[it] = make_uint4(out[0], out[1], out[2], out[3]);
-    }
-  };
-  // every reader of the unit's old page has its loads landed
-  auto readers_done = [&](const Tile &t) -> bool {
-    // counts only grow: if every reader had landed when the unit was loaded,
-    // the store may go ahead (it is issued only after that read returned)
-    if (t.seen >= a.n_lanes) return true;
-    for (int rw = t.dlo; rw <= t.dhi; ++rw)
-      if (!wait_landed(&pd.dep[rw].landed, a.n_lanes, abort_flag)) return false;
-    return true;
-  };
-
-  const int mover = blockIdx.x * kMovers + wid;
-  const int my_units = mover < n_slots ? (n_slots - 1 - mover) / nm + 1 : 0;
-  // the unit's (kk, j, tl) advance by nm slots without a division
-  const int step_kk = nm / row_size, step_pos = nm - step_kk * row_size;
-  const int step_j = step_pos / a.n_lanes, step_tl = step_pos - step_j * a.n_lanes;
-  int kk = mover / row_size, pos = mover - kk * row_size;
-  int j = pos / a.n_lanes, tl = pos - j * a.n_lanes;
-  auto advance = [&]() {
-    kk += step_kk;
-    j += step_j;
-    tl += step_tl;
-    if (tl >= a.n_lanes) {
-      tl -= a.n_lanes;
-      ++j;
-    }
-    if (j >= n_active) {
-      j -= n_active;
-      ++kk;
-    }
-  };
-  Tile A, B;
-  Meta M;   // the descriptors of the next unit to load
-  if (my_units > 0) {
-    fetch(kk, j, tl, M);
-    advance();
-    load(M, A);
-    fetch(kk, j, tl, M);
-    advance();
-    load(M, B);
-    fetch(kk, j, tl, M);
-    advance();
-    land_and_count(A);
-    rotate(A);
-    // unit u in `cur` (landed, counted, rotated), unit u + 1 in flight in `next`:
-    // u is stored and u + 2's loads are issued before waiting for u + 1's, so
-    // two units' loads are in flight during that wait.  Every unit is still
-    // counted before it is stored, so the lowest-numbered unstored unit can
-    // always proceed.
-    auto step = [&](Tile &cur, Tile &next) -> bool {
-      if (!readers_done(cur)) return false;
-      store(cur);
-      load(M, cur);   // unit u + 2
-      fetch(kk, j, tl, M);
-      advance();
-      land_and_count(next);
-      rotate(next);
-      return true;
-    };
-    for (int u = 0; u < my_units; u += 2) {
-      bool ok = step(A, B);
-      if (ok && u + 1 < my_units) ok = step(B, A);
-      if (!ok) {
-        if (lane == 0) {
-          set_error(a.status, UMIM_ERR_TIMEOUT);
-          atomicExch(abort_flag, 1);
-        }
-        break;
-      }
-    }
-  }
-
-  finish_rollback(a, arr, s_last);
-}
-
-
 // ---------------------------------------------------------------------------
-// The move with TMA bulk copies (keys moved verbatim).  Same units, plan,
-// landed counters and ordering argument as rollback_move_kernel; a unit's 16
-// rows go through shared memory instead of registers.  Each slot's source is
+// The move, with TMA bulk copies.  A unit's 16 rows go through shared memory:
+// each slot's source is
 // a moved entry, a surrogate row, or -- for a slot inside the written range
 // that keeps its entry -- the row itself; slots whose sources are consecutive
 // rows of one old page form a run that its first lane copies with one
 // cp.async.bulk into the unit's stage.  The stage's mbarrier completes, the
 // unit is counted into its row, and once its page's reader rows have landed
 // one bulk store writes the unit's written slot range [ra, rb) back (a
-// contiguous part of the 16 x D tile).  Each warp keeps three units in its
-// ring.  The copy engine's reads and writes of the same pages keep their full
-// rate, where 16-byte loads and stores of a 4 KB tile written back in place a
-// few tiles behind its reads lose about a seventh.
+// contiguous part of the 16 x D tile).  With RoPE, the moved keys are re-rotated
+// in shared memory between the copies and the store.  Each warp keeps three
+// units in its ring.  The copy engine's reads and writes of the same pages keep
+// their full rate, where 16-byte loads and stores of a 4 KB tile written back in
+// place a few tiles behind its reads lose about a seventh.
 // ---------------------------------------------------------------------------
 constexpr int kBulkThreads = 512;   // 16 mover warps, one CTA per SM
 constexpr int kBulkMovers = kBulkThreads / 32;
@@ -574,7 +229,7 @@ __device__ __forceinline__ void fence_proxy_async_global() {
   asm volatile("fence.proxy.async.global;" ::: "memory");
 }
 
-template <int D>
+template <int D, bool ROPE>
 __global__ void __launch_bounds__(kBulkThreads, 1) rollback_bulk_kernel(MoveArgs a, PlanArrays arr, PageDesc pd) {
   constexpr int ROW = D * 2;                 // bytes of one entry of one (K|V, head)
   constexpr int TILE = kPageSize * ROW;      // bytes of a unit
@@ -585,10 +240,13 @@ __global__ void __launch_bounds__(kBulkThreads, 1) rollback_bulk_kernel(MoveArgs
   __shared__ int s_sq[kSmemSeqs], s_nd[kSmemSeqs], s_ub[kSmemSeqs], s_fp[kSmemSeqs];
   __shared__ int64_t s_toff[kSmemLanes];
   __shared__ int32_t s_tlh[kSmemLanes];
+  __shared__ float s_w[ROPE ? D / 2 : 1];   // RoPE angular frequencies
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
   const int nm = gridDim.x * kBulkMovers;
   uint8_t *ring = bulk_smem + (size_t)wid * kBulkStages * TILE;
 
+  if (ROPE)
+    for (int i = threadIdx.x; i < a.rotary_dim / 2; i += blockDim.x) s_w[i] = a.rope_inv_freq[i];
   if (lane == 0) {
     for (int st = 0; st < kBulkStages; ++st) mbar_init(&bars[wid][st], 1);
     fence_mbar_init();
@@ -638,6 +296,7 @@ __global__ void __launch_bounds__(kBulkThreads, 1) rollback_bulk_kernel(MoveArgs
     int64_t my_src;   // lanes < 16: the source of slot `lane` (kNoWrite: the slot keeps its entry)
     int64_t tile;     // offset of its (layer, K|V, head) tile in page 0 of the layer
     int32_t valid, idx, page, lh, kv, ra, rb, dlo, dhi, seen;
+    int32_t shift;    // lanes < 16: positions removed before slot `lane`'s moved entry (re-rotated keys)
   };
   auto fetch = [&](int kk, int j, int tl, Unit &m) {
     m.valid = 0;
@@ -661,6 +320,7 @@ __global__ void __launch_bounds__(kBulkThreads, 1) rollback_bulk_kernel(MoveArgs
       m.tile = layer * layer_stride + (int)(m.kv * kv_stride32 + h * kHead);
     }
     m.my_src = lane < kPageSize ? pd.src[(int64_t)m.idx * kPageSize + lane] : kNoWrite;
+    m.shift = (ROPE && lane < kPageSize) ? pd.shift[(int64_t)m.idx * kPageSize + lane] : 0;
     m.page = a.block_table[(int64_t)b * a.max_pages + fp_of(j) + kk];
     const RowDep dep = pd.dep[m.idx];
     m.dlo = dep.lo;
@@ -713,6 +373,51 @@ __global__ void __launch_bounds__(kBulkThreads, 1) rollback_bulk_kernel(MoveArgs
     m.seen = a.n_lanes;
     if (lane == 0)
       for (int rw = m.dlo; rw <= m.dhi; ++rw) m.seen = min(m.seen, ld_relaxed(&pd.dep[rw].landed));
+  };
+  // RoPE: a moved key (shift r > 0) is rotated in shared memory by -r w_m on the
+  // pairs (m, m + rotary_dim/2): x' = x cos + y sin, y' = y cos - x sin, with the
+  // angle r w rounded plus its exact rounding error (an fma) folded into the sine
+  // and cosine to first order, and the rounded angle reduced to [-pi, pi] (Cody
+  // and Waite's three-part reduction) for the hardware sine and cosine.  Lane l
+  // takes the pairs m = l and l + 32 of every row; consecutive rows with the same
+  // shift (a run of moved entries between two spans) reuse the lane's angles.
+  static_assert(D / 2 <= 64, "two pairs per lane");
+  auto rotate_rows = [&](const Unit &m, uint8_t *stage) {
+    const int half = a.rotary_dim / 2;
+    float prev = 0.f, snc[2] = {0.f, 0.f}, csc[2] = {1.f, 1.f};
+    for (int r = m.ra; r < m.rb; ++r) {
+      const float rf = (float)__shfl_sync(0xffffffffu, m.shift, r);
+      if (rf == 0.f) continue;   // a surrogate or an entry that keeps its position
+      if (rf != prev) {
+#pragma unroll
+        for (int i = 0; i < 2; ++i) {
+          const int q = lane + 32 * i;
+          if (q < half) {
+            const float w = s_w[q];
+            const float ang = rf * w;
+            const float err = fmaf(rf, w, -ang);
+            const float kq = rintf(ang * 0.15915493667125702f);
+            float red = fmaf(-kq, 6.28125f, ang);
+            red = fmaf(-kq, 0.0019354820251464844f, red);
+            red = fmaf(-kq, -1.7484555314695172e-07f, red);
+            const float sn0 = __sinf(red), cs0 = __cosf(red);
+            snc[i] = fmaf(err, cs0, sn0);
+            csc[i] = fmaf(-err, sn0, cs0);
+          }
+        }
+        prev = rf;
+      }
+      __nv_bfloat16 *row = reinterpret_cast<__nv_bfloat16 *>(stage + r * ROW);
+#pragma unroll
+      for (int i = 0; i < 2; ++i) {
+        const int q = lane + 32 * i;
+        if (q < half) {
+          const float x = __bfloat162float(row[q]), y = __bfloat162float(row[q + half]);
+          row[q] = __float2bfloat16_rn(fmaf(x, csc[i], y * snc[i]));
+          row[q + half] = __float2bfloat16_rn(fmaf(y, csc[i], -(x * snc[i])));
+        }
+      }
+    }
   };
   // every reader row of the unit's old page has its loads landed
   auto readers_done = [&](const Unit &m) -> bool {
@@ -770,6 +475,11 @@ __global__ void __launch_bounds__(kBulkThreads, 1) rollback_bulk_kernel(MoveArgs
       if (k + S < my_units) next_unit(Nx);
     }
     if (!__all_sync(0xffffffffu, mbar_wait(&bars[wid][st], (uint32_t)(k / S) & 1u))) return false;
+    if (ROPE && cur.valid && cur.kv == 0) {
+      rotate_rows(cur, ring + st * TILE);
+      fence_proxy_async_smem();   // the rotated rows, written by the lanes, are what the bulk store reads
+      __syncwarp();
+    }
     bool ok = true;
     if (lane == 0 && cur.valid) {
       // the unit's rows are in shared memory, so its reads of the old pages are done: count it
@@ -873,15 +583,13 @@ umim_status kv_rollback(const umim_paged_kv *kv, int32_t *block_table, int32_t m
   ma.status = status;
   ma.rope_inv_freq = rope_inv_freq;
   ma.rotary_dim = rope_inv_freq ? rotary_dim : 0;
-  ma.zero = 0;
   const bool rope = rope_inv_freq != nullptr;
-  // verbatim moves go through the copy engine; re-rotated keys through registers
-  auto kern = rope ? (D == 128 ? rollback_move_kernel<128, true> : rollback_move_kernel<64, true>)
-                   : (D == 128 ? rollback_bulk_kernel<128> : rollback_bulk_kernel<64>);
-  const int threads = rope ? kMoveThreads : kBulkThreads;
-  const int smem = rope ? 0 : kBulkMovers * kBulkStages * kPageSize * D * 2;
+  auto kern = rope ? (D == 128 ? rollback_bulk_kernel<128, true> : rollback_bulk_kernel<64, true>)
+                   : (D == 128 ? rollback_bulk_kernel<128, false> : rollback_bulk_kernel<64, false>);
+  const int threads = kBulkThreads;
+  const int smem = kBulkMovers * kBulkStages * kPageSize * D * 2;
   // set on every call: the attribute belongs to the current device
-  if (!rope && cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
     return UMIM_ERR_CUDA;
   int per_sm = 0;
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, threads, smem) != cudaSuccess || per_sm < 1)
