@@ -272,3 +272,22 @@ def test_merge_needs_a_token_per_span(lib):
     null = ctypes.c_void_p(0)
     w = MergeWeightsC(*([1 << 20] * 9), 512, 4, 1e-5)
     assert lib.umim_merge_spans(null, 10, null, 3, null, 4, ctypes.byref(w), null, null, 0, null, null) == 1
+
+
+def test_binding_switches_library_and_decodes_bounds_words():
+    """use_debug_library routes the binding's calls to libumim_debug.so and back;
+    a UMIM_ERR_BOUNDS word raises an error naming its access site."""
+    import paper_2609_27233_gb300 as umim
+    from paper_2609_27233_gb300 import build, _lib
+    for path, v in ((_lib.LIB_PATH, "release"), (_lib.DEBUG_LIB_PATH, "debug")):
+        if not os.path.exists(path):
+            build.build(variants=(v,))
+    try:
+        umim.use_debug_library(True)
+        assert umim.umim_debug_build() == 1
+        err = umim.UmimError(umim.UMIM_ERR_BOUNDS | (12 << 8), "step")
+        assert err.site == "decode_step.cache_write" and "UMIM_ERR_BOUNDS at decode_step.cache_write" in str(err)
+    finally:
+        umim.use_debug_library(False)
+    assert umim.umim_debug_build() == 0
+    assert "UMIM_ERR_TIMEOUT" in str(umim.UmimError(4, "x")) and umim.UmimError(4).site == ""
