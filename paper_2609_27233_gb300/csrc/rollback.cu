@@ -183,19 +183,18 @@ __device__ __forceinline__ bool wait_landed(const int32_t *cnt, int target, cons
 }
 
 // ---------------------------------------------------------------------------
-// The move, with TMA bulk copies.  A unit's 16 rows go through shared memory:
-// each slot's source is
-// a moved entry, a surrogate row, or -- for a slot inside the written range
-// that keeps its entry -- the row itself; slots whose sources are consecutive
-// rows of one old page form a run that its first lane copies with one
-// cp.async.bulk into the unit's stage.  The stage's mbarrier completes, the
-// unit is counted into its row, and once its page's reader rows have landed
-// one bulk store writes the unit's written slot range [ra, rb) back (a
-// contiguous part of the 16 x D tile).  With RoPE, the moved keys are re-rotated
-// in shared memory between the copies and the store.  Each warp keeps three
-// units in its ring.  The copy engine's reads and writes of the same pages keep
-// their full rate, where 16-byte loads and stores of a 4 KB tile written back in
-// place a few tiles behind its reads lose about a seventh.
+// The move, with TMA bulk copies.  A unit's 16 rows go through shared memory.
+// Each slot's source is a moved entry, a surrogate row, or -- for a slot inside
+// the written range that keeps its entry -- the row itself; slots whose sources
+// are consecutive rows of one old page form a run that its first lane copies
+// with one cp.async.bulk into the unit's stage.  The stage's mbarrier
+// completes, the unit is counted into its row, and once its page's reader rows
+// have landed one bulk store writes the unit's written slot range [ra, rb) back
+// (a contiguous part of the 16 x D tile).  With RoPE, the moved keys are
+// re-rotated in shared memory between the copies and the store.  Each warp
+// keeps three units in its ring.  The copy engine's reads and writes of the
+// same pages keep their full rate, where 16-byte loads and stores of a 4 KB
+// tile written back in place a few tiles behind its reads lose about a seventh.
 // ---------------------------------------------------------------------------
 constexpr int kBulkThreads = 512;   // 16 mover warps, one CTA per SM
 constexpr int kBulkMovers = kBulkThreads / 32;
